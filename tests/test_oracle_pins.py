@@ -1,0 +1,409 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Every check here computes its expectation by a route other than the oracle's
+own code: brute force on tiny inputs, a textbook top-k MoE written with torch
+CPU ops, closed forms, or invariants the paper states. No test here needs a GPU.
+"""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import decomoe_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+rng = np.random.default_rng(1234)
+
+
+def _logits(T, E, seed, bias=None, std=1.0):
+    r = np.random.default_rng(seed)
+    a = r.standard_normal((T, E)) * std
+    if bias is not None:
+        a = a + bias[None, :]
+    return a.astype(np.float32)
+
+
+# ---------------------------------------------------------------- router (Eq. 1)
+
+def test_router_logits_bruteforce_fsum():
+    r = np.random.default_rng(0)
+    x = r.standard_normal((5, 7)).astype(np.float32)
+    w = r.standard_normal((4, 7)).astype(np.float32)
+    b = r.standard_normal(4).astype(np.float32)
+    a = O.router_logits(x, w, b)
+    assert a.dtype == np.float32
+    for t in range(5):
+        for e in range(4):
+            exact = math.fsum([float(x[t, j]) * float(w[e, j]) for j in range(7)] + [float(b[e])])
+            # both round a float64-accurate value once to float32: at most 1 ulp apart
+            assert abs(float(a[t, e]) - exact) <= np.spacing(np.float32(abs(exact)))
+
+
+def test_router_logits_onehot_closed_form():
+    d, E = 6, 5
+    w = np.arange(E * d, dtype=np.float32).reshape(E, d) / 7.0
+    b = np.linspace(1, -1, E).astype(np.float32)
+    x = np.eye(d, dtype=np.float32)
+    a = O.router_logits(x, w, b)
+    np.testing.assert_array_equal(a, (w.T + b[None, :]).astype(np.float32))
+
+
+def test_softmax_closed_forms():
+    a, c = 0.3, -1.7
+    s = O.softmax(np.array([[a, c]]))
+    assert s[0, 0] == pytest.approx(1.0 / (1.0 + math.exp(c - a)), rel=1e-15)
+    v = rng.standard_normal((3, 9))
+    np.testing.assert_allclose(O.softmax(v).sum(-1), 1.0, rtol=0, atol=1e-15)
+    np.testing.assert_allclose(O.softmax(v + 11.0), O.softmax(v), rtol=1e-13)
+
+
+# ---------------------------------------------------------------- top-k (Eqs. 7, 10)
+
+def test_topk_bruteforce_subsets():
+    for seed in range(20):
+        E, k = 7, 3
+        v = np.random.default_rng(seed).standard_normal(E).astype(np.float32)
+        got = O.topk(v[None, :], k)[0]
+        best = max(itertools.combinations(range(E), k), key=lambda S: sum(float(v[e]) for e in S))
+        assert set(got.tolist()) == set(best)
+        assert all(v[got[i]] >= v[got[i + 1]] for i in range(k - 1))
+
+
+def test_topk_ties_lower_index_first():
+    v = np.array([[0.5, 2.0, 0.5, 2.0, 0.5]], np.float32)
+    assert O.topk(v, 3)[0].tolist() == [1, 3, 0]
+
+
+def test_full_pool_route_matches_textbook_torch():
+    a = _logits(40, 16, 3)
+    R, w = O.full_pool_route(a, 4)
+    t = torch.from_numpy(a.astype(np.float64))
+    p = torch.softmax(t, dim=-1)
+    tv, ti = torch.topk(p, 4, dim=-1, sorted=True)
+    tw = tv / tv.sum(-1, keepdim=True)
+    assert np.array_equal(R, ti.numpy())
+    np.testing.assert_allclose(w, tw.numpy(), rtol=1e-13, atol=1e-15)
+
+
+def test_ranking_by_probability_equals_ranking_by_logit():
+    a = _logits(200, 32, 9, std=3.0)
+    by_q = np.argsort(-O.softmax(a), axis=-1, kind="stable")[:, :8]
+    assert np.array_equal(O.topk(a, 8), by_q)
+
+
+# ---------------------------------------------------------------- activated mass (Eq. 11)
+
+def test_activated_mass_bruteforce_per_expert():
+    T, E, k = 12, 9, 3
+    a = _logits(T, E, 5)
+    s = O.activated_mass(a, k)
+    s_bf = np.zeros(E)
+    for e in range(E):
+        for i in range(T):
+            row = [float(v) for v in a[i]]
+            q = [math.exp(v - max(row)) for v in row]
+            top = sorted(range(E), key=lambda j: (-row[j], j))[:k]
+            if e in top:
+                s_bf[e] += q[e] / sum(q[j] for j in top)
+    np.testing.assert_allclose(s, s_bf, rtol=1e-13, atol=1e-15)
+
+
+def test_activated_mass_total_is_token_count():
+    a = _logits(300, 64, 7)
+    s = O.activated_mass(a, 8)
+    assert s.sum() == pytest.approx(300.0, rel=1e-13)
+    assert (s >= 0).all()
+
+
+def test_activated_mass_equal_top_logits_split_evenly():
+    # two tokens whose two largest logits are equal: each gets weight 1/2
+    a = np.array([[3.0, 3.0, -1.0, -2.0], [-5.0, 0.0, 7.0, 7.0]], np.float32)
+    s = O.activated_mass(a, 2)
+    np.testing.assert_allclose(s, [0.5, 0.5, 0.5, 0.5], rtol=0, atol=1e-15)
+
+
+# ---------------------------------------------------------------- prefix length (Eq. 12)
+
+def _select_bruteforce(s, p, k):
+    E = len(s)
+    tot = math.fsum(s)
+    ok = [K for K in range(1, E + 1) if math.fsum(s[:K]) >= p * tot * (1 - 1e-12)]
+    return max(k, min(ok))
+
+
+def test_select_prefix_bruteforce():
+    for seed in range(50):
+        r = np.random.default_rng(seed)
+        E = int(r.integers(2, 40))
+        k = int(r.integers(1, E + 1))
+        s = r.random(E) ** 3 * 10
+        for p in (0.05, 0.3, 0.5, 0.7, 0.9, 0.999):
+            K = O.select_prefix(s, p, k)
+            # tolerance-free brute force can differ only when a partial ratio
+            # is within rounding of p; such draws are skipped
+            ratios = np.cumsum(s) / s.sum()
+            if np.min(np.abs(ratios - p)) < 1e-9:
+                continue
+            assert K == _select_bruteforce(list(s), p, k)
+
+
+def test_select_prefix_invariants_from_paper():
+    # K >= k always; K monotone non-decreasing in p; p = 1 keeps the full pool
+    # (Appendix sweep: average prefix 128.0 of 128 at p = 1.0)
+    with open(os.path.join(GOLDEN, "rcep_prefix_vs_p.json")) as f:
+        g = json.load(f)
+    E, k = g["E"], g["k_moe"]
+    for seed in range(30):
+        r = np.random.default_rng(100 + seed)
+        # Zipf-like skew over the reordered index, like a calibrated order
+        s = (1.0 / (np.arange(E) + 1.0) ** r.uniform(0.5, 2.0)) * r.uniform(0.5, 1.5, E)
+        Ks = [O.select_prefix(s, p, k) for p in g["p"]]
+        assert all(K >= k for K in Ks)
+        assert all(Ks[i] <= Ks[i + 1] for i in range(len(Ks) - 1))
+        assert Ks[-1] == E
+        # mass concentrated so that the first k experts cover >= 20%: the
+        # clamp gives exactly k at p = 0.1 and 0.2 (sweep: 8.0 = k_moe there)
+        if np.cumsum(s)[k - 1] / s.sum() >= 0.2:
+            assert Ks[0] == k and Ks[1] == k
+    # the published sweep itself is monotone, starts at k_moe and ends at E
+    avg = g["avg_prefix"]
+    assert avg[0] == k and avg[1] == k and avg[-1] == E
+    assert all(avg[i] <= avg[i + 1] for i in range(len(avg) - 1))
+
+
+def test_select_prefix_edge_cases():
+    s = np.array([0.0, 0.0, 5.0, 0.0])
+    assert O.select_prefix(s, 0.5, 1) == 3
+    assert O.select_prefix(s, 1.0, 1) == 4          # p = 1 -> E
+    assert O.select_prefix(np.zeros(4), 0.7, 2) == 2  # empty invocation -> k
+    with pytest.raises(ValueError):
+        O.select_prefix(s, 0.0, 1)
+    with pytest.raises(ValueError):
+        O.select_prefix(s, 1.5, 1)
+
+
+# ---------------------------------------------------------------- prefix routing
+
+def test_route_prefix_full_span_is_ordinary_topk_moe():
+    a = _logits(50, 16, 11)
+    i1, w1 = O.route_prefix(a, 16, 2)
+    i2, w2 = O.full_pool_route(a, 2)
+    assert np.array_equal(i1, i2)
+    np.testing.assert_allclose(w1, w2, rtol=1e-13)
+
+
+def test_route_prefix_bruteforce_and_softmax_over_picks():
+    for seed in range(10):
+        a = _logits(6, 10, 20 + seed)
+        for K in (3, 5, 10):
+            idx, w = O.route_prefix(a, K, 3)
+            assert (idx < K).all()
+            np.testing.assert_allclose(w.sum(-1), 1.0, atol=1e-14)
+            for t in range(6):
+                best = max(itertools.combinations(range(K), 3),
+                           key=lambda S: sum(float(a[t, e]) for e in S))
+                assert set(idx[t].tolist()) == set(best)
+                picks = [float(a[t, e]) for e in idx[t]]
+                z = [math.exp(v - max(picks)) for v in picks]
+                np.testing.assert_allclose(w[t], np.array(z) / sum(z), rtol=1e-13)
+
+
+def test_route_prefix_does_not_intersect_full_pool_topk():
+    # full-pool top-2 of this token is {7, 6}, both outside the prefix K=4.
+    # Intersecting would leave no expert; the paper's rule reruns top-k
+    # inside the prefix and still returns exactly k experts.
+    a = np.array([[0.1, 0.4, 0.2, 0.3, -1.0, -2.0, 5.0, 6.0]], np.float32)
+    idx, w = O.route_prefix(a, 4, 2)
+    assert idx[0].tolist() == [1, 3]
+    v = a[0, [1, 3]].astype(np.float64)
+    e = np.exp(v - v[0])
+    np.testing.assert_allclose(w[0], e / e.sum(), rtol=1e-14)
+
+
+def test_route_prefix_weights_invariant_to_K_when_set_unchanged():
+    a = _logits(30, 20, 4, bias=-np.log(np.arange(20) + 1.0))
+    i1, w1 = O.route_prefix(a, 20, 4)
+    i2, w2 = O.route_prefix(a, 12, 4)
+    same = (i1 == i2).all(-1)
+    assert same.any()
+    np.testing.assert_allclose(w1[same], w2[same], rtol=1e-13)
+
+
+def test_route_prefix_K_equals_k_takes_whole_prefix():
+    a = _logits(8, 12, 8)
+    idx, _ = O.route_prefix(a, 3, 3)
+    assert all(sorted(r) == [0, 1, 2] for r in idx.tolist())
+
+
+# ---------------------------------------------------------------- dispatch
+
+def test_dispatch_is_stable_sort_by_expert():
+    for seed in range(10):
+        r = np.random.default_rng(seed)
+        T, k, K = int(r.integers(1, 60)), int(r.integers(1, 5)), int(r.integers(1, 9))
+        idx = r.integers(0, K, size=(T, k))
+        counts, offsets, perm_token, inv_slot = O.dispatch(idx, K)
+        order = np.argsort(idx.reshape(-1), kind="stable")
+        assert np.array_equal(perm_token, order // k)
+        assert counts.sum() == T * k and offsets[-1] == T * k and offsets[0] == 0
+        assert np.array_equal(np.bincount(idx.reshape(-1), minlength=K), counts)
+        assert np.array_equal(inv_slot[order], np.arange(T * k))
+        assert sorted(inv_slot.tolist()) == list(range(T * k))
+        # within one expert, rows follow increasing flat index
+        for e in range(K):
+            fl = order[offsets[e]:offsets[e + 1]]
+            assert (np.diff(fl) > 0).all() and (idx.reshape(-1)[fl] == e).all()
+
+
+def test_dispatch_empty_and_single_expert():
+    counts, offsets, perm, inv = O.dispatch(np.zeros((0, 2), np.int64), 4)
+    assert counts.tolist() == [0, 0, 0, 0] and offsets.tolist() == [0] * 5 and len(perm) == 0
+    counts, offsets, perm, inv = O.dispatch(np.full((5, 1), 2), 3)
+    assert counts.tolist() == [0, 0, 5] and perm.tolist() == [0, 1, 2, 3, 4]
+
+
+# ---------------------------------------------------------------- expert FFN + combine
+
+def _tiny_layer(seed, T=9, d=6, m=5, E=6):
+    r = np.random.default_rng(seed)
+    x = r.standard_normal((T, d))
+    wg = r.standard_normal((E, m, d)) * 0.5
+    wu = r.standard_normal((E, m, d)) * 0.5
+    wd = r.standard_normal((E, d, m)) * 0.5
+    return x, wg, wu, wd
+
+
+def test_silu_closed_forms():
+    assert O.silu(0.0) == 0.0
+    assert O.silu(1.0) == pytest.approx(1.0 / (1.0 + math.exp(-1.0)), rel=1e-15)
+    assert O.silu(-40.0) == pytest.approx(-40.0 * math.exp(-40.0), rel=1e-9)
+    np.testing.assert_allclose(O.silu(np.array([3.0])), torch.nn.functional.silu(
+        torch.tensor([3.0], dtype=torch.float64)).numpy(), rtol=1e-15)
+
+
+def test_layer_matches_dense_equivalent_formulation():
+    # Appendix "Dense-equivalent expert convention": run every retained expert
+    # on every token, then apply the sparse routing weights. It must equal the
+    # sparse grouped computation.
+    for seed in range(4):
+        x, wg, wu, wd = _tiny_layer(seed)
+        T, E, k, K = x.shape[0], wg.shape[0], 2, 4
+        a = _logits(T, E, 50 + seed)
+        idx, w = O.route_prefix(a, K, k)
+        counts, offsets, perm, inv = O.dispatch(idx, K)
+        y = O.expert_swiglu(x[perm], offsets, wg, wu, wd)
+        out = O.combine(y, inv, w)
+        xt = torch.from_numpy(x)
+        dense = torch.stack([
+            torch.nn.functional.linear(
+                torch.nn.functional.silu(torch.nn.functional.linear(xt, torch.from_numpy(wg[e])))
+                * torch.nn.functional.linear(xt, torch.from_numpy(wu[e])),
+                torch.from_numpy(wd[e]))
+            for e in range(K)])                                    # [K, T, d]
+        Wsp = torch.zeros(T, K, dtype=torch.float64)
+        Wsp.scatter_(1, torch.from_numpy(idx), torch.from_numpy(w))
+        ref = torch.einsum("tk,ktd->td", Wsp, dense).numpy()
+        np.testing.assert_allclose(out, ref, rtol=1e-12, atol=1e-12)
+
+
+def test_expert_swiglu_diagonal_closed_form():
+    d = m = 4
+    al, be, ga = 0.7, -1.3, 2.0
+    wg = np.stack([al * np.eye(d)] * 2)
+    wu = np.stack([be * np.eye(d)] * 2)
+    wd = np.stack([ga * np.eye(d)] * 2)
+    x = np.array([[1.0, -2.0, 0.5, 0.0], [3.0, 0.25, -1.0, 2.0]])
+    y = O.expert_swiglu(x, np.array([0, 1, 2]), wg, wu, wd)
+    z = al * x
+    np.testing.assert_allclose(y, ga * (z / (1 + np.exp(-z))) * (be * x), rtol=1e-14)
+
+
+def test_combine_single_slot_and_residual():
+    y = np.arange(12.0).reshape(4, 3)
+    inv = np.array([2, 0, 3, 1])
+    w = np.ones((4, 1))
+    res = np.full((4, 3), 0.5)
+    out = O.combine(y, inv, w, res)
+    np.testing.assert_array_equal(out, y[[2, 0, 3, 1]] + 0.5)
+
+
+def test_full_span_layer_matches_textbook_moe_torch():
+    # K = E reduces to the ordinary top-k MoE (reordering only permutes storage)
+    x, wg, wu, wd = _tiny_layer(7, T=11, E=5)
+    r = np.random.default_rng(3)
+    w_r = r.standard_normal((5, x.shape[1])).astype(np.float32)
+    b = np.linspace(0.5, -0.5, 5).astype(np.float32)
+    x32 = x.astype(np.float32)
+    res = O.moe_layer(x32, w_r, b, wg, wu, wd, k=2, K=5)
+    xt = torch.from_numpy(x32.astype(np.float64))
+    logits = (xt @ torch.from_numpy(w_r.astype(np.float64)).T + torch.from_numpy(b.astype(np.float64))).float()
+    prob = torch.softmax(logits.double(), -1)
+    tv, ti = torch.topk(prob, 2, -1)
+    tw = tv / tv.sum(-1, keepdim=True)
+    ref = torch.zeros_like(xt)
+    for t in range(xt.shape[0]):
+        for j in range(2):
+            e = int(ti[t, j])
+            h = torch.nn.functional.silu(torch.from_numpy(wg[e]) @ xt[t]) * (torch.from_numpy(wu[e]) @ xt[t])
+            ref[t] += tw[t, j] * (torch.from_numpy(wd[e]) @ h)
+    np.testing.assert_allclose(res["out"], ref.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_moe_token_equals_layer_rows():
+    x, wg, wu, wd = _tiny_layer(9, T=7, E=6)
+    a = _logits(7, 6, 77)
+    idx, w = O.route_prefix(a, 4, 2)
+    counts, offsets, perm, inv = O.dispatch(idx, 4)
+    out = O.combine(O.expert_swiglu(x[perm], offsets, wg, wu, wd), inv, w)
+    for t in range(7):
+        o, _, _ = O.moe_token(x[t], a[t], wg, wu, wd, 4, 2)
+        np.testing.assert_allclose(o, out[t], rtol=1e-12, atol=1e-13)
+
+
+def test_adaptive_K_path_uses_select_prefix():
+    x, wg, wu, wd = _tiny_layer(2, T=20, E=6)
+    r = np.random.default_rng(1)
+    w_r = r.standard_normal((6, x.shape[1])).astype(np.float32)
+    b = (-1.1 * np.log(np.arange(6) + 1.0)).astype(np.float32)
+    res = O.moe_layer(x.astype(np.float32), w_r, b, wg, wu, wd, k=2, p=0.7)
+    a = O.router_logits(x.astype(np.float32), w_r, b)
+    assert res["K"] == _select_bruteforce(list(O.activated_mass(a, 2)), 0.7, 2)
+
+
+# ---------------------------------------------------------------- SAVB removal
+
+def test_drop_visual_block_keeps_text_rows_in_order():
+    rows = np.arange(40).reshape(10, 4)
+    out = O.drop_visual_block(rows, 3, 4)
+    np.testing.assert_array_equal(out, np.delete(rows, np.s_[3:7], axis=0))
+    assert out.shape[0] == 6
+    np.testing.assert_array_equal(O.drop_visual_block(rows, 5, 0), rows)
+    np.testing.assert_array_equal(O.drop_visual_block(rows, 0, 10), rows[:0])
+    np.testing.assert_array_equal(O.drop_visual_block(rows, 0, 3), rows[3:])
+    np.testing.assert_array_equal(O.drop_visual_block(rows, 7, 3), rows[:7])
+
+
+# ---------------------------------------------------------------- stack
+
+def test_rmsnorm_closed_form():
+    x = np.full((1, 8), -3.0)
+    np.testing.assert_allclose(O.rmsnorm(x, eps=0.0), -np.ones((1, 8)), rtol=1e-15)
+    y = O.rmsnorm(np.array([[3.0, 4.0]]), eps=0.0)
+    np.testing.assert_allclose(y, [[3.0 / math.sqrt(12.5), 4.0 / math.sqrt(12.5)]], rtol=1e-15)
+
+
+def test_stack_one_layer_is_residual_moe():
+    x, wg, wu, wd = _tiny_layer(5, T=4, E=6)
+    r = np.random.default_rng(2)
+    w_r = r.standard_normal((6, x.shape[1])).astype(np.float32)
+    b = np.zeros(6, np.float32)
+    layer = dict(w_r=w_r, bias=b, w_gate=wg, w_up=wu, w_down=wd)
+    for t in range(4):
+        h, _ = O.stack_token(x[t], [layer], [4], 2)
+        xn = O.rmsnorm(x[t:t + 1])
+        ref = O.moe_layer(xn, w_r, b, wg, wu, wd, k=2, K=4)["out"][0] + x[t]
+        np.testing.assert_allclose(h, ref, rtol=1e-13, atol=1e-13)
