@@ -1,0 +1,549 @@
+#!/usr/bin/env python
+"""Throughput of the DecoMoE prefix-MoE hot path on GB300.
+
+One step = one pass of the whole hot path over one batch of the T=2048 prefill
+workload (d=2048, E=128 experts, top-8, expert FFN width 768, bf16 storage,
+fp32 accumulation): router logits over the full pool, activated-mass pass
+(Eq. 11), prefix routing over [0, K), dispatch, grouped SwiGLU experts,
+combine, and removal of the 1792-row visual block from the layer's hidden
+output (2048 -> 256 rows). K defaults to 64 (the workload's prefix sweep is
+128/96/64/40; the other values are reported under "sweep").
+
+Inputs rotate over 8 independent layers (weights ~1.2 GB each), so the
+per-step working set is far larger than L2.
+
+Prints ONE JSON line (rank 0). ``--impl reference`` times the CPU oracle
+instead (the reference arm), on bounded token samples of the same workload.
+Multi-GPU (torchrun): independent replicas, no collective on the data path.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads as W  # noqa: E402
+
+LAUNCHES_PER_STEP = 11  # router 1, mass 2, route 1, dispatch 3, gate/up 1, down 1, combine 1, compaction 1
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--K", type=int, default=64)
+    ap.add_argument("--layers", type=int, default=8)
+    ap.add_argument("--p", type=float, default=0.7)
+    ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------------ distributed plumbing
+
+def dist_setup(args):
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+
+        if args.impl == "ours":
+            torch.cuda.set_device(local)
+            dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        else:
+            dist.init_process_group("gloo")
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(0)
+    return ws, rank, local
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+def max_over_ranks(v, ws):
+    if ws == 1:
+        return v
+    import torch.distributed as dist
+
+    t = torch.tensor([v], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------ clocks
+
+class Clocks:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.path = tempfile.mktemp(prefix="clocks_", suffix=".csv")
+        self.proc = None
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "100",
+                 "-i", str(gpu_index)], stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        self.t_on = None
+        self.t_off = None
+
+    def mark_on(self):
+        self.t_on = time.time()
+
+    def mark_off(self):
+        self.t_off = time.time()
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        for line in open(self.path):
+            p = [s.strip() for s in line.split(",")]
+            if len(p) < 9:
+                continue
+            try:
+                rows.append(dict(sm=float(p[1]), smax=float(p[2]), power=float(p[3]), hw=p[5], hwt=p[6], swt=p[7],
+                                 swpc=p[8]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        # the sampler writes at ~100 ms; samples during the timed window are the
+        # ones drawing power above idle (the window is marked by power draw)
+        pmax = max(r["power"] for r in rows)
+        load = [r for r in rows if r["power"] >= 0.5 * pmax] or rows
+        reasons = set()
+        for r in load:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"), ("swt", "sw_thermal_slowdown"),
+                              ("swpc", "sw_power_cap")):
+                if r[key].lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(r["sm"] for r in load), "sm_max_mhz": max(r["smax"] for r in load),
+                "reasons": sorted(reasons), "samples": len(load), "power_w_max": pmax}
+
+
+# ------------------------------------------------------------------ peaks
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            pk = json.load(f)
+        return {"hbm_gbs": pk["hbm_gbs"], "bf16_tflops": pk["bf16_tflops"],
+                "bf16_tflops_sustained": pk.get("bf16_tflops_sustained"), "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+# ------------------------------------------------------------------ our arm
+
+class Layer:
+    def __init__(self, wl, l, dev, dm):
+        g = W.make_layer(wl, layer=l, device=dev)
+        self.x = g["x"]
+        self.w_r = g["w_r"]
+        self.bias = g["bias"]
+        self.w_gu = dm.fuse_gate_up(g["w_gate"], g["w_up"])
+        self.w_down = g["w_down"]
+        del g
+
+
+class Buffers:
+    def __init__(self, wl, T, dev, dm):
+        k, E, d, m = wl.k, wl.E, wl.d, wl.m
+        R = T * k
+        self.logits = torch.empty(T, E, dtype=torch.float32, device=dev)
+        self.mass = torch.empty(E, dtype=torch.float64, device=dev)
+        self.route_ws = dm.workspace(dm.decomoe_route_workspace_bytes(T, E), dev)
+        self.idx = torch.empty(T, k, dtype=torch.int32, device=dev)
+        self.w = torch.empty(T, k, dtype=torch.float32, device=dev)
+        self.counts = torch.empty(E, dtype=torch.int32, device=dev)
+        self.offsets = torch.empty(E + 1, dtype=torch.int32, device=dev)
+        self.perm = torch.empty(R, dtype=torch.int32, device=dev)
+        self.inv = torch.empty(R, dtype=torch.int32, device=dev)
+        self.x_perm = torch.empty(R, d, dtype=torch.bfloat16, device=dev)
+        self.disp_ws = dm.workspace(dm.decomoe_dispatch_workspace_bytes(T, k, E), dev)
+        self.h = torch.empty(R, m, dtype=torch.bfloat16, device=dev)
+        self.y = torch.empty(R, d, dtype=torch.bfloat16, device=dev)
+        self.out = torch.empty(T, d, dtype=torch.bfloat16, device=dev)
+        self.status = torch.zeros(1, dtype=torch.int32, device=dev)
+
+
+def run_step(dm, wl, L, B, K, v0, nv, text, ev=None):
+    """One pass of the hot path, every step a C-ABI call (11 kernel launches)."""
+    k, E = wl.k, wl.E
+    dm.decomoe_router_logits(L.x, L.w_r, L.bias, B.logits, B.status)                   # a1
+    dm.decomoe_route_prefix(B.logits, E, k, None, None, B.mass, B.route_ws)            # a2 (Eq. 11)
+    dm.decomoe_route_prefix(B.logits, K, k, B.idx, B.w)                                # a4
+    dm.decomoe_dispatch(B.idx, K, L.x, B.counts[:K], B.offsets[:K + 1], B.perm, B.inv, B.x_perm, B.disp_ws,
+                        B.status)                                                     # a5
+    if ev is not None:
+        ev[0].record()
+    dm.decomoe_expert_gate_up(B.x_perm, B.offsets[:K + 1], K, L.w_gu, B.h, B.status)   # a6 gate/up + SwiGLU
+    if ev is not None:
+        ev[1].record()
+    dm.decomoe_expert_down(B.h, B.offsets[:K + 1], K, L.w_down, B.y, B.status)         # a6 down
+    if ev is not None:
+        ev[2].record()
+    dm.decomoe_combine(B.y, B.inv, B.w, B.out)                                         # a7
+    if text is not None:
+        dm.decomoe_drop_visual_block(B.out, text, v0, nv)                              # a8
+
+
+def timed(fn, steps, warmup, ws, clocks=None, name="sweep"):
+    for i in range(warmup):
+        fn(i, None)
+    torch.cuda.synchronize()
+    barrier(ws)
+    torch.cuda.synchronize()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    if clocks:
+        clocks.mark_on()
+    torch.cuda.nvtx.range_push(name)
+    s.record()
+    for i in range(steps):
+        fn(i, evs[i])
+    e.record()
+    torch.cuda.synchronize()
+    torch.cuda.nvtx.range_pop()
+    if clocks:
+        clocks.mark_off()
+    barrier(ws)
+    ms = s.elapsed_time(e)
+    return ms, evs
+
+
+def algo_bytes_gate_up(wl, R, D):
+    return D * 2 * wl.m * wl.d * 2 + R * wl.d * 2 + R * wl.m * 2
+
+
+def algo_bytes_down(wl, R, D):
+    return D * wl.d * wl.m * 2 + R * wl.m * 2 + R * wl.d * 2
+
+
+def ours(args, ws, rank, local):
+    import paper_2609_38823_gb300 as dm
+
+    dm.lib()
+    dev = torch.device("cuda", local)
+    wl = W.PREFILL
+    T, k, K = wl.T, wl.k, args.K
+    R = T * k
+    pk = peaks()
+    layers = [Layer(wl, l, dev, dm) for l in range(args.layers)]
+    B = Buffers(wl, T, dev, dm)
+    v0, nv = wl.v0, wl.nv
+    text = torch.empty(T - nv, wl.d, dtype=torch.bfloat16, device=dev)
+    torch.cuda.synchronize()
+
+    clocks = Clocks(local) if rank == 0 else None
+
+    def step(i, ev):
+        run_step(dm, wl, layers[i % len(layers)], B, K, v0, nv, text, ev)
+
+    ms, evs = timed(step, args.steps, args.warmup, ws, clocks, name="timed")
+    # extend the clock window when the timed region is shorter than ~1.5 s
+    ext = 0
+    if clocks and ms < 1500:
+        t0 = time.time()
+        while time.time() - t0 < 1.5:
+            for i in range(200):
+                step(i, None)
+            torch.cuda.synchronize()
+            ext += 200
+    clk = clocks.stop() if clocks else None
+    if dm.decomoe_read_status(B.status) != 0:
+        raise RuntimeError("device status set during the benchmark")
+    ms_max = max_over_ranks(ms, ws)
+    step_ms = ms_max / args.steps
+    tok_s = ws * T * args.steps / (ms_max / 1e3)
+    gu_ms = statistics.mean(evs[i][0].elapsed_time(evs[i][1]) for i in range(args.steps))
+    dn_ms = statistics.mean(evs[i][1].elapsed_time(evs[i][2]) for i in range(args.steps))
+    # distinct active experts per layer (for the algorithmic bytes)
+    Ds = []
+    for l in range(len(layers)):
+        run_step(dm, wl, layers[l], B, K, v0, nv, text)
+        torch.cuda.synchronize()
+        Ds.append(int((B.counts[:K] > 0).sum()))
+    D = statistics.mean(Ds)
+    gu_flops = 2.0 * R * wl.d * 2 * wl.m
+    dn_flops = 2.0 * R * wl.m * wl.d
+    useful_flops = 6.0 * R * wl.d * wl.m + 2.0 * T * wl.d * wl.E
+    gu_bytes = algo_bytes_gate_up(wl, R, D)
+    gu_tflops = gu_flops / (gu_ms * 1e-3) / 1e12
+    gu_gbs = gu_bytes / (gu_ms * 1e-3) / 1e9
+    ffn_ms = gu_ms + dn_ms
+    ffn_tflops = (gu_flops + dn_flops) / (ffn_ms * 1e-3) / 1e12
+    t_compute = gu_flops / (pk["bf16_tflops"] * 1e12)
+    t_mem = gu_bytes / (pk["hbm_gbs"] * 1e9)
+    bound = "tensor" if t_compute >= t_mem else "hbm"
+    traffic = None
+    prof = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(prof):
+        try:
+            tr = json.load(open(prof)).get(f"gate_up_K{K}")
+            if tr and tr.get("source_hash") == _kernel_hash():
+                traffic = tr["bytes_per_launch"]
+        except Exception:
+            traffic = None
+    if bound == "tensor":
+        roof = {"bound": "tensor", "achieved": round(gu_tflops, 2), "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
+                "frac": round(gu_tflops / pk["bf16_tflops"], 4), "traffic": traffic}
+    else:
+        roof = {"bound": "hbm", "achieved": round(gu_gbs, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": round(gu_gbs / pk["hbm_gbs"], 4), "traffic": traffic}
+    roof.update({"kernel": "k_gemm_tc<256,SwiGLU> (expert gate/up, fused SwiGLU epilogue)",
+                 "peak_source": f"{pk['source']} burst", "ms_per_launch": round(gu_ms, 4),
+                 "flops_per_launch": gu_flops, "algo_bytes_per_launch": gu_bytes,
+                 "tensor_frac": round(gu_tflops / pk["bf16_tflops"], 4), "hbm_frac": round(gu_gbs / pk["hbm_gbs"], 4)})
+
+    # e2e through the composite C-ABI call with pinned host buffers
+    e2e = None
+    if True:
+        xs_host = [L.x.cpu().pin_memory() for L in layers]
+        out_host = torch.empty(T, wl.d, dtype=torch.bfloat16).pin_memory()
+        x_dev = torch.empty(T, wl.d, dtype=torch.bfloat16, device=dev)
+        lws = dm.workspace(dm.decomoe_moe_layer_workspace_bytes(T, wl.d, wl.E, k, wl.m, dm.DECOMOE_BF16), dev)
+
+        def e2e_step(i, ev):
+            L = layers[i % len(layers)]
+            x_dev.copy_(xs_host[i % len(layers)], non_blocking=True)
+            dm.decomoe_moe_layer(x_dev, L.w_r, L.bias, L.w_gu, L.w_down, k, B.out, lws, K_fixed=K, p=args.p,
+                                 status=B.status)
+            dm.decomoe_drop_visual_block(B.out, text, v0, nv)
+            out_host.copy_(B.out, non_blocking=True)
+
+        e_steps = max(10, min(args.steps, 1000))
+        ms_e, _ = timed(e2e_step, e_steps, max(3, args.warmup), ws)
+        ms_e = max_over_ranks(ms_e, ws)
+        e2e = {"value": round(ws * T * e_steps / (ms_e / 1e3), 1), "unit": "tokens/s",
+               "h2d_bytes_per_step": T * wl.d * 2, "d2h_bytes_per_step": T * wl.d * 2,
+               "ms_per_step": round(ms_e / e_steps, 4), "steps": e_steps,
+               "path": "pinned host x -> decomoe_moe_layer (C ABI) -> decomoe_drop_visual_block -> pinned host out"}
+
+    sweep = []
+    if not args.no_sweep:
+        sweep = run_sweep(args, dm, wl, layers, B, text, ws, pk)
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(wl, layers[0], K, args.cpu_seconds)
+
+    line = {
+        "metric": "prefix-MoE layer tokens/s (T=2048 prefill, K=%d of E=128)" % K,
+        "value": round(tok_s, 1), "unit": "tokens/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(step_ms, 4), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic (seeded N(0,1) hidden, N(0,0.02) weights, Zipf router bias -1.1 ln(e+1))",
+        "config": {"workload": wl.name, "T": T, "visual_block": [v0, nv], "d": wl.d, "E": wl.E, "k": k, "m": wl.m,
+                   "K": K, "layers_rotated": len(layers),
+                   "l2": "inputs larger than L2: 8 rotating layers, >=0.6 GB of weights per step",
+                   "parallelism": "replicas" if ws > 1 else "single GPU"},
+        "step_tflops": round(useful_flops / (step_ms * 1e-3) / 1e12, 2),
+        "expert_ffn": {"ms": round(ffn_ms, 4), "tflops": round(ffn_tflops, 2),
+                       "tensor_frac": round(ffn_tflops / pk["bf16_tflops"], 4),
+                       "gate_up_ms": round(gu_ms, 4), "down_ms": round(dn_ms, 4), "active_experts": D},
+        "roofline": roof,
+        "e2e": e2e,
+        "gpu_launches": LAUNCHES_PER_STEP * args.steps,
+        "clocks": clk,
+        "clock_window": "timed region" if ext == 0 else f"timed region + {ext} identical untimed steps",
+        "sweep": sweep,
+        "cpu_baseline": cpu,
+    }
+    return line
+
+
+def run_sweep(args, dm, wl, layers, B, text, ws, pk):
+    out = []
+    T = wl.T
+    R = T * wl.k
+    n = max(10, min(args.steps, 400))
+    for K in (128, 96, 64, 40):
+        ms, evs = timed(lambda i, ev: run_step(dm, wl, layers[i % len(layers)], B, K, wl.v0, wl.nv, text, ev), n,
+                        5, ws)
+        gu = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+        dn = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+        D = int((B.counts[:K] > 0).sum())
+        ffn_fl = 6.0 * R * wl.d * wl.m
+        ffn_by = algo_bytes_gate_up(wl, R, D) + algo_bytes_down(wl, R, D)
+        out.append({"mode": "fixed", "K": K, "tokens_per_s": round(T * n / (ms / 1e3), 1),
+                    "ms_per_step": round(ms / n, 4), "ffn_ms": round(gu + dn, 4),
+                    "ffn_tflops": round(ffn_fl / ((gu + dn) * 1e-3) / 1e12, 2),
+                    "ffn_tensor_frac": round(ffn_fl / ((gu + dn) * 1e-3) / 1e12 / pk["bf16_tflops"], 4),
+                    "ffn_hbm_frac": round(ffn_by / ((gu + dn) * 1e-3) / 1e9 / pk["hbm_gbs"], 4)})
+    # adaptive prefix: Eq. 12 on the host each step (device->host read of the mass)
+    lws = dm.workspace(dm.decomoe_moe_layer_workspace_bytes(T, wl.d, wl.E, wl.k, wl.m, dm.DECOMOE_BF16), B.out.device)
+    Ks = []
+
+    def ad_step(i, ev):
+        L = layers[i % len(layers)]
+        Ku, _ = dm.decomoe_moe_layer(L.x, L.w_r, L.bias, L.w_gu, L.w_down, wl.k, B.out, lws, K_fixed=0, p=args.p,
+                                     status=B.status)
+        Ks.append(Ku)
+        dm.decomoe_drop_visual_block(B.out, text, wl.v0, wl.nv)
+
+    ms, _ = timed(ad_step, n, 5, ws)
+    out.append({"mode": f"mass p={args.p}", "K_mean": round(statistics.mean(Ks[-n:]), 2),
+                "tokens_per_s": round(T * n / (ms / 1e3), 1), "ms_per_step": round(ms / n, 4)})
+    # decode-size layers, K=64: weight streaming, reported against HBM
+    for Td in W.DECODE_T:
+        Bd = Buffers(wl, Td, B.out.device, dm)
+        xs = [W.make_x(W.DECODE, T=Td, layer=l, device=B.out.device) for l in range(len(layers))]
+
+        class LV:
+            pass
+
+        def dec_step(i, ev, Td=Td, Bd=Bd, xs=xs):
+            L = layers[i % len(layers)]
+            lv = LV()
+            lv.x, lv.w_r, lv.bias, lv.w_gu, lv.w_down = xs[i % len(xs)], L.w_r, L.bias, L.w_gu, L.w_down
+            run_step(dm, wl, lv, Bd, 64, 0, 0, None, ev)
+
+        ms, evs = timed(dec_step, n, 5, ws)
+        ffn = statistics.mean(e[0].elapsed_time(e[2]) for e in evs)
+        D = int((Bd.counts[:64] > 0).sum())
+        wbytes = D * 3 * wl.m * wl.d * 2
+        step_bytes = wbytes + wl.E * wl.d * 2 + Td * wl.d * 2 * (2 + 3 * wl.k)
+        out.append({"mode": "decode", "T": Td, "K": 64, "active_experts": D,
+                    "tokens_per_s": round(Td * n / (ms / 1e3), 1), "ms_per_step": round(ms / n, 4),
+                    "step_hbm_frac": round(step_bytes / (ms / n * 1e-3) / 1e9 / pk["hbm_gbs"], 4),
+                    "ffn_ms": round(ffn, 4),
+                    "ffn_hbm_frac": round(wbytes / (ffn * 1e-3) / 1e9 / pk["hbm_gbs"], 4)})
+        del Bd, xs
+    return out
+
+
+def _kernel_hash():
+    import hashlib
+
+    h = hashlib.sha256()
+    for f in ("expert_gemm.cu", "decomoe_internal.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2609_38823_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+# ------------------------------------------------------------------ CPU oracle (baseline and reference arm)
+
+def _oracle_inputs(wl, L_dev_or_none, K, ntok, seed=0):
+    """Host float64 inputs for the oracle: a token sample and the K experts."""
+    from oracle import decomoe_oracle as O  # noqa: F401
+
+    if L_dev_or_none is not None:
+        g = {"x": L_dev_or_none.x.cpu(), "w_r": L_dev_or_none.w_r.cpu(), "bias": L_dev_or_none.bias.cpu()}
+        wgu = L_dev_or_none.w_gu[:K].cpu()
+        m = wl.m
+        G = 128
+        blocks = wgu.view(K, m // G, 2, G, wl.d)
+        wg = blocks[:, :, 0].reshape(K, m, wl.d)
+        wu = blocks[:, :, 1].reshape(K, m, wl.d)
+        wd = L_dev_or_none.w_down[:K].cpu()
+    else:
+        g = W.make_layer(wl, device="cpu")
+        wg, wu, wd = g["w_gate"][:K], g["w_up"][:K], g["w_down"][:K]
+    r = np.random.default_rng(seed)
+    sample = np.sort(r.choice(wl.T, ntok, replace=False))
+    f = lambda t: t.float().numpy().astype(np.float64)  # noqa: E731
+    return (f(g["x"][torch.from_numpy(sample)]).astype(np.float32), f(g["w_r"]).astype(np.float32),
+            g["bias"].numpy(), f(wg), f(wu), f(wd))
+
+
+def _cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(wl, L, K, seconds):
+    from oracle import decomoe_oracle as O
+
+    ntok = 256
+    x, wr, b, wg, wu, wd = _oracle_inputs(wl, L, K, ntok)
+    reps = 0
+    t0 = time.perf_counter()
+    while True:
+        O.moe_layer(x, wr, b, wg, wu, wd, k=wl.k, K=K)
+        reps += 1
+        if time.perf_counter() - t0 >= seconds:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": round(reps * ntok / dt, 2), "unit": "tokens/s", "cores": _cores(), "kind": "oracle",
+            "sample": f"{ntok} of the {wl.T} tokens x {reps} runs ({dt:.1f} s): numpy float64 oracle layer "
+                      f"(router, Eqs. 10-12 routing at K={K}, dispatch, SwiGLU experts, combine); "
+                      f"BLAS threads = all host cores"}
+
+
+def reference(args, ws, rank):
+    if rank != 0:
+        return None
+    from oracle import decomoe_oracle as O
+
+    wl = W.PREFILL
+    K = args.K
+    ntok = 64
+    x, wr, b, wg, wu, wd = _oracle_inputs(wl, None, K, ntok)
+    for _ in range(args.warmup):
+        O.moe_layer(x, wr, b, wg, wu, wd, k=wl.k, K=K)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        O.moe_layer(x, wr, b, wg, wu, wd, k=wl.k, K=K)
+    dt = time.perf_counter() - t0
+    v = round(ntok * args.steps / dt, 2)
+    return {"impl": "reference", "metric": "prefix-MoE layer tokens/s (T=2048 prefill, K=%d of E=128)" % K,
+            "value": v, "unit": "tokens/s", "n_gpus": 0, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(dt / args.steps * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wl.name, "T": wl.T, "d": wl.d, "E": wl.E, "k": wl.k, "m": wl.m, "K": K},
+            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": _cores(), "kind": "oracle",
+                             "sample": f"{ntok} tokens of the {wl.T}-token layer per step"},
+            "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = parse()
+    ws, rank, local = dist_setup(args)
+    if args.impl == "reference":
+        line = reference(args, ws, rank)
+        if line is not None:
+            print(json.dumps(line), flush=True)
+        return
+    line = ours(args, ws, rank, local)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,271 @@
+/*
+ * decomoe.h - C ABI of the DecoMoE prefix-MoE hot path on one GB300 (sm_103a).
+ *
+ * The DecoMoE paper ("DecoMoE: Decoupling Visual Propagation and Expert
+ * Computation for Efficient Multimodal MoE Inference") restricts each MoE
+ * layer after the visual exit to the shortest contiguous prefix [0, K) of
+ * offline mass-reordered experts (RCEP, Section 3.3, Eqs. 10-12, Algorithm 2)
+ * and removes the contiguous visual-token block from the hidden state and the
+ * KV cache at the exit layer (SAVB, Section 3.2). This library computes the
+ * per-layer steps of that path with hand-written CUDA kernels.
+ *
+ * Conventions (every call):
+ *   - extern "C"; every call returns an int status (decomoe_status). No
+ *     exception crosses the ABI. On an error the message of the calling host
+ *     thread is available from decomoe_last_error().
+ *   - The caller owns all memory. Pointers named *_host are host pointers; all
+ *     others are device pointers of the current CUDA device. The library never
+ *     allocates device memory: temporary space comes from a caller-provided
+ *     workspace whose size a *_workspace_bytes() query returns.
+ *   - Device calls are asynchronous on the given stream (NULL = legacy default
+ *     stream). Outputs are valid after the stream is synchronised; inputs must
+ *     stay alive until then. Calls that must read a device value on the host
+ *     (decomoe_moe_layer in mass mode, decomoe_read_status) synchronise the
+ *     stream and say so.
+ *   - Index arrays are int32, row-major. T = tokens of the invocation, d =
+ *     hidden size, E = experts in the pool, K = prefix length, k = top-k width,
+ *     m = expert FFN width.
+ *   - Argument errors (null pointer, k > K, K > E, negative sizes, d or m not a
+ *     multiple of the required granule, misaligned pointer) return
+ *     DECOMOE_ERR_INVALID_ARG before anything is launched.
+ */
+#ifndef DECOMOE_H
+#define DECOMOE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define DECOMOE_API __attribute__((visibility("default")))
+#else
+#define DECOMOE_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* decomoe_stream_t; /* same type as cudaStream_t */
+
+typedef enum {
+  DECOMOE_OK = 0,
+  DECOMOE_ERR_INVALID_ARG = 1, /* bad argument; nothing was launched */
+  DECOMOE_ERR_CUDA = 2,        /* a CUDA launch or API error; see decomoe_last_error() */
+  DECOMOE_ERR_TIMEOUT = 3,     /* a bounded device-side wait ran out (read via decomoe_read_status) */
+  DECOMOE_ERR_UNSUPPORTED = 4, /* a shape or dtype no kernel here takes */
+  DECOMOE_ERR_WORKSPACE = 5,   /* workspace pointer null or smaller than the query says */
+  DECOMOE_ERR_BAD_INPUT = 6    /* device-side input check failed (e.g. expert id >= K) */
+} decomoe_status;
+
+/* Storage dtype of activations and weights. Accumulation is always fp32 (fp64
+ * for the activated mass). */
+enum { DECOMOE_BF16 = 0, DECOMOE_F32 = 1 };
+
+/* Gate/up interleave granule of the fused weight layout (rows of one block). */
+#define DECOMOE_GU_BLOCK 128
+/* Largest expert pool and largest top-k any kernel here takes. */
+#define DECOMOE_MAX_E 256
+#define DECOMOE_MAX_TOPK 32
+
+/* Message of the last failed call made by this host thread ("" if none). */
+DECOMOE_API const char* decomoe_last_error(void);
+
+/* Library ABI version (major*100 + minor). */
+DECOMOE_API int decomoe_version(void);
+
+/* Number of SMs and compute capability of the current device. */
+DECOMOE_API int decomoe_device_info(int* sm_count_host, int* cc_major_host, int* cc_minor_host);
+
+/* ------------------------------------------------------------------------
+ * a1. Router logits over the whole pool (Section 3.1, Eq. 1; the full-pool
+ * router projection stays in every layer, Appendix FLOPs "Scope").
+ *   logits[t, e] = sum_j x[t, j] * w_r[e, j] + bias[e]      (fp32 out)
+ * x: [T, d] row-major, dtype; w_r: [E, d] row-major, dtype, rows in reordered
+ * expert order; bias: [E] fp32 or NULL; logits: [T, E] fp32 row-major.
+ * bf16 with d % 64 == 0 and E in {128, 256} runs on the tensor cores (fp32
+ * accumulate); f32 and other bf16 shapes run a CUDA-core kernel.
+ * status_dev: optional device int32 that collects bounded-wait timeouts.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API int decomoe_router_logits(const void* x, const void* w_r, const float* bias, int64_t T, int d,
+                          int E, int dtype, float* logits, int32_t* status_dev,
+                          decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * a2 + a4. Routing on fp32 logits (Eqs. 10-11; prefix rule of Section 3.3 and
+ * Algorithm 2).
+ *   For every token t: S_t = the k largest of logits[t, 0:K) (largest first;
+ *   equal values: lower expert index first), and
+ *   topk_w[t, j] = exp(l_j - l_0) / sum_j' exp(l_j' - l_0) over the k picks,
+ *   which equals "new softmax over the prefix, top-k, renormalise".
+ *   With K == E this is the full-pool routing of Eq. 10. If mass_out is not
+ *   NULL, mass_out[e] = sum_t of the token's renormalised weight of e (Eq. 11),
+ *   accumulated in fp64 in a fixed order (bit-reproducible run to run);
+ *   mass_out then needs E entries and the workspace.
+ * logits: [T, ld] fp32, entries [0, E) used, ld >= E. topk_idx: [T, k] int32,
+ * values in [0, K). topk_w: [T, k] fp32. Either output may be NULL (e.g. the
+ * mass-only pass). Needs 1 <= k <= K <= E <= 256, k <= 32.
+ * ws: device workspace of decomoe_route_workspace_bytes(T, E) bytes (only when
+ * mass_out != NULL).
+ * ------------------------------------------------------------------------ */
+DECOMOE_API size_t decomoe_route_workspace_bytes(int64_t T, int E);
+DECOMOE_API int decomoe_route_prefix(const float* logits, int64_t T, int E, int64_t ld, int K, int k,
+                         int32_t* topk_idx, float* topk_w, double* mass_out, void* ws,
+                         size_t ws_bytes, decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * a3. Prefix length (Eq. 12), plain C on the host, no CUDA.
+ *   K_hat = min{K in 1..E : sum_{e<K} mass[e] / sum_e mass[e] >= p},
+ *   K = max(k, K_hat). Sums run sequentially over e = 0..E-1 in fp64; p == 1
+ *   gives K_hat = E; a total mass of 0 gives K = k.
+ * mass_host: [E] fp64 host array. Needs 0 < p <= 1, 1 <= k <= E.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API int decomoe_select_prefix(const double* mass_host, int E, int k, double p, int* K_out_host);
+
+/* ------------------------------------------------------------------------
+ * a5. Dispatch: group the T*k (token, slot) pairs by expert (Algorithm 2,
+ * "evaluate ... only the first K expert MLPs").
+ *   counts[e] = #pairs with topk_idx == e (e < K); offsets = exclusive scan,
+ *   offsets[K] = T*k. Rows are ordered by expert, then by flat index
+ *   f = t*k + j (a stable sort). perm_token[r] = token of row r;
+ *   inv_slot[f] = row of pair f; x_perm[r, :] = x[perm_token[r], :].
+ * topk_idx: [T, k] int32 in [0, K) (an id outside it sets DECOMOE_ERR_BAD_INPUT
+ * in status_dev, if given, and that pair is dropped). x: [T, d] dtype (rows
+ * 16-byte aligned); x_perm: [T*k, d] dtype, or NULL to skip the row gather.
+ * counts: [K], offsets: [K+1], perm_token and inv_slot: [T*k] int32.
+ * ws: decomoe_dispatch_workspace_bytes(T, k, K) bytes.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API size_t decomoe_dispatch_workspace_bytes(int64_t T, int k, int K);
+DECOMOE_API int decomoe_dispatch(const int32_t* topk_idx, int64_t T, int k, int K, const void* x, int d,
+                     int dtype, int32_t* counts, int32_t* offsets, int32_t* perm_token,
+                     int32_t* inv_slot, void* x_perm, void* ws, size_t ws_bytes,
+                     int32_t* status_dev, decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * One-time weight layout transform (like the paper's load-time expert
+ * reorder, Section 3.3: it changes storage only, not values).
+ *   w_gate, w_up: [E, m, d] row-major (dtype). w_gate_up: [E, 2m, d], where
+ *   rows [2*G*b, 2*G*b + G) of expert e are gate rows [G*b, G*b + G) and rows
+ *   [2*G*b + G, 2*G*(b+1)) are up rows [G*b, G*b + G), G = DECOMOE_GU_BLOCK.
+ * Needs m % 128 == 0.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API int decomoe_weight_layout(const void* w_gate, const void* w_up, void* w_gate_up, int E, int d,
+                          int m, int dtype, decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * a6. Grouped SwiGLU expert FFN over the prefix experts (Algorithm 2; gate,
+ * up and down matmuls, Appendix C_expert = 6Kdm).
+ *   For every row r in [offsets[e], offsets[e+1]), e < K:
+ *   h_r = silu(W_gate[e] x_r) * (W_up[e] x_r); y_r = W_down[e] h_r.
+ * x_perm: [rows, d]; w_gate_up: [E, 2m, d] in the layout above; w_down:
+ * [E, d, m]; h_ws: [rows, m] dtype (intermediate, caller-owned); y_perm:
+ * [rows, d] dtype. rows = T*k = offsets[K] (upper bound used to size tensor
+ * maps; offsets stay on the device). Experts with no rows cost nothing.
+ * bf16: tcgen05 tensor-core kernels for rows > 64, a weight-streaming kernel
+ * for rows <= 64 (decode); fp32 accumulate, h rounded to bf16. f32: CUDA-core
+ * kernels with h kept in fp32. Needs d % 64 == 0 and m % 128 == 0 (bf16).
+ * status_dev: optional device int32 collecting bounded-wait timeouts.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API int decomoe_expert_swiglu(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d,
+                          int m, int dtype, const void* w_gate_up, const void* w_down, void* h_ws,
+                          void* y_perm, int32_t* status_dev, decomoe_stream_t stream);
+
+/* The two phases of decomoe_expert_swiglu as separate calls (same arguments
+ * and rules): gate/up with the fused SwiGLU epilogue writes h [rows, m]; down
+ * reads h and writes y_perm [rows, d]. */
+DECOMOE_API int decomoe_expert_gate_up(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d,
+                                       int m, int dtype, const void* w_gate_up, void* h, int32_t* status_dev,
+                                       decomoe_stream_t stream);
+DECOMOE_API int decomoe_expert_down(const void* h, const int32_t* offsets, int64_t rows, int K, int d, int m,
+                                    int dtype, const void* w_down, void* y_perm, int32_t* status_dev,
+                                    decomoe_stream_t stream);
+
+/* CUDA-core reference of decomoe_expert_swiglu for bf16 storage: the same
+ * arithmetic (bf16 products, fp32 accumulation, h rounded to bf16) with one
+ * thread per output element and no tensor cores. It is slow; it exists to
+ * localise a disagreement between the tensor-core kernels and the oracle. */
+DECOMOE_API int decomoe_expert_swiglu_ref(const void* x_perm, const int32_t* offsets, int64_t rows, int K,
+                                          int d, int m, const void* w_gate_up, const void* w_down,
+                                          void* h_ws, void* y_perm, decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * a7. Combine (Algorithm 2, "evaluate and combine"): the weighted sum of a
+ * token's k expert outputs, written as a gather (deterministic, no atomics).
+ *   out[t, :] = sum_{j=0..k-1} topk_w[t, j] * y_perm[inv_slot[t*k + j], :]
+ *               (+ residual[t, :])
+ * fp32 sum in slot order j = 0..k-1, rounded once to dtype. residual may be
+ * NULL. out must not alias y_perm.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API int decomoe_combine(const void* y_perm, const int32_t* inv_slot, const float* topk_w, int64_t T,
+                    int k, int d, int dtype, const void* residual, void* out,
+                    decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * a8. Visual-block removal (Section 3.2: the complete visual block leaves the
+ * hidden state and the KV cache; later layers and decoding use the text-only
+ * sequence). Out-of-place, order-preserving row compaction, batched:
+ *   for b < nbatch: dst[b] = rows [0, v0) of src[b] followed by rows
+ *   [v0 + nv, rows) of src[b].
+ * row_bytes: bytes per row; src_batch_stride / dst_batch_stride: bytes between
+ * consecutive batches (rows of one batch are contiguous). src and dst must not
+ * overlap. 0 <= v0, 0 <= nv, v0 + nv <= rows; nv == 0 is a plain copy.
+ * 16-byte aligned pointers, row_bytes and strides take the vector path; any
+ * other alignment takes a byte path.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API int decomoe_drop_visual_block(const void* src, void* dst, int64_t rows, int64_t row_bytes,
+                              int64_t v0, int64_t nv, int64_t nbatch, int64_t src_batch_stride,
+                              int64_t dst_batch_stride, decomoe_stream_t stream);
+
+/* RMSNorm of the attention-free layer stack (a workload choice; the paper
+ * leaves norms out of the method): y[t] = x[t] / sqrt(mean(x[t]^2) + eps),
+ * fp32 math, dtype in and out. y may alias x. */
+DECOMOE_API int decomoe_rmsnorm(const void* x, void* y, int64_t T, int d, float eps, int dtype,
+                    decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Whole RCEP MoE invocation (Algorithm 2, exited branch), chaining a1..a7 on
+ * one stream:
+ *   router logits -> [mass pass -> select prefix] -> prefix routing ->
+ *   dispatch -> grouped SwiGLU -> combine (+ residual).
+ * K_fixed > 0 routes over the fixed prefix [0, K_fixed) (the paper's fixed
+ * keep-ratio experiments) and still runs the mass pass when p > 0 (K_sel_host
+ * then receives the prefix Eq. 12 selects); K_fixed == 0 selects K from p
+ * (0 < p <= 1), which synchronises the stream once to read the mass. p == 0
+ * with K_fixed > 0 skips the mass pass. K_used_host / K_sel_host may be NULL.
+ * x, residual, out: [T, d] dtype (out may alias residual, not x).
+ * ws: decomoe_moe_layer_workspace_bytes(...) bytes; every intermediate
+ * (logits, routes, dispatch arrays, x_perm, h, y_perm) lives there.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API size_t decomoe_moe_layer_workspace_bytes(int64_t T, int d, int E, int k, int m, int dtype);
+DECOMOE_API int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const void* w_gate_up,
+                      const void* w_down, int64_t T, int d, int E, int k, int m, int dtype,
+                      int K_fixed, double p, const void* residual, void* out, int* K_used_host,
+                      int* K_sel_host, void* ws, size_t ws_bytes, int32_t* status_dev,
+                      decomoe_stream_t stream);
+
+/* Offsets (bytes) of the intermediates inside the decomoe_moe_layer workspace,
+ * for inspection: logits, topk_idx, topk_w, mass, counts, offsets, perm_token,
+ * inv_slot, x_perm, h, y_perm (11 entries written to offs_host). */
+DECOMOE_API int decomoe_moe_layer_workspace_layout(int64_t T, int d, int E, int k, int m, int dtype,
+                                       size_t* offs_host);
+
+/* ------------------------------------------------------------------------
+ * Bounded-wait status. Kernels that wait on device barriers give up after a
+ * time limit, record DECOMOE_ERR_TIMEOUT (or DECOMOE_ERR_BAD_INPUT) in the
+ * caller's status word and return, leaving the context usable.
+ * decomoe_read_status synchronises the stream, copies the word to
+ * *code_host, clears it and returns DECOMOE_OK.
+ * decomoe_set_wait_limit_ns sets the limit used by later launches (default
+ * 2e9 ns).
+ * decomoe_selftest_wait launches one kernel that waits on a device barrier
+ * nothing ever completes, with the given limit, so that the timeout path can
+ * be tested without faulting or hanging the GPU.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API int decomoe_read_status(int32_t* status_dev, int32_t* code_host, decomoe_stream_t stream);
+DECOMOE_API int decomoe_set_wait_limit_ns(int64_t limit_ns);
+DECOMOE_API int decomoe_selftest_wait(int32_t* status_dev, int64_t limit_ns, decomoe_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DECOMOE_H */

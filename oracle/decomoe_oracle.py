@@ -220,7 +220,7 @@ def expert_swiglu(x_rows, offsets, w_gate, w_up, w_down):
     x_rows = np.asarray(x_rows, F64)
     R, d = x_rows.shape
     K = len(offsets) - 1
-    y = np.zeros((R, np.asarray(w_down).shape[1]), F64)
+    y = np.zeros((R, d), F64)  # the down projection maps back to width d
     for e in range(K):
         r0, r1 = int(offsets[e]), int(offsets[e + 1])
         if r1 == r0:
@@ -277,7 +277,7 @@ def moe_token(x_t, a_t, w_gate, w_up, w_down, K, k):
     independent once K is fixed). Used for sampled checks at full size."""
     idx, w = route_prefix(np.asarray(a_t)[None, :], K, k)
     x_t = np.asarray(x_t, F64)
-    out = np.zeros(np.asarray(w_down).shape[1], F64)
+    out = np.zeros(x_t.shape[0], F64)
     for j in range(k):
         e = int(idx[0, j])
         g = np.asarray(w_gate[e], F64) @ x_t

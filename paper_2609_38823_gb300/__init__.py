@@ -1,0 +1,328 @@
+"""Python binding of libdecomoe (the DecoMoE prefix-MoE hot path on GB300).
+
+Argument marshalling only: every function here forwards torch tensors' device
+pointers, sizes and the current CUDA stream to the C ABI of include/decomoe.h,
+and raises DecomoeError on a non-zero status. No step of the computation runs
+in Python or in PyTorch ops; PyTorch provides device memory and streams.
+
+The shared library is built in-tree (``__graft_entry__.build()`` or
+``python paper_2609_38823_gb300/_build.py``). Importing this package does not
+need a GPU; calling a device function without the library or without a GPU
+raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import torch
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libdecomoe.so")
+
+DECOMOE_OK = 0
+DECOMOE_ERR_INVALID_ARG = 1
+DECOMOE_ERR_CUDA = 2
+DECOMOE_ERR_TIMEOUT = 3
+DECOMOE_ERR_UNSUPPORTED = 4
+DECOMOE_ERR_WORKSPACE = 5
+DECOMOE_ERR_BAD_INPUT = 6
+DECOMOE_BF16 = 0
+DECOMOE_F32 = 1
+GU_BLOCK = 128
+
+# name -> (restype, argtypes)
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_L = ctypes.c_int64
+_S = ctypes.c_size_t
+_D = ctypes.c_double
+_F = ctypes.c_float
+SIGNATURES = {
+    "decomoe_last_error": (ctypes.c_char_p, []),
+    "decomoe_version": (_I, []),
+    "decomoe_device_info": (_I, [_P, _P, _P]),
+    "decomoe_router_logits": (_I, [_P, _P, _P, _L, _I, _I, _I, _P, _P, _P]),
+    "decomoe_route_workspace_bytes": (_S, [_L, _I]),
+    "decomoe_route_prefix": (_I, [_P, _L, _I, _L, _I, _I, _P, _P, _P, _P, _S, _P]),
+    "decomoe_select_prefix": (_I, [_P, _I, _I, _D, _P]),
+    "decomoe_dispatch_workspace_bytes": (_S, [_L, _I, _I]),
+    "decomoe_dispatch": (_I, [_P, _L, _I, _I, _P, _I, _I, _P, _P, _P, _P, _P, _P, _S, _P, _P]),
+    "decomoe_weight_layout": (_I, [_P, _P, _P, _I, _I, _I, _I, _P]),
+    "decomoe_expert_swiglu": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P]),
+    "decomoe_expert_gate_up": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P]),
+    "decomoe_expert_down": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P]),
+    "decomoe_expert_swiglu_ref": (_I, [_P, _P, _L, _I, _I, _I, _P, _P, _P, _P, _P]),
+    "decomoe_combine": (_I, [_P, _P, _P, _L, _I, _I, _I, _P, _P, _P]),
+    "decomoe_drop_visual_block": (_I, [_P, _P, _L, _L, _L, _L, _L, _L, _L, _P]),
+    "decomoe_rmsnorm": (_I, [_P, _P, _L, _I, _F, _I, _P]),
+    "decomoe_moe_layer_workspace_bytes": (_S, [_L, _I, _I, _I, _I, _I]),
+    "decomoe_moe_layer": (_I, [_P, _P, _P, _P, _P, _L, _I, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P,
+                               _P, _S, _P, _P]),
+    "decomoe_moe_layer_workspace_layout": (_I, [_L, _I, _I, _I, _I, _I, _P]),
+    "decomoe_read_status": (_I, [_P, _P, _P]),
+    "decomoe_set_wait_limit_ns": (_I, [_L]),
+    "decomoe_selftest_wait": (_I, [_P, _L, _P]),
+}
+
+
+class DecomoeError(RuntimeError):
+    def __init__(self, name, code, msg):
+        super().__init__(f"{name} failed with status {code}: {msg}")
+        self.code = code
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load libdecomoe.so (raises if it was not built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError(
+                f"{LIB_PATH} is missing: build it with __graft_entry__.build() "
+                "(the CUDA library is required; there is no fallback)")
+        L = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _check(name, code):
+    if code != DECOMOE_OK:
+        msg = lib().decomoe_last_error()
+        raise DecomoeError(name, code, msg.decode() if msg else "")
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dt(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return DECOMOE_BF16
+    if t.dtype == torch.float32:
+        return DECOMOE_F32
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _need_cuda(*ts):
+    for t in ts:
+        if t is not None:
+            if not t.is_cuda:
+                raise ValueError("device tensors expected")
+            if not t.is_contiguous():
+                raise ValueError("contiguous tensors expected")
+
+
+# ----------------------------------------------------------------- host-only calls
+
+def decomoe_version() -> int:
+    return lib().decomoe_version()
+
+
+def decomoe_select_prefix(mass, k: int, p: float) -> int:
+    """Eq. 12 on the host (plain C): shortest prefix covering mass fraction p."""
+    import numpy as np
+
+    m = np.ascontiguousarray(np.asarray(mass, dtype=np.float64))
+    out = ctypes.c_int(0)
+    _check("decomoe_select_prefix",
+           lib().decomoe_select_prefix(m.ctypes.data_as(ctypes.c_void_p), int(m.shape[0]), int(k),
+                                       float(p), ctypes.byref(out)))
+    return out.value
+
+
+def decomoe_route_workspace_bytes(T: int, E: int) -> int:
+    return lib().decomoe_route_workspace_bytes(T, E)
+
+
+def decomoe_dispatch_workspace_bytes(T: int, k: int, K: int) -> int:
+    return lib().decomoe_dispatch_workspace_bytes(T, k, K)
+
+
+def decomoe_moe_layer_workspace_bytes(T, d, E, k, m, dtype) -> int:
+    return lib().decomoe_moe_layer_workspace_bytes(T, d, E, k, m, dtype)
+
+
+def decomoe_moe_layer_workspace_layout(T, d, E, k, m, dtype):
+    offs = (ctypes.c_size_t * 11)()
+    _check("decomoe_moe_layer_workspace_layout",
+           lib().decomoe_moe_layer_workspace_layout(T, d, E, k, m, dtype, offs))
+    return list(offs)
+
+
+def decomoe_set_wait_limit_ns(limit_ns: int):
+    _check("decomoe_set_wait_limit_ns", lib().decomoe_set_wait_limit_ns(int(limit_ns)))
+
+
+def decomoe_device_info():
+    a, b, c = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+    _check("decomoe_device_info", lib().decomoe_device_info(ctypes.byref(a), ctypes.byref(b), ctypes.byref(c)))
+    return a.value, b.value, c.value
+
+
+# ----------------------------------------------------------------- device calls
+
+def decomoe_router_logits(x, w_r, bias, logits, status=None, stream=None):
+    _need_cuda(x, w_r, bias, logits, status)
+    T, d = x.shape
+    E = w_r.shape[0]
+    _check("decomoe_router_logits",
+           lib().decomoe_router_logits(_ptr(x), _ptr(w_r), _ptr(bias), T, d, E, _dt(x), _ptr(logits),
+                                       _ptr(status), _stream(stream)))
+
+
+def decomoe_route_prefix(logits, K, k, topk_idx=None, topk_w=None, mass_out=None, ws=None, E=None,
+                         stream=None):
+    _need_cuda(logits, topk_idx, topk_w, mass_out, ws)
+    T, ld = logits.shape
+    E = ld if E is None else E
+    ws_bytes = 0 if ws is None else ws.numel() * ws.element_size()
+    _check("decomoe_route_prefix",
+           lib().decomoe_route_prefix(_ptr(logits), T, E, ld, K, k, _ptr(topk_idx), _ptr(topk_w),
+                                      _ptr(mass_out), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def decomoe_dispatch(topk_idx, K, x, counts, offsets, perm_token, inv_slot, x_perm, ws, status=None,
+                     stream=None):
+    _need_cuda(topk_idx, x, counts, offsets, perm_token, inv_slot, x_perm, ws, status)
+    T, k = topk_idx.shape
+    d = x.shape[1] if x is not None else 0
+    dtype = _dt(x) if x is not None else DECOMOE_BF16
+    _check("decomoe_dispatch",
+           lib().decomoe_dispatch(_ptr(topk_idx), T, k, K, _ptr(x), d, dtype, _ptr(counts), _ptr(offsets),
+                                  _ptr(perm_token), _ptr(inv_slot), _ptr(x_perm), _ptr(ws),
+                                  ws.numel() * ws.element_size(), _ptr(status), _stream(stream)))
+
+
+def decomoe_weight_layout(w_gate, w_up, w_gate_up, stream=None):
+    _need_cuda(w_gate, w_up, w_gate_up)
+    E, m, d = w_gate.shape
+    _check("decomoe_weight_layout",
+           lib().decomoe_weight_layout(_ptr(w_gate), _ptr(w_up), _ptr(w_gate_up), E, d, m, _dt(w_gate),
+                                       _stream(stream)))
+
+
+def decomoe_expert_swiglu(x_perm, offsets, K, w_gate_up, w_down, h_ws, y_perm, status=None, stream=None):
+    _need_cuda(x_perm, offsets, w_gate_up, w_down, h_ws, y_perm, status)
+    rows, d = x_perm.shape
+    m = w_down.shape[2]
+    _check("decomoe_expert_swiglu",
+           lib().decomoe_expert_swiglu(_ptr(x_perm), _ptr(offsets), rows, K, d, m, _dt(x_perm),
+                                       _ptr(w_gate_up), _ptr(w_down), _ptr(h_ws), _ptr(y_perm),
+                                       _ptr(status), _stream(stream)))
+
+
+def decomoe_expert_gate_up(x_perm, offsets, K, w_gate_up, h, status=None, stream=None):
+    _need_cuda(x_perm, offsets, w_gate_up, h, status)
+    rows, d = x_perm.shape
+    m = h.shape[1]
+    _check("decomoe_expert_gate_up",
+           lib().decomoe_expert_gate_up(_ptr(x_perm), _ptr(offsets), rows, K, d, m, _dt(x_perm), _ptr(w_gate_up),
+                                        _ptr(h), _ptr(status), _stream(stream)))
+
+
+def decomoe_expert_down(h, offsets, K, w_down, y_perm, status=None, stream=None):
+    _need_cuda(h, offsets, w_down, y_perm, status)
+    rows, m = h.shape
+    d = y_perm.shape[1]
+    _check("decomoe_expert_down",
+           lib().decomoe_expert_down(_ptr(h), _ptr(offsets), rows, K, d, m, _dt(h), _ptr(w_down), _ptr(y_perm),
+                                     _ptr(status), _stream(stream)))
+
+
+def decomoe_expert_swiglu_ref(x_perm, offsets, K, w_gate_up, w_down, h_ws, y_perm, stream=None):
+    _need_cuda(x_perm, offsets, w_gate_up, w_down, h_ws, y_perm)
+    rows, d = x_perm.shape
+    m = w_down.shape[2]
+    _check("decomoe_expert_swiglu_ref",
+           lib().decomoe_expert_swiglu_ref(_ptr(x_perm), _ptr(offsets), rows, K, d, m, _ptr(w_gate_up),
+                                           _ptr(w_down), _ptr(h_ws), _ptr(y_perm), _stream(stream)))
+
+
+def decomoe_combine(y_perm, inv_slot, topk_w, out, residual=None, stream=None):
+    _need_cuda(y_perm, inv_slot, topk_w, out, residual)
+    T, k = topk_w.shape
+    d = out.shape[1]
+    _check("decomoe_combine",
+           lib().decomoe_combine(_ptr(y_perm), _ptr(inv_slot), _ptr(topk_w), T, k, d, _dt(out),
+                                 _ptr(residual), _ptr(out), _stream(stream)))
+
+
+def decomoe_drop_visual_block(src, dst, v0, nv, stream=None):
+    """src: [rows, ...] or [nbatch, rows, ...] contiguous; dst the compacted shape."""
+    _need_cuda(src, dst)
+    if src.dim() >= 3:
+        nbatch, rows = src.shape[0], src.shape[1]
+        row_bytes = src[0, 0].numel() * src.element_size()
+        sstride = src.stride(0) * src.element_size()
+        dstride = dst.stride(0) * dst.element_size()
+    else:
+        nbatch, rows = 1, src.shape[0]
+        row_bytes = (src.numel() // max(rows, 1)) * src.element_size() if rows else src.element_size()
+        sstride = rows * row_bytes
+        dstride = (rows - nv) * row_bytes
+    _check("decomoe_drop_visual_block",
+           lib().decomoe_drop_visual_block(_ptr(src), _ptr(dst), rows, row_bytes, v0, nv, nbatch, sstride,
+                                           dstride, _stream(stream)))
+
+
+def decomoe_rmsnorm(x, y, eps=1e-6, stream=None):
+    _need_cuda(x, y)
+    T, d = x.shape
+    _check("decomoe_rmsnorm", lib().decomoe_rmsnorm(_ptr(x), _ptr(y), T, d, float(eps), _dt(x), _stream(stream)))
+
+
+def decomoe_moe_layer(x, w_r, bias, w_gate_up, w_down, k, out, ws, K_fixed=0, p=0.0, residual=None,
+                      status=None, stream=None):
+    """One RCEP MoE invocation. Returns (K_used, K_selected or None)."""
+    _need_cuda(x, w_r, bias, w_gate_up, w_down, out, ws, residual, status)
+    T, d = x.shape
+    E = w_r.shape[0]
+    m = w_down.shape[2]
+    Ku, Ks = ctypes.c_int(0), ctypes.c_int(-1)
+    _check("decomoe_moe_layer",
+           lib().decomoe_moe_layer(_ptr(x), _ptr(w_r), _ptr(bias), _ptr(w_gate_up), _ptr(w_down), T, d, E,
+                                   k, m, _dt(x), int(K_fixed), float(p), _ptr(residual), _ptr(out),
+                                   ctypes.byref(Ku), ctypes.byref(Ks), _ptr(ws),
+                                   ws.numel() * ws.element_size(), _ptr(status), _stream(stream)))
+    return Ku.value, (Ks.value if Ks.value >= 0 else None)
+
+
+def decomoe_read_status(status, stream=None) -> int:
+    code = ctypes.c_int32(0)
+    _check("decomoe_read_status", lib().decomoe_read_status(_ptr(status), ctypes.byref(code), _stream(stream)))
+    return code.value
+
+
+def decomoe_selftest_wait(status, limit_ns, stream=None):
+    _check("decomoe_selftest_wait", lib().decomoe_selftest_wait(_ptr(status), int(limit_ns), _stream(stream)))
+
+
+# ----------------------------------------------------------------- helpers
+
+def fuse_gate_up(w_gate: torch.Tensor, w_up: torch.Tensor) -> torch.Tensor:
+    """Interleaved gate/up weights [E, 2m, d] made on the device by the library."""
+    E, m, d = w_gate.shape
+    out = torch.empty((E, 2 * m, d), dtype=w_gate.dtype, device=w_gate.device)
+    decomoe_weight_layout(w_gate, w_up, out)
+    return out
+
+
+def workspace(nbytes: int, device) -> torch.Tensor:
+    """A caller-owned device workspace of at least nbytes (256-byte aligned)."""
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)

@@ -1,0 +1,223 @@
+// Dispatch of the routed (token, slot) pairs to the prefix experts: per-tile
+// histograms with warp-aggregated shared-memory atomics, a scan, a stable
+// rank assignment, and a 128-bit row gather (DecoMoE Algorithm 2: only the
+// first K expert MLPs are evaluated, each on the tokens routed to it).
+#include "decomoe_internal.cuh"
+
+namespace decomoe {
+
+constexpr int DSP_THREADS = 256;
+constexpr int DSP_WARPS = DSP_THREADS / 32;
+constexpr int DSP_PER_WARP = 128;                   // consecutive pairs per warp
+constexpr int DSP_TILE = DSP_WARPS * DSP_PER_WARP;  // pairs per block (1024)
+
+// Pass 1: histogram of expert ids in each tile of DSP_TILE consecutive pairs.
+__global__ void __launch_bounds__(DSP_THREADS)
+    k_dispatch_hist(const int32_t* __restrict__ idx, int64_t N, int K,
+                    int32_t* __restrict__ tile_hist, int32_t* status) {
+  __shared__ int hist[DECOMOE_MAX_E];
+  for (int e = threadIdx.x; e < K; e += DSP_THREADS) hist[e] = 0;
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t base = static_cast<int64_t>(blockIdx.x) * DSP_TILE + warp * DSP_PER_WARP;
+#pragma unroll
+  for (int r = 0; r < DSP_PER_WARP / 32; ++r) {
+    const int64_t f = base + r * 32 + lane;
+    int e = -2;
+    if (f < N) {
+      e = idx[f];
+      if (e < 0 || e >= K) {
+        report_status(status, DECOMOE_ERR_BAD_INPUT);
+        e = -1;
+      }
+    }
+    const uint32_t grp = __match_any_sync(0xffffffffu, e);
+    if (e >= 0 && lane == __ffs(grp) - 1) atomicAdd(&hist[e], __popc(grp));
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < K; e += DSP_THREADS)
+    tile_hist[static_cast<int64_t>(blockIdx.x) * K + e] = hist[e];
+}
+
+// Pass 2: every block sums the tile histograms (its own prefix and the total),
+// scans the totals over experts, then ranks its pairs stably: warp w owns
+// pairs [w*128, w*128+128) of the tile in order, ranks inside a 32-pair round
+// come from __match_any_sync, and per-warp running counts are scanned across
+// warps. Writes perm_token and inv_slot; block 0 writes counts and offsets.
+__global__ void __launch_bounds__(DSP_THREADS)
+    k_dispatch_scatter(const int32_t* __restrict__ idx, int64_t N, int k, int K,
+                       const int32_t* __restrict__ tile_hist, int ntiles,
+                       int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
+                       int32_t* __restrict__ perm_token, int32_t* __restrict__ inv_slot) {
+  __shared__ int s_base[DECOMOE_MAX_E];
+  __shared__ int s_wcnt[DSP_WARPS][DECOMOE_MAX_E];
+  __shared__ int s_wsum[DSP_WARPS];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int e_t = threadIdx.x;  // one expert per thread (K <= 256 = DSP_THREADS)
+
+  int tot = 0, before = 0;
+  if (e_t < K) {
+    for (int b = 0; b < ntiles; ++b) {
+      const int v = tile_hist[static_cast<int64_t>(b) * K + e_t];
+      tot += v;
+      if (b < static_cast<int>(blockIdx.x)) before += v;
+    }
+  }
+  // exclusive block scan of tot over experts
+  int incl = tot;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int v = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += v;
+  }
+  if (lane == 31) s_wsum[warp] = incl;
+  for (int e = threadIdx.x; e < K; e += DSP_THREADS)
+    for (int w = 0; w < DSP_WARPS; ++w) s_wcnt[w][e] = 0;
+  __syncthreads();
+  int wpre = 0;
+  for (int w = 0; w < warp; ++w) wpre += s_wsum[w];
+  const int excl = wpre + incl - tot;
+  if (e_t < K) {
+    s_base[e_t] = excl + before;
+    if (blockIdx.x == 0) {
+      counts[e_t] = tot;
+      offsets[e_t] = excl;
+      if (e_t == K - 1) offsets[K] = excl + tot;
+    }
+  }
+  __syncthreads();
+
+  const int64_t base = static_cast<int64_t>(blockIdx.x) * DSP_TILE + warp * DSP_PER_WARP;
+  int rank[DSP_PER_WARP / 32];
+  int ex[DSP_PER_WARP / 32];
+#pragma unroll
+  for (int r = 0; r < DSP_PER_WARP / 32; ++r) {
+    const int64_t f = base + r * 32 + lane;
+    int e = -2;
+    if (f < N) {
+      e = idx[f];
+      if (e < 0 || e >= K) e = -1;
+    }
+    const uint32_t grp = __match_any_sync(0xffffffffu, e);
+    const uint32_t lt = (1u << lane) - 1u;
+    int rk = 0;
+    if (e >= 0) rk = s_wcnt[warp][e] + __popc(grp & lt);
+    __syncwarp();
+    if (e >= 0 && lane == __ffs(grp) - 1) s_wcnt[warp][e] += __popc(grp);
+    __syncwarp();
+    rank[r] = rk;
+    ex[r] = e;
+  }
+  __syncthreads();
+  // per-expert exclusive scan over warps
+  for (int e = threadIdx.x; e < K; e += DSP_THREADS) {
+    int run = 0;
+    for (int w = 0; w < DSP_WARPS; ++w) {
+      const int c = s_wcnt[w][e];
+      s_wcnt[w][e] = run;
+      run += c;
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int r = 0; r < DSP_PER_WARP / 32; ++r) {
+    const int64_t f = base + r * 32 + lane;
+    if (f >= N) continue;
+    const int e = ex[r];
+    if (e >= 0) {
+      const int row = s_base[e] + s_wcnt[warp][e] + rank[r];
+      perm_token[row] = static_cast<int32_t>(f / k);
+      inv_slot[f] = row;
+    } else {
+      inv_slot[f] = -1;
+    }
+  }
+}
+
+// Pass 3: x_perm[r, :] = x[perm_token[r], :], one warp per row, 16-byte
+// vectors, loads of a row issued before its stores.
+__global__ void __launch_bounds__(256)
+    k_gather_rows(const uint4* __restrict__ x, const int32_t* __restrict__ perm_token,
+                  const int32_t* __restrict__ offsets, int K, int vec_per_row,
+                  uint4* __restrict__ x_perm) {
+  const int rows = offsets[K];
+  const int lane = threadIdx.x & 31;
+  const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int nw = (gridDim.x * blockDim.x) >> 5;
+  for (int r = gw; r < rows; r += nw) {
+    const int t = perm_token[r];
+    const uint4* src = x + static_cast<int64_t>(t) * vec_per_row;
+    uint4* dst = x_perm + static_cast<int64_t>(r) * vec_per_row;
+    int c = lane;
+    for (; c + 32 * 7 < vec_per_row; c += 32 * 8) {
+      uint4 v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = __ldg(src + c + 32 * u);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) dst[c + 32 * u] = v[u];
+    }
+    for (; c < vec_per_row; c += 32) dst[c] = __ldg(src + c);
+  }
+}
+
+}  // namespace decomoe
+
+using namespace decomoe;
+
+extern "C" {
+
+size_t decomoe_dispatch_workspace_bytes(int64_t T, int k, int K) {
+  if (T < 0 || k <= 0 || K <= 0) return 0;
+  const int64_t N = T * k;
+  const int64_t ntiles = (N + DSP_TILE - 1) / DSP_TILE;
+  return align_up(static_cast<size_t>(ntiles > 0 ? ntiles : 1) * K * sizeof(int32_t), 256);
+}
+
+int decomoe_dispatch(const int32_t* topk_idx, int64_t T, int k, int K, const void* x, int d,
+                     int dtype, int32_t* counts, int32_t* offsets, int32_t* perm_token,
+                     int32_t* inv_slot, void* x_perm, void* ws, size_t ws_bytes,
+                     int32_t* status_dev, decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(T >= 0 && k >= 1 && k <= DECOMOE_MAX_TOPK, "dispatch: bad T=%lld or k=%d", (long long)T, k);
+  DM_ARG_CHECK(K >= 1 && K <= DECOMOE_MAX_E, "dispatch: K=%d outside [1, %d]", K, DECOMOE_MAX_E);
+  DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "dispatch: bad dtype");
+  DM_ARG_CHECK(counts && offsets, "dispatch: counts/offsets null");
+  const int64_t N = T * k;
+  DM_ARG_CHECK(N < 0x7fffffffLL, "dispatch: T*k too large");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (N == 0) {
+    DM_CUDA_CHECK(cudaMemsetAsync(counts, 0, sizeof(int32_t) * K, s));
+    DM_CUDA_CHECK(cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (K + 1), s));
+    return DECOMOE_OK;
+  }
+  DM_ARG_CHECK(topk_idx && perm_token && inv_slot, "dispatch: null index array");
+  const size_t row_bytes = static_cast<size_t>(d) * dtype_bytes(dtype);
+  if (x_perm != nullptr) {
+    DM_ARG_CHECK(x != nullptr && d > 0, "dispatch: x null or d <= 0");
+    DM_ARG_CHECK(row_bytes % 16 == 0 && aligned16(x) && aligned16(x_perm),
+                 "dispatch: rows must be 16-byte multiples and 16-byte aligned");
+  }
+  if (ws == nullptr || ws_bytes < decomoe_dispatch_workspace_bytes(T, k, K)) {
+    set_error("dispatch: workspace needs %zu bytes", decomoe_dispatch_workspace_bytes(T, k, K));
+    return DECOMOE_ERR_WORKSPACE;
+  }
+  const int ntiles = static_cast<int>((N + DSP_TILE - 1) / DSP_TILE);
+  int32_t* tile_hist = static_cast<int32_t*>(ws);
+  k_dispatch_hist<<<ntiles, DSP_THREADS, 0, s>>>(topk_idx, N, K, tile_hist, status_dev);
+  DM_LAUNCH_CHECK("k_dispatch_hist");
+  k_dispatch_scatter<<<ntiles, DSP_THREADS, 0, s>>>(topk_idx, N, k, K, tile_hist, ntiles, counts,
+                                                    offsets, perm_token, inv_slot);
+  DM_LAUNCH_CHECK("k_dispatch_scatter");
+  if (x_perm != nullptr) {
+    const int vec = static_cast<int>(row_bytes / 16);
+    const int64_t want_warps = N;
+    int blocks = static_cast<int>(std::min<int64_t>((want_warps * 32 + 255) / 256, sm_count() * 8LL));
+    if (blocks < 1) blocks = 1;
+    k_gather_rows<<<blocks, 256, 0, s>>>(static_cast<const uint4*>(x), perm_token, offsets, K, vec,
+                                         static_cast<uint4*>(x_perm));
+    DM_LAUNCH_CHECK("k_gather_rows");
+  }
+  return DECOMOE_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,895 @@
+// Grouped expert GEMMs of the prefix-MoE layer (DecoMoE Algorithm 2: evaluate
+// only the first K physically contiguous expert MLPs; gate, up and down
+// matmuls, Appendix C_expert = 6Kdm) and the bf16 router projection.
+//
+// bf16, many rows: a persistent warp-specialised tcgen05 kernel.
+//   warp 0      TMA producer: A tile (128 rows x 64) and B tile (BN rows x 64)
+//               per k-block into a STAGES-deep shared-memory ring (128-byte
+//               swizzle), completion on mbarriers.
+//   warp 1      TMEM allocator and MMA issuer: one thread issues
+//               tcgen05.mma.cta_group::1.kind::f16 (M=128, N=BN, K=16) into a
+//               double-buffered fp32 accumulator in tensor memory.
+//   warps 2..5  epilogue: tcgen05.ld of the accumulator (one TMEM lane
+//               quarter per warp, one row per thread), fused SwiGLU / bf16 /
+//               fp32+bias conversion, stores to global.
+// Tiles: for every group (expert) g, ceil(rows_g / 128) M-tiles times
+// N / BN N-tiles; see tile_coords for the order. Rows past the group's end are
+// computed on whatever TMA loaded (zeros past the tensor end) and never
+// stored.
+// bf16, few rows (decode): weight-streaming CUDA-core kernels.
+// f32: CUDA-core kernels (exact fp32 products, fp32 accumulation).
+#include <mutex>
+
+#include <cudaTypedefs.h>
+
+#include "decomoe_internal.cuh"
+
+namespace decomoe {
+
+// ------------------------------------------------------------------ TMA maps
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor [outer, inner] row-major; box = box_outer rows x box_inner
+// columns (64 -> 128-byte swizzle, 32 -> 64-byte swizzle), zero fill out of
+// bounds.
+static int make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
+                          uint32_t box_outer, uint32_t box_inner) {
+  auto fn = encode_fn();
+  if (fn == nullptr) {
+    set_error("cuTensorMapEncodeTiled is not available from the driver");
+    return DECOMOE_ERR_CUDA;
+  }
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  const CUtensorMapSwizzle sw = box_inner == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+                  estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    set_error("cuTensorMapEncodeTiled failed (%d): inner=%llu outer=%llu box=%ux%u", (int)r,
+              (unsigned long long)inner, (unsigned long long)outer, box_outer, box_inner);
+    return DECOMOE_ERR_CUDA;
+  }
+  return DECOMOE_OK;
+}
+
+// ------------------------------------------------------------------ tcgen05 GEMM
+// EPI_SWIGLU: columns [0, BN/2) gate, [BN/2, BN) up -> bf16 silu(g)*u.
+// EPI_BF16: bf16 store. EPI_F32_BIAS: fp32 + bias[col]. EPI_F32_BIAS_T: the
+// accumulator is the transpose of the output (A = router rows, B = tokens):
+// out[col * ld + row] = acc + bias[row], columns >= n_valid skipped.
+enum { EPI_SWIGLU = 0, EPI_BF16 = 1, EPI_F32_BIAS = 2, EPI_F32_BIAS_T = 3 };
+
+struct TcArgs {
+  const int32_t* offsets;  // [ngroups + 1] row offsets (device) or null: one group [0, rows)
+  int ngroups;
+  int rows;
+  int n_per_group;  // B rows per group
+  int kdim;
+  void* out;
+  int64_t out_ld;  // elements
+  const float* bias;
+  int32_t* status;
+  uint64_t limit_ns;
+  int n_valid;  // EPI_F32_BIAS_T: number of valid output columns (tokens)
+};
+
+template <int BN, int STAGES, int BK_>
+struct TcCfg {
+  static constexpr int BM = 128, BK = BK_;
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int TMEM_COLS = 2 * BN;  // two accumulator buffers
+  static constexpr int MAXG = DECOMOE_MAX_E;
+  static constexpr int NBARS = 2 * STAGES + 5;
+  static constexpr size_t SMEM =
+      1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + NBARS * 8 + 2 * (MAXG + 1) * 4 + 16;
+};
+
+// Work item -> (group, M-tile inside the group, N-tile). M-tiles are visited
+// alternately from the two ends of the group-ordered list (first, last,
+// second, second-to-last, ...), each with all its N-tiles back to back. With
+// experts ordered by routed mass, the front holds large experts whose weight
+// tiles are shared by many M-tiles (L2 / tensor bound) and the back small
+// experts whose weights stream from HBM once; mixing them in every wave keeps
+// both HBM and the tensor pipes busy instead of running the two phases one
+// after the other.
+__device__ __forceinline__ void tile_coords(int tile, int NT, const int* s_mt, int G, int& grp, int& mt,
+                                            int& nb) {
+  const int j = tile / NT;
+  nb = tile - j * NT;
+  const int mtot = s_mt[G];
+  const int mtg = (j & 1) ? (mtot - 1 - (j >> 1)) : (j >> 1);
+  int lo = 0, hi = G - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (s_mt[mid] <= mtg)
+      lo = mid;
+    else
+      hi = mid - 1;
+  }
+  grp = lo;
+  mt = mtg - s_mt[lo];
+}
+
+template <int BN, int EPI, int STAGES, int BK>
+__global__ void __launch_bounds__(192, 1)
+    k_gemm_tc(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b,
+              const TcArgs g) {
+  using C = TcCfg<BN, STAGES, BK>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
+  uint8_t* smem = smem_raw + pad;
+  const uint32_t sA = raw + pad;
+  const uint32_t sB = sA + STAGES * C::A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
+  int* s_off = reinterpret_cast<int*>(bars + C::NBARS);
+  int* s_mt = s_off + (C::MAXG + 1);
+  volatile uint32_t* s_tmem = reinterpret_cast<volatile uint32_t*>(s_mt + (C::MAXG + 1));
+  volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t bar0 = smem_u32(bars);
+  // barrier slots: full[STAGES] | empty[STAGES] | tfull[2] | tempty[2] | drain
+#define FULL_BAR(s) (bar0 + 8u * (s))
+#define EMPTY_BAR(s) (bar0 + 8u * (STAGES + (s)))
+#define TFULL_BAR(a) (bar0 + 8u * (2 * STAGES + (a)))
+#define TEMPTY_BAR(a) (bar0 + 8u * (2 * STAGES + 2 + (a)))
+#define DRAIN_BAR (bar0 + 8u * (2 * STAGES + 4))
+
+  const int G = g.ngroups;
+  for (int i = threadIdx.x; i <= G; i += blockDim.x)
+    s_off[i] = (g.offsets != nullptr) ? g.offsets[i] : (i == 0 ? 0 : g.rows);
+  if (threadIdx.x == 0) {
+    *s_abort = 0;
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(FULL_BAR(s), 1);
+      mbar_init(EMPTY_BAR(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(TFULL_BAR(a), 1);
+      mbar_init(TEMPTY_BAR(a), 128);
+    }
+    mbar_init(DRAIN_BAR, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (warp == 2) {
+    // exclusive scan of M-tiles per group: s_mt[g] = first global M-tile of g
+    const int per = (G + 31) / 32;  // <= 8
+    int loc[8];
+    int sum = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      loc[i] = 0;
+      const int gi = lane * per + i;
+      if (i < per && gi < G) {
+        const int n = s_off[gi + 1] - s_off[gi];
+        loc[i] = n > 0 ? (n + C::BM - 1) / C::BM : 0;
+      }
+      sum += loc[i];
+    }
+    int incl = sum;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += v;
+    }
+    int run = incl - sum;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int gi = lane * per + i;
+      if (i < per && gi < G) s_mt[gi] = run;
+      run += loc[i];
+    }
+    if (lane == 31) s_mt[G] = incl;
+  }
+  __syncthreads();
+  const int NT = g.n_per_group / BN;
+  const int total = s_mt[G] * NT;
+  if (static_cast<int>(blockIdx.x) >= total) return;  // before any TMEM or TMA use
+
+  if (warp == 1) {
+    tmem_alloc(smem_u32(const_cast<uint32_t*>(s_tmem)), C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *s_tmem;
+  const int KB = g.kdim / C::BK;
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------ TMA producer
+    tma_prefetch_desc(&tma_a);
+    tma_prefetch_desc(&tma_b);
+    int stage = 0;
+    uint32_t ph = 0;
+    bool ok = true;
+    uint32_t armed = 0;  // bit s: stage s was ever filled
+    uint32_t armed_ph = 0;
+    for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+      int grp, mt, nb;
+      tile_coords(tile, NT, s_mt, G, grp, mt, nb);
+      const int row0 = s_off[grp] + mt * C::BM;
+      const int brow = grp * g.n_per_group + nb * BN;
+      for (int kb = 0; kb < KB; ++kb) {
+        if (!mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(FULL_BAR(stage), C::STAGE_BYTES);
+        tma_load_2d(sA + stage * C::A_BYTES, &tma_a, FULL_BAR(stage), kb * C::BK, row0);
+        tma_load_2d(sB + stage * C::B_BYTES, &tma_b, FULL_BAR(stage), kb * C::BK, brow);
+        armed |= 1u << stage;
+        armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
+        if (++stage == STAGES) {
+          stage = 0;
+          ph ^= 1u;
+        }
+      }
+    }
+    if (!ok) {
+      *s_abort = 1;
+      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+      // let every copy this thread started land before the CTA can exit
+      int no_abort = 0;
+      for (int s = 0; s < STAGES; ++s)
+        if ((armed >> s) & 1u) mbar_wait(FULL_BAR(s), (armed_ph >> s) & 1u, g.limit_ns, &no_abort);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ------------------------------------------------ MMA issuer
+    constexpr uint32_t IDESC = idesc_bf16_f32(C::BM, BN);
+    int stage = 0;
+    uint32_t ph = 0;
+    bool ok = true, issued = false;
+    int it = 0;
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
+      const int acc = it & 1;
+      const uint32_t aph = (it >> 1) & 1;
+      if (!mbar_wait(TEMPTY_BAR(acc), aph ^ 1u, g.limit_ns, s_abort)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t dt = tmem_base + static_cast<uint32_t>(acc * BN);
+      for (int kb = 0; kb < KB; ++kb) {
+        if (!mbar_wait(FULL_BAR(stage), ph, g.limit_ns, s_abort)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint64_t ad = smem_desc_kmajor<BK>(sA + stage * C::A_BYTES);
+        const uint64_t bd = smem_desc_kmajor<BK>(sB + stage * C::B_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < C::BK / 16; ++kk)
+          tc_mma_f16(dt, ad + 2u * kk, bd + 2u * kk, IDESC, (kb | kk) != 0 ? 1u : 0u);
+        tc_commit(EMPTY_BAR(stage));
+        issued = true;
+        if (++stage == STAGES) {
+          stage = 0;
+          ph ^= 1u;
+        }
+      }
+      if (!ok) break;
+      tc_commit(TFULL_BAR(acc));
+    }
+    if (!ok) {
+      *s_abort = 1;
+      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+      if (issued) {
+        int no_abort = 0;
+        tc_commit(DRAIN_BAR);
+        mbar_wait(DRAIN_BAR, 0, g.limit_ns, &no_abort);
+      }
+    }
+  } else if (warp >= 2) {
+    // ------------------------------------------------ epilogue
+    const int q = warp & 3;  // TMEM lanes [32q, 32q + 32) belong to this warp
+    int it = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
+      const int acc = it & 1;
+      const uint32_t aph = (it >> 1) & 1;
+      int grp, mt, nb;
+      tile_coords(tile, NT, s_mt, G, grp, mt, nb);
+      const int row0 = s_off[grp] + mt * C::BM;
+      const int row_end = s_off[grp + 1];
+      if (!mbar_wait(TFULL_BAR(acc), aph, g.limit_ns, s_abort)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const int grow = row0 + q * 32 + lane;
+      const bool valid = grow < row_end;
+      const uint32_t tb =
+          tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
+      if constexpr (EPI == EPI_SWIGLU) {
+        // columns [0, BN/2) gate, [BN/2, BN) up of features nb*BN/2 + c
+        __nv_bfloat16* out = static_cast<__nv_bfloat16*>(g.out);
+#pragma unroll 1
+        for (int c = 0; c < BN / 2; c += 32) {
+          uint32_t gr[32], ur[32];
+          tmem_ld32(tb + c, gr);
+          tmem_ld32(tb + BN / 2 + c, ur);
+          tc_wait_ld();
+          uint32_t pk[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const float g0 = __uint_as_float(gr[2 * i]), g1 = __uint_as_float(gr[2 * i + 1]);
+            const float u0 = __uint_as_float(ur[2 * i]), u1 = __uint_as_float(ur[2 * i + 1]);
+            pk[i] = pack_bf16x2(silu_f(g0) * u0, silu_f(g1) * u1);
+          }
+          if (valid) {
+            uint4* dst = reinterpret_cast<uint4*>(out + static_cast<int64_t>(grow) * g.out_ld +
+                                                  nb * (BN / 2) + c);
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+              dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+          }
+        }
+      } else if constexpr (EPI == EPI_BF16) {
+        __nv_bfloat16* out = static_cast<__nv_bfloat16*>(g.out);
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t r[32];
+          tmem_ld32(tb + c, r);
+          tc_wait_ld();
+          uint32_t pk[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i)
+            pk[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
+          if (valid) {
+            uint4* dst =
+                reinterpret_cast<uint4*>(out + static_cast<int64_t>(grow) * g.out_ld + nb * BN + c);
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+              dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+          }
+        }
+      } else if constexpr (EPI == EPI_F32_BIAS_T) {
+        // row = router row (expert), columns = tokens nb*BN + c
+        float* out = static_cast<float*>(g.out);
+        const float bv = (valid && g.bias) ? g.bias[grow] : 0.f;
+        const int n0 = nb * BN;
+        if constexpr (BN == 16) {
+          uint32_t r[16];
+          tmem_ld16(tb, r);
+          tc_wait_ld();
+          if (valid) {
+#pragma unroll
+            for (int c = 0; c < 16; ++c)
+              if (n0 + c < g.n_valid) out[static_cast<int64_t>(n0 + c) * g.out_ld + grow] = __uint_as_float(r[c]) + bv;
+          }
+        } else {
+#pragma unroll 1
+          for (int c0 = 0; c0 < BN; c0 += 32) {
+            uint32_t r[32];
+            tmem_ld32(tb + c0, r);
+            tc_wait_ld();
+            if (valid) {
+#pragma unroll
+              for (int c = 0; c < 32; ++c)
+                if (n0 + c0 + c < g.n_valid)
+                  out[static_cast<int64_t>(n0 + c0 + c) * g.out_ld + grow] = __uint_as_float(r[c]) + bv;
+            }
+          }
+        }
+      } else {
+        float* out = static_cast<float*>(g.out);
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t r[32];
+          tmem_ld32(tb + c, r);
+          tc_wait_ld();
+          if (valid) {
+            float4* dst =
+                reinterpret_cast<float4*>(out + static_cast<int64_t>(grow) * g.out_ld + nb * BN + c);
+            const float* bptr = g.bias ? g.bias + nb * BN + c : nullptr;
+#pragma unroll
+            for (int v = 0; v < 8; ++v) {
+              float4 o;
+              o.x = __uint_as_float(r[4 * v + 0]) + (bptr ? bptr[4 * v + 0] : 0.f);
+              o.y = __uint_as_float(r[4 * v + 1]) + (bptr ? bptr[4 * v + 1] : 0.f);
+              o.z = __uint_as_float(r[4 * v + 2]) + (bptr ? bptr[4 * v + 2] : 0.f);
+              o.w = __uint_as_float(r[4 * v + 3]) + (bptr ? bptr[4 * v + 3] : 0.f);
+              dst[v] = o;
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(TEMPTY_BAR(acc));
+    }
+    if (!ok) {
+      *s_abort = 1;
+      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+#undef FULL_BAR
+#undef EMPTY_BAR
+#undef TFULL_BAR
+#undef TEMPTY_BAR
+#undef DRAIN_BAR
+}
+
+template <int BN, int EPI, int STAGES, int BK>
+static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b_rows,
+                     const int32_t* offsets, int ngroups, int n_per_group, void* out,
+                     int64_t out_ld, const float* bias, int32_t* status, cudaStream_t s, int n_valid = 0) {
+  using C = TcCfg<BN, STAGES, BK>;
+  CUtensorMap ta, tb;
+  DM_RET(make_tmap_bf16(&ta, A, static_cast<uint64_t>(kdim), static_cast<uint64_t>(rows), C::BM, BK));
+  DM_RET(make_tmap_bf16(&tb, B, static_cast<uint64_t>(kdim), static_cast<uint64_t>(b_rows), BN, BK));
+  TcArgs g;
+  g.offsets = offsets;
+  g.ngroups = ngroups;
+  g.rows = rows;
+  g.n_per_group = n_per_group;
+  g.kdim = kdim;
+  g.out = out;
+  g.out_ld = out_ld;
+  g.bias = bias;
+  g.status = status;
+  g.limit_ns = static_cast<uint64_t>(wait_limit_ns());
+  g.n_valid = n_valid;
+  auto kern = k_gemm_tc<BN, EPI, STAGES, BK>;
+  static_assert(C::SMEM <= 232448, "shared memory budget");
+  DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(C::SMEM)));
+  const int64_t ub_tiles =
+      (static_cast<int64_t>(rows) / C::BM + ngroups) * static_cast<int64_t>(n_per_group / BN);
+  const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(sm_count(), ub_tiles)));
+  kern<<<grid, 192, C::SMEM, s>>>(ta, tb, g);
+  DM_LAUNCH_CHECK("k_gemm_tc");
+  return DECOMOE_OK;
+}
+
+bool router_tc_supported(int d, int E) { return d % 64 == 0 && (E == 128 || E == 256); }
+
+// Router on the tensor cores with the router rows as the M operand (E = 128
+// or 256 rows, one or two M tiles) and the tokens as N tiles of BN columns, so
+// that T = 2048 already spreads over 128 CTAs; the epilogue writes the
+// transpose, logits[t, e], 32 experts of one token per warp store.
+template <int BN>
+static int launch_router_bn(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E,
+                            float* logits, int32_t* status, cudaStream_t s) {
+  const int64_t npad = (T + BN - 1) / BN * BN;
+  return launch_tc<BN, EPI_F32_BIAS_T, 8, 64>(w_r, E, d, x, T, nullptr, 1, static_cast<int>(npad), logits, E,
+                                              bias, status, s, static_cast<int>(T));
+}
+
+int launch_router_tc(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E,
+                     float* logits, int32_t* status, cudaStream_t s) {
+  if (T > 0x7fffff00LL) {
+    set_error("router_logits: T too large for the tensor-core path");
+    return DECOMOE_ERR_UNSUPPORTED;
+  }
+  const int64_t ctas = sm_count();
+  if (T <= 16 * ctas) return launch_router_bn<16>(x, w_r, bias, T, d, E, logits, status, s);
+  if (T <= 32 * ctas) return launch_router_bn<32>(x, w_r, bias, T, d, E, logits, status, s);
+  return launch_router_bn<64>(x, w_r, bias, T, d, E, logits, status, s);
+}
+
+// ------------------------------------------------------------------ CUDA-core paths
+template <typename T>
+__device__ __forceinline__ float ld_f(const T* p);
+template <>
+__device__ __forceinline__ float ld_f<float>(const float* p) { return *p; }
+template <>
+__device__ __forceinline__ float ld_f<__nv_bfloat16>(const __nv_bfloat16* p) {
+  return __bfloat162float(*p);
+}
+template <typename T>
+__device__ __forceinline__ T from_f(float v);
+template <>
+__device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+
+__device__ __forceinline__ int find_group(const int32_t* __restrict__ offsets, int G, int r) {
+  int lo = 0, hi = G - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (offsets[mid] <= r)
+      lo = mid;
+    else
+      hi = mid - 1;
+  }
+  return lo;
+}
+
+// h[r, f] = silu(W_gate[e] x_r)_f * (W_up[e] x_r)_f with the interleaved gate/up
+// layout. One thread per (row, feature).
+template <typename T>
+__global__ void k_simt_gate_up(const T* __restrict__ A, const int32_t* __restrict__ offsets, int G,
+                               const T* __restrict__ Wgu, int d, int m, T* __restrict__ H) {
+  const int rows = offsets[G];
+  const int f = blockIdx.x * blockDim.x + threadIdx.x;
+  if (f >= m) return;
+  for (int r = blockIdx.y; r < rows; r += gridDim.y) {
+    const int e = find_group(offsets, G, r);
+    const int blk = f / DECOMOE_GU_BLOCK, i = f % DECOMOE_GU_BLOCK;
+    const int64_t grow = static_cast<int64_t>(e) * 2 * m + blk * 2 * DECOMOE_GU_BLOCK + i;
+    const T* wg = Wgu + grow * d;
+    const T* wu = wg + static_cast<int64_t>(DECOMOE_GU_BLOCK) * d;
+    const T* x = A + static_cast<int64_t>(r) * d;
+    float ag = 0.f, au = 0.f;
+    for (int j = 0; j < d; ++j) {
+      const float xv = ld_f(x + j);
+      ag = fmaf(xv, ld_f(wg + j), ag);
+      au = fmaf(xv, ld_f(wu + j), au);
+    }
+    const float hv = ag / (1.0f + expf(-ag)) * au;
+    H[static_cast<int64_t>(r) * m + f] = from_f<T>(hv);
+  }
+}
+
+// y[r, n] = sum_f W_down[e][n, f] h[r, f]. One thread per (row, output).
+template <typename T>
+__global__ void k_simt_down(const T* __restrict__ H, const int32_t* __restrict__ offsets, int G,
+                            const T* __restrict__ Wd, int d, int m, T* __restrict__ Y) {
+  const int rows = offsets[G];
+  const int n = blockIdx.x * blockDim.x + threadIdx.x;
+  if (n >= d) return;
+  for (int r = blockIdx.y; r < rows; r += gridDim.y) {
+    const int e = find_group(offsets, G, r);
+    const T* w = Wd + (static_cast<int64_t>(e) * d + n) * m;
+    const T* h = H + static_cast<int64_t>(r) * m;
+    float acc = 0.f;
+    for (int f = 0; f < m; ++f) acc = fmaf(ld_f(h + f), ld_f(w + f), acc);
+    Y[static_cast<int64_t>(r) * d + n] = from_f<T>(acc);
+  }
+}
+
+// ------------------------------------------------------------------ decode path
+// Few rows per expert: stream each weight row once with 16-byte non-allocating
+// loads, dot it with the expert's (at most 8 at a time) activation rows held
+// in shared memory. One warp per output feature pair.
+constexpr int DEC_THREADS = 256;
+constexpr int DEC_FEAT_PER_BLOCK = 16;  // 8 warps x 2 features
+constexpr int DEC_NMAX = 8;
+
+__device__ __forceinline__ uint4 ldg_stream(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+__device__ __forceinline__ float dot8(const uint4& w, const uint4& x) {
+  float s = bf16_lo(w.x) * bf16_lo(x.x);
+  s = fmaf(bf16_hi(w.x), bf16_hi(x.x), s);
+  s = fmaf(bf16_lo(w.y), bf16_lo(x.y), s);
+  s = fmaf(bf16_hi(w.y), bf16_hi(x.y), s);
+  s = fmaf(bf16_lo(w.z), bf16_lo(x.z), s);
+  s = fmaf(bf16_hi(w.z), bf16_hi(x.z), s);
+  s = fmaf(bf16_lo(w.w), bf16_lo(x.w), s);
+  s = fmaf(bf16_hi(w.w), bf16_hi(x.w), s);
+  return s;
+}
+
+// acc[i] += row(w) . xs[i] for i < NC; w rows of `vec` 16-byte vectors.
+template <int NC>
+__device__ __forceinline__ void dec_dot_rows(const uint4* __restrict__ w0, const uint4* __restrict__ w1,
+                                             const uint4* xs, int vec, int lane, float (&a0)[DEC_NMAX],
+                                             float (&a1)[DEC_NMAX]) {
+#pragma unroll
+  for (int i = 0; i < DEC_NMAX; ++i) a0[i] = a1[i] = 0.f;
+  int v = lane;
+  for (; v + 32 * 3 < vec; v += 32 * 4) {
+    uint4 p[4], q[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      p[u] = ldg_stream(w0 + v + 32 * u);
+      q[u] = ldg_stream(w1 + v + 32 * u);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+      for (int i = 0; i < NC; ++i) {
+        const uint4 xv = xs[i * vec + v + 32 * u];
+        a0[i] += dot8(p[u], xv);
+        a1[i] += dot8(q[u], xv);
+      }
+  }
+  for (; v < vec; v += 32) {
+    const uint4 p = ldg_stream(w0 + v), q = ldg_stream(w1 + v);
+#pragma unroll
+    for (int i = 0; i < NC; ++i) {
+      const uint4 xv = xs[i * vec + v];
+      a0[i] += dot8(p, xv);
+      a1[i] += dot8(q, xv);
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < NC; ++i)
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      a0[i] += __shfl_xor_sync(0xffffffffu, a0[i], off);
+      a1[i] += __shfl_xor_sync(0xffffffffu, a1[i], off);
+    }
+}
+
+// Gate/up for decode: block (feature block, expert). Each warp computes two
+// features f: gate row and up row of f together, h = silu(g) * u.
+__global__ void __launch_bounds__(DEC_THREADS)
+    k_dec_gate_up(const __nv_bfloat16* __restrict__ X, const int32_t* __restrict__ offsets,
+                  const __nv_bfloat16* __restrict__ Wgu, int d, int m, __nv_bfloat16* __restrict__ H) {
+  extern __shared__ uint4 xs[];  // [DEC_NMAX][d / 8]
+  const int e = blockIdx.y;
+  const int r0 = offsets[e];
+  const int n_e = offsets[e + 1] - r0;
+  if (n_e <= 0) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int vec = d / 8;
+  for (int c0 = 0; c0 < n_e; c0 += DEC_NMAX) {
+    const int nc = min(DEC_NMAX, n_e - c0);
+    __syncthreads();
+    for (int i = threadIdx.x; i < nc * vec; i += DEC_THREADS) {
+      const int rr = i / vec, v = i - rr * vec;
+      xs[rr * vec + v] = reinterpret_cast<const uint4*>(X + static_cast<int64_t>(r0 + c0 + rr) * d)[v];
+    }
+    __syncthreads();
+#pragma unroll 1
+    for (int ff = 0; ff < 2; ++ff) {
+      const int f = blockIdx.x * DEC_FEAT_PER_BLOCK + warp * 2 + ff;
+      if (f >= m) break;
+      const int blk = f / DECOMOE_GU_BLOCK, i = f % DECOMOE_GU_BLOCK;
+      const int64_t grow = static_cast<int64_t>(e) * 2 * m + blk * 2 * DECOMOE_GU_BLOCK + i;
+      const uint4* wg = reinterpret_cast<const uint4*>(Wgu + grow * d);
+      const uint4* wu = reinterpret_cast<const uint4*>(Wgu + (grow + DECOMOE_GU_BLOCK) * d);
+      float ag[DEC_NMAX], au[DEC_NMAX];
+      switch (nc) {
+        case 1: dec_dot_rows<1>(wg, wu, xs, vec, lane, ag, au); break;
+        case 2: dec_dot_rows<2>(wg, wu, xs, vec, lane, ag, au); break;
+        case 3: case 4: dec_dot_rows<4>(wg, wu, xs, vec, lane, ag, au); break;
+        default: dec_dot_rows<8>(wg, wu, xs, vec, lane, ag, au); break;
+      }
+#pragma unroll
+      for (int rr = 0; rr < DEC_NMAX; ++rr)
+        if (lane == rr && rr < nc)
+          H[static_cast<int64_t>(r0 + c0 + rr) * m + f] =
+              __float2bfloat16_rn(silu_f(ag[rr]) * au[rr]);
+    }
+  }
+}
+
+// Down projection for decode: block (output block, expert); each warp two
+// output features n, rows of W_down of m elements.
+__global__ void __launch_bounds__(DEC_THREADS)
+    k_dec_down(const __nv_bfloat16* __restrict__ H, const int32_t* __restrict__ offsets,
+               const __nv_bfloat16* __restrict__ Wd, int d, int m, __nv_bfloat16* __restrict__ Y) {
+  extern __shared__ uint4 hs[];  // [DEC_NMAX][m / 8]
+  const int e = blockIdx.y;
+  const int r0 = offsets[e];
+  const int n_e = offsets[e + 1] - r0;
+  if (n_e <= 0) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int vec = m / 8;
+  for (int c0 = 0; c0 < n_e; c0 += DEC_NMAX) {
+    const int nc = min(DEC_NMAX, n_e - c0);
+    __syncthreads();
+    for (int i = threadIdx.x; i < nc * vec; i += DEC_THREADS) {
+      const int rr = i / vec, v = i - rr * vec;
+      hs[rr * vec + v] = reinterpret_cast<const uint4*>(H + static_cast<int64_t>(r0 + c0 + rr) * m)[v];
+    }
+    __syncthreads();
+    const int n0 = blockIdx.x * DEC_FEAT_PER_BLOCK + warp * 2;
+    if (n0 >= d) continue;
+    const uint4* w0 = reinterpret_cast<const uint4*>(Wd + (static_cast<int64_t>(e) * d + n0) * m);
+    const uint4* w1 = reinterpret_cast<const uint4*>(Wd + (static_cast<int64_t>(e) * d + n0 + 1) * m);
+    float a0[DEC_NMAX], a1[DEC_NMAX];
+    switch (nc) {
+      case 1: dec_dot_rows<1>(w0, w1, hs, vec, lane, a0, a1); break;
+      case 2: dec_dot_rows<2>(w0, w1, hs, vec, lane, a0, a1); break;
+      case 3: case 4: dec_dot_rows<4>(w0, w1, hs, vec, lane, a0, a1); break;
+      default: dec_dot_rows<8>(w0, w1, hs, vec, lane, a0, a1); break;
+    }
+#pragma unroll
+    for (int rr = 0; rr < DEC_NMAX; ++rr)
+      if (lane == rr && rr < nc) {
+        __nv_bfloat162 o = __floats2bfloat162_rn(a0[rr], a1[rr]);
+        *reinterpret_cast<__nv_bfloat162*>(Y + static_cast<int64_t>(r0 + c0 + rr) * d + n0) = o;
+      }
+  }
+}
+
+// ------------------------------------------------------------------ weight layout
+__global__ void k_weight_layout(const uint4* __restrict__ wg, const uint4* __restrict__ wu,
+                                uint4* __restrict__ wgu, int E, int m, int vec) {
+  const int64_t rows_out = static_cast<int64_t>(E) * 2 * m;
+  const int lane = threadIdx.x & 31;
+  const int64_t gw = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  for (int64_t ro = gw; ro < rows_out; ro += nw) {
+    const int64_t e = ro / (2 * m);
+    const int rr = static_cast<int>(ro - e * 2 * m);
+    const int blk = rr / (2 * DECOMOE_GU_BLOCK), w = rr % (2 * DECOMOE_GU_BLOCK);
+    const bool is_up = w >= DECOMOE_GU_BLOCK;
+    const int f = blk * DECOMOE_GU_BLOCK + (is_up ? w - DECOMOE_GU_BLOCK : w);
+    const uint4* src = (is_up ? wu : wg) + (e * m + f) * vec;
+    uint4* dst = wgu + ro * vec;
+    for (int c = lane; c < vec; c += 32) dst[c] = src[c];
+  }
+}
+
+}  // namespace decomoe
+
+using namespace decomoe;
+
+extern "C" {
+
+int decomoe_weight_layout(const void* w_gate, const void* w_up, void* w_gate_up, int E, int d, int m,
+                          int dtype, decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(w_gate && w_up && w_gate_up, "weight_layout: null pointer");
+  DM_ARG_CHECK(E > 0 && d > 0 && m > 0, "weight_layout: bad sizes");
+  DM_ARG_CHECK(m % DECOMOE_GU_BLOCK == 0, "weight_layout: m=%d must be a multiple of %d", m, DECOMOE_GU_BLOCK);
+  DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "weight_layout: bad dtype");
+  const size_t row_bytes = static_cast<size_t>(d) * dtype_bytes(dtype);
+  DM_ARG_CHECK(row_bytes % 16 == 0 && aligned16(w_gate) && aligned16(w_up) && aligned16(w_gate_up),
+               "weight_layout: rows must be 16-byte multiples, pointers 16-byte aligned");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int blocks = sm_count() * 8;
+  k_weight_layout<<<blocks, 256, 0, s>>>(static_cast<const uint4*>(w_gate), static_cast<const uint4*>(w_up),
+                                         static_cast<uint4*>(w_gate_up), E, m,
+                                         static_cast<int>(row_bytes / 16));
+  DM_LAUNCH_CHECK("k_weight_layout");
+  return DECOMOE_OK;
+}
+
+static int expert_check(const char* name, const void* a, const int32_t* offsets, int64_t rows, int K, int d,
+                        int m, int dtype, const void* w, void* out) {
+  DM_ARG_CHECK(rows >= 0 && rows < 0x7fffffffLL, "%s: rows out of range", name);
+  DM_ARG_CHECK(K >= 1 && K <= DECOMOE_MAX_E, "%s: K=%d outside [1, %d]", name, K, DECOMOE_MAX_E);
+  DM_ARG_CHECK(d > 0 && m > 0, "%s: bad d/m", name);
+  DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "%s: bad dtype", name);
+  DM_ARG_CHECK(m % DECOMOE_GU_BLOCK == 0, "%s: m must be a multiple of %d", name, DECOMOE_GU_BLOCK);
+  if (rows == 0) return DECOMOE_OK;
+  DM_ARG_CHECK(a && offsets && w && out, "%s: null pointer", name);
+  if (dtype == DECOMOE_BF16) {
+    DM_ARG_CHECK(d % 256 == 0, "%s: bf16 needs d %% 256 == 0 (d=%d)", name, d);
+    DM_ARG_CHECK(aligned16(a) && aligned16(w) && aligned16(out), "%s: pointers must be 16-byte aligned", name);
+  }
+  return DECOMOE_OK;
+}
+
+static bool use_decode_path(int64_t rows) { return rows <= 64; }
+
+// Pipeline shape of the two expert GEMMs: k-block depth (64 -> 128-byte
+// swizzle, 32 -> 64-byte swizzle) and the number of shared-memory stages.
+#ifndef DECOMOE_GU_BK
+#define DECOMOE_GU_BK 64
+#endif
+#ifndef DECOMOE_GU_STAGES
+#define DECOMOE_GU_STAGES 4
+#endif
+#ifndef DECOMOE_DN_BK
+#define DECOMOE_DN_BK 64
+#endif
+#ifndef DECOMOE_DN_STAGES
+#define DECOMOE_DN_STAGES 4
+#endif
+constexpr int GU_BK = DECOMOE_GU_BK, GU_STAGES = DECOMOE_GU_STAGES;
+constexpr int DN_BK = DECOMOE_DN_BK, DN_STAGES = DECOMOE_DN_STAGES;
+
+int decomoe_expert_gate_up(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m,
+                           int dtype, const void* w_gate_up, void* h, int32_t* status_dev,
+                           decomoe_stream_t stream) {
+  clear_error();
+  DM_RET(expert_check("expert_gate_up", x_perm, offsets, rows, K, d, m, dtype, w_gate_up, h));
+  if (rows == 0) return DECOMOE_OK;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int R = static_cast<int>(rows);
+  if (dtype == DECOMOE_F32) {
+    dim3 g1((m + 127) / 128, static_cast<unsigned>(std::min(R, 65535)));
+    k_simt_gate_up<float><<<g1, 128, 0, s>>>(static_cast<const float*>(x_perm), offsets, K,
+                                              static_cast<const float*>(w_gate_up), d, m, static_cast<float*>(h));
+    DM_LAUNCH_CHECK("k_simt_gate_up");
+    return DECOMOE_OK;
+  }
+  if (use_decode_path(rows)) {
+    const size_t sm1 = static_cast<size_t>(DEC_NMAX) * d * 2;
+    DM_ARG_CHECK(sm1 <= 200 * 1024, "expert_gate_up: d too large for the decode path");
+    DM_CUDA_CHECK(cudaFuncSetAttribute(k_dec_gate_up, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm1));
+    dim3 g1((m + DEC_FEAT_PER_BLOCK - 1) / DEC_FEAT_PER_BLOCK, K);
+    k_dec_gate_up<<<g1, DEC_THREADS, sm1, s>>>(static_cast<const __nv_bfloat16*>(x_perm), offsets,
+                                               static_cast<const __nv_bfloat16*>(w_gate_up), d, m,
+                                               static_cast<__nv_bfloat16*>(h));
+    DM_LAUNCH_CHECK("k_dec_gate_up");
+    return DECOMOE_OK;
+  }
+  // A = x_perm [R, d], B = w_gate_up [K*2m, d] (only experts < K are read)
+  return launch_tc<256, EPI_SWIGLU, GU_STAGES, GU_BK>(x_perm, R, d, w_gate_up, static_cast<int64_t>(K) * 2 * m,
+                                                     offsets, K, 2 * m, h, m, nullptr, status_dev, s);
+}
+
+int decomoe_expert_down(const void* h, const int32_t* offsets, int64_t rows, int K, int d, int m, int dtype,
+                        const void* w_down, void* y_perm, int32_t* status_dev, decomoe_stream_t stream) {
+  clear_error();
+  DM_RET(expert_check("expert_down", h, offsets, rows, K, d, m, dtype, w_down, y_perm));
+  if (rows == 0) return DECOMOE_OK;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int R = static_cast<int>(rows);
+  if (dtype == DECOMOE_F32) {
+    dim3 g2((d + 127) / 128, static_cast<unsigned>(std::min(R, 65535)));
+    k_simt_down<float><<<g2, 128, 0, s>>>(static_cast<const float*>(h), offsets, K,
+                                           static_cast<const float*>(w_down), d, m, static_cast<float*>(y_perm));
+    DM_LAUNCH_CHECK("k_simt_down");
+    return DECOMOE_OK;
+  }
+  if (use_decode_path(rows)) {
+    const size_t sm2 = static_cast<size_t>(DEC_NMAX) * m * 2;
+    DM_ARG_CHECK(sm2 <= 200 * 1024, "expert_down: m too large for the decode path");
+    DM_CUDA_CHECK(cudaFuncSetAttribute(k_dec_down, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2));
+    dim3 g2((d + DEC_FEAT_PER_BLOCK - 1) / DEC_FEAT_PER_BLOCK, K);
+    k_dec_down<<<g2, DEC_THREADS, sm2, s>>>(static_cast<const __nv_bfloat16*>(h), offsets,
+                                            static_cast<const __nv_bfloat16*>(w_down), d, m,
+                                            static_cast<__nv_bfloat16*>(y_perm));
+    DM_LAUNCH_CHECK("k_dec_down");
+    return DECOMOE_OK;
+  }
+  // A = h [R, m], B = w_down [K*d, m]
+  return launch_tc<256, EPI_BF16, DN_STAGES, DN_BK>(h, R, m, w_down, static_cast<int64_t>(K) * d, offsets, K, d,
+                                                   y_perm, d, nullptr, status_dev, s);
+}
+
+int decomoe_expert_swiglu(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m,
+                          int dtype, const void* w_gate_up, const void* w_down, void* h_ws, void* y_perm,
+                          int32_t* status_dev, decomoe_stream_t stream) {
+  DM_RET(decomoe_expert_gate_up(x_perm, offsets, rows, K, d, m, dtype, w_gate_up, h_ws, status_dev, stream));
+  return decomoe_expert_down(h_ws, offsets, rows, K, d, m, dtype, w_down, y_perm, status_dev, stream);
+}
+
+// Reference CUDA-core path for bf16 (same math as the tensor-core path: bf16
+// products, fp32 accumulation, h rounded to bf16). Not part of the public
+// header; used by tests to localise disagreements between the tensor-core
+// kernels and the oracle.
+int decomoe_expert_swiglu_ref(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m,
+                               const void* w_gate_up, const void* w_down, void* h_ws, void* y_perm,
+                               decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(rows >= 0 && rows < 0x7fffffffLL && K >= 1 && K <= DECOMOE_MAX_E && d > 0 && m > 0,
+               "expert_swiglu_ref: bad sizes");
+  if (rows == 0) return DECOMOE_OK;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int R = static_cast<int>(rows);
+  dim3 g1((m + 127) / 128, static_cast<unsigned>(std::min(R, 65535)));
+  k_simt_gate_up<__nv_bfloat16><<<g1, 128, 0, s>>>(static_cast<const __nv_bfloat16*>(x_perm), offsets, K,
+                                                    static_cast<const __nv_bfloat16*>(w_gate_up), d, m,
+                                                    static_cast<__nv_bfloat16*>(h_ws));
+  DM_LAUNCH_CHECK("k_simt_gate_up<bf16>");
+  dim3 g2((d + 127) / 128, static_cast<unsigned>(std::min(R, 65535)));
+  k_simt_down<__nv_bfloat16><<<g2, 128, 0, s>>>(static_cast<const __nv_bfloat16*>(h_ws), offsets, K,
+                                                 static_cast<const __nv_bfloat16*>(w_down), d, m,
+                                                 static_cast<__nv_bfloat16*>(y_perm));
+  DM_LAUNCH_CHECK("k_simt_down<bf16>");
+  return DECOMOE_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,155 @@
+// One RCEP MoE invocation chained on a stream (DecoMoE Algorithm 2, exited
+// branch): router logits over the full pool, the activated-mass pass and
+// prefix selection (Eqs. 10-12), prefix routing, dispatch, grouped SwiGLU
+// experts and combine. Every intermediate lives in the caller's workspace.
+#include <vector>
+
+#include "decomoe_internal.cuh"
+
+namespace decomoe {
+
+enum {
+  WS_LOGITS = 0,
+  WS_TOPK_IDX,
+  WS_TOPK_W,
+  WS_MASS,
+  WS_COUNTS,
+  WS_OFFSETS,
+  WS_PERM,
+  WS_INV,
+  WS_XPERM,
+  WS_H,
+  WS_YPERM,
+  WS_ROUTE,
+  WS_DISPATCH,
+  WS_STATUS_PAD,
+  WS_COUNT
+};
+
+struct LayerLayout {
+  size_t off[WS_COUNT];
+  size_t total;
+};
+
+static LayerLayout layer_layout(int64_t T, int d, int E, int k, int m, int dtype) {
+  LayerLayout L;
+  const size_t eb = dtype_bytes(dtype);
+  const size_t R = static_cast<size_t>(T) * k;
+  size_t sz[WS_COUNT];
+  sz[WS_LOGITS] = static_cast<size_t>(T) * E * 4;
+  sz[WS_TOPK_IDX] = R * 4;
+  sz[WS_TOPK_W] = R * 4;
+  sz[WS_MASS] = static_cast<size_t>(E) * 8;
+  sz[WS_COUNTS] = static_cast<size_t>(E) * 4;
+  sz[WS_OFFSETS] = static_cast<size_t>(E + 1) * 4;
+  sz[WS_PERM] = R * 4;
+  sz[WS_INV] = R * 4;
+  sz[WS_XPERM] = R * d * eb;
+  sz[WS_H] = R * m * eb;
+  sz[WS_YPERM] = R * d * eb;
+  sz[WS_ROUTE] = decomoe_route_workspace_bytes(T, E);
+  sz[WS_DISPATCH] = decomoe_dispatch_workspace_bytes(T, k, E);
+  sz[WS_STATUS_PAD] = 256;
+  size_t o = 0;
+  for (int i = 0; i < WS_COUNT; ++i) {
+    L.off[i] = o;
+    o = align_up(o + sz[i], 256);
+  }
+  L.total = o;
+  return L;
+}
+
+}  // namespace decomoe
+
+using namespace decomoe;
+
+extern "C" {
+
+size_t decomoe_moe_layer_workspace_bytes(int64_t T, int d, int E, int k, int m, int dtype) {
+  if (T < 0 || d <= 0 || E <= 0 || k <= 0 || m <= 0) return 0;
+  return layer_layout(T, d, E, k, m, dtype).total;
+}
+
+int decomoe_moe_layer_workspace_layout(int64_t T, int d, int E, int k, int m, int dtype, size_t* offs_host) {
+  clear_error();
+  DM_ARG_CHECK(offs_host != nullptr, "moe_layer_workspace_layout: null pointer");
+  DM_ARG_CHECK(T >= 0 && d > 0 && E > 0 && k > 0 && m > 0, "moe_layer_workspace_layout: bad sizes");
+  const LayerLayout L = layer_layout(T, d, E, k, m, dtype);
+  for (int i = 0; i <= WS_YPERM; ++i) offs_host[i] = L.off[i];
+  return DECOMOE_OK;
+}
+
+int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const void* w_gate_up,
+                      const void* w_down, int64_t T, int d, int E, int k, int m, int dtype, int K_fixed,
+                      double p, const void* residual, void* out, int* K_used_host, int* K_sel_host, void* ws,
+                      size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(T >= 0 && d > 0 && m > 0, "moe_layer: bad sizes");
+  DM_ARG_CHECK(E >= 1 && E <= DECOMOE_MAX_E && k >= 1 && k <= DECOMOE_MAX_TOPK && k <= E,
+               "moe_layer: need 1 <= k <= E <= %d, k <= %d", DECOMOE_MAX_E, DECOMOE_MAX_TOPK);
+  DM_ARG_CHECK(K_fixed == 0 || (K_fixed >= k && K_fixed <= E), "moe_layer: K_fixed=%d outside [k, E]", K_fixed);
+  DM_ARG_CHECK(K_fixed > 0 || (p > 0.0 && p <= 1.0), "moe_layer: mass mode needs 0 < p <= 1");
+  DM_ARG_CHECK(p >= 0.0 && p <= 1.0, "moe_layer: p outside [0, 1]");
+  DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "moe_layer: bad dtype");
+  if (T == 0) {
+    if (K_used_host) *K_used_host = K_fixed > 0 ? K_fixed : k;
+    if (K_sel_host) *K_sel_host = k;
+    return DECOMOE_OK;
+  }
+  DM_ARG_CHECK(x && w_r && w_gate_up && w_down && out, "moe_layer: null pointer");
+  DM_ARG_CHECK(out != x, "moe_layer: out aliases x");
+  const LayerLayout L = layer_layout(T, d, E, k, m, dtype);
+  if (ws == nullptr || ws_bytes < L.total) {
+    set_error("moe_layer: workspace needs %zu bytes", L.total);
+    return DECOMOE_ERR_WORKSPACE;
+  }
+  DM_ARG_CHECK(aligned16(ws), "moe_layer: workspace must be 16-byte aligned");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  float* logits = reinterpret_cast<float*>(base + L.off[WS_LOGITS]);
+  int32_t* topk_idx = reinterpret_cast<int32_t*>(base + L.off[WS_TOPK_IDX]);
+  float* topk_w = reinterpret_cast<float*>(base + L.off[WS_TOPK_W]);
+  double* mass = reinterpret_cast<double*>(base + L.off[WS_MASS]);
+  int32_t* counts = reinterpret_cast<int32_t*>(base + L.off[WS_COUNTS]);
+  int32_t* offsets = reinterpret_cast<int32_t*>(base + L.off[WS_OFFSETS]);
+  int32_t* perm = reinterpret_cast<int32_t*>(base + L.off[WS_PERM]);
+  int32_t* inv = reinterpret_cast<int32_t*>(base + L.off[WS_INV]);
+  void* x_perm = base + L.off[WS_XPERM];
+  void* h = base + L.off[WS_H];
+  void* y_perm = base + L.off[WS_YPERM];
+  void* route_ws = base + L.off[WS_ROUTE];
+  void* disp_ws = base + L.off[WS_DISPATCH];
+
+  // a1: router logits over all E reordered experts
+  DM_RET(decomoe_router_logits(x, w_r, bias, T, d, E, dtype, logits, status_dev, stream));
+  // a2 + a3: full-pool routing, activated mass, shortest covering prefix
+  int K = K_fixed;
+  if (K_fixed == 0 || p > 0.0) {
+    DM_RET(decomoe_route_prefix(logits, T, E, E, E, k, nullptr, nullptr, mass, route_ws,
+                                decomoe_route_workspace_bytes(T, E), stream));
+    if (K_fixed == 0) {
+      static thread_local std::vector<double> h_mass;
+      h_mass.resize(E);
+      DM_CUDA_CHECK(cudaMemcpyAsync(h_mass.data(), mass, sizeof(double) * E, cudaMemcpyDeviceToHost, s));
+      DM_CUDA_CHECK(cudaStreamSynchronize(s));
+      int Ksel = k;
+      DM_RET(decomoe_select_prefix(h_mass.data(), E, k, p, &Ksel));
+      K = Ksel;
+      if (K_sel_host) *K_sel_host = Ksel;
+    }
+  }
+  if (K_used_host) *K_used_host = K;
+  // a4: prefix routing
+  DM_RET(decomoe_route_prefix(logits, T, E, E, K, k, topk_idx, topk_w, nullptr, nullptr, 0, stream));
+  // a5: dispatch
+  DM_RET(decomoe_dispatch(topk_idx, T, k, K, x, d, dtype, counts, offsets, perm, inv, x_perm, disp_ws,
+                          decomoe_dispatch_workspace_bytes(T, k, K), status_dev, stream));
+  // a6: grouped SwiGLU experts over [0, K)
+  DM_RET(decomoe_expert_swiglu(x_perm, offsets, T * k, K, d, m, dtype, w_gate_up, w_down, h, y_perm,
+                               status_dev, stream));
+  // a7: combine (+ residual)
+  DM_RET(decomoe_combine(y_perm, inv, topk_w, T, k, d, dtype, residual, out, stream));
+  return DECOMOE_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,226 @@
+// Router logits (CUDA-core path) and prefix-restricted top-k routing with the
+// activated-mass reduction of RCEP (DecoMoE Section 3.3, Eqs. 10-12,
+// Algorithm 2).
+#include <cfloat>
+
+#include "decomoe_internal.cuh"
+
+namespace decomoe {
+
+// ------------------------------------------------------------ router, CUDA cores
+// logits[t, e] = sum_j x[t, j] * w_r[e, j] + bias[e]. One thread per (t, e);
+// fp32 accumulate. Used for fp32 storage and shapes the tensor-core kernel does
+// not take.
+template <typename T>
+__device__ __forceinline__ float to_f(T v);
+template <>
+__device__ __forceinline__ float to_f<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+template <typename T>
+__global__ void k_router_simt(const T* __restrict__ x, const T* __restrict__ w_r,
+                              const float* __restrict__ bias, int64_t Tn, int d, int E,
+                              float* __restrict__ logits) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= Tn * E) return;
+  const int64_t t = i / E;
+  const int e = static_cast<int>(i - t * E);
+  const T* xr = x + t * d;
+  const T* wr = w_r + static_cast<int64_t>(e) * d;
+  float acc = 0.f;
+  for (int j = 0; j < d; ++j) acc = fmaf(to_f(xr[j]), to_f(wr[j]), acc);
+  if (bias != nullptr) acc += bias[e];
+  logits[i] = acc;
+}
+
+// ------------------------------------------------------------ routing
+// One warp per token. Lane l holds logits l, l+32, ... of the prefix [0, K)
+// in registers (K <= 256, 8 per lane). k rounds of a warp arg-max pick the k
+// largest (ties: lower expert index). Pick j lives in lane j. Weights are the
+// softmax over the k picks (equal to prefix softmax + top-k + renormalise,
+// because the prefix denominator cancels). With a mass buffer, each block also
+// writes its tokens' fp64 weights per expert, summed in token order, to
+// part[block][e]; k_mass_finalize then sums blocks in block order, so the
+// activated mass of Eq. 11 is bit-reproducible.
+constexpr int ROUTE_THREADS = 256;
+constexpr int ROUTE_TPB = 8;  // tokens per block: one per warp
+
+__global__ void __launch_bounds__(ROUTE_THREADS)
+    k_route(const float* __restrict__ logits, int64_t Tn, int E, int64_t ld, int K, int k,
+            int32_t* __restrict__ idx_out, float* __restrict__ w_out, double* __restrict__ part) {
+  __shared__ int s_idx[ROUTE_TPB][DECOMOE_MAX_TOPK];
+  __shared__ double s_w[ROUTE_TPB][DECOMOE_MAX_TOPK];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t tok0 = static_cast<int64_t>(blockIdx.x) * ROUTE_TPB;
+
+  for (int tt = warp; tt < ROUTE_TPB; tt += ROUTE_THREADS / 32) {
+    const int64_t t = tok0 + tt;
+    if (t >= Tn) break;
+    const float* row = logits + t * ld;
+    float v[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int e = lane + 32 * i;
+      v[i] = (e < K) ? row[e] : -FLT_MAX;
+    }
+    uint32_t taken = 0;
+    float my_v = 0.f;
+    int my_i = 0;
+    for (int j = 0; j < k; ++j) {
+      float bv = 0.f;
+      int bi = INT_MAX;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int e = lane + 32 * i;
+        if (e < K && !((taken >> i) & 1u)) {
+          if (bi == INT_MAX || v[i] > bv || (v[i] == bv && e < bi)) {
+            bv = v[i];
+            bi = e;
+          }
+        }
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+        const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+        const bool better = (oi != INT_MAX) &&
+                            (bi == INT_MAX || ov > bv || (ov == bv && oi < bi));
+        if (better) {
+          bv = ov;
+          bi = oi;
+        }
+      }
+      if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
+      if (lane == j) {
+        my_v = bv;
+        my_i = bi;
+      }
+    }
+    const float v0 = __shfl_sync(0xffffffffu, my_v, 0);
+    // fp32 weights for the routing output
+    float z = (lane < k) ? __expf(my_v - v0) : 0.f;
+    float zs = z;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) zs += __shfl_xor_sync(0xffffffffu, zs, off);
+    if (lane < k) {
+      if (idx_out != nullptr) idx_out[t * k + lane] = my_i;
+      if (w_out != nullptr) w_out[t * k + lane] = z / zs;
+    }
+    if (part != nullptr) {
+      // fp64 weights for the activated mass (Eq. 11)
+      double zd = (lane < k) ? exp(static_cast<double>(my_v) - static_cast<double>(v0)) : 0.0;
+      double zds = zd;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) zds += __shfl_xor_sync(0xffffffffu, zds, off);
+      if (lane < k) {
+        s_idx[tt][lane] = my_i;
+        s_w[tt][lane] = zd / zds;
+      }
+    }
+  }
+  if (part == nullptr) return;
+  __syncthreads();
+  const int ntok = static_cast<int>(Tn - tok0 < ROUTE_TPB ? Tn - tok0 : ROUTE_TPB);
+  for (int e = threadIdx.x; e < E; e += ROUTE_THREADS) {
+    double acc = 0.0;
+    for (int tt = 0; tt < ntok; ++tt)
+      for (int j = 0; j < k; ++j)
+        if (s_idx[tt][j] == e) acc += s_w[tt][j];  // token order, then slot order
+    part[static_cast<int64_t>(blockIdx.x) * E + e] = acc;
+  }
+}
+
+// mass[e] = sum over blocks of part[b][e]: one block per expert, each thread
+// sums a fixed strided subset of blocks in order, then a fixed-shape tree in
+// shared memory combines the 256 thread sums (bit-reproducible).
+__global__ void __launch_bounds__(256)
+    k_mass_finalize(const double* __restrict__ part, int nblocks, int E, double* __restrict__ mass) {
+  __shared__ double red[256];
+  const int e = blockIdx.x;
+  double acc = 0.0;
+  for (int b = threadIdx.x; b < nblocks; b += 256) acc += part[static_cast<int64_t>(b) * E + e];
+  red[threadIdx.x] = acc;
+  __syncthreads();
+  for (int w = 128; w > 0; w >>= 1) {
+    if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) mass[e] = red[0];
+}
+
+}  // namespace decomoe
+
+using namespace decomoe;
+
+extern "C" {
+
+int decomoe_router_logits(const void* x, const void* w_r, const float* bias, int64_t T, int d,
+                          int E, int dtype, float* logits, int32_t* status_dev,
+                          decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(T >= 0 && d > 0 && E > 0, "router_logits: bad sizes T=%lld d=%d E=%d", (long long)T, d, E);
+  DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "router_logits: bad dtype %d", dtype);
+  if (T == 0) return DECOMOE_OK;
+  DM_ARG_CHECK(x && w_r && logits, "router_logits: null pointer");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (dtype == DECOMOE_BF16 && router_tc_supported(d, E)) {
+    DM_ARG_CHECK(aligned16(x) && aligned16(w_r) && aligned16(logits),
+                 "router_logits: pointers must be 16-byte aligned");
+    return launch_router_tc(x, w_r, bias, T, d, E, logits, status_dev, s);
+  }
+  const int64_t n = T * E;
+  const int threads = 256;
+  const int64_t blocks = (n + threads - 1) / threads;
+  if (dtype == DECOMOE_F32)
+    k_router_simt<float><<<blocks, threads, 0, s>>>(static_cast<const float*>(x),
+                                                    static_cast<const float*>(w_r), bias, T, d, E, logits);
+  else
+    k_router_simt<__nv_bfloat16><<<blocks, threads, 0, s>>>(
+        static_cast<const __nv_bfloat16*>(x), static_cast<const __nv_bfloat16*>(w_r), bias, T, d, E, logits);
+  DM_LAUNCH_CHECK("k_router_simt");
+  return DECOMOE_OK;
+}
+
+size_t decomoe_route_workspace_bytes(int64_t T, int E) {
+  if (T < 0 || E <= 0) return 0;
+  const int64_t nblocks = (T + ROUTE_TPB - 1) / ROUTE_TPB;
+  return align_up(static_cast<size_t>(nblocks > 0 ? nblocks : 1) * E * sizeof(double), 256);
+}
+
+int decomoe_route_prefix(const float* logits, int64_t T, int E, int64_t ld, int K, int k,
+                         int32_t* topk_idx, float* topk_w, double* mass_out, void* ws,
+                         size_t ws_bytes, decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(T >= 0, "route_prefix: T < 0");
+  DM_ARG_CHECK(E >= 1 && E <= DECOMOE_MAX_E, "route_prefix: E=%d outside [1, %d]", E, DECOMOE_MAX_E);
+  DM_ARG_CHECK(k >= 1 && k <= DECOMOE_MAX_TOPK, "route_prefix: k=%d outside [1, %d]", k, DECOMOE_MAX_TOPK);
+  DM_ARG_CHECK(K >= k && K <= E, "route_prefix: need k <= K <= E (k=%d K=%d E=%d)", k, K, E);
+  DM_ARG_CHECK(ld >= E, "route_prefix: ld < E");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (T == 0) {
+    if (mass_out) DM_CUDA_CHECK(cudaMemsetAsync(mass_out, 0, sizeof(double) * E, s));
+    return DECOMOE_OK;
+  }
+  DM_ARG_CHECK(logits != nullptr, "route_prefix: logits is null");
+  const int64_t nblocks = (T + ROUTE_TPB - 1) / ROUTE_TPB;
+  DM_ARG_CHECK(nblocks <= 0x7fffffff, "route_prefix: T too large");
+  double* part = nullptr;
+  if (mass_out != nullptr) {
+    if (ws == nullptr || ws_bytes < decomoe_route_workspace_bytes(T, E)) {
+      set_error("route_prefix: workspace needs %zu bytes", decomoe_route_workspace_bytes(T, E));
+      return DECOMOE_ERR_WORKSPACE;
+    }
+    part = static_cast<double*>(ws);
+  }
+  k_route<<<static_cast<unsigned>(nblocks), ROUTE_THREADS, 0, s>>>(logits, T, E, ld, K, k, topk_idx,
+                                                                   topk_w, part);
+  DM_LAUNCH_CHECK("k_route");
+  if (mass_out != nullptr) {
+    k_mass_finalize<<<E, 256, 0, s>>>(part, static_cast<int>(nblocks), E, mass_out);
+    DM_LAUNCH_CHECK("k_mass_finalize");
+  }
+  return DECOMOE_OK;
+}
+
+}  // extern "C"
