@@ -141,6 +141,32 @@ DECOMOE_API int decomoe_dispatch(const int32_t* topk_idx, int64_t T, int k, int 
                      int32_t* status_dev, decomoe_stream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Allocation-free dispatch (the paper has no counterpart: this is a library
+ * convenience). Same arguments, outputs and errors as decomoe_dispatch, minus
+ * the workspace: for callers that cannot allocate device memory, e.g. a
+ * serving runtime that owns all of HBM in a fixed arena from start-up and
+ * forbids later cudaMalloc (it can synchronise the device and fragment the
+ * arena). The per-tile histograms then live in a fixed array inside the
+ * library image, of DECOMOE_NOALLOC_DISPATCH_SCRATCH_INTS int32 entries
+ * (256 KiB), which every GPU that loads the library keeps until the process
+ * exits. Requires ceil(T*k / 1024) * K <= that size, else
+ * DECOMOE_ERR_INVALID_ARG with a message and nothing launched.
+ *   - The first call on a device looks up the array's device address (once
+ *     per device, with that device current); make that first call before any
+ *     stream capture.
+ *   - Calls never allocate or free device memory.
+ *   - All calls on a device share the one array and it keeps the last call's
+ *     contents; nothing in it needs to start at zero (each call writes every
+ *     entry it reads). Calls whose execution overlaps on the GPU (different
+ *     streams, or other threads) race on the array: serialise them.
+ * ------------------------------------------------------------------------ */
+#define DECOMOE_NOALLOC_DISPATCH_SCRATCH_INTS 65536
+DECOMOE_API int decomoe_dispatch_noalloc(const int32_t* topk_idx, int64_t T, int k, int K, const void* x,
+                                         int d, int dtype, int32_t* counts, int32_t* offsets,
+                                         int32_t* perm_token, int32_t* inv_slot, void* x_perm,
+                                         int32_t* status_dev, decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * One-time weight layout transform (like the paper's load-time expert
  * reorder, Section 3.3: it changes storage only, not values).
  *   w_gate, w_up: [E, m, d] row-major (dtype). w_gate_up: [E, 2m, d], where

@@ -49,6 +49,7 @@ SIGNATURES = {
     "decomoe_select_prefix": (_I, [_P, _I, _I, _D, _P]),
     "decomoe_dispatch_workspace_bytes": (_S, [_L, _I, _I]),
     "decomoe_dispatch": (_I, [_P, _L, _I, _I, _P, _I, _I, _P, _P, _P, _P, _P, _P, _S, _P, _P]),
+    "decomoe_dispatch_noalloc": (_I, [_P, _L, _I, _I, _P, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
     "decomoe_weight_layout": (_I, [_P, _P, _P, _I, _I, _I, _I, _P]),
     "decomoe_expert_swiglu": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P]),
     "decomoe_expert_gate_up": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P]),
@@ -207,6 +208,21 @@ def decomoe_dispatch(topk_idx, K, x, counts, offsets, perm_token, inv_slot, x_pe
            lib().decomoe_dispatch(_ptr(topk_idx), T, k, K, _ptr(x), d, dtype, _ptr(counts), _ptr(offsets),
                                   _ptr(perm_token), _ptr(inv_slot), _ptr(x_perm), _ptr(ws),
                                   ws.numel() * ws.element_size(), _ptr(status), _stream(stream)))
+
+
+def decomoe_dispatch_noalloc(topk_idx, K, x, counts, offsets, perm_token, inv_slot, x_perm, status=None,
+                             stream=None):
+    """decomoe_dispatch without a workspace: for callers that cannot allocate
+    device memory; its scratch is a fixed array inside the library (see the
+    header for the size limit and the rule that overlapping calls race)."""
+    _need_cuda(topk_idx, x, counts, offsets, perm_token, inv_slot, x_perm, status)
+    T, k = topk_idx.shape
+    d = x.shape[1] if x is not None else 0
+    dtype = _dt(x) if x is not None else DECOMOE_BF16
+    _check("decomoe_dispatch_noalloc",
+           lib().decomoe_dispatch_noalloc(_ptr(topk_idx), T, k, K, _ptr(x), d, dtype, _ptr(counts), _ptr(offsets),
+                                          _ptr(perm_token), _ptr(inv_slot), _ptr(x_perm), _ptr(status),
+                                          _stream(stream)))
 
 
 def decomoe_weight_layout(w_gate, w_up, w_gate_up, stream=None):

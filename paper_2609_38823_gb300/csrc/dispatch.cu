@@ -2,6 +2,8 @@
 // histograms with warp-aggregated shared-memory atomics, a scan, a stable
 // rank assignment, and a 128-bit row gather (DecoMoE Algorithm 2: only the
 // first K expert MLPs are evaluated, each on the tokens routed to it).
+#include <mutex>
+
 #include "decomoe_internal.cuh"
 
 namespace decomoe {
@@ -221,3 +223,96 @@ int decomoe_dispatch(const int32_t* topk_idx, int64_t T, int k, int K, const voi
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free dispatch.
+//
+// Some callers cannot hand the library a workspace: their runtime owns every
+// device allocation up front (a serving engine that carves all of HBM into a
+// fixed arena at start-up and forbids any later cudaMalloc, because cudaMalloc
+// can synchronise the device and fragment that arena). For them this entry
+// point keeps the per-tile histograms in a fixed array that is part of the
+// library image itself, so the call needs nothing beyond its inputs and
+// outputs.
+//
+// Limit: ceil(T*k / 1024) * K <= DECOMOE_NOALLOC_DISPATCH_SCRATCH_INTS
+// (65536 int32 = 256 KiB, e.g. T*k up to 524288 pairs at K = 128). Every GPU
+// that loads the library holds this array until the process exits.
+// ---------------------------------------------------------------------------
+namespace decomoe {
+
+static __device__ __align__(256) int32_t g_noalloc_dispatch_scratch[DECOMOE_NOALLOC_DISPATCH_SCRATCH_INTS];
+
+// Device address of the array, looked up once per device (host code cannot
+// use the symbol itself as a device pointer).
+static int noalloc_scratch_ptr(int32_t** out) {
+  static std::mutex mu;
+  static int32_t* ptrs[64] = {nullptr};
+  int dev = 0;
+  DM_CUDA_CHECK(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= 64) {
+    set_error("dispatch_noalloc: device ordinal %d out of range", dev);
+    return DECOMOE_ERR_UNSUPPORTED;
+  }
+  std::lock_guard<std::mutex> lk(mu);
+  if (ptrs[dev] == nullptr) {
+    void* p = nullptr;
+    DM_CUDA_CHECK(cudaGetSymbolAddress(&p, g_noalloc_dispatch_scratch));
+    ptrs[dev] = static_cast<int32_t*>(p);
+  }
+  *out = ptrs[dev];
+  return DECOMOE_OK;
+}
+
+}  // namespace decomoe
+
+extern "C" int decomoe_dispatch_noalloc(const int32_t* topk_idx, int64_t T, int k, int K, const void* x, int d,
+                                        int dtype, int32_t* counts, int32_t* offsets, int32_t* perm_token,
+                                        int32_t* inv_slot, void* x_perm, int32_t* status_dev,
+                                        decomoe_stream_t stream) {
+  using namespace decomoe;
+  clear_error();
+  DM_ARG_CHECK(T >= 0 && k >= 1 && k <= DECOMOE_MAX_TOPK, "dispatch_noalloc: bad T=%lld or k=%d", (long long)T, k);
+  DM_ARG_CHECK(K >= 1 && K <= DECOMOE_MAX_E, "dispatch_noalloc: K=%d outside [1, %d]", K, DECOMOE_MAX_E);
+  DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "dispatch_noalloc: bad dtype");
+  DM_ARG_CHECK(counts && offsets, "dispatch_noalloc: counts/offsets null");
+  const int64_t N = T * k;
+  DM_ARG_CHECK(N < 0x7fffffffLL, "dispatch_noalloc: T*k too large");
+  const int64_t ntiles64 = (N + DSP_TILE - 1) / DSP_TILE;
+  DM_ARG_CHECK(ntiles64 * K <= DECOMOE_NOALLOC_DISPATCH_SCRATCH_INTS,
+               "dispatch_noalloc: ceil(T*k/%d)*K = %lld exceeds the fixed scratch of %d entries; "
+               "use decomoe_dispatch with a workspace", DSP_TILE, (long long)(ntiles64 * K),
+               DECOMOE_NOALLOC_DISPATCH_SCRATCH_INTS);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (N == 0) {
+    DM_CUDA_CHECK(cudaMemsetAsync(counts, 0, sizeof(int32_t) * K, s));
+    DM_CUDA_CHECK(cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (K + 1), s));
+    return DECOMOE_OK;
+  }
+  DM_ARG_CHECK(topk_idx && perm_token && inv_slot, "dispatch_noalloc: null index array");
+  const size_t row_bytes = static_cast<size_t>(d) * dtype_bytes(dtype);
+  if (x_perm != nullptr) {
+    DM_ARG_CHECK(x != nullptr && d > 0, "dispatch_noalloc: x null or d <= 0");
+    DM_ARG_CHECK(row_bytes % 16 == 0 && aligned16(x) && aligned16(x_perm),
+                 "dispatch_noalloc: rows must be 16-byte multiples and 16-byte aligned");
+  }
+  int32_t* tile_hist = nullptr;
+  DM_RET(noalloc_scratch_ptr(&tile_hist));
+  // k_dispatch_hist writes every entry the scatter pass reads, so nothing
+  // left in the array by an earlier call is ever used.
+  const int ntiles = static_cast<int>(ntiles64);
+  k_dispatch_hist<<<ntiles, DSP_THREADS, 0, s>>>(topk_idx, N, K, tile_hist, status_dev);
+  DM_LAUNCH_CHECK("k_dispatch_hist");
+  k_dispatch_scatter<<<ntiles, DSP_THREADS, 0, s>>>(topk_idx, N, k, K, tile_hist, ntiles, counts, offsets,
+                                                    perm_token, inv_slot);
+  DM_LAUNCH_CHECK("k_dispatch_scatter");
+  if (x_perm != nullptr) {
+    const int vec = static_cast<int>(row_bytes / 16);
+    int blocks = static_cast<int>(std::min<int64_t>((N * 32 + 255) / 256, sm_count() * 8LL));
+    if (blocks < 1) blocks = 1;
+    k_gather_rows<<<blocks, 256, 0, s>>>(static_cast<const uint4*>(x), perm_token, offsets, K, vec,
+                                         static_cast<uint4*>(x_perm));
+    DM_LAUNCH_CHECK("k_gather_rows");
+  }
+  return DECOMOE_OK;
+}
