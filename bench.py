@@ -33,7 +33,7 @@ sys.path.insert(0, ROOT)
 
 import workloads as W  # noqa: E402
 
-LAUNCHES_PER_STEP = 11  # router 1, mass 2, route 1, dispatch 3, gate/up 1, down 1, combine 1, compaction 1
+LAUNCHES_PER_STEP = 10  # router 1, route+mass 2, dispatch 3, gate/up 1, down 1, combine 1, compaction 1
 
 
 def parse():
@@ -198,11 +198,10 @@ class Buffers:
 
 
 def run_step(dm, wl, L, B, K, v0, nv, text, ev=None):
-    """One pass of the hot path, every step a C-ABI call (11 kernel launches)."""
+    """One pass of the hot path, every step a C-ABI call (10 kernel launches)."""
     k, E = wl.k, wl.E
     dm.decomoe_router_logits(L.x, L.w_r, L.bias, B.logits, B.status)                   # a1
-    dm.decomoe_route_prefix(B.logits, E, k, None, None, B.mass, B.route_ws)            # a2 (Eq. 11)
-    dm.decomoe_route_prefix(B.logits, K, k, B.idx, B.w)                                # a4
+    dm.decomoe_route_prefix(B.logits, K, k, B.idx, B.w, B.mass, B.route_ws)           # a2 (Eq. 11) + a4
     dm.decomoe_dispatch(B.idx, K, L.x, B.counts[:K], B.offsets[:K + 1], B.perm, B.inv, B.x_perm, B.disp_ws,
                         B.status)                                                     # a5
     if ev is not None:
@@ -414,6 +413,12 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
     ms, _ = timed(ad_step, n, 5, ws)
     out.append({"mode": f"mass p={args.p}", "K_mean": round(statistics.mean(Ks[-n:]), 2),
                 "tokens_per_s": round(T * n / (ms / 1e3), 1), "ms_per_step": round(ms / n, 4)})
+    # the same fixed-K step replayed from CUDA graphs (one per rotated layer)
+    graphs = [dm.capture_graph(lambda L=L: run_step(dm, wl, L, B, args.K, wl.v0, wl.nv, text)) for L in layers]
+    ms, _ = timed(lambda i, ev: graphs[i % len(graphs)].replay(), n, 5, ws)
+    out.append({"mode": "fixed, CUDA graph", "K": args.K, "tokens_per_s": round(T * n / (ms / 1e3), 1),
+                "ms_per_step": round(ms / n, 4)})
+    del graphs
     # decode-size layers, K=64: weight streaming, reported against HBM
     for Td in W.DECODE_T:
         Bd = Buffers(wl, Td, B.out.device, dm)
@@ -433,12 +438,15 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
         D = int((Bd.counts[:64] > 0).sum())
         wbytes = D * 3 * wl.m * wl.d * 2
         step_bytes = wbytes + wl.E * wl.d * 2 + Td * wl.d * 2 * (2 + 3 * wl.k)
+        graphs = [dm.capture_graph(lambda i=i: dec_step(i, None)) for i in range(len(layers))]
+        msg, _ = timed(lambda i, ev: graphs[i % len(graphs)].replay(), n, 5, ws)
         out.append({"mode": "decode", "T": Td, "K": 64, "active_experts": D,
                     "tokens_per_s": round(Td * n / (ms / 1e3), 1), "ms_per_step": round(ms / n, 4),
-                    "step_hbm_frac": round(step_bytes / (ms / n * 1e-3) / 1e9 / pk["hbm_gbs"], 4),
+                    "graph_tokens_per_s": round(Td * n / (msg / 1e3), 1), "graph_ms_per_step": round(msg / n, 4),
+                    "graph_step_hbm_frac": round(step_bytes / (msg / n * 1e-3) / 1e9 / pk["hbm_gbs"], 4),
                     "ffn_ms": round(ffn, 4),
                     "ffn_hbm_frac": round(wbytes / (ffn * 1e-3) / 1e9 / pk["hbm_gbs"], 4)})
-        del Bd, xs
+        del Bd, xs, graphs
     return out
 
 
@@ -461,7 +469,7 @@ def _oracle_inputs(wl, L_dev_or_none, K, ntok, seed=0):
         g = {"x": L_dev_or_none.x.cpu(), "w_r": L_dev_or_none.w_r.cpu(), "bias": L_dev_or_none.bias.cpu()}
         wgu = L_dev_or_none.w_gu[:K].cpu()
         m = wl.m
-        G = 128
+        G = 64
         blocks = wgu.view(K, m // G, 2, G, wl.d)
         wg = blocks[:, :, 0].reshape(K, m, wl.d)
         wu = blocks[:, :, 1].reshape(K, m, wl.d)

@@ -62,7 +62,7 @@ typedef enum {
 enum { DECOMOE_BF16 = 0, DECOMOE_F32 = 1 };
 
 /* Gate/up interleave granule of the fused weight layout (rows of one block). */
-#define DECOMOE_GU_BLOCK 128
+#define DECOMOE_GU_BLOCK 64
 /* Largest expert pool and largest top-k any kernel here takes. */
 #define DECOMOE_MAX_E 256
 #define DECOMOE_MAX_TOPK 32
@@ -98,9 +98,11 @@ DECOMOE_API int decomoe_router_logits(const void* x, const void* w_r, const floa
  *   topk_w[t, j] = exp(l_j - l_0) / sum_j' exp(l_j' - l_0) over the k picks,
  *   which equals "new softmax over the prefix, top-k, renormalise".
  *   With K == E this is the full-pool routing of Eq. 10. If mass_out is not
- *   NULL, mass_out[e] = sum_t of the token's renormalised weight of e (Eq. 11),
- *   accumulated in fp64 in a fixed order (bit-reproducible run to run);
- *   mass_out then needs E entries and the workspace.
+ *   NULL the same launch also computes the activated mass of Eq. 11 over the
+ *   full pool [0, E) whatever K is: mass_out[e] = sum over tokens of the
+ *   renormalised full-pool top-k weight of e (fp32 weights, fp64 sum across
+ *   blocks in a fixed order: bit-reproducible run to run, relative error of a
+ *   few 1e-7); mass_out then needs E entries and the workspace.
  * logits: [T, ld] fp32, entries [0, E) used, ld >= E. topk_idx: [T, k] int32,
  * values in [0, K). topk_w: [T, k] fp32. Either output may be NULL (e.g. the
  * mass-only pass). Needs 1 <= k <= K <= E <= 256, k <= 32.

@@ -30,7 +30,7 @@ DECOMOE_ERR_WORKSPACE = 5
 DECOMOE_ERR_BAD_INPUT = 6
 DECOMOE_BF16 = 0
 DECOMOE_F32 = 1
-GU_BLOCK = 128
+GU_BLOCK = 64
 
 # name -> (restype, argtypes)
 _P = ctypes.c_void_p
@@ -337,6 +337,23 @@ def fuse_gate_up(w_gate: torch.Tensor, w_up: torch.Tensor) -> torch.Tensor:
     out = torch.empty((E, 2 * m, d), dtype=w_gate.dtype, device=w_gate.device)
     decomoe_weight_layout(w_gate, w_up, out)
     return out
+
+
+def capture_graph(fn, warmup: int = 1) -> "torch.cuda.CUDAGraph":
+    """Capture fn() (a sequence of the calls above with fixed sizes, e.g. one
+    fixed-K MoE layer) into a CUDA graph; replay it with g.replay(). Calls
+    that synchronise (decomoe_moe_layer with K_fixed == 0, decomoe_read_status)
+    cannot be captured."""
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for _ in range(warmup):
+            fn()
+    torch.cuda.current_stream().wait_stream(side)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        fn()
+    return g
 
 
 def workspace(nbytes: int, device) -> torch.Tensor:

@@ -112,45 +112,36 @@ static void launch_combine(int grid, cudaStream_t s, const uint4* y, const int32
 }
 
 // ------------------------------------------------------------------ compaction
-// dst[b, r'] = src[b, r'] for r' < v0, src[b, r' + nv] otherwise. Each warp
-// copies 4 rows per step (16-byte vectors, all loads issued before stores).
+// dst[b, r'] = src[b, r'] for r' < v0, src[b, r' + nv] otherwise. A flat grid
+// over the output's 16-byte vectors (batch, row, column; column fastest, so a
+// warp moves 512 contiguous bytes), four vectors per thread in flight.
 __global__ void __launch_bounds__(256)
     k_compact_vec(const uint4* __restrict__ src, uint4* __restrict__ dst, int64_t rows_out,
                   int64_t vec, int64_t v0, int64_t nv, int64_t nbatch, int64_t sstride,
                   int64_t dstride) {
-  const int lane = threadIdx.x & 31;
-  const int64_t gw = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-  const int64_t nw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
-  const int64_t total = nbatch * rows_out;
-  constexpr int RPW = 4;
-  for (int64_t q0 = gw * RPW; q0 < total; q0 += nw * RPW) {
-    const uint4* s[RPW];
-    uint4* d[RPW];
-    int nr = 0;
+  constexpr int U = 4;
+  const int64_t total = nbatch * rows_out * vec;
+  const int64_t step = static_cast<int64_t>(gridDim.x) * blockDim.x * U;
+  for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x * U + threadIdx.x; base < total; base += step) {
+    uint4 v[U];
+    int64_t di[U];
 #pragma unroll
-    for (int u = 0; u < RPW; ++u) {
-      const int64_t q = q0 + u;
-      if (q < total) {
+    for (int u = 0; u < U; ++u) {
+      const int64_t i = base + static_cast<int64_t>(u) * blockDim.x;
+      di[u] = -1;
+      if (i < total) {
+        const int64_t c = i % vec;
+        const int64_t q = i / vec;
         const int64_t b = q / rows_out;
         const int64_t r = q - b * rows_out;
         const int64_t rs = r < v0 ? r : r + nv;
-        s[u] = src + b * sstride + rs * vec;
-        d[u] = dst + b * dstride + r * vec;
-        nr = u + 1;
-      } else {
-        s[u] = nullptr;
-        d[u] = nullptr;
+        v[u] = __ldcs(src + b * sstride + rs * vec + c);
+        di[u] = b * dstride + r * vec + c;
       }
     }
-    for (int64_t c = lane; c < vec; c += 32) {
-      uint4 v[RPW];
 #pragma unroll
-      for (int u = 0; u < RPW; ++u)
-        if (u < nr) v[u] = __ldcs(s[u] + c);
-#pragma unroll
-      for (int u = 0; u < RPW; ++u)
-        if (u < nr) __stcs(d[u] + c, v[u]);
-    }
+    for (int u = 0; u < U; ++u)
+      if (di[u] >= 0) __stcs(dst + di[u], v[u]);
   }
 }
 
@@ -282,7 +273,8 @@ int decomoe_drop_visual_block(const void* src, void* dst, int64_t rows, int64_t 
   const bool vec_ok = row_bytes % 16 == 0 && aligned16(src) && aligned16(dst) &&
                       (nbatch == 1 || (src_batch_stride % 16 == 0 && dst_batch_stride % 16 == 0));
   if (vec_ok) {
-    const int grid = grid_for_warps((nbatch * rows_out + 3) / 4);
+    const int64_t nvec = nbatch * rows_out * (row_bytes / 16);
+    const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>((nvec + 1023) / 1024, sm_count() * 16LL)));
     k_compact_vec<<<grid, 256, 0, s>>>(static_cast<const uint4*>(src), static_cast<uint4*>(dst), rows_out,
                                        row_bytes / 16, v0, nv, nbatch, src_batch_stride / 16,
                                        dst_batch_stride / 16);

@@ -24,6 +24,17 @@
 
 #include "decomoe_internal.cuh"
 
+// Kernel choice for the bf16 expert GEMMs: the weights-stationary k_moe_ws
+// when the average expert gets at most DECOMOE_WS_MAX_AVG_ROWS rows (decode
+// sizes: every tile streams its own weight slice), the tokens-as-M k_gemm_tc
+// otherwise (prefill: faster when many rows share an expert's weights).
+#ifndef DECOMOE_WS_MAX_AVG_ROWS
+#define DECOMOE_WS_MAX_AVG_ROWS 8
+#endif
+#ifndef DECOMOE_DECODE_ROWS
+#define DECOMOE_DECODE_ROWS 0  // rows at or below which the CUDA-core decode kernels run
+#endif
+
 namespace decomoe {
 
 // ------------------------------------------------------------------ TMA maps
@@ -109,12 +120,28 @@ struct TcCfg {
 // experts whose weights stream from HBM once; mixing them in every wave keeps
 // both HBM and the tensor pipes busy instead of running the two phases one
 // after the other.
+#ifndef DECOMOE_TILE_ORDER
+#define DECOMOE_TILE_ORDER 1
+#endif
 __device__ __forceinline__ void tile_coords(int tile, int NT, const int* s_mt, int G, int& grp, int& mt,
                                             int& nb) {
+  const int mtot = s_mt[G];
+#if DECOMOE_TILE_ORDER == 2
+  {
+    // multiplicative permutation of the work items (a bijection when the
+    // multiplier is coprime with their count)
+    const int total = mtot * NT;
+    const int P = (total % 7919 != 0) ? 7919 : 7907;
+    tile = static_cast<int>((static_cast<long long>(tile) * P) % total);
+  }
+#endif
   const int j = tile / NT;
   nb = tile - j * NT;
-  const int mtot = s_mt[G];
+#if DECOMOE_TILE_ORDER == 1
   const int mtg = (j & 1) ? (mtot - 1 - (j >> 1)) : (j >> 1);
+#else
+  const int mtg = j;
+#endif
   int lo = 0, hi = G - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
@@ -321,13 +348,17 @@ __global__ void __launch_bounds__(192, 1)
       const uint32_t tb =
           tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
       if constexpr (EPI == EPI_SWIGLU) {
-        // columns [0, BN/2) gate, [BN/2, BN) up of features nb*BN/2 + c
+        // columns hold blocks of GU gate then GU up columns of the same
+        // features: features nb*BN/2 + half*GU + c
+        constexpr int GU = DECOMOE_GU_BLOCK;
+        static_assert(BN % (2 * GU) == 0, "N tile must hold whole gate/up blocks");
         __nv_bfloat16* out = static_cast<__nv_bfloat16*>(g.out);
 #pragma unroll 1
-        for (int c = 0; c < BN / 2; c += 32) {
+        for (int cc = 0; cc < BN / 2; cc += 32) {
+          const int half = cc / GU, c = cc % GU;
           uint32_t gr[32], ur[32];
-          tmem_ld32(tb + c, gr);
-          tmem_ld32(tb + BN / 2 + c, ur);
+          tmem_ld32(tb + half * 2 * GU + c, gr);
+          tmem_ld32(tb + half * 2 * GU + GU + c, ur);
           tc_wait_ld();
           uint32_t pk[16];
 #pragma unroll
@@ -338,7 +369,7 @@ __global__ void __launch_bounds__(192, 1)
           }
           if (valid) {
             uint4* dst = reinterpret_cast<uint4*>(out + static_cast<int64_t>(grow) * g.out_ld +
-                                                  nb * (BN / 2) + c);
+                                                  nb * (BN / 2) + cc);
 #pragma unroll
             for (int v = 0; v < 4; ++v)
               dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
@@ -462,9 +493,390 @@ static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b
                                      static_cast<int>(C::SMEM)));
   const int64_t ub_tiles =
       (static_cast<int64_t>(rows) / C::BM + ngroups) * static_cast<int64_t>(n_per_group / BN);
-  const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(sm_count(), ub_tiles)));
+#ifdef DECOMOE_GRID_CAP
+  const int64_t cap = std::min<int64_t>(sm_count(), DECOMOE_GRID_CAP);
+#else
+  const int64_t cap = sm_count();
+#endif
+  const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(cap, ub_tiles)));
   kern<<<grid, 192, C::SMEM, s>>>(ta, tb, g);
   DM_LAUNCH_CHECK("k_gemm_tc");
+  return DECOMOE_OK;
+}
+
+// ------------------------------------------------------------------ weights-stationary grouped GEMM
+// D[w, t] = sum_k W[e][wrow0 + w, k] * X[row0 + t, k]: the expert's weight rows
+// are the M operand (128 per tile, always full) and its tokens the N operand
+// (up to 256 per tile, MMA width rounded up to 16). No M padding, so a ragged,
+// skewed expert population costs only what it routes; small experts (and the
+// decode sizes) become pure weight streaming with every tile reading its own
+// 128-row weight slice once. Roles as in k_gemm_tc (TMA warp, MMA warp, four
+// epilogue warps, double-buffered 256-column TMEM accumulators).
+//
+// Tiles: per expert e, (wrows / 128) weight blocks x ceil(n_e / 256) token
+// chunks, chunk innermost (consecutive tiles share a weight block, so it is
+// read from HBM once and from L2 after); the global list is visited
+// alternately from both ends, as in k_gemm_tc.
+//
+// SwiGLU epilogue: with the 64-row gate/up interleave a weight block holds 64
+// gate rows (TMEM lanes 0..63) and the 64 up rows of the same features (lanes
+// 64..127). The warps owning lanes 64..127 pass their up values through a
+// small double-buffered shared-memory exchange to the warps owning the gate
+// lanes of the same features, which write h.
+struct WsArgs {
+  const int32_t* offsets;  // [G + 1] token row offsets per expert
+  int G;                   // experts [0, G)
+  int rows;                // token rows of the activation tensor
+  int wrows;               // weight rows per expert (2m gate/up, d down)
+  int kdim;
+  void* out;
+  int64_t out_ld;
+  int32_t* status;
+  uint64_t limit_ns;
+};
+
+#ifndef DECOMOE_WS_BOX
+#define DECOMOE_WS_BOX 32
+#endif
+#ifndef DECOMOE_WS_ORDER
+#define DECOMOE_WS_ORDER 0  // 0: weight block outer, token chunk inner; 1: chunk outer
+#endif
+constexpr int WS_BM = 128, WS_BK = 64, WS_BN = 256, WS_BOX = DECOMOE_WS_BOX;
+
+template <int STAGES, bool SWIGLU>
+struct WsCfg {
+  static constexpr int A_BYTES = WS_BM * WS_BK * 2;
+  static constexpr int B_BYTES = WS_BN * WS_BK * 2;
+  static constexpr int BOX_BYTES = WS_BOX * WS_BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int TMEM_COLS = 2 * WS_BN;
+  static constexpr int MAXG = DECOMOE_MAX_E;
+  static constexpr int NBARS = 2 * STAGES + 5;
+  static constexpr int XCH_BYTES = SWIGLU ? 2 * 2 * 32 * 32 * 4 : 0;  // up values, double-buffered
+  static constexpr int OUT_COLS = SWIGLU ? WS_BM / 2 : WS_BM;            // output features per tile
+  static constexpr int STILE_BYTES = 2 * 32 * OUT_COLS * 2;              // [2][32 tokens][OUT_COLS] bf16
+  static constexpr size_t SMEM = 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + XCH_BYTES + STILE_BYTES +
+                                 NBARS * 8 + 2 * (MAXG + 1) * 4 + 16;
+};
+
+struct WsTile {
+  int g, wb, row0, ntok;
+};
+
+__device__ __forceinline__ WsTile ws_tile(int t, int total, const int* s_tt, const int* s_off, int G, int nwb) {
+  const int tp = (t & 1) ? (total - 1 - (t >> 1)) : (t >> 1);
+  int lo = 0, hi = G - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (s_tt[mid] <= tp)
+      lo = mid;
+    else
+      hi = mid - 1;
+  }
+  WsTile r;
+  r.g = lo;
+  const int n = s_off[lo + 1] - s_off[lo];
+  const int nch = (n + WS_BN - 1) / WS_BN;
+  const int local = tp - s_tt[lo];
+#if DECOMOE_WS_ORDER == 1
+  const int c = local / nwb;
+  r.wb = local - c * nwb;
+#else
+  r.wb = local / nch;
+  const int c = local - r.wb * nch;
+#endif
+  r.row0 = s_off[lo] + c * WS_BN;
+  r.ntok = min(WS_BN, n - c * WS_BN);
+  return r;
+}
+
+__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+template <bool SWIGLU, int STAGES>
+__global__ void __launch_bounds__(192, 1)
+    k_moe_ws(const __grid_constant__ CUtensorMap tma_w, const __grid_constant__ CUtensorMap tma_x,
+             const WsArgs g) {
+  using C = WsCfg<STAGES, SWIGLU>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
+  uint8_t* smem = smem_raw + pad;
+  const uint32_t sA = raw + pad;
+  const uint32_t sB = sA + STAGES * C::A_BYTES;
+  float* xch = reinterpret_cast<float*>(smem + STAGES * C::STAGE_BYTES);
+  __nv_bfloat16* stile = reinterpret_cast<__nv_bfloat16*>(smem + STAGES * C::STAGE_BYTES + C::XCH_BYTES);
+  uint64_t* bars =
+      reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES + C::XCH_BYTES + C::STILE_BYTES);
+  int* s_off = reinterpret_cast<int*>(bars + C::NBARS);
+  int* s_tt = s_off + (C::MAXG + 1);
+  volatile uint32_t* s_tmem = reinterpret_cast<volatile uint32_t*>(s_tt + (C::MAXG + 1));
+  volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t bar0 = smem_u32(bars);
+#define FULL_BAR(s) (bar0 + 8u * (s))
+#define EMPTY_BAR(s) (bar0 + 8u * (STAGES + (s)))
+#define TFULL_BAR(a) (bar0 + 8u * (2 * STAGES + (a)))
+#define TEMPTY_BAR(a) (bar0 + 8u * (2 * STAGES + 2 + (a)))
+#define DRAIN_BAR (bar0 + 8u * (2 * STAGES + 4))
+
+  const int G = g.G;
+  const int nwb = g.wrows / WS_BM;
+  for (int i = threadIdx.x; i <= G; i += blockDim.x) s_off[i] = g.offsets[i];
+  if (threadIdx.x == 0) {
+    *s_abort = 0;
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(FULL_BAR(s), 1);
+      mbar_init(EMPTY_BAR(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(TFULL_BAR(a), 1);
+      mbar_init(TEMPTY_BAR(a), 128);
+    }
+    mbar_init(DRAIN_BAR, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (warp == 2) {
+    // s_tt[e] = first tile of expert e = sum over earlier experts of nwb * chunks
+    const int per = (G + 31) / 32;
+    int loc[8];
+    int sum = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      loc[i] = 0;
+      const int gi = lane * per + i;
+      if (i < per && gi < G) {
+        const int n = s_off[gi + 1] - s_off[gi];
+        loc[i] = n > 0 ? ((n + WS_BN - 1) / WS_BN) * nwb : 0;
+      }
+      sum += loc[i];
+    }
+    int incl = sum;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += v;
+    }
+    int run = incl - sum;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int gi = lane * per + i;
+      if (i < per && gi < G) s_tt[gi] = run;
+      run += loc[i];
+    }
+    if (lane == 31) s_tt[G] = incl;
+  }
+  __syncthreads();
+  const int total = s_tt[G];
+  if (static_cast<int>(blockIdx.x) >= total) return;
+
+  if (warp == 1) {
+    tmem_alloc(smem_u32(const_cast<uint32_t*>(s_tmem)), C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *s_tmem;
+  const int KB = g.kdim / WS_BK;
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------ TMA producer
+    tma_prefetch_desc(&tma_w);
+    tma_prefetch_desc(&tma_x);
+    int stage = 0;
+    uint32_t ph = 0;
+    bool ok = true;
+    uint32_t armed = 0, armed_ph = 0;
+    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+      const WsTile T = ws_tile(t, total, s_tt, s_off, G, nwb);
+      const int wrow0 = T.g * g.wrows + T.wb * WS_BM;
+      const int nbox = (T.ntok + WS_BOX - 1) / WS_BOX;
+      const uint32_t bytes = C::A_BYTES + nbox * C::BOX_BYTES;
+      for (int kb = 0; kb < KB; ++kb) {
+        if (!mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(FULL_BAR(stage), bytes);
+        tma_load_2d(sA + stage * C::A_BYTES, &tma_w, FULL_BAR(stage), kb * WS_BK, wrow0);
+        for (int i = 0; i < nbox; ++i)
+          tma_load_2d(sB + stage * C::B_BYTES + i * C::BOX_BYTES, &tma_x, FULL_BAR(stage), kb * WS_BK,
+                      T.row0 + i * WS_BOX);
+        armed |= 1u << stage;
+        armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
+        if (++stage == STAGES) {
+          stage = 0;
+          ph ^= 1u;
+        }
+      }
+    }
+    if (!ok) {
+      *s_abort = 1;
+      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+      int no_abort = 0;
+      for (int s = 0; s < STAGES; ++s)
+        if ((armed >> s) & 1u) mbar_wait(FULL_BAR(s), (armed_ph >> s) & 1u, g.limit_ns, &no_abort);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ------------------------------------------------ MMA issuer
+    int stage = 0;
+    uint32_t ph = 0;
+    bool ok = true, issued = false;
+    int it = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
+      const WsTile T = ws_tile(t, total, s_tt, s_off, G, nwb);
+      const uint32_t idesc = idesc_bf16_f32(WS_BM, (T.ntok + 15) & ~15);
+      const int acc = it & 1;
+      const uint32_t aph = (it >> 1) & 1;
+      if (!mbar_wait(TEMPTY_BAR(acc), aph ^ 1u, g.limit_ns, s_abort)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t dt = tmem_base + static_cast<uint32_t>(acc * WS_BN);
+      for (int kb = 0; kb < KB; ++kb) {
+        if (!mbar_wait(FULL_BAR(stage), ph, g.limit_ns, s_abort)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint64_t ad = smem_desc_kmajor<WS_BK>(sA + stage * C::A_BYTES);
+        const uint64_t bd = smem_desc_kmajor<WS_BK>(sB + stage * C::B_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < WS_BK / 16; ++kk)
+          tc_mma_f16(dt, ad + 2u * kk, bd + 2u * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+        tc_commit(EMPTY_BAR(stage));
+        issued = true;
+        if (++stage == STAGES) {
+          stage = 0;
+          ph ^= 1u;
+        }
+      }
+      if (!ok) break;
+      tc_commit(TFULL_BAR(acc));
+    }
+    if (!ok) {
+      *s_abort = 1;
+      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+      if (issued) {
+        int no_abort = 0;
+        tc_commit(DRAIN_BAR);
+        mbar_wait(DRAIN_BAR, 0, g.limit_ns, &no_abort);
+      }
+    }
+  } else if (warp >= 2) {
+    // ------------------------------------------------ epilogue
+    const int q = warp & 3;  // TMEM lanes [32q, 32q + 32)
+    __nv_bfloat16* out = static_cast<__nv_bfloat16*>(g.out);
+    int it = 0;
+    int xpar = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
+      const WsTile T = ws_tile(t, total, s_tt, s_off, G, nwb);
+      const int acc = it & 1;
+      const uint32_t aph = (it >> 1) & 1;
+      if (!mbar_wait(TFULL_BAR(acc), aph, g.limit_ns, s_abort)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t tb =
+          tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * WS_BN);
+      // Each 32-token chunk: accumulator columns -> registers -> (SwiGLU) ->
+      // bf16 tile [32 tokens][OUT_COLS features] in shared memory -> 16-byte
+      // row stores to out[token, feature]. Two named barriers per chunk over
+      // the four epilogue warps; the exchange and tile buffers alternate.
+      constexpr int OC = C::OUT_COLS;
+      const int et = threadIdx.x - 64;  // 0..127 among the epilogue warps
+      const int fbase = T.wb * OC;      // first output feature of this tile
+#pragma unroll 1
+      for (int c0 = 0; c0 < T.ntok; c0 += 32) {
+        uint32_t r[32];
+        tmem_ld32(tb + c0, r);
+        tc_wait_ld();
+        __nv_bfloat16* st = stile + xpar * (32 * OC);
+        if constexpr (SWIGLU) {
+          const bool is_gate = q < 2;
+          const int pr = q & 1;
+          float* xb = xch + (xpar * 2 + pr) * 1024;  // [32 columns][32 lanes]
+          if (!is_gate) {
+#pragma unroll
+            for (int c = 0; c < 32; ++c) xb[c * 32 + lane] = __uint_as_float(r[c]);
+          }
+          named_bar_sync(1, 128);
+          if (is_gate) {
+#pragma unroll
+            for (int c = 0; c < 32; ++c)
+              st[c * OC + pr * 32 + lane] = __float2bfloat16_rn(silu_f(__uint_as_float(r[c])) * xb[c * 32 + lane]);
+          }
+        } else {
+#pragma unroll
+          for (int c = 0; c < 32; ++c) st[c * OC + q * 32 + lane] = __float2bfloat16_rn(__uint_as_float(r[c]));
+        }
+        named_bar_sync(1, 128);
+        const int nc = min(32, T.ntok - c0);
+        constexpr int VPR = OC / 8;  // 16-byte vectors per token row
+#pragma unroll
+        for (int v = et; v < 32 * VPR; v += 128) {
+          const int row = v / VPR, cv = v - row * VPR;
+          if (row < nc) {
+            const uint4 val = *reinterpret_cast<const uint4*>(st + row * OC + cv * 8);
+            *reinterpret_cast<uint4*>(out + static_cast<int64_t>(T.row0 + c0 + row) * g.out_ld + fbase + cv * 8) = val;
+          }
+        }
+        xpar ^= 1;
+      }
+      tc_fence_before();
+      mbar_arrive(TEMPTY_BAR(acc));
+    }
+    if (!ok) {
+      *s_abort = 1;
+      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+#undef FULL_BAR
+#undef EMPTY_BAR
+#undef TFULL_BAR
+#undef TEMPTY_BAR
+#undef DRAIN_BAR
+}
+
+// X: [rows, kdim] token rows grouped by expert; W: [G * wrows, kdim].
+template <bool SWIGLU, int STAGES>
+static int launch_ws(const void* X, int rows, int kdim, const void* W, int wrows, const int32_t* offsets, int G,
+                     void* out, int64_t out_ld, int32_t* status, cudaStream_t s) {
+  using C = WsCfg<STAGES, SWIGLU>;
+  CUtensorMap tw, tx;
+  DM_RET(make_tmap_bf16(&tw, W, static_cast<uint64_t>(kdim), static_cast<uint64_t>(G) * wrows, WS_BM, WS_BK));
+  DM_RET(make_tmap_bf16(&tx, X, static_cast<uint64_t>(kdim), static_cast<uint64_t>(rows), WS_BOX, WS_BK));
+  WsArgs g;
+  g.offsets = offsets;
+  g.G = G;
+  g.rows = rows;
+  g.wrows = wrows;
+  g.kdim = kdim;
+  g.out = out;
+  g.out_ld = out_ld;
+  g.status = status;
+  g.limit_ns = static_cast<uint64_t>(wait_limit_ns());
+  auto kern = k_moe_ws<SWIGLU, STAGES>;
+  static_assert(C::SMEM <= 232448, "shared memory budget");
+  DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(C::SMEM)));
+  const int64_t ub_tiles = (static_cast<int64_t>(rows) / WS_BN + G) * (wrows / WS_BM);
+  const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(sm_count(), ub_tiles)));
+  kern<<<grid, 192, C::SMEM, s>>>(tw, tx, g);
+  DM_LAUNCH_CHECK("k_moe_ws");
   return DECOMOE_OK;
 }
 
@@ -779,7 +1191,7 @@ static int expert_check(const char* name, const void* a, const int32_t* offsets,
   return DECOMOE_OK;
 }
 
-static bool use_decode_path(int64_t rows) { return rows <= 64; }
+static bool use_decode_path(int64_t rows) { return rows <= DECOMOE_DECODE_ROWS; }
 
 // Pipeline shape of the two expert GEMMs: k-block depth (64 -> 128-byte
 // swizzle, 32 -> 64-byte swizzle) and the number of shared-memory stages.
@@ -824,6 +1236,8 @@ int decomoe_expert_gate_up(const void* x_perm, const int32_t* offsets, int64_t r
     DM_LAUNCH_CHECK("k_dec_gate_up");
     return DECOMOE_OK;
   }
+  if (static_cast<int64_t>(R) <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K)
+    return launch_ws<true, 4>(x_perm, R, d, w_gate_up, 2 * m, offsets, K, h, m, status_dev, s);
   // A = x_perm [R, d], B = w_gate_up [K*2m, d] (only experts < K are read)
   return launch_tc<256, EPI_SWIGLU, GU_STAGES, GU_BK>(x_perm, R, d, w_gate_up, static_cast<int64_t>(K) * 2 * m,
                                                      offsets, K, 2 * m, h, m, nullptr, status_dev, s);
@@ -854,6 +1268,8 @@ int decomoe_expert_down(const void* h, const int32_t* offsets, int64_t rows, int
     DM_LAUNCH_CHECK("k_dec_down");
     return DECOMOE_OK;
   }
+  if (static_cast<int64_t>(R) <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K)
+    return launch_ws<false, 4>(h, R, m, w_down, d, offsets, K, y_perm, d, status_dev, s);
   // A = h [R, m], B = w_down [K*d, m]
   return launch_tc<256, EPI_BF16, DN_STAGES, DN_BK>(h, R, m, w_down, static_cast<int64_t>(K) * d, offsets, K, d,
                                                    y_perm, d, nullptr, status_dev, s);

@@ -122,25 +122,27 @@ int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const v
 
   // a1: router logits over all E reordered experts
   DM_RET(decomoe_router_logits(x, w_r, bias, T, d, E, dtype, logits, status_dev, stream));
-  // a2 + a3: full-pool routing, activated mass, shortest covering prefix
+  // a2 (+ a3) and a4: full-pool activated mass and prefix routing
   int K = K_fixed;
-  if (K_fixed == 0 || p > 0.0) {
+  if (K_fixed > 0) {
+    // one launch: prefix routing over [0, K_fixed) and, when p > 0, the
+    // full-pool mass of Eq. 11 (left in the workspace, no host sync)
+    DM_RET(decomoe_route_prefix(logits, T, E, E, K, k, topk_idx, topk_w, p > 0.0 ? mass : nullptr, route_ws,
+                                decomoe_route_workspace_bytes(T, E), stream));
+  } else {
     DM_RET(decomoe_route_prefix(logits, T, E, E, E, k, nullptr, nullptr, mass, route_ws,
                                 decomoe_route_workspace_bytes(T, E), stream));
-    if (K_fixed == 0) {
-      static thread_local std::vector<double> h_mass;
-      h_mass.resize(E);
-      DM_CUDA_CHECK(cudaMemcpyAsync(h_mass.data(), mass, sizeof(double) * E, cudaMemcpyDeviceToHost, s));
-      DM_CUDA_CHECK(cudaStreamSynchronize(s));
-      int Ksel = k;
-      DM_RET(decomoe_select_prefix(h_mass.data(), E, k, p, &Ksel));
-      K = Ksel;
-      if (K_sel_host) *K_sel_host = Ksel;
-    }
+    static thread_local std::vector<double> h_mass;
+    h_mass.resize(E);
+    DM_CUDA_CHECK(cudaMemcpyAsync(h_mass.data(), mass, sizeof(double) * E, cudaMemcpyDeviceToHost, s));
+    DM_CUDA_CHECK(cudaStreamSynchronize(s));
+    int Ksel = k;
+    DM_RET(decomoe_select_prefix(h_mass.data(), E, k, p, &Ksel));
+    K = Ksel;
+    if (K_sel_host) *K_sel_host = Ksel;
+    DM_RET(decomoe_route_prefix(logits, T, E, E, K, k, topk_idx, topk_w, nullptr, nullptr, 0, stream));
   }
   if (K_used_host) *K_used_host = K;
-  // a4: prefix routing
-  DM_RET(decomoe_route_prefix(logits, T, E, E, K, k, topk_idx, topk_w, nullptr, nullptr, 0, stream));
   // a5: dispatch
   DM_RET(decomoe_dispatch(topk_idx, T, k, K, x, d, dtype, counts, offsets, perm, inv, x_perm, disp_ws,
                           decomoe_dispatch_workspace_bytes(T, k, K), status_dev, stream));

@@ -35,99 +35,117 @@ __global__ void k_router_simt(const T* __restrict__ x, const T* __restrict__ w_r
 }
 
 // ------------------------------------------------------------ routing
-// One warp per token. Lane l holds logits l, l+32, ... of the prefix [0, K)
-// in registers (K <= 256, 8 per lane). k rounds of a warp arg-max pick the k
-// largest (ties: lower expert index). Pick j lives in lane j. Weights are the
+// One warp per token; lane l holds logits l, l+32, ... (E <= 256, 8 per lane)
+// in registers. A pass of k rounds of warp arg-max picks the k largest of a
+// range (ties: lower expert index); pick j ends in lane j. Weights are the
 // softmax over the k picks (equal to prefix softmax + top-k + renormalise,
-// because the prefix denominator cancels). With a mass buffer, each block also
-// writes its tokens' fp64 weights per expert, summed in token order, to
-// part[block][e]; k_mass_finalize then sums blocks in block order, so the
-// activated mass of Eq. 11 is bit-reproducible.
+// because the prefix denominator cancels).
+//
+// With a mass buffer the same launch also computes the activated mass of
+// Eq. 11 over the full pool [0, E): the full-pool picks are found first; if
+// they all lie inside [0, K) they are also the prefix picks, else a second
+// pass runs over [0, K). Each block writes its tokens' fp32 full-pool weights
+// per expert, summed in token order, to part[block][e]; k_mass_finalize sums
+// the blocks in a fixed order in fp64, so the mass is bit-reproducible.
 constexpr int ROUTE_THREADS = 256;
 constexpr int ROUTE_TPB = 8;  // tokens per block: one per warp
+
+// k rounds of warp arg-max over entries e < lim not yet taken; returns the
+// pick of round `lane` in (my_v, my_i) and whether every pick is < K.
+__device__ __forceinline__ void warp_topk(const float (&v)[8], int lim, int k, int lane, float& my_v, int& my_i) {
+  uint32_t taken = 0;
+  my_v = 0.f;
+  my_i = 0;
+  for (int j = 0; j < k; ++j) {
+    float bv = 0.f;
+    int bi = INT_MAX;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int e = lane + 32 * i;
+      if (e < lim && !((taken >> i) & 1u)) {
+        if (bi == INT_MAX || v[i] > bv || (v[i] == bv && e < bi)) {
+          bv = v[i];
+          bi = e;
+        }
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+      const bool better = (oi != INT_MAX) && (bi == INT_MAX || ov > bv || (ov == bv && oi < bi));
+      if (better) {
+        bv = ov;
+        bi = oi;
+      }
+    }
+    if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
+    if (lane == j) {
+      my_v = bv;
+      my_i = bi;
+    }
+  }
+}
+
+// Renormalised weight of this lane's pick (lanes >= k get 0).
+__device__ __forceinline__ float pick_weight(float my_v, int lane, int k) {
+  const float v0 = __shfl_sync(0xffffffffu, my_v, 0);
+  const float z = (lane < k) ? __expf(my_v - v0) : 0.f;
+  float zs = z;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) zs += __shfl_xor_sync(0xffffffffu, zs, off);
+  return z / zs;
+}
 
 __global__ void __launch_bounds__(ROUTE_THREADS)
     k_route(const float* __restrict__ logits, int64_t Tn, int E, int64_t ld, int K, int k,
             int32_t* __restrict__ idx_out, float* __restrict__ w_out, double* __restrict__ part) {
   __shared__ int s_idx[ROUTE_TPB][DECOMOE_MAX_TOPK];
-  __shared__ double s_w[ROUTE_TPB][DECOMOE_MAX_TOPK];
+  __shared__ float s_w[ROUTE_TPB][DECOMOE_MAX_TOPK];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t tok0 = static_cast<int64_t>(blockIdx.x) * ROUTE_TPB;
-
-  for (int tt = warp; tt < ROUTE_TPB; tt += ROUTE_THREADS / 32) {
-    const int64_t t = tok0 + tt;
-    if (t >= Tn) break;
+  const int64_t t = static_cast<int64_t>(blockIdx.x) * ROUTE_TPB + warp;
+  const bool mass = part != nullptr;
+  if (t < Tn) {
     const float* row = logits + t * ld;
+    const int lim = mass ? E : K;
     float v[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const int e = lane + 32 * i;
-      v[i] = (e < K) ? row[e] : -FLT_MAX;
+      v[i] = (e < lim) ? row[e] : -FLT_MAX;
     }
-    uint32_t taken = 0;
-    float my_v = 0.f;
-    int my_i = 0;
-    for (int j = 0; j < k; ++j) {
-      float bv = 0.f;
-      int bi = INT_MAX;
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int e = lane + 32 * i;
-        if (e < K && !((taken >> i) & 1u)) {
-          if (bi == INT_MAX || v[i] > bv || (v[i] == bv && e < bi)) {
-            bv = v[i];
-            bi = e;
-          }
-        }
-      }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
-        const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-        const bool better = (oi != INT_MAX) &&
-                            (bi == INT_MAX || ov > bv || (ov == bv && oi < bi));
-        if (better) {
-          bv = ov;
-          bi = oi;
-        }
-      }
-      if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
-      if (lane == j) {
-        my_v = bv;
-        my_i = bi;
-      }
-    }
-    const float v0 = __shfl_sync(0xffffffffu, my_v, 0);
-    // fp32 weights for the routing output
-    float z = (lane < k) ? __expf(my_v - v0) : 0.f;
-    float zs = z;
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) zs += __shfl_xor_sync(0xffffffffu, zs, off);
-    if (lane < k) {
-      if (idx_out != nullptr) idx_out[t * k + lane] = my_i;
-      if (w_out != nullptr) w_out[t * k + lane] = z / zs;
-    }
-    if (part != nullptr) {
-      // fp64 weights for the activated mass (Eq. 11)
-      double zd = (lane < k) ? exp(static_cast<double>(my_v) - static_cast<double>(v0)) : 0.0;
-      double zds = zd;
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) zds += __shfl_xor_sync(0xffffffffu, zds, off);
+    float my_v;
+    int my_i;
+    warp_topk(v, lim, k, lane, my_v, my_i);
+    if (mass) {
+      const float wf = pick_weight(my_v, lane, k);
       if (lane < k) {
-        s_idx[tt][lane] = my_i;
-        s_w[tt][lane] = zd / zds;
+        s_idx[warp][lane] = my_i;
+        s_w[warp][lane] = wf;
+      }
+      // full-pool picks all inside the prefix: they are the prefix picks too
+      const bool inside = __all_sync(0xffffffffu, lane >= k || my_i < K);
+      if (!inside) warp_topk(v, K, k, lane, my_v, my_i);
+    }
+    if (idx_out != nullptr || w_out != nullptr) {
+      const float w = pick_weight(my_v, lane, k);
+      if (lane < k) {
+        if (idx_out != nullptr) idx_out[t * k + lane] = my_i;
+        if (w_out != nullptr) w_out[t * k + lane] = w;
       }
     }
   }
-  if (part == nullptr) return;
+  if (!mass) return;
   __syncthreads();
-  const int ntok = static_cast<int>(Tn - tok0 < ROUTE_TPB ? Tn - tok0 : ROUTE_TPB);
+  const int ntok = static_cast<int>(Tn - static_cast<int64_t>(blockIdx.x) * ROUTE_TPB < ROUTE_TPB
+                                        ? Tn - static_cast<int64_t>(blockIdx.x) * ROUTE_TPB
+                                        : ROUTE_TPB);
   for (int e = threadIdx.x; e < E; e += ROUTE_THREADS) {
-    double acc = 0.0;
+    float acc = 0.f;
     for (int tt = 0; tt < ntok; ++tt)
       for (int j = 0; j < k; ++j)
         if (s_idx[tt][j] == e) acc += s_w[tt][j];  // token order, then slot order
-    part[static_cast<int64_t>(blockIdx.x) * E + e] = acc;
+    part[static_cast<int64_t>(blockIdx.x) * E + e] = static_cast<double>(acc);
   }
 }
 

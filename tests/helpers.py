@@ -12,6 +12,12 @@ F32_REL_L2 = 1e-5
 F32_MAX_ABS = 1e-5
 # Routing weights: |delta| bound on the renormalised top-k weights.
 W_ABS = 1e-6
+# Activated mass (Eq. 11) from fp32 per-token weights: relative error bound
+# (expf <= 2 ulp, one division, renormalising sum over k <= 32 terms and the
+# in-block sum of <= 8 token weights, each ~2^-24 relative), and the band
+# around p inside which the prefix length is reported but not compared.
+MASS_REL = 4e-6
+MASS_P_BAND = 2e-5
 # Tokens whose k-th/(k+1)-th logit gap inside the prefix is below this are
 # reported and left out of index-exact comparisons when both sides use the same
 # fp32 logits.

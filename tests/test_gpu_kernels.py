@@ -12,7 +12,8 @@ import torch
 import paper_2609_38823_gb300 as dm
 import workloads as W
 from oracle import decomoe_oracle as O
-from tests.helpers import (BF16_MAX_ABS, BF16_REL_L2, F32_MAX_ABS, F32_REL_L2, MARGIN_SAME_LOGITS, W_ABS,
+from tests.helpers import (BF16_MAX_ABS, BF16_REL_L2, F32_MAX_ABS, F32_REL_L2, MARGIN_SAME_LOGITS, MASS_P_BAND,
+                           MASS_REL, W_ABS,
                            assert_close_out, bf16_round, f64, logit_error_bound)
 
 pytestmark = pytest.mark.gpu
@@ -99,19 +100,25 @@ def test_route_full_pool_topk_not_intersected():
     assert idx[0].tolist() == [1, 3]
 
 
-@pytest.mark.parametrize("T", [1, 64, 100, 2048, 16384])
-def test_activated_mass_parity_and_reproducible(T):
+@pytest.mark.parametrize("T,K", [(1, 128), (64, 128), (100, 40), (2048, 64), (16384, 128), (777, 8)])
+def test_activated_mass_parity_and_reproducible(T, K):
+    # the mass is Eq. 11 over the full pool whatever prefix K the same launch routes
     E, k = 128, 8
     a = W.make_logits(T, E, std=0.9, bias=_zipf_bias(E), seed=1, wid=20)
-    _, _, m1 = _route_gpu(a, E, k, mass=True)
-    _, _, m2 = _route_gpu(a, E, k, mass=True)
+    idx, w, m1 = _route_gpu(a, K, k, mass=True)
+    _, _, m2 = _route_gpu(a, K, k, mass=True)
+    ri, rw = O.route_prefix(a.numpy(), K, k)
+    keep = O.prefix_margin(a.numpy(), K, k) >= MARGIN_SAME_LOGITS
+    assert np.array_equal(idx[keep], ri[keep]) and np.abs(w[keep] - rw[keep]).max() <= W_ABS
     assert np.array_equal(m1.view(np.uint64), m2.view(np.uint64)), "mass not bit-reproducible"
     ref = O.activated_mass(a.numpy(), k)
-    assert np.abs(m1 - ref).max() <= 1e-12 * max(T, 1)
-    assert abs(m1.sum() - T) <= 1e-9 * T
+    # fp32 per-token weights (expf, one division, sums of <= 8 terms per
+    # block): a few fp32 ulps relative to each expert's mass
+    assert (np.abs(m1 - ref) <= MASS_REL * ref + 1e-30).all()
+    assert abs(m1.sum() - T) <= MASS_REL * T
     cum = np.cumsum(ref) / ref.sum()
     for p in (0.3, 0.5, 0.7, 0.9, 1.0):
-        if p < 1.0 and np.abs(cum - p).min() < 1e-9:
+        if p < 1.0 and np.abs(cum - p).min() < MASS_P_BAND:
             continue  # ratio within rounding of p: K is reported, not compared
         assert dm.decomoe_select_prefix(m1, k, p) == O.select_prefix(ref, p, k)
 
