@@ -189,8 +189,8 @@ class Buffers:
         self.offsets = torch.empty(E + 1, dtype=torch.int32, device=dev)
         self.perm = torch.empty(R, dtype=torch.int32, device=dev)
         self.inv = torch.empty(R, dtype=torch.int32, device=dev)
-        self.x_perm = torch.empty(R, d, dtype=torch.bfloat16, device=dev)
         self.disp_ws = dm.workspace(dm.decomoe_dispatch_workspace_bytes(T, k, E), dev)
+        self.x_perm = torch.empty(R, d, dtype=torch.bfloat16, device=dev)
         self.h = torch.empty(R, m, dtype=torch.bfloat16, device=dev)
         self.y = torch.empty(R, d, dtype=torch.bfloat16, device=dev)
         self.out = torch.empty(T, d, dtype=torch.bfloat16, device=dev)
@@ -242,6 +242,7 @@ def timed(fn, steps, warmup, ws, clocks=None, name="sweep"):
 
 
 def algo_bytes_gate_up(wl, R, D):
+    # weights of the active experts, x_perm rows read, h written
     return D * 2 * wl.m * wl.d * 2 + R * wl.d * 2 + R * wl.m * 2
 
 

@@ -207,6 +207,23 @@ DECOMOE_API int decomoe_expert_down(const void* h, const int32_t* offsets, int64
                                     int dtype, const void* w_down, void* y_perm, int32_t* status_dev,
                                     decomoe_stream_t stream);
 
+/* Gather forms: the expert rows are read straight from the token-ordered
+ * hidden state, row r of the grouped order being x[perm_token[r], :] (TMA
+ * tile::gather4 on the tensor cores), so dispatch need not materialise x_perm
+ * (saves T*k*d elements of memory). Same results bit for bit as the x_perm
+ * forms; slower at prefill sizes, where the four-row gathers, not the tensor
+ * cores, bound the gate/up GEMM. x: [T, d] dtype; perm_token: [rows] int32
+ * from decomoe_dispatch; other arguments and rules as decomoe_expert_gate_up /
+ * decomoe_expert_swiglu. */
+DECOMOE_API int decomoe_expert_gate_up_gather(const void* x, int64_t T, const int32_t* perm_token,
+                                              const int32_t* offsets, int64_t rows, int K, int d, int m,
+                                              int dtype, const void* w_gate_up, void* h, int32_t* status_dev,
+                                              decomoe_stream_t stream);
+DECOMOE_API int decomoe_expert_swiglu_gather(const void* x, int64_t T, const int32_t* perm_token,
+                                             const int32_t* offsets, int64_t rows, int K, int d, int m, int dtype,
+                                             const void* w_gate_up, const void* w_down, void* h_ws,
+                                             void* y_perm, int32_t* status_dev, decomoe_stream_t stream);
+
 /* CUDA-core reference of decomoe_expert_swiglu for bf16 storage: the same
  * arithmetic (bf16 products, fp32 accumulation, h rounded to bf16) with one
  * thread per output element and no tensor cores. It is slow; it exists to

@@ -54,6 +54,8 @@ SIGNATURES = {
     "decomoe_expert_swiglu": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P]),
     "decomoe_expert_gate_up": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P]),
     "decomoe_expert_down": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P]),
+    "decomoe_expert_gate_up_gather": (_I, [_P, _L, _P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P]),
+    "decomoe_expert_swiglu_gather": (_I, [_P, _L, _P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P]),
     "decomoe_expert_swiglu_ref": (_I, [_P, _P, _L, _I, _I, _I, _P, _P, _P, _P, _P]),
     "decomoe_combine": (_I, [_P, _P, _P, _L, _I, _I, _I, _P, _P, _P]),
     "decomoe_drop_visual_block": (_I, [_P, _P, _L, _L, _L, _L, _L, _L, _L, _P]),
@@ -259,6 +261,28 @@ def decomoe_expert_down(h, offsets, K, w_down, y_perm, status=None, stream=None)
     _check("decomoe_expert_down",
            lib().decomoe_expert_down(_ptr(h), _ptr(offsets), rows, K, d, m, _dt(h), _ptr(w_down), _ptr(y_perm),
                                      _ptr(status), _stream(stream)))
+
+
+def decomoe_expert_gate_up_gather(x, perm_token, offsets, K, w_gate_up, h, status=None, stream=None):
+    _need_cuda(x, perm_token, offsets, w_gate_up, h, status)
+    T, d = x.shape
+    rows = perm_token.shape[0]
+    m = h.shape[1]
+    _check("decomoe_expert_gate_up_gather",
+           lib().decomoe_expert_gate_up_gather(_ptr(x), T, _ptr(perm_token), _ptr(offsets), rows, K, d, m, _dt(x),
+                                               _ptr(w_gate_up), _ptr(h), _ptr(status), _stream(stream)))
+
+
+def decomoe_expert_swiglu_gather(x, perm_token, offsets, K, w_gate_up, w_down, h_ws, y_perm, status=None,
+                                 stream=None):
+    _need_cuda(x, perm_token, offsets, w_gate_up, w_down, h_ws, y_perm, status)
+    T, d = x.shape
+    rows = perm_token.shape[0]
+    m = w_down.shape[2]
+    _check("decomoe_expert_swiglu_gather",
+           lib().decomoe_expert_swiglu_gather(_ptr(x), T, _ptr(perm_token), _ptr(offsets), rows, K, d, m, _dt(x),
+                                              _ptr(w_gate_up), _ptr(w_down), _ptr(h_ws), _ptr(y_perm),
+                                              _ptr(status), _stream(stream)))
 
 
 def decomoe_expert_swiglu_ref(x_perm, offsets, K, w_gate_up, w_down, h_ws, y_perm, stream=None):

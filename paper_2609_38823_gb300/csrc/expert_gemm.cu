@@ -97,6 +97,7 @@ struct TcArgs {
   int32_t* status;
   uint64_t limit_ns;
   int n_valid;  // EPI_F32_BIAS_T: number of valid output columns (tokens)
+  const int32_t* a_rows;  // GATHER_A: A row r is row a_rows[r] of the A tensor (rows entries)
 };
 
 template <int BN, int STAGES, int BK_>
@@ -154,11 +155,12 @@ __device__ __forceinline__ void tile_coords(int tile, int NT, const int* s_mt, i
   mt = mtg - s_mt[lo];
 }
 
-template <int BN, int EPI, int STAGES, int BK>
+template <int BN, int EPI, int STAGES, int BK, bool GATHER_A = false>
 __global__ void __launch_bounds__(192, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b,
               const TcArgs g) {
   using C = TcCfg<BN, STAGES, BK>;
+  __shared__ int s_arow[GATHER_A ? 128 : 1];
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
@@ -242,37 +244,78 @@ __global__ void __launch_bounds__(192, 1)
   const uint32_t tmem_base = *s_tmem;
   const int KB = g.kdim / C::BK;
 
-  if (warp == 0 && lane == 0) {
-    // ------------------------------------------------ TMA producer
-    tma_prefetch_desc(&tma_a);
-    tma_prefetch_desc(&tma_b);
+  if (warp == 0) {
+    // ------------------------------------------------ TMA producer (lane 0
+    // issues; with GATHER_A the whole warp first reads the tile's 128 A row
+    // indices into shared memory)
+    if (lane == 0) {
+      tma_prefetch_desc(&tma_a);
+      tma_prefetch_desc(&tma_b);
+    }
     int stage = 0;
     uint32_t ph = 0;
     bool ok = true;
     uint32_t armed = 0;  // bit s: stage s was ever filled
     uint32_t armed_ph = 0;
-    for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
       int grp, mt, nb;
       tile_coords(tile, NT, s_mt, G, grp, mt, nb);
       const int row0 = s_off[grp] + mt * C::BM;
       const int brow = grp * g.n_per_group + nb * BN;
-      for (int kb = 0; kb < KB; ++kb) {
-        if (!mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort)) {
-          ok = false;
-          break;
+      if constexpr (GATHER_A) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int r = row0 + lane * 4 + i;
+          s_arow[lane * 4 + i] = (r < g.rows) ? g.a_rows[r] : 0;  // rows past the end: any valid row, not stored
         }
-        mbar_arrive_expect_tx(FULL_BAR(stage), C::STAGE_BYTES);
-        tma_load_2d(sA + stage * C::A_BYTES, &tma_a, FULL_BAR(stage), kb * C::BK, row0);
-        tma_load_2d(sB + stage * C::B_BYTES, &tma_b, FULL_BAR(stage), kb * C::BK, brow);
-        armed |= 1u << stage;
-        armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
-        if (++stage == STAGES) {
-          stage = 0;
-          ph ^= 1u;
+        __syncwarp();
+      }
+      if constexpr (GATHER_A) {
+        // the warp issues the 32 four-row gathers of a k-block in parallel
+        for (int kb = 0; kb < KB; ++kb) {
+          bool got = true;
+          if (lane == 0) got = mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort);
+          got = __shfl_sync(0xffffffffu, got, 0);
+          if (!got) {
+            ok = false;
+            break;
+          }
+          if (lane == 0) {
+            mbar_arrive_expect_tx(FULL_BAR(stage), C::STAGE_BYTES);
+            tma_load_2d(sB + stage * C::B_BYTES, &tma_b, FULL_BAR(stage), kb * C::BK, brow);
+          }
+          __syncwarp();
+          const uint32_t dA = sA + stage * C::A_BYTES;
+          tma_gather4(dA + lane * 4 * (C::BK * 2), &tma_a, FULL_BAR(stage), kb * C::BK, s_arow[4 * lane],
+                      s_arow[4 * lane + 1], s_arow[4 * lane + 2], s_arow[4 * lane + 3]);
+          armed |= 1u << stage;
+          armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            ph ^= 1u;
+          }
+        }
+      } else if (lane == 0) {
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(FULL_BAR(stage), C::STAGE_BYTES);
+          tma_load_2d(sA + stage * C::A_BYTES, &tma_a, FULL_BAR(stage), kb * C::BK, row0);
+          tma_load_2d(sB + stage * C::B_BYTES, &tma_b, FULL_BAR(stage), kb * C::BK, brow);
+          armed |= 1u << stage;
+          armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            ph ^= 1u;
+          }
         }
       }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
     }
-    if (!ok) {
+    if (lane == 0 && !ok) {
       *s_abort = 1;
       report_status(g.status, DECOMOE_ERR_TIMEOUT);
       // let every copy this thread started land before the CTA can exit
@@ -467,13 +510,19 @@ __global__ void __launch_bounds__(192, 1)
 #undef DRAIN_BAR
 }
 
-template <int BN, int EPI, int STAGES, int BK>
+// A: [rows, kdim], or with GATHER_A the source tensor [a_tensor_rows, kdim]
+// whose row a_rows[r] is A row r.
+template <int BN, int EPI, int STAGES, int BK, bool GATHER_A = false>
 static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b_rows,
                      const int32_t* offsets, int ngroups, int n_per_group, void* out,
-                     int64_t out_ld, const float* bias, int32_t* status, cudaStream_t s, int n_valid = 0) {
+                     int64_t out_ld, const float* bias, int32_t* status, cudaStream_t s, int n_valid = 0,
+                     const int32_t* a_rows = nullptr, int64_t a_tensor_rows = 0) {
   using C = TcCfg<BN, STAGES, BK>;
   CUtensorMap ta, tb;
-  DM_RET(make_tmap_bf16(&ta, A, static_cast<uint64_t>(kdim), static_cast<uint64_t>(rows), C::BM, BK));
+  if (GATHER_A)
+    DM_RET(make_tmap_bf16(&ta, A, static_cast<uint64_t>(kdim), static_cast<uint64_t>(a_tensor_rows), 1, BK));
+  else
+    DM_RET(make_tmap_bf16(&ta, A, static_cast<uint64_t>(kdim), static_cast<uint64_t>(rows), C::BM, BK));
   DM_RET(make_tmap_bf16(&tb, B, static_cast<uint64_t>(kdim), static_cast<uint64_t>(b_rows), BN, BK));
   TcArgs g;
   g.offsets = offsets;
@@ -487,7 +536,8 @@ static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b
   g.status = status;
   g.limit_ns = static_cast<uint64_t>(wait_limit_ns());
   g.n_valid = n_valid;
-  auto kern = k_gemm_tc<BN, EPI, STAGES, BK>;
+  g.a_rows = a_rows;
+  auto kern = k_gemm_tc<BN, EPI, STAGES, BK, GATHER_A>;
   static_assert(C::SMEM <= 232448, "shared memory budget");
   DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(C::SMEM)));
@@ -533,6 +583,7 @@ struct WsArgs {
   int64_t out_ld;
   int32_t* status;
   uint64_t limit_ns;
+  const int32_t* b_rows;  // GATHER_B: token row r is row b_rows[r] of the activation tensor
 };
 
 #ifndef DECOMOE_WS_BOX
@@ -594,11 +645,12 @@ __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
-template <bool SWIGLU, int STAGES>
+template <bool SWIGLU, int STAGES, bool GATHER_B = false>
 __global__ void __launch_bounds__(192, 1)
     k_moe_ws(const __grid_constant__ CUtensorMap tma_w, const __grid_constant__ CUtensorMap tma_x,
              const WsArgs g) {
   using C = WsCfg<STAGES, SWIGLU>;
+  __shared__ int s_brow[GATHER_B ? WS_BN : 1];
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
@@ -683,38 +735,61 @@ __global__ void __launch_bounds__(192, 1)
   const uint32_t tmem_base = *s_tmem;
   const int KB = g.kdim / WS_BK;
 
-  if (warp == 0 && lane == 0) {
-    // ------------------------------------------------ TMA producer
-    tma_prefetch_desc(&tma_w);
-    tma_prefetch_desc(&tma_x);
+  if (warp == 0) {
+    // ------------------------------------------------ TMA producer (lane 0
+    // issues; with GATHER_B the warp first reads the tile's token row indices)
+    if (lane == 0) {
+      tma_prefetch_desc(&tma_w);
+      tma_prefetch_desc(&tma_x);
+    }
     int stage = 0;
     uint32_t ph = 0;
     bool ok = true;
     uint32_t armed = 0, armed_ph = 0;
-    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+    for (int t = blockIdx.x; t < total; t += gridDim.x) {
       const WsTile T = ws_tile(t, total, s_tt, s_off, G, nwb);
       const int wrow0 = T.g * g.wrows + T.wb * WS_BM;
-      const int nbox = (T.ntok + WS_BOX - 1) / WS_BOX;
-      const uint32_t bytes = C::A_BYTES + nbox * C::BOX_BYTES;
-      for (int kb = 0; kb < KB; ++kb) {
-        if (!mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort)) {
-          ok = false;
-          break;
-        }
-        mbar_arrive_expect_tx(FULL_BAR(stage), bytes);
-        tma_load_2d(sA + stage * C::A_BYTES, &tma_w, FULL_BAR(stage), kb * WS_BK, wrow0);
-        for (int i = 0; i < nbox; ++i)
-          tma_load_2d(sB + stage * C::B_BYTES + i * C::BOX_BYTES, &tma_x, FULL_BAR(stage), kb * WS_BK,
-                      T.row0 + i * WS_BOX);
-        armed |= 1u << stage;
-        armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
-        if (++stage == STAGES) {
-          stage = 0;
-          ph ^= 1u;
+      int nload;       // TMA copies for B per k-block
+      uint32_t bytes;  // bytes landing per stage
+      if constexpr (GATHER_B) {
+        for (int i = lane; i < WS_BN; i += 32)
+          s_brow[i] = (i < T.ntok) ? g.b_rows[T.row0 + i] : 0;  // padding rows: any valid row, never stored
+        __syncwarp();
+        nload = (T.ntok + 3) / 4;
+        bytes = C::A_BYTES + nload * 4 * WS_BK * 2;
+      } else {
+        nload = (T.ntok + WS_BOX - 1) / WS_BOX;
+        bytes = C::A_BYTES + nload * C::BOX_BYTES;
+      }
+      if (lane == 0) {
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(FULL_BAR(stage), bytes);
+          tma_load_2d(sA + stage * C::A_BYTES, &tma_w, FULL_BAR(stage), kb * WS_BK, wrow0);
+          const uint32_t dB = sB + stage * C::B_BYTES;
+          if constexpr (GATHER_B) {
+            for (int i = 0; i < nload; ++i)
+              tma_gather4(dB + i * 4 * WS_BK * 2, &tma_x, FULL_BAR(stage), kb * WS_BK, s_brow[4 * i],
+                          s_brow[4 * i + 1], s_brow[4 * i + 2], s_brow[4 * i + 3]);
+          } else {
+            for (int i = 0; i < nload; ++i)
+              tma_load_2d(dB + i * C::BOX_BYTES, &tma_x, FULL_BAR(stage), kb * WS_BK, T.row0 + i * WS_BOX);
+          }
+          armed |= 1u << stage;
+          armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            ph ^= 1u;
+          }
         }
       }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
     }
-    if (!ok) {
+    if (lane == 0 && !ok) {
       *s_abort = 1;
       report_status(g.status, DECOMOE_ERR_TIMEOUT);
       int no_abort = 0;
@@ -852,14 +927,20 @@ __global__ void __launch_bounds__(192, 1)
 #undef DRAIN_BAR
 }
 
-// X: [rows, kdim] token rows grouped by expert; W: [G * wrows, kdim].
-template <bool SWIGLU, int STAGES>
+// X: [rows, kdim] token rows grouped by expert, or with GATHER_B the source
+// tensor [x_tensor_rows, kdim] whose row b_rows[r] is token row r;
+// W: [G * wrows, kdim].
+template <bool SWIGLU, int STAGES, bool GATHER_B = false>
 static int launch_ws(const void* X, int rows, int kdim, const void* W, int wrows, const int32_t* offsets, int G,
-                     void* out, int64_t out_ld, int32_t* status, cudaStream_t s) {
+                     void* out, int64_t out_ld, int32_t* status, cudaStream_t s, const int32_t* b_rows = nullptr,
+                     int64_t x_tensor_rows = 0) {
   using C = WsCfg<STAGES, SWIGLU>;
   CUtensorMap tw, tx;
   DM_RET(make_tmap_bf16(&tw, W, static_cast<uint64_t>(kdim), static_cast<uint64_t>(G) * wrows, WS_BM, WS_BK));
-  DM_RET(make_tmap_bf16(&tx, X, static_cast<uint64_t>(kdim), static_cast<uint64_t>(rows), WS_BOX, WS_BK));
+  if (GATHER_B)
+    DM_RET(make_tmap_bf16(&tx, X, static_cast<uint64_t>(kdim), static_cast<uint64_t>(x_tensor_rows), 1, WS_BK));
+  else
+    DM_RET(make_tmap_bf16(&tx, X, static_cast<uint64_t>(kdim), static_cast<uint64_t>(rows), WS_BOX, WS_BK));
   WsArgs g;
   g.offsets = offsets;
   g.G = G;
@@ -870,7 +951,8 @@ static int launch_ws(const void* X, int rows, int kdim, const void* W, int wrows
   g.out_ld = out_ld;
   g.status = status;
   g.limit_ns = static_cast<uint64_t>(wait_limit_ns());
-  auto kern = k_moe_ws<SWIGLU, STAGES>;
+  g.b_rows = b_rows;
+  auto kern = k_moe_ws<SWIGLU, STAGES, GATHER_B>;
   static_assert(C::SMEM <= 232448, "shared memory budget");
   DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(C::SMEM)));
   const int64_t ub_tiles = (static_cast<int64_t>(rows) / WS_BN + G) * (wrows / WS_BM);
@@ -938,7 +1020,8 @@ __device__ __forceinline__ int find_group(const int32_t* __restrict__ offsets, i
 // layout. One thread per (row, feature).
 template <typename T>
 __global__ void k_simt_gate_up(const T* __restrict__ A, const int32_t* __restrict__ offsets, int G,
-                               const T* __restrict__ Wgu, int d, int m, T* __restrict__ H) {
+                               const T* __restrict__ Wgu, int d, int m, T* __restrict__ H,
+                               const int32_t* __restrict__ a_rows) {
   const int rows = offsets[G];
   const int f = blockIdx.x * blockDim.x + threadIdx.x;
   if (f >= m) return;
@@ -948,7 +1031,7 @@ __global__ void k_simt_gate_up(const T* __restrict__ A, const int32_t* __restric
     const int64_t grow = static_cast<int64_t>(e) * 2 * m + blk * 2 * DECOMOE_GU_BLOCK + i;
     const T* wg = Wgu + grow * d;
     const T* wu = wg + static_cast<int64_t>(DECOMOE_GU_BLOCK) * d;
-    const T* x = A + static_cast<int64_t>(r) * d;
+    const T* x = A + static_cast<int64_t>(a_rows ? a_rows[r] : r) * d;
     float ag = 0.f, au = 0.f;
     for (int j = 0; j < d; ++j) {
       const float xv = ld_f(x + j);
@@ -1221,7 +1304,8 @@ int decomoe_expert_gate_up(const void* x_perm, const int32_t* offsets, int64_t r
   if (dtype == DECOMOE_F32) {
     dim3 g1((m + 127) / 128, static_cast<unsigned>(std::min(R, 65535)));
     k_simt_gate_up<float><<<g1, 128, 0, s>>>(static_cast<const float*>(x_perm), offsets, K,
-                                              static_cast<const float*>(w_gate_up), d, m, static_cast<float*>(h));
+                                              static_cast<const float*>(w_gate_up), d, m, static_cast<float*>(h),
+                                              nullptr);
     DM_LAUNCH_CHECK("k_simt_gate_up");
     return DECOMOE_OK;
   }
@@ -1275,6 +1359,39 @@ int decomoe_expert_down(const void* h, const int32_t* offsets, int64_t rows, int
                                                    y_perm, d, nullptr, status_dev, s);
 }
 
+int decomoe_expert_gate_up_gather(const void* x, int64_t T, const int32_t* perm_token, const int32_t* offsets,
+                                  int64_t rows, int K, int d, int m, int dtype, const void* w_gate_up, void* h,
+                                  int32_t* status_dev, decomoe_stream_t stream) {
+  clear_error();
+  DM_RET(expert_check("expert_gate_up_gather", x, offsets, rows, K, d, m, dtype, w_gate_up, h));
+  if (rows == 0) return DECOMOE_OK;
+  DM_ARG_CHECK(perm_token != nullptr && T > 0 && T < 0x7fffffffLL, "expert_gate_up_gather: bad perm_token or T");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int R = static_cast<int>(rows);
+  if (dtype == DECOMOE_F32) {
+    dim3 g1((m + 127) / 128, static_cast<unsigned>(std::min(R, 65535)));
+    k_simt_gate_up<float><<<g1, 128, 0, s>>>(static_cast<const float*>(x), offsets, K,
+                                              static_cast<const float*>(w_gate_up), d, m, static_cast<float*>(h),
+                                              perm_token);
+    DM_LAUNCH_CHECK("k_simt_gate_up");
+    return DECOMOE_OK;
+  }
+  if (static_cast<int64_t>(R) <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K)
+    return launch_ws<true, 4, true>(x, R, d, w_gate_up, 2 * m, offsets, K, h, m, status_dev, s, perm_token, T);
+  return launch_tc<256, EPI_SWIGLU, GU_STAGES, GU_BK, true>(x, R, d, w_gate_up, static_cast<int64_t>(K) * 2 * m,
+                                                            offsets, K, 2 * m, h, m, nullptr, status_dev, s, 0,
+                                                            perm_token, T);
+}
+
+int decomoe_expert_swiglu_gather(const void* x, int64_t T, const int32_t* perm_token, const int32_t* offsets,
+                                 int64_t rows, int K, int d, int m, int dtype, const void* w_gate_up,
+                                 const void* w_down, void* h_ws, void* y_perm, int32_t* status_dev,
+                                 decomoe_stream_t stream) {
+  DM_RET(decomoe_expert_gate_up_gather(x, T, perm_token, offsets, rows, K, d, m, dtype, w_gate_up, h_ws,
+                                       status_dev, stream));
+  return decomoe_expert_down(h_ws, offsets, rows, K, d, m, dtype, w_down, y_perm, status_dev, stream);
+}
+
 int decomoe_expert_swiglu(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m,
                           int dtype, const void* w_gate_up, const void* w_down, void* h_ws, void* y_perm,
                           int32_t* status_dev, decomoe_stream_t stream) {
@@ -1298,7 +1415,7 @@ int decomoe_expert_swiglu_ref(const void* x_perm, const int32_t* offsets, int64_
   dim3 g1((m + 127) / 128, static_cast<unsigned>(std::min(R, 65535)));
   k_simt_gate_up<__nv_bfloat16><<<g1, 128, 0, s>>>(static_cast<const __nv_bfloat16*>(x_perm), offsets, K,
                                                     static_cast<const __nv_bfloat16*>(w_gate_up), d, m,
-                                                    static_cast<__nv_bfloat16*>(h_ws));
+                                                    static_cast<__nv_bfloat16*>(h_ws), nullptr);
   DM_LAUNCH_CHECK("k_simt_gate_up<bf16>");
   dim3 g2((d + 127) / 128, static_cast<unsigned>(std::min(R, 65535)));
   k_simt_down<__nv_bfloat16><<<g2, 128, 0, s>>>(static_cast<const __nv_bfloat16*>(h_ws), offsets, K,

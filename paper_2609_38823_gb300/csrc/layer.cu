@@ -143,7 +143,7 @@ int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const v
     DM_RET(decomoe_route_prefix(logits, T, E, E, K, k, topk_idx, topk_w, nullptr, nullptr, 0, stream));
   }
   if (K_used_host) *K_used_host = K;
-  // a5: dispatch
+  // a5: dispatch (counts, offsets, permutation, x_perm rows)
   DM_RET(decomoe_dispatch(topk_idx, T, k, K, x, d, dtype, counts, offsets, perm, inv, x_perm, disp_ws,
                           decomoe_dispatch_workspace_bytes(T, k, K), status_dev, stream));
   // a6: grouped SwiGLU experts over [0, K)

@@ -97,6 +97,6 @@ def test_workspace_queries():
     assert dm.decomoe_route_workspace_bytes(2048, 128) >= 32 * 128 * 8
     assert dm.decomoe_dispatch_workspace_bytes(2048, 8, 128) >= 16 * 128 * 4
     b = dm.decomoe_moe_layer_workspace_bytes(2048, 2048, 128, 8, 768, 0)
-    assert b >= 2048 * 8 * (2048 * 2 * 2 + 768 * 2)
+    assert b >= 2048 * 8 * (2048 * 2 * 2 + 768 * 2)  # x_perm, y_perm and h
     offs = dm.decomoe_moe_layer_workspace_layout(2048, 2048, 128, 8, 768, 0)
     assert offs == sorted(offs) and all(o % 256 == 0 for o in offs)

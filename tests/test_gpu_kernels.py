@@ -196,6 +196,7 @@ def _expert_case(T, k, K, d, m, pattern, seed, dtype=torch.bfloat16):
     idx = _idx_pattern(T, k, K, pattern, seed)
     counts, offsets, perm, inv = O.dispatch(idx, K)
     x_perm = L["x"][torch.from_numpy(perm)]
+    L["perm"] = perm
     return L, x_perm, offsets
 
 
@@ -235,6 +236,15 @@ def test_expert_swiglu_bf16_parity(T, k, K, d, m, pattern):
     dm.decomoe_expert_swiglu_ref(xp, off, K, w_gu, g["w_down"], h2, y2)
     torch.cuda.synchronize()
     assert_close_out(f64(y), f64(y2), 2e-3, 1e-2, "tensor-core vs CUDA-core reference")
+    # gather form: rows read from the token-ordered x through perm_token give
+    # the same shared-memory tiles, so the same bits
+    h3 = torch.empty_like(h)
+    y3 = torch.empty_like(y)
+    perm_d = torch.from_numpy(L["perm"].astype(np.int32)).to(DEV)
+    dm.decomoe_expert_swiglu_gather(L["x"].to(DEV), perm_d, off, K, w_gu, g["w_down"], h3, y3, status)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(status) == 0
+    assert torch.equal(y3, y) and torch.equal(h3, h)
 
 
 def test_expert_swiglu_f32_parity():
@@ -249,6 +259,11 @@ def test_expert_swiglu_f32_parity():
     torch.cuda.synchronize()
     ref = O.expert_swiglu(f64(x_perm), offsets, f64(L["w_gate"]), f64(L["w_up"]), f64(L["w_down"]))
     assert_close_out(f64(y), ref, F32_REL_L2, F32_MAX_ABS, "fp32 expert_swiglu")
+    y3 = torch.empty_like(y)
+    perm_d = torch.from_numpy(L["perm"].astype(np.int32)).to(DEV)
+    dm.decomoe_expert_swiglu_gather(L["x"].to(DEV), perm_d, off, K, w_gu, g["w_down"], torch.empty_like(h), y3)
+    torch.cuda.synchronize()
+    assert torch.equal(y3, y)
 
 
 def test_weight_layout_interleave():
