@@ -267,10 +267,29 @@ def ours(args, ws, rank, local):
 
     clocks = Clocks(local) if rank == 0 else None
 
+    # The timed steps replay one CUDA graph per rotated layer (launch overhead
+    # out of the way); events captured into each graph bracket its two expert
+    # GEMMs, so after the loop they hold the durations of the last replay of
+    # every graph. Without event capture support the steps run eagerly.
+    timing_mode = "cuda-graph replay"
+    try:
+        gevs = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(3)] for _ in layers]
+        graphs = [dm.capture_graph(lambda L=L, ev=ev: run_step(dm, wl, L, B, K, v0, nv, text, ev))
+                  for L, ev in zip(layers, gevs)]
+    except (TypeError, RuntimeError):
+        torch.cuda.synchronize()
+        timing_mode = "eager"
+        graphs = None
+
     def step(i, ev):
-        run_step(dm, wl, layers[i % len(layers)], B, K, v0, nv, text, ev)
+        if graphs is not None:
+            graphs[i % len(graphs)].replay()
+        else:
+            run_step(dm, wl, layers[i % len(layers)], B, K, v0, nv, text, ev)
 
     ms, evs = timed(step, args.steps, args.warmup, ws, clocks, name="timed")
+    if graphs is not None:
+        evs = gevs[:min(len(gevs), args.steps)]
     # extend the clock window when the timed region is shorter than ~1.5 s
     ext = 0
     if clocks and ms < 1500:
@@ -286,8 +305,9 @@ def ours(args, ws, rank, local):
     ms_max = max_over_ranks(ms, ws)
     step_ms = ms_max / args.steps
     tok_s = ws * T * args.steps / (ms_max / 1e3)
-    gu_ms = statistics.mean(evs[i][0].elapsed_time(evs[i][1]) for i in range(args.steps))
-    dn_ms = statistics.mean(evs[i][1].elapsed_time(evs[i][2]) for i in range(args.steps))
+    gu_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    dn_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    del graphs
     # distinct active experts per layer (for the algorithmic bytes)
     Ds = []
     for l in range(len(layers)):
@@ -374,6 +394,7 @@ def ours(args, ws, rank, local):
         "roofline": roof,
         "e2e": e2e,
         "gpu_launches": LAUNCHES_PER_STEP * args.steps,
+        "timing_mode": timing_mode,
         "clocks": clk,
         "clock_window": "timed region" if ext == 0 else f"timed region + {ext} identical untimed steps",
         "sweep": sweep,
@@ -395,7 +416,7 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
         D = int((B.counts[:K] > 0).sum())
         ffn_fl = 6.0 * R * wl.d * wl.m
         ffn_by = algo_bytes_gate_up(wl, R, D) + algo_bytes_down(wl, R, D)
-        out.append({"mode": "fixed", "K": K, "tokens_per_s": round(T * n / (ms / 1e3), 1),
+        out.append({"mode": "fixed (eager launches)", "K": K, "tokens_per_s": round(T * n / (ms / 1e3), 1),
                     "ms_per_step": round(ms / n, 4), "ffn_ms": round(gu + dn, 4),
                     "ffn_tflops": round(ffn_fl / ((gu + dn) * 1e-3) / 1e12, 2),
                     "ffn_tensor_frac": round(ffn_fl / ((gu + dn) * 1e-3) / 1e12 / pk["bf16_tflops"], 4),
@@ -414,12 +435,6 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
     ms, _ = timed(ad_step, n, 5, ws)
     out.append({"mode": f"mass p={args.p}", "K_mean": round(statistics.mean(Ks[-n:]), 2),
                 "tokens_per_s": round(T * n / (ms / 1e3), 1), "ms_per_step": round(ms / n, 4)})
-    # the same fixed-K step replayed from CUDA graphs (one per rotated layer)
-    graphs = [dm.capture_graph(lambda L=L: run_step(dm, wl, L, B, args.K, wl.v0, wl.nv, text)) for L in layers]
-    ms, _ = timed(lambda i, ev: graphs[i % len(graphs)].replay(), n, 5, ws)
-    out.append({"mode": "fixed, CUDA graph", "K": args.K, "tokens_per_s": round(T * n / (ms / 1e3), 1),
-                "ms_per_step": round(ms / n, 4)})
-    del graphs
     # decode-size layers, K=64: weight streaming, reported against HBM
     for Td in W.DECODE_T:
         Bd = Buffers(wl, Td, B.out.device, dm)

@@ -100,13 +100,18 @@ struct TcArgs {
   const int32_t* a_rows;  // GATHER_A: A row r is row a_rows[r] of the A tensor (rows entries)
 };
 
-template <int BN, int STAGES, int BK_>
+// MP = M-tiles per work item. MP = 1: one 128-row A tile per B tile, two
+// accumulator buffers (epilogue overlaps the next tile's MMAs). MP = 2: two
+// M-tiles of the same group share each B tile (two M=128 MMAs per k-step,
+// 2/3 of the shared-memory traffic per MMA), one buffer of two accumulators.
+template <int BN, int STAGES, int BK_, int MP_ = 1>
 struct TcCfg {
-  static constexpr int BM = 128, BK = BK_;
-  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int BM = 128, BK = BK_, MP = MP_;
+  static constexpr int A_BYTES = BM * BK * 2;  // one M-tile
   static constexpr int B_BYTES = BN * BK * 2;
-  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int TMEM_COLS = 2 * BN;  // two accumulator buffers
+  static constexpr int STAGE_BYTES = MP * A_BYTES + B_BYTES;
+  static constexpr int NBUF = MP == 1 ? 2 : 1;  // accumulator buffers
+  static constexpr int TMEM_COLS = 2 * BN;      // NBUF * MP accumulators of BN columns
   static constexpr int MAXG = DECOMOE_MAX_E;
   static constexpr int NBARS = 2 * STAGES + 5;
   static constexpr size_t SMEM =
@@ -155,18 +160,21 @@ __device__ __forceinline__ void tile_coords(int tile, int NT, const int* s_mt, i
   mt = mtg - s_mt[lo];
 }
 
-template <int BN, int EPI, int STAGES, int BK, bool GATHER_A = false>
-__global__ void __launch_bounds__(192, 1)
+// EW epilogue warps (4 or 8): with 8, two warps share each 32-lane TMEM
+// quarter and split its column chunks, so the epilogue's latency is hidden.
+template <int BN, int EPI, int STAGES, int BK, bool GATHER_A = false, int MP = 1, int EW = 8>
+__global__ void __launch_bounds__(64 + 32 * EW, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b,
               const TcArgs g) {
-  using C = TcCfg<BN, STAGES, BK>;
+  using C = TcCfg<BN, STAGES, BK, MP>;
+  static_assert(!(GATHER_A && MP != 1), "gathered A takes one M-tile per work item");
   __shared__ int s_arow[GATHER_A ? 128 : 1];
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
   uint8_t* smem = smem_raw + pad;
   const uint32_t sA = raw + pad;
-  const uint32_t sB = sA + STAGES * C::A_BYTES;
+  const uint32_t sB = sA + STAGES * MP * C::A_BYTES;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
   int* s_off = reinterpret_cast<int*>(bars + C::NBARS);
   int* s_mt = s_off + (C::MAXG + 1);
@@ -193,14 +201,14 @@ __global__ void __launch_bounds__(192, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(TFULL_BAR(a), 1);
-      mbar_init(TEMPTY_BAR(a), 128);
+      mbar_init(TEMPTY_BAR(a), 32 * EW);
     }
     mbar_init(DRAIN_BAR, 1);
     fence_mbar_init();
   }
   __syncthreads();
   if (warp == 2) {
-    // exclusive scan of M-tiles per group: s_mt[g] = first global M-tile of g
+    // exclusive scan of work units (MP M-tiles) per group: s_mt[g] = first unit of g
     const int per = (G + 31) / 32;  // <= 8
     int loc[8];
     int sum = 0;
@@ -210,7 +218,7 @@ __global__ void __launch_bounds__(192, 1)
       const int gi = lane * per + i;
       if (i < per && gi < G) {
         const int n = s_off[gi + 1] - s_off[gi];
-        loc[i] = n > 0 ? (n + C::BM - 1) / C::BM : 0;
+        loc[i] = n > 0 ? (n + C::BM * MP - 1) / (C::BM * MP) : 0;
       }
       sum += loc[i];
     }
@@ -260,8 +268,9 @@ __global__ void __launch_bounds__(192, 1)
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
       int grp, mt, nb;
       tile_coords(tile, NT, s_mt, G, grp, mt, nb);
-      const int row0 = s_off[grp] + mt * C::BM;
+      const int row0 = s_off[grp] + mt * MP * C::BM;
       const int brow = grp * g.n_per_group + nb * BN;
+      const bool has2 = MP == 2 && row0 + C::BM < s_off[grp + 1];  // second M-tile has rows
       if constexpr (GATHER_A) {
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
@@ -301,8 +310,10 @@ __global__ void __launch_bounds__(192, 1)
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(FULL_BAR(stage), C::STAGE_BYTES);
-          tma_load_2d(sA + stage * C::A_BYTES, &tma_a, FULL_BAR(stage), kb * C::BK, row0);
+          mbar_arrive_expect_tx(FULL_BAR(stage), (has2 ? 2 : 1) * C::A_BYTES + C::B_BYTES);
+          tma_load_2d(sA + stage * MP * C::A_BYTES, &tma_a, FULL_BAR(stage), kb * C::BK, row0);
+          if (has2)
+            tma_load_2d(sA + (stage * MP + 1) * C::A_BYTES, &tma_a, FULL_BAR(stage), kb * C::BK, row0 + C::BM);
           tma_load_2d(sB + stage * C::B_BYTES, &tma_b, FULL_BAR(stage), kb * C::BK, brow);
           armed |= 1u << stage;
           armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
@@ -331,8 +342,14 @@ __global__ void __launch_bounds__(192, 1)
     bool ok = true, issued = false;
     int it = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
-      const int acc = it & 1;
-      const uint32_t aph = (it >> 1) & 1;
+      const int acc = it % C::NBUF;
+      const uint32_t aph = (it / C::NBUF) & 1;
+      bool has2 = false;
+      if constexpr (MP == 2) {
+        int grp, mt, nb;
+        tile_coords(tile, NT, s_mt, G, grp, mt, nb);
+        has2 = s_off[grp] + (mt * 2 + 1) * C::BM < s_off[grp + 1];
+      }
       if (!mbar_wait(TEMPTY_BAR(acc), aph ^ 1u, g.limit_ns, s_abort)) {
         ok = false;
         break;
@@ -345,11 +362,15 @@ __global__ void __launch_bounds__(192, 1)
           break;
         }
         tc_fence_after();
-        const uint64_t ad = smem_desc_kmajor<BK>(sA + stage * C::A_BYTES);
+        const uint64_t ad = smem_desc_kmajor<BK>(sA + stage * MP * C::A_BYTES);
         const uint64_t bd = smem_desc_kmajor<BK>(sB + stage * C::B_BYTES);
 #pragma unroll
-        for (int kk = 0; kk < C::BK / 16; ++kk)
+        for (int kk = 0; kk < C::BK / 16; ++kk) {
           tc_mma_f16(dt, ad + 2u * kk, bd + 2u * kk, IDESC, (kb | kk) != 0 ? 1u : 0u);
+          if (MP == 2 && has2)
+            tc_mma_f16(tmem_base + BN, ad + static_cast<uint64_t>(C::A_BYTES >> 4) + 2u * kk, bd + 2u * kk, IDESC,
+                       (kb | kk) != 0 ? 1u : 0u);
+        }
         tc_commit(EMPTY_BAR(stage));
         issued = true;
         if (++stage == STAGES) {
@@ -371,25 +392,30 @@ __global__ void __launch_bounds__(192, 1)
     }
   } else if (warp >= 2) {
     // ------------------------------------------------ epilogue
-    const int q = warp & 3;  // TMEM lanes [32q, 32q + 32) belong to this warp
+    const int q = warp & 3;            // TMEM lanes [32q, 32q + 32) belong to this warp
+    const int wp = (warp - 2) >> 2;    // which of the quarter's warps (0 .. EW/4 - 1)
+    constexpr int WPQ = EW / 4;        // warps per quarter: column chunks are dealt round robin
     int it = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
-      const int acc = it & 1;
-      const uint32_t aph = (it >> 1) & 1;
+      const int acc = it % C::NBUF;
+      const uint32_t aph = (it / C::NBUF) & 1;
       int grp, mt, nb;
       tile_coords(tile, NT, s_mt, G, grp, mt, nb);
-      const int row0 = s_off[grp] + mt * C::BM;
       const int row_end = s_off[grp + 1];
       if (!mbar_wait(TFULL_BAR(acc), aph, g.limit_ns, s_abort)) {
         ok = false;
         break;
       }
       tc_fence_after();
+#pragma unroll 1
+      for (int sub = 0; sub < MP; ++sub) {
+      const int row0 = s_off[grp] + (mt * MP + sub) * C::BM;
+      if (sub > 0 && row0 >= row_end) break;  // no second M-tile in this unit
       const int grow = row0 + q * 32 + lane;
       const bool valid = grow < row_end;
       const uint32_t tb =
-          tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
+          tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>((acc + sub) * BN);
       if constexpr (EPI == EPI_SWIGLU) {
         // columns hold blocks of GU gate then GU up columns of the same
         // features: features nb*BN/2 + half*GU + c
@@ -397,7 +423,7 @@ __global__ void __launch_bounds__(192, 1)
         static_assert(BN % (2 * GU) == 0, "N tile must hold whole gate/up blocks");
         __nv_bfloat16* out = static_cast<__nv_bfloat16*>(g.out);
 #pragma unroll 1
-        for (int cc = 0; cc < BN / 2; cc += 32) {
+        for (int cc = 32 * wp; cc < BN / 2; cc += 32 * WPQ) {
           const int half = cc / GU, c = cc % GU;
           uint32_t gr[32], ur[32];
           tmem_ld32(tb + half * 2 * GU + c, gr);
@@ -421,7 +447,7 @@ __global__ void __launch_bounds__(192, 1)
       } else if constexpr (EPI == EPI_BF16) {
         __nv_bfloat16* out = static_cast<__nv_bfloat16*>(g.out);
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
+        for (int c = 32 * wp; c < BN; c += 32 * WPQ) {
           uint32_t r[32];
           tmem_ld32(tb + c, r);
           tc_wait_ld();
@@ -443,6 +469,7 @@ __global__ void __launch_bounds__(192, 1)
         const float bv = (valid && g.bias) ? g.bias[grow] : 0.f;
         const int n0 = nb * BN;
         if constexpr (BN == 16) {
+          if (wp == 0) {
           uint32_t r[16];
           tmem_ld16(tb, r);
           tc_wait_ld();
@@ -451,9 +478,10 @@ __global__ void __launch_bounds__(192, 1)
             for (int c = 0; c < 16; ++c)
               if (n0 + c < g.n_valid) out[static_cast<int64_t>(n0 + c) * g.out_ld + grow] = __uint_as_float(r[c]) + bv;
           }
+          }
         } else {
 #pragma unroll 1
-          for (int c0 = 0; c0 < BN; c0 += 32) {
+          for (int c0 = 32 * wp; c0 < BN; c0 += 32 * WPQ) {
             uint32_t r[32];
             tmem_ld32(tb + c0, r);
             tc_wait_ld();
@@ -468,7 +496,7 @@ __global__ void __launch_bounds__(192, 1)
       } else {
         float* out = static_cast<float*>(g.out);
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
+        for (int c = 32 * wp; c < BN; c += 32 * WPQ) {
           uint32_t r[32];
           tmem_ld32(tb + c, r);
           tc_wait_ld();
@@ -488,6 +516,7 @@ __global__ void __launch_bounds__(192, 1)
           }
         }
       }
+      }  // sub
       tc_fence_before();
       mbar_arrive(TEMPTY_BAR(acc));
     }
@@ -512,12 +541,12 @@ __global__ void __launch_bounds__(192, 1)
 
 // A: [rows, kdim], or with GATHER_A the source tensor [a_tensor_rows, kdim]
 // whose row a_rows[r] is A row r.
-template <int BN, int EPI, int STAGES, int BK, bool GATHER_A = false>
+template <int BN, int EPI, int STAGES, int BK, bool GATHER_A = false, int MP = 1>
 static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b_rows,
                      const int32_t* offsets, int ngroups, int n_per_group, void* out,
                      int64_t out_ld, const float* bias, int32_t* status, cudaStream_t s, int n_valid = 0,
                      const int32_t* a_rows = nullptr, int64_t a_tensor_rows = 0) {
-  using C = TcCfg<BN, STAGES, BK>;
+  using C = TcCfg<BN, STAGES, BK, MP>;
   CUtensorMap ta, tb;
   if (GATHER_A)
     DM_RET(make_tmap_bf16(&ta, A, static_cast<uint64_t>(kdim), static_cast<uint64_t>(a_tensor_rows), 1, BK));
@@ -537,7 +566,7 @@ static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b
   g.limit_ns = static_cast<uint64_t>(wait_limit_ns());
   g.n_valid = n_valid;
   g.a_rows = a_rows;
-  auto kern = k_gemm_tc<BN, EPI, STAGES, BK, GATHER_A>;
+  auto kern = k_gemm_tc<BN, EPI, STAGES, BK, GATHER_A, MP>;
   static_assert(C::SMEM <= 232448, "shared memory budget");
   DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(C::SMEM)));
@@ -549,7 +578,7 @@ static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b
   const int64_t cap = sm_count();
 #endif
   const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(cap, ub_tiles)));
-  kern<<<grid, 192, C::SMEM, s>>>(ta, tb, g);
+  kern<<<grid, 64 + 32 * 8, C::SMEM, s>>>(ta, tb, g);
   DM_LAUNCH_CHECK("k_gemm_tc");
   return DECOMOE_OK;
 }
@@ -1287,11 +1316,18 @@ static bool use_decode_path(int64_t rows) { return rows <= DECOMOE_DECODE_ROWS; 
 #ifndef DECOMOE_DN_BK
 #define DECOMOE_DN_BK 64
 #endif
+#ifndef DECOMOE_GU_MP
+#define DECOMOE_GU_MP 1
+#endif
+#ifndef DECOMOE_DN_MP
+#define DECOMOE_DN_MP 1
+#endif
 #ifndef DECOMOE_DN_STAGES
 #define DECOMOE_DN_STAGES 4
 #endif
 constexpr int GU_BK = DECOMOE_GU_BK, GU_STAGES = DECOMOE_GU_STAGES;
 constexpr int DN_BK = DECOMOE_DN_BK, DN_STAGES = DECOMOE_DN_STAGES;
+constexpr int GU_MP = DECOMOE_GU_MP, DN_MP = DECOMOE_DN_MP;
 
 int decomoe_expert_gate_up(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m,
                            int dtype, const void* w_gate_up, void* h, int32_t* status_dev,
@@ -1323,8 +1359,8 @@ int decomoe_expert_gate_up(const void* x_perm, const int32_t* offsets, int64_t r
   if (static_cast<int64_t>(R) <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K)
     return launch_ws<true, 4>(x_perm, R, d, w_gate_up, 2 * m, offsets, K, h, m, status_dev, s);
   // A = x_perm [R, d], B = w_gate_up [K*2m, d] (only experts < K are read)
-  return launch_tc<256, EPI_SWIGLU, GU_STAGES, GU_BK>(x_perm, R, d, w_gate_up, static_cast<int64_t>(K) * 2 * m,
-                                                     offsets, K, 2 * m, h, m, nullptr, status_dev, s);
+  return launch_tc<256, EPI_SWIGLU, GU_STAGES, GU_BK, false, GU_MP>(
+      x_perm, R, d, w_gate_up, static_cast<int64_t>(K) * 2 * m, offsets, K, 2 * m, h, m, nullptr, status_dev, s);
 }
 
 int decomoe_expert_down(const void* h, const int32_t* offsets, int64_t rows, int K, int d, int m, int dtype,
@@ -1355,8 +1391,8 @@ int decomoe_expert_down(const void* h, const int32_t* offsets, int64_t rows, int
   if (static_cast<int64_t>(R) <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K)
     return launch_ws<false, 4>(h, R, m, w_down, d, offsets, K, y_perm, d, status_dev, s);
   // A = h [R, m], B = w_down [K*d, m]
-  return launch_tc<256, EPI_BF16, DN_STAGES, DN_BK>(h, R, m, w_down, static_cast<int64_t>(K) * d, offsets, K, d,
-                                                   y_perm, d, nullptr, status_dev, s);
+  return launch_tc<256, EPI_BF16, DN_STAGES, DN_BK, false, DN_MP>(h, R, m, w_down, static_cast<int64_t>(K) * d, offsets,
+                                                                  K, d, y_perm, d, nullptr, status_dev, s);
 }
 
 int decomoe_expert_gate_up_gather(const void* x, int64_t T, const int32_t* perm_token, const int32_t* offsets,
