@@ -435,6 +435,8 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
     ms, _ = timed(ad_step, n, 5, ws)
     out.append({"mode": f"mass p={args.p}", "K_mean": round(statistics.mean(Ks[-n:]), 2),
                 "tokens_per_s": round(T * n / (ms / 1e3), 1), "ms_per_step": round(ms / n, 4)})
+    out += run_large(dm, ws, pk, n)
+    out += run_stack(dm, ws, pk)
     # decode-size layers, K=64: weight streaming, reported against HBM
     for Td in W.DECODE_T:
         Bd = Buffers(wl, Td, B.out.device, dm)
@@ -464,6 +466,83 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
                     "ffn_hbm_frac": round(wbytes / (ffn * 1e-3) / 1e9 / pk["hbm_gbs"], 4)})
         del Bd, xs, graphs
     return out
+
+
+def run_large(dm, ws, pk, n):
+    """T=16384 prefill (14336 visual + 2048 text rows): one layer at each
+    prefix fraction and Zipf skew, plus the visual-block removal from the
+    layer output and from 48 layers of K and V caches, as one graph replay."""
+    out = []
+    dev = torch.device("cuda")
+    base = W.LARGE
+    kv = [W.make_kv(base, device=dev, seed=s) for s in (0, 1)]
+    kv_out = [torch.empty(base.layers, base.T - base.nv, base.kv_width, dtype=torch.bfloat16, device=dev)
+              for _ in range(2)]
+    for zipf in W.LARGE_ZIPF:
+        wl = W.with_(base, zipf_s=zipf)
+        g = W.make_layer(wl, device=dev)
+        w_gu = dm.fuse_gate_up(g["w_gate"], g["w_up"])
+        del g["w_gate"], g["w_up"]
+        lws = dm.workspace(dm.decomoe_moe_layer_workspace_bytes(wl.T, wl.d, wl.E, wl.k, wl.m, dm.DECOMOE_BF16), dev)
+        o = torch.empty_like(g["x"])
+        text = torch.empty(wl.T - wl.nv, wl.d, dtype=torch.bfloat16, device=dev)
+        for f in W.LARGE_FRACTIONS:
+            K = W.large_K(f)
+
+            def step(K=K):
+                dm.decomoe_moe_layer(g["x"], g["w_r"], g["bias"], w_gu, g["w_down"], wl.k, o, lws, K_fixed=K,
+                                     p=0.7)
+                dm.decomoe_drop_visual_block(o, text, wl.v0, wl.nv)
+                for src, dst in zip(kv, kv_out):
+                    dm.decomoe_drop_visual_block(src, dst, wl.v0, wl.nv)
+
+            gr = dm.capture_graph(step)
+            nn = max(5, min(n, 50))
+            ms, _ = timed(lambda i, ev: gr.replay(), nn, 3, ws)
+            ms_step = ms / nn
+            fl = 6.0 * wl.T * wl.k * wl.d * wl.m + 2.0 * wl.T * wl.d * wl.E
+            out.append({"mode": "large T=16384", "zipf_s": zipf, "K": K, "fraction": f,
+                        "ms_per_step": round(ms_step, 4), "tokens_per_s": round(wl.T / (ms_step * 1e-3), 1),
+                        "step_tflops": round(fl / (ms_step * 1e-3) / 1e12, 2),
+                        "includes": "layer + hidden and 2x48-layer KV compaction (1.61 GB in)"})
+            del gr
+        del g, w_gu, lws
+    del kv, kv_out
+    torch.cuda.empty_cache()
+    return out
+
+
+def run_stack(dm, ws, pk):
+    """48-layer attention-free stack, 16 system + 1280 visual + 256 text rows:
+    layers 0..19 at K=128 on 1552 rows, visual block removed from hidden and
+    both 48-layer KV caches at layer 20, layers 20..47 on 272 rows with K_l
+    drawn from 32..96. One pass = one graph replay."""
+    from paper_2609_38823_gb300.stack import Stack, StackLayer
+
+    wl = W.STACK
+    dev = torch.device("cuda")
+    layers = []
+    for l in range(wl.layers):
+        g = W.make_layer(wl, layer=l, device=dev, with_x=False)
+        layers.append(StackLayer(g["w_r"], g["bias"], dm.fuse_gate_up(g["w_gate"], g["w_up"]), g["w_down"]))
+        del g
+    K_sched = W.stack_K_schedule(wl)
+    st = Stack(layers, K_sched, wl.k, wl.exit_layer, wl.v0, wl.nv, wl.T)
+    h0 = W.make_x(wl, device=dev)
+    kv = [W.make_kv(wl, device=dev, seed=s) for s in (0, 1)]
+    kv_out = [torch.empty(wl.layers, wl.T - wl.nv, wl.kv_width, dtype=torch.bfloat16, device=dev) for _ in range(2)]
+    gr = dm.capture_graph(lambda: st.forward(h0, kv, kv_out))
+    nn = 10
+    ms, _ = timed(lambda i, ev: gr.replay(), nn, 3, ws)
+    ms_pass = ms / nn
+    Tt = wl.T - wl.nv
+    fl = sum(6.0 * (wl.T if l < wl.exit_layer else Tt) * wl.k * wl.d * wl.m for l in range(wl.layers))
+    res = [{"mode": "stack48", "pass_ms": round(ms_pass, 3), "tokens_per_s": round(wl.T / (ms_pass * 1e-3), 1),
+            "useful_tflops": round(fl / (ms_pass * 1e-3) / 1e12, 2), "exit_layer": wl.exit_layer,
+            "K_after_exit_mean": round(statistics.mean(K_sched[wl.exit_layer:]), 2)}]
+    del gr, st, layers, kv, kv_out
+    torch.cuda.empty_cache()
+    return res
 
 
 def _kernel_hash():

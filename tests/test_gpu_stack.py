@@ -1,0 +1,153 @@
+"""The attention-free layer stack (RMSNorm -> prefix MoE + residual, visual
+block removed from the hidden state and the KV caches at the exit layer) and
+the T=16384 prefill layer, against the oracle.
+
+Tokens are independent once every layer's prefix K_l is fixed (no attention),
+so the oracle follows sampled tokens through the layers one by one
+(stack_token). Tokens whose routing margin at some layer is too small for the
+two sides' rounding are counted and left out of the output comparison.
+"""
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_38823_gb300 as dm
+import workloads as W
+from oracle import decomoe_oracle as O
+from paper_2609_38823_gb300.stack import Stack, StackLayer
+from tests.helpers import assert_close_out, bf16_round, f64
+
+pytestmark = pytest.mark.gpu
+DEV = torch.device("cuda")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    import __graft_entry__
+
+    __graft_entry__.build()
+    dm.lib()
+
+
+class ExpertView:
+    def __init__(self, t):
+        self.t = t
+
+    def __getitem__(self, e):
+        return self.t[e].double().cpu().numpy()
+
+
+def _layers(wl, n, device, first=0):
+    out_dev, out_ref = [], []
+    for l in range(first, first + n):
+        g = W.make_layer(wl, layer=l, device=device, with_x=False)
+        w_gu = dm.fuse_gate_up(g["w_gate"].to(DEV), g["w_up"].to(DEV))
+        out_dev.append(StackLayer(g["w_r"].to(DEV), g["bias"].to(DEV), w_gu, g["w_down"].to(DEV)))
+        out_ref.append(dict(w_r=f64(g["w_r"]).astype(np.float32) if wl.dtype == "f32" else f64(g["w_r"]),
+                            bias=g["bias"].cpu().numpy(), w_gate=ExpertView(g["w_gate"]),
+                            w_up=ExpertView(g["w_up"]), w_down=ExpertView(g["w_down"])))
+    return out_dev, out_ref
+
+
+def _trajectories(h0, ref_layers, K_sched, k, rows, round_fn):
+    outs, margins = [], []
+    for t in rows:
+        h, mg = O.stack_token(h0[t], ref_layers, K_sched, k, round_bf16=round_fn)
+        outs.append(h)
+        margins.append(min(mg))
+    return np.stack(outs), np.array(margins)
+
+
+def test_small_fp32_stack_with_exit():
+    wl = W.with_(W.TINY, layers=6, exit_layer=3)
+    L, R = _layers(wl, 6, "cpu")
+    K_sched = [16, 16, 16, 10, 6, 12]
+    h0 = W.make_x(wl)
+    st = Stack(L, K_sched, wl.k, exit_layer=3, v0=wl.v0, nv=wl.nv, T=wl.T)
+    kv = [torch.randn(6, wl.T, 64, generator=torch.Generator().manual_seed(s)).to(DEV) for s in (1, 2)]
+    kv_out = [torch.empty(6, wl.T - wl.nv, 64, device=DEV) for _ in range(2)]
+    out = st.forward(h0.to(DEV), kv, kv_out)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(st.status) == 0
+    text = [t for t in range(wl.T) if not (wl.v0 <= t < wl.v0 + wl.nv)]
+    assert out.shape == (len(text), wl.d)
+    ref, margins = _trajectories(f64(h0), R, K_sched, wl.k, text, None)
+    keep = margins > 1e-4
+    assert keep.mean() > 0.8
+    assert_close_out(f64(out)[keep], ref[keep], 1e-4, 1e-4, "fp32 stack output")
+    for src, dst in zip(kv, kv_out):
+        ref_kv = np.stack([O.drop_visual_block(src[l].cpu().numpy(), wl.v0, wl.nv) for l in range(6)])
+        assert np.array_equal(dst.cpu().numpy(), ref_kv)
+
+
+@pytest.fixture(scope="module")
+def stack48():
+    wl = W.STACK
+    L, R = _layers(wl, wl.layers, "cuda")
+    return wl, L, R
+
+
+def test_stack48_exit_layer_compaction_and_window_parity(stack48):
+    """Full 48-layer stack at its real size: finite text-only output, KV
+    compaction bit-exact, and sampled tokens followed by the oracle through a
+    three-layer window around the exit layer (19, 20, 21), where the bf16
+    drift of the hidden state stays within the output tolerance."""
+    wl, L, R = stack48
+    K_sched = W.stack_K_schedule(wl)
+    assert K_sched[:20] == [128] * 20 and all(32 <= v <= 96 for v in K_sched[20:])
+    h0 = W.make_x(wl, device="cuda")
+    kv = [W.make_kv(wl, device="cuda", seed=s) for s in (0, 1)]
+    kv_out = [torch.empty(wl.layers, wl.T - wl.nv, wl.kv_width, dtype=torch.bfloat16, device=DEV) for _ in range(2)]
+    st = Stack(L, K_sched, wl.k, exit_layer=wl.exit_layer, v0=wl.v0, nv=wl.nv, T=wl.T)
+    out = st.forward(h0, kv, kv_out)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(st.status) == 0
+    assert out.shape == (wl.T - wl.nv, wl.d) and torch.isfinite(out.float()).all()
+    for src, dst in zip(kv, kv_out):
+        for l in (0, 19, 20, 47):
+            ref = O.drop_visual_block(src[l].view(torch.int16).cpu().numpy(), wl.v0, wl.nv)
+            assert np.array_equal(dst[l].view(torch.int16).cpu().numpy(), ref)
+    # window around the exit: layers 19 (full sequence), 20 and 21 (text only)
+    win = Stack(L[19:22], K_sched[19:22], wl.k, exit_layer=1, v0=wl.v0, nv=wl.nv, T=wl.T)
+    hw = win.forward(h0)
+    torch.cuda.synchronize()
+    text = [t for t in range(wl.T) if not (wl.v0 <= t < wl.v0 + wl.nv)]
+    r = np.random.default_rng(7)
+    pick = np.sort(r.choice(len(text), 12, replace=False))
+    rows = [text[i] for i in pick]
+    ref, margins = _trajectories(f64(h0), R[19:22], K_sched[19:22], wl.k, rows, bf16_round)
+    keep = margins > 2e-2
+    assert keep.sum() >= 3, f"only {keep.sum()} sampled tokens clear of near-ties"
+    assert_close_out(f64(hw)[pick][keep], ref[keep], 5e-3, 2e-2, "stack window output")
+
+
+@pytest.mark.parametrize("K,zipf", [(39, 1.2), (128, 0.8)])
+def test_large_T16384_layer_sampled_and_compaction(K, zipf):
+    wl = W.with_(W.LARGE, zipf_s=zipf)
+    g = W.make_layer(wl, device="cuda")
+    w_gu = dm.fuse_gate_up(g["w_gate"], g["w_up"])
+    out = torch.empty_like(g["x"])
+    ws = dm.workspace(dm.decomoe_moe_layer_workspace_bytes(wl.T, wl.d, wl.E, wl.k, wl.m, dm.DECOMOE_BF16), DEV)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    dm.decomoe_moe_layer(g["x"], g["w_r"], g["bias"], w_gu, g["w_down"], wl.k, out, ws, K_fixed=K, p=0.7, status=st)
+    text = torch.empty(wl.T - wl.nv, wl.d, dtype=torch.bfloat16, device=DEV)
+    dm.decomoe_drop_visual_block(out, text, wl.v0, wl.nv)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(st) == 0
+    # compaction of the layer output: bit-exact against the oracle
+    ref_text = O.drop_visual_block(out.view(torch.int16).cpu().numpy(), wl.v0, wl.nv)
+    assert np.array_equal(text.view(torch.int16).cpu().numpy(), ref_text)
+    # sampled tokens through the layer
+    r = np.random.default_rng(K)
+    sample = np.sort(r.choice(wl.T, 24, replace=False))
+    x64 = f64(g["x"][torch.from_numpy(sample).to(DEV)])
+    wr64 = f64(g["w_r"])
+    b64 = g["bias"].cpu().numpy().astype(np.float64)
+    from tests.helpers import logit_error_bound
+    bound = logit_error_bound(x64, wr64, b64)
+    a = O.router_logits(x64, wr64, b64).astype(np.float64)
+    keep = O.prefix_margin(a, K, wl.k) > 2 * bound.max()
+    ref = O.moe_layer(x64, wr64, b64, ExpertView(g["w_gate"]), ExpertView(g["w_up"]), ExpertView(g["w_down"]),
+                      k=wl.k, K=K)
+    assert_close_out(f64(out[torch.from_numpy(sample).to(DEV)])[keep], ref["out"][keep], 5e-3, 2e-2,
+                     "T=16384 layer output")
