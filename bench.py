@@ -433,8 +433,17 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
         dm.decomoe_drop_visual_block(B.out, text, wl.v0, wl.nv)
 
     ms, _ = timed(ad_step, n, 5, ws)
-    out.append({"mode": f"mass p={args.p}", "K_mean": round(statistics.mean(Ks[-n:]), 2),
+    out.append({"mode": f"mass p={args.p}, host-selected K (one sync per step)", "K_mean": round(statistics.mean(Ks[-n:]), 2),
                 "tokens_per_s": round(T * n / (ms / 1e3), 1), "ms_per_step": round(ms / n, 4)})
+    # the same with the prefix selected on the device: no sync, CUDA-graph replay
+    graphs = [dm.capture_graph(lambda L=L: (dm.decomoe_moe_layer(L.x, L.w_r, L.bias, L.w_gu, L.w_down, wl.k, B.out,
+                                                                  lws, K_fixed=-1, p=args.p, status=B.status),
+                                             dm.decomoe_drop_visual_block(B.out, text, wl.v0, wl.nv)))
+              for L in layers]
+    ms, _ = timed(lambda i, ev: graphs[i % len(graphs)].replay(), n, 5, ws)
+    out.append({"mode": f"mass p={args.p}, device-selected K (graph replay)",
+                "tokens_per_s": round(T * n / (ms / 1e3), 1), "ms_per_step": round(ms / n, 4)})
+    del graphs
     out += run_large(dm, ws, pk, n)
     out += run_stack(dm, ws, pk)
     # decode-size layers, K=64: weight streaming, reported against HBM

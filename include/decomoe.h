@@ -124,6 +124,20 @@ DECOMOE_API int decomoe_route_prefix(const float* logits, int64_t T, int E, int6
 DECOMOE_API int decomoe_select_prefix(const double* mass_host, int E, int k, double p, int* K_out_host);
 
 /* ------------------------------------------------------------------------
+ * Prefix selection on the device (Eq. 12 as decomoe_select_prefix, same
+ * sequential fp64 arithmetic, so the same K bit for bit): reads mass [E]
+ * (e.g. the mass_out of decomoe_route_prefix) and writes K to K_dev (one
+ * int32 on the device). With decomoe_route_prefix_dk, which routes over the
+ * prefix [0, *K_dev), the mass-selected RCEP layer needs no host
+ * synchronisation: dispatch and the expert GEMMs then take K = E (experts at
+ * or beyond *K_dev receive no rows and cost nothing).
+ * ------------------------------------------------------------------------ */
+DECOMOE_API int decomoe_select_prefix_device(const double* mass, int E, int k, double p, int32_t* K_dev,
+                                             decomoe_stream_t stream);
+DECOMOE_API int decomoe_route_prefix_dk(const float* logits, int64_t T, int E, int64_t ld, const int32_t* K_dev,
+                                        int k, int32_t* topk_idx, float* topk_w, decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * a5. Dispatch: group the T*k (token, slot) pairs by expert (Algorithm 2,
  * "evaluate ... only the first K expert MLPs").
  *   counts[e] = #pairs with topk_idx == e (e < K); offsets = exclusive scan,
@@ -272,10 +286,15 @@ DECOMOE_API int decomoe_rmsnorm(const void* x, void* y, int64_t T, int d, float 
  *   router logits -> [mass pass -> select prefix] -> prefix routing ->
  *   dispatch -> grouped SwiGLU -> combine (+ residual).
  * K_fixed > 0 routes over the fixed prefix [0, K_fixed) (the paper's fixed
- * keep-ratio experiments) and still runs the mass pass when p > 0 (K_sel_host
- * then receives the prefix Eq. 12 selects); K_fixed == 0 selects K from p
- * (0 < p <= 1), which synchronises the stream once to read the mass. p == 0
- * with K_fixed > 0 skips the mass pass. K_used_host / K_sel_host may be NULL.
+ * keep-ratio experiments); with p > 0 the same routing launch also leaves the
+ * full-pool activated mass in the workspace (no host sync). K_fixed == 0
+ * selects K from p (0 < p <= 1) on the host: the stream is synchronised once
+ * to read the mass and K_used_host / K_sel_host receive K. K_fixed == -1
+ * selects K from p on the device (decomoe_select_prefix_device): no host
+ * synchronisation, capturable in a CUDA graph; K is left as an int32 in the
+ * workspace (entry 11 of decomoe_moe_layer_workspace_layout) and the host
+ * outputs are set to -1. p == 0 with K_fixed > 0 skips the mass pass.
+ * K_used_host / K_sel_host may be NULL.
  * x, residual, out: [T, d] dtype (out may alias residual, not x).
  * ws: decomoe_moe_layer_workspace_bytes(...) bytes; every intermediate
  * (logits, routes, dispatch arrays, x_perm, h, y_perm) lives there.
@@ -289,7 +308,7 @@ DECOMOE_API int decomoe_moe_layer(const void* x, const void* w_r, const float* b
 
 /* Offsets (bytes) of the intermediates inside the decomoe_moe_layer workspace,
  * for inspection: logits, topk_idx, topk_w, mass, counts, offsets, perm_token,
- * inv_slot, x_perm, h, y_perm (11 entries written to offs_host). */
+ * inv_slot, x_perm, h, y_perm, device K (12 entries written to offs_host). */
 DECOMOE_API int decomoe_moe_layer_workspace_layout(int64_t T, int d, int E, int k, int m, int dtype,
                                        size_t* offs_host);
 

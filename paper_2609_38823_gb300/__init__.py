@@ -47,6 +47,8 @@ SIGNATURES = {
     "decomoe_route_workspace_bytes": (_S, [_L, _I]),
     "decomoe_route_prefix": (_I, [_P, _L, _I, _L, _I, _I, _P, _P, _P, _P, _S, _P]),
     "decomoe_select_prefix": (_I, [_P, _I, _I, _D, _P]),
+    "decomoe_select_prefix_device": (_I, [_P, _I, _I, _D, _P, _P]),
+    "decomoe_route_prefix_dk": (_I, [_P, _L, _I, _L, _P, _I, _P, _P, _P]),
     "decomoe_dispatch_workspace_bytes": (_S, [_L, _I, _I]),
     "decomoe_dispatch": (_I, [_P, _L, _I, _I, _P, _I, _I, _P, _P, _P, _P, _P, _P, _S, _P, _P]),
     "decomoe_dispatch_noalloc": (_I, [_P, _L, _I, _I, _P, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
@@ -162,7 +164,7 @@ def decomoe_moe_layer_workspace_bytes(T, d, E, k, m, dtype) -> int:
 
 
 def decomoe_moe_layer_workspace_layout(T, d, E, k, m, dtype):
-    offs = (ctypes.c_size_t * 11)()
+    offs = (ctypes.c_size_t * 12)()
     _check("decomoe_moe_layer_workspace_layout",
            lib().decomoe_moe_layer_workspace_layout(T, d, E, k, m, dtype, offs))
     return list(offs)
@@ -198,6 +200,20 @@ def decomoe_route_prefix(logits, K, k, topk_idx=None, topk_w=None, mass_out=None
     _check("decomoe_route_prefix",
            lib().decomoe_route_prefix(_ptr(logits), T, E, ld, K, k, _ptr(topk_idx), _ptr(topk_w),
                                       _ptr(mass_out), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def decomoe_select_prefix_device(mass, k, p, K_dev, stream=None):
+    _need_cuda(mass, K_dev)
+    _check("decomoe_select_prefix_device",
+           lib().decomoe_select_prefix_device(_ptr(mass), mass.shape[0], k, float(p), _ptr(K_dev), _stream(stream)))
+
+
+def decomoe_route_prefix_dk(logits, K_dev, k, topk_idx, topk_w, stream=None):
+    _need_cuda(logits, K_dev, topk_idx, topk_w)
+    T, E = logits.shape
+    _check("decomoe_route_prefix_dk",
+           lib().decomoe_route_prefix_dk(_ptr(logits), T, E, E, _ptr(K_dev), k, _ptr(topk_idx), _ptr(topk_w),
+                                         _stream(stream)))
 
 
 def decomoe_dispatch(topk_idx, K, x, counts, offsets, perm_token, inv_slot, x_perm, ws, status=None,

@@ -22,6 +22,7 @@ enum {
   WS_YPERM,
   WS_ROUTE,
   WS_DISPATCH,
+  WS_KDEV,
   WS_STATUS_PAD,
   WS_COUNT
 };
@@ -49,6 +50,7 @@ static LayerLayout layer_layout(int64_t T, int d, int E, int k, int m, int dtype
   sz[WS_YPERM] = R * d * eb;
   sz[WS_ROUTE] = decomoe_route_workspace_bytes(T, E);
   sz[WS_DISPATCH] = decomoe_dispatch_workspace_bytes(T, k, E);
+  sz[WS_KDEV] = 16;
   sz[WS_STATUS_PAD] = 256;
   size_t o = 0;
   for (int i = 0; i < WS_COUNT; ++i) {
@@ -76,6 +78,7 @@ int decomoe_moe_layer_workspace_layout(int64_t T, int d, int E, int k, int m, in
   DM_ARG_CHECK(T >= 0 && d > 0 && E > 0 && k > 0 && m > 0, "moe_layer_workspace_layout: bad sizes");
   const LayerLayout L = layer_layout(T, d, E, k, m, dtype);
   for (int i = 0; i <= WS_YPERM; ++i) offs_host[i] = L.off[i];
+  offs_host[11] = L.off[WS_KDEV];
   return DECOMOE_OK;
 }
 
@@ -87,7 +90,8 @@ int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const v
   DM_ARG_CHECK(T >= 0 && d > 0 && m > 0, "moe_layer: bad sizes");
   DM_ARG_CHECK(E >= 1 && E <= DECOMOE_MAX_E && k >= 1 && k <= DECOMOE_MAX_TOPK && k <= E,
                "moe_layer: need 1 <= k <= E <= %d, k <= %d", DECOMOE_MAX_E, DECOMOE_MAX_TOPK);
-  DM_ARG_CHECK(K_fixed == 0 || (K_fixed >= k && K_fixed <= E), "moe_layer: K_fixed=%d outside [k, E]", K_fixed);
+  DM_ARG_CHECK(K_fixed == 0 || K_fixed == -1 || (K_fixed >= k && K_fixed <= E),
+               "moe_layer: K_fixed=%d outside [k, E] (0: host-selected, -1: device-selected)", K_fixed);
   DM_ARG_CHECK(K_fixed > 0 || (p > 0.0 && p <= 1.0), "moe_layer: mass mode needs 0 < p <= 1");
   DM_ARG_CHECK(p >= 0.0 && p <= 1.0, "moe_layer: p outside [0, 1]");
   DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "moe_layer: bad dtype");
@@ -124,7 +128,19 @@ int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const v
   DM_RET(decomoe_router_logits(x, w_r, bias, T, d, E, dtype, logits, status_dev, stream));
   // a2 (+ a3) and a4: full-pool activated mass and prefix routing
   int K = K_fixed;
-  if (K_fixed > 0) {
+  int32_t* K_dev = reinterpret_cast<int32_t*>(base + L.off[WS_KDEV]);
+  if (K_fixed == -1) {
+    // device-selected prefix: mass pass, Eq. 12 on the device, routing over
+    // [0, *K_dev); dispatch and experts run over all E groups (those at or
+    // beyond *K_dev are empty)
+    DM_RET(decomoe_route_prefix(logits, T, E, E, E, k, nullptr, nullptr, mass, route_ws,
+                                decomoe_route_workspace_bytes(T, E), stream));
+    DM_RET(decomoe_select_prefix_device(mass, E, k, p, K_dev, stream));
+    DM_RET(decomoe_route_prefix_dk(logits, T, E, E, K_dev, k, topk_idx, topk_w, stream));
+    K = E;
+    if (K_sel_host) *K_sel_host = -1;
+    if (K_used_host) *K_used_host = -1;
+  } else if (K_fixed > 0) {
     // one launch: prefix routing over [0, K_fixed) and, when p > 0, the
     // full-pool mass of Eq. 11 (left in the workspace, no host sync)
     DM_RET(decomoe_route_prefix(logits, T, E, E, K, k, topk_idx, topk_w, p > 0.0 ? mass : nullptr, route_ws,
@@ -142,7 +158,7 @@ int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const v
     if (K_sel_host) *K_sel_host = Ksel;
     DM_RET(decomoe_route_prefix(logits, T, E, E, K, k, topk_idx, topk_w, nullptr, nullptr, 0, stream));
   }
-  if (K_used_host) *K_used_host = K;
+  if (K_used_host && K_fixed != -1) *K_used_host = K;
   // a5: dispatch (counts, offsets, permutation, x_perm rows)
   DM_RET(decomoe_dispatch(topk_idx, T, k, K, x, d, dtype, counts, offsets, perm, inv, x_perm, disp_ws,
                           decomoe_dispatch_workspace_bytes(T, k, K), status_dev, stream));

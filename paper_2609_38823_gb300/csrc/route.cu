@@ -99,7 +99,9 @@ __device__ __forceinline__ float pick_weight(float my_v, int lane, int k) {
 
 __global__ void __launch_bounds__(ROUTE_THREADS)
     k_route(const float* __restrict__ logits, int64_t Tn, int E, int64_t ld, int K, int k,
-            int32_t* __restrict__ idx_out, float* __restrict__ w_out, double* __restrict__ part) {
+            int32_t* __restrict__ idx_out, float* __restrict__ w_out, double* __restrict__ part,
+            const int32_t* __restrict__ K_dev) {
+  if (K_dev != nullptr) K = *K_dev;  // prefix chosen on the device (k <= K <= E by construction)
   __shared__ int s_idx[ROUTE_TPB][DECOMOE_MAX_TOPK];
   __shared__ float s_w[ROUTE_TPB][DECOMOE_MAX_TOPK];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -167,6 +169,31 @@ __global__ void __launch_bounds__(256)
   if (threadIdx.x == 0) mass[e] = red[0];
 }
 
+// Eq. 12 on the device, one thread: the same sequential fp64 sums, division
+// and comparison as decomoe_select_prefix, so the prefix is bit-identical to
+// the host selection on the same mass.
+__global__ void k_select_prefix(const double* __restrict__ mass, int E, int k, double p, int32_t* __restrict__ K_dev) {
+  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+  double tot = 0.0;
+  for (int e = 0; e < E; ++e) tot = __dadd_rn(tot, mass[e]);
+  int K = k;
+  if (tot > 0.0) {
+    int K_hat = E;
+    if (p < 1.0) {
+      double acc = 0.0;
+      for (int Kc = 1; Kc <= E; ++Kc) {
+        acc = __dadd_rn(acc, mass[Kc - 1]);
+        if (__ddiv_rn(acc, tot) >= p) {
+          K_hat = Kc;
+          break;
+        }
+      }
+    }
+    K = K_hat > k ? K_hat : k;
+  }
+  *K_dev = K;
+}
+
 }  // namespace decomoe
 
 using namespace decomoe;
@@ -232,12 +259,39 @@ int decomoe_route_prefix(const float* logits, int64_t T, int E, int64_t ld, int 
     part = static_cast<double*>(ws);
   }
   k_route<<<static_cast<unsigned>(nblocks), ROUTE_THREADS, 0, s>>>(logits, T, E, ld, K, k, topk_idx,
-                                                                   topk_w, part);
+                                                                   topk_w, part, nullptr);
   DM_LAUNCH_CHECK("k_route");
   if (mass_out != nullptr) {
     k_mass_finalize<<<E, 256, 0, s>>>(part, static_cast<int>(nblocks), E, mass_out);
     DM_LAUNCH_CHECK("k_mass_finalize");
   }
+  return DECOMOE_OK;
+}
+
+
+int decomoe_select_prefix_device(const double* mass, int E, int k, double p, int32_t* K_dev,
+                                 decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(mass && K_dev, "select_prefix_device: null pointer");
+  DM_ARG_CHECK(E >= 1 && k >= 1 && k <= E, "select_prefix_device: need 1 <= k <= E");
+  DM_ARG_CHECK(p > 0.0 && p <= 1.0, "select_prefix_device: p must lie in (0, 1]");
+  k_select_prefix<<<1, 32, 0, reinterpret_cast<cudaStream_t>(stream)>>>(mass, E, k, p, K_dev);
+  DM_LAUNCH_CHECK("k_select_prefix");
+  return DECOMOE_OK;
+}
+
+int decomoe_route_prefix_dk(const float* logits, int64_t T, int E, int64_t ld, const int32_t* K_dev, int k,
+                            int32_t* topk_idx, float* topk_w, decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(T >= 0 && E >= 1 && E <= DECOMOE_MAX_E && k >= 1 && k <= DECOMOE_MAX_TOPK && k <= E && ld >= E,
+               "route_prefix_dk: bad sizes");
+  if (T == 0) return DECOMOE_OK;
+  DM_ARG_CHECK(logits && K_dev, "route_prefix_dk: null pointer");
+  const int64_t nblocks = (T + ROUTE_TPB - 1) / ROUTE_TPB;
+  DM_ARG_CHECK(nblocks <= 0x7fffffff, "route_prefix_dk: T too large");
+  k_route<<<static_cast<unsigned>(nblocks), ROUTE_THREADS, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+      logits, T, E, ld, E, k, topk_idx, topk_w, nullptr, K_dev);
+  DM_LAUNCH_CHECK("k_route");
   return DECOMOE_OK;
 }
 

@@ -158,3 +158,64 @@ def test_layer_decode_bf16(prefill_layer, T):
     gc = dict(g_cpu, x=x.cpu())
     out, Ku, _, logits, idx, w, _ = _run_layer(gd, wl.k, T, K_fixed=64, p=0.7)
     _compare(gc, out, logits, idx, w, 64, wl.k, np.arange(T), (BF16_REL_L2, BF16_MAX_ABS))
+
+
+# ----------------------------------------------------------------- prefix selected on the device
+
+def test_select_prefix_device_matches_host_c():
+    r = np.random.default_rng(11)
+    for trial in range(60):
+        E = int(r.choice([8, 16, 128, 256]))
+        k = int(r.integers(1, min(E, 32) + 1))
+        s = (1.0 / (np.arange(E) + 1.0) ** r.uniform(0.0, 2.0)) * r.uniform(0.0, 2.0, E) * r.uniform(1, 3000)
+        if trial % 7 == 0:
+            s[r.integers(0, E, size=E // 2)] = 0.0
+        if trial % 11 == 0:
+            s[:] = 0.0
+        md = torch.from_numpy(s).to(DEV)
+        Kd = torch.zeros(1, dtype=torch.int32, device=DEV)
+        for p in (0.05, 0.3, 0.7, 0.9, 1.0):
+            dm.decomoe_select_prefix_device(md, k, p, Kd)
+            torch.cuda.synchronize()
+            assert int(Kd) == dm.decomoe_select_prefix(s, k, p) == O.select_prefix(s, p, k)
+
+
+@pytest.mark.parametrize("which", ["tiny", "prefill"])
+def test_layer_device_selected_prefix_equals_host_selected(which, prefill_layer):
+    if which == "tiny":
+        wl = W.TINY
+        g_cpu = W.make_layer(wl, device="cpu")
+        g = {n: t.to(DEV) for n, t in g_cpu.items()}
+    else:
+        wl, g, g_cpu = prefill_layer
+    p = 0.9 if which == "prefill" else 0.7
+    out_h, Ku, Ks, logits, idx, w, mass = _run_layer(g, wl.k, wl.T, K_fixed=0, p=p)
+    out_d, Kud, Ksd, logits_d, idx_d, w_d, mass_d = _run_layer(g, wl.k, wl.T, K_fixed=-1, p=p)
+    assert Kud == -1 and Ksd is None
+    assert torch.equal(out_h, out_d)
+    assert np.array_equal(idx, idx_d) and np.array_equal(w, w_d)
+    assert np.array_equal(mass, mass_d)
+
+
+def test_layer_device_selected_prefix_in_cuda_graph(prefill_layer):
+    wl, g, _ = prefill_layer
+    T, d, E, k, m = wl.T, wl.d, wl.E, wl.k, wl.m
+    w_gu = g.get("w_gu")
+    if w_gu is None:
+        w_gu = dm.fuse_gate_up(g["w_gate"], g["w_up"])
+        g["w_gu"] = w_gu
+    ws = dm.workspace(dm.decomoe_moe_layer_workspace_bytes(T, d, E, k, m, dm.DECOMOE_BF16), DEV)
+    out_e = torch.empty_like(g["x"])
+    dm.decomoe_moe_layer(g["x"], g["w_r"], g["bias"], w_gu, g["w_down"], k, out_e, ws, K_fixed=-1, p=0.8)
+    torch.cuda.synchronize()
+    out_g = torch.zeros_like(g["x"])
+    graph = dm.capture_graph(lambda: dm.decomoe_moe_layer(g["x"], g["w_r"], g["bias"], w_gu, g["w_down"], k, out_g,
+                                                          ws, K_fixed=-1, p=0.8))
+    out_g.zero_()
+    graph.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(out_e, out_g)
+    offs = dm.decomoe_moe_layer_workspace_layout(T, d, E, k, m, dm.DECOMOE_BF16)
+    Kdev = int(ws[offs[11]:offs[11] + 4].view(torch.int32))
+    mass = ws[offs[3]:offs[3] + E * 8].view(torch.float64).cpu().numpy()
+    assert Kdev == dm.decomoe_select_prefix(mass, k, 0.8)
