@@ -34,6 +34,7 @@ sys.path.insert(0, ROOT)
 import workloads as W  # noqa: E402
 
 LAUNCHES_PER_STEP = 10  # router 1, route+mass 2, dispatch 3, gate/up 1, down 1, combine 1, compaction 1
+# (plus two 4-byte memsets zeroing the expert GEMMs' tile counter)
 
 
 def parse():
@@ -195,6 +196,7 @@ class Buffers:
         self.y = torch.empty(R, d, dtype=torch.bfloat16, device=dev)
         self.out = torch.empty(T, d, dtype=torch.bfloat16, device=dev)
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
+        self.sched = torch.zeros(4, dtype=torch.int32, device=dev)  # dynamic tile counter of the expert GEMMs
 
 
 def run_step(dm, wl, L, B, K, v0, nv, text, ev=None):
@@ -206,10 +208,10 @@ def run_step(dm, wl, L, B, K, v0, nv, text, ev=None):
                         B.status)                                                     # a5
     if ev is not None:
         ev[0].record()
-    dm.decomoe_expert_gate_up(B.x_perm, B.offsets[:K + 1], K, L.w_gu, B.h, B.status)   # a6 gate/up + SwiGLU
+    dm.decomoe_expert_gate_up(B.x_perm, B.offsets[:K + 1], K, L.w_gu, B.h, B.status, B.sched)  # a6 gate/up
     if ev is not None:
         ev[1].record()
-    dm.decomoe_expert_down(B.h, B.offsets[:K + 1], K, L.w_down, B.y, B.status)         # a6 down
+    dm.decomoe_expert_down(B.h, B.offsets[:K + 1], K, L.w_down, B.y, B.status, B.sched)  # a6 down
     if ev is not None:
         ev[2].record()
     dm.decomoe_combine(B.y, B.inv, B.w, B.out)                                         # a7

@@ -206,20 +206,25 @@ DECOMOE_API int decomoe_weight_layout(const void* w_gate, const void* w_up, void
  * for rows <= 64 (decode); fp32 accumulate, h rounded to bf16. f32: CUDA-core
  * kernels with h kept in fp32. Needs d % 64 == 0 and m % 128 == 0 (bf16).
  * status_dev: optional device int32 collecting bounded-wait timeouts.
+ * sched_dev: optional device int32 (4 bytes, caller-owned). Given, the
+ * tensor-core kernels hand tiles out dynamically from this counter (the call
+ * zeroes it first) instead of a fixed round robin, which balances the mix of
+ * weight-streaming and weight-reusing tiles. Launches that may overlap on the
+ * GPU need distinct counters. NULL keeps the static order.
  * ------------------------------------------------------------------------ */
 DECOMOE_API int decomoe_expert_swiglu(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d,
                           int m, int dtype, const void* w_gate_up, const void* w_down, void* h_ws,
-                          void* y_perm, int32_t* status_dev, decomoe_stream_t stream);
+                          void* y_perm, int32_t* status_dev, int32_t* sched_dev, decomoe_stream_t stream);
 
 /* The two phases of decomoe_expert_swiglu as separate calls (same arguments
  * and rules): gate/up with the fused SwiGLU epilogue writes h [rows, m]; down
  * reads h and writes y_perm [rows, d]. */
 DECOMOE_API int decomoe_expert_gate_up(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d,
                                        int m, int dtype, const void* w_gate_up, void* h, int32_t* status_dev,
-                                       decomoe_stream_t stream);
+                                       int32_t* sched_dev, decomoe_stream_t stream);
 DECOMOE_API int decomoe_expert_down(const void* h, const int32_t* offsets, int64_t rows, int K, int d, int m,
                                     int dtype, const void* w_down, void* y_perm, int32_t* status_dev,
-                                    decomoe_stream_t stream);
+                                    int32_t* sched_dev, decomoe_stream_t stream);
 
 /* Gather forms: the expert rows are read straight from the token-ordered
  * hidden state, row r of the grouped order being x[perm_token[r], :] (TMA
@@ -232,11 +237,12 @@ DECOMOE_API int decomoe_expert_down(const void* h, const int32_t* offsets, int64
 DECOMOE_API int decomoe_expert_gate_up_gather(const void* x, int64_t T, const int32_t* perm_token,
                                               const int32_t* offsets, int64_t rows, int K, int d, int m,
                                               int dtype, const void* w_gate_up, void* h, int32_t* status_dev,
-                                              decomoe_stream_t stream);
+                                              int32_t* sched_dev, decomoe_stream_t stream);
 DECOMOE_API int decomoe_expert_swiglu_gather(const void* x, int64_t T, const int32_t* perm_token,
                                              const int32_t* offsets, int64_t rows, int K, int d, int m, int dtype,
                                              const void* w_gate_up, const void* w_down, void* h_ws,
-                                             void* y_perm, int32_t* status_dev, decomoe_stream_t stream);
+                                             void* y_perm, int32_t* status_dev, int32_t* sched_dev,
+                                             decomoe_stream_t stream);
 
 /* CUDA-core reference of decomoe_expert_swiglu for bf16 storage: the same
  * arithmetic (bf16 products, fp32 accumulation, h rounded to bf16) with one

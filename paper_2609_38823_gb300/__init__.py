@@ -53,11 +53,11 @@ SIGNATURES = {
     "decomoe_dispatch": (_I, [_P, _L, _I, _I, _P, _I, _I, _P, _P, _P, _P, _P, _P, _S, _P, _P]),
     "decomoe_dispatch_noalloc": (_I, [_P, _L, _I, _I, _P, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
     "decomoe_weight_layout": (_I, [_P, _P, _P, _I, _I, _I, _I, _P]),
-    "decomoe_expert_swiglu": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P]),
-    "decomoe_expert_gate_up": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P]),
-    "decomoe_expert_down": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P]),
-    "decomoe_expert_gate_up_gather": (_I, [_P, _L, _P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P]),
-    "decomoe_expert_swiglu_gather": (_I, [_P, _L, _P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P]),
+    "decomoe_expert_swiglu": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
+    "decomoe_expert_gate_up": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P]),
+    "decomoe_expert_down": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P]),
+    "decomoe_expert_gate_up_gather": (_I, [_P, _L, _P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P]),
+    "decomoe_expert_swiglu_gather": (_I, [_P, _L, _P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
     "decomoe_expert_swiglu_ref": (_I, [_P, _P, _L, _I, _I, _I, _P, _P, _P, _P, _P]),
     "decomoe_combine": (_I, [_P, _P, _P, _L, _I, _I, _I, _P, _P, _P]),
     "decomoe_drop_visual_block": (_I, [_P, _P, _L, _L, _L, _L, _L, _L, _L, _P]),
@@ -251,32 +251,33 @@ def decomoe_weight_layout(w_gate, w_up, w_gate_up, stream=None):
                                        _stream(stream)))
 
 
-def decomoe_expert_swiglu(x_perm, offsets, K, w_gate_up, w_down, h_ws, y_perm, status=None, stream=None):
-    _need_cuda(x_perm, offsets, w_gate_up, w_down, h_ws, y_perm, status)
+def decomoe_expert_swiglu(x_perm, offsets, K, w_gate_up, w_down, h_ws, y_perm, status=None, sched=None,
+                          stream=None):
+    _need_cuda(x_perm, offsets, w_gate_up, w_down, h_ws, y_perm, status, sched)
     rows, d = x_perm.shape
     m = w_down.shape[2]
     _check("decomoe_expert_swiglu",
            lib().decomoe_expert_swiglu(_ptr(x_perm), _ptr(offsets), rows, K, d, m, _dt(x_perm),
                                        _ptr(w_gate_up), _ptr(w_down), _ptr(h_ws), _ptr(y_perm),
-                                       _ptr(status), _stream(stream)))
+                                       _ptr(status), _ptr(sched), _stream(stream)))
 
 
-def decomoe_expert_gate_up(x_perm, offsets, K, w_gate_up, h, status=None, stream=None):
-    _need_cuda(x_perm, offsets, w_gate_up, h, status)
+def decomoe_expert_gate_up(x_perm, offsets, K, w_gate_up, h, status=None, sched=None, stream=None):
+    _need_cuda(x_perm, offsets, w_gate_up, h, status, sched)
     rows, d = x_perm.shape
     m = h.shape[1]
     _check("decomoe_expert_gate_up",
            lib().decomoe_expert_gate_up(_ptr(x_perm), _ptr(offsets), rows, K, d, m, _dt(x_perm), _ptr(w_gate_up),
-                                        _ptr(h), _ptr(status), _stream(stream)))
+                                        _ptr(h), _ptr(status), _ptr(sched), _stream(stream)))
 
 
-def decomoe_expert_down(h, offsets, K, w_down, y_perm, status=None, stream=None):
-    _need_cuda(h, offsets, w_down, y_perm, status)
+def decomoe_expert_down(h, offsets, K, w_down, y_perm, status=None, sched=None, stream=None):
+    _need_cuda(h, offsets, w_down, y_perm, status, sched)
     rows, m = h.shape
     d = y_perm.shape[1]
     _check("decomoe_expert_down",
            lib().decomoe_expert_down(_ptr(h), _ptr(offsets), rows, K, d, m, _dt(h), _ptr(w_down), _ptr(y_perm),
-                                     _ptr(status), _stream(stream)))
+                                     _ptr(status), _ptr(sched), _stream(stream)))
 
 
 def decomoe_expert_gate_up_gather(x, perm_token, offsets, K, w_gate_up, h, status=None, stream=None):
@@ -286,7 +287,7 @@ def decomoe_expert_gate_up_gather(x, perm_token, offsets, K, w_gate_up, h, statu
     m = h.shape[1]
     _check("decomoe_expert_gate_up_gather",
            lib().decomoe_expert_gate_up_gather(_ptr(x), T, _ptr(perm_token), _ptr(offsets), rows, K, d, m, _dt(x),
-                                               _ptr(w_gate_up), _ptr(h), _ptr(status), _stream(stream)))
+                                               _ptr(w_gate_up), _ptr(h), _ptr(status), None, _stream(stream)))
 
 
 def decomoe_expert_swiglu_gather(x, perm_token, offsets, K, w_gate_up, w_down, h_ws, y_perm, status=None,
@@ -298,7 +299,7 @@ def decomoe_expert_swiglu_gather(x, perm_token, offsets, K, w_gate_up, w_down, h
     _check("decomoe_expert_swiglu_gather",
            lib().decomoe_expert_swiglu_gather(_ptr(x), T, _ptr(perm_token), _ptr(offsets), rows, K, d, m, _dt(x),
                                               _ptr(w_gate_up), _ptr(w_down), _ptr(h_ws), _ptr(y_perm),
-                                              _ptr(status), _stream(stream)))
+                                              _ptr(status), None, _stream(stream)))
 
 
 def decomoe_expert_swiglu_ref(x_perm, offsets, K, w_gate_up, w_down, h_ws, y_perm, stream=None):

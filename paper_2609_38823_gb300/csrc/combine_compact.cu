@@ -48,10 +48,13 @@ __global__ void __launch_bounds__(256)
               const float* __restrict__ w, int64_t Tn, int k, int vec,
               const uint4* __restrict__ residual, uint4* __restrict__ out) {
   constexpr int NE = BF16 ? 8 : 4;
+  constexpr int WPT = 2;  // warps per token: each takes alternate 32-vector chunks
   const int lane = threadIdx.x & 31;
   const int64_t gw = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int64_t nw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
-  for (int64_t t = gw; t < Tn; t += nw) {
+  for (int64_t wt = gw; wt < Tn * WPT; wt += nw) {
+    const int64_t t = wt / WPT;
+    const int part = static_cast<int>(wt - t * WPT);
     int my_row = -1;
     float my_w = 0.f;
     if (lane < k) {
@@ -66,21 +69,30 @@ __global__ void __launch_bounds__(256)
         rows[j] = __shfl_sync(0xffffffffu, my_row, j);
         wts[j] = __shfl_sync(0xffffffffu, my_w, j);
       }
-      for (int c = lane; c < vec; c += 32) {
-        uint4 v[KT];
+      // two chunks (64 vectors apart) per iteration: 2*KT loads in flight
+      for (int c = part * 32 + lane; c < vec; c += 64 * WPT) {
+        const int c2 = c + 32 * WPT;
+        const bool two = c2 < vec;
+        uint4 v[KT], v2[KT];
 #pragma unroll
-        for (int j = 0; j < KT; ++j)
+        for (int j = 0; j < KT; ++j) {
           v[j] = rows[j] >= 0 ? __ldg(y + static_cast<int64_t>(rows[j]) * vec + c) : make_uint4(0, 0, 0, 0);
-        float acc[NE];
+          v2[j] = (rows[j] >= 0 && two) ? __ldg(y + static_cast<int64_t>(rows[j]) * vec + c2) : make_uint4(0, 0, 0, 0);
+        }
+        float acc[NE], acc2[NE];
 #pragma unroll
-        for (int i = 0; i < NE; ++i) acc[i] = 0.f;
+        for (int i = 0; i < NE; ++i) acc[i] = acc2[i] = 0.f;
 #pragma unroll
         for (int j = 0; j < KT; ++j)
-          if (rows[j] >= 0) acc_vec<BF16>(acc, v[j], wts[j]);
+          if (rows[j] >= 0) {
+            acc_vec<BF16>(acc, v[j], wts[j]);
+            acc_vec<BF16>(acc2, v2[j], wts[j]);
+          }
         out[t * vec + c] = finish_vec<BF16>(acc, residual, t * vec + c);
+        if (two) out[t * vec + c2] = finish_vec<BF16>(acc2, residual, t * vec + c2);
       }
     } else {
-      for (int c0 = 0; c0 < vec; c0 += 32) {
+      for (int c0 = part * 32; c0 < vec; c0 += 32 * WPT) {
         // every lane takes part in the shuffles; only lanes with c < vec load/store
         const int c = c0 + lane;
         const bool active = c < vec;
@@ -238,7 +250,7 @@ int decomoe_combine(const void* y_perm, const int32_t* inv_slot, const float* to
   DM_ARG_CHECK(out != y_perm, "combine: out aliases y_perm");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const int vec = static_cast<int>(row_bytes / 16);
-  const int grid = grid_for_warps(T);
+  const int grid = grid_for_warps(2 * T);  // two warps per token
   if (dtype == DECOMOE_BF16)
     launch_combine<true>(grid, s, static_cast<const uint4*>(y_perm), inv_slot, topk_w, T, k, vec,
                          static_cast<const uint4*>(residual), static_cast<uint4*>(out));

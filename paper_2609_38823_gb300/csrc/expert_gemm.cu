@@ -98,24 +98,29 @@ struct TcArgs {
   uint64_t limit_ns;
   int n_valid;  // EPI_F32_BIAS_T: number of valid output columns (tokens)
   const int32_t* a_rows;  // GATHER_A: A row r is row a_rows[r] of the A tensor (rows entries)
+  int* sched;             // dynamic scheduling: tile counter, zero at launch (null: static round robin)
 };
 
 // MP = M-tiles per work item. MP = 1: one 128-row A tile per B tile, two
 // accumulator buffers (epilogue overlaps the next tile's MMAs). MP = 2: two
 // M-tiles of the same group share each B tile (two M=128 MMAs per k-step,
 // 2/3 of the shared-memory traffic per MMA), one buffer of two accumulators.
-template <int BN, int STAGES, int BK_, int MP_ = 1>
+// OCC = resident CTAs per SM. OCC = 2 halves each CTA's shared memory and
+// TMEM (one accumulator, no double buffer): two tiles then share an SM, so
+// one CTA's weight streaming overlaps the other's tensor-core work.
+template <int BN, int STAGES, int BK_, int MP_ = 1, int OCC_ = 1>
 struct TcCfg {
-  static constexpr int BM = 128, BK = BK_, MP = MP_;
+  static constexpr int BM = 128, BK = BK_, MP = MP_, OCC = OCC_;
   static constexpr int A_BYTES = BM * BK * 2;  // one M-tile
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = MP * A_BYTES + B_BYTES;
-  static constexpr int NBUF = MP == 1 ? 2 : 1;  // accumulator buffers
-  static constexpr int TMEM_COLS = 2 * BN;      // NBUF * MP accumulators of BN columns
+  static constexpr int NBUF = (MP == 1 && OCC == 1) ? 2 : 1;  // accumulator buffers
+  static constexpr int TMEM_COLS = NBUF * MP * BN;             // power of two for BN in {128, 256}
   static constexpr int MAXG = DECOMOE_MAX_E;
-  static constexpr int NBARS = 2 * STAGES + 5;
+  static constexpr int TQ = 4;  // depth of the tile-id queue (dynamic scheduling)
+  static constexpr int NBARS = 2 * STAGES + 5 + 2 * TQ;
   static constexpr size_t SMEM =
-      1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + NBARS * 8 + 2 * (MAXG + 1) * 4 + 16;
+      1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + NBARS * 8 + 2 * (MAXG + 1) * 4 + 16 + TQ * 4;
 };
 
 // Work item -> (group, M-tile inside the group, N-tile). M-tiles are visited
@@ -162,11 +167,11 @@ __device__ __forceinline__ void tile_coords(int tile, int NT, const int* s_mt, i
 
 // EW epilogue warps (4 or 8): with 8, two warps share each 32-lane TMEM
 // quarter and split its column chunks, so the epilogue's latency is hidden.
-template <int BN, int EPI, int STAGES, int BK, bool GATHER_A = false, int MP = 1, int EW = 8>
-__global__ void __launch_bounds__(64 + 32 * EW, 1)
+template <int BN, int EPI, int STAGES, int BK, bool GATHER_A = false, int MP = 1, int EW = 8, int OCC = 1>
+__global__ void __launch_bounds__(64 + 32 * EW, OCC)
     k_gemm_tc(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b,
               const TcArgs g) {
-  using C = TcCfg<BN, STAGES, BK, MP>;
+  using C = TcCfg<BN, STAGES, BK, MP, OCC>;
   static_assert(!(GATHER_A && MP != 1), "gathered A takes one M-tile per work item");
   __shared__ int s_arow[GATHER_A ? 128 : 1];
   extern __shared__ uint8_t smem_raw[];
@@ -180,15 +185,18 @@ __global__ void __launch_bounds__(64 + 32 * EW, 1)
   int* s_mt = s_off + (C::MAXG + 1);
   volatile uint32_t* s_tmem = reinterpret_cast<volatile uint32_t*>(s_mt + (C::MAXG + 1));
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
+  volatile int* s_tq = reinterpret_cast<volatile int*>(s_tmem + 4);  // [TQ] tile ids
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t bar0 = smem_u32(bars);
-  // barrier slots: full[STAGES] | empty[STAGES] | tfull[2] | tempty[2] | drain
+  // barrier slots: full[STAGES] | empty[STAGES] | tfull[2] | tempty[2] | drain | tqfull[TQ] | tqempty[TQ]
 #define FULL_BAR(s) (bar0 + 8u * (s))
 #define EMPTY_BAR(s) (bar0 + 8u * (STAGES + (s)))
 #define TFULL_BAR(a) (bar0 + 8u * (2 * STAGES + (a)))
 #define TEMPTY_BAR(a) (bar0 + 8u * (2 * STAGES + 2 + (a)))
 #define DRAIN_BAR (bar0 + 8u * (2 * STAGES + 4))
+#define TQF_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + (i)))
+#define TQE_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + C::TQ + (i)))
 
   const int G = g.ngroups;
   for (int i = threadIdx.x; i <= G; i += blockDim.x)
@@ -204,6 +212,10 @@ __global__ void __launch_bounds__(64 + 32 * EW, 1)
       mbar_init(TEMPTY_BAR(a), 32 * EW);
     }
     mbar_init(DRAIN_BAR, 1);
+    for (int i = 0; i < C::TQ; ++i) {
+      mbar_init(TQF_BAR(i), 1);
+      mbar_init(TQE_BAR(i), 1 + EW);  // the MMA thread and lane 0 of every epilogue warp
+    }
     fence_mbar_init();
   }
   __syncthreads();
@@ -252,6 +264,35 @@ __global__ void __launch_bounds__(64 + 32 * EW, 1)
   const uint32_t tmem_base = *s_tmem;
   const int KB = g.kdim / C::BK;
 
+  // Tile sequence of this CTA. Static: blockIdx.x, + gridDim.x, ... Dynamic:
+  // the producer takes the next id from the global counter and passes it to
+  // the MMA and epilogue warps through a TQ-deep shared-memory queue; -1 ends.
+  const bool dyn = !GATHER_A && g.sched != nullptr;
+  auto static_tile = [&](int i) -> int {
+    const int t = static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x);
+    return t < total ? t : -1;
+  };
+  auto produce_tile = [&](int i) -> int {  // producer thread; returns -2 on timeout
+    if (!dyn) return static_tile(i);
+    const int slot = i % C::TQ;
+    const uint32_t qph = (i / C::TQ) & 1;
+    if (!mbar_wait(TQE_BAR(slot), qph ^ 1u, g.limit_ns, s_abort)) return -2;
+    int t = atomicAdd(g.sched, 1);
+    if (t >= total) t = -1;
+    s_tq[slot] = t;
+    mbar_arrive(TQF_BAR(slot));
+    return t;
+  };
+  auto consume_tile = [&](int i, bool arrive) -> int {  // returns -2 on timeout
+    if (!dyn) return static_tile(i);
+    const int slot = i % C::TQ;
+    const uint32_t qph = (i / C::TQ) & 1;
+    if (!mbar_wait(TQF_BAR(slot), qph, g.limit_ns, s_abort)) return -2;
+    const int t = s_tq[slot];
+    if (arrive) mbar_arrive(TQE_BAR(slot));
+    return t;
+  };
+
   if (warp == 0) {
     // ------------------------------------------------ TMA producer (lane 0
     // issues; with GATHER_A the whole warp first reads the tile's 128 A row
@@ -265,7 +306,15 @@ __global__ void __launch_bounds__(64 + 32 * EW, 1)
     bool ok = true;
     uint32_t armed = 0;  // bit s: stage s was ever filled
     uint32_t armed_ph = 0;
-    for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+    for (int ti = 0;; ++ti) {
+      int tile = 0;
+      if (lane == 0) tile = produce_tile(ti);
+      tile = __shfl_sync(0xffffffffu, tile, 0);
+      if (tile == -2) {
+        ok = false;
+        break;
+      }
+      if (tile < 0) break;
       int grp, mt, nb;
       tile_coords(tile, NT, s_mt, G, grp, mt, nb);
       const int row0 = s_off[grp] + mt * MP * C::BM;
@@ -340,8 +389,13 @@ __global__ void __launch_bounds__(64 + 32 * EW, 1)
     int stage = 0;
     uint32_t ph = 0;
     bool ok = true, issued = false;
-    int it = 0;
-    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
+    for (int it = 0;; ++it) {
+      const int tile = consume_tile(it, true);
+      if (tile == -2) {
+        ok = false;
+        break;
+      }
+      if (tile < 0) break;
       const int acc = it % C::NBUF;
       const uint32_t aph = (it / C::NBUF) & 1;
       bool has2 = false;
@@ -395,9 +449,16 @@ __global__ void __launch_bounds__(64 + 32 * EW, 1)
     const int q = warp & 3;            // TMEM lanes [32q, 32q + 32) belong to this warp
     const int wp = (warp - 2) >> 2;    // which of the quarter's warps (0 .. EW/4 - 1)
     constexpr int WPQ = EW / 4;        // warps per quarter: column chunks are dealt round robin
-    int it = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
+    for (int it = 0;; ++it) {
+      int tile = 0;
+      if (lane == 0) tile = consume_tile(it, true);
+      tile = __shfl_sync(0xffffffffu, tile, 0);
+      if (tile == -2) {
+        ok = false;
+        break;
+      }
+      if (tile < 0) break;
       const int acc = it % C::NBUF;
       const uint32_t aph = (it / C::NBUF) & 1;
       int grp, mt, nb;
@@ -537,16 +598,18 @@ __global__ void __launch_bounds__(64 + 32 * EW, 1)
 #undef TFULL_BAR
 #undef TEMPTY_BAR
 #undef DRAIN_BAR
+#undef TQF_BAR
+#undef TQE_BAR
 }
 
 // A: [rows, kdim], or with GATHER_A the source tensor [a_tensor_rows, kdim]
 // whose row a_rows[r] is A row r.
-template <int BN, int EPI, int STAGES, int BK, bool GATHER_A = false, int MP = 1>
+template <int BN, int EPI, int STAGES, int BK, bool GATHER_A = false, int MP = 1, int EW = 8, int OCC = 1>
 static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b_rows,
                      const int32_t* offsets, int ngroups, int n_per_group, void* out,
                      int64_t out_ld, const float* bias, int32_t* status, cudaStream_t s, int n_valid = 0,
-                     const int32_t* a_rows = nullptr, int64_t a_tensor_rows = 0) {
-  using C = TcCfg<BN, STAGES, BK, MP>;
+                     const int32_t* a_rows = nullptr, int64_t a_tensor_rows = 0, int* sched = nullptr) {
+  using C = TcCfg<BN, STAGES, BK, MP, OCC>;
   CUtensorMap ta, tb;
   if (GATHER_A)
     DM_RET(make_tmap_bf16(&ta, A, static_cast<uint64_t>(kdim), static_cast<uint64_t>(a_tensor_rows), 1, BK));
@@ -566,19 +629,21 @@ static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b
   g.limit_ns = static_cast<uint64_t>(wait_limit_ns());
   g.n_valid = n_valid;
   g.a_rows = a_rows;
-  auto kern = k_gemm_tc<BN, EPI, STAGES, BK, GATHER_A, MP>;
+  g.sched = sched;
+  if (sched != nullptr) DM_CUDA_CHECK(cudaMemsetAsync(sched, 0, sizeof(int), s));
+  auto kern = k_gemm_tc<BN, EPI, STAGES, BK, GATHER_A, MP, EW, OCC>;
   static_assert(C::SMEM <= 232448, "shared memory budget");
   DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(C::SMEM)));
   const int64_t ub_tiles =
       (static_cast<int64_t>(rows) / C::BM + ngroups) * static_cast<int64_t>(n_per_group / BN);
 #ifdef DECOMOE_GRID_CAP
-  const int64_t cap = std::min<int64_t>(sm_count(), DECOMOE_GRID_CAP);
+  const int64_t cap = std::min<int64_t>(static_cast<int64_t>(sm_count()) * OCC, DECOMOE_GRID_CAP);
 #else
-  const int64_t cap = sm_count();
+  const int64_t cap = static_cast<int64_t>(sm_count()) * OCC;
 #endif
   const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(cap, ub_tiles)));
-  kern<<<grid, 64 + 32 * 8, C::SMEM, s>>>(ta, tb, g);
+  kern<<<grid, 64 + 32 * EW, C::SMEM, s>>>(ta, tb, g);
   DM_LAUNCH_CHECK("k_gemm_tc");
   return DECOMOE_OK;
 }
@@ -1319,6 +1384,18 @@ static bool use_decode_path(int64_t rows) { return rows <= DECOMOE_DECODE_ROWS; 
 #ifndef DECOMOE_GU_MP
 #define DECOMOE_GU_MP 1
 #endif
+#ifndef DECOMOE_GU_OCC
+#define DECOMOE_GU_OCC 1
+#endif
+#ifndef DECOMOE_DN_OCC
+#define DECOMOE_DN_OCC 1
+#endif
+#ifndef DECOMOE_GU_EW
+#define DECOMOE_GU_EW 8
+#endif
+#ifndef DECOMOE_DN_EW
+#define DECOMOE_DN_EW 8
+#endif
 #ifndef DECOMOE_DN_MP
 #define DECOMOE_DN_MP 1
 #endif
@@ -1328,9 +1405,10 @@ static bool use_decode_path(int64_t rows) { return rows <= DECOMOE_DECODE_ROWS; 
 constexpr int GU_BK = DECOMOE_GU_BK, GU_STAGES = DECOMOE_GU_STAGES;
 constexpr int DN_BK = DECOMOE_DN_BK, DN_STAGES = DECOMOE_DN_STAGES;
 constexpr int GU_MP = DECOMOE_GU_MP, DN_MP = DECOMOE_DN_MP;
+constexpr int GU_OCC = DECOMOE_GU_OCC, DN_OCC = DECOMOE_DN_OCC, GU_EW = DECOMOE_GU_EW, DN_EW = DECOMOE_DN_EW;
 
 int decomoe_expert_gate_up(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m,
-                           int dtype, const void* w_gate_up, void* h, int32_t* status_dev,
+                           int dtype, const void* w_gate_up, void* h, int32_t* status_dev, int32_t* sched_dev,
                            decomoe_stream_t stream) {
   clear_error();
   DM_RET(expert_check("expert_gate_up", x_perm, offsets, rows, K, d, m, dtype, w_gate_up, h));
@@ -1359,12 +1437,14 @@ int decomoe_expert_gate_up(const void* x_perm, const int32_t* offsets, int64_t r
   if (static_cast<int64_t>(R) <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K)
     return launch_ws<true, 4>(x_perm, R, d, w_gate_up, 2 * m, offsets, K, h, m, status_dev, s);
   // A = x_perm [R, d], B = w_gate_up [K*2m, d] (only experts < K are read)
-  return launch_tc<256, EPI_SWIGLU, GU_STAGES, GU_BK, false, GU_MP>(
-      x_perm, R, d, w_gate_up, static_cast<int64_t>(K) * 2 * m, offsets, K, 2 * m, h, m, nullptr, status_dev, s);
+  return launch_tc<256, EPI_SWIGLU, GU_STAGES, GU_BK, false, GU_MP, GU_EW, GU_OCC>(
+      x_perm, R, d, w_gate_up, static_cast<int64_t>(K) * 2 * m, offsets, K, 2 * m, h, m, nullptr, status_dev, s, 0,
+      nullptr, 0, sched_dev);
 }
 
 int decomoe_expert_down(const void* h, const int32_t* offsets, int64_t rows, int K, int d, int m, int dtype,
-                        const void* w_down, void* y_perm, int32_t* status_dev, decomoe_stream_t stream) {
+                        const void* w_down, void* y_perm, int32_t* status_dev, int32_t* sched_dev,
+                        decomoe_stream_t stream) {
   clear_error();
   DM_RET(expert_check("expert_down", h, offsets, rows, K, d, m, dtype, w_down, y_perm));
   if (rows == 0) return DECOMOE_OK;
@@ -1391,13 +1471,15 @@ int decomoe_expert_down(const void* h, const int32_t* offsets, int64_t rows, int
   if (static_cast<int64_t>(R) <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K)
     return launch_ws<false, 4>(h, R, m, w_down, d, offsets, K, y_perm, d, status_dev, s);
   // A = h [R, m], B = w_down [K*d, m]
-  return launch_tc<256, EPI_BF16, DN_STAGES, DN_BK, false, DN_MP>(h, R, m, w_down, static_cast<int64_t>(K) * d, offsets,
-                                                                  K, d, y_perm, d, nullptr, status_dev, s);
+  return launch_tc<256, EPI_BF16, DN_STAGES, DN_BK, false, DN_MP, DN_EW, DN_OCC>(h, R, m, w_down, static_cast<int64_t>(K) * d, offsets,
+                                                                  K, d, y_perm, d, nullptr, status_dev, s, 0,
+                                                                  nullptr, 0, sched_dev);
 }
 
 int decomoe_expert_gate_up_gather(const void* x, int64_t T, const int32_t* perm_token, const int32_t* offsets,
                                   int64_t rows, int K, int d, int m, int dtype, const void* w_gate_up, void* h,
-                                  int32_t* status_dev, decomoe_stream_t stream) {
+                                  int32_t* status_dev, int32_t* sched_dev, decomoe_stream_t stream) {
+  (void)sched_dev;  // the gathered form keeps the static tile order
   clear_error();
   DM_RET(expert_check("expert_gate_up_gather", x, offsets, rows, K, d, m, dtype, w_gate_up, h));
   if (rows == 0) return DECOMOE_OK;
@@ -1422,17 +1504,18 @@ int decomoe_expert_gate_up_gather(const void* x, int64_t T, const int32_t* perm_
 int decomoe_expert_swiglu_gather(const void* x, int64_t T, const int32_t* perm_token, const int32_t* offsets,
                                  int64_t rows, int K, int d, int m, int dtype, const void* w_gate_up,
                                  const void* w_down, void* h_ws, void* y_perm, int32_t* status_dev,
-                                 decomoe_stream_t stream) {
+                                 int32_t* sched_dev, decomoe_stream_t stream) {
   DM_RET(decomoe_expert_gate_up_gather(x, T, perm_token, offsets, rows, K, d, m, dtype, w_gate_up, h_ws,
-                                       status_dev, stream));
-  return decomoe_expert_down(h_ws, offsets, rows, K, d, m, dtype, w_down, y_perm, status_dev, stream);
+                                       status_dev, sched_dev, stream));
+  return decomoe_expert_down(h_ws, offsets, rows, K, d, m, dtype, w_down, y_perm, status_dev, sched_dev, stream);
 }
 
 int decomoe_expert_swiglu(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m,
                           int dtype, const void* w_gate_up, const void* w_down, void* h_ws, void* y_perm,
-                          int32_t* status_dev, decomoe_stream_t stream) {
-  DM_RET(decomoe_expert_gate_up(x_perm, offsets, rows, K, d, m, dtype, w_gate_up, h_ws, status_dev, stream));
-  return decomoe_expert_down(h_ws, offsets, rows, K, d, m, dtype, w_down, y_perm, status_dev, stream);
+                          int32_t* status_dev, int32_t* sched_dev, decomoe_stream_t stream) {
+  DM_RET(decomoe_expert_gate_up(x_perm, offsets, rows, K, d, m, dtype, w_gate_up, h_ws, status_dev, sched_dev,
+                                stream));
+  return decomoe_expert_down(h_ws, offsets, rows, K, d, m, dtype, w_down, y_perm, status_dev, sched_dev, stream);
 }
 
 // Reference CUDA-core path for bf16 (same math as the tensor-core path: bf16

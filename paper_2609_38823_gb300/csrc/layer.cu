@@ -23,6 +23,7 @@ enum {
   WS_ROUTE,
   WS_DISPATCH,
   WS_KDEV,
+  WS_SCHED,
   WS_STATUS_PAD,
   WS_COUNT
 };
@@ -51,6 +52,7 @@ static LayerLayout layer_layout(int64_t T, int d, int E, int k, int m, int dtype
   sz[WS_ROUTE] = decomoe_route_workspace_bytes(T, E);
   sz[WS_DISPATCH] = decomoe_dispatch_workspace_bytes(T, k, E);
   sz[WS_KDEV] = 16;
+  sz[WS_SCHED] = 16;
   sz[WS_STATUS_PAD] = 256;
   size_t o = 0;
   for (int i = 0; i < WS_COUNT; ++i) {
@@ -163,8 +165,9 @@ int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const v
   DM_RET(decomoe_dispatch(topk_idx, T, k, K, x, d, dtype, counts, offsets, perm, inv, x_perm, disp_ws,
                           decomoe_dispatch_workspace_bytes(T, k, K), status_dev, stream));
   // a6: grouped SwiGLU experts over [0, K)
+  int32_t* sched = reinterpret_cast<int32_t*>(base + L.off[WS_SCHED]);
   DM_RET(decomoe_expert_swiglu(x_perm, offsets, T * k, K, d, m, dtype, w_gate_up, w_down, h, y_perm,
-                               status_dev, stream));
+                               status_dev, sched, stream));
   // a7: combine (+ residual)
   DM_RET(decomoe_combine(y_perm, inv, topk_w, T, k, d, dtype, residual, out, stream));
   return DECOMOE_OK;

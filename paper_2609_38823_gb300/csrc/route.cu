@@ -50,39 +50,48 @@ __global__ void k_router_simt(const T* __restrict__ x, const T* __restrict__ w_r
 constexpr int ROUTE_THREADS = 256;
 constexpr int ROUTE_TPB = 8;  // tokens per block: one per warp
 
-// k rounds of warp arg-max over entries e < lim not yet taken; returns the
-// pick of round `lane` in (my_v, my_i) and whether every pick is < K.
-__device__ __forceinline__ void warp_topk(const float (&v)[8], int lim, int k, int lane, float& my_v, int& my_i) {
-  uint32_t taken = 0;
+// Order-preserving 32-bit key of a float (larger float -> larger key; -0 and
+// +0 share a key so equal values tie). Key 0 is below every float's key and
+// marks entries that are out of range or already picked.
+__device__ __forceinline__ uint32_t fkey(float f) {
+  const uint32_t u = (f == 0.0f) ? 0u : __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float fkey_inv(uint32_t k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
+}
+
+// k rounds of warp arg-max over entries e < lim: each round one redux.sync
+// max over the lanes' best keys, then one redux.sync min over the indices of
+// the lanes holding that key (lower index wins a tie). Pick j ends in lane j.
+__device__ __forceinline__ void warp_topk(const uint32_t (&key_in)[8], int lim, int k, int lane, float& my_v,
+                                          int& my_i) {
+  uint32_t key[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) key[i] = (lane + 32 * i < lim) ? key_in[i] : 0u;
   my_v = 0.f;
   my_i = 0;
   for (int j = 0; j < k; ++j) {
-    float bv = 0.f;
-    int bi = INT_MAX;
+    uint32_t bk = 0;
+    int bs = 0;  // slot of the lane's best (entries ascend with the slot, so strict > keeps the lowest index)
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int e = lane + 32 * i;
-      if (e < lim && !((taken >> i) & 1u)) {
-        if (bi == INT_MAX || v[i] > bv || (v[i] == bv && e < bi)) {
-          bv = v[i];
-          bi = e;
-        }
+    for (int i = 0; i < 8; ++i)
+      if (key[i] > bk) {
+        bk = key[i];
+        bs = i;
       }
-    }
+    const uint32_t mk = __reduce_max_sync(0xffffffffu, bk);
+    const uint32_t cand = (bk == mk) ? static_cast<uint32_t>(lane + 32 * bs) : 0xffffffffu;
+    const uint32_t wi = __reduce_min_sync(0xffffffffu, cand);
+    {
+      const bool mine = (wi & 31u) == static_cast<uint32_t>(lane);
+      const int sl = static_cast<int>(wi >> 5);
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
-      const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-      const bool better = (oi != INT_MAX) && (bi == INT_MAX || ov > bv || (ov == bv && oi < bi));
-      if (better) {
-        bv = ov;
-        bi = oi;
-      }
+      for (int i = 0; i < 8; ++i) key[i] = (mine && i == sl) ? 0u : key[i];  // selects keep key[] in registers
     }
-    if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
     if (lane == j) {
-      my_v = bv;
-      my_i = bi;
+      my_v = fkey_inv(mk);
+      my_i = static_cast<int>(wi);
     }
   }
 }
@@ -110,11 +119,11 @@ __global__ void __launch_bounds__(ROUTE_THREADS)
   if (t < Tn) {
     const float* row = logits + t * ld;
     const int lim = mass ? E : K;
-    float v[8];
+    uint32_t v[8];  // order-preserving keys of the row's logits
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const int e = lane + 32 * i;
-      v[i] = (e < lim) ? row[e] : -FLT_MAX;
+      v[i] = (e < lim) ? fkey(row[e]) : 0u;
     }
     float my_v;
     int my_i;

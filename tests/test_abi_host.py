@@ -82,7 +82,7 @@ def test_argument_errors_are_caught_before_launch():
     # visual block past the end
     assert L.decomoe_drop_visual_block(fake, fake, 10, 16, 8, 3, 1, 160, 112, None) == 1
     # m not a multiple of the gate/up block
-    assert L.decomoe_expert_swiglu(fake, fake, 100, 4, 256, 100, 0, fake, fake, fake, fake, None, None) == 1
+    assert L.decomoe_expert_swiglu(fake, fake, 100, 4, 256, 100, 0, fake, fake, fake, fake, None, None, None) == 1
     # K_fixed < k
     assert L.decomoe_moe_layer(fake, fake, None, fake, fake, 4, 256, 16, 4, 128, 0, 2, 0.0, None, fake,
                                None, None, fake, 1 << 30, None, None) == 1

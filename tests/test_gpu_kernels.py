@@ -236,6 +236,14 @@ def test_expert_swiglu_bf16_parity(T, k, K, d, m, pattern):
     dm.decomoe_expert_swiglu_ref(xp, off, K, w_gu, g["w_down"], h2, y2)
     torch.cuda.synchronize()
     assert_close_out(f64(y), f64(y2), 2e-3, 1e-2, "tensor-core vs CUDA-core reference")
+    # dynamic tile scheduling hands the same tiles out in another order: same bits
+    sched = torch.zeros(1, dtype=torch.int32, device=DEV)
+    h4 = torch.empty_like(h)
+    y4 = torch.empty_like(y)
+    dm.decomoe_expert_swiglu(xp, off, K, w_gu, g["w_down"], h4, y4, status, sched)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(status) == 0
+    assert torch.equal(y4, y) and torch.equal(h4, h)
     # gather form: rows read from the token-ordered x through perm_token give
     # the same shared-memory tiles, so the same bits
     h3 = torch.empty_like(h)
