@@ -1,4 +1,5 @@
-"""CPU oracle of the DecoMoE prefix-restricted MoE layer and visual-block removal.
+"""CPU oracle of the DecoMoE prefix-restricted MoE layer, its offline Mean-Mass
+expert calibration, the SAVB exit gate and visual-block removal.
 
 TEST INFRASTRUCTURE ONLY. This module is the plain, slow, obviously-correct
 statement of what the DecoMoE paper's method computes, in float64 with numpy.
@@ -284,6 +285,113 @@ def moe_token(x_t, a_t, w_gate, w_up, w_down, K, k):
         u = np.asarray(w_up[e], F64) @ x_t
         out += w[0, j] * (np.asarray(w_down[e], F64) @ (silu(g) * u))
     return out, idx[0], w[0]
+
+
+# ---------------------------------------------------------------------------
+# RCEP offline calibration: text-token routed mass and the Mean-Mass expert
+# order (Section 3.3, Eqs. 8-9; Algorithm 1, last two loops; Appendix, "RCEP
+# Calibration and Text-Routing Alignment")
+# ---------------------------------------------------------------------------
+
+def text_routed_mass(a_text, k):
+    """Eq. 9: M_{c,l,e} = (1/|T|) * sum over the case's text tokens i of the
+    renormalised full-pool top-k weight of expert e (rho_e / sum of rho over
+    the k selected experts; zero where e is not selected).
+
+    ``a_text``: float32 router logits [n, E] of the case's text tokens at one
+    layer (n >= 1). The top-k sets and weights are those of Eq. 10 / Eq. 11
+    (full_pool_route), summed in token order in float64, then divided by n.
+    Returns M [E] float64 (it sums to 1 up to rounding).
+    """
+    a_text = np.asarray(a_text)
+    n = a_text.shape[0]
+    if n < 1:
+        raise ValueError("a case needs at least one text token")
+    return activated_mass(a_text, k) / F64(n)
+
+
+def mean_mass_order(case_masses):
+    """Eq. 8: pi_l = argsort over experts of the case-mean routed mass,
+    descending. The Appendix averages within a case first (Eq. 9) and then
+    across cases, so every case has equal weight.
+
+    Reading where the paper is silent: equal means keep ascending expert index
+    (a stable sort), so pi is unique. The mean is the float64 sum over cases in
+    their given order divided by the case count.
+    ``case_masses``: [C, E]. Returns (pi [E] int64, mean [E] float64): new
+    expert position i holds original expert pi[i].
+    """
+    M = np.asarray(case_masses, F64)
+    C, E = M.shape
+    if C < 1:
+        raise ValueError("need at least one calibration case")
+    tot = np.zeros(E, F64)
+    for c in range(C):
+        tot = tot + M[c]
+    mean = tot / F64(C)
+    pi = np.argsort(-mean, kind="stable")
+    return pi.astype(np.int64), mean
+
+
+def apply_expert_order(pi, w_r, bias, w_gate, w_up, w_down):
+    """Algorithm 1, last loop; Section 3.3 after Eq. 8: the same permutation
+    applied to the router output rows (and the per-expert router bias of the
+    synthetic workload) and to the gate/up and down tensors of the experts.
+    Only the storage order changes. Returns the reordered copies."""
+    pi = np.asarray(pi, np.int64)
+    return (np.asarray(w_r)[pi], None if bias is None else np.asarray(bias)[pi], np.asarray(w_gate)[pi],
+            np.asarray(w_up)[pi], np.asarray(w_down)[pi])
+
+
+# ---------------------------------------------------------------------------
+# SAVB gate (Section 3.2, Eqs. 2-3; Appendix, "SAVB Supervision")
+# ---------------------------------------------------------------------------
+
+def candidate_layers(n_layers, first=3, step=4):
+    """The sparse candidate set G = {3, 7, 11, ...} (zero-based layer indices,
+    Appendix "Offline Calibration"), every fourth decoder layer."""
+    return list(range(first, n_layers, step))
+
+
+def gate_feature(h, v0, nv):
+    """Eq. 2: x = [mean of text states 1..n-1 ; text state n] in R^{2d}.
+
+    Reading: the text tokens are the rows outside the contiguous visual block
+    [v0, v0+nv), in sequence order (system-prompt rows before the block and the
+    text after it). With a single text row the pooled half is zero. Float64.
+    """
+    T = drop_visual_block(np.asarray(h, F64), v0, nv)
+    n, d = T.shape
+    if n < 1:
+        raise ValueError("no text rows")
+    pooled = np.zeros(d, F64)
+    for j in range(n - 1):
+        pooled = pooled + T[j]
+    if n > 1:
+        pooled = pooled / F64(n - 1)
+    return np.concatenate([pooled, T[n - 1]])
+
+
+def gate_logits(x, w1, b1, w2, b2):
+    """The two-class MLP g_phi of Eq. 3 with one hidden layer (512 wide in the
+    Appendix): z = W2 relu(W1 x + b1) + b2, z in R^2.
+
+    Reading: the paper does not name the hidden activation; ReLU is taken.
+    w1: [H, 2d], b1: [H], w2: [2, H], b2: [2]. Float64.
+    """
+    hdn = np.asarray(w1, F64) @ np.asarray(x, F64) + np.asarray(b1, F64)
+    hdn = np.maximum(hdn, 0.0)
+    return np.asarray(w2, F64) @ hdn + np.asarray(b2, F64)
+
+
+def gate_exit_prob(z):
+    """Eq. 3: p_exit = softmax(z)_1 (class 1 is "exit")."""
+    return float(softmax(np.asarray(z, F64)[None, :])[0, 1])
+
+
+def gate_decision(p_exit, theta):
+    """Eq. 3: Exit = [p_exit >= theta]."""
+    return bool(p_exit >= theta)
 
 
 # ---------------------------------------------------------------------------

@@ -40,7 +40,8 @@ def build(verbose: bool = False, ptxas_info: bool = False, force: bool = False) 
     os.makedirs(BUILD, exist_ok=True)
     nvcc = nvcc_path()
     srcs = [os.path.join(CSRC, s) for s in CU_SOURCES + C_SOURCES]
-    hdrs = [os.path.join(CSRC, "decomoe_internal.cuh"), os.path.join(ROOT, "include", "decomoe.h")]
+    hdrs = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cuh")]
+    hdrs.append(os.path.join(ROOT, "include", "decomoe.h"))
     if not force and os.path.exists(LIB):
         lib_t = os.path.getmtime(LIB)
         if all(os.path.getmtime(p) < lib_t for p in srcs + hdrs + [__file__]):

@@ -407,3 +407,121 @@ def test_stack_one_layer_is_residual_moe():
         xn = O.rmsnorm(x[t:t + 1])
         ref = O.moe_layer(xn, w_r, b, wg, wu, wd, k=2, K=4)["out"][0] + x[t]
         np.testing.assert_allclose(h, ref, rtol=1e-13, atol=1e-13)
+
+
+# ---------------------------------------------------------------- calibration (Eqs. 8-9)
+
+def test_text_routed_mass_closed_form_and_sum():
+    # token 0 ties its top 2 at 3.0 (weights 1/2, 1/2); token 1 picks experts
+    # 3 and 1 with logits differing by ln 3 (weights 3/4, 1/4)
+    a = np.array([[3.0, -9.0, 3.0, -9.0, -9.0],
+                  [-9.0, 1.0, -9.0, 1.0 + math.log(3.0), -9.0]], dtype=np.float32)
+    M = O.text_routed_mass(a, 2)
+    w1 = math.exp(float(np.float32(1.0))) / (math.exp(float(np.float32(1.0))) + math.exp(float(a[1, 3])))
+    expect = np.array([0.25, w1 / 2, 0.25, (1 - w1) / 2, 0.0])
+    assert np.allclose(M, expect, rtol=0, atol=1e-15)
+    r = np.random.default_rng(3)
+    for n, E, k in ((1, 16, 2), (37, 128, 8), (200, 64, 4)):
+        M = O.text_routed_mass(r.standard_normal((n, E)).astype(np.float32), k)
+        assert abs(M.sum() - 1.0) < 1e-12 and (M >= 0).all()
+        assert (M > 0).sum() <= min(E, n * k)
+
+
+def test_mean_mass_order_ties_and_case_weighting():
+    # case means: e0 (0.1+0.3)/2 = 0.2, e1 0.4, e2 0.2, e3 0.2 -> ties keep index order
+    M = np.array([[0.1, 0.5, 0.2, 0.2], [0.3, 0.3, 0.2, 0.2]])
+    pi, mean = O.mean_mass_order(M)
+    assert pi.tolist() == [1, 0, 2, 3]
+    assert np.allclose(mean, [0.2, 0.4, 0.2, 0.2])
+    # every case counts once, however many tokens it had: duplicating the
+    # cases leaves the order unchanged
+    pi2, _ = O.mean_mass_order(np.concatenate([M, M]))
+    assert pi2.tolist() == pi.tolist()
+
+
+def test_mean_mass_order_maximises_every_prefix_bruteforce():
+    # the sorted order puts the largest total mean mass into every prefix
+    r = np.random.default_rng(11)
+    M = r.dirichlet(np.ones(6), size=5)
+    pi, mean = O.mean_mass_order(M)
+    for K in range(1, 7):
+        best = max(sum(mean[list(c)]) for c in itertools.combinations(range(6), K))
+        assert abs(sum(mean[pi[:K]]) - best) < 1e-15
+    assert sorted(pi.tolist()) == list(range(6))
+
+
+def _calib_layer(seed, E=6, d=8, m=4):
+    r = np.random.default_rng(seed)
+    return dict(w_r=r.standard_normal((E, d)) * 0.5, bias=r.standard_normal(E) * 0.3,
+                w_gate=r.standard_normal((E, m, d)) * 0.3, w_up=r.standard_normal((E, m, d)) * 0.3,
+                w_down=r.standard_normal((E, d, m)) * 0.3)
+
+
+def test_reorder_is_identity_on_unsliced_layer():
+    # Section 3.3 / Appendix: the permutation of router rows and expert tensors
+    # changes only the storage order; with every expert kept (K = E) the layer
+    # output is unchanged
+    L = _calib_layer(5)
+    x = np.random.default_rng(6).standard_normal((9, 8))
+    pi = np.array([4, 0, 5, 2, 1, 3])
+    w_r, b, wg, wu, wd = O.apply_expert_order(pi, L["w_r"], L["bias"], L["w_gate"], L["w_up"], L["w_down"])
+    ref = O.moe_layer(x, L["w_r"], L["bias"], L["w_gate"], L["w_up"], L["w_down"], k=2, K=6)["out"]
+    got = O.moe_layer(x, w_r, b, wg, wu, wd, k=2, K=6)["out"]
+    assert np.allclose(got, ref, rtol=0, atol=1e-12)
+    # a mistake in one tensor (gate/up permuted, down not) breaks it
+    bad = O.moe_layer(x, w_r, b, wg, wu, L["w_down"], k=2, K=6)["out"]
+    assert np.abs(bad - ref).max() > 1e-3
+
+
+def test_reorder_by_calibrated_order_sorts_the_calibration_mass():
+    # after applying pi, recomputing the cases' routed mass gives experts in
+    # non-increasing mean mass: the leading positions form the mass prefix
+    L = _calib_layer(8, E=6)
+    r = np.random.default_rng(9)
+    cases = [r.standard_normal((int(n), 8)) for n in (3, 11, 6)]
+    Ms = [O.text_routed_mass(O.router_logits(c, L["w_r"], L["bias"]), 2) for c in cases]
+    pi, mean = O.mean_mass_order(np.stack(Ms))
+    w_r, b, _, _, _ = O.apply_expert_order(pi, L["w_r"], L["bias"], L["w_gate"], L["w_up"], L["w_down"])
+    Ms2 = [O.text_routed_mass(O.router_logits(c, w_r, b), 2) for c in cases]
+    _, mean2 = O.mean_mass_order(np.stack(Ms2))
+    assert np.allclose(mean2, mean[pi], rtol=0, atol=1e-12)
+    assert (np.diff(mean2) <= 1e-15).all()
+
+
+# ---------------------------------------------------------------- SAVB gate (Eqs. 2-3)
+
+def test_candidate_layers_every_fourth_from_three():
+    assert O.candidate_layers(48) == [3 + 4 * i for i in range(12)]
+    assert O.candidate_layers(48)[-1] == 47 and 19 in O.candidate_layers(48)
+
+
+def test_gate_feature_pooling_closed_forms():
+    h = np.arange(7 * 3, dtype=np.float64).reshape(7, 3)
+    # visual rows 1..3 removed: text rows 0, 4, 5, 6; pooled over 0, 4, 5; last = 6
+    x = O.gate_feature(h, 1, 3)
+    assert np.allclose(x[:3], (h[0] + h[4] + h[5]) / 3) and np.array_equal(x[3:], h[6])
+    # n = 2: the pooled half is the first text row itself
+    x2 = O.gate_feature(h[:2], 0, 0)
+    assert np.array_equal(x2, np.concatenate([h[0], h[1]]))
+    # one text row: pooled half zero
+    assert np.array_equal(O.gate_feature(h[:3], 0, 2), np.concatenate([np.zeros(3), h[2]]))
+    # the pooled half does not depend on the order of the preceding text rows
+    perm = h[[5, 0, 4, 6]]
+    assert np.allclose(O.gate_feature(perm, 0, 0)[:3], x[:3])
+
+
+def test_gate_mlp_closed_form_sigmoid():
+    # W1 picks x0 and -x0 through the ReLU, W2 subtracts them: z = [0, x0],
+    # so p_exit = softmax(z)_1 = 1 / (1 + exp(-x0))
+    w1 = np.zeros((2, 4)); w1[0, 0] = 1.0; w1[1, 0] = -1.0
+    w2 = np.array([[0.0, 0.0], [1.0, -1.0]])
+    for x0 in (-3.0, -0.5, 0.0, 0.7, 4.0):
+        x = np.array([x0, 9.0, -2.0, 1.0])
+        z = O.gate_logits(x, w1, np.zeros(2), w2, np.zeros(2))
+        assert np.allclose(z, [0.0, x0])
+        assert abs(O.gate_exit_prob(z) - 1.0 / (1.0 + math.exp(-x0))) < 1e-15
+    assert O.gate_decision(0.5, 0.5) and not O.gate_decision(0.4999, 0.5)
+    # the hidden layer really is rectified: a negative pre-activation is dropped
+    z = O.gate_logits(np.array([-1.0, 0, 0, 0]), np.array([[1.0, 0, 0, 0]]), np.zeros(1),
+                      np.array([[0.0], [5.0]]), np.array([0.25, 0.0]))
+    assert np.allclose(z, [0.25, 0.0])
