@@ -280,6 +280,65 @@ DECOMOE_API int decomoe_drop_visual_block(const void* src, void* dst, int64_t ro
                               int64_t v0, int64_t nv, int64_t nbatch, int64_t src_batch_stride,
                               int64_t dst_batch_stride, decomoe_stream_t stream);
 
+/* ------------------------------------------------------------------------
+ * SAVB exit gate (Section 3.2, Eqs. 2-3), evaluated at the candidate layers
+ * {3, 7, ..., 47} (zero-based, Appendix) on the hidden state h [T, d]:
+ *   text rows = rows outside the visual block [v0, v0+nv), in order (n of
+ *   them, n >= 1); x = [mean of text rows 0..n-2 ; text row n-1] (fp32 sums
+ *   in a fixed order; the pooled half is 0 when n == 1);
+ *   z = W2 relu(W1 x + b1) + b2 (hidden width H; ReLU is this library's
+ *   reading, the paper does not name the activation);
+ *   p_exit = softmax(z)_1, exit = [p_exit >= theta].
+ * h: dtype (DECOMOE_BF16 or DECOMOE_F32), d a multiple of 64, 16-byte
+ * aligned. w1 [H, 2d], b1 [H], w2 [2, H], b2 [2]: fp32 device arrays (w1
+ * 16-byte aligned). p_exit, exit_flag: one fp32 / int32 on the device.
+ * ws: decomoe_savb_gate_workspace_bytes(d, H) bytes, 16-byte aligned; it
+ * need not start at zero. Two launches; no host synchronisation (the caller
+ * reads exit_flag to decide whether to remove the visual block before the
+ * next layer, which changes the shapes of every later launch).
+ * ------------------------------------------------------------------------ */
+DECOMOE_API size_t decomoe_savb_gate_workspace_bytes(int d, int H);
+DECOMOE_API int decomoe_savb_gate(const void* h, int64_t T, int d, int dtype, int64_t v0, int64_t nv,
+                                  const float* w1, const float* b1, const float* w2, const float* b2, int H,
+                                  float theta, float* p_exit, int32_t* exit_flag, void* ws, size_t ws_bytes,
+                                  decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Offline RCEP calibration (Section 3.3, Eqs. 8-9; Algorithm 1).
+ *
+ * decomoe_calib_case_mass: one calibration case at one layer. logits [T, ld]
+ * fp32 are the router logits of the case's sequence; its text tokens are the
+ * rows outside the visual block [v0, v0+nv) (n = T - nv >= 1). Adds the
+ * case's text-token routed mass of Eq. 9 to accum:
+ *   accum[e] += (1/n) * sum over text tokens of the renormalised full-pool
+ *               top-k weight of e
+ * (the same fp32 weights and fixed-order fp64 sums as the activated mass of
+ * decomoe_route_prefix, then one fp64 division; cases add in call order).
+ * accum: [E] fp64 on the device, zeroed by the caller before the first case.
+ * ws: decomoe_calib_workspace_bytes(T, E) bytes. Needs 1 <= k <= E <= 256.
+ *
+ * decomoe_mean_mass_order: Eq. 8. mean[e] = accum[e] / n_cases; pi[i] = the
+ * expert at new position i, by descending mean, equal means in ascending
+ * expert index. pi: [E] int32 on the device; mean_out: [E] fp64 or NULL. A
+ * NaN mean sets DECOMOE_ERR_BAD_INPUT in status_dev.
+ *
+ * decomoe_permute_experts: the one-time reorder of Algorithm 1's last loop:
+ * dst expert block i = src expert block pi[i], for a tensor stored as E
+ * consecutive blocks of bytes_per_expert bytes (router rows [E, d], the
+ * router bias [E], gate/up [E, 2m, d] in either layout, down [E, d, m]).
+ * Out of place (src and dst must not overlap). An index outside [0, E) sets
+ * DECOMOE_ERR_BAD_INPUT and leaves that block unwritten; pi must be a
+ * permutation for dst to hold every expert.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API size_t decomoe_calib_workspace_bytes(int64_t T, int E);
+DECOMOE_API int decomoe_calib_case_mass(const float* logits, int64_t T, int E, int64_t ld, int k, int64_t v0,
+                                        int64_t nv, double* accum, void* ws, size_t ws_bytes,
+                                        decomoe_stream_t stream);
+DECOMOE_API int decomoe_mean_mass_order(const double* accum, int E, int n_cases, int32_t* pi, double* mean_out,
+                                        int32_t* status_dev, decomoe_stream_t stream);
+DECOMOE_API int decomoe_permute_experts(const void* src, void* dst, const int32_t* pi, int E,
+                                        int64_t bytes_per_expert, int32_t* status_dev, decomoe_stream_t stream);
+
 /* RMSNorm of the attention-free layer stack (a workload choice; the paper
  * leaves norms out of the method): y[t] = x[t] / sqrt(mean(x[t]^2) + eps),
  * fp32 math, dtype in and out. y may alias x. */

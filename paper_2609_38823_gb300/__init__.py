@@ -50,6 +50,12 @@ SIGNATURES = {
     "decomoe_select_prefix_device": (_I, [_P, _I, _I, _D, _P, _P]),
     "decomoe_route_prefix_dk": (_I, [_P, _L, _I, _L, _P, _I, _P, _P, _P]),
     "decomoe_dispatch_workspace_bytes": (_S, [_L, _I, _I]),
+    "decomoe_savb_gate_workspace_bytes": (_S, [_I, _I]),
+    "decomoe_savb_gate": (_I, [_P, _L, _I, _I, _L, _L, _P, _P, _P, _P, _I, _F, _P, _P, _P, _S, _P]),
+    "decomoe_calib_workspace_bytes": (_S, [_L, _I]),
+    "decomoe_calib_case_mass": (_I, [_P, _L, _I, _L, _I, _L, _L, _P, _P, _S, _P]),
+    "decomoe_mean_mass_order": (_I, [_P, _I, _I, _P, _P, _P, _P]),
+    "decomoe_permute_experts": (_I, [_P, _P, _P, _I, _L, _P, _P]),
     "decomoe_dispatch": (_I, [_P, _L, _I, _I, _P, _I, _I, _P, _P, _P, _P, _P, _P, _S, _P, _P]),
     "decomoe_dispatch_noalloc": (_I, [_P, _L, _I, _I, _P, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
     "decomoe_weight_layout": (_I, [_P, _P, _P, _I, _I, _I, _I, _P]),
@@ -241,6 +247,57 @@ def decomoe_dispatch_noalloc(topk_idx, K, x, counts, offsets, perm_token, inv_sl
            lib().decomoe_dispatch_noalloc(_ptr(topk_idx), T, k, K, _ptr(x), d, dtype, _ptr(counts), _ptr(offsets),
                                           _ptr(perm_token), _ptr(inv_slot), _ptr(x_perm), _ptr(status),
                                           _stream(stream)))
+
+
+# ----------------------------------------------------------------- SAVB gate and RCEP calibration
+
+def decomoe_savb_gate_workspace_bytes(d, H):
+    return int(lib().decomoe_savb_gate_workspace_bytes(d, H))
+
+
+def decomoe_savb_gate(h, v0, nv, w1, b1, w2, b2, theta, p_exit, exit_flag, ws, stream=None):
+    """SAVB exit gate on hidden h [T, d] (Eqs. 2-3); writes p_exit [1] fp32 and
+    exit_flag [1] int32 on the device."""
+    _need_cuda(h, w1, b1, w2, b2, p_exit, exit_flag, ws)
+    T, d = h.shape
+    H = w1.shape[0]
+    _check("decomoe_savb_gate",
+           lib().decomoe_savb_gate(_ptr(h), T, d, _dt(h), v0, nv, _ptr(w1), _ptr(b1), _ptr(w2), _ptr(b2), H,
+                                   float(theta), _ptr(p_exit), _ptr(exit_flag), _ptr(ws),
+                                   ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def decomoe_calib_workspace_bytes(T, E):
+    return int(lib().decomoe_calib_workspace_bytes(T, E))
+
+
+def decomoe_calib_case_mass(logits, k, v0, nv, accum, ws, E=None, stream=None):
+    """accum [E] fp64 += the case's text-token routed mass (Eq. 9)."""
+    _need_cuda(logits, accum, ws)
+    T, ld = logits.shape
+    E = ld if E is None else E
+    _check("decomoe_calib_case_mass",
+           lib().decomoe_calib_case_mass(_ptr(logits), T, E, ld, k, v0, nv, _ptr(accum), _ptr(ws),
+                                         ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def decomoe_mean_mass_order(accum, n_cases, pi, mean_out=None, status=None, stream=None):
+    """Eq. 8: pi [E] int32 = experts by descending case-mean routed mass."""
+    _need_cuda(accum, pi, mean_out, status)
+    _check("decomoe_mean_mass_order",
+           lib().decomoe_mean_mass_order(_ptr(accum), accum.shape[0], n_cases, _ptr(pi), _ptr(mean_out),
+                                         _ptr(status), _stream(stream)))
+
+
+def decomoe_permute_experts(src, dst, pi, status=None, stream=None):
+    """dst[i] = src[pi[i]] over the leading (expert) dimension, out of place."""
+    _need_cuda(src, dst, pi, status)
+    E = src.shape[0]
+    if dst.shape != src.shape or dst.dtype != src.dtype or pi.shape[0] != E:
+        raise ValueError("src, dst and pi must agree in shape")
+    _check("decomoe_permute_experts",
+           lib().decomoe_permute_experts(_ptr(src), _ptr(dst), _ptr(pi), E, src[0].numel() * src.element_size()
+                                         if E > 0 else 0, _ptr(status), _stream(stream)))
 
 
 def decomoe_weight_layout(w_gate, w_up, w_gate_up, stream=None):

@@ -67,6 +67,8 @@ int sm_count();  // cached per device
 int launch_router_tc(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E,
                      float* logits, int32_t* status, cudaStream_t s);
 bool router_tc_supported(int d, int E);
+int launch_skip_mass(const float* logits, int64_t n, int E, int64_t ld, int k, int64_t skip_at, int64_t skip_len,
+                     double* part, double* mass, cudaStream_t s);
 
 // ---------------------------------------------------------------- device side
 

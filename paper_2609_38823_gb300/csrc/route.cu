@@ -2,6 +2,7 @@
 // activated-mass reduction of RCEP (DecoMoE Section 3.3, Eqs. 10-12,
 // Algorithm 2).
 #include <cfloat>
+#include <cstdint>
 
 #include "decomoe_internal.cuh"
 
@@ -109,7 +110,7 @@ __device__ __forceinline__ float pick_weight(float my_v, int lane, int k) {
 __global__ void __launch_bounds__(ROUTE_THREADS)
     k_route(const float* __restrict__ logits, int64_t Tn, int E, int64_t ld, int K, int k,
             int32_t* __restrict__ idx_out, float* __restrict__ w_out, double* __restrict__ part,
-            const int32_t* __restrict__ K_dev) {
+            const int32_t* __restrict__ K_dev, int64_t skip_at = INT64_MAX, int64_t skip_len = 0) {
   if (K_dev != nullptr) K = *K_dev;  // prefix chosen on the device (k <= K <= E by construction)
   __shared__ int s_idx[ROUTE_TPB][DECOMOE_MAX_TOPK];
   __shared__ float s_w[ROUTE_TPB][DECOMOE_MAX_TOPK];
@@ -117,7 +118,9 @@ __global__ void __launch_bounds__(ROUTE_THREADS)
   const int64_t t = static_cast<int64_t>(blockIdx.x) * ROUTE_TPB + warp;
   const bool mass = part != nullptr;
   if (t < Tn) {
-    const float* row = logits + t * ld;
+    // token t reads logit row t, or t + skip_len from skip_at on (the text
+    // tokens around a removed visual block)
+    const float* row = logits + (t < skip_at ? t : t + skip_len) * ld;
     const int lim = mass ? E : K;
     uint32_t v[8];  // order-preserving keys of the row's logits
 #pragma unroll
@@ -201,6 +204,20 @@ __global__ void k_select_prefix(const double* __restrict__ mass, int E, int k, d
     K = K_hat > k ? K_hat : k;
   }
   *K_dev = K;
+}
+
+// Activated mass (Eq. 11) over n tokens whose logit rows skip a block:
+// token t reads row t, or t + skip_len from skip_at on. part needs
+// ceil(n / ROUTE_TPB) * E doubles.
+int launch_skip_mass(const float* logits, int64_t n, int E, int64_t ld, int k, int64_t skip_at, int64_t skip_len,
+                     double* part, double* mass, cudaStream_t s) {
+  const int64_t nblocks = (n + ROUTE_TPB - 1) / ROUTE_TPB;
+  k_route<<<static_cast<unsigned>(nblocks), ROUTE_THREADS, 0, s>>>(logits, n, E, ld, E, k, nullptr, nullptr, part,
+                                                                   nullptr, skip_at, skip_len);
+  DM_LAUNCH_CHECK("k_route");
+  k_mass_finalize<<<E, 256, 0, s>>>(part, static_cast<int>(nblocks), E, mass);
+  DM_LAUNCH_CHECK("k_mass_finalize");
+  return DECOMOE_OK;
 }
 
 }  // namespace decomoe

@@ -88,6 +88,15 @@ def test_argument_errors_are_caught_before_launch():
                                None, None, fake, 1 << 30, None, None) == 1
     msg = L.decomoe_last_error().decode()
     assert "K_fixed" in msg
+    # SAVB gate: d not a multiple of 64; no text rows
+    assert L.decomoe_savb_gate(fake, 10, 100, 0, 0, 0, fake, fake, fake, fake, 8, 0.5, fake, fake, fake, 1 << 20,
+                               None) == 1
+    assert L.decomoe_savb_gate(fake, 10, 64, 0, 0, 10, fake, fake, fake, fake, 8, 0.5, fake, fake, fake, 1 << 20,
+                               None) == 1
+    # calibration: a case without text tokens; overlapping permutation buffers
+    assert L.decomoe_calib_case_mass(fake, 8, 16, 16, 2, 0, 8, fake, fake, 1 << 20, None) == 1
+    assert L.decomoe_permute_experts(fake, ctypes.c_void_p(0x1000 + 64), fake, 4, 64, None, None) == 1
+    assert L.decomoe_mean_mass_order(fake, 300, 1, fake, None, None, None) == 1
     # too-small workspace
     assert L.decomoe_dispatch(fake, 4, 2, 4, None, 0, 0, fake, fake, fake, fake, None, fake, 1, None,
                               None) == dm.DECOMOE_ERR_WORKSPACE
