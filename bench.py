@@ -448,6 +448,7 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
     del graphs
     out += run_large(dm, ws, pk, n)
     out += run_stack(dm, ws, pk)
+    out += run_calib_gate(dm, ws, pk)
     # decode-size layers, K=64: weight streaming, reported against HBM
     for Td in W.DECODE_T:
         Bd = Buffers(wl, Td, B.out.device, dm)
@@ -528,7 +529,7 @@ def run_stack(dm, ws, pk):
     layers 0..19 at K=128 on 1552 rows, visual block removed from hidden and
     both 48-layer KV caches at layer 20, layers 20..47 on 272 rows with K_l
     drawn from 32..96. One pass = one graph replay."""
-    from paper_2609_38823_gb300.stack import Stack, StackLayer
+    from paper_2609_38823_gb300.stack import SavbGate, Stack, StackLayer
 
     wl = W.STACK
     dev = torch.device("cuda")
@@ -551,7 +552,73 @@ def run_stack(dm, ws, pk):
     res = [{"mode": "stack48", "pass_ms": round(ms_pass, 3), "tokens_per_s": round(wl.T / (ms_pass * 1e-3), 1),
             "useful_tflops": round(fl / (ms_pass * 1e-3) / 1e12, 2), "exit_layer": wl.exit_layer,
             "K_after_exit_mean": round(statistics.mean(K_sched[wl.exit_layer:]), 2)}]
-    del gr, st, layers, kv, kv_out
+    del gr
+    # Algorithm 2 with the SAVB gate at candidates 3, 7, ..., 19 (synthetic
+    # gate parameters that fire at 19, so layer 20 is the first text-only
+    # layer), eager launches with one 4-byte decision read per candidate;
+    # beside it the same fixed-exit stack, eager, for the gate's cost
+    gate = SavbGate(W.make_gate_params(wl.d, 512, [c for c in range(3, wl.layers, 4)], fire_at=wl.exit_layer - 1,
+                                       device=dev), theta=0.5)
+    variants = [("stack48 eager, fixed exit", st),
+                ("stack48 eager, SAVB gate", Stack(layers, K_sched, wl.k, None, wl.v0, wl.nv, wl.T, gate=gate)),
+                ("stack48 eager, SAVB gate + mass-selected K (p=0.7, on device)",
+                 Stack(layers, K_sched, wl.k, None, wl.v0, wl.nv, wl.T, gate=gate, p_after_exit=0.7))]
+    for name, sv in variants:
+        ms, _ = timed(lambda i, ev, sv=sv: sv.forward(h0, kv, kv_out), 3, 1, ws)
+        res.append({"mode": name, "pass_ms": round(ms / 3, 3), "tokens_per_s": round(wl.T / (ms / 3 * 1e-3), 1),
+                    "exit_layer": sv.exit_taken})
+    del st, variants, layers, kv, kv_out
+    torch.cuda.empty_cache()
+    return res
+
+
+def run_calib_gate(dm, ws, pk):
+    """Offline Mean-Mass calibration of one prefill-size layer (Eqs. 8-9): the
+    routed mass of one case (1552 rows, 272 text), the order, and the one-time
+    reorder of the layer's four tensors (1.21 GB read + written); and the SAVB
+    gate on the stack's and the large prefill's sequences."""
+    dev = torch.device("cuda")
+    wl = W.PREFILL
+    E, d, m, k = wl.E, wl.d, wl.m, wl.k
+    res = []
+    logits = W.make_logits(1552, E, std=0.9, bias=None, seed=0, wid=7).to(dev)
+    cws = dm.workspace(dm.decomoe_calib_workspace_bytes(1552, E), dev)
+    accum = torch.zeros(E, dtype=torch.float64, device=dev)
+    pi = torch.empty(E, dtype=torch.int32, device=dev)
+    g = dm.capture_graph(lambda: [dm.decomoe_calib_case_mass(logits, k, 16, 1280, accum, cws) for _ in range(20)])
+    ms, _ = timed(lambda i, ev: g.replay(), 5, 2, ws)
+    res.append({"mode": "calibration: text routed mass of one case (Eq. 9)", "rows": 1552, "text_rows": 272,
+                "us_per_case_layer": round(ms / 5 / 20 * 1e3, 2)})
+    g = dm.capture_graph(lambda: [dm.decomoe_mean_mass_order(accum, 8, pi) for _ in range(20)])
+    ms, _ = timed(lambda i, ev: g.replay(), 5, 2, ws)
+    res.append({"mode": "calibration: Mean-Mass order (Eq. 8)", "E": E, "us": round(ms / 5 / 20 * 1e3, 2)})
+    L = W.make_layer(wl, device=dev, with_x=False)
+    tensors = [L["w_r"], L["bias"], dm.fuse_gate_up(L["w_gate"], L["w_up"]), L["w_down"]]
+    del L
+    outs = [torch.empty_like(t) for t in tensors]
+    pi.copy_(torch.randperm(E, device=dev).to(torch.int32))
+    nbytes = sum(t.numel() * t.element_size() for t in tensors)
+
+    def reorder(i, ev):
+        for a, b in zip(tensors, outs):
+            dm.decomoe_permute_experts(a, b, pi)
+
+    ms, _ = timed(reorder, 5, 2, ws)
+    res.append({"mode": "calibration: reorder one layer (4 tensors)", "bytes_moved": 2 * nbytes,
+                "ms": round(ms / 5, 4), "gbs": round(2 * nbytes / (ms / 5 * 1e-3) / 1e9, 1),
+                "hbm_frac": round(2 * nbytes / (ms / 5 * 1e-3) / 1e9 / pk["hbm_gbs"], 4)})
+    del tensors, outs
+    for T, v0, nv in ((1552, 16, 1280), (16384, 0, 14336)):
+        h = W.make_x(W.with_(wl, T=T), device=dev)
+        prm = W.make_gate_params(d, 512, [19], fire_at=19, device=dev)[19]
+        p = torch.empty(1, dtype=torch.float32, device=dev)
+        ex = torch.empty(1, dtype=torch.int32, device=dev)
+        gws = dm.workspace(dm.decomoe_savb_gate_workspace_bytes(d, 512), dev)
+        g = dm.capture_graph(lambda: [dm.decomoe_savb_gate(h, v0, nv, *prm, 0.5, p, ex, gws) for _ in range(20)])
+        ms, _ = timed(lambda i, ev: g.replay(), 5, 2, ws)
+        res.append({"mode": "SAVB gate (Eqs. 2-3)", "T": T, "text_rows": T - nv, "hidden": 512,
+                    "us": round(ms / 5 / 20 * 1e3, 2)})
+        del h
     torch.cuda.empty_cache()
     return res
 

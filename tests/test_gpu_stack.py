@@ -15,7 +15,7 @@ import paper_2609_38823_gb300 as dm
 import workloads as W
 from oracle import decomoe_oracle as O
 from paper_2609_38823_gb300.stack import Stack, StackLayer
-from tests.helpers import assert_close_out, bf16_round, f64
+from tests.helpers import MASS_P_BAND, assert_close_out, bf16_round, f64
 
 pytestmark = pytest.mark.gpu
 DEV = torch.device("cuda")
@@ -151,3 +151,85 @@ def test_large_T16384_layer_sampled_and_compaction(K, zipf):
                       k=wl.k, K=K)
     assert_close_out(f64(out[torch.from_numpy(sample).to(DEV)])[keep], ref["out"][keep], 5e-3, 2e-2,
                      "T=16384 layer output")
+
+
+def _gate_dev(wl, candidates, fire_at, H=64, seed=0):
+    from paper_2609_38823_gb300.stack import SavbGate
+
+    prm = W.make_gate_params(wl.d, H, candidates, fire_at, seed=seed, device="cuda")
+    return SavbGate(prm, theta=0.5), prm
+
+
+def test_gate_driven_exit_equals_fixed_exit_and_gate_parity():
+    """Algorithm 2 with the SAVB gate: candidates 1 and 3; the synthetic gate
+    fires at 3, so the visual block leaves before layer 4. The output and the
+    compacted KV equal the fixed-exit stack's bit for bit, and the gate's
+    p_exit at each candidate matches the oracle gate on that layer's output."""
+    wl = W.with_(W.TINY, layers=6)
+    L, _ = _layers(wl, 6, "cpu")
+    K_sched = [16, 16, 16, 16, 10, 6]
+    h0 = W.make_x(wl).to(DEV)
+    gate, prm = _gate_dev(wl, [1, 3], fire_at=3)
+    kvs = [torch.randn(6, wl.T, 64, generator=torch.Generator().manual_seed(s)).to(DEV) for s in (1, 2)]
+    outs = []
+    for kind in ("gate", "fixed"):
+        kv_out = [torch.empty(6, wl.T - wl.nv, 64, device=DEV) for _ in range(2)]
+        if kind == "gate":
+            st = Stack(L, K_sched, wl.k, exit_layer=None, v0=wl.v0, nv=wl.nv, T=wl.T, gate=gate)
+        else:
+            st = Stack(L, K_sched, wl.k, exit_layer=4, v0=wl.v0, nv=wl.nv, T=wl.T)
+        out = st.forward(h0, kvs, kv_out).clone()
+        torch.cuda.synchronize()
+        assert dm.decomoe_read_status(st.status) == 0
+        assert st.exit_taken == 4
+        outs.append((out, [t.clone() for t in kv_out], st))
+    assert torch.equal(outs[0][0], outs[1][0])
+    for a, b in zip(outs[0][1], outs[1][1]):
+        assert torch.equal(a, b)
+    gst = outs[0][2]
+    assert gst.exit_flag.cpu().tolist()[1] == 0 and gst.exit_flag.cpu().tolist()[3] == 1
+    # teacher-forced gate parity: hidden after layers 0..l from a window stack
+    for l in (1, 3):
+        win = Stack(L[:l + 1], K_sched[:l + 1], wl.k, exit_layer=None, v0=wl.v0, nv=wl.nv, T=wl.T)
+        hl = win.forward(h0)
+        torch.cuda.synchronize()
+        w1, b1, w2, b2 = (t.cpu().numpy() for t in prm[l])
+        p_ref = O.gate_exit_prob(O.gate_logits(O.gate_feature(f64(hl), wl.v0, wl.nv), w1, b1, w2, b2))
+        assert abs(float(gst.p_exit[l]) - p_ref) <= 2e-5
+
+
+def test_mass_selected_prefix_after_exit_device_equals_host():
+    """After the exit, each layer's prefix is selected from its activated mass
+    (Eq. 12 with p); the device selection gives the same output bits as the
+    host selection, and the first post-exit layer matches the oracle run with
+    the oracle's own K."""
+    wl = W.with_(W.TINY, layers=5)
+    L, R = _layers(wl, 5, "cpu")
+    K_sched = [16] * 5
+    h0 = W.make_x(wl).to(DEV)
+    res = []
+    for host in (False, True):
+        st = Stack(L, K_sched, wl.k, exit_layer=2, v0=wl.v0, nv=wl.nv, T=wl.T, p_after_exit=0.7,
+                   select_on_host=host)
+        res.append(st.forward(h0).clone())
+        torch.cuda.synchronize()
+        assert dm.decomoe_read_status(st.status) == 0
+    assert torch.equal(res[0], res[1])
+    # layer 2 (first text-only layer) from the GPU's own input, K by the oracle
+    pre = Stack(L[:2], K_sched[:2], wl.k, exit_layer=None, v0=wl.v0, nv=wl.nv, T=wl.T)
+    h2 = O.drop_visual_block(f64(pre.forward(h0)), wl.v0, wl.nv)
+    # already text-only (nv = 0): the mass-selected branch from its first layer
+    one = Stack(L[2:3], [16], wl.k, exit_layer=0, v0=0, nv=0, T=h2.shape[0], p_after_exit=0.7)
+    got = one.forward(torch.from_numpy(h2).to(DEV, torch.float32))
+    torch.cuda.synchronize()
+    xn = O.rmsnorm(h2)
+    a = O.router_logits(xn, R[2]["w_r"], R[2]["bias"]).astype(np.float64)
+    s_ref = O.activated_mass(a, wl.k)
+    cum = np.cumsum(s_ref) / s_ref.sum()
+    if np.abs(cum - 0.7).min() < MASS_P_BAND:
+        pytest.skip("mass ratio within rounding of p: K is reported, not compared")
+    K = O.select_prefix(s_ref, 0.7, wl.k)
+    keep = O.prefix_margin(a, K, wl.k) > 1e-4
+    ref = O.moe_layer(xn, R[2]["w_r"], R[2]["bias"], R[2]["w_gate"], R[2]["w_up"], R[2]["w_down"], k=wl.k,
+                      K=K)["out"] + h2
+    assert_close_out(f64(got)[keep], ref[keep], 1e-4, 1e-4, "mass-selected layer")

@@ -195,3 +195,22 @@ def stack_K_schedule(wl: Workload, seed: int = 0) -> List[int]:
 def large_K(fraction: float, E: int = 128) -> int:
     """Prefix length for a retained fraction f of the pool: ceil(f*E) (0.3*128 -> 39)."""
     return int(math.ceil(fraction * E - 1e-9))
+
+
+def make_gate_params(d: int, H: int, candidates, fire_at: Optional[int], seed: int = 0, device="cpu",
+                     margin: float = 8.0):
+    """Synthetic SAVB gate parameters for each candidate layer (the trained
+    checkpoint is not available): W1 ~ N(0, 1/(2d)), b1 ~ N(0, 0.1),
+    W2 ~ N(0, 1/H), and an output bias b2 = (+margin, -margin) at every
+    candidate except ``fire_at``, where it is (-margin, +margin), so the gate
+    computes its full MLP everywhere and fires at that candidate.
+    Returns {layer: (w1 [H, 2d], b1 [H], w2 [2, H], b2 [2])} fp32."""
+    out = {}
+    for l in candidates:
+        g = _gen("cpu", stream(seed, 90, l, 0))
+        w1 = torch.randn(H, 2 * d, generator=g) / (2 * d) ** 0.5
+        b1 = torch.randn(H, generator=g) * 0.1
+        w2 = torch.randn(2, H, generator=g) / H ** 0.5
+        b2 = torch.tensor([-margin, margin] if l == fire_at else [margin, -margin])
+        out[l] = tuple(t.to(device=device, dtype=torch.float32).contiguous() for t in (w1, b1, w2, b2))
+    return out
