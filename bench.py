@@ -463,13 +463,16 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
             lv.x, lv.w_r, lv.bias, lv.w_gu, lv.w_down = xs[i % len(xs)], L.w_r, L.bias, L.w_gu, L.w_down
             run_step(dm, wl, lv, Bd, 64, 0, 0, None, ev)
 
-        ms, evs = timed(dec_step, n, 5, ws)
-        ffn = statistics.mean(e[0].elapsed_time(e[2]) for e in evs)
+        ms, _ = timed(dec_step, n, 5, ws)
         D = int((Bd.counts[:64] > 0).sum())
         wbytes = D * 3 * wl.m * wl.d * 2
         step_bytes = wbytes + wl.E * wl.d * 2 + Td * wl.d * 2 * (2 + 3 * wl.k)
-        graphs = [dm.capture_graph(lambda i=i: dec_step(i, None)) for i in range(len(layers))]
+        # graph replay (no host launch gaps); events captured in each graph
+        # bracket its two expert GEMMs
+        gevs = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(3)] for _ in layers]
+        graphs = [dm.capture_graph(lambda i=i: dec_step(i, gevs[i])) for i in range(len(layers))]
         msg, _ = timed(lambda i, ev: graphs[i % len(graphs)].replay(), n, 5, ws)
+        ffn = statistics.mean(e[0].elapsed_time(e[2]) for e in gevs)
         out.append({"mode": "decode", "T": Td, "K": 64, "active_experts": D,
                     "tokens_per_s": round(Td * n / (ms / 1e3), 1), "ms_per_step": round(ms / n, 4),
                     "graph_tokens_per_s": round(Td * n / (msg / 1e3), 1), "graph_ms_per_step": round(msg / n, 4),

@@ -9,14 +9,16 @@
 //   warp 1      TMEM allocator and MMA issuer: one thread issues
 //               tcgen05.mma.cta_group::1.kind::f16 (M=128, N=BN, K=16) into a
 //               double-buffered fp32 accumulator in tensor memory.
-//   warps 2..5  epilogue: tcgen05.ld of the accumulator (one TMEM lane
-//               quarter per warp, one row per thread), fused SwiGLU / bf16 /
+//   warps 2..   epilogue (EW warps, 8 by default: two per TMEM lane
+//               quarter, each on half of the tile's columns): tcgen05.ld of
+//               the accumulator, one row per thread, fused SwiGLU / bf16 /
 //               fp32+bias conversion, stores to global.
 // Tiles: for every group (expert) g, ceil(rows_g / 128) M-tiles times
 // N / BN N-tiles; see tile_coords for the order. Rows past the group's end are
 // computed on whatever TMA loaded (zeros past the tensor end) and never
 // stored.
-// bf16, few rows (decode): weight-streaming CUDA-core kernels.
+// bf16, few rows per expert (decode): the weights-stationary tcgen05 kernel
+// k_moe_ws (expert weights as M, the expert's tokens as N).
 // f32: CUDA-core kernels (exact fp32 products, fp32 accumulation).
 #include <mutex>
 
@@ -30,9 +32,6 @@
 // otherwise (prefill: faster when many rows share an expert's weights).
 #ifndef DECOMOE_WS_MAX_AVG_ROWS
 #define DECOMOE_WS_MAX_AVG_ROWS 8
-#endif
-#ifndef DECOMOE_DECODE_ROWS
-#define DECOMOE_DECODE_ROWS 0  // rows at or below which the CUDA-core decode kernels run
 #endif
 
 namespace decomoe {
@@ -686,10 +685,14 @@ struct WsArgs {
 #ifndef DECOMOE_WS_ORDER
 #define DECOMOE_WS_ORDER 0  // 0: weight block outer, token chunk inner; 1: chunk outer
 #endif
-constexpr int WS_BM = 128, WS_BK = 64, WS_BN = 256, WS_BOX = DECOMOE_WS_BOX;
+constexpr int WS_BM = 128, WS_BK = 64, WS_BOX = DECOMOE_WS_BOX;
 
-template <int STAGES, bool SWIGLU>
+// BN: token chunk (the MMA's N), one chunk per (expert, weight block) tile
+// when an expert has at most BN rows; smaller chunks leave shared memory for
+// a deeper weight-streaming ring.
+template <int STAGES, bool SWIGLU, int BN = 256>
 struct WsCfg {
+  static constexpr int WS_BN = BN;
   static constexpr int A_BYTES = WS_BM * WS_BK * 2;
   static constexpr int B_BYTES = WS_BN * WS_BK * 2;
   static constexpr int BOX_BYTES = WS_BOX * WS_BK * 2;
@@ -704,10 +707,20 @@ struct WsCfg {
                                  NBARS * 8 + 2 * (MAXG + 1) * 4 + 16;
 };
 
+// Most stages of a WsCfg<., SWIGLU, BN> that fit the shared-memory budget.
+template <bool SWIGLU, int BN>
+constexpr int ws_max_stages() {
+  constexpr size_t fixed = WsCfg<1, SWIGLU, BN>::SMEM - WsCfg<1, SWIGLU, BN>::STAGE_BYTES - 2 * 8;
+  constexpr size_t per = WsCfg<1, SWIGLU, BN>::STAGE_BYTES + 2 * 8;
+  constexpr int n = static_cast<int>((232448 - fixed) / per);
+  return n > 12 ? 12 : n;
+}
+
 struct WsTile {
   int g, wb, row0, ntok;
 };
 
+template <int WS_BN>
 __device__ __forceinline__ WsTile ws_tile(int t, int total, const int* s_tt, const int* s_off, int G, int nwb) {
   const int tp = (t & 1) ? (total - 1 - (t >> 1)) : (t >> 1);
   int lo = 0, hi = G - 1;
@@ -739,11 +752,12 @@ __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
-template <bool SWIGLU, int STAGES, bool GATHER_B = false>
+template <bool SWIGLU, int STAGES, bool GATHER_B = false, int BN = 256>
 __global__ void __launch_bounds__(192, 1)
     k_moe_ws(const __grid_constant__ CUtensorMap tma_w, const __grid_constant__ CUtensorMap tma_x,
              const WsArgs g) {
-  using C = WsCfg<STAGES, SWIGLU>;
+  using C = WsCfg<STAGES, SWIGLU, BN>;
+  constexpr int WS_BN = BN;
   __shared__ int s_brow[GATHER_B ? WS_BN : 1];
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -841,7 +855,7 @@ __global__ void __launch_bounds__(192, 1)
     bool ok = true;
     uint32_t armed = 0, armed_ph = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
-      const WsTile T = ws_tile(t, total, s_tt, s_off, G, nwb);
+      const WsTile T = ws_tile<WS_BN>(t, total, s_tt, s_off, G, nwb);
       const int wrow0 = T.g * g.wrows + T.wb * WS_BM;
       int nload;       // TMA copies for B per k-block
       uint32_t bytes;  // bytes landing per stage
@@ -897,7 +911,7 @@ __global__ void __launch_bounds__(192, 1)
     bool ok = true, issued = false;
     int it = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
-      const WsTile T = ws_tile(t, total, s_tt, s_off, G, nwb);
+      const WsTile T = ws_tile<WS_BN>(t, total, s_tt, s_off, G, nwb);
       const uint32_t idesc = idesc_bf16_f32(WS_BM, (T.ntok + 15) & ~15);
       const int acc = it & 1;
       const uint32_t aph = (it >> 1) & 1;
@@ -945,7 +959,7 @@ __global__ void __launch_bounds__(192, 1)
     int xpar = 0;
     bool ok = true;
     for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
-      const WsTile T = ws_tile(t, total, s_tt, s_off, G, nwb);
+      const WsTile T = ws_tile<WS_BN>(t, total, s_tt, s_off, G, nwb);
       const int acc = it & 1;
       const uint32_t aph = (it >> 1) & 1;
       if (!mbar_wait(TFULL_BAR(acc), aph, g.limit_ns, s_abort)) {
@@ -1024,11 +1038,12 @@ __global__ void __launch_bounds__(192, 1)
 // X: [rows, kdim] token rows grouped by expert, or with GATHER_B the source
 // tensor [x_tensor_rows, kdim] whose row b_rows[r] is token row r;
 // W: [G * wrows, kdim].
-template <bool SWIGLU, int STAGES, bool GATHER_B = false>
+template <bool SWIGLU, int STAGES, bool GATHER_B = false, int BN = 256>
 static int launch_ws(const void* X, int rows, int kdim, const void* W, int wrows, const int32_t* offsets, int G,
                      void* out, int64_t out_ld, int32_t* status, cudaStream_t s, const int32_t* b_rows = nullptr,
                      int64_t x_tensor_rows = 0) {
-  using C = WsCfg<STAGES, SWIGLU>;
+  using C = WsCfg<STAGES, SWIGLU, BN>;
+  constexpr int WS_BN = BN;
   CUtensorMap tw, tx;
   DM_RET(make_tmap_bf16(&tw, W, static_cast<uint64_t>(kdim), static_cast<uint64_t>(G) * wrows, WS_BM, WS_BK));
   if (GATHER_B)
@@ -1046,7 +1061,7 @@ static int launch_ws(const void* X, int rows, int kdim, const void* W, int wrows
   g.status = status;
   g.limit_ns = static_cast<uint64_t>(wait_limit_ns());
   g.b_rows = b_rows;
-  auto kern = k_moe_ws<SWIGLU, STAGES, GATHER_B>;
+  auto kern = k_moe_ws<SWIGLU, STAGES, GATHER_B, BN>;
   static_assert(C::SMEM <= 232448, "shared memory budget");
   DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(C::SMEM)));
   const int64_t ub_tiles = (static_cast<int64_t>(rows) / WS_BN + G) * (wrows / WS_BM);
@@ -1054,6 +1069,25 @@ static int launch_ws(const void* X, int rows, int kdim, const void* W, int wrows
   kern<<<grid, 192, C::SMEM, s>>>(tw, tx, g);
   DM_LAUNCH_CHECK("k_moe_ws");
   return DECOMOE_OK;
+}
+
+// Weights-stationary launch with the token chunk sized to the row count: an
+// expert never gets more rows than there are tokens, and rows = T * k with
+// k >= 1, so for rows <= 256 a 32-token chunk usually covers every expert in
+// one chunk (decode); smaller chunks buy a deeper weight-streaming ring.
+template <bool SWIGLU>
+static int launch_ws_auto(const void* X, int rows, int kdim, const void* W, int wrows, const int32_t* offsets,
+                          int G, void* out, int64_t out_ld, int32_t* status, cudaStream_t s) {
+  if (rows <= 256)
+    return launch_ws<SWIGLU, ws_max_stages<SWIGLU, 32>(), false, 32>(X, rows, kdim, W, wrows, offsets, G, out,
+                                                                     out_ld, status, s);
+  if (rows <= 512)
+    return launch_ws<SWIGLU, ws_max_stages<SWIGLU, 64>(), false, 64>(X, rows, kdim, W, wrows, offsets, G, out,
+                                                                     out_ld, status, s);
+  if (rows <= 1024)
+    return launch_ws<SWIGLU, ws_max_stages<SWIGLU, 128>(), false, 128>(X, rows, kdim, W, wrows, offsets, G, out,
+                                                                       out_ld, status, s);
+  return launch_ws<SWIGLU, 4, false, 256>(X, rows, kdim, W, wrows, offsets, G, out, out_ld, status, s);
 }
 
 bool router_tc_supported(int d, int E) { return d % 64 == 0 && (E == 128 || E == 256); }
@@ -1154,160 +1188,6 @@ __global__ void k_simt_down(const T* __restrict__ H, const int32_t* __restrict__
   }
 }
 
-// ------------------------------------------------------------------ decode path
-// Few rows per expert: stream each weight row once with 16-byte non-allocating
-// loads, dot it with the expert's (at most 8 at a time) activation rows held
-// in shared memory. One warp per output feature pair.
-constexpr int DEC_THREADS = 256;
-constexpr int DEC_FEAT_PER_BLOCK = 16;  // 8 warps x 2 features
-constexpr int DEC_NMAX = 8;
-
-__device__ __forceinline__ uint4 ldg_stream(const void* p) {
-  uint4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-               : "l"(p));
-  return v;
-}
-
-__device__ __forceinline__ float dot8(const uint4& w, const uint4& x) {
-  float s = bf16_lo(w.x) * bf16_lo(x.x);
-  s = fmaf(bf16_hi(w.x), bf16_hi(x.x), s);
-  s = fmaf(bf16_lo(w.y), bf16_lo(x.y), s);
-  s = fmaf(bf16_hi(w.y), bf16_hi(x.y), s);
-  s = fmaf(bf16_lo(w.z), bf16_lo(x.z), s);
-  s = fmaf(bf16_hi(w.z), bf16_hi(x.z), s);
-  s = fmaf(bf16_lo(w.w), bf16_lo(x.w), s);
-  s = fmaf(bf16_hi(w.w), bf16_hi(x.w), s);
-  return s;
-}
-
-// acc[i] += row(w) . xs[i] for i < NC; w rows of `vec` 16-byte vectors.
-template <int NC>
-__device__ __forceinline__ void dec_dot_rows(const uint4* __restrict__ w0, const uint4* __restrict__ w1,
-                                             const uint4* xs, int vec, int lane, float (&a0)[DEC_NMAX],
-                                             float (&a1)[DEC_NMAX]) {
-#pragma unroll
-  for (int i = 0; i < DEC_NMAX; ++i) a0[i] = a1[i] = 0.f;
-  int v = lane;
-  for (; v + 32 * 3 < vec; v += 32 * 4) {
-    uint4 p[4], q[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      p[u] = ldg_stream(w0 + v + 32 * u);
-      q[u] = ldg_stream(w1 + v + 32 * u);
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u)
-#pragma unroll
-      for (int i = 0; i < NC; ++i) {
-        const uint4 xv = xs[i * vec + v + 32 * u];
-        a0[i] += dot8(p[u], xv);
-        a1[i] += dot8(q[u], xv);
-      }
-  }
-  for (; v < vec; v += 32) {
-    const uint4 p = ldg_stream(w0 + v), q = ldg_stream(w1 + v);
-#pragma unroll
-    for (int i = 0; i < NC; ++i) {
-      const uint4 xv = xs[i * vec + v];
-      a0[i] += dot8(p, xv);
-      a1[i] += dot8(q, xv);
-    }
-  }
-#pragma unroll
-  for (int i = 0; i < NC; ++i)
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      a0[i] += __shfl_xor_sync(0xffffffffu, a0[i], off);
-      a1[i] += __shfl_xor_sync(0xffffffffu, a1[i], off);
-    }
-}
-
-// Gate/up for decode: block (feature block, expert). Each warp computes two
-// features f: gate row and up row of f together, h = silu(g) * u.
-__global__ void __launch_bounds__(DEC_THREADS)
-    k_dec_gate_up(const __nv_bfloat16* __restrict__ X, const int32_t* __restrict__ offsets,
-                  const __nv_bfloat16* __restrict__ Wgu, int d, int m, __nv_bfloat16* __restrict__ H) {
-  extern __shared__ uint4 xs[];  // [DEC_NMAX][d / 8]
-  const int e = blockIdx.y;
-  const int r0 = offsets[e];
-  const int n_e = offsets[e + 1] - r0;
-  if (n_e <= 0) return;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int vec = d / 8;
-  for (int c0 = 0; c0 < n_e; c0 += DEC_NMAX) {
-    const int nc = min(DEC_NMAX, n_e - c0);
-    __syncthreads();
-    for (int i = threadIdx.x; i < nc * vec; i += DEC_THREADS) {
-      const int rr = i / vec, v = i - rr * vec;
-      xs[rr * vec + v] = reinterpret_cast<const uint4*>(X + static_cast<int64_t>(r0 + c0 + rr) * d)[v];
-    }
-    __syncthreads();
-#pragma unroll 1
-    for (int ff = 0; ff < 2; ++ff) {
-      const int f = blockIdx.x * DEC_FEAT_PER_BLOCK + warp * 2 + ff;
-      if (f >= m) break;
-      const int blk = f / DECOMOE_GU_BLOCK, i = f % DECOMOE_GU_BLOCK;
-      const int64_t grow = static_cast<int64_t>(e) * 2 * m + blk * 2 * DECOMOE_GU_BLOCK + i;
-      const uint4* wg = reinterpret_cast<const uint4*>(Wgu + grow * d);
-      const uint4* wu = reinterpret_cast<const uint4*>(Wgu + (grow + DECOMOE_GU_BLOCK) * d);
-      float ag[DEC_NMAX], au[DEC_NMAX];
-      switch (nc) {
-        case 1: dec_dot_rows<1>(wg, wu, xs, vec, lane, ag, au); break;
-        case 2: dec_dot_rows<2>(wg, wu, xs, vec, lane, ag, au); break;
-        case 3: case 4: dec_dot_rows<4>(wg, wu, xs, vec, lane, ag, au); break;
-        default: dec_dot_rows<8>(wg, wu, xs, vec, lane, ag, au); break;
-      }
-#pragma unroll
-      for (int rr = 0; rr < DEC_NMAX; ++rr)
-        if (lane == rr && rr < nc)
-          H[static_cast<int64_t>(r0 + c0 + rr) * m + f] =
-              __float2bfloat16_rn(silu_f(ag[rr]) * au[rr]);
-    }
-  }
-}
-
-// Down projection for decode: block (output block, expert); each warp two
-// output features n, rows of W_down of m elements.
-__global__ void __launch_bounds__(DEC_THREADS)
-    k_dec_down(const __nv_bfloat16* __restrict__ H, const int32_t* __restrict__ offsets,
-               const __nv_bfloat16* __restrict__ Wd, int d, int m, __nv_bfloat16* __restrict__ Y) {
-  extern __shared__ uint4 hs[];  // [DEC_NMAX][m / 8]
-  const int e = blockIdx.y;
-  const int r0 = offsets[e];
-  const int n_e = offsets[e + 1] - r0;
-  if (n_e <= 0) return;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int vec = m / 8;
-  for (int c0 = 0; c0 < n_e; c0 += DEC_NMAX) {
-    const int nc = min(DEC_NMAX, n_e - c0);
-    __syncthreads();
-    for (int i = threadIdx.x; i < nc * vec; i += DEC_THREADS) {
-      const int rr = i / vec, v = i - rr * vec;
-      hs[rr * vec + v] = reinterpret_cast<const uint4*>(H + static_cast<int64_t>(r0 + c0 + rr) * m)[v];
-    }
-    __syncthreads();
-    const int n0 = blockIdx.x * DEC_FEAT_PER_BLOCK + warp * 2;
-    if (n0 >= d) continue;
-    const uint4* w0 = reinterpret_cast<const uint4*>(Wd + (static_cast<int64_t>(e) * d + n0) * m);
-    const uint4* w1 = reinterpret_cast<const uint4*>(Wd + (static_cast<int64_t>(e) * d + n0 + 1) * m);
-    float a0[DEC_NMAX], a1[DEC_NMAX];
-    switch (nc) {
-      case 1: dec_dot_rows<1>(w0, w1, hs, vec, lane, a0, a1); break;
-      case 2: dec_dot_rows<2>(w0, w1, hs, vec, lane, a0, a1); break;
-      case 3: case 4: dec_dot_rows<4>(w0, w1, hs, vec, lane, a0, a1); break;
-      default: dec_dot_rows<8>(w0, w1, hs, vec, lane, a0, a1); break;
-    }
-#pragma unroll
-    for (int rr = 0; rr < DEC_NMAX; ++rr)
-      if (lane == rr && rr < nc) {
-        __nv_bfloat162 o = __floats2bfloat162_rn(a0[rr], a1[rr]);
-        *reinterpret_cast<__nv_bfloat162*>(Y + static_cast<int64_t>(r0 + c0 + rr) * d + n0) = o;
-      }
-  }
-}
-
 // ------------------------------------------------------------------ weight layout
 __global__ void k_weight_layout(const uint4* __restrict__ wg, const uint4* __restrict__ wu,
                                 uint4* __restrict__ wgu, int E, int m, int vec) {
@@ -1368,8 +1248,6 @@ static int expert_check(const char* name, const void* a, const int32_t* offsets,
   return DECOMOE_OK;
 }
 
-static bool use_decode_path(int64_t rows) { return rows <= DECOMOE_DECODE_ROWS; }
-
 // Pipeline shape of the two expert GEMMs: k-block depth (64 -> 128-byte
 // swizzle, 32 -> 64-byte swizzle) and the number of shared-memory stages.
 #ifndef DECOMOE_GU_BK
@@ -1423,19 +1301,8 @@ int decomoe_expert_gate_up(const void* x_perm, const int32_t* offsets, int64_t r
     DM_LAUNCH_CHECK("k_simt_gate_up");
     return DECOMOE_OK;
   }
-  if (use_decode_path(rows)) {
-    const size_t sm1 = static_cast<size_t>(DEC_NMAX) * d * 2;
-    DM_ARG_CHECK(sm1 <= 200 * 1024, "expert_gate_up: d too large for the decode path");
-    DM_CUDA_CHECK(cudaFuncSetAttribute(k_dec_gate_up, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm1));
-    dim3 g1((m + DEC_FEAT_PER_BLOCK - 1) / DEC_FEAT_PER_BLOCK, K);
-    k_dec_gate_up<<<g1, DEC_THREADS, sm1, s>>>(static_cast<const __nv_bfloat16*>(x_perm), offsets,
-                                               static_cast<const __nv_bfloat16*>(w_gate_up), d, m,
-                                               static_cast<__nv_bfloat16*>(h));
-    DM_LAUNCH_CHECK("k_dec_gate_up");
-    return DECOMOE_OK;
-  }
   if (static_cast<int64_t>(R) <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K)
-    return launch_ws<true, 4>(x_perm, R, d, w_gate_up, 2 * m, offsets, K, h, m, status_dev, s);
+    return launch_ws_auto<true>(x_perm, R, d, w_gate_up, 2 * m, offsets, K, h, m, status_dev, s);
   // A = x_perm [R, d], B = w_gate_up [K*2m, d] (only experts < K are read)
   return launch_tc<256, EPI_SWIGLU, GU_STAGES, GU_BK, false, GU_MP, GU_EW, GU_OCC>(
       x_perm, R, d, w_gate_up, static_cast<int64_t>(K) * 2 * m, offsets, K, 2 * m, h, m, nullptr, status_dev, s, 0,
@@ -1457,19 +1324,8 @@ int decomoe_expert_down(const void* h, const int32_t* offsets, int64_t rows, int
     DM_LAUNCH_CHECK("k_simt_down");
     return DECOMOE_OK;
   }
-  if (use_decode_path(rows)) {
-    const size_t sm2 = static_cast<size_t>(DEC_NMAX) * m * 2;
-    DM_ARG_CHECK(sm2 <= 200 * 1024, "expert_down: m too large for the decode path");
-    DM_CUDA_CHECK(cudaFuncSetAttribute(k_dec_down, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2));
-    dim3 g2((d + DEC_FEAT_PER_BLOCK - 1) / DEC_FEAT_PER_BLOCK, K);
-    k_dec_down<<<g2, DEC_THREADS, sm2, s>>>(static_cast<const __nv_bfloat16*>(h), offsets,
-                                            static_cast<const __nv_bfloat16*>(w_down), d, m,
-                                            static_cast<__nv_bfloat16*>(y_perm));
-    DM_LAUNCH_CHECK("k_dec_down");
-    return DECOMOE_OK;
-  }
   if (static_cast<int64_t>(R) <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K)
-    return launch_ws<false, 4>(h, R, m, w_down, d, offsets, K, y_perm, d, status_dev, s);
+    return launch_ws_auto<false>(h, R, m, w_down, d, offsets, K, y_perm, d, status_dev, s);
   // A = h [R, m], B = w_down [K*d, m]
   return launch_tc<256, EPI_BF16, DN_STAGES, DN_BK, false, DN_MP, DN_EW, DN_OCC>(h, R, m, w_down, static_cast<int64_t>(K) * d, offsets,
                                                                   K, d, y_perm, d, nullptr, status_dev, s, 0,
