@@ -47,6 +47,8 @@ def parse():
     ap.add_argument("--layers", type=int, default=8)
     ap.add_argument("--p", type=float, default=0.7)
     ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--only-decode", type=int, default=0, metavar="T",
+                    help="run only the decode layer at T tokens (K=64) for --steps graph replays (profiling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     return ap.parse_args()
@@ -626,6 +628,35 @@ def run_calib_gate(dm, ws, pk):
     return res
 
 
+def only_decode(args, local):
+    """The decode-size layer alone (T = --only-decode tokens, K = 64), one
+    CUDA graph per rotated layer, replayed --steps times after --warmup."""
+    import paper_2609_38823_gb300 as dm
+
+    dm.lib()
+    dev = torch.device("cuda", local)
+    wl = W.PREFILL
+    Td = args.only_decode
+    layers = [Layer(wl, l, dev, dm) for l in range(args.layers)]
+    Bd = Buffers(wl, Td, dev, dm)
+    xs = [W.make_x(W.DECODE, T=Td, layer=l, device=dev) for l in range(len(layers))]
+
+    class LV:
+        pass
+
+    def dec_step(i):
+        L = layers[i % len(layers)]
+        lv = LV()
+        lv.x, lv.w_r, lv.bias, lv.w_gu, lv.w_down = xs[i % len(xs)], L.w_r, L.bias, L.w_gu, L.w_down
+        run_step(dm, wl, lv, Bd, 64, 0, 0, None, None)
+
+    graphs = [dm.capture_graph(lambda i=i: dec_step(i)) for i in range(len(layers))]
+    ms, _ = timed(lambda i, ev: graphs[i % len(graphs)].replay(), args.steps, args.warmup, 1)
+    if dm.decomoe_read_status(Bd.status) != 0:
+        raise RuntimeError("device status set during the decode run")
+    return {"mode": "decode only", "T": Td, "K": 64, "steps": args.steps, "ms_per_step": round(ms / args.steps, 4)}
+
+
 def _kernel_hash():
     import hashlib
 
@@ -718,6 +749,11 @@ def main():
     if args.impl == "reference":
         line = reference(args, ws, rank)
         if line is not None:
+            print(json.dumps(line), flush=True)
+        return
+    if args.only_decode:
+        line = only_decode(args, local)
+        if rank == 0:
             print(json.dumps(line), flush=True)
         return
     line = ours(args, ws, rank, local)
