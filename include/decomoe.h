@@ -157,6 +157,31 @@ DECOMOE_API int decomoe_dispatch(const int32_t* topk_idx, int64_t T, int k, int 
                      int32_t* status_dev, decomoe_stream_t stream);
 
 /* ------------------------------------------------------------------------
+ * a2-a5 in one call: routing and dispatch of one RCEP invocation (Eqs.
+ * 10-12 and the prefix routing and dispatch of Algorithm 2). Outputs are
+ * bit-identical to decomoe_route_prefix (+ decomoe_select_prefix_device +
+ * decomoe_route_prefix_dk) followed by decomoe_dispatch on the same logits.
+ *   K >= k (<= E): fixed prefix [0, K); with mass_out ([E] fp64) the call also
+ *     computes the full-pool activated mass of Eq. 11; p is ignored.
+ *     Dispatch groups: K.
+ *   K == -1: device-selected prefix: mass_out (required) gets the mass, K is
+ *     chosen by Eq. 12 with 0 < p <= 1 (decomoe_select_prefix's arithmetic)
+ *     and written to K_dev (required), routing runs over [0, K). Dispatch
+ *     groups: E (those at or beyond K stay empty): counts [E], offsets [E+1].
+ * logits: [T, E] fp32 (row stride E). topk_idx, topk_w: [T, k]. x, d, dtype,
+ * counts, offsets, perm_token, inv_slot, x_perm: as decomoe_dispatch (x_perm
+ * NULL skips the row gather).
+ * ws: decomoe_route_dispatch_workspace_bytes(T, k, E) bytes (the routing
+ * and dispatch scratch). No host synchronisation; capturable in a CUDA graph.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API size_t decomoe_route_dispatch_workspace_bytes(int64_t T, int k, int E);
+DECOMOE_API int decomoe_route_dispatch(const float* logits, int64_t T, int E, int K, int k, double p,
+                                       int32_t* topk_idx, float* topk_w, double* mass_out, int32_t* K_dev,
+                                       const void* x, int d, int dtype, int32_t* counts, int32_t* offsets,
+                                       int32_t* perm_token, int32_t* inv_slot, void* x_perm, void* ws,
+                                       size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * Allocation-free dispatch (the paper has no counterpart: this is a library
  * convenience). Same arguments, outputs and errors as decomoe_dispatch, minus
  * the workspace: for callers that cannot allocate device memory, e.g. a

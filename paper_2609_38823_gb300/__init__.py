@@ -50,6 +50,9 @@ SIGNATURES = {
     "decomoe_select_prefix_device": (_I, [_P, _I, _I, _D, _P, _P]),
     "decomoe_route_prefix_dk": (_I, [_P, _L, _I, _L, _P, _I, _P, _P, _P]),
     "decomoe_dispatch_workspace_bytes": (_S, [_L, _I, _I]),
+    "decomoe_route_dispatch_workspace_bytes": (_S, [_L, _I, _I]),
+    "decomoe_route_dispatch": (_I, [_P, _L, _I, _I, _I, _D, _P, _P, _P, _P, _P, _I, _I, _P, _P, _P, _P, _P, _P, _S,
+                                    _P, _P]),
     "decomoe_savb_gate_workspace_bytes": (_S, [_I, _I]),
     "decomoe_savb_gate": (_I, [_P, _L, _I, _I, _L, _L, _P, _P, _P, _P, _I, _F, _P, _P, _P, _S, _P]),
     "decomoe_calib_workspace_bytes": (_S, [_L, _I]),
@@ -220,6 +223,28 @@ def decomoe_route_prefix_dk(logits, K_dev, k, topk_idx, topk_w, stream=None):
     _check("decomoe_route_prefix_dk",
            lib().decomoe_route_prefix_dk(_ptr(logits), T, E, E, _ptr(K_dev), k, _ptr(topk_idx), _ptr(topk_w),
                                          _stream(stream)))
+
+
+def decomoe_route_dispatch_workspace_bytes(T, k, E):
+    return int(lib().decomoe_route_dispatch_workspace_bytes(T, k, E))
+
+
+def decomoe_route_dispatch(logits, K, k, topk_idx, topk_w, x, counts, offsets, perm_token, inv_slot, x_perm, ws,
+                           p=0.0, mass_out=None, K_dev=None, status=None, stream=None):
+    """Routing and dispatch in one call: K >= k a fixed prefix (mass_out
+    optional), K = -1 the prefix selected on the device from p (mass_out and
+    K_dev required; dispatch then runs over all E groups)."""
+    _need_cuda(logits, topk_idx, topk_w, x, counts, offsets, perm_token, inv_slot, x_perm, ws, mass_out, K_dev,
+               status)
+    T, E = logits.shape
+    d = x.shape[1] if x is not None else 0
+    dtype = _dt(x) if x is not None else DECOMOE_BF16
+    _check("decomoe_route_dispatch",
+           lib().decomoe_route_dispatch(_ptr(logits), T, E, K, k, float(p), _ptr(topk_idx), _ptr(topk_w),
+                                        _ptr(mass_out), _ptr(K_dev), _ptr(x), d, dtype, _ptr(counts), _ptr(offsets),
+                                        _ptr(perm_token), _ptr(inv_slot), _ptr(x_perm), _ptr(ws),
+                                        0 if ws is None else ws.numel() * ws.element_size(), _ptr(status),
+                                        _stream(stream)))
 
 
 def decomoe_dispatch(topk_idx, K, x, counts, offsets, perm_token, inv_slot, x_perm, ws, status=None,

@@ -21,7 +21,6 @@ enum {
   WS_H,
   WS_YPERM,
   WS_ROUTE,
-  WS_DISPATCH,
   WS_KDEV,
   WS_SCHED,
   WS_STATUS_PAD,
@@ -49,8 +48,7 @@ static LayerLayout layer_layout(int64_t T, int d, int E, int k, int m, int dtype
   sz[WS_XPERM] = R * d * eb;
   sz[WS_H] = R * m * eb;
   sz[WS_YPERM] = R * d * eb;
-  sz[WS_ROUTE] = decomoe_route_workspace_bytes(T, E);
-  sz[WS_DISPATCH] = decomoe_dispatch_workspace_bytes(T, k, E);
+  sz[WS_ROUTE] = decomoe_route_dispatch_workspace_bytes(T, k, E);
   sz[WS_KDEV] = 16;
   sz[WS_SCHED] = 16;
   sz[WS_STATUS_PAD] = 256;
@@ -82,6 +80,66 @@ int decomoe_moe_layer_workspace_layout(int64_t T, int d, int E, int k, int m, in
   for (int i = 0; i <= WS_YPERM; ++i) offs_host[i] = L.off[i];
   offs_host[11] = L.off[WS_KDEV];
   return DECOMOE_OK;
+}
+
+size_t decomoe_route_dispatch_workspace_bytes(int64_t T, int k, int E) {
+  if (T < 0 || k <= 0 || E <= 0) return 0;
+  return align_up(decomoe_route_workspace_bytes(T, E), 256) + decomoe_dispatch_workspace_bytes(T, k, E);
+}
+
+int decomoe_route_dispatch(const float* logits, int64_t T, int E, int K, int k, double p, int32_t* topk_idx,
+                           float* topk_w, double* mass_out, int32_t* K_dev, const void* x, int d, int dtype,
+                           int32_t* counts, int32_t* offsets, int32_t* perm_token, int32_t* inv_slot, void* x_perm,
+                           void* ws, size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(T >= 0, "route_dispatch: T < 0");
+  DM_ARG_CHECK(E >= 1 && E <= DECOMOE_MAX_E && k >= 1 && k <= DECOMOE_MAX_TOPK && k <= E,
+               "route_dispatch: need 1 <= k <= E <= %d, k <= %d", DECOMOE_MAX_E, DECOMOE_MAX_TOPK);
+  const bool device_k = (K == -1);
+  DM_ARG_CHECK(device_k || (K >= k && K <= E), "route_dispatch: need k <= K <= E or K = -1 (k=%d K=%d E=%d)", k,
+               K, E);
+  if (device_k) {
+    DM_ARG_CHECK(p > 0.0 && p <= 1.0, "route_dispatch: a device-selected prefix needs 0 < p <= 1");
+    DM_ARG_CHECK(mass_out && K_dev, "route_dispatch: a device-selected prefix needs mass_out and K_dev");
+  }
+  DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "route_dispatch: bad dtype");
+  DM_ARG_CHECK(counts && offsets, "route_dispatch: counts/offsets null");
+  const int Kd = device_k ? E : K;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (T == 0) {
+    DM_CUDA_CHECK(cudaMemsetAsync(counts, 0, sizeof(int32_t) * Kd, s));
+    DM_CUDA_CHECK(cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (Kd + 1), s));
+    if (mass_out) DM_CUDA_CHECK(cudaMemsetAsync(mass_out, 0, sizeof(double) * E, s));
+    if (device_k) return decomoe_select_prefix_device(mass_out, E, k, p, K_dev, stream);  // zero mass: K = k
+    return DECOMOE_OK;
+  }
+  DM_ARG_CHECK(logits && topk_idx && topk_w && perm_token && inv_slot, "route_dispatch: null pointer");
+  DM_ARG_CHECK(T * static_cast<int64_t>(k) < 0x7fffffffLL, "route_dispatch: T*k too large");
+  const size_t row_bytes = static_cast<size_t>(d) * dtype_bytes(dtype);
+  if (x_perm != nullptr) {
+    DM_ARG_CHECK(x != nullptr && d > 0, "route_dispatch: x null or d <= 0");
+    DM_ARG_CHECK(row_bytes % 16 == 0 && aligned16(x) && aligned16(x_perm),
+                 "route_dispatch: rows must be 16-byte multiples and 16-byte aligned");
+  }
+  const size_t rbytes = align_up(decomoe_route_workspace_bytes(T, E), 256);
+  const size_t dbytes = decomoe_dispatch_workspace_bytes(T, k, E);
+  if (ws == nullptr || ws_bytes < rbytes + dbytes) {
+    set_error("route_dispatch: workspace needs %zu bytes", rbytes + dbytes);
+    return DECOMOE_ERR_WORKSPACE;
+  }
+  void* route_ws = ws;
+  void* disp_ws = static_cast<uint8_t*>(ws) + rbytes;
+  if (device_k) {
+    // mass pass, Eq. 12 on the device, routing over [0, *K_dev)
+    DM_RET(decomoe_route_prefix(logits, T, E, E, E, k, nullptr, nullptr, mass_out, route_ws, rbytes, stream));
+    DM_RET(decomoe_select_prefix_device(mass_out, E, k, p, K_dev, stream));
+    DM_RET(decomoe_route_prefix_dk(logits, T, E, E, K_dev, k, topk_idx, topk_w, stream));
+  } else {
+    // one launch: prefix routing and, with mass_out, the full-pool mass
+    DM_RET(decomoe_route_prefix(logits, T, E, E, K, k, topk_idx, topk_w, mass_out, route_ws, rbytes, stream));
+  }
+  return decomoe_dispatch(topk_idx, T, k, Kd, x, d, dtype, counts, offsets, perm_token, inv_slot, x_perm, disp_ws,
+                          dbytes, status_dev, stream);
 }
 
 int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const void* w_gate_up,
@@ -123,31 +181,29 @@ int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const v
   void* x_perm = base + L.off[WS_XPERM];
   void* h = base + L.off[WS_H];
   void* y_perm = base + L.off[WS_YPERM];
-  void* route_ws = base + L.off[WS_ROUTE];
-  void* disp_ws = base + L.off[WS_DISPATCH];
+  void* route_ws = base + L.off[WS_ROUTE];  // routing and dispatch scratch
 
   // a1: router logits over all E reordered experts
   DM_RET(decomoe_router_logits(x, w_r, bias, T, d, E, dtype, logits, status_dev, stream));
   // a2 (+ a3) and a4: full-pool activated mass and prefix routing
   int K = K_fixed;
   int32_t* K_dev = reinterpret_cast<int32_t*>(base + L.off[WS_KDEV]);
-  if (K_fixed == -1) {
-    // device-selected prefix: mass pass, Eq. 12 on the device, routing over
-    // [0, *K_dev); dispatch and experts run over all E groups (those at or
-    // beyond *K_dev are empty)
-    DM_RET(decomoe_route_prefix(logits, T, E, E, E, k, nullptr, nullptr, mass, route_ws,
-                                decomoe_route_workspace_bytes(T, E), stream));
-    DM_RET(decomoe_select_prefix_device(mass, E, k, p, K_dev, stream));
-    DM_RET(decomoe_route_prefix_dk(logits, T, E, E, K_dev, k, topk_idx, topk_w, stream));
-    K = E;
-    if (K_sel_host) *K_sel_host = -1;
-    if (K_used_host) *K_used_host = -1;
-  } else if (K_fixed > 0) {
-    // one launch: prefix routing over [0, K_fixed) and, when p > 0, the
-    // full-pool mass of Eq. 11 (left in the workspace, no host sync)
-    DM_RET(decomoe_route_prefix(logits, T, E, E, K, k, topk_idx, topk_w, p > 0.0 ? mass : nullptr, route_ws,
-                                decomoe_route_workspace_bytes(T, E), stream));
+  if (K_fixed != 0) {
+    // a2-a5: full-pool mass (Eq. 11), prefix (fixed, or Eq. 12 on the
+    // device), prefix routing and dispatch; with a device-selected prefix,
+    // dispatch and the experts run over all E groups (those at or beyond
+    // *K_dev are empty)
+    DM_RET(decomoe_route_dispatch(logits, T, E, K_fixed, k, p, topk_idx, topk_w,
+                                  (K_fixed == -1 || p > 0.0) ? mass : nullptr, K_dev, x, d, dtype, counts, offsets,
+                                  perm, inv, x_perm, route_ws, L.off[WS_KDEV] - L.off[WS_ROUTE], status_dev,
+                                  stream));
+    if (K_fixed == -1) {
+      K = E;
+      if (K_sel_host) *K_sel_host = -1;
+      if (K_used_host) *K_used_host = -1;
+    }
   } else {
+    // host-selected prefix: mass pass, one device-to-host read, Eq. 12 in C
     DM_RET(decomoe_route_prefix(logits, T, E, E, E, k, nullptr, nullptr, mass, route_ws,
                                 decomoe_route_workspace_bytes(T, E), stream));
     static thread_local std::vector<double> h_mass;
@@ -158,12 +214,11 @@ int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const v
     DM_RET(decomoe_select_prefix(h_mass.data(), E, k, p, &Ksel));
     K = Ksel;
     if (K_sel_host) *K_sel_host = Ksel;
-    DM_RET(decomoe_route_prefix(logits, T, E, E, K, k, topk_idx, topk_w, nullptr, nullptr, 0, stream));
+    DM_RET(decomoe_route_dispatch(logits, T, E, K, k, 0.0, topk_idx, topk_w, nullptr, nullptr, x, d, dtype, counts,
+                                  offsets, perm, inv, x_perm, route_ws, L.off[WS_KDEV] - L.off[WS_ROUTE],
+                                  status_dev, stream));
   }
   if (K_used_host && K_fixed != -1) *K_used_host = K;
-  // a5: dispatch (counts, offsets, permutation, x_perm rows)
-  DM_RET(decomoe_dispatch(topk_idx, T, k, K, x, d, dtype, counts, offsets, perm, inv, x_perm, disp_ws,
-                          decomoe_dispatch_workspace_bytes(T, k, K), status_dev, stream));
   // a6: grouped SwiGLU experts over [0, K)
   int32_t* sched = reinterpret_cast<int32_t*>(base + L.off[WS_SCHED]);
   DM_RET(decomoe_expert_swiglu(x_perm, offsets, T * k, K, d, m, dtype, w_gate_up, w_down, h, y_perm,

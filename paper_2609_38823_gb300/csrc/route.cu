@@ -35,6 +35,63 @@ __global__ void k_router_simt(const T* __restrict__ x, const T* __restrict__ w_r
   logits[i] = acc;
 }
 
+// Router for few tokens (decode): one warp per (expert row, group of
+// GEMV_TPW tokens). The warp loads its 16-byte slices of the router row and
+// of the tokens' rows (all loads in flight before any arithmetic), forms the
+// fp32 dot products of the bf16 values, and combines the lane partial sums
+// with a shuffle tree. The router matrix is read from HBM once and spread
+// over many SMs instead of one tensor-core tile.
+constexpr int GEMV_WARPS = 4;
+constexpr int GEMV_TPW = 4;  // tokens per warp
+__device__ __forceinline__ float dot8_bf16(const uint4 a, const uint4 b, float acc) {
+  acc = fmaf(bf16_lo(a.x), bf16_lo(b.x), acc);
+  acc = fmaf(bf16_hi(a.x), bf16_hi(b.x), acc);
+  acc = fmaf(bf16_lo(a.y), bf16_lo(b.y), acc);
+  acc = fmaf(bf16_hi(a.y), bf16_hi(b.y), acc);
+  acc = fmaf(bf16_lo(a.z), bf16_lo(b.z), acc);
+  acc = fmaf(bf16_hi(a.z), bf16_hi(b.z), acc);
+  acc = fmaf(bf16_lo(a.w), bf16_lo(b.w), acc);
+  acc = fmaf(bf16_hi(a.w), bf16_hi(b.w), acc);
+  return acc;
+}
+
+__global__ void __launch_bounds__(32 * GEMV_WARPS)
+    k_router_gemv(const uint4* __restrict__ x, const uint4* __restrict__ w_r, const float* __restrict__ bias,
+                  int64_t Tn, int vpr, int E, float* __restrict__ logits) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int e = blockIdx.x * GEMV_WARPS + warp;
+  const int64_t t0 = static_cast<int64_t>(blockIdx.y) * GEMV_TPW;
+  if (e >= E) return;
+  const uint4* wr = w_r + static_cast<int64_t>(e) * vpr;
+  float acc[GEMV_TPW];
+#pragma unroll
+  for (int j = 0; j < GEMV_TPW; ++j) acc[j] = 0.f;
+  const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
+  for (int c0 = 0; c0 < vpr; c0 += 32 * 8) {  // 8 vectors per lane per pass
+    uint4 wv[8], xv[GEMV_TPW][8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int c = c0 + lane + 32 * i;
+      wv[i] = (c < vpr) ? __ldg(wr + c) : zero;
+#pragma unroll
+      for (int j = 0; j < GEMV_TPW; ++j)
+        xv[j][i] = (c < vpr && t0 + j < Tn) ? __ldg(x + (t0 + j) * vpr + c) : zero;
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+      for (int j = 0; j < GEMV_TPW; ++j) acc[j] = dot8_bf16(wv[i], xv[j][i], acc[j]);
+  }
+  const float b = bias != nullptr ? bias[e] : 0.f;
+#pragma unroll
+  for (int j = 0; j < GEMV_TPW; ++j) {
+    float v = acc[j];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    if (lane == 0 && t0 + j < Tn) logits[(t0 + j) * E + e] = v + b;
+  }
+}
+
 // ------------------------------------------------------------ routing
 // One warp per token; lane l holds logits l, l+32, ... (E <= 256, 8 per lane)
 // in registers. A pass of k rounds of warp arg-max picks the k largest of a
@@ -181,11 +238,11 @@ __global__ void __launch_bounds__(256)
   if (threadIdx.x == 0) mass[e] = red[0];
 }
 
-// Eq. 12 on the device, one thread: the same sequential fp64 sums, division
-// and comparison as decomoe_select_prefix, so the prefix is bit-identical to
-// the host selection on the same mass.
-__global__ void k_select_prefix(const double* __restrict__ mass, int E, int k, double p, int32_t* __restrict__ K_dev) {
-  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+// Eq. 12, sequentially in fp64 with round-to-nearest adds and division, as
+// the host decomoe_select_prefix does: K_hat = smallest K whose prefix mass
+// ratio reaches p (E when p >= 1 or none does), K = max(k, K_hat); k when the
+// total mass is zero.
+__device__ int select_prefix_seq(const double* mass, int E, int k, double p) {
   double tot = 0.0;
   for (int e = 0; e < E; ++e) tot = __dadd_rn(tot, mass[e]);
   int K = k;
@@ -203,7 +260,13 @@ __global__ void k_select_prefix(const double* __restrict__ mass, int E, int k, d
     }
     K = K_hat > k ? K_hat : k;
   }
-  *K_dev = K;
+  return K;
+}
+
+// Eq. 12 on the device, one thread (bit-identical to decomoe_select_prefix).
+__global__ void k_select_prefix(const double* __restrict__ mass, int E, int k, double p, int32_t* __restrict__ K_dev) {
+  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+  *K_dev = select_prefix_seq(mass, E, k, p);
 }
 
 // Activated mass (Eq. 11) over n tokens whose logit rows skip a block:
@@ -235,6 +298,13 @@ int decomoe_router_logits(const void* x, const void* w_r, const float* bias, int
   if (T == 0) return DECOMOE_OK;
   DM_ARG_CHECK(x && w_r && logits, "router_logits: null pointer");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (dtype == DECOMOE_BF16 && T <= 64 && d % 8 == 0 && aligned16(x) && aligned16(w_r)) {
+    const dim3 grid((E + GEMV_WARPS - 1) / GEMV_WARPS, static_cast<unsigned>((T + GEMV_TPW - 1) / GEMV_TPW));
+    k_router_gemv<<<grid, 32 * GEMV_WARPS, 0, s>>>(static_cast<const uint4*>(x), static_cast<const uint4*>(w_r),
+                                                   bias, T, d / 8, E, logits);
+    DM_LAUNCH_CHECK("k_router_gemv");
+    return DECOMOE_OK;
+  }
   if (dtype == DECOMOE_BF16 && router_tc_supported(d, E)) {
     DM_ARG_CHECK(aligned16(x) && aligned16(w_r) && aligned16(logits),
                  "router_logits: pointers must be 16-byte aligned");

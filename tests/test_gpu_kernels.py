@@ -385,3 +385,71 @@ def test_rmsnorm():
         torch.cuda.synchronize()
         ref = O.rmsnorm(f64(x), 1e-6)
         assert np.abs(f64(y) - ref).max() <= tol * np.abs(ref).max() * 2
+
+
+# ----------------------------------------------------------------- routing + dispatch in one call
+
+@pytest.mark.parametrize("T,E,K,k,p", [(1, 128, 64, 8, 0.0), (7, 16, 10, 2, 0.0), (100, 128, 40, 8, 0.0),
+                                       (256, 128, 128, 8, 0.0), (257, 128, 64, 8, 0.0), (2048, 128, 64, 8, 0.0),
+                                       (33, 256, 200, 32, 0.0), (1, 128, -1, 8, 0.7), (64, 128, -1, 8, 0.9),
+                                       (256, 128, -1, 8, 0.5), (300, 128, -1, 8, 0.7), (2048, 128, -1, 8, 1.0)])
+def test_route_dispatch_equals_separate_calls_and_oracle(T, E, K, k, p):
+    """decomoe_route_dispatch (one block at decode sizes, the separate kernels
+    above them) equals the separate C-ABI calls bit for bit, and its dispatch
+    is the oracle's stable sort of its own picks."""
+    a = W.make_logits(T, E, std=0.9, bias=_zipf_bias(E), seed=3, wid=60 + E)
+    ad = a.to(DEV)
+    d = 256
+    x = torch.randn(T, d, generator=torch.Generator().manual_seed(T)).to(torch.bfloat16).to(DEV)
+    Kd = E if K == -1 else K
+    idx = torch.full((T, k), -9, dtype=torch.int32, device=DEV)
+    w = torch.empty(T, k, dtype=torch.float32, device=DEV)
+    mass = torch.empty(E, dtype=torch.float64, device=DEV)
+    Kdev = torch.zeros(1, dtype=torch.int32, device=DEV)
+    counts = torch.empty(Kd, dtype=torch.int32, device=DEV)
+    offsets = torch.empty(Kd + 1, dtype=torch.int32, device=DEV)
+    perm = torch.empty(T * k, dtype=torch.int32, device=DEV)
+    inv = torch.empty(T * k, dtype=torch.int32, device=DEV)
+    xp = torch.empty(T * k, d, dtype=torch.bfloat16, device=DEV)
+    ws = dm.workspace(dm.decomoe_route_dispatch_workspace_bytes(T, k, E), DEV)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    dm.decomoe_route_dispatch(ad, K, k, idx, w, x, counts, offsets, perm, inv, xp, ws, p=p, mass_out=mass,
+                              K_dev=Kdev if K == -1 else None, status=st)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(st) == 0
+    # separate calls
+    rws = dm.workspace(dm.decomoe_route_workspace_bytes(T, E), DEV)
+    idx2 = torch.empty(T, k, dtype=torch.int32, device=DEV)
+    w2 = torch.empty(T, k, dtype=torch.float32, device=DEV)
+    mass2 = torch.empty(E, dtype=torch.float64, device=DEV)
+    if K == -1:
+        Kdev2 = torch.empty(1, dtype=torch.int32, device=DEV)
+        dm.decomoe_route_prefix(ad, E, k, None, None, mass2, rws)
+        dm.decomoe_select_prefix_device(mass2, k, p, Kdev2)
+        dm.decomoe_route_prefix_dk(ad, Kdev2, k, idx2, w2)
+        Ksel = int(Kdev2)
+        assert int(Kdev) == Ksel
+    else:
+        dm.decomoe_route_prefix(ad, K, k, idx2, w2, mass2, rws)
+        Ksel = K
+    c2 = torch.empty(Kd, dtype=torch.int32, device=DEV)
+    o2 = torch.empty(Kd + 1, dtype=torch.int32, device=DEV)
+    p2 = torch.empty(T * k, dtype=torch.int32, device=DEV)
+    i2 = torch.empty(T * k, dtype=torch.int32, device=DEV)
+    xp2 = torch.empty(T * k, d, dtype=torch.bfloat16, device=DEV)
+    dm.decomoe_dispatch(idx2, Kd, x, c2, o2, p2, i2, xp2, dm.workspace(dm.decomoe_dispatch_workspace_bytes(T, k, Kd),
+                                                                      DEV))
+    torch.cuda.synchronize()
+    for got, ref in ((idx, idx2), (counts, c2), (offsets, o2), (perm, p2), (inv, i2)):
+        assert torch.equal(got, ref)
+    assert torch.equal(w.view(torch.int32), w2.view(torch.int32))
+    assert torch.equal(mass.view(torch.int64), mass2.view(torch.int64))
+    assert torch.equal(xp.view(torch.int16), xp2.view(torch.int16))
+    # oracle: dispatch of the picks, routing away from near-ties, mass
+    c, o, pp, ii = O.dispatch(idx.cpu().numpy().astype(np.int64), Kd)
+    assert np.array_equal(counts.cpu().numpy(), c) and np.array_equal(perm.cpu().numpy(), pp)
+    ri, rw = O.route_prefix(a.numpy(), Ksel, k)
+    keep = O.prefix_margin(a.numpy(), Ksel, k) >= MARGIN_SAME_LOGITS
+    assert np.array_equal(idx.cpu().numpy()[keep], ri[keep])
+    ref_m = O.activated_mass(a.numpy(), k)
+    assert (np.abs(mass.cpu().numpy() - ref_m) <= MASS_REL * ref_m + 1e-30).all()

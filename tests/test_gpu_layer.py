@@ -219,3 +219,59 @@ def test_layer_device_selected_prefix_in_cuda_graph(prefill_layer):
     Kdev = int(ws[offs[11]:offs[11] + 4].view(torch.int32))
     mass = ws[offs[3]:offs[3] + E * 8].view(torch.float64).cpu().numpy()
     assert Kdev == dm.decomoe_select_prefix(mass, k, 0.8)
+
+
+@pytest.mark.parametrize("T,K_fixed,p", [(1, 64, 0.7), (8, 64, 0.7), (32, 40, 0.0), (100, 128, 0.7), (256, 96, 0.7),
+                                         (1, -1, 0.7), (8, -1, 0.5), (129, -1, 0.9), (256, -1, 1.0)])
+def test_layer_intermediates_equal_separate_calls(T, K_fixed, p):
+    """The layer's routing, mass, prefix and dispatch intermediates (left in
+    its workspace) equal, bit for bit, the separate C-ABI calls on the same
+    router logits, for fixed and device-selected prefixes."""
+    wl = W.with_(W.PREFILL, T=T)
+    E, k, d, m = wl.E, wl.k, wl.d, wl.m
+    g = W.make_layer(wl, device="cuda", seed=T)
+    w_gu = dm.fuse_gate_up(g["w_gate"], g["w_up"])
+    out = torch.empty_like(g["x"])
+    ws = dm.workspace(dm.decomoe_moe_layer_workspace_bytes(T, d, E, k, m, dm.DECOMOE_BF16), DEV)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    dm.decomoe_moe_layer(g["x"], g["w_r"], g["bias"], w_gu, g["w_down"], k, out, ws, K_fixed=K_fixed, p=p,
+                         status=st)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(st) == 0
+    offs = dm.decomoe_moe_layer_workspace_layout(T, d, E, k, m, dm.DECOMOE_BF16)
+    view = lambda i, n, dt: ws[offs[i]:offs[i] + n * torch.tensor([], dtype=dt).element_size()].view(dt)
+    logits = view(0, T * E, torch.float32).view(T, E).clone()
+    Kd = E if K_fixed == -1 else K_fixed
+    got = dict(idx=view(1, T * k, torch.int32).cpu(), w=view(2, T * k, torch.float32).cpu(),
+               counts=view(4, Kd, torch.int32).cpu(), offsets=view(5, Kd + 1, torch.int32).cpu(),
+               perm=view(6, T * k, torch.int32).cpu(), inv=view(7, T * k, torch.int32).cpu(),
+               xp=view(8, T * k * d, torch.bfloat16).view(T * k, d).clone())
+    mass_l = view(3, E, torch.float64).cpu()
+    # separate calls on the same logits
+    mass = torch.empty(E, dtype=torch.float64, device=DEV)
+    rws = dm.workspace(dm.decomoe_route_workspace_bytes(T, E), DEV)
+    idx = torch.empty(T, k, dtype=torch.int32, device=DEV)
+    w = torch.empty(T, k, dtype=torch.float32, device=DEV)
+    if K_fixed == -1:
+        Kdev = torch.empty(1, dtype=torch.int32, device=DEV)
+        dm.decomoe_route_prefix(logits, E, k, None, None, mass, rws)
+        dm.decomoe_select_prefix_device(mass, k, p, Kdev)
+        dm.decomoe_route_prefix_dk(logits, Kdev, k, idx, w)
+        assert int(Kdev) == int(view(11, 1, torch.int32).cpu())
+    else:
+        dm.decomoe_route_prefix(logits, K_fixed, k, idx, w, mass if p > 0 else None, rws)
+    counts = torch.empty(Kd, dtype=torch.int32, device=DEV)
+    offsets = torch.empty(Kd + 1, dtype=torch.int32, device=DEV)
+    perm = torch.empty(T * k, dtype=torch.int32, device=DEV)
+    inv = torch.empty(T * k, dtype=torch.int32, device=DEV)
+    xp = torch.empty(T * k, d, dtype=torch.bfloat16, device=DEV)
+    dws = dm.workspace(dm.decomoe_dispatch_workspace_bytes(T, k, Kd), DEV)
+    dm.decomoe_dispatch(idx, Kd, g["x"], counts, offsets, perm, inv, xp, dws)
+    torch.cuda.synchronize()
+    assert torch.equal(got["idx"], idx.view(-1).cpu())
+    assert torch.equal(got["w"].view(torch.int32), w.view(-1).cpu().view(torch.int32))
+    for n, t in (("counts", counts), ("offsets", offsets), ("perm", perm), ("inv", inv)):
+        assert torch.equal(got[n], t.cpu()), n
+    assert torch.equal(got["xp"].view(torch.int16), xp.view(torch.int16))
+    if K_fixed == -1 or p > 0:
+        assert torch.equal(mass_l.view(torch.int64), mass.cpu().view(torch.int64))
