@@ -41,6 +41,9 @@ __global__ void k_router_simt(const T* __restrict__ x, const T* __restrict__ w_r
 // fp32 dot products of the bf16 values, and combines the lane partial sums
 // with a shuffle tree. The router matrix is read from HBM once and spread
 // over many SMs instead of one tensor-core tile.
+#ifndef DECOMOE_ROUTER_GEMV_MAX_T
+#define DECOMOE_ROUTER_GEMV_MAX_T 192  // token counts up to which the router runs on CUDA cores
+#endif
 constexpr int GEMV_WARPS = 4;
 constexpr int GEMV_TPW = 4;  // tokens per warp
 __device__ __forceinline__ float dot8_bf16(const uint4 a, const uint4 b, float acc) {
@@ -298,7 +301,7 @@ int decomoe_router_logits(const void* x, const void* w_r, const float* bias, int
   if (T == 0) return DECOMOE_OK;
   DM_ARG_CHECK(x && w_r && logits, "router_logits: null pointer");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (dtype == DECOMOE_BF16 && T <= 64 && d % 8 == 0 && aligned16(x) && aligned16(w_r)) {
+  if (dtype == DECOMOE_BF16 && T <= DECOMOE_ROUTER_GEMV_MAX_T && d % 8 == 0 && aligned16(x) && aligned16(w_r)) {
     const dim3 grid((E + GEMV_WARPS - 1) / GEMV_WARPS, static_cast<unsigned>((T + GEMV_TPW - 1) / GEMV_TPW));
     k_router_gemv<<<grid, 32 * GEMV_WARPS, 0, s>>>(static_cast<const uint4*>(x), static_cast<const uint4*>(w_r),
                                                    bias, T, d / 8, E, logits);
