@@ -1,6 +1,7 @@
 // Error reporting, device queries, the bounded-wait status word and its
 // self-test kernel.
 #include <atomic>
+#include <cstdlib>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -24,6 +25,21 @@ void set_error(const char* fmt, ...) {
 void clear_error() { t_last_error.clear(); }
 
 int64_t wait_limit_ns() { return g_wait_limit_ns.load(std::memory_order_relaxed); }
+
+// Programmatic launch pays for grids of at most one block per SM (the
+// persistent GEMMs and the decode-size kernels); kernels of many blocks ran
+// slower with it, so they launch plainly. DECOMOE_PDL=0 turns it off;
+// DECOMOE_PDL_MAX_BLOCKS overrides the grid-size limit.
+bool pdl_enabled(int64_t blocks) {
+  static const int64_t max_blocks = [] {
+    const char* on = getenv("DECOMOE_PDL");
+    if (on != nullptr && on[0] == '0') return static_cast<int64_t>(-1);
+    const char* v = getenv("DECOMOE_PDL_MAX_BLOCKS");
+    if (v != nullptr) return static_cast<int64_t>(atoll(v));
+    return static_cast<int64_t>(0);  // 0: one block per SM of the current device
+  }();
+  return blocks <= (max_blocks == 0 ? static_cast<int64_t>(sm_count()) : max_blocks);
+}
 
 int sm_count() {
   static std::mutex mu;

@@ -47,6 +47,7 @@ __global__ void __launch_bounds__(256)
     k_combine(const uint4* __restrict__ y, const int32_t* __restrict__ inv_slot,
               const float* __restrict__ w, int64_t Tn, int k, int vec,
               const uint4* __restrict__ residual, uint4* __restrict__ out) {
+  pdl_enter();
   constexpr int NE = BF16 ? 8 : 4;
   constexpr int WPT = 2;  // warps per token: each takes alternate 32-vector chunks
   const int lane = threadIdx.x & 31;
@@ -112,14 +113,14 @@ __global__ void __launch_bounds__(256)
 }
 
 template <bool BF16>
-static void launch_combine(int grid, cudaStream_t s, const uint4* y, const int32_t* inv, const float* w, int64_t T,
-                           int k, int vec, const uint4* res, uint4* out) {
+static cudaError_t launch_combine(int grid, cudaStream_t s, const uint4* y, const int32_t* inv, const float* w,
+                                  int64_t T, int k, int vec, const uint4* res, uint4* out) {
   switch (k) {
-    case 1: k_combine<BF16, 1><<<grid, 256, 0, s>>>(y, inv, w, T, k, vec, res, out); break;
-    case 2: k_combine<BF16, 2><<<grid, 256, 0, s>>>(y, inv, w, T, k, vec, res, out); break;
-    case 4: k_combine<BF16, 4><<<grid, 256, 0, s>>>(y, inv, w, T, k, vec, res, out); break;
-    case 8: k_combine<BF16, 8><<<grid, 256, 0, s>>>(y, inv, w, T, k, vec, res, out); break;
-    default: k_combine<BF16, 0><<<grid, 256, 0, s>>>(y, inv, w, T, k, vec, res, out); break;
+    case 1: return launch_pdl(k_combine<BF16, 1>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out);
+    case 2: return launch_pdl(k_combine<BF16, 2>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out);
+    case 4: return launch_pdl(k_combine<BF16, 4>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out);
+    case 8: return launch_pdl(k_combine<BF16, 8>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out);
+    default: return launch_pdl(k_combine<BF16, 0>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out);
   }
 }
 
@@ -131,6 +132,7 @@ __global__ void __launch_bounds__(256)
     k_compact_vec(const uint4* __restrict__ src, uint4* __restrict__ dst, int64_t rows_out,
                   int64_t vec, int64_t v0, int64_t nv, int64_t nbatch, int64_t sstride,
                   int64_t dstride) {
+  pdl_enter();
   constexpr int U = 4;
   const int64_t total = nbatch * rows_out * vec;
   const int64_t step = static_cast<int64_t>(gridDim.x) * blockDim.x * U;
@@ -161,6 +163,7 @@ __global__ void __launch_bounds__(256)
 __global__ void k_compact_bytes(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst,
                                 int64_t rows_out, int64_t row_bytes, int64_t v0, int64_t nv,
                                 int64_t nbatch, int64_t sstride, int64_t dstride) {
+  pdl_enter();
   const int64_t total = nbatch * rows_out * row_bytes;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -178,6 +181,7 @@ template <bool BF16>
 __global__ void __launch_bounds__(256)
     k_rmsnorm(const uint4* __restrict__ x, uint4* __restrict__ y, int64_t Tn, int vec, int d,
               float eps) {
+  pdl_enter();
   const int lane = threadIdx.x & 31;
   const int64_t gw = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int64_t nw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
@@ -252,12 +256,11 @@ int decomoe_combine(const void* y_perm, const int32_t* inv_slot, const float* to
   const int vec = static_cast<int>(row_bytes / 16);
   const int grid = grid_for_warps(2 * T);  // two warps per token
   if (dtype == DECOMOE_BF16)
-    launch_combine<true>(grid, s, static_cast<const uint4*>(y_perm), inv_slot, topk_w, T, k, vec,
-                         static_cast<const uint4*>(residual), static_cast<uint4*>(out));
+    DM_CUDA_CHECK(launch_combine<true>(grid, s, static_cast<const uint4*>(y_perm), inv_slot, topk_w, T, k, vec,
+                                       static_cast<const uint4*>(residual), static_cast<uint4*>(out)));
   else
-    launch_combine<false>(grid, s, static_cast<const uint4*>(y_perm), inv_slot, topk_w, T, k, vec,
-                          static_cast<const uint4*>(residual), static_cast<uint4*>(out));
-  DM_LAUNCH_CHECK("k_combine");
+    DM_CUDA_CHECK(launch_combine<false>(grid, s, static_cast<const uint4*>(y_perm), inv_slot, topk_w, T, k, vec,
+                                        static_cast<const uint4*>(residual), static_cast<uint4*>(out)));
   return DECOMOE_OK;
 }
 
@@ -287,15 +290,14 @@ int decomoe_drop_visual_block(const void* src, void* dst, int64_t rows, int64_t 
   if (vec_ok) {
     const int64_t nvec = nbatch * rows_out * (row_bytes / 16);
     const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>((nvec + 1023) / 1024, sm_count() * 16LL)));
-    k_compact_vec<<<grid, 256, 0, s>>>(static_cast<const uint4*>(src), static_cast<uint4*>(dst), rows_out,
-                                       row_bytes / 16, v0, nv, nbatch, src_batch_stride / 16,
-                                       dst_batch_stride / 16);
-    DM_LAUNCH_CHECK("k_compact_vec");
+    DM_CUDA_CHECK(launch_pdl(k_compact_vec, dim3(grid), dim3(256), 0, s, static_cast<const uint4*>(src),
+                             static_cast<uint4*>(dst), rows_out, row_bytes / 16, v0, nv, nbatch,
+                             src_batch_stride / 16, dst_batch_stride / 16));
   } else {
     const int grid = sm_count() * 8;
-    k_compact_bytes<<<grid, 256, 0, s>>>(static_cast<const uint8_t*>(src), static_cast<uint8_t*>(dst), rows_out,
-                                         row_bytes, v0, nv, nbatch, src_batch_stride, dst_batch_stride);
-    DM_LAUNCH_CHECK("k_compact_bytes");
+    DM_CUDA_CHECK(launch_pdl(k_compact_bytes, dim3(grid), dim3(256), 0, s, static_cast<const uint8_t*>(src),
+                             static_cast<uint8_t*>(dst), rows_out, row_bytes, v0, nv, nbatch, src_batch_stride,
+                             dst_batch_stride));
   }
   return DECOMOE_OK;
 }
@@ -312,10 +314,11 @@ int decomoe_rmsnorm(const void* x, void* y, int64_t T, int d, float eps, int dty
   const int vec = static_cast<int>(row_bytes / 16);
   const int grid = grid_for_warps(T);
   if (dtype == DECOMOE_BF16)
-    k_rmsnorm<true><<<grid, 256, 0, s>>>(static_cast<const uint4*>(x), static_cast<uint4*>(y), T, vec, d, eps);
+    DM_CUDA_CHECK(launch_pdl(k_rmsnorm<true>, dim3(grid), dim3(256), 0, s, static_cast<const uint4*>(x),
+                             static_cast<uint4*>(y), T, vec, d, eps));
   else
-    k_rmsnorm<false><<<grid, 256, 0, s>>>(static_cast<const uint4*>(x), static_cast<uint4*>(y), T, vec, d, eps);
-  DM_LAUNCH_CHECK("k_rmsnorm");
+    DM_CUDA_CHECK(launch_pdl(k_rmsnorm<false>, dim3(grid), dim3(256), 0, s, static_cast<const uint4*>(x),
+                             static_cast<uint4*>(y), T, vec, d, eps));
   return DECOMOE_OK;
 }
 

@@ -62,6 +62,28 @@ inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 inline size_t dtype_bytes(int dtype) { return dtype == DECOMOE_BF16 ? 2 : 4; }
 
 int sm_count();  // cached per device
+bool pdl_enabled(int64_t blocks);  // programmatic dependent launch for a grid of this many blocks
+
+// Launch with programmatic stream serialisation: the kernel's CTAs may start
+// while the previous kernel on the stream is still running; every kernel
+// launched this way calls pdl_wait() before it reads anything an earlier
+// kernel wrote (or writes anything an earlier kernel reads).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed =
+      pdl_enabled(static_cast<int64_t>(grid.x) * grid.y * grid.z) ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
 
 // Internal entry points shared between translation units.
 int launch_router_tc(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E,
@@ -80,6 +102,16 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
+}
+
+// Programmatic dependent launch: let the next kernel on the stream be
+// scheduled now, and wait until the previous kernel has completed and its
+// memory is visible (a no-op for kernels launched without the attribute).
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_enter() {
+  pdl_trigger();
+  pdl_wait();
 }
 
 // Record the first error code in the caller's status word (if given).

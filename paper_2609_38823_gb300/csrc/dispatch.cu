@@ -17,6 +17,7 @@ constexpr int DSP_TILE = DSP_WARPS * DSP_PER_WARP;  // pairs per block (1024)
 __global__ void __launch_bounds__(DSP_THREADS)
     k_dispatch_hist(const int32_t* __restrict__ idx, int64_t N, int K,
                     int32_t* __restrict__ tile_hist, int32_t* status) {
+  pdl_enter();
   __shared__ int hist[DECOMOE_MAX_E];
   for (int e = threadIdx.x; e < K; e += DSP_THREADS) hist[e] = 0;
   __syncthreads();
@@ -51,6 +52,7 @@ __global__ void __launch_bounds__(DSP_THREADS)
                        const int32_t* __restrict__ tile_hist, int ntiles,
                        int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
                        int32_t* __restrict__ perm_token, int32_t* __restrict__ inv_slot) {
+  pdl_enter();
   __shared__ int s_base[DECOMOE_MAX_E];
   __shared__ int s_wcnt[DSP_WARPS][DECOMOE_MAX_E];
   __shared__ int s_wsum[DSP_WARPS];
@@ -142,6 +144,7 @@ __global__ void __launch_bounds__(256)
     k_gather_rows(const uint4* __restrict__ x, const int32_t* __restrict__ perm_token,
                   const int32_t* __restrict__ offsets, int K, int vec_per_row,
                   uint4* __restrict__ x_perm) {
+  pdl_enter();
   const int rows = offsets[K];
   const int lane = threadIdx.x & 31;
   const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -205,19 +208,18 @@ int decomoe_dispatch(const int32_t* topk_idx, int64_t T, int k, int K, const voi
   }
   const int ntiles = static_cast<int>((N + DSP_TILE - 1) / DSP_TILE);
   int32_t* tile_hist = static_cast<int32_t*>(ws);
-  k_dispatch_hist<<<ntiles, DSP_THREADS, 0, s>>>(topk_idx, N, K, tile_hist, status_dev);
-  DM_LAUNCH_CHECK("k_dispatch_hist");
-  k_dispatch_scatter<<<ntiles, DSP_THREADS, 0, s>>>(topk_idx, N, k, K, tile_hist, ntiles, counts,
-                                                    offsets, perm_token, inv_slot);
-  DM_LAUNCH_CHECK("k_dispatch_scatter");
+  DM_CUDA_CHECK(launch_pdl(k_dispatch_hist, dim3(ntiles), dim3(DSP_THREADS), 0, s, topk_idx, N, K, tile_hist,
+                           status_dev));
+  DM_CUDA_CHECK(launch_pdl(k_dispatch_scatter, dim3(ntiles), dim3(DSP_THREADS), 0, s, topk_idx, N, k, K,
+                           static_cast<const int32_t*>(tile_hist), ntiles, counts, offsets, perm_token, inv_slot));
   if (x_perm != nullptr) {
     const int vec = static_cast<int>(row_bytes / 16);
     const int64_t want_warps = N;
     int blocks = static_cast<int>(std::min<int64_t>((want_warps * 32 + 255) / 256, sm_count() * 8LL));
     if (blocks < 1) blocks = 1;
-    k_gather_rows<<<blocks, 256, 0, s>>>(static_cast<const uint4*>(x), perm_token, offsets, K, vec,
-                                         static_cast<uint4*>(x_perm));
-    DM_LAUNCH_CHECK("k_gather_rows");
+    DM_CUDA_CHECK(launch_pdl(k_gather_rows, dim3(blocks), dim3(256), 0, s, static_cast<const uint4*>(x),
+                             static_cast<const int32_t*>(perm_token), static_cast<const int32_t*>(offsets), K, vec,
+                             static_cast<uint4*>(x_perm)));
   }
   return DECOMOE_OK;
 }
@@ -301,8 +303,8 @@ extern "C" int decomoe_dispatch_noalloc(const int32_t* topk_idx, int64_t T, int 
   // k_dispatch_hist writes every entry the scatter pass reads, so nothing
   // left in the array by an earlier call is ever used.
   const int ntiles = static_cast<int>(ntiles64);
-  k_dispatch_hist<<<ntiles, DSP_THREADS, 0, s>>>(topk_idx, N, K, tile_hist, status_dev);
-  DM_LAUNCH_CHECK("k_dispatch_hist");
+  DM_CUDA_CHECK(launch_pdl(k_dispatch_hist, dim3(ntiles), dim3(DSP_THREADS), 0, s, topk_idx, N, K, tile_hist,
+                           status_dev));
   k_dispatch_scatter<<<ntiles, DSP_THREADS, 0, s>>>(topk_idx, N, k, K, tile_hist, ntiles, counts, offsets,
                                                     perm_token, inv_slot);
   DM_LAUNCH_CHECK("k_dispatch_scatter");
@@ -310,9 +312,9 @@ extern "C" int decomoe_dispatch_noalloc(const int32_t* topk_idx, int64_t T, int 
     const int vec = static_cast<int>(row_bytes / 16);
     int blocks = static_cast<int>(std::min<int64_t>((N * 32 + 255) / 256, sm_count() * 8LL));
     if (blocks < 1) blocks = 1;
-    k_gather_rows<<<blocks, 256, 0, s>>>(static_cast<const uint4*>(x), perm_token, offsets, K, vec,
-                                         static_cast<uint4*>(x_perm));
-    DM_LAUNCH_CHECK("k_gather_rows");
+    DM_CUDA_CHECK(launch_pdl(k_gather_rows, dim3(blocks), dim3(256), 0, s, static_cast<const uint4*>(x),
+                             static_cast<const int32_t*>(perm_token), static_cast<const int32_t*>(offsets), K, vec,
+                             static_cast<uint4*>(x_perm)));
   }
   return DECOMOE_OK;
 }

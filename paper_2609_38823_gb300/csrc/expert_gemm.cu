@@ -198,8 +198,6 @@ __global__ void __launch_bounds__(64 + 32 * EW, OCC)
 #define TQE_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + C::TQ + (i)))
 
   const int G = g.ngroups;
-  for (int i = threadIdx.x; i <= G; i += blockDim.x)
-    s_off[i] = (g.offsets != nullptr) ? g.offsets[i] : (i == 0 ? 0 : g.rows);
   if (threadIdx.x == 0) {
     *s_abort = 0;
     for (int s = 0; s < STAGES; ++s) {
@@ -217,6 +215,11 @@ __global__ void __launch_bounds__(64 + 32 * EW, OCC)
     }
     fence_mbar_init();
   }
+  // wait for the earlier kernels' results; the next kernel is released only
+  // at the end (its CTAs would otherwise sit resident through this one)
+  pdl_wait();
+  for (int i = threadIdx.x; i <= G; i += blockDim.x)
+    s_off[i] = (g.offsets != nullptr) ? g.offsets[i] : (i == 0 ? 0 : g.rows);
   __syncthreads();
   if (warp == 2) {
     // exclusive scan of work units (MP M-tiles) per group: s_mt[g] = first unit of g
@@ -585,6 +588,7 @@ __global__ void __launch_bounds__(64 + 32 * EW, OCC)
       report_status(g.status, DECOMOE_ERR_TIMEOUT);
     }
   }
+  pdl_trigger();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -642,8 +646,7 @@ static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b
   const int64_t cap = static_cast<int64_t>(sm_count()) * OCC;
 #endif
   const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(cap, ub_tiles)));
-  kern<<<grid, 64 + 32 * EW, C::SMEM, s>>>(ta, tb, g);
-  DM_LAUNCH_CHECK("k_gemm_tc");
+  DM_CUDA_CHECK(launch_pdl(kern, dim3(grid), dim3(64 + 32 * EW), C::SMEM, s, ta, tb, g));
   return DECOMOE_OK;
 }
 
@@ -784,7 +787,6 @@ __global__ void __launch_bounds__(192, 1)
 
   const int G = g.G;
   const int nwb = g.wrows / WS_BM;
-  for (int i = threadIdx.x; i <= G; i += blockDim.x) s_off[i] = g.offsets[i];
   if (threadIdx.x == 0) {
     *s_abort = 0;
     for (int s = 0; s < STAGES; ++s) {
@@ -798,6 +800,10 @@ __global__ void __launch_bounds__(192, 1)
     mbar_init(DRAIN_BAR, 1);
     fence_mbar_init();
   }
+  // wait for the earlier kernels' results; the next kernel is released only
+  // at the end (its CTAs would otherwise sit resident through this one)
+  pdl_wait();
+  for (int i = threadIdx.x; i <= G; i += blockDim.x) s_off[i] = g.offsets[i];
   __syncthreads();
   if (warp == 2) {
     // s_tt[e] = first tile of expert e = sum over earlier experts of nwb * chunks
@@ -1021,6 +1027,7 @@ __global__ void __launch_bounds__(192, 1)
       report_status(g.status, DECOMOE_ERR_TIMEOUT);
     }
   }
+  pdl_trigger();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -1066,8 +1073,7 @@ static int launch_ws(const void* X, int rows, int kdim, const void* W, int wrows
   DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(C::SMEM)));
   const int64_t ub_tiles = (static_cast<int64_t>(rows) / WS_BN + G) * (wrows / WS_BM);
   const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(sm_count(), ub_tiles)));
-  kern<<<grid, 192, C::SMEM, s>>>(tw, tx, g);
-  DM_LAUNCH_CHECK("k_moe_ws");
+  DM_CUDA_CHECK(launch_pdl(kern, dim3(grid), dim3(192), C::SMEM, s, tw, tx, g));
   return DECOMOE_OK;
 }
 

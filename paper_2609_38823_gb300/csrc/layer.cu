@@ -220,9 +220,10 @@ int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const v
   }
   if (K_used_host && K_fixed != -1) *K_used_host = K;
   // a6: grouped SwiGLU experts over [0, K)
-  int32_t* sched = reinterpret_cast<int32_t*>(base + L.off[WS_SCHED]);
+  // static tile order (as fast as the dynamic queue here, and no counter
+  // reset between the launches, which keeps them chained programmatically)
   DM_RET(decomoe_expert_swiglu(x_perm, offsets, T * k, K, d, m, dtype, w_gate_up, w_down, h, y_perm,
-                               status_dev, sched, stream));
+                               status_dev, nullptr, stream));
   // a7: combine (+ residual)
   DM_RET(decomoe_combine(y_perm, inv, topk_w, T, k, d, dtype, residual, out, stream));
   return DECOMOE_OK;

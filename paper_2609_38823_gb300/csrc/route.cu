@@ -61,6 +61,7 @@ __device__ __forceinline__ float dot8_bf16(const uint4 a, const uint4 b, float a
 __global__ void __launch_bounds__(32 * GEMV_WARPS)
     k_router_gemv(const uint4* __restrict__ x, const uint4* __restrict__ w_r, const float* __restrict__ bias,
                   int64_t Tn, int vpr, int E, float* __restrict__ logits) {
+  pdl_enter();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int e = blockIdx.x * GEMV_WARPS + warp;
   const int64_t t0 = static_cast<int64_t>(blockIdx.y) * GEMV_TPW;
@@ -171,6 +172,7 @@ __global__ void __launch_bounds__(ROUTE_THREADS)
     k_route(const float* __restrict__ logits, int64_t Tn, int E, int64_t ld, int K, int k,
             int32_t* __restrict__ idx_out, float* __restrict__ w_out, double* __restrict__ part,
             const int32_t* __restrict__ K_dev, int64_t skip_at = INT64_MAX, int64_t skip_len = 0) {
+  pdl_enter();
   if (K_dev != nullptr) K = *K_dev;  // prefix chosen on the device (k <= K <= E by construction)
   __shared__ int s_idx[ROUTE_TPB][DECOMOE_MAX_TOPK];
   __shared__ float s_w[ROUTE_TPB][DECOMOE_MAX_TOPK];
@@ -228,6 +230,7 @@ __global__ void __launch_bounds__(ROUTE_THREADS)
 // shared memory combines the 256 thread sums (bit-reproducible).
 __global__ void __launch_bounds__(256)
     k_mass_finalize(const double* __restrict__ part, int nblocks, int E, double* __restrict__ mass) {
+  pdl_enter();
   __shared__ double red[256];
   const int e = blockIdx.x;
   double acc = 0.0;
@@ -268,6 +271,7 @@ __device__ int select_prefix_seq(const double* mass, int E, int k, double p) {
 
 // Eq. 12 on the device, one thread (bit-identical to decomoe_select_prefix).
 __global__ void k_select_prefix(const double* __restrict__ mass, int E, int k, double p, int32_t* __restrict__ K_dev) {
+  pdl_enter();
   if (threadIdx.x != 0 || blockIdx.x != 0) return;
   *K_dev = select_prefix_seq(mass, E, k, p);
 }
@@ -303,9 +307,8 @@ int decomoe_router_logits(const void* x, const void* w_r, const float* bias, int
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (dtype == DECOMOE_BF16 && T <= DECOMOE_ROUTER_GEMV_MAX_T && d % 8 == 0 && aligned16(x) && aligned16(w_r)) {
     const dim3 grid((E + GEMV_WARPS - 1) / GEMV_WARPS, static_cast<unsigned>((T + GEMV_TPW - 1) / GEMV_TPW));
-    k_router_gemv<<<grid, 32 * GEMV_WARPS, 0, s>>>(static_cast<const uint4*>(x), static_cast<const uint4*>(w_r),
-                                                   bias, T, d / 8, E, logits);
-    DM_LAUNCH_CHECK("k_router_gemv");
+    DM_CUDA_CHECK(launch_pdl(k_router_gemv, grid, dim3(32 * GEMV_WARPS), 0, s, static_cast<const uint4*>(x),
+                             static_cast<const uint4*>(w_r), bias, static_cast<int64_t>(T), d / 8, E, logits));
     return DECOMOE_OK;
   }
   if (dtype == DECOMOE_BF16 && router_tc_supported(d, E)) {
@@ -357,13 +360,12 @@ int decomoe_route_prefix(const float* logits, int64_t T, int E, int64_t ld, int 
     }
     part = static_cast<double*>(ws);
   }
-  k_route<<<static_cast<unsigned>(nblocks), ROUTE_THREADS, 0, s>>>(logits, T, E, ld, K, k, topk_idx,
-                                                                   topk_w, part, nullptr);
-  DM_LAUNCH_CHECK("k_route");
-  if (mass_out != nullptr) {
-    k_mass_finalize<<<E, 256, 0, s>>>(part, static_cast<int>(nblocks), E, mass_out);
-    DM_LAUNCH_CHECK("k_mass_finalize");
-  }
+  DM_CUDA_CHECK(launch_pdl(k_route, dim3(static_cast<unsigned>(nblocks)), dim3(ROUTE_THREADS), 0, s, logits, T, E,
+                           ld, K, k, topk_idx, topk_w, part, static_cast<const int32_t*>(nullptr), INT64_MAX,
+                           static_cast<int64_t>(0)));
+  if (mass_out != nullptr)
+    DM_CUDA_CHECK(launch_pdl(k_mass_finalize, dim3(E), dim3(256), 0, s, static_cast<const double*>(part),
+                             static_cast<int>(nblocks), E, mass_out));
   return DECOMOE_OK;
 }
 
@@ -374,8 +376,8 @@ int decomoe_select_prefix_device(const double* mass, int E, int k, double p, int
   DM_ARG_CHECK(mass && K_dev, "select_prefix_device: null pointer");
   DM_ARG_CHECK(E >= 1 && k >= 1 && k <= E, "select_prefix_device: need 1 <= k <= E");
   DM_ARG_CHECK(p > 0.0 && p <= 1.0, "select_prefix_device: p must lie in (0, 1]");
-  k_select_prefix<<<1, 32, 0, reinterpret_cast<cudaStream_t>(stream)>>>(mass, E, k, p, K_dev);
-  DM_LAUNCH_CHECK("k_select_prefix");
+  DM_CUDA_CHECK(launch_pdl(k_select_prefix, dim3(1), dim3(32), 0, reinterpret_cast<cudaStream_t>(stream), mass, E, k,
+                           p, K_dev));
   return DECOMOE_OK;
 }
 
@@ -388,9 +390,9 @@ int decomoe_route_prefix_dk(const float* logits, int64_t T, int E, int64_t ld, c
   DM_ARG_CHECK(logits && K_dev, "route_prefix_dk: null pointer");
   const int64_t nblocks = (T + ROUTE_TPB - 1) / ROUTE_TPB;
   DM_ARG_CHECK(nblocks <= 0x7fffffff, "route_prefix_dk: T too large");
-  k_route<<<static_cast<unsigned>(nblocks), ROUTE_THREADS, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-      logits, T, E, ld, E, k, topk_idx, topk_w, nullptr, K_dev);
-  DM_LAUNCH_CHECK("k_route");
+  DM_CUDA_CHECK(launch_pdl(k_route, dim3(static_cast<unsigned>(nblocks)), dim3(ROUTE_THREADS), 0,
+                           reinterpret_cast<cudaStream_t>(stream), logits, T, E, ld, E, k, topk_idx, topk_w,
+                           static_cast<double*>(nullptr), K_dev, INT64_MAX, static_cast<int64_t>(0)));
   return DECOMOE_OK;
 }
 

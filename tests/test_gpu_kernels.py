@@ -346,7 +346,8 @@ def test_drop_visual_block_bit_exact(shape, v0, nv, dt):
 # ----------------------------------------------------------------- router logits
 
 @pytest.mark.parametrize("T,d,E", [(2048, 2048, 128), (1, 2048, 128), (300, 2048, 256), (1552, 2048, 128),
-                                   (129, 256, 128)])
+                                   (129, 256, 128), (7, 2048, 128), (192, 2048, 128), (193, 2048, 256),
+                                   (33, 4096, 64), (5, 2056, 16)])
 def test_router_logits_bf16_tensor_cores(T, d, E):
     g = torch.Generator().manual_seed(T + E)
     x = torch.randn(T, d, generator=g).to(torch.bfloat16)
