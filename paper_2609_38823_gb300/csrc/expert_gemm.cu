@@ -30,6 +30,11 @@
 // when the average expert gets at most DECOMOE_WS_MAX_AVG_ROWS rows (decode
 // sizes: every tile streams its own weight slice), the tokens-as-M k_gemm_tc
 // otherwise (prefill: faster when many rows share an expert's weights).
+// How the gathered gate/up entry loads its A rows: 2 = cp.async rows by four
+// extra warps, 1 = TMA tile::gather4.
+#ifndef DECOMOE_GATHER_MODE
+#define DECOMOE_GATHER_MODE 2
+#endif
 #ifndef DECOMOE_WS_MAX_AVG_ROWS
 #define DECOMOE_WS_MAX_AVG_ROWS 8
 #endif
@@ -96,7 +101,8 @@ struct TcArgs {
   int32_t* status;
   uint64_t limit_ns;
   int n_valid;  // EPI_F32_BIAS_T: number of valid output columns (tokens)
-  const int32_t* a_rows;  // GATHER_A: A row r is row a_rows[r] of the A tensor (rows entries)
+  const int32_t* a_rows;  // GA != 0: A row r is row a_rows[r] of the A tensor (rows entries)
+  const uint8_t* a_ptr;   // GA == 2: the A tensor itself (rows of kdim bf16)
   int* sched;             // dynamic scheduling: tile counter, zero at launch (null: static round robin)
 };
 
@@ -166,12 +172,19 @@ __device__ __forceinline__ void tile_coords(int tile, int NT, const int* s_mt, i
 
 // EW epilogue warps (4 or 8): with 8, two warps share each 32-lane TMEM
 // quarter and split its column chunks, so the epilogue's latency is hidden.
-template <int BN, int EPI, int STAGES, int BK, bool GATHER_A = false, int MP = 1, int EW = 8, int OCC = 1>
-__global__ void __launch_bounds__(64 + 32 * EW, OCC)
+// GA: how A tiles reach shared memory. 0: tiled TMA of rows [row0, row0+128)
+// of A. 1: TMA tile::gather4 of the rows a_rows[row0 ..] (warp 0). 2: four
+// extra warps, one A row per thread, 16-byte cp.async of the rows
+// a_rows[row0 ..] into the 128-byte-swizzled layout the TMA would produce;
+// each thread's copies complete on the stage's full barrier.
+template <int BN, int EPI, int STAGES, int BK, int GA = 0, int MP = 1, int EW = 8, int OCC = 1>
+__global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
     k_gemm_tc(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b,
               const TcArgs g) {
   using C = TcCfg<BN, STAGES, BK, MP, OCC>;
-  static_assert(!(GATHER_A && MP != 1), "gathered A takes one M-tile per work item");
+  static_assert(!(GA != 0 && MP != 1), "gathered A takes one M-tile per work item");
+  static_assert(GA != 2 || BK == 64, "the cp.async gather writes 128-byte swizzled rows");
+  constexpr bool GATHER_A = GA == 1;
   __shared__ int s_arow[GATHER_A ? 128 : 1];
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -201,7 +214,7 @@ __global__ void __launch_bounds__(64 + 32 * EW, OCC)
   if (threadIdx.x == 0) {
     *s_abort = 0;
     for (int s = 0; s < STAGES; ++s) {
-      mbar_init(FULL_BAR(s), 1);
+      mbar_init(FULL_BAR(s), GA == 2 ? 1 + 128 : 1);  // + one arrival per cp.async A-row thread
       mbar_init(EMPTY_BAR(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -269,7 +282,7 @@ __global__ void __launch_bounds__(64 + 32 * EW, OCC)
   // Tile sequence of this CTA. Static: blockIdx.x, + gridDim.x, ... Dynamic:
   // the producer takes the next id from the global counter and passes it to
   // the MMA and epilogue warps through a TQ-deep shared-memory queue; -1 ends.
-  const bool dyn = !GATHER_A && g.sched != nullptr;
+  const bool dyn = GA == 0 && g.sched != nullptr;
   auto static_tile = [&](int i) -> int {
     const int t = static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x);
     return t < total ? t : -1;
@@ -361,10 +374,12 @@ __global__ void __launch_bounds__(64 + 32 * EW, OCC)
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(FULL_BAR(stage), (has2 ? 2 : 1) * C::A_BYTES + C::B_BYTES);
-          tma_load_2d(sA + stage * MP * C::A_BYTES, &tma_a, FULL_BAR(stage), kb * C::BK, row0);
-          if (has2)
-            tma_load_2d(sA + (stage * MP + 1) * C::A_BYTES, &tma_a, FULL_BAR(stage), kb * C::BK, row0 + C::BM);
+          mbar_arrive_expect_tx(FULL_BAR(stage), (GA == 2 ? 0 : (has2 ? 2 : 1) * C::A_BYTES) + C::B_BYTES);
+          if constexpr (GA == 0) {
+            tma_load_2d(sA + stage * MP * C::A_BYTES, &tma_a, FULL_BAR(stage), kb * C::BK, row0);
+            if (has2)
+              tma_load_2d(sA + (stage * MP + 1) * C::A_BYTES, &tma_a, FULL_BAR(stage), kb * C::BK, row0 + C::BM);
+          }
           tma_load_2d(sB + stage * C::B_BYTES, &tma_b, FULL_BAR(stage), kb * C::BK, brow);
           armed |= 1u << stage;
           armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
@@ -418,6 +433,7 @@ __global__ void __launch_bounds__(64 + 32 * EW, OCC)
           break;
         }
         tc_fence_after();
+        if constexpr (GA == 2) fence_proxy_async_smem();  // A rows came through the generic proxy
         const uint64_t ad = smem_desc_kmajor<BK>(sA + stage * MP * C::A_BYTES);
         const uint64_t bd = smem_desc_kmajor<BK>(sB + stage * C::B_BYTES);
 #pragma unroll
@@ -445,6 +461,60 @@ __global__ void __launch_bounds__(64 + 32 * EW, OCC)
         tc_commit(DRAIN_BAR);
         mbar_wait(DRAIN_BAR, 0, g.limit_ns, &no_abort);
       }
+    }
+  } else if (GA == 2 && warp >= 2 + EW) {
+    // ------------------------------------------------ A rows by cp.async:
+    // the 128 threads copy the tile's 128 A rows (token rows a_rows[row0 +
+    // i] of the A tensor), 8 x 16 bytes per row per k-block, eight lanes per
+    // row so each warp instruction reads four whole 128-byte row segments.
+    // Chunk c of tile row i lands at i*128 + ((c ^ (i & 7)) * 16): the
+    // 128-byte-swizzled layout the TMA would write.
+    const int t = threadIdx.x - 32 * (2 + EW);
+    const int c = lane & 7;                      // 16-byte chunk of the row
+    const int i0 = (t >> 5) * 32 + (lane >> 3);  // rows i0 + 4j, j < 8
+    int stage = 0;
+    uint32_t ph = 0;
+    bool ok = true;
+    for (int ti = 0;; ++ti) {
+      const int tile = static_tile(ti);
+      if (tile < 0) break;
+      int grp, mt, nb;
+      tile_coords(tile, NT, s_mt, G, grp, mt, nb);
+      const int row0 = s_off[grp] + mt * C::BM;
+      const uint8_t* src[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int r = row0 + i0 + 4 * j;
+        const int src_row = (r < g.rows) ? g.a_rows[r] : 0;  // rows past the end: any valid row, never stored
+        src[j] = g.a_ptr + static_cast<int64_t>(src_row) * g.kdim * 2 + c * 16;
+      }
+      for (int kb = 0; kb < KB; ++kb) {
+        bool got = true;
+        if (lane == 0) got = mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort);
+        got = __shfl_sync(0xffffffffu, got, 0);
+        if (!got) {
+          ok = false;
+          break;
+        }
+        const uint32_t dst = sA + stage * C::A_BYTES;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int i = i0 + 4 * j;
+          cp_async16(dst + static_cast<uint32_t>(i) * 128u + (static_cast<uint32_t>(c ^ (i & 7)) << 4),
+                     src[j] + kb * (C::BK * 2));
+        }
+        cp_async_mbar_arrive_noinc(FULL_BAR(stage));
+        if (++stage == STAGES) {
+          stage = 0;
+          ph ^= 1u;
+        }
+      }
+      if (!ok) break;
+    }
+    cp_async_wait_all();  // every copy lands before the CTA can exit
+    if (!ok && lane == 0) {
+      *s_abort = 1;
+      report_status(g.status, DECOMOE_ERR_TIMEOUT);
     }
   } else if (warp >= 2) {
     // ------------------------------------------------ epilogue
@@ -607,15 +677,17 @@ __global__ void __launch_bounds__(64 + 32 * EW, OCC)
 
 // A: [rows, kdim], or with GATHER_A the source tensor [a_tensor_rows, kdim]
 // whose row a_rows[r] is A row r.
-template <int BN, int EPI, int STAGES, int BK, bool GATHER_A = false, int MP = 1, int EW = 8, int OCC = 1>
+template <int BN, int EPI, int STAGES, int BK, int GA = 0, int MP = 1, int EW = 8, int OCC = 1>
 static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b_rows,
                      const int32_t* offsets, int ngroups, int n_per_group, void* out,
                      int64_t out_ld, const float* bias, int32_t* status, cudaStream_t s, int n_valid = 0,
                      const int32_t* a_rows = nullptr, int64_t a_tensor_rows = 0, int* sched = nullptr) {
   using C = TcCfg<BN, STAGES, BK, MP, OCC>;
   CUtensorMap ta, tb;
-  if (GATHER_A)
+  if (GA == 1)
     DM_RET(make_tmap_bf16(&ta, A, static_cast<uint64_t>(kdim), static_cast<uint64_t>(a_tensor_rows), 1, BK));
+  else if (GA == 2)
+    ta = CUtensorMap{};  // A is read with cp.async, not TMA
   else
     DM_RET(make_tmap_bf16(&ta, A, static_cast<uint64_t>(kdim), static_cast<uint64_t>(rows), C::BM, BK));
   DM_RET(make_tmap_bf16(&tb, B, static_cast<uint64_t>(kdim), static_cast<uint64_t>(b_rows), BN, BK));
@@ -632,9 +704,10 @@ static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b
   g.limit_ns = static_cast<uint64_t>(wait_limit_ns());
   g.n_valid = n_valid;
   g.a_rows = a_rows;
+  g.a_ptr = static_cast<const uint8_t*>(A);
   g.sched = sched;
   if (sched != nullptr) DM_CUDA_CHECK(cudaMemsetAsync(sched, 0, sizeof(int), s));
-  auto kern = k_gemm_tc<BN, EPI, STAGES, BK, GATHER_A, MP, EW, OCC>;
+  auto kern = k_gemm_tc<BN, EPI, STAGES, BK, GA, MP, EW, OCC>;
   static_assert(C::SMEM <= 232448, "shared memory budget");
   DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(C::SMEM)));
@@ -646,7 +719,7 @@ static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b
   const int64_t cap = static_cast<int64_t>(sm_count()) * OCC;
 #endif
   const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(cap, ub_tiles)));
-  DM_CUDA_CHECK(launch_pdl(kern, dim3(grid), dim3(64 + 32 * EW), C::SMEM, s, ta, tb, g));
+  DM_CUDA_CHECK(launch_pdl(kern, dim3(grid), dim3(64 + 32 * EW + (GA == 2 ? 128 : 0)), C::SMEM, s, ta, tb, g));
   return DECOMOE_OK;
 }
 
@@ -1358,9 +1431,9 @@ int decomoe_expert_gate_up_gather(const void* x, int64_t T, const int32_t* perm_
   }
   if (static_cast<int64_t>(R) <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K)
     return launch_ws<true, 4, true>(x, R, d, w_gate_up, 2 * m, offsets, K, h, m, status_dev, s, perm_token, T);
-  return launch_tc<256, EPI_SWIGLU, GU_STAGES, GU_BK, true>(x, R, d, w_gate_up, static_cast<int64_t>(K) * 2 * m,
-                                                            offsets, K, 2 * m, h, m, nullptr, status_dev, s, 0,
-                                                            perm_token, T);
+  return launch_tc<256, EPI_SWIGLU, GU_STAGES, GU_BK, DECOMOE_GATHER_MODE>(
+      x, R, d, w_gate_up, static_cast<int64_t>(K) * 2 * m, offsets, K, 2 * m, h, m, nullptr, status_dev, s, 0,
+      perm_token, T);
 }
 
 int decomoe_expert_swiglu_gather(const void* x, int64_t T, const int32_t* perm_token, const int32_t* offsets,
