@@ -56,20 +56,24 @@ def parse():
 
 # ------------------------------------------------------------------ distributed plumbing
 
-def dist_setup(args):
+def dist_setup(args, backend=None):
+    """One process per GPU (torchrun env). The replicas exchange nothing but
+    the timing barrier and the max-over-ranks reduction: NCCL for our arm,
+    gloo for the CPU reference arm (and for CPU tests of this logic)."""
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if ws > 1:
         import torch.distributed as dist
 
-        if args.impl == "ours":
+        backend = backend or ("nccl" if args.impl == "ours" else "gloo")
+        if backend == "nccl":
             torch.cuda.set_device(local)
             dist.init_process_group("nccl", device_id=torch.device("cuda", local))
         else:
-            dist.init_process_group("gloo")
+            dist.init_process_group(backend)
     elif torch.cuda.is_available():
-        torch.cuda.set_device(0)
+        torch.cuda.set_device(local)
     return ws, rank, local
 
 
@@ -81,13 +85,21 @@ def barrier(ws):
 
 
 def max_over_ranks(v, ws):
+    """The slowest rank's value (the job's time is its last rank's time)."""
     if ws == 1:
         return v
     import torch.distributed as dist
 
-    t = torch.tensor([v], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([v], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_rate(units_per_rank, ws, ms_max):
+    """Whole-job throughput: the units every replica processed, over the
+    slowest replica's time (weak scaling: fixed work per rank)."""
+    return ws * units_per_rank / (ms_max / 1e3)
 
 
 # ------------------------------------------------------------------ clocks
@@ -314,7 +326,7 @@ def ours(args, ws, rank, local):
         raise RuntimeError("device status set during the benchmark")
     ms_max = max_over_ranks(ms, ws)
     step_ms = ms_max / args.steps
-    tok_s = ws * T * args.steps / (ms_max / 1e3)
+    tok_s = job_rate(T * args.steps, ws, ms_max)
     gu_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
     dn_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
     del graphs
@@ -377,7 +389,7 @@ def ours(args, ws, rank, local):
         e_steps = max(10, min(args.steps, 1000))
         ms_e, _ = timed(e2e_step, e_steps, max(3, args.warmup), ws)
         ms_e = max_over_ranks(ms_e, ws)
-        e2e = {"value": round(ws * T * e_steps / (ms_e / 1e3), 1), "unit": "tokens/s",
+        e2e = {"value": round(job_rate(T * e_steps, ws, ms_e), 1), "unit": "tokens/s",
                "h2d_bytes_per_step": T * wl.d * 2, "d2h_bytes_per_step": T * wl.d * 2,
                "ms_per_step": round(ms_e / e_steps, 4), "steps": e_steps,
                "path": "pinned host x -> decomoe_moe_layer (C ABI) -> decomoe_drop_visual_block -> pinned host out"}
