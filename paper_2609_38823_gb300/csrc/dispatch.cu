@@ -47,20 +47,48 @@ __global__ void __launch_bounds__(DSP_THREADS)
 // pairs [w*128, w*128+128) of the tile in order, ranks inside a 32-pair round
 // come from __match_any_sync, and per-warp running counts are scanned across
 // warps. Writes perm_token and inv_slot; block 0 writes counts and offsets.
+// SINGLE: one tile in one block (decode sizes): the block also counts the
+// histogram itself and may copy the rows (x_perm != null).
+template <bool SINGLE>
 __global__ void __launch_bounds__(DSP_THREADS)
     k_dispatch_scatter(const int32_t* __restrict__ idx, int64_t N, int k, int K,
                        const int32_t* __restrict__ tile_hist, int ntiles,
                        int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
-                       int32_t* __restrict__ perm_token, int32_t* __restrict__ inv_slot) {
+                       int32_t* __restrict__ perm_token, int32_t* __restrict__ inv_slot,
+                       int32_t* status = nullptr, const uint4* __restrict__ x = nullptr, int row_vec = 0,
+                       uint4* __restrict__ x_perm = nullptr) {
   pdl_enter();
   __shared__ int s_base[DECOMOE_MAX_E];
   __shared__ int s_wcnt[DSP_WARPS][DECOMOE_MAX_E];
   __shared__ int s_wsum[DSP_WARPS];
+  __shared__ int s_row[SINGLE ? DSP_TILE : 1];  // rows of this tile's pairs (for the in-block gather)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int e_t = threadIdx.x;  // one expert per thread (K <= 256 = DSP_THREADS)
 
   int tot = 0, before = 0;
-  if (e_t < K) {
+  if constexpr (SINGLE) {
+    // a single tile (one block): count its pairs here, as k_dispatch_hist does
+    int* s_cnt = &s_wcnt[0][0];
+    for (int e = threadIdx.x; e < K; e += DSP_THREADS) s_cnt[e] = 0;
+    __syncthreads();
+#pragma unroll
+    for (int r = 0; r < DSP_PER_WARP / 32; ++r) {
+      const int64_t f = static_cast<int64_t>(warp) * DSP_PER_WARP + r * 32 + lane;
+      int e = -2;
+      if (f < N) {
+        e = idx[f];
+        if (e < 0 || e >= K) {
+          report_status(status, DECOMOE_ERR_BAD_INPUT);
+          e = -1;
+        }
+      }
+      const uint32_t grp = __match_any_sync(0xffffffffu, e);
+      if (e >= 0 && lane == __ffs(grp) - 1) atomicAdd(&s_cnt[e], __popc(grp));
+    }
+    __syncthreads();
+    if (e_t < K) tot = s_cnt[e_t];
+    __syncthreads();
+  } else if (e_t < K) {
     for (int b = 0; b < ntiles; ++b) {
       const int v = tile_hist[static_cast<int64_t>(b) * K + e_t];
       tot += v;
@@ -128,13 +156,35 @@ __global__ void __launch_bounds__(DSP_THREADS)
     const int64_t f = base + r * 32 + lane;
     if (f >= N) continue;
     const int e = ex[r];
+    int row = -1;
     if (e >= 0) {
-      const int row = s_base[e] + s_wcnt[warp][e] + rank[r];
+      row = s_base[e] + s_wcnt[warp][e] + rank[r];
       perm_token[row] = static_cast<int32_t>(f / k);
-      inv_slot[f] = row;
-    } else {
-      inv_slot[f] = -1;
     }
+    inv_slot[f] = row;
+    if constexpr (SINGLE) s_row[warp * DSP_PER_WARP + r * 32 + lane] = row;
+  }
+  if (!SINGLE || x_perm == nullptr) return;
+  // in-block gather (single small tile): warp per pair, 16-byte vectors
+  __syncthreads();
+  const int64_t n_here = (N - static_cast<int64_t>(blockIdx.x) * DSP_TILE < DSP_TILE)
+                             ? N - static_cast<int64_t>(blockIdx.x) * DSP_TILE
+                             : DSP_TILE;
+  for (int i = warp; i < n_here; i += DSP_WARPS) {
+    const int row = s_row[i];
+    if (row < 0) continue;
+    const int64_t f = static_cast<int64_t>(blockIdx.x) * DSP_TILE + i;
+    const uint4* src = x + (f / k) * row_vec;
+    uint4* dst = x_perm + static_cast<int64_t>(row) * row_vec;
+    int c = lane;
+    for (; c + 32 * 3 < row_vec; c += 32 * 4) {
+      uint4 v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) v[u] = __ldg(src + c + 32 * u);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) dst[c + 32 * u] = v[u];
+    }
+    for (; c < row_vec; c += 32) dst[c] = __ldg(src + c);
   }
 }
 
@@ -208,10 +258,23 @@ int decomoe_dispatch(const int32_t* topk_idx, int64_t T, int k, int K, const voi
   }
   const int ntiles = static_cast<int>((N + DSP_TILE - 1) / DSP_TILE);
   int32_t* tile_hist = static_cast<int32_t*>(ws);
-  DM_CUDA_CHECK(launch_pdl(k_dispatch_hist, dim3(ntiles), dim3(DSP_THREADS), 0, s, topk_idx, N, K, tile_hist,
-                           status_dev));
-  DM_CUDA_CHECK(launch_pdl(k_dispatch_scatter, dim3(ntiles), dim3(DSP_THREADS), 0, s, topk_idx, N, k, K,
-                           static_cast<const int32_t*>(tile_hist), ntiles, counts, offsets, perm_token, inv_slot));
+  if (ntiles == 1) {
+    // one tile (decode sizes): count, scan and rank in one block, and copy
+    // the rows there too when they are few
+    const bool gather_here = x_perm != nullptr && static_cast<size_t>(N) * row_bytes <= 64 * 1024;
+    DM_CUDA_CHECK(launch_pdl(k_dispatch_scatter<true>, dim3(1), dim3(DSP_THREADS), 0, s, topk_idx, N, k, K,
+                             static_cast<const int32_t*>(nullptr), 1, counts, offsets, perm_token, inv_slot,
+                             status_dev, static_cast<const uint4*>(x), static_cast<int>(row_bytes / 16),
+                             gather_here ? static_cast<uint4*>(x_perm) : static_cast<uint4*>(nullptr)));
+    if (gather_here) return DECOMOE_OK;
+  } else {
+    DM_CUDA_CHECK(launch_pdl(k_dispatch_hist, dim3(ntiles), dim3(DSP_THREADS), 0, s, topk_idx, N, K, tile_hist,
+                             status_dev));
+    DM_CUDA_CHECK(launch_pdl(k_dispatch_scatter<false>, dim3(ntiles), dim3(DSP_THREADS), 0, s, topk_idx, N, k, K,
+                             static_cast<const int32_t*>(tile_hist), ntiles, counts, offsets, perm_token, inv_slot,
+                             static_cast<int32_t*>(nullptr), static_cast<const uint4*>(nullptr), 0,
+                             static_cast<uint4*>(nullptr)));
+  }
   if (x_perm != nullptr) {
     const int vec = static_cast<int>(row_bytes / 16);
     const int64_t want_warps = N;
@@ -305,7 +368,7 @@ extern "C" int decomoe_dispatch_noalloc(const int32_t* topk_idx, int64_t T, int 
   const int ntiles = static_cast<int>(ntiles64);
   DM_CUDA_CHECK(launch_pdl(k_dispatch_hist, dim3(ntiles), dim3(DSP_THREADS), 0, s, topk_idx, N, K, tile_hist,
                            status_dev));
-  k_dispatch_scatter<<<ntiles, DSP_THREADS, 0, s>>>(topk_idx, N, k, K, tile_hist, ntiles, counts, offsets,
+  k_dispatch_scatter<false><<<ntiles, DSP_THREADS, 0, s>>>(topk_idx, N, k, K, tile_hist, ntiles, counts, offsets,
                                                     perm_token, inv_slot);
   DM_LAUNCH_CHECK("k_dispatch_scatter");
   if (x_perm != nullptr) {

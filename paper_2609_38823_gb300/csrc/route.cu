@@ -358,12 +358,14 @@ int decomoe_route_prefix(const float* logits, int64_t T, int E, int64_t ld, int 
       set_error("route_prefix: workspace needs %zu bytes", decomoe_route_workspace_bytes(T, E));
       return DECOMOE_ERR_WORKSPACE;
     }
-    part = static_cast<double*>(ws);
+    // one routing block: its partial is the mass itself (the fixed-order
+    // finalize would only add zeros), so it is written in place
+    part = nblocks == 1 ? mass_out : static_cast<double*>(ws);
   }
   DM_CUDA_CHECK(launch_pdl(k_route, dim3(static_cast<unsigned>(nblocks)), dim3(ROUTE_THREADS), 0, s, logits, T, E,
                            ld, K, k, topk_idx, topk_w, part, static_cast<const int32_t*>(nullptr), INT64_MAX,
                            static_cast<int64_t>(0)));
-  if (mass_out != nullptr)
+  if (mass_out != nullptr && nblocks > 1)
     DM_CUDA_CHECK(launch_pdl(k_mass_finalize, dim3(E), dim3(256), 0, s, static_cast<const double*>(part),
                              static_cast<int>(nblocks), E, mass_out));
   return DECOMOE_OK;
