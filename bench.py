@@ -33,7 +33,7 @@ sys.path.insert(0, ROOT)
 
 import workloads as W  # noqa: E402
 
-LAUNCHES_PER_STEP = 10  # router 1, route+mass 2, dispatch 3, gate/up 1, down 1, combine 1, compaction 1
+LAUNCHES_PER_STEP = 11  # router 2 (k slices + reduction), route+mass 2, dispatch 3, gate/up, down, combine, compaction
 # (plus two 4-byte memsets zeroing the expert GEMMs' tile counter)
 
 
@@ -196,6 +196,7 @@ class Buffers:
         k, E, d, m = wl.k, wl.E, wl.d, wl.m
         R = T * k
         self.logits = torch.empty(T, E, dtype=torch.float32, device=dev)
+        self.router_ws = dm.workspace(dm.decomoe_router_logits_ws_bytes(T, wl.d, E), dev)
         self.mass = torch.empty(E, dtype=torch.float64, device=dev)
         self.route_ws = dm.workspace(dm.decomoe_route_workspace_bytes(T, E), dev)
         self.idx = torch.empty(T, k, dtype=torch.int32, device=dev)
@@ -215,7 +216,7 @@ class Buffers:
 def run_step(dm, wl, L, B, K, v0, nv, text, ev=None):
     """One pass of the hot path, every step a C-ABI call (10 kernel launches)."""
     k, E = wl.k, wl.E
-    dm.decomoe_router_logits(L.x, L.w_r, L.bias, B.logits, B.status)                   # a1
+    dm.decomoe_router_logits_ws(L.x, L.w_r, L.bias, B.logits, B.router_ws, B.status)   # a1
     dm.decomoe_route_dispatch(B.logits, K, k, B.idx, B.w, L.x, B.counts[:K], B.offsets[:K + 1], B.perm, B.inv,
                               B.x_perm, B.rd_ws, mass_out=B.mass, status=B.status)   # a2 (Eq. 11) + a4 + a5
     if ev is not None:

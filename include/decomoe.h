@@ -91,6 +91,19 @@ DECOMOE_API int decomoe_router_logits(const void* x, const void* w_r, const floa
                           decomoe_stream_t stream);
 
 /* ------------------------------------------------------------------------
+ * a1 with a workspace: the same logits as decomoe_router_logits (within the
+ * fp32 summation bound; the order of the additions differs). Above the
+ * CUDA-core token range the tensor-core router then splits the k loop into
+ * slices that run on more CTAs and adds their partial sums in slice order,
+ * the bias last. ws: decomoe_router_logits_ws_bytes(T, d, E) bytes (0 means
+ * no split at this size; ws may then be NULL), 16-byte aligned.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API size_t decomoe_router_logits_ws_bytes(int64_t T, int d, int E);
+DECOMOE_API int decomoe_router_logits_ws(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E,
+                                         int dtype, float* logits, void* ws, size_t ws_bytes, int32_t* status_dev,
+                                         decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * a2 + a4. Routing on fp32 logits (Eqs. 10-11; prefix rule of Section 3.3 and
  * Algorithm 2).
  *   For every token t: S_t = the k largest of logits[t, 0:K) (largest first;

@@ -44,6 +44,8 @@ SIGNATURES = {
     "decomoe_version": (_I, []),
     "decomoe_device_info": (_I, [_P, _P, _P]),
     "decomoe_router_logits": (_I, [_P, _P, _P, _L, _I, _I, _I, _P, _P, _P]),
+    "decomoe_router_logits_ws_bytes": (_S, [_L, _I, _I]),
+    "decomoe_router_logits_ws": (_I, [_P, _P, _P, _L, _I, _I, _I, _P, _P, _S, _P, _P]),
     "decomoe_route_workspace_bytes": (_S, [_L, _I]),
     "decomoe_route_prefix": (_I, [_P, _L, _I, _L, _I, _I, _P, _P, _P, _P, _S, _P]),
     "decomoe_select_prefix": (_I, [_P, _I, _I, _D, _P]),
@@ -198,6 +200,21 @@ def decomoe_router_logits(x, w_r, bias, logits, status=None, stream=None):
     _check("decomoe_router_logits",
            lib().decomoe_router_logits(_ptr(x), _ptr(w_r), _ptr(bias), T, d, E, _dt(x), _ptr(logits),
                                        _ptr(status), _stream(stream)))
+
+
+def decomoe_router_logits_ws_bytes(T, d, E):
+    return int(lib().decomoe_router_logits_ws_bytes(T, d, E))
+
+
+def decomoe_router_logits_ws(x, w_r, bias, logits, ws, status=None, stream=None):
+    """Router logits with a workspace (k-split tensor-core path at large T)."""
+    _need_cuda(x, w_r, bias, logits, ws, status)
+    T, d = x.shape
+    E = w_r.shape[0]
+    _check("decomoe_router_logits_ws",
+           lib().decomoe_router_logits_ws(_ptr(x), _ptr(w_r), _ptr(bias), T, d, E, _dt(x), _ptr(logits), _ptr(ws),
+                                          0 if ws is None else ws.numel() * ws.element_size(), _ptr(status),
+                                          _stream(stream)))
 
 
 def decomoe_route_prefix(logits, K, k, topk_idx=None, topk_w=None, mass_out=None, ws=None, E=None,

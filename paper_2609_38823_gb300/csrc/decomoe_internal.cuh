@@ -89,6 +89,9 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
 int launch_router_tc(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E,
                      float* logits, int32_t* status, cudaStream_t s);
 bool router_tc_supported(int d, int E);
+int router_split_ks(int64_t T, int d, int E);  // k slices of the split router at T tokens (1: no split)
+int launch_router_split(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E, float* logits,
+                        float* scratch, int32_t* status, cudaStream_t s);
 int launch_skip_mass(const float* logits, int64_t n, int E, int64_t ld, int k, int64_t skip_at, int64_t skip_len,
                      double* part, double* mass, cudaStream_t s);
 

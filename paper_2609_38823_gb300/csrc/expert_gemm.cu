@@ -104,6 +104,7 @@ struct TcArgs {
   const int32_t* a_rows;  // GA != 0: A row r is row a_rows[r] of the A tensor (rows entries)
   const uint8_t* a_ptr;   // GA == 2: the A tensor itself (rows of kdim bf16)
   int* sched;             // dynamic scheduling: tile counter, zero at launch (null: static round robin)
+  int64_t split_stride;   // KS > 1: elements between the k slices' partial outputs
 };
 
 // MP = M-tiles per work item. MP = 1: one 128-row A tile per B tile, two
@@ -177,13 +178,17 @@ __device__ __forceinline__ void tile_coords(int tile, int NT, const int* s_mt, i
 // extra warps, one A row per thread, 16-byte cp.async of the rows
 // a_rows[row0 ..] into the 128-byte-swizzled layout the TMA would produce;
 // each thread's copies complete on the stage's full barrier.
-template <int BN, int EPI, int STAGES, int BK, int GA = 0, int MP = 1, int EW = 8, int OCC = 1>
+// KS: split of the k loop. Work item = (output tile, k slice); slice s runs
+// k-blocks [s*KB/KS, (s+1)*KB/KS) and writes its partial sums to
+// out + s * split_stride (EPI_F32_BIAS_T only; the caller adds the slices).
+template <int BN, int EPI, int STAGES, int BK, int GA = 0, int MP = 1, int EW = 8, int OCC = 1, int KS = 1>
 __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
     k_gemm_tc(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b,
               const TcArgs g) {
   using C = TcCfg<BN, STAGES, BK, MP, OCC>;
   static_assert(!(GA != 0 && MP != 1), "gathered A takes one M-tile per work item");
   static_assert(GA != 2 || BK == 64, "the cp.async gather writes 128-byte swizzled rows");
+  static_assert(KS == 1 || (EPI == EPI_F32_BIAS_T && MP == 1 && GA == 0), "k split: transposed fp32 partials only");
   constexpr bool GATHER_A = GA == 1;
   __shared__ int s_arow[GATHER_A ? 128 : 1];
   extern __shared__ uint8_t smem_raw[];
@@ -266,7 +271,7 @@ __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
   }
   __syncthreads();
   const int NT = g.n_per_group / BN;
-  const int total = s_mt[G] * NT;
+  const int total = s_mt[G] * NT * KS;
   if (static_cast<int>(blockIdx.x) >= total) return;  // before any TMEM or TMA use
 
   if (warp == 1) {
@@ -277,7 +282,7 @@ __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *s_tmem;
-  const int KB = g.kdim / C::BK;
+  const int KB = g.kdim / C::BK / KS;  // k-blocks per work item
 
   // Tile sequence of this CTA. Static: blockIdx.x, + gridDim.x, ... Dynamic:
   // the producer takes the next id from the global counter and passes it to
@@ -331,9 +336,10 @@ __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
       }
       if (tile < 0) break;
       int grp, mt, nb;
-      tile_coords(tile, NT, s_mt, G, grp, mt, nb);
+      tile_coords(tile / KS, NT, s_mt, G, grp, mt, nb);
       const int row0 = s_off[grp] + mt * MP * C::BM;
       const int brow = grp * g.n_per_group + nb * BN;
+      const int kbase = (tile % KS) * KB;  // first k-block of this work item's slice
       const bool has2 = MP == 2 && row0 + C::BM < s_off[grp + 1];  // second M-tile has rows
       if constexpr (GATHER_A) {
 #pragma unroll
@@ -376,11 +382,12 @@ __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
           }
           mbar_arrive_expect_tx(FULL_BAR(stage), (GA == 2 ? 0 : (has2 ? 2 : 1) * C::A_BYTES) + C::B_BYTES);
           if constexpr (GA == 0) {
-            tma_load_2d(sA + stage * MP * C::A_BYTES, &tma_a, FULL_BAR(stage), kb * C::BK, row0);
+            tma_load_2d(sA + stage * MP * C::A_BYTES, &tma_a, FULL_BAR(stage), (kbase + kb) * C::BK, row0);
             if (has2)
-              tma_load_2d(sA + (stage * MP + 1) * C::A_BYTES, &tma_a, FULL_BAR(stage), kb * C::BK, row0 + C::BM);
+              tma_load_2d(sA + (stage * MP + 1) * C::A_BYTES, &tma_a, FULL_BAR(stage), (kbase + kb) * C::BK,
+                          row0 + C::BM);
           }
-          tma_load_2d(sB + stage * C::B_BYTES, &tma_b, FULL_BAR(stage), kb * C::BK, brow);
+          tma_load_2d(sB + stage * C::B_BYTES, &tma_b, FULL_BAR(stage), (kbase + kb) * C::BK, brow);
           armed |= 1u << stage;
           armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
           if (++stage == STAGES) {
@@ -418,7 +425,7 @@ __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
       bool has2 = false;
       if constexpr (MP == 2) {
         int grp, mt, nb;
-        tile_coords(tile, NT, s_mt, G, grp, mt, nb);
+        tile_coords(tile / KS, NT, s_mt, G, grp, mt, nb);
         has2 = s_off[grp] + (mt * 2 + 1) * C::BM < s_off[grp + 1];
       }
       if (!mbar_wait(TEMPTY_BAR(acc), aph ^ 1u, g.limit_ns, s_abort)) {
@@ -479,7 +486,7 @@ __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
       const int tile = static_tile(ti);
       if (tile < 0) break;
       int grp, mt, nb;
-      tile_coords(tile, NT, s_mt, G, grp, mt, nb);
+      tile_coords(tile / KS, NT, s_mt, G, grp, mt, nb);
       const int row0 = s_off[grp] + mt * C::BM;
       const uint8_t* src[8];
 #pragma unroll
@@ -534,7 +541,7 @@ __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
       const int acc = it % C::NBUF;
       const uint32_t aph = (it / C::NBUF) & 1;
       int grp, mt, nb;
-      tile_coords(tile, NT, s_mt, G, grp, mt, nb);
+      tile_coords(tile / KS, NT, s_mt, G, grp, mt, nb);
       const int row_end = s_off[grp + 1];
       if (!mbar_wait(TFULL_BAR(acc), aph, g.limit_ns, s_abort)) {
         ok = false;
@@ -597,9 +604,10 @@ __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
           }
         }
       } else if constexpr (EPI == EPI_F32_BIAS_T) {
-        // row = router row (expert), columns = tokens nb*BN + c
-        float* out = static_cast<float*>(g.out);
-        const float bv = (valid && g.bias) ? g.bias[grow] : 0.f;
+        // row = router row (expert), columns = tokens nb*BN + c; with a k
+        // split, slice (tile % KS) writes its partial sums without the bias
+        float* out = static_cast<float*>(g.out) + static_cast<int64_t>(tile % KS) * g.split_stride;
+        const float bv = (KS == 1 && valid && g.bias) ? g.bias[grow] : 0.f;
         const int n0 = nb * BN;
         if constexpr (BN == 16) {
           if (wp == 0) {
@@ -677,11 +685,12 @@ __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
 
 // A: [rows, kdim], or with GATHER_A the source tensor [a_tensor_rows, kdim]
 // whose row a_rows[r] is A row r.
-template <int BN, int EPI, int STAGES, int BK, int GA = 0, int MP = 1, int EW = 8, int OCC = 1>
+template <int BN, int EPI, int STAGES, int BK, int GA = 0, int MP = 1, int EW = 8, int OCC = 1, int KS = 1>
 static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b_rows,
                      const int32_t* offsets, int ngroups, int n_per_group, void* out,
                      int64_t out_ld, const float* bias, int32_t* status, cudaStream_t s, int n_valid = 0,
-                     const int32_t* a_rows = nullptr, int64_t a_tensor_rows = 0, int* sched = nullptr) {
+                     const int32_t* a_rows = nullptr, int64_t a_tensor_rows = 0, int* sched = nullptr,
+                     int64_t split_stride = 0) {
   using C = TcCfg<BN, STAGES, BK, MP, OCC>;
   CUtensorMap ta, tb;
   if (GA == 1)
@@ -706,13 +715,14 @@ static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b
   g.a_rows = a_rows;
   g.a_ptr = static_cast<const uint8_t*>(A);
   g.sched = sched;
+  g.split_stride = split_stride;
   if (sched != nullptr) DM_CUDA_CHECK(cudaMemsetAsync(sched, 0, sizeof(int), s));
-  auto kern = k_gemm_tc<BN, EPI, STAGES, BK, GA, MP, EW, OCC>;
+  auto kern = k_gemm_tc<BN, EPI, STAGES, BK, GA, MP, EW, OCC, KS>;
   static_assert(C::SMEM <= 232448, "shared memory budget");
   DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(C::SMEM)));
   const int64_t ub_tiles =
-      (static_cast<int64_t>(rows) / C::BM + ngroups) * static_cast<int64_t>(n_per_group / BN);
+      (static_cast<int64_t>(rows) / C::BM + ngroups) * static_cast<int64_t>(n_per_group / BN) * KS;
 #ifdef DECOMOE_GRID_CAP
   const int64_t cap = std::min<int64_t>(static_cast<int64_t>(sm_count()) * OCC, DECOMOE_GRID_CAP);
 #else
@@ -1193,6 +1203,72 @@ int launch_router_tc(const void* x, const void* w_r, const float* bias, int64_t 
   if (T <= 16 * ctas) return launch_router_bn<16>(x, w_r, bias, T, d, E, logits, status, s);
   if (T <= 32 * ctas) return launch_router_bn<32>(x, w_r, bias, T, d, E, logits, status, s);
   return launch_router_bn<64>(x, w_r, bias, T, d, E, logits, status, s);
+}
+
+// k-split router: KS k slices of the router GEMM write partial logits
+// [KS][T][E] (no bias) to the scratch, then k_router_reduce adds the slices in
+// slice order and the bias last: logits = (((p0 + p1) + ...) + p_{KS-1}) + b.
+// More CTAs with fewer k-blocks each (and N = 64 tokens per MMA instead of
+// 16) than the unsplit kernel at the same token count.
+template <int KS>
+__global__ void __launch_bounds__(256)
+    k_router_reduce(const float4* __restrict__ part, int64_t n4, const float* __restrict__ bias, int E,
+                    float4* __restrict__ logits) {
+  pdl_enter();
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    float4 v[KS];
+#pragma unroll
+    for (int sl = 0; sl < KS; ++sl) v[sl] = __ldcs(part + sl * n4 + i);  // every slice load in flight
+    float4 acc = v[0];
+#pragma unroll
+    for (int sl = 1; sl < KS; ++sl) {
+      acc.x += v[sl].x;
+      acc.y += v[sl].y;
+      acc.z += v[sl].z;
+      acc.w += v[sl].w;
+    }
+    if (bias != nullptr) {
+      const int e = static_cast<int>((i * 4) % E);
+      acc.x += bias[e];
+      acc.y += bias[e + 1];
+      acc.z += bias[e + 2];
+      acc.w += bias[e + 3];
+    }
+    logits[i] = acc;
+  }
+}
+
+int router_split_ks(int64_t T, int d, int E) {
+  if (!router_tc_supported(d, E) || d % (64 * 16) != 0) return 1;
+  const int64_t tiles = (T + 63) / 64, ctas = sm_count();
+  if (tiles * 16 <= ctas) return 16;
+  if (tiles * 4 <= ctas) return 4;
+  return 1;
+}
+
+template <int KS>
+static int launch_router_split_ks(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E,
+                                  float* logits, float* scratch, int32_t* status, cudaStream_t s) {
+  const int64_t npad = (T + 63) / 64 * 64;
+  const int64_t n = T * E;
+  DM_RET((launch_tc<64, EPI_F32_BIAS_T, 8, 64, 0, 1, 8, 1, KS>(w_r, E, d, x, T, nullptr, 1, static_cast<int>(npad),
+                                                               scratch, E, nullptr, status, s, static_cast<int>(T),
+                                                               nullptr, 0, nullptr, n)));
+  const int64_t n4 = n / 4;
+  const int blocks = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>((n4 + 255) / 256, sm_count())));
+  DM_CUDA_CHECK(launch_pdl(k_router_reduce<KS>, dim3(blocks), dim3(256), 0, s,
+                           reinterpret_cast<const float4*>(scratch), n4, bias, E, reinterpret_cast<float4*>(logits)));
+  return DECOMOE_OK;
+}
+
+int launch_router_split(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E, float* logits,
+                        float* scratch, int32_t* status, cudaStream_t s) {
+  switch (router_split_ks(T, d, E)) {
+    case 16: return launch_router_split_ks<16>(x, w_r, bias, T, d, E, logits, scratch, status, s);
+    case 4: return launch_router_split_ks<4>(x, w_r, bias, T, d, E, logits, scratch, status, s);
+    default: return launch_router_tc(x, w_r, bias, T, d, E, logits, status, s);
+  }
 }
 
 // ------------------------------------------------------------------ CUDA-core paths

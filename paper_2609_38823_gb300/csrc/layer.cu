@@ -23,6 +23,7 @@ enum {
   WS_ROUTE,
   WS_KDEV,
   WS_SCHED,
+  WS_RSPLIT,
   WS_STATUS_PAD,
   WS_COUNT
 };
@@ -51,6 +52,7 @@ static LayerLayout layer_layout(int64_t T, int d, int E, int k, int m, int dtype
   sz[WS_ROUTE] = decomoe_route_dispatch_workspace_bytes(T, k, E);
   sz[WS_KDEV] = 16;
   sz[WS_SCHED] = 16;
+  sz[WS_RSPLIT] = decomoe_router_logits_ws_bytes(T, d, E);
   sz[WS_STATUS_PAD] = 256;
   size_t o = 0;
   for (int i = 0; i < WS_COUNT; ++i) {
@@ -184,7 +186,8 @@ int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const v
   void* route_ws = base + L.off[WS_ROUTE];  // routing and dispatch scratch
 
   // a1: router logits over all E reordered experts
-  DM_RET(decomoe_router_logits(x, w_r, bias, T, d, E, dtype, logits, status_dev, stream));
+  DM_RET(decomoe_router_logits_ws(x, w_r, bias, T, d, E, dtype, logits, base + L.off[WS_RSPLIT],
+                                  decomoe_router_logits_ws_bytes(T, d, E), status_dev, stream));
   // a2 (+ a3) and a4: full-pool activated mass and prefix routing
   int K = K_fixed;
   int32_t* K_dev = reinterpret_cast<int32_t*>(base + L.off[WS_KDEV]);

@@ -329,6 +329,30 @@ int decomoe_router_logits(const void* x, const void* w_r, const float* bias, int
   return DECOMOE_OK;
 }
 
+size_t decomoe_router_logits_ws_bytes(int64_t T, int d, int E) {
+  if (T <= 0 || d <= 0 || E <= 0) return 0;
+  if (T <= DECOMOE_ROUTER_GEMV_MAX_T) return 0;
+  const int ks = router_split_ks(T, d, E);
+  return ks > 1 ? align_up(static_cast<size_t>(ks) * T * E * sizeof(float), 256) : 0;
+}
+
+int decomoe_router_logits_ws(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E, int dtype,
+                             float* logits, void* ws, size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream) {
+  clear_error();
+  const size_t need = decomoe_router_logits_ws_bytes(T, d, E);
+  if (dtype != DECOMOE_BF16 || need == 0 || T <= DECOMOE_ROUTER_GEMV_MAX_T)
+    return decomoe_router_logits(x, w_r, bias, T, d, E, dtype, logits, status_dev, stream);
+  DM_ARG_CHECK(x && w_r && logits, "router_logits_ws: null pointer");
+  DM_ARG_CHECK(aligned16(x) && aligned16(w_r) && aligned16(logits) && aligned16(ws),
+               "router_logits_ws: pointers must be 16-byte aligned");
+  if (ws == nullptr || ws_bytes < need) {
+    set_error("router_logits_ws: workspace needs %zu bytes", need);
+    return DECOMOE_ERR_WORKSPACE;
+  }
+  return launch_router_split(x, w_r, bias, T, d, E, logits, static_cast<float*>(ws), status_dev,
+                             reinterpret_cast<cudaStream_t>(stream));
+}
+
 size_t decomoe_route_workspace_bytes(int64_t T, int E) {
   if (T < 0 || E <= 0) return 0;
   const int64_t nblocks = (T + ROUTE_TPB - 1) / ROUTE_TPB;

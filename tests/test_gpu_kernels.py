@@ -454,3 +454,28 @@ def test_route_dispatch_equals_separate_calls_and_oracle(T, E, K, k, p):
     assert np.array_equal(idx.cpu().numpy()[keep], ri[keep])
     ref_m = O.activated_mass(a.numpy(), k)
     assert (np.abs(mass.cpu().numpy() - ref_m) <= MASS_REL * ref_m + 1e-30).all()
+
+
+@pytest.mark.parametrize("T,E", [(193, 128), (300, 256), (576, 128), (577, 128), (2048, 128), (2432, 256),
+                                 (2433, 128), (16384, 128), (100, 128)])
+def test_router_logits_k_split(T, E):
+    """The workspace router (k slices on the tensor cores, partial sums added
+    in slice order, the bias last) stays within the fp32 summation bound at
+    every slice count it picks (16, 4, or none)."""
+    d = 2048
+    g = torch.Generator().manual_seed(T + 7 * E)
+    x = torch.randn(T, d, generator=g).to(torch.bfloat16)
+    w = (torch.randn(E, d, generator=g) * 0.02).to(torch.bfloat16)
+    b = _zipf_bias(E)
+    lg = torch.full((T, E), float("nan"), dtype=torch.float32, device=DEV)
+    ws = dm.workspace(dm.decomoe_router_logits_ws_bytes(T, d, E), DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    dm.decomoe_router_logits_ws(x.to(DEV), w.to(DEV), b.to(DEV), lg, ws, status)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(status) == 0
+    x64, w64, b64 = f64(x), f64(w), b.numpy().astype(np.float64)
+    rows = np.arange(T) if T <= 2433 else np.random.default_rng(T).choice(T, 512, replace=False)
+    ref = O.router_logits(x64[rows], w64, b64).astype(np.float64)
+    err = np.abs(f64(lg)[rows] - ref)
+    assert np.isfinite(f64(lg)).all()
+    assert (err <= logit_error_bound(x64[rows], w64, b64)).all(), f"max err {err.max():.3e}"
