@@ -17,6 +17,7 @@ instead (the reference arm), on bounded token samples of the same workload.
 Multi-GPU (torchrun): independent replicas, no collective on the data path.
 """
 import argparse
+import types
 import json
 import os
 import statistics
@@ -599,11 +600,26 @@ def run_large(dm, ws, pk, n):
             ms, _ = timed(lambda i, ev: gr.replay(), nn, 3, ws)
             ms_step = ms / nn
             fl = 6.0 * wl.T * wl.k * wl.d * wl.m + 2.0 * wl.T * wl.d * wl.E
+            # the expert FFN alone: the same layer as separate C-ABI calls, with
+            # events captured around the two expert GEMMs
+            Bl = Buffers(wl, wl.T, dev, dm)
+            lv = types.SimpleNamespace(x=g["x"], w_r=g["w_r"], bias=g["bias"], w_gu=w_gu, w_down=g["w_down"])
+            evs = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(3)]
+            gr2 = dm.capture_graph(lambda K=K: run_step(dm, wl, lv, Bl, K, 0, 0, None, evs))
+            ffn = []
+            for _ in range(5):
+                gr2.replay()
+                torch.cuda.synchronize()
+                ffn.append(evs[0].elapsed_time(evs[2]))
+            ffn_ms = statistics.median(ffn)
+            ffn_fl = 6.0 * wl.T * wl.k * wl.d * wl.m
             out.append({"mode": "large T=16384", "zipf_s": zipf, "K": K, "fraction": f,
                         "ms_per_step": round(ms_step, 4), "tokens_per_s": round(wl.T / (ms_step * 1e-3), 1),
                         "step_tflops": round(fl / (ms_step * 1e-3) / 1e12, 2),
+                        "ffn_ms": round(ffn_ms, 4), "ffn_tflops": round(ffn_fl / (ffn_ms * 1e-3) / 1e12, 1),
+                        "ffn_tensor_frac": round(ffn_fl / (ffn_ms * 1e-3) / 1e12 / pk["bf16_tflops"], 4),
                         "includes": "layer + hidden and 2x48-layer KV compaction (1.61 GB in)"})
-            del gr
+            del gr, gr2, Bl
         del g, w_gu, lws
     del kv, kv_out
     torch.cuda.empty_cache()
