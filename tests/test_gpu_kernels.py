@@ -135,7 +135,15 @@ def _idx_pattern(T, k, K, pattern, seed):
         return np.full((T, k), K - 1, np.int64)
     if pattern == "uniform":
         return r.integers(0, K, size=(T, k))
+    if pattern == "sizes":  # k = 1, expert e routed SIZES[e] tokens, in random token order
+        assert k == 1 and K == len(SIZES) and T == sum(SIZES)
+        return r.permutation(np.repeat(np.arange(K), SIZES))[:, None].astype(np.int64)
     raise ValueError(pattern)
+
+
+# expert row counts around the swapped-tile boundaries: 16-row MMA widths, the
+# 32-token epilogue chunks, the 128-row threshold and empty experts
+SIZES = [1, 15, 16, 17, 31, 32, 33, 63, 64, 65, 96, 127, 128, 129, 200, 0, 5]
 
 
 DISPATCH_CASES = [
@@ -211,6 +219,8 @@ EXPERT_CASES = [
     (8, 8, 64, 2048, 768, "route"),       # decode T=8 (64 rows)
     (9, 8, 64, 2048, 768, "route"),       # 72 rows: smallest tensor-core case
     (40, 2, 4, 2048, 768, "one_expert"),  # decode path, 40 rows on one expert (> 8 per chunk)
+    (sum(SIZES), 1, len(SIZES), 2048, 768, "sizes"),  # swapped (<= 128 rows) and tokens-as-M experts
+    (sum(SIZES), 1, len(SIZES), 256, 128, "sizes"),   # one N-tile per GEMM
 ]
 
 
