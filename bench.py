@@ -34,7 +34,10 @@ sys.path.insert(0, ROOT)
 
 import workloads as W  # noqa: E402
 
-LAUNCHES_PER_STEP = 11  # router 2 (k slices + reduction), route+mass 2, dispatch 3, gate/up, down, combine, compaction
+# at T=2048: router k slices, routing (reads the slices) with mass partials,
+# dispatch 3 (histogram + mass sum, ranks, row gather), gate/up, down,
+# combine, compaction
+LAUNCHES_PER_STEP = 9
 # (plus two 4-byte memsets zeroing the expert GEMMs' tile counter)
 
 
@@ -207,6 +210,7 @@ class Buffers:
         self.perm = torch.empty(R, dtype=torch.int32, device=dev)
         self.inv = torch.empty(R, dtype=torch.int32, device=dev)
         self.rd_ws = dm.workspace(dm.decomoe_route_dispatch_workspace_bytes(T, k, E), dev)
+        self.rrd_ws = dm.workspace(dm.decomoe_router_route_dispatch_workspace_bytes(T, wl.d, E, k), dev)
         self.x_perm = torch.empty(R, d, dtype=torch.bfloat16, device=dev)
         self.h = torch.empty(R, m, dtype=torch.bfloat16, device=dev)
         self.y = torch.empty(R, d, dtype=torch.bfloat16, device=dev)
@@ -215,11 +219,12 @@ class Buffers:
 
 
 def run_step(dm, wl, L, B, K, v0, nv, text, ev=None):
-    """One pass of the hot path, every step a C-ABI call (10 kernel launches)."""
+    """One pass of the hot path, every step a C-ABI call."""
     k, E = wl.k, wl.E
-    dm.decomoe_router_logits_ws(L.x, L.w_r, L.bias, B.logits, B.router_ws, B.status)   # a1
-    dm.decomoe_route_dispatch(B.logits, K, k, B.idx, B.w, L.x, B.counts[:K], B.offsets[:K + 1], B.perm, B.inv,
-                              B.x_perm, B.rd_ws, mass_out=B.mass, status=B.status)   # a2 (Eq. 11) + a4 + a5
+    # a1 + a2 (Eq. 11) + a4 + a5: router logits, routing with the activated
+    # mass, dispatch
+    dm.decomoe_router_route_dispatch(L.x, L.w_r, L.bias, B.logits, K, k, B.idx, B.w, B.counts[:K], B.offsets[:K + 1],
+                                     B.perm, B.inv, B.x_perm, B.rrd_ws, mass_out=B.mass, status=B.status)
     if ev is not None:
         ev[0].record()
     dm.decomoe_expert_gate_up(B.x_perm, B.offsets[:K + 1], K, L.w_gu, B.h, B.status)  # a6 gate/up

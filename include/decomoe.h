@@ -195,6 +195,32 @@ DECOMOE_API int decomoe_route_dispatch(const float* logits, int64_t T, int E, in
                                        size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream);
 
 /* ------------------------------------------------------------------------
+ * a1-a5 in one call: the router logits over the full pool (Eq. 10's input),
+ * then decomoe_route_dispatch on them. Outputs (logits included) are
+ * bit-identical to decomoe_router_logits_ws followed by
+ * decomoe_route_dispatch with the same arguments. Where the router splits
+ * its k loop (bf16, 192 < T, k slices that fit the SMs), the routing kernel
+ * reads the router's partial sums itself, adding them in slice order and the
+ * bias last exactly as the router's own reduction does, and writes the summed
+ * logits; with a fixed K and mass_out the activated mass is added up by the
+ * dispatch launch. Two launches fewer than the separate calls.
+ * x: [T, d] dtype; w_r: [E, d] dtype; bias: [E] fp32 or NULL; logits: [T, E]
+ * fp32 output (required). K, k, p, topk_idx, topk_w, mass_out, K_dev,
+ * counts, offsets, perm_token, inv_slot, x_perm: as decomoe_route_dispatch
+ * (x, d and dtype are the dispatch's too).
+ * ws: decomoe_router_route_dispatch_workspace_bytes(T, d, E, k) bytes, 16-byte
+ * aligned (the split router's partials, then the routing and dispatch
+ * scratch). No host synchronisation; capturable in a CUDA graph.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API size_t decomoe_router_route_dispatch_workspace_bytes(int64_t T, int d, int E, int k);
+DECOMOE_API int decomoe_router_route_dispatch(const void* x, const void* w_r, const float* bias, int64_t T,
+                                              int d, int E, int dtype, int K, int k, double p, float* logits,
+                                              int32_t* topk_idx, float* topk_w, double* mass_out,
+                                              int32_t* K_dev, int32_t* counts, int32_t* offsets,
+                                              int32_t* perm_token, int32_t* inv_slot, void* x_perm, void* ws,
+                                              size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * Allocation-free dispatch (the paper has no counterpart: this is a library
  * convenience). Same arguments, outputs and errors as decomoe_dispatch, minus
  * the workspace: for callers that cannot allocate device memory, e.g. a

@@ -55,6 +55,9 @@ SIGNATURES = {
     "decomoe_route_dispatch_workspace_bytes": (_S, [_L, _I, _I]),
     "decomoe_route_dispatch": (_I, [_P, _L, _I, _I, _I, _D, _P, _P, _P, _P, _P, _I, _I, _P, _P, _P, _P, _P, _P, _S,
                                     _P, _P]),
+    "decomoe_router_route_dispatch_workspace_bytes": (_S, [_L, _I, _I, _I]),
+    "decomoe_router_route_dispatch": (_I, [_P, _P, _P, _L, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P, _P, _P, _P, _P,
+                                           _P, _P, _S, _P, _P]),
     "decomoe_savb_gate_workspace_bytes": (_S, [_I, _I]),
     "decomoe_savb_gate": (_I, [_P, _L, _I, _I, _L, _L, _P, _P, _P, _P, _I, _F, _P, _P, _P, _S, _P]),
     "decomoe_calib_workspace_bytes": (_S, [_L, _I]),
@@ -262,6 +265,27 @@ def decomoe_route_dispatch(logits, K, k, topk_idx, topk_w, x, counts, offsets, p
                                         _ptr(perm_token), _ptr(inv_slot), _ptr(x_perm), _ptr(ws),
                                         0 if ws is None else ws.numel() * ws.element_size(), _ptr(status),
                                         _stream(stream)))
+
+
+def decomoe_router_route_dispatch_workspace_bytes(T, d, E, k):
+    return int(lib().decomoe_router_route_dispatch_workspace_bytes(T, d, E, k))
+
+
+def decomoe_router_route_dispatch(x, w_r, bias, logits, K, k, topk_idx, topk_w, counts, offsets, perm_token,
+                                  inv_slot, x_perm, ws, p=0.0, mass_out=None, K_dev=None, status=None, stream=None):
+    """Router logits, routing and dispatch in one call (the same results as
+    decomoe_router_logits_ws followed by decomoe_route_dispatch)."""
+    _need_cuda(x, w_r, bias, logits, topk_idx, topk_w, counts, offsets, perm_token, inv_slot, x_perm, ws, mass_out,
+               K_dev, status)
+    T, d = x.shape
+    E = w_r.shape[0]
+    _check("decomoe_router_route_dispatch",
+           lib().decomoe_router_route_dispatch(_ptr(x), _ptr(w_r), _ptr(bias), T, d, E, _dt(x), K, k, float(p),
+                                               _ptr(logits), _ptr(topk_idx), _ptr(topk_w), _ptr(mass_out),
+                                               _ptr(K_dev), _ptr(counts), _ptr(offsets), _ptr(perm_token),
+                                               _ptr(inv_slot), _ptr(x_perm), _ptr(ws),
+                                               0 if ws is None else ws.numel() * ws.element_size(), _ptr(status),
+                                               _stream(stream)))
 
 
 def decomoe_dispatch(topk_idx, K, x, counts, offsets, perm_token, inv_slot, x_perm, ws, status=None,

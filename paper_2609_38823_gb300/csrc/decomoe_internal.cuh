@@ -95,10 +95,61 @@ int launch_router_split(const void* x, const void* w_r, const float* bias, int64
 int launch_skip_mass(const float* logits, int64_t n, int E, int64_t ld, int k, int64_t skip_at, int64_t skip_len,
                      double* part, double* mass, cudaStream_t s);
 
+// Where the routing kernel reads its logits: row t is
+// parts[t*ld + e] + parts[part_stride + t*ld + e] + ... (nparts slices, in
+// slice order) + bias[e] (when bias is set), the sum the k-split router's
+// reduction forms, so routing can read the router's partial sums directly;
+// logits_out (optional) receives the summed rows. Plain logits: nparts = 1,
+// no bias, no logits_out.
+struct RouteSrc {
+  int nparts = 1;
+  int64_t part_stride = 0;
+  const float* bias = nullptr;
+  float* logits_out = nullptr;
+};
+// decomoe_route_prefix reading its logits through src. defer_finalize: with
+// mass_out and more than one routing block, the per-block partial masses are
+// left in the workspace (their count returned in *mass_blocks) for a later
+// kernel to add up (launch_dispatch's extra blocks) instead of a separate
+// finalize launch.
+int route_prefix_src(const float* logits, const RouteSrc& src, int64_t T, int E, int64_t ld, int K, int k,
+                     int32_t* topk_idx, float* topk_w, double* mass_out, void* ws, size_t ws_bytes,
+                     bool defer_finalize, int* mass_blocks, cudaStream_t s);
+// decomoe_dispatch that also finishes a deferred activated mass: mass[e] =
+// fixed-order fp64 sum of mass_part[b][e] over mass_blocks blocks (no-op when
+// mass_part is null).
+int dispatch_with_mass(const int32_t* topk_idx, int64_t T, int k, int K, const void* x, int d, int dtype,
+                       int32_t* counts, int32_t* offsets, int32_t* perm_token, int32_t* inv_slot, void* x_perm,
+                       void* ws, size_t ws_bytes, int32_t* status_dev, const double* mass_part, int mass_blocks,
+                       int mass_E, double* mass, cudaStream_t s);
+// The k-split router's GEMM alone: KS slices of partial logits [KS][T][E]
+// (no bias) into scratch; returns KS (1: no split at this size, nothing
+// launched).
+int launch_router_parts(const void* x, const void* w_r, int64_t T, int d, int E, float* scratch, int32_t* status,
+                        cudaStream_t s, int* ks_out);
+
 // ---------------------------------------------------------------- device side
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// Activated mass of expert e (Eq. 11) from the routing blocks' partial sums,
+// by one block of 256 threads: thread i adds blocks i, i + 256, ... in order,
+// then a fixed-shape tree combines the 256 thread sums (bit-reproducible, the
+// same order wherever it runs).
+__device__ __forceinline__ void mass_finalize_block(const double* __restrict__ part, int nblocks, int E, int e,
+                                                    double* __restrict__ mass) {
+  __shared__ double red[256];
+  double acc = 0.0;
+  for (int b = threadIdx.x; b < nblocks; b += 256) acc += part[static_cast<int64_t>(b) * E + e];
+  red[threadIdx.x] = acc;
+  __syncthreads();
+  for (int w = 128; w > 0; w >>= 1) {
+    if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) mass[e] = red[0];
 }
 
 __device__ __forceinline__ uint64_t globaltimer_ns() {

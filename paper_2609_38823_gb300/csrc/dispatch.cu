@@ -13,11 +13,26 @@ constexpr int DSP_WARPS = DSP_THREADS / 32;
 constexpr int DSP_PER_WARP = 128;                   // consecutive pairs per warp
 constexpr int DSP_TILE = DSP_WARPS * DSP_PER_WARP;  // pairs per block (1024)
 
-// Pass 1: histogram of expert ids in each tile of DSP_TILE consecutive pairs.
+// Deferred activated mass (Eq. 11) carried by a dispatch launch: blocks
+// [first, first + E) of the grid add up the routing blocks' partial masses,
+// one expert each, in the fixed order of mass_finalize_block.
+struct MassFinish {
+  const double* part = nullptr;  // null: nothing to finish
+  int nblocks = 0;
+  int E = 0;
+  double* mass = nullptr;
+};
+
+// Pass 1: histogram of expert ids in each tile of DSP_TILE consecutive pairs
+// (blocks [0, ntiles)); blocks from ntiles on finish a deferred mass.
 __global__ void __launch_bounds__(DSP_THREADS)
     k_dispatch_hist(const int32_t* __restrict__ idx, int64_t N, int K,
-                    int32_t* __restrict__ tile_hist, int32_t* status) {
+                    int32_t* __restrict__ tile_hist, int32_t* status, int ntiles, MassFinish mf) {
   pdl_enter();
+  if (static_cast<int>(blockIdx.x) >= ntiles) {
+    mass_finalize_block(mf.part, mf.nblocks, mf.E, static_cast<int>(blockIdx.x) - ntiles, mf.mass);
+    return;
+  }
   __shared__ int hist[DECOMOE_MAX_E];
   for (int e = threadIdx.x; e < K; e += DSP_THREADS) hist[e] = 0;
   __syncthreads();
@@ -48,7 +63,8 @@ __global__ void __launch_bounds__(DSP_THREADS)
 // come from __match_any_sync, and per-warp running counts are scanned across
 // warps. Writes perm_token and inv_slot; block 0 writes counts and offsets.
 // SINGLE: one tile in one block (decode sizes): the block also counts the
-// histogram itself and may copy the rows (x_perm != null).
+// histogram itself and may copy the rows (x_perm != null); blocks from 1 on
+// finish a deferred mass.
 template <bool SINGLE>
 __global__ void __launch_bounds__(DSP_THREADS)
     k_dispatch_scatter(const int32_t* __restrict__ idx, int64_t N, int k, int K,
@@ -56,8 +72,12 @@ __global__ void __launch_bounds__(DSP_THREADS)
                        int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
                        int32_t* __restrict__ perm_token, int32_t* __restrict__ inv_slot,
                        int32_t* status = nullptr, const uint4* __restrict__ x = nullptr, int row_vec = 0,
-                       uint4* __restrict__ x_perm = nullptr) {
+                       uint4* __restrict__ x_perm = nullptr, MassFinish mf = MassFinish{}) {
   pdl_enter();
+  if (SINGLE && blockIdx.x > 0) {
+    mass_finalize_block(mf.part, mf.nblocks, mf.E, static_cast<int>(blockIdx.x) - 1, mf.mass);
+    return;
+  }
   __shared__ int s_base[DECOMOE_MAX_E];
   __shared__ int s_wcnt[DSP_WARPS][DECOMOE_MAX_E];
   __shared__ int s_wsum[DSP_WARPS];
@@ -233,13 +253,34 @@ int decomoe_dispatch(const int32_t* topk_idx, int64_t T, int k, int K, const voi
                      int32_t* inv_slot, void* x_perm, void* ws, size_t ws_bytes,
                      int32_t* status_dev, decomoe_stream_t stream) {
   clear_error();
+  return dispatch_with_mass(topk_idx, T, k, K, x, d, dtype, counts, offsets, perm_token, inv_slot, x_perm, ws,
+                            ws_bytes, status_dev, nullptr, 0, 0, nullptr, reinterpret_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"
+
+namespace decomoe {
+
+int dispatch_with_mass(const int32_t* topk_idx, int64_t T, int k, int K, const void* x, int d, int dtype,
+                       int32_t* counts, int32_t* offsets, int32_t* perm_token, int32_t* inv_slot, void* x_perm,
+                       void* ws, size_t ws_bytes, int32_t* status_dev, const double* mass_part, int mass_blocks,
+                       int mass_E, double* mass, cudaStream_t s) {
+  MassFinish mf;
+  if (mass_part != nullptr && mass_blocks > 0) {
+    DM_ARG_CHECK(mass != nullptr && mass_E >= 1 && mass_E <= DECOMOE_MAX_E, "dispatch: bad deferred mass");
+    mf.part = mass_part;
+    mf.nblocks = mass_blocks;
+    mf.E = mass_E;
+    mf.mass = mass;
+  }
+  const int mblocks = mf.part != nullptr ? mf.E : 0;
   DM_ARG_CHECK(T >= 0 && k >= 1 && k <= DECOMOE_MAX_TOPK, "dispatch: bad T=%lld or k=%d", (long long)T, k);
   DM_ARG_CHECK(K >= 1 && K <= DECOMOE_MAX_E, "dispatch: K=%d outside [1, %d]", K, DECOMOE_MAX_E);
   DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "dispatch: bad dtype");
   DM_ARG_CHECK(counts && offsets, "dispatch: counts/offsets null");
   const int64_t N = T * k;
   DM_ARG_CHECK(N < 0x7fffffffLL, "dispatch: T*k too large");
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  DM_ARG_CHECK(N > 0 || mblocks == 0, "dispatch: a deferred mass needs routed pairs");
   if (N == 0) {
     DM_CUDA_CHECK(cudaMemsetAsync(counts, 0, sizeof(int32_t) * K, s));
     DM_CUDA_CHECK(cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (K + 1), s));
@@ -262,18 +303,18 @@ int decomoe_dispatch(const int32_t* topk_idx, int64_t T, int k, int K, const voi
     // one tile (decode sizes): count, scan and rank in one block, and copy
     // the rows there too when they are few
     const bool gather_here = x_perm != nullptr && static_cast<size_t>(N) * row_bytes <= 64 * 1024;
-    DM_CUDA_CHECK(launch_pdl(k_dispatch_scatter<true>, dim3(1), dim3(DSP_THREADS), 0, s, topk_idx, N, k, K,
-                             static_cast<const int32_t*>(nullptr), 1, counts, offsets, perm_token, inv_slot,
+    DM_CUDA_CHECK(launch_pdl(k_dispatch_scatter<true>, dim3(1 + mblocks), dim3(DSP_THREADS), 0, s, topk_idx, N,
+                             k, K, static_cast<const int32_t*>(nullptr), 1, counts, offsets, perm_token, inv_slot,
                              status_dev, static_cast<const uint4*>(x), static_cast<int>(row_bytes / 16),
-                             gather_here ? static_cast<uint4*>(x_perm) : static_cast<uint4*>(nullptr)));
+                             gather_here ? static_cast<uint4*>(x_perm) : static_cast<uint4*>(nullptr), mf));
     if (gather_here) return DECOMOE_OK;
   } else {
-    DM_CUDA_CHECK(launch_pdl(k_dispatch_hist, dim3(ntiles), dim3(DSP_THREADS), 0, s, topk_idx, N, K, tile_hist,
-                             status_dev));
+    DM_CUDA_CHECK(launch_pdl(k_dispatch_hist, dim3(ntiles + mblocks), dim3(DSP_THREADS), 0, s, topk_idx, N, K,
+                             tile_hist, status_dev, ntiles, mf));
     DM_CUDA_CHECK(launch_pdl(k_dispatch_scatter<false>, dim3(ntiles), dim3(DSP_THREADS), 0, s, topk_idx, N, k, K,
                              static_cast<const int32_t*>(tile_hist), ntiles, counts, offsets, perm_token, inv_slot,
                              static_cast<int32_t*>(nullptr), static_cast<const uint4*>(nullptr), 0,
-                             static_cast<uint4*>(nullptr)));
+                             static_cast<uint4*>(nullptr), MassFinish{}));
   }
   if (x_perm != nullptr) {
     const int vec = static_cast<int>(row_bytes / 16);
@@ -287,7 +328,7 @@ int decomoe_dispatch(const int32_t* topk_idx, int64_t T, int k, int K, const voi
   return DECOMOE_OK;
 }
 
-}  // extern "C"
+}  // namespace decomoe
 
 // ---------------------------------------------------------------------------
 // Allocation-free dispatch.
@@ -367,7 +408,7 @@ extern "C" int decomoe_dispatch_noalloc(const int32_t* topk_idx, int64_t T, int 
   // left in the array by an earlier call is ever used.
   const int ntiles = static_cast<int>(ntiles64);
   DM_CUDA_CHECK(launch_pdl(k_dispatch_hist, dim3(ntiles), dim3(DSP_THREADS), 0, s, topk_idx, N, K, tile_hist,
-                           status_dev));
+                           status_dev, ntiles, MassFinish{}));
   k_dispatch_scatter<false><<<ntiles, DSP_THREADS, 0, s>>>(topk_idx, N, k, K, tile_hist, ntiles, counts, offsets,
                                                     perm_token, inv_slot);
   DM_LAUNCH_CHECK("k_dispatch_scatter");

@@ -1262,6 +1262,26 @@ static int launch_router_split_ks(const void* x, const void* w_r, const float* b
   return DECOMOE_OK;
 }
 
+int launch_router_parts(const void* x, const void* w_r, int64_t T, int d, int E, float* scratch, int32_t* status,
+                        cudaStream_t s, int* ks_out) {
+  const int ks = router_split_ks(T, d, E);
+  *ks_out = ks;
+  const int64_t npad = (T + 63) / 64 * 64;
+  const int64_t n = T * E;
+  switch (ks) {
+    case 16:
+      return launch_tc<64, EPI_F32_BIAS_T, 8, 64, 0, 1, 8, 1, 16>(w_r, E, d, x, T, nullptr, 1, static_cast<int>(npad),
+                                                                  scratch, E, nullptr, status, s, static_cast<int>(T),
+                                                                  nullptr, 0, nullptr, n);
+    case 4:
+      return launch_tc<64, EPI_F32_BIAS_T, 8, 64, 0, 1, 8, 1, 4>(w_r, E, d, x, T, nullptr, 1, static_cast<int>(npad),
+                                                                 scratch, E, nullptr, status, s, static_cast<int>(T),
+                                                                 nullptr, 0, nullptr, n);
+    default:
+      return DECOMOE_OK;  // no split at this size: nothing launched
+  }
+}
+
 int launch_router_split(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E, float* logits,
                         float* scratch, int32_t* status, cudaStream_t s) {
   switch (router_split_ks(T, d, E)) {

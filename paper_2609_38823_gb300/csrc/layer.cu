@@ -28,6 +28,107 @@ enum {
   WS_COUNT
 };
 
+// a2-a5 over logits read through src (plain logits, or the k-split
+// router's partial sums): mass pass, prefix (fixed, or Eq. 12 on the
+// device), prefix routing and dispatch. With a fixed prefix and mass_out the
+// activated mass is finished by the dispatch launch's extra blocks.
+static int route_dispatch_src(const float* logits, const RouteSrc& src, int64_t T, int E, int K, int k, double p,
+                              int32_t* topk_idx, float* topk_w, double* mass_out, int32_t* K_dev, const void* x,
+                              int d, int dtype, int32_t* counts, int32_t* offsets, int32_t* perm_token,
+                              int32_t* inv_slot, void* x_perm, void* ws, size_t ws_bytes, int32_t* status_dev,
+                              cudaStream_t s) {
+  DM_ARG_CHECK(T >= 0, "route_dispatch: T < 0");
+  DM_ARG_CHECK(E >= 1 && E <= DECOMOE_MAX_E && k >= 1 && k <= DECOMOE_MAX_TOPK && k <= E,
+               "route_dispatch: need 1 <= k <= E <= %d, k <= %d", DECOMOE_MAX_E, DECOMOE_MAX_TOPK);
+  const bool device_k = (K == -1);
+  DM_ARG_CHECK(device_k || (K >= k && K <= E), "route_dispatch: need k <= K <= E or K = -1 (k=%d K=%d E=%d)", k,
+               K, E);
+  if (device_k) {
+    DM_ARG_CHECK(p > 0.0 && p <= 1.0, "route_dispatch: a device-selected prefix needs 0 < p <= 1");
+    DM_ARG_CHECK(mass_out && K_dev, "route_dispatch: a device-selected prefix needs mass_out and K_dev");
+  }
+  DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "route_dispatch: bad dtype");
+  DM_ARG_CHECK(counts && offsets, "route_dispatch: counts/offsets null");
+  const int Kd = device_k ? E : K;
+  decomoe_stream_t stream = reinterpret_cast<decomoe_stream_t>(s);
+  if (T == 0) {
+    DM_CUDA_CHECK(cudaMemsetAsync(counts, 0, sizeof(int32_t) * Kd, s));
+    DM_CUDA_CHECK(cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (Kd + 1), s));
+    if (mass_out) DM_CUDA_CHECK(cudaMemsetAsync(mass_out, 0, sizeof(double) * E, s));
+    if (device_k) return decomoe_select_prefix_device(mass_out, E, k, p, K_dev, stream);  // zero mass: K = k
+    return DECOMOE_OK;
+  }
+  DM_ARG_CHECK(logits && topk_idx && topk_w && perm_token && inv_slot, "route_dispatch: null pointer");
+  DM_ARG_CHECK(T * static_cast<int64_t>(k) < 0x7fffffffLL, "route_dispatch: T*k too large");
+  const size_t row_bytes = static_cast<size_t>(d) * dtype_bytes(dtype);
+  if (x_perm != nullptr) {
+    DM_ARG_CHECK(x != nullptr && d > 0, "route_dispatch: x null or d <= 0");
+    DM_ARG_CHECK(row_bytes % 16 == 0 && aligned16(x) && aligned16(x_perm),
+                 "route_dispatch: rows must be 16-byte multiples and 16-byte aligned");
+  }
+  const size_t rbytes = align_up(decomoe_route_workspace_bytes(T, E), 256);
+  const size_t dbytes = decomoe_dispatch_workspace_bytes(T, k, E);
+  if (ws == nullptr || ws_bytes < rbytes + dbytes) {
+    set_error("route_dispatch: workspace needs %zu bytes", rbytes + dbytes);
+    return DECOMOE_ERR_WORKSPACE;
+  }
+  void* route_ws = ws;
+  void* disp_ws = static_cast<uint8_t*>(ws) + rbytes;
+  int mass_blocks = 0;
+  if (device_k) {
+    // mass pass, Eq. 12 on the device, routing over [0, *K_dev) (from the
+    // summed logits when the first pass read the router's partials)
+    DM_RET(route_prefix_src(logits, src, T, E, E, E, k, nullptr, nullptr, mass_out, route_ws, rbytes, false, nullptr,
+                            s));
+    DM_RET(decomoe_select_prefix_device(mass_out, E, k, p, K_dev, stream));
+    DM_RET(decomoe_route_prefix_dk(src.logits_out != nullptr ? src.logits_out : logits, T, E, E, K_dev, k, topk_idx,
+                                   topk_w, stream));
+  } else {
+    // one launch: prefix routing and, with mass_out, the full-pool partial
+    // masses (finished by the dispatch launch)
+    DM_RET(route_prefix_src(logits, src, T, E, E, K, k, topk_idx, topk_w, mass_out, route_ws, rbytes, true,
+                            &mass_blocks, s));
+  }
+  return dispatch_with_mass(topk_idx, T, k, Kd, x, d, dtype, counts, offsets, perm_token, inv_slot, x_perm, disp_ws,
+                            dbytes, status_dev, mass_blocks > 0 ? static_cast<const double*>(route_ws) : nullptr,
+                            mass_blocks, E, mass_out, s);
+}
+
+// a1-a5: router logits (as partial sums read by the routing kernel when the
+// router splits its k loop, else written out first), then route_dispatch_src.
+// scratch: the split router's partials (decomoe_router_logits_ws_bytes).
+static int router_route_dispatch_impl(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E,
+                                      int dtype, int K, int k, double p, float* logits, int32_t* topk_idx,
+                                      float* topk_w, double* mass_out, int32_t* K_dev, int32_t* counts,
+                                      int32_t* offsets, int32_t* perm_token, int32_t* inv_slot, void* x_perm,
+                                      float* scratch, void* rd_ws, size_t rd_bytes, int32_t* status_dev,
+                                      cudaStream_t s) {
+  DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "router_route_dispatch: bad dtype");
+  RouteSrc src;
+  const float* lg = logits;
+  if (T > 0) {
+    DM_ARG_CHECK(x && w_r && logits, "router_route_dispatch: null pointer");
+    int ks = 1;
+    if (dtype == DECOMOE_BF16 && decomoe_router_logits_ws_bytes(T, d, E) > 0) {
+      DM_ARG_CHECK(aligned16(x) && aligned16(w_r) && aligned16(scratch),
+                   "router_route_dispatch: pointers must be 16-byte aligned");
+      DM_RET(launch_router_parts(x, w_r, T, d, E, scratch, status_dev, s, &ks));
+    }
+    if (ks > 1) {
+      src.nparts = ks;
+      src.part_stride = T * E;
+      src.bias = bias;
+      src.logits_out = logits;
+      lg = scratch;
+    } else {
+      DM_RET(decomoe_router_logits(x, w_r, bias, T, d, E, dtype, logits, status_dev,
+                                   reinterpret_cast<decomoe_stream_t>(s)));
+    }
+  }
+  return route_dispatch_src(lg, src, T, E, K, k, p, topk_idx, topk_w, mass_out, K_dev, x, d, dtype, counts, offsets,
+                            perm_token, inv_slot, x_perm, rd_ws, rd_bytes, status_dev, s);
+}
+
 struct LayerLayout {
   size_t off[WS_COUNT];
   size_t total;
@@ -94,54 +195,34 @@ int decomoe_route_dispatch(const float* logits, int64_t T, int E, int K, int k, 
                            int32_t* counts, int32_t* offsets, int32_t* perm_token, int32_t* inv_slot, void* x_perm,
                            void* ws, size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream) {
   clear_error();
-  DM_ARG_CHECK(T >= 0, "route_dispatch: T < 0");
-  DM_ARG_CHECK(E >= 1 && E <= DECOMOE_MAX_E && k >= 1 && k <= DECOMOE_MAX_TOPK && k <= E,
-               "route_dispatch: need 1 <= k <= E <= %d, k <= %d", DECOMOE_MAX_E, DECOMOE_MAX_TOPK);
-  const bool device_k = (K == -1);
-  DM_ARG_CHECK(device_k || (K >= k && K <= E), "route_dispatch: need k <= K <= E or K = -1 (k=%d K=%d E=%d)", k,
-               K, E);
-  if (device_k) {
-    DM_ARG_CHECK(p > 0.0 && p <= 1.0, "route_dispatch: a device-selected prefix needs 0 < p <= 1");
-    DM_ARG_CHECK(mass_out && K_dev, "route_dispatch: a device-selected prefix needs mass_out and K_dev");
-  }
-  DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "route_dispatch: bad dtype");
-  DM_ARG_CHECK(counts && offsets, "route_dispatch: counts/offsets null");
-  const int Kd = device_k ? E : K;
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (T == 0) {
-    DM_CUDA_CHECK(cudaMemsetAsync(counts, 0, sizeof(int32_t) * Kd, s));
-    DM_CUDA_CHECK(cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (Kd + 1), s));
-    if (mass_out) DM_CUDA_CHECK(cudaMemsetAsync(mass_out, 0, sizeof(double) * E, s));
-    if (device_k) return decomoe_select_prefix_device(mass_out, E, k, p, K_dev, stream);  // zero mass: K = k
-    return DECOMOE_OK;
-  }
-  DM_ARG_CHECK(logits && topk_idx && topk_w && perm_token && inv_slot, "route_dispatch: null pointer");
-  DM_ARG_CHECK(T * static_cast<int64_t>(k) < 0x7fffffffLL, "route_dispatch: T*k too large");
-  const size_t row_bytes = static_cast<size_t>(d) * dtype_bytes(dtype);
-  if (x_perm != nullptr) {
-    DM_ARG_CHECK(x != nullptr && d > 0, "route_dispatch: x null or d <= 0");
-    DM_ARG_CHECK(row_bytes % 16 == 0 && aligned16(x) && aligned16(x_perm),
-                 "route_dispatch: rows must be 16-byte multiples and 16-byte aligned");
-  }
-  const size_t rbytes = align_up(decomoe_route_workspace_bytes(T, E), 256);
-  const size_t dbytes = decomoe_dispatch_workspace_bytes(T, k, E);
-  if (ws == nullptr || ws_bytes < rbytes + dbytes) {
-    set_error("route_dispatch: workspace needs %zu bytes", rbytes + dbytes);
+  return route_dispatch_src(logits, RouteSrc{}, T, E, K, k, p, topk_idx, topk_w, mass_out, K_dev, x, d, dtype,
+                            counts, offsets, perm_token, inv_slot, x_perm, ws, ws_bytes, status_dev,
+                            reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t decomoe_router_route_dispatch_workspace_bytes(int64_t T, int d, int E, int k) {
+  if (T < 0 || d <= 0 || E <= 0 || k <= 0) return 0;
+  return align_up(decomoe_router_logits_ws_bytes(T, d, E), 256) + decomoe_route_dispatch_workspace_bytes(T, k, E);
+}
+
+int decomoe_router_route_dispatch(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E,
+                                  int dtype, int K, int k, double p, float* logits, int32_t* topk_idx, float* topk_w,
+                                  double* mass_out, int32_t* K_dev, int32_t* counts, int32_t* offsets,
+                                  int32_t* perm_token, int32_t* inv_slot, void* x_perm, void* ws, size_t ws_bytes,
+                                  int32_t* status_dev, decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(T >= 0 && d > 0, "router_route_dispatch: bad sizes");
+  const size_t rs = align_up(decomoe_router_logits_ws_bytes(T, d, E), 256);
+  const size_t need = decomoe_router_route_dispatch_workspace_bytes(T, d, E, k);
+  if (T > 0 && (ws == nullptr || ws_bytes < need)) {
+    set_error("router_route_dispatch: workspace needs %zu bytes", need);
     return DECOMOE_ERR_WORKSPACE;
   }
-  void* route_ws = ws;
-  void* disp_ws = static_cast<uint8_t*>(ws) + rbytes;
-  if (device_k) {
-    // mass pass, Eq. 12 on the device, routing over [0, *K_dev)
-    DM_RET(decomoe_route_prefix(logits, T, E, E, E, k, nullptr, nullptr, mass_out, route_ws, rbytes, stream));
-    DM_RET(decomoe_select_prefix_device(mass_out, E, k, p, K_dev, stream));
-    DM_RET(decomoe_route_prefix_dk(logits, T, E, E, K_dev, k, topk_idx, topk_w, stream));
-  } else {
-    // one launch: prefix routing and, with mass_out, the full-pool mass
-    DM_RET(decomoe_route_prefix(logits, T, E, E, K, k, topk_idx, topk_w, mass_out, route_ws, rbytes, stream));
-  }
-  return decomoe_dispatch(topk_idx, T, k, Kd, x, d, dtype, counts, offsets, perm_token, inv_slot, x_perm, disp_ws,
-                          dbytes, status_dev, stream);
+  return router_route_dispatch_impl(x, w_r, bias, T, d, E, dtype, K, k, p, logits, topk_idx, topk_w, mass_out, K_dev,
+                                    counts, offsets, perm_token, inv_slot, x_perm,
+                                    T > 0 ? static_cast<float*>(ws) : nullptr,
+                                    T > 0 ? static_cast<uint8_t*>(ws) + rs : nullptr, T > 0 ? ws_bytes - rs : 0,
+                                    status_dev, reinterpret_cast<cudaStream_t>(stream));
 }
 
 int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const void* w_gate_up,
@@ -185,28 +266,27 @@ int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const v
   void* y_perm = base + L.off[WS_YPERM];
   void* route_ws = base + L.off[WS_ROUTE];  // routing and dispatch scratch
 
-  // a1: router logits over all E reordered experts
-  DM_RET(decomoe_router_logits_ws(x, w_r, bias, T, d, E, dtype, logits, base + L.off[WS_RSPLIT],
-                                  decomoe_router_logits_ws_bytes(T, d, E), status_dev, stream));
-  // a2 (+ a3) and a4: full-pool activated mass and prefix routing
   int K = K_fixed;
   int32_t* K_dev = reinterpret_cast<int32_t*>(base + L.off[WS_KDEV]);
+  float* rsplit = reinterpret_cast<float*>(base + L.off[WS_RSPLIT]);
   if (K_fixed != 0) {
-    // a2-a5: full-pool mass (Eq. 11), prefix (fixed, or Eq. 12 on the
-    // device), prefix routing and dispatch; with a device-selected prefix,
-    // dispatch and the experts run over all E groups (those at or beyond
-    // *K_dev are empty)
-    DM_RET(decomoe_route_dispatch(logits, T, E, K_fixed, k, p, topk_idx, topk_w,
-                                  (K_fixed == -1 || p > 0.0) ? mass : nullptr, K_dev, x, d, dtype, counts, offsets,
-                                  perm, inv, x_perm, route_ws, L.off[WS_KDEV] - L.off[WS_ROUTE], status_dev,
-                                  stream));
+    // a1-a5: router logits over all E reordered experts, full-pool mass
+    // (Eq. 11), prefix (fixed, or Eq. 12 on the device), prefix routing and
+    // dispatch; with a device-selected prefix, dispatch and the experts run
+    // over all E groups (those at or beyond *K_dev are empty)
+    DM_RET(router_route_dispatch_impl(x, w_r, bias, T, d, E, dtype, K_fixed, k, p, logits, topk_idx, topk_w,
+                                      (K_fixed == -1 || p > 0.0) ? mass : nullptr, K_dev, counts, offsets, perm, inv,
+                                      x_perm, rsplit, route_ws, L.off[WS_KDEV] - L.off[WS_ROUTE], status_dev, s));
     if (K_fixed == -1) {
       K = E;
       if (K_sel_host) *K_sel_host = -1;
       if (K_used_host) *K_used_host = -1;
     }
   } else {
-    // host-selected prefix: mass pass, one device-to-host read, Eq. 12 in C
+    // host-selected prefix: router logits, mass pass, one device-to-host
+    // read, Eq. 12 in C
+    DM_RET(decomoe_router_logits_ws(x, w_r, bias, T, d, E, dtype, logits, rsplit,
+                                    decomoe_router_logits_ws_bytes(T, d, E), status_dev, stream));
     DM_RET(decomoe_route_prefix(logits, T, E, E, E, k, nullptr, nullptr, mass, route_ws,
                                 decomoe_route_workspace_bytes(T, E), stream));
     static thread_local std::vector<double> h_mass;

@@ -171,7 +171,7 @@ __device__ __forceinline__ float pick_weight(float my_v, int lane, int k) {
 __global__ void __launch_bounds__(ROUTE_THREADS)
     k_route(const float* __restrict__ logits, int64_t Tn, int E, int64_t ld, int K, int k,
             int32_t* __restrict__ idx_out, float* __restrict__ w_out, double* __restrict__ part,
-            const int32_t* __restrict__ K_dev, int64_t skip_at = INT64_MAX, int64_t skip_len = 0) {
+            const int32_t* __restrict__ K_dev, int64_t skip_at, int64_t skip_len, RouteSrc src) {
   pdl_enter();
   if (K_dev != nullptr) K = *K_dev;  // prefix chosen on the device (k <= K <= E by construction)
   __shared__ int s_idx[ROUTE_TPB][DECOMOE_MAX_TOPK];
@@ -182,13 +182,30 @@ __global__ void __launch_bounds__(ROUTE_THREADS)
   if (t < Tn) {
     // token t reads logit row t, or t + skip_len from skip_at on (the text
     // tokens around a removed visual block)
-    const float* row = logits + (t < skip_at ? t : t + skip_len) * ld;
+    const int64_t roff = (t < skip_at ? t : t + skip_len) * ld;
+    const float* row = logits + roff;
     const int lim = mass ? E : K;
     uint32_t v[8];  // order-preserving keys of the row's logits
+    if (src.nparts == 1 && src.bias == nullptr && src.logits_out == nullptr) {
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int e = lane + 32 * i;
-      v[i] = (e < lim) ? fkey(row[e]) : 0u;
+      for (int i = 0; i < 8; ++i) {
+        const int e = lane + 32 * i;
+        v[i] = (e < lim) ? fkey(row[e]) : 0u;
+      }
+    } else {
+      // partial sums of the k-split router, added in slice order, bias last
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int e = lane + 32 * i;
+        v[i] = 0u;
+        if (e < E) {
+          float a = row[e];
+          for (int sl = 1; sl < src.nparts; ++sl) a += row[sl * src.part_stride + e];
+          if (src.bias != nullptr) a += src.bias[e];
+          if (src.logits_out != nullptr) src.logits_out[roff + e] = a;
+          if (e < lim) v[i] = fkey(a);
+        }
+      }
     }
     float my_v;
     int my_i;
@@ -231,17 +248,7 @@ __global__ void __launch_bounds__(ROUTE_THREADS)
 __global__ void __launch_bounds__(256)
     k_mass_finalize(const double* __restrict__ part, int nblocks, int E, double* __restrict__ mass) {
   pdl_enter();
-  __shared__ double red[256];
-  const int e = blockIdx.x;
-  double acc = 0.0;
-  for (int b = threadIdx.x; b < nblocks; b += 256) acc += part[static_cast<int64_t>(b) * E + e];
-  red[threadIdx.x] = acc;
-  __syncthreads();
-  for (int w = 128; w > 0; w >>= 1) {
-    if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
-    __syncthreads();
-  }
-  if (threadIdx.x == 0) mass[e] = red[0];
+  mass_finalize_block(part, nblocks, E, static_cast<int>(blockIdx.x), mass);
 }
 
 // Eq. 12, sequentially in fp64 with round-to-nearest adds and division, as
@@ -283,7 +290,7 @@ int launch_skip_mass(const float* logits, int64_t n, int E, int64_t ld, int k, i
                      double* part, double* mass, cudaStream_t s) {
   const int64_t nblocks = (n + ROUTE_TPB - 1) / ROUTE_TPB;
   k_route<<<static_cast<unsigned>(nblocks), ROUTE_THREADS, 0, s>>>(logits, n, E, ld, E, k, nullptr, nullptr, part,
-                                                                   nullptr, skip_at, skip_len);
+                                                                   nullptr, skip_at, skip_len, RouteSrc{});
   DM_LAUNCH_CHECK("k_route");
   k_mass_finalize<<<E, 256, 0, s>>>(part, static_cast<int>(nblocks), E, mass);
   DM_LAUNCH_CHECK("k_mass_finalize");
@@ -363,12 +370,24 @@ int decomoe_route_prefix(const float* logits, int64_t T, int E, int64_t ld, int 
                          int32_t* topk_idx, float* topk_w, double* mass_out, void* ws,
                          size_t ws_bytes, decomoe_stream_t stream) {
   clear_error();
+  return route_prefix_src(logits, RouteSrc{}, T, E, ld, K, k, topk_idx, topk_w, mass_out, ws, ws_bytes, false,
+                          nullptr, reinterpret_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"
+
+namespace decomoe {
+
+int route_prefix_src(const float* logits, const RouteSrc& src, int64_t T, int E, int64_t ld, int K, int k,
+                     int32_t* topk_idx, float* topk_w, double* mass_out, void* ws, size_t ws_bytes,
+                     bool defer_finalize, int* mass_blocks, cudaStream_t s) {
+  if (mass_blocks != nullptr) *mass_blocks = 0;
   DM_ARG_CHECK(T >= 0, "route_prefix: T < 0");
   DM_ARG_CHECK(E >= 1 && E <= DECOMOE_MAX_E, "route_prefix: E=%d outside [1, %d]", E, DECOMOE_MAX_E);
   DM_ARG_CHECK(k >= 1 && k <= DECOMOE_MAX_TOPK, "route_prefix: k=%d outside [1, %d]", k, DECOMOE_MAX_TOPK);
   DM_ARG_CHECK(K >= k && K <= E, "route_prefix: need k <= K <= E (k=%d K=%d E=%d)", k, K, E);
   DM_ARG_CHECK(ld >= E, "route_prefix: ld < E");
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  DM_ARG_CHECK(src.nparts >= 1, "route_prefix: no logit slices");
   if (T == 0) {
     if (mass_out) DM_CUDA_CHECK(cudaMemsetAsync(mass_out, 0, sizeof(double) * E, s));
     return DECOMOE_OK;
@@ -388,12 +407,21 @@ int decomoe_route_prefix(const float* logits, int64_t T, int E, int64_t ld, int 
   }
   DM_CUDA_CHECK(launch_pdl(k_route, dim3(static_cast<unsigned>(nblocks)), dim3(ROUTE_THREADS), 0, s, logits, T, E,
                            ld, K, k, topk_idx, topk_w, part, static_cast<const int32_t*>(nullptr), INT64_MAX,
-                           static_cast<int64_t>(0)));
-  if (mass_out != nullptr && nblocks > 1)
-    DM_CUDA_CHECK(launch_pdl(k_mass_finalize, dim3(E), dim3(256), 0, s, static_cast<const double*>(part),
-                             static_cast<int>(nblocks), E, mass_out));
+                           static_cast<int64_t>(0), src));
+  if (mass_out != nullptr && nblocks > 1) {
+    if (defer_finalize && mass_blocks != nullptr) {
+      *mass_blocks = static_cast<int>(nblocks);  // the caller's next kernel adds the partials up
+    } else {
+      DM_CUDA_CHECK(launch_pdl(k_mass_finalize, dim3(E), dim3(256), 0, s, static_cast<const double*>(part),
+                               static_cast<int>(nblocks), E, mass_out));
+    }
+  }
   return DECOMOE_OK;
 }
+
+}  // namespace decomoe
+
+extern "C" {
 
 
 int decomoe_select_prefix_device(const double* mass, int E, int k, double p, int32_t* K_dev,
@@ -418,7 +446,7 @@ int decomoe_route_prefix_dk(const float* logits, int64_t T, int E, int64_t ld, c
   DM_ARG_CHECK(nblocks <= 0x7fffffff, "route_prefix_dk: T too large");
   DM_CUDA_CHECK(launch_pdl(k_route, dim3(static_cast<unsigned>(nblocks)), dim3(ROUTE_THREADS), 0,
                            reinterpret_cast<cudaStream_t>(stream), logits, T, E, ld, E, k, topk_idx, topk_w,
-                           static_cast<double*>(nullptr), K_dev, INT64_MAX, static_cast<int64_t>(0)));
+                           static_cast<double*>(nullptr), K_dev, INT64_MAX, static_cast<int64_t>(0), RouteSrc{}));
   return DECOMOE_OK;
 }
 

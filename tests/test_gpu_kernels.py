@@ -489,3 +489,54 @@ def test_router_logits_k_split(T, E):
     err = np.abs(f64(lg)[rows] - ref)
     assert np.isfinite(f64(lg)).all()
     assert (err <= logit_error_bound(x64[rows], w64, b64)).all(), f"max err {err.max():.3e}"
+
+
+@pytest.mark.parametrize("T,E,K,p", [(1, 128, 64, 0.7), (100, 128, 64, 0.7), (193, 128, 64, 0.7), (300, 256, -1, 0.7),
+                                     (576, 128, 64, 0.0), (577, 128, -1, 0.5), (2048, 128, 64, 0.7),
+                                     (2048, 128, -1, 0.7), (2432, 256, 40, 0.7), (2433, 128, 64, 0.7),
+                                     (4096, 128, -1, 0.9)])
+def test_router_route_dispatch_equals_separate_calls(T, E, K, p):
+    """The one-call front half (router logits, routing, dispatch) equals
+    decomoe_router_logits_ws + decomoe_route_dispatch bit for bit, whether
+    the routing kernel reads the split router's partial sums (193 <= T <=
+    2432) or plain logits, with the mass finished by the dispatch launch or by
+    its own kernel."""
+    d, k = 2048, 8
+    g = torch.Generator().manual_seed(T + 3 * E)
+    x = torch.randn(T, d, generator=g).to(torch.bfloat16).to(DEV)
+    w_r = (torch.randn(E, d, generator=g) * 0.02).to(torch.bfloat16).to(DEV)
+    bias = _zipf_bias(E).to(DEV)
+    Kd = E if K == -1 else K
+
+    def outs():
+        return dict(logits=torch.empty(T, E, device=DEV), idx=torch.full((T, k), -9, dtype=torch.int32, device=DEV),
+                    w=torch.empty(T, k, device=DEV), mass=torch.full((E,), -1.0, dtype=torch.float64, device=DEV),
+                    Kdev=torch.zeros(1, dtype=torch.int32, device=DEV),
+                    counts=torch.empty(Kd, dtype=torch.int32, device=DEV),
+                    offsets=torch.empty(Kd + 1, dtype=torch.int32, device=DEV),
+                    perm=torch.empty(T * k, dtype=torch.int32, device=DEV),
+                    inv=torch.empty(T * k, dtype=torch.int32, device=DEV),
+                    xp=torch.empty(T * k, d, dtype=torch.bfloat16, device=DEV))
+
+    a, b = outs(), outs()
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    ws = dm.workspace(dm.decomoe_router_route_dispatch_workspace_bytes(T, d, E, k), DEV)
+    dm.decomoe_router_route_dispatch(x, w_r, bias, a["logits"], K, k, a["idx"], a["w"], a["counts"], a["offsets"],
+                                     a["perm"], a["inv"], a["xp"], ws, p=p, mass_out=a["mass"] if p > 0 else None,
+                                     K_dev=a["Kdev"] if K == -1 else None, status=st)
+    rws = dm.workspace(dm.decomoe_router_logits_ws_bytes(T, d, E), DEV)
+    dm.decomoe_router_logits_ws(x, w_r, bias, b["logits"], rws, st)
+    dws = dm.workspace(dm.decomoe_route_dispatch_workspace_bytes(T, k, E), DEV)
+    dm.decomoe_route_dispatch(b["logits"], K, k, b["idx"], b["w"], x, b["counts"], b["offsets"], b["perm"], b["inv"],
+                              b["xp"], dws, p=p, mass_out=b["mass"] if p > 0 else None,
+                              K_dev=b["Kdev"] if K == -1 else None, status=st)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(st) == 0
+    for key in a:
+        u, v = a[key], b[key]
+        if u.dtype in (torch.float32, torch.float64, torch.bfloat16):
+            u = u.view({torch.float32: torch.int32, torch.float64: torch.int64, torch.bfloat16: torch.int16}[u.dtype])
+            v = v.view(u.dtype)
+        assert torch.equal(u, v), key
+    if p > 0:
+        assert (a["mass"] >= 0).all()
