@@ -109,11 +109,10 @@ static int router_route_dispatch_impl(const void* x, const void* w_r, const floa
   if (T > 0) {
     DM_ARG_CHECK(x && w_r && logits, "router_route_dispatch: null pointer");
     int ks = 1;
-    if (dtype == DECOMOE_BF16 && decomoe_router_logits_ws_bytes(T, d, E) > 0) {
-      DM_ARG_CHECK(aligned16(x) && aligned16(w_r) && aligned16(scratch),
-                   "router_route_dispatch: pointers must be 16-byte aligned");
+    const size_t split_bytes = dtype == DECOMOE_BF16 ? decomoe_router_logits_ws_bytes(T, d, E) : 0;
+    if (split_bytes > 0 && aligned16(x) && aligned16(w_r) && aligned16(scratch) && aligned16(logits) &&
+        (bias == nullptr || aligned16(bias)))
       DM_RET(launch_router_parts(x, w_r, T, d, E, scratch, status_dev, s, &ks));
-    }
     if (ks > 1) {
       src.nparts = ks;
       src.part_stride = T * E;
@@ -121,8 +120,10 @@ static int router_route_dispatch_impl(const void* x, const void* w_r, const floa
       src.logits_out = logits;
       lg = scratch;
     } else {
-      DM_RET(decomoe_router_logits(x, w_r, bias, T, d, E, dtype, logits, status_dev,
-                                   reinterpret_cast<decomoe_stream_t>(s)));
+      // unsplit router, or operands the slice-reading routing kernel cannot
+      // take: the logits first, exactly as decomoe_router_logits_ws forms them
+      DM_RET(decomoe_router_logits_ws(x, w_r, bias, T, d, E, dtype, logits, scratch, split_bytes, status_dev,
+                                      reinterpret_cast<decomoe_stream_t>(s)));
     }
   }
   return route_dispatch_src(lg, src, T, E, K, k, p, topk_idx, topk_w, mass_out, K_dev, x, d, dtype, counts, offsets,

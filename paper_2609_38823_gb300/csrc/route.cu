@@ -168,6 +168,12 @@ __device__ __forceinline__ float pick_weight(float my_v, int lane, int k) {
   return z / zs;
 }
 
+// NP: 1 reads plain logit rows; NP > 1 reads NP k slices of the split
+// router (src), each warp loading its row's slices as coalesced 16-byte
+// vectors (all NP in flight), adding them in slice order and the bias last,
+// storing the sums to src.logits_out and, through shared memory, into the
+// key layout (E % 4 == 0, 16-byte aligned rows).
+template <int NP>
 __global__ void __launch_bounds__(ROUTE_THREADS)
     k_route(const float* __restrict__ logits, int64_t Tn, int E, int64_t ld, int K, int k,
             int32_t* __restrict__ idx_out, float* __restrict__ w_out, double* __restrict__ part,
@@ -176,6 +182,7 @@ __global__ void __launch_bounds__(ROUTE_THREADS)
   if (K_dev != nullptr) K = *K_dev;  // prefix chosen on the device (k <= K <= E by construction)
   __shared__ int s_idx[ROUTE_TPB][DECOMOE_MAX_TOPK];
   __shared__ float s_w[ROUTE_TPB][DECOMOE_MAX_TOPK];
+  __shared__ float s_row[NP > 1 ? ROUTE_TPB : 1][NP > 1 ? DECOMOE_MAX_E : 1];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t t = static_cast<int64_t>(blockIdx.x) * ROUTE_TPB + warp;
   const bool mass = part != nullptr;
@@ -186,7 +193,7 @@ __global__ void __launch_bounds__(ROUTE_THREADS)
     const float* row = logits + roff;
     const int lim = mass ? E : K;
     uint32_t v[8];  // order-preserving keys of the row's logits
-    if (src.nparts == 1 && src.bias == nullptr && src.logits_out == nullptr) {
+    if constexpr (NP == 1) {
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         const int e = lane + 32 * i;
@@ -194,17 +201,35 @@ __global__ void __launch_bounds__(ROUTE_THREADS)
       }
     } else {
       // partial sums of the k-split router, added in slice order, bias last
+      const float4* r4 = reinterpret_cast<const float4*>(row);
+      const int64_t s4 = src.part_stride / 4;
+      for (int c = lane; c < E / 4; c += 32) {
+        float4 p[NP];
+#pragma unroll
+        for (int sl = 0; sl < NP; ++sl) p[sl] = __ldcs(r4 + sl * s4 + c);
+        float4 a = p[0];
+#pragma unroll
+        for (int sl = 1; sl < NP; ++sl) {
+          a.x += p[sl].x;
+          a.y += p[sl].y;
+          a.z += p[sl].z;
+          a.w += p[sl].w;
+        }
+        if (src.bias != nullptr) {
+          const float4 b = reinterpret_cast<const float4*>(src.bias)[c];
+          a.x += b.x;
+          a.y += b.y;
+          a.z += b.z;
+          a.w += b.w;
+        }
+        if (src.logits_out != nullptr) reinterpret_cast<float4*>(src.logits_out + roff)[c] = a;
+        reinterpret_cast<float4*>(s_row[warp])[c] = a;
+      }
+      __syncwarp();
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         const int e = lane + 32 * i;
-        v[i] = 0u;
-        if (e < E) {
-          float a = row[e];
-          for (int sl = 1; sl < src.nparts; ++sl) a += row[sl * src.part_stride + e];
-          if (src.bias != nullptr) a += src.bias[e];
-          if (src.logits_out != nullptr) src.logits_out[roff + e] = a;
-          if (e < lim) v[i] = fkey(a);
-        }
+        v[i] = (e < lim) ? fkey(s_row[warp][e]) : 0u;
       }
     }
     float my_v;
@@ -289,8 +314,8 @@ __global__ void k_select_prefix(const double* __restrict__ mass, int E, int k, d
 int launch_skip_mass(const float* logits, int64_t n, int E, int64_t ld, int k, int64_t skip_at, int64_t skip_len,
                      double* part, double* mass, cudaStream_t s) {
   const int64_t nblocks = (n + ROUTE_TPB - 1) / ROUTE_TPB;
-  k_route<<<static_cast<unsigned>(nblocks), ROUTE_THREADS, 0, s>>>(logits, n, E, ld, E, k, nullptr, nullptr, part,
-                                                                   nullptr, skip_at, skip_len, RouteSrc{});
+  k_route<1><<<static_cast<unsigned>(nblocks), ROUTE_THREADS, 0, s>>>(logits, n, E, ld, E, k, nullptr, nullptr, part,
+                                                                      nullptr, skip_at, skip_len, RouteSrc{});
   DM_LAUNCH_CHECK("k_route");
   k_mass_finalize<<<E, 256, 0, s>>>(part, static_cast<int>(nblocks), E, mass);
   DM_LAUNCH_CHECK("k_mass_finalize");
@@ -387,7 +412,11 @@ int route_prefix_src(const float* logits, const RouteSrc& src, int64_t T, int E,
   DM_ARG_CHECK(k >= 1 && k <= DECOMOE_MAX_TOPK, "route_prefix: k=%d outside [1, %d]", k, DECOMOE_MAX_TOPK);
   DM_ARG_CHECK(K >= k && K <= E, "route_prefix: need k <= K <= E (k=%d K=%d E=%d)", k, K, E);
   DM_ARG_CHECK(ld >= E, "route_prefix: ld < E");
-  DM_ARG_CHECK(src.nparts >= 1, "route_prefix: no logit slices");
+  DM_ARG_CHECK(src.nparts == 1 || ((src.nparts == 4 || src.nparts == 16) && E % 4 == 0 && ld == E &&
+                                    src.part_stride % 4 == 0 && aligned16(logits) &&
+                                    (src.bias == nullptr || aligned16(src.bias)) &&
+                                    (src.logits_out == nullptr || aligned16(src.logits_out))),
+               "route_prefix: logit slices need 4 or 16 slices of 16-byte aligned rows");
   if (T == 0) {
     if (mass_out) DM_CUDA_CHECK(cudaMemsetAsync(mass_out, 0, sizeof(double) * E, s));
     return DECOMOE_OK;
@@ -405,8 +434,9 @@ int route_prefix_src(const float* logits, const RouteSrc& src, int64_t T, int E,
     // finalize would only add zeros), so it is written in place
     part = nblocks == 1 ? mass_out : static_cast<double*>(ws);
   }
-  DM_CUDA_CHECK(launch_pdl(k_route, dim3(static_cast<unsigned>(nblocks)), dim3(ROUTE_THREADS), 0, s, logits, T, E,
-                           ld, K, k, topk_idx, topk_w, part, static_cast<const int32_t*>(nullptr), INT64_MAX,
+  auto kern = src.nparts == 16 ? k_route<16> : src.nparts == 4 ? k_route<4> : k_route<1>;
+  DM_CUDA_CHECK(launch_pdl(kern, dim3(static_cast<unsigned>(nblocks)), dim3(ROUTE_THREADS), 0, s, logits, T, E, ld,
+                           K, k, topk_idx, topk_w, part, static_cast<const int32_t*>(nullptr), INT64_MAX,
                            static_cast<int64_t>(0), src));
   if (mass_out != nullptr && nblocks > 1) {
     if (defer_finalize && mass_blocks != nullptr) {
@@ -444,7 +474,7 @@ int decomoe_route_prefix_dk(const float* logits, int64_t T, int E, int64_t ld, c
   DM_ARG_CHECK(logits && K_dev, "route_prefix_dk: null pointer");
   const int64_t nblocks = (T + ROUTE_TPB - 1) / ROUTE_TPB;
   DM_ARG_CHECK(nblocks <= 0x7fffffff, "route_prefix_dk: T too large");
-  DM_CUDA_CHECK(launch_pdl(k_route, dim3(static_cast<unsigned>(nblocks)), dim3(ROUTE_THREADS), 0,
+  DM_CUDA_CHECK(launch_pdl(k_route<1>, dim3(static_cast<unsigned>(nblocks)), dim3(ROUTE_THREADS), 0,
                            reinterpret_cast<cudaStream_t>(stream), logits, T, E, ld, E, k, topk_idx, topk_w,
                            static_cast<double*>(nullptr), K_dev, INT64_MAX, static_cast<int64_t>(0), RouteSrc{}));
   return DECOMOE_OK;
