@@ -36,8 +36,8 @@ import workloads as W  # noqa: E402
 
 # at T=2048: router k slices, routing (reads the slices) with mass partials,
 # dispatch 3 (histogram + mass sum, ranks, row gather), gate/up, down,
-# combine, compaction
-LAUNCHES_PER_STEP = 9
+# combine with the visual-block removal
+LAUNCHES_PER_STEP = 8
 # (plus two 4-byte memsets zeroing the expert GEMMs' tile counter)
 
 
@@ -233,9 +233,11 @@ def run_step(dm, wl, L, B, K, v0, nv, text, ev=None):
     dm.decomoe_expert_down(B.h, B.offsets[:K + 1], K, L.w_down, B.y, B.status)  # a6 down
     if ev is not None:
         ev[2].record()
-    dm.decomoe_combine(B.y, B.inv, B.w, B.out)                                         # a7
     if text is not None:
-        dm.decomoe_drop_visual_block(B.out, text, v0, nv)                              # a8
+        # a7 + a8: combine, the text rows also stored to the compacted buffer
+        dm.decomoe_combine_drop_visual_block(B.y, B.inv, B.w, B.out, text, v0, nv)
+    else:
+        dm.decomoe_combine(B.y, B.inv, B.w, B.out)                                     # a7
 
 
 def timed(fn, steps, warmup, ws, clocks=None, name="sweep"):

@@ -328,6 +328,18 @@ DECOMOE_API int decomoe_combine(const void* y_perm, const int32_t* inv_slot, con
                     int k, int d, int dtype, const void* residual, void* out,
                     decomoe_stream_t stream);
 
+/* a7 + a8 in one launch: decomoe_combine, and every text row of its output
+ * (t < v0 or t >= v0 + nv, the rows outside the visual block of Section 3.2)
+ * also stored to text_out [T - nv, d] in order, the block's rows skipped.
+ * out and text_out are bit-identical to decomoe_combine followed by
+ * decomoe_drop_visual_block(out, text_out, T, d * elem, v0, nv, 1, ...).
+ * Needs 0 <= v0, 0 <= nv, v0 + nv <= T; text_out 16-byte aligned and not
+ * overlapping out (else DECOMOE_ERR_INVALID_ARG, nothing launched). */
+DECOMOE_API int decomoe_combine_drop_visual_block(const void* y_perm, const int32_t* inv_slot,
+                                                  const float* topk_w, int64_t T, int k, int d, int dtype,
+                                                  const void* residual, void* out, void* text_out, int64_t v0,
+                                                  int64_t nv, decomoe_stream_t stream);
+
 /* ------------------------------------------------------------------------
  * a8. Visual-block removal (Section 3.2: the complete visual block leaves the
  * hidden state and the KV cache; later layers and decoding use the text-only

@@ -74,6 +74,7 @@ SIGNATURES = {
     "decomoe_expert_swiglu_gather": (_I, [_P, _L, _P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
     "decomoe_expert_swiglu_ref": (_I, [_P, _P, _L, _I, _I, _I, _P, _P, _P, _P, _P]),
     "decomoe_combine": (_I, [_P, _P, _P, _L, _I, _I, _I, _P, _P, _P]),
+    "decomoe_combine_drop_visual_block": (_I, [_P, _P, _P, _L, _I, _I, _I, _P, _P, _P, _L, _L, _P]),
     "decomoe_drop_visual_block": (_I, [_P, _P, _L, _L, _L, _L, _L, _L, _L, _P]),
     "decomoe_rmsnorm": (_I, [_P, _P, _L, _I, _F, _I, _P]),
     "decomoe_moe_layer_workspace_bytes": (_S, [_L, _I, _I, _I, _I, _I]),
@@ -441,6 +442,18 @@ def decomoe_combine(y_perm, inv_slot, topk_w, out, residual=None, stream=None):
     _check("decomoe_combine",
            lib().decomoe_combine(_ptr(y_perm), _ptr(inv_slot), _ptr(topk_w), T, k, d, _dt(out),
                                  _ptr(residual), _ptr(out), _stream(stream)))
+
+
+def decomoe_combine_drop_visual_block(y_perm, inv_slot, topk_w, out, text_out, v0, nv, residual=None, stream=None):
+    """Combine, and the output's text rows (outside [v0, v0 + nv)) also
+    stored to text_out [T - nv, d] in the same launch."""
+    _need_cuda(y_perm, inv_slot, topk_w, out, text_out, residual)
+    T, k = topk_w.shape
+    d = out.shape[1]
+    _check("decomoe_combine_drop_visual_block",
+           lib().decomoe_combine_drop_visual_block(_ptr(y_perm), _ptr(inv_slot), _ptr(topk_w), T, k, d, _dt(out),
+                                                   _ptr(residual), _ptr(out), _ptr(text_out), v0, nv,
+                                                   _stream(stream)))
 
 
 def decomoe_drop_visual_block(src, dst, v0, nv, stream=None):

@@ -42,11 +42,20 @@ __device__ __forceinline__ uint4 finish_vec(float* acc, const uint4* __restrict_
                       __float_as_uint(acc[3]));
 }
 
-template <bool BF16, int KT>
+// Visual-block removal fused into the combine: every output vector of a text
+// row (t < v0 or t >= v0 + nv) is also stored to text[t'] with t' = t, or
+// t - nv past the block: the rows decomoe_drop_visual_block would copy from
+// out, written while they are in registers.
+struct DropRows {
+  uint4* text = nullptr;  // null: no second store
+  int64_t v0 = 0, nv = 0;
+};
+
+template <bool BF16, int KT, bool DROP>
 __global__ void __launch_bounds__(256)
     k_combine(const uint4* __restrict__ y, const int32_t* __restrict__ inv_slot,
               const float* __restrict__ w, int64_t Tn, int k, int vec,
-              const uint4* __restrict__ residual, uint4* __restrict__ out) {
+              const uint4* __restrict__ residual, uint4* __restrict__ out, DropRows drop) {
   pdl_enter();
   constexpr int NE = BF16 ? 8 : 4;
   constexpr int WPT = 2;  // warps per token: each takes alternate 32-vector chunks
@@ -56,6 +65,8 @@ __global__ void __launch_bounds__(256)
   for (int64_t wt = gw; wt < Tn * WPT; wt += nw) {
     const int64_t t = wt / WPT;
     const int part = static_cast<int>(wt - t * WPT);
+    const bool text_row = DROP && (t < drop.v0 || t >= drop.v0 + drop.nv);
+    const int64_t trow = t < drop.v0 ? t : t - drop.nv;
     int my_row = -1;
     float my_w = 0.f;
     if (lane < k) {
@@ -89,8 +100,14 @@ __global__ void __launch_bounds__(256)
             acc_vec<BF16>(acc, v[j], wts[j]);
             acc_vec<BF16>(acc2, v2[j], wts[j]);
           }
-        out[t * vec + c] = finish_vec<BF16>(acc, residual, t * vec + c);
-        if (two) out[t * vec + c2] = finish_vec<BF16>(acc2, residual, t * vec + c2);
+        const uint4 o1 = finish_vec<BF16>(acc, residual, t * vec + c);
+        out[t * vec + c] = o1;
+        if (text_row) drop.text[trow * vec + c] = o1;
+        if (two) {
+          const uint4 o2 = finish_vec<BF16>(acc2, residual, t * vec + c2);
+          out[t * vec + c2] = o2;
+          if (text_row) drop.text[trow * vec + c2] = o2;
+        }
       }
     } else {
       for (int c0 = part * 32; c0 < vec; c0 += 32 * WPT) {
@@ -106,22 +123,33 @@ __global__ void __launch_bounds__(256)
           if (row < 0 || !active) continue;
           acc_vec<BF16>(acc, __ldg(y + static_cast<int64_t>(row) * vec + c), wj);
         }
-        if (active) out[t * vec + c] = finish_vec<BF16>(acc, residual, t * vec + c);
+        if (active) {
+          const uint4 o1 = finish_vec<BF16>(acc, residual, t * vec + c);
+          out[t * vec + c] = o1;
+          if (text_row) drop.text[trow * vec + c] = o1;
+        }
       }
     }
   }
 }
 
+template <bool BF16, bool DROP>
+static cudaError_t launch_combine_k(int grid, cudaStream_t s, const uint4* y, const int32_t* inv, const float* w,
+                                    int64_t T, int k, int vec, const uint4* res, uint4* out, DropRows drop) {
+  switch (k) {
+    case 1: return launch_pdl(k_combine<BF16, 1, DROP>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out, drop);
+    case 2: return launch_pdl(k_combine<BF16, 2, DROP>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out, drop);
+    case 4: return launch_pdl(k_combine<BF16, 4, DROP>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out, drop);
+    case 8: return launch_pdl(k_combine<BF16, 8, DROP>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out, drop);
+    default:
+      return launch_pdl(k_combine<BF16, 0, DROP>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out, drop);
+  }
+}
 template <bool BF16>
 static cudaError_t launch_combine(int grid, cudaStream_t s, const uint4* y, const int32_t* inv, const float* w,
-                                  int64_t T, int k, int vec, const uint4* res, uint4* out) {
-  switch (k) {
-    case 1: return launch_pdl(k_combine<BF16, 1>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out);
-    case 2: return launch_pdl(k_combine<BF16, 2>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out);
-    case 4: return launch_pdl(k_combine<BF16, 4>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out);
-    case 8: return launch_pdl(k_combine<BF16, 8>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out);
-    default: return launch_pdl(k_combine<BF16, 0>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out);
-  }
+                                  int64_t T, int k, int vec, const uint4* res, uint4* out, DropRows drop) {
+  return drop.text != nullptr ? launch_combine_k<BF16, true>(grid, s, y, inv, w, T, k, vec, res, out, drop)
+                              : launch_combine_k<BF16, false>(grid, s, y, inv, w, T, k, vec, res, out, drop);
 }
 
 // ------------------------------------------------------------------ compaction
@@ -243,6 +271,29 @@ extern "C" {
 int decomoe_combine(const void* y_perm, const int32_t* inv_slot, const float* topk_w, int64_t T, int k,
                     int d, int dtype, const void* residual, void* out, decomoe_stream_t stream) {
   clear_error();
+  return combine_impl(y_perm, inv_slot, topk_w, T, k, d, dtype, residual, out, nullptr, 0, 0, stream);
+}
+
+int decomoe_combine_drop_visual_block(const void* y_perm, const int32_t* inv_slot, const float* topk_w, int64_t T,
+                                      int k, int d, int dtype, const void* residual, void* out, void* text_out,
+                                      int64_t v0, int64_t nv, decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(v0 >= 0 && nv >= 0 && v0 + nv <= T,
+               "combine_drop_visual_block: visual block [%lld, %lld) outside [0, %lld)", (long long)v0,
+               (long long)(v0 + nv), (long long)T);
+  const bool any_text = T - nv > 0;  // an all-visual sequence leaves no text row to store
+  DM_ARG_CHECK(text_out != nullptr || !any_text, "combine_drop_visual_block: text_out is null");
+  return combine_impl(y_perm, inv_slot, topk_w, T, k, d, dtype, residual, out, any_text ? text_out : nullptr, v0,
+                      nv, stream);
+}
+
+}  // extern "C"
+
+namespace decomoe {
+
+int combine_impl(const void* y_perm, const int32_t* inv_slot, const float* topk_w, int64_t T, int k, int d,
+                 int dtype, const void* residual, void* out, void* text_out, int64_t v0, int64_t nv,
+                 decomoe_stream_t stream) {
   DM_ARG_CHECK(T >= 0 && k >= 1 && k <= DECOMOE_MAX_TOPK && d > 0, "combine: bad sizes");
   DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "combine: bad dtype");
   if (T == 0) return DECOMOE_OK;
@@ -252,17 +303,33 @@ int decomoe_combine(const void* y_perm, const int32_t* inv_slot, const float* to
                    (residual == nullptr || aligned16(residual)),
                "combine: rows must be 16-byte multiples, pointers 16-byte aligned");
   DM_ARG_CHECK(out != y_perm, "combine: out aliases y_perm");
+  DropRows drop;
+  if (text_out != nullptr) {
+    DM_ARG_CHECK(v0 >= 0 && nv >= 0 && v0 + nv <= T, "combine: visual block [%lld, %lld) outside [0, %lld)",
+                 (long long)v0, (long long)(v0 + nv), (long long)T);
+    DM_ARG_CHECK(aligned16(text_out), "combine: text_out must be 16-byte aligned");
+    const uintptr_t o0 = reinterpret_cast<uintptr_t>(out), o1 = o0 + static_cast<uintptr_t>(T) * row_bytes;
+    const uintptr_t t0 = reinterpret_cast<uintptr_t>(text_out), t1 = t0 + static_cast<uintptr_t>(T - nv) * row_bytes;
+    DM_ARG_CHECK(o1 <= t0 || t1 <= o0, "combine: text_out overlaps out");
+    drop.text = static_cast<uint4*>(text_out);
+    drop.v0 = v0;
+    drop.nv = nv;
+  }
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const int vec = static_cast<int>(row_bytes / 16);
   const int grid = grid_for_warps(2 * T);  // two warps per token
   if (dtype == DECOMOE_BF16)
     DM_CUDA_CHECK(launch_combine<true>(grid, s, static_cast<const uint4*>(y_perm), inv_slot, topk_w, T, k, vec,
-                                       static_cast<const uint4*>(residual), static_cast<uint4*>(out)));
+                                       static_cast<const uint4*>(residual), static_cast<uint4*>(out), drop));
   else
     DM_CUDA_CHECK(launch_combine<false>(grid, s, static_cast<const uint4*>(y_perm), inv_slot, topk_w, T, k, vec,
-                                        static_cast<const uint4*>(residual), static_cast<uint4*>(out)));
+                                        static_cast<const uint4*>(residual), static_cast<uint4*>(out), drop));
   return DECOMOE_OK;
 }
+
+}  // namespace decomoe
+
+extern "C" {
 
 int decomoe_drop_visual_block(const void* src, void* dst, int64_t rows, int64_t row_bytes, int64_t v0,
                               int64_t nv, int64_t nbatch, int64_t src_batch_stride,

@@ -122,6 +122,11 @@ int dispatch_with_mass(const int32_t* topk_idx, int64_t T, int k, int K, const v
                        int32_t* counts, int32_t* offsets, int32_t* perm_token, int32_t* inv_slot, void* x_perm,
                        void* ws, size_t ws_bytes, int32_t* status_dev, const double* mass_part, int mass_blocks,
                        int mass_E, double* mass, cudaStream_t s);
+// decomoe_combine, and with text_out also the visual-block removal of its
+// output rows (decomoe_combine_drop_visual_block).
+int combine_impl(const void* y_perm, const int32_t* inv_slot, const float* topk_w, int64_t T, int k, int d,
+                 int dtype, const void* residual, void* out, void* text_out, int64_t v0, int64_t nv,
+                 decomoe_stream_t stream);
 // The k-split router's GEMM alone: KS slices of partial logits [KS][T][E]
 // (no bias) into scratch; returns KS (1: no split at this size, nothing
 // launched).

@@ -323,6 +323,45 @@ def test_combine_parity(T, k, d, dt, resid):
         assert_close_out(got, ref, BF16_REL_L2, BF16_MAX_ABS, "combine bf16")
 
 
+@pytest.mark.parametrize("T,k,d,dt,resid,v0,nv", [(2048, 8, 2048, "bf16", True, 0, 1792),
+                                                   (333, 3, 128, "bf16", False, 100, 200),
+                                                   (64, 2, 256, "f32", True, 10, 0),
+                                                   (50, 1, 64, "f32", False, 0, 50),
+                                                   (40, 8, 2048, "bf16", False, 39, 1)])
+def test_combine_drop_visual_block_equals_two_calls(T, k, d, dt, resid, v0, nv):
+    """The fused combine + visual-block removal writes the same out and the
+    same compacted text rows as decomoe_combine followed by
+    decomoe_drop_visual_block, bit for bit (a block at the start, in the
+    middle, empty, the whole sequence, the last row)."""
+    dtype = torch.bfloat16 if dt == "bf16" else torch.float32
+    g = torch.Generator().manual_seed(T * 5 + k)
+    y = torch.randn(T * k, d, generator=g).to(dtype).to(DEV)
+    inv = torch.randperm(T * k, generator=g).to(torch.int32).to(DEV)
+    w = torch.softmax(torch.randn(T, k, generator=g), -1).float().to(DEV)
+    res = torch.randn(T, d, generator=g).to(dtype).to(DEV) if resid else None
+    out1, out2 = (torch.empty(T, d, dtype=dtype, device=DEV) for _ in range(2))
+    text1 = torch.full((T - nv, d), 7, dtype=dtype, device=DEV)
+    text2 = torch.full((T - nv, d), -7, dtype=dtype, device=DEV)
+    dm.decomoe_combine_drop_visual_block(y, inv, w, out1, text1, v0, nv, res)
+    dm.decomoe_combine(y, inv, w, out2, res)
+    dm.decomoe_drop_visual_block(out2, text2, v0, nv)
+    torch.cuda.synchronize()
+    iv = torch.int16 if dtype == torch.bfloat16 else torch.int32
+    assert torch.equal(out1.view(iv), out2.view(iv))
+    assert torch.equal(text1.view(iv), text2.view(iv))
+
+
+def test_combine_drop_visual_block_rejects_bad_block():
+    T, k, d = 16, 2, 64
+    y = torch.zeros(T * k, d, device=DEV)
+    inv = torch.arange(T * k, dtype=torch.int32, device=DEV)
+    w = torch.full((T, k), 0.5, device=DEV)
+    out = torch.empty(T, d, device=DEV)
+    with pytest.raises(dm.DecomoeError) as e:
+        dm.decomoe_combine_drop_visual_block(y, inv, w, out, torch.empty(4, d, device=DEV), 10, 12)
+    assert e.value.code == dm.DECOMOE_ERR_INVALID_ARG
+
+
 # ----------------------------------------------------------------- visual-block removal
 
 @pytest.mark.parametrize("shape,v0,nv,dt", [
