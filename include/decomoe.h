@@ -356,6 +356,19 @@ DECOMOE_API int decomoe_drop_visual_block(const void* src, void* dst, int64_t ro
                               int64_t v0, int64_t nv, int64_t nbatch, int64_t src_batch_stride,
                               int64_t dst_batch_stride, decomoe_stream_t stream);
 
+/* The SAVB trigger fused into the removal (Section 3.2, Eq. 3): the same
+ * call with the gate's device-side decision exit_flag (decomoe_savb_gate's
+ * exit_flag_dev). The kernel reads *exit_flag: 1 performs the removal above,
+ * any other value writes nothing to dst. A caller can queue the removal of
+ * the hidden state and of the KV slices right behind the gate and read the
+ * decision back afterwards, instead of between the gate and the removal.
+ * Arguments and errors as decomoe_drop_visual_block; exit_flag must not be
+ * NULL (DECOMOE_ERR_INVALID_ARG). */
+DECOMOE_API int decomoe_drop_visual_block_if(const int32_t* exit_flag, const void* src, void* dst, int64_t rows,
+                                             int64_t row_bytes, int64_t v0, int64_t nv, int64_t nbatch,
+                                             int64_t src_batch_stride, int64_t dst_batch_stride,
+                                             decomoe_stream_t stream);
+
 /* ------------------------------------------------------------------------
  * SAVB exit gate (Section 3.2, Eqs. 2-3), evaluated at the candidate layers
  * {3, 7, ..., 47} (zero-based, Appendix) on the hidden state h [T, d]:

@@ -76,6 +76,7 @@ SIGNATURES = {
     "decomoe_combine": (_I, [_P, _P, _P, _L, _I, _I, _I, _P, _P, _P]),
     "decomoe_combine_drop_visual_block": (_I, [_P, _P, _P, _L, _I, _I, _I, _P, _P, _P, _L, _L, _P]),
     "decomoe_drop_visual_block": (_I, [_P, _P, _L, _L, _L, _L, _L, _L, _L, _P]),
+    "decomoe_drop_visual_block_if": (_I, [_P, _P, _P, _L, _L, _L, _L, _L, _L, _L, _P]),
     "decomoe_rmsnorm": (_I, [_P, _P, _L, _I, _F, _I, _P]),
     "decomoe_moe_layer_workspace_bytes": (_S, [_L, _I, _I, _I, _I, _I]),
     "decomoe_moe_layer": (_I, [_P, _P, _P, _P, _P, _L, _I, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P,
@@ -456,9 +457,7 @@ def decomoe_combine_drop_visual_block(y_perm, inv_slot, topk_w, out, text_out, v
                                                    _stream(stream)))
 
 
-def decomoe_drop_visual_block(src, dst, v0, nv, stream=None):
-    """src: [rows, ...] or [nbatch, rows, ...] contiguous; dst the compacted shape."""
-    _need_cuda(src, dst)
+def _drop_geometry(src, dst, nv):
     if src.dim() >= 3:
         nbatch, rows = src.shape[0], src.shape[1]
         row_bytes = src[0, 0].numel() * src.element_size()
@@ -469,9 +468,26 @@ def decomoe_drop_visual_block(src, dst, v0, nv, stream=None):
         row_bytes = (src.numel() // max(rows, 1)) * src.element_size() if rows else src.element_size()
         sstride = rows * row_bytes
         dstride = (rows - nv) * row_bytes
+    return nbatch, rows, row_bytes, sstride, dstride
+
+
+def decomoe_drop_visual_block(src, dst, v0, nv, stream=None):
+    """src: [rows, ...] or [nbatch, rows, ...] contiguous; dst the compacted shape."""
+    _need_cuda(src, dst)
+    nbatch, rows, row_bytes, sstride, dstride = _drop_geometry(src, dst, nv)
     _check("decomoe_drop_visual_block",
            lib().decomoe_drop_visual_block(_ptr(src), _ptr(dst), rows, row_bytes, v0, nv, nbatch, sstride,
                                            dstride, _stream(stream)))
+
+
+def decomoe_drop_visual_block_if(exit_flag, src, dst, v0, nv, stream=None):
+    """decomoe_drop_visual_block when the device int32 exit_flag holds 1 (the
+    SAVB gate's decision); otherwise dst is left as it is."""
+    _need_cuda(exit_flag, src, dst)
+    nbatch, rows, row_bytes, sstride, dstride = _drop_geometry(src, dst, nv)
+    _check("decomoe_drop_visual_block_if",
+           lib().decomoe_drop_visual_block_if(_ptr(exit_flag), _ptr(src), _ptr(dst), rows, row_bytes, v0, nv, nbatch,
+                                              sstride, dstride, _stream(stream)))
 
 
 def decomoe_rmsnorm(x, y, eps=1e-6, stream=None):

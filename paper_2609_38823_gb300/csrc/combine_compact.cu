@@ -156,11 +156,14 @@ static cudaError_t launch_combine(int grid, cudaStream_t s, const uint4* y, cons
 // dst[b, r'] = src[b, r'] for r' < v0, src[b, r' + nv] otherwise. A flat grid
 // over the output's 16-byte vectors (batch, row, column; column fastest, so a
 // warp moves 512 contiguous bytes), four vectors per thread in flight.
+// flag (optional): the removal runs only when *flag == 1 (the SAVB gate's
+// exit decision, read on the device); any other value leaves dst untouched.
 __global__ void __launch_bounds__(256)
     k_compact_vec(const uint4* __restrict__ src, uint4* __restrict__ dst, int64_t rows_out,
                   int64_t vec, int64_t v0, int64_t nv, int64_t nbatch, int64_t sstride,
-                  int64_t dstride) {
+                  int64_t dstride, const int32_t* __restrict__ flag) {
   pdl_enter();
+  if (flag != nullptr && *flag != 1) return;
   constexpr int U = 4;
   const int64_t total = nbatch * rows_out * vec;
   const int64_t step = static_cast<int64_t>(gridDim.x) * blockDim.x * U;
@@ -190,8 +193,9 @@ __global__ void __launch_bounds__(256)
 // Byte path for rows or strides that are not 16-byte multiples.
 __global__ void k_compact_bytes(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst,
                                 int64_t rows_out, int64_t row_bytes, int64_t v0, int64_t nv,
-                                int64_t nbatch, int64_t sstride, int64_t dstride) {
+                                int64_t nbatch, int64_t sstride, int64_t dstride, const int32_t* __restrict__ flag) {
   pdl_enter();
+  if (flag != nullptr && *flag != 1) return;
   const int64_t total = nbatch * rows_out * row_bytes;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -335,6 +339,26 @@ int decomoe_drop_visual_block(const void* src, void* dst, int64_t rows, int64_t 
                               int64_t nv, int64_t nbatch, int64_t src_batch_stride,
                               int64_t dst_batch_stride, decomoe_stream_t stream) {
   clear_error();
+  return drop_visual_block_impl(nullptr, src, dst, rows, row_bytes, v0, nv, nbatch, src_batch_stride,
+                                dst_batch_stride, stream);
+}
+
+int decomoe_drop_visual_block_if(const int32_t* exit_flag, const void* src, void* dst, int64_t rows,
+                                 int64_t row_bytes, int64_t v0, int64_t nv, int64_t nbatch,
+                                 int64_t src_batch_stride, int64_t dst_batch_stride, decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(exit_flag != nullptr, "drop_visual_block_if: exit_flag is null");
+  return drop_visual_block_impl(exit_flag, src, dst, rows, row_bytes, v0, nv, nbatch, src_batch_stride,
+                                dst_batch_stride, stream);
+}
+
+}  // extern "C"
+
+namespace decomoe {
+
+int drop_visual_block_impl(const int32_t* flag, const void* src, void* dst, int64_t rows, int64_t row_bytes,
+                           int64_t v0, int64_t nv, int64_t nbatch, int64_t src_batch_stride,
+                           int64_t dst_batch_stride, decomoe_stream_t stream) {
   DM_ARG_CHECK(rows >= 0 && row_bytes > 0 && nbatch >= 0, "drop_visual_block: bad sizes");
   DM_ARG_CHECK(v0 >= 0 && nv >= 0 && v0 + nv <= rows, "drop_visual_block: block [%lld, %lld) outside [0, %lld)",
                (long long)v0, (long long)(v0 + nv), (long long)rows);
@@ -359,15 +383,19 @@ int decomoe_drop_visual_block(const void* src, void* dst, int64_t rows, int64_t 
     const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>((nvec + 1023) / 1024, sm_count() * 16LL)));
     DM_CUDA_CHECK(launch_pdl(k_compact_vec, dim3(grid), dim3(256), 0, s, static_cast<const uint4*>(src),
                              static_cast<uint4*>(dst), rows_out, row_bytes / 16, v0, nv, nbatch,
-                             src_batch_stride / 16, dst_batch_stride / 16));
+                             src_batch_stride / 16, dst_batch_stride / 16, flag));
   } else {
     const int grid = sm_count() * 8;
     DM_CUDA_CHECK(launch_pdl(k_compact_bytes, dim3(grid), dim3(256), 0, s, static_cast<const uint8_t*>(src),
                              static_cast<uint8_t*>(dst), rows_out, row_bytes, v0, nv, nbatch, src_batch_stride,
-                             dst_batch_stride));
+                             dst_batch_stride, flag));
   }
   return DECOMOE_OK;
 }
+
+}  // namespace decomoe
+
+extern "C" {
 
 int decomoe_rmsnorm(const void* x, void* y, int64_t T, int d, float eps, int dtype, decomoe_stream_t stream) {
   clear_error();

@@ -18,7 +18,7 @@ from typing import Dict, List, Optional, Sequence, Tuple
 
 import torch
 
-from . import (DECOMOE_BF16, DECOMOE_F32, decomoe_drop_visual_block, decomoe_moe_layer,
+from . import (DECOMOE_BF16, DECOMOE_F32, decomoe_drop_visual_block, decomoe_drop_visual_block_if, decomoe_moe_layer,
                decomoe_moe_layer_workspace_bytes, decomoe_rmsnorm, decomoe_savb_gate,
                decomoe_savb_gate_workspace_bytes, workspace)
 
@@ -80,12 +80,21 @@ class Stack:
             self.exit_flag = torch.zeros(len(layers), dtype=torch.int32, device=dev)
         self.exit_taken: Optional[int] = None  # first text-only layer of the last forward
 
-    def _compact(self, cur, kv, kv_out):
+    def _compact(self, cur, kv, kv_out, flag=None):
+        """Remove the visual block from the hidden state (into ht[0]) and the
+        KV caches; with flag (the gate's device-side decision) only when it
+        holds 1."""
         dst = self.ht[0]
-        decomoe_drop_visual_block(cur, dst, self.v0, self.nv)
+        if flag is None:
+            decomoe_drop_visual_block(cur, dst, self.v0, self.nv)
+        else:
+            decomoe_drop_visual_block_if(flag, cur, dst, self.v0, self.nv)
         if kv is not None:
             for src, out in zip(kv, kv_out):
-                decomoe_drop_visual_block(src, out, self.v0, self.nv)
+                if flag is None:
+                    decomoe_drop_visual_block(src, out, self.v0, self.nv)
+                else:
+                    decomoe_drop_visual_block_if(flag, src, out, self.v0, self.nv)
         return dst
 
     def forward(self, h0: torch.Tensor, kv: Optional[List[torch.Tensor]] = None,
@@ -117,10 +126,15 @@ class Stack:
             cur, nxt = out, 1 - nxt
             if self.gate is not None and not exited and l in self.gate.params and l + 1 < len(self.layers):
                 w1, b1, w2, b2 = self.gate.params[l]
+                flag = self.exit_flag[l:l + 1]
                 decomoe_savb_gate(cur, self.v0, self.nv, w1, b1, w2, b2, self.gate.theta, self.p_exit[l:l + 1],
-                                  self.exit_flag[l:l + 1], self.gate_ws)
-                if int(self.exit_flag[l].item()) == 1:
-                    cur = self._compact(cur, kv, kv_out)
+                                  flag, self.gate_ws)
+                # the removal is queued behind the gate and reads its decision
+                # on the device; the host reads the decision afterwards (the
+                # later launches' shapes depend on it)
+                dst = self._compact(cur, kv, kv_out, flag)
+                if int(flag.item()) == 1:
+                    cur = dst
                     bufs, xn, nxt, exited = self.ht, self.xn_t, 1, True
                     self.exit_taken = l + 1
         return cur

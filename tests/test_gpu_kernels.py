@@ -392,6 +392,30 @@ def test_drop_visual_block_bit_exact(shape, v0, nv, dt):
     assert got.shape == ref.shape and np.array_equal(got, ref)
 
 
+@pytest.mark.parametrize("shape,v0,nv,dt", [((300, 2048), 16, 256, torch.bfloat16),
+                                             ((4, 100, 512), 10, 80, torch.bfloat16),
+                                             ((9, 7, 6), 2, 3, torch.float32)])  # byte path (24-byte rows)
+def test_drop_visual_block_if_follows_the_device_flag(shape, v0, nv, dt):
+    """The gate-triggered removal compacts exactly when the device flag holds
+    1 (then bit-identical to the unconditional call) and leaves dst untouched
+    for 0 or any other value."""
+    src = torch.randn(*shape, generator=torch.Generator().manual_seed(9)).to(dt).to(DEV)
+    out_shape = (shape[0] - nv,) + tuple(shape[1:]) if len(shape) == 2 else \
+        (shape[0], shape[1] - nv) + tuple(shape[2:])
+    iv = torch.int16 if dt == torch.bfloat16 else torch.int32
+    ref = torch.empty(out_shape, dtype=dt, device=DEV)
+    dm.decomoe_drop_visual_block(src, ref, v0, nv)
+    for fv in (0, 1, 2, -1):
+        flag = torch.tensor([fv], dtype=torch.int32, device=DEV)
+        dst = torch.full(out_shape, 3.0, dtype=dt, device=DEV)
+        dm.decomoe_drop_visual_block_if(flag, src, dst, v0, nv)
+        torch.cuda.synchronize()
+        if fv == 1:
+            assert torch.equal(dst.view(iv), ref.view(iv))
+        else:
+            assert (dst == 3.0).all()
+
+
 # ----------------------------------------------------------------- router logits
 
 @pytest.mark.parametrize("T,d,E", [(2048, 2048, 128), (1, 2048, 128), (300, 2048, 256), (1552, 2048, 128),
