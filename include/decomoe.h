@@ -199,7 +199,7 @@ DECOMOE_API int decomoe_route_dispatch(const float* logits, int64_t T, int E, in
  * then decomoe_route_dispatch on them. Outputs (logits included) are
  * bit-identical to decomoe_router_logits_ws followed by
  * decomoe_route_dispatch with the same arguments. Where the router splits
- * its k loop (bf16, 192 < T, k slices that fit the SMs), the routing kernel
+ * its k loop (bf16, 96 < T, k slices that fit the SMs), the routing kernel
  * reads the router's partial sums itself, adding them in slice order and the
  * bias last exactly as the router's own reduction does, and writes the summed
  * logits; with a fixed K and mass_out the activated mass is added up by the

@@ -42,8 +42,17 @@ __global__ void k_router_simt(const T* __restrict__ x, const T* __restrict__ w_r
 // with a shuffle tree. The router matrix is read from HBM once and spread
 // over many SMs instead of one tensor-core tile.
 #ifndef DECOMOE_ROUTER_GEMV_MAX_T
-#define DECOMOE_ROUTER_GEMV_MAX_T 192  // token counts up to which the router runs on CUDA cores
+#define DECOMOE_ROUTER_GEMV_MAX_T 96  // token counts up to which the router runs on CUDA cores
 #endif
+// DECOMOE_ROUTER_GEMV_MAX_T in the environment overrides the compiled value
+// (read once per process).
+static int64_t router_gemv_max_t() {
+  static const int64_t v = [] {
+    const char* e = getenv("DECOMOE_ROUTER_GEMV_MAX_T");
+    return e != nullptr ? static_cast<int64_t>(atoll(e)) : static_cast<int64_t>(DECOMOE_ROUTER_GEMV_MAX_T);
+  }();
+  return v;
+}
 constexpr int GEMV_WARPS = 4;
 constexpr int GEMV_TPW = 4;  // tokens per warp
 __device__ __forceinline__ float dot8_bf16(const uint4 a, const uint4 b, float acc) {
@@ -337,7 +346,7 @@ int decomoe_router_logits(const void* x, const void* w_r, const float* bias, int
   if (T == 0) return DECOMOE_OK;
   DM_ARG_CHECK(x && w_r && logits, "router_logits: null pointer");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (dtype == DECOMOE_BF16 && T <= DECOMOE_ROUTER_GEMV_MAX_T && d % 8 == 0 && aligned16(x) && aligned16(w_r)) {
+  if (dtype == DECOMOE_BF16 && T <= router_gemv_max_t() && d % 8 == 0 && aligned16(x) && aligned16(w_r)) {
     const dim3 grid((E + GEMV_WARPS - 1) / GEMV_WARPS, static_cast<unsigned>((T + GEMV_TPW - 1) / GEMV_TPW));
     DM_CUDA_CHECK(launch_pdl(k_router_gemv, grid, dim3(32 * GEMV_WARPS), 0, s, static_cast<const uint4*>(x),
                              static_cast<const uint4*>(w_r), bias, static_cast<int64_t>(T), d / 8, E, logits));
@@ -363,7 +372,7 @@ int decomoe_router_logits(const void* x, const void* w_r, const float* bias, int
 
 size_t decomoe_router_logits_ws_bytes(int64_t T, int d, int E) {
   if (T <= 0 || d <= 0 || E <= 0) return 0;
-  if (T <= DECOMOE_ROUTER_GEMV_MAX_T) return 0;
+  if (T <= router_gemv_max_t()) return 0;
   const int ks = router_split_ks(T, d, E);
   return ks > 1 ? align_up(static_cast<size_t>(ks) * T * E * sizeof(float), 256) : 0;
 }
@@ -372,7 +381,7 @@ int decomoe_router_logits_ws(const void* x, const void* w_r, const float* bias, 
                              float* logits, void* ws, size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream) {
   clear_error();
   const size_t need = decomoe_router_logits_ws_bytes(T, d, E);
-  if (dtype != DECOMOE_BF16 || need == 0 || T <= DECOMOE_ROUTER_GEMV_MAX_T)
+  if (dtype != DECOMOE_BF16 || need == 0 || T <= router_gemv_max_t())
     return decomoe_router_logits(x, w_r, bias, T, d, E, dtype, logits, status_dev, stream);
   DM_ARG_CHECK(x && w_r && logits, "router_logits_ws: null pointer");
   DM_ARG_CHECK(aligned16(x) && aligned16(w_r) && aligned16(logits) && aligned16(ws),

@@ -529,8 +529,8 @@ def test_route_dispatch_equals_separate_calls_and_oracle(T, E, K, k, p):
     assert (np.abs(mass.cpu().numpy() - ref_m) <= MASS_REL * ref_m + 1e-30).all()
 
 
-@pytest.mark.parametrize("T,E", [(193, 128), (300, 256), (576, 128), (577, 128), (2048, 128), (2432, 256),
-                                 (2433, 128), (16384, 128), (100, 128)])
+@pytest.mark.parametrize("T,E", [(97, 128), (193, 128), (300, 256), (576, 128), (577, 128), (2048, 128),
+                                 (2432, 256), (2433, 128), (16384, 128), (100, 128)])
 def test_router_logits_k_split(T, E):
     """The workspace router (k slices on the tensor cores, partial sums added
     in slice order, the bias last) stays within the fp32 summation bound at
@@ -554,14 +554,15 @@ def test_router_logits_k_split(T, E):
     assert (err <= logit_error_bound(x64[rows], w64, b64)).all(), f"max err {err.max():.3e}"
 
 
-@pytest.mark.parametrize("T,E,K,p", [(1, 128, 64, 0.7), (100, 128, 64, 0.7), (193, 128, 64, 0.7), (300, 256, -1, 0.7),
+@pytest.mark.parametrize("T,E,K,p", [(1, 128, 64, 0.7), (96, 128, 64, 0.7), (97, 128, 64, 0.7), (100, 128, -1, 0.7),
+                                     (193, 128, 64, 0.7), (300, 256, -1, 0.7),
                                      (576, 128, 64, 0.0), (577, 128, -1, 0.5), (2048, 128, 64, 0.7),
                                      (2048, 128, -1, 0.7), (2432, 256, 40, 0.7), (2433, 128, 64, 0.7),
                                      (4096, 128, -1, 0.9)])
 def test_router_route_dispatch_equals_separate_calls(T, E, K, p):
     """The one-call front half (router logits, routing, dispatch) equals
     decomoe_router_logits_ws + decomoe_route_dispatch bit for bit, whether
-    the routing kernel reads the split router's partial sums (193 <= T <=
+    the routing kernel reads the split router's partial sums (97 <= T <=
     2432) or plain logits, with the mass finished by the dispatch launch or by
     its own kernel."""
     d, k = 2048, 8
