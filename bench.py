@@ -331,6 +331,20 @@ def ours(args, ws, rank, local):
             torch.cuda.synchronize()
             ext += 200
     clk = clocks.stop() if clocks else None
+    # per-step spread: 200 further steps, each bracketed by its own events
+    # between graph launches (outside any graph, so no launch chain is cut)
+    spread = None
+    if graphs is not None:
+        n_sp = 200
+        sp = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_sp)]
+        for i in range(n_sp):
+            sp[i][0].record()
+            step(i, None)
+            sp[i][1].record()
+        torch.cuda.synchronize()
+        d_ms = sorted(a.elapsed_time(b) for a, b in sp)
+        spread = {"steps": n_sp, "p10_ms": round(d_ms[n_sp // 10], 4), "median_ms": round(d_ms[n_sp // 2], 4),
+                  "p90_ms": round(d_ms[(9 * n_sp) // 10], 4)}
     if dm.decomoe_read_status(B.status) != 0:
         raise RuntimeError("device status set during the benchmark")
     ms_max = max_over_ranks(ms, ws)
@@ -482,6 +496,7 @@ def ours(args, ws, rank, local):
         "e2e": e2e,
         "gpu_launches": LAUNCHES_PER_STEP * args.steps,
         "timing_mode": timing_mode,
+        "step_spread": spread,
         "clocks": clk,
         "clock_window": "timed region" if ext == 0 else f"timed region + {ext} identical untimed steps",
         "sweep": sweep,

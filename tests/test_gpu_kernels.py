@@ -151,6 +151,9 @@ DISPATCH_CASES = [
     (2048, 8, 40, 2048, "bf16", "route"), (16384, 8, 39, 2048, "bf16", "route"), (100, 4, 8, 256, "bf16", "one_expert"),
     (1000, 3, 256, 64, "bf16", "uniform"), (129, 8, 16, 2048, "bf16", "uniform"), (1552, 8, 128, 2048, "bf16", "route"),
     (272, 8, 37, 2048, "bf16", "route"),
+    # row sizes around the bulk-copy gather's ring limits: 6 KiB (32 buffers),
+    # 8 KiB (16 buffers), 16 KiB (warp-per-row kernel)
+    (300, 4, 16, 3072, "bf16", "route"), (300, 4, 16, 4096, "bf16", "uniform"), (64, 2, 8, 4096, "f32", "uniform"),
 ]
 
 
