@@ -107,14 +107,37 @@ struct RouteSrc {
   const float* bias = nullptr;
   float* logits_out = nullptr;
 };
+// Tokens per routing block (one warp per token): up to this many tokens the
+// routing launch is a single block.
+constexpr int ROUTE_TOKENS_PER_BLOCK = 8;
+// Dispatch done by a single routing block right after it has routed its
+// tokens (T <= 8): the arguments of decomoe_dispatch for Kd groups, x_perm
+// null when the rows are copied by a separate launch. counts null: none.
+struct RouteDispatch {
+  int32_t* counts = nullptr;
+  int32_t* offsets = nullptr;
+  int32_t* perm_token = nullptr;
+  int32_t* inv_slot = nullptr;
+  int32_t* status = nullptr;
+  const void* x = nullptr;
+  int row_vec = 0;  // 16-byte vectors per row
+  void* x_perm = nullptr;
+  int Kd = 0;
+};
 // decomoe_route_prefix reading its logits through src. defer_finalize: with
 // mass_out and more than one routing block, the per-block partial masses are
 // left in the workspace (their count returned in *mass_blocks) for a later
 // kernel to add up (launch_dispatch's extra blocks) instead of a separate
-// finalize launch.
+// finalize launch. K_dev: the prefix is read on the device (no mass).
+// rd: with one routing block, that block also dispatches its picks.
 int route_prefix_src(const float* logits, const RouteSrc& src, int64_t T, int E, int64_t ld, int K, int k,
                      int32_t* topk_idx, float* topk_w, double* mass_out, void* ws, size_t ws_bytes,
-                     bool defer_finalize, int* mass_blocks, cudaStream_t s);
+                     bool defer_finalize, int* mass_blocks, cudaStream_t s, const int32_t* K_dev = nullptr,
+                     const RouteDispatch* rd = nullptr);
+// The row gather of decomoe_dispatch: x_perm[r] = x[perm_token[r]] for the
+// offsets[K] routed rows (N = T*k rows at most).
+int launch_gather_rows(const void* x, const int32_t* perm_token, const int32_t* offsets, int K, size_t row_bytes,
+                       int64_t N, void* x_perm, cudaStream_t s);
 // decomoe_dispatch that also finishes a deferred activated mass: mass[e] =
 // fixed-order fp64 sum of mass_part[b][e] over mass_blocks blocks (no-op when
 // mass_part is null).

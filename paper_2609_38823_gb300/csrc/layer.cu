@@ -75,19 +75,41 @@ static int route_dispatch_src(const float* logits, const RouteSrc& src, int64_t 
   void* route_ws = ws;
   void* disp_ws = static_cast<uint8_t*>(ws) + rbytes;
   int mass_blocks = 0;
+  // decode sizes (one routing block): that block also counts, ranks and, for
+  // up to 64 KiB of rows, gathers its picks; larger rows are copied by the
+  // gather launch
+  const bool one_block = T <= ROUTE_TOKENS_PER_BLOCK;
+  RouteDispatch rd;
+  if (one_block) {
+    rd.counts = counts;
+    rd.offsets = offsets;
+    rd.perm_token = perm_token;
+    rd.inv_slot = inv_slot;
+    rd.status = status_dev;
+    rd.x = x;
+    rd.row_vec = static_cast<int>(row_bytes / 16);
+    rd.x_perm = (x_perm != nullptr && static_cast<size_t>(T) * k * row_bytes <= 64 * 1024) ? x_perm : nullptr;
+    rd.Kd = Kd;
+  }
   if (device_k) {
     // mass pass, Eq. 12 on the device, routing over [0, *K_dev) (from the
     // summed logits when the first pass read the router's partials)
     DM_RET(route_prefix_src(logits, src, T, E, E, E, k, nullptr, nullptr, mass_out, route_ws, rbytes, false, nullptr,
                             s));
     DM_RET(decomoe_select_prefix_device(mass_out, E, k, p, K_dev, stream));
-    DM_RET(decomoe_route_prefix_dk(src.logits_out != nullptr ? src.logits_out : logits, T, E, E, K_dev, k, topk_idx,
-                                   topk_w, stream));
+    DM_RET(route_prefix_src(src.logits_out != nullptr ? src.logits_out : logits, RouteSrc{}, T, E, E, E, k, topk_idx,
+                            topk_w, nullptr, nullptr, 0, false, nullptr, s, K_dev, one_block ? &rd : nullptr));
   } else {
     // one launch: prefix routing and, with mass_out, the full-pool partial
     // masses (finished by the dispatch launch)
     DM_RET(route_prefix_src(logits, src, T, E, E, K, k, topk_idx, topk_w, mass_out, route_ws, rbytes, true,
-                            &mass_blocks, s));
+                            &mass_blocks, s, nullptr, one_block ? &rd : nullptr));
+  }
+  if (one_block) {
+    // one routing block: the mass was written in place and the picks are dispatched
+    if (x_perm != nullptr && rd.x_perm == nullptr)
+      DM_RET(launch_gather_rows(x, perm_token, offsets, Kd, row_bytes, T * k, x_perm, s));
+    return DECOMOE_OK;
   }
   return dispatch_with_mass(topk_idx, T, k, Kd, x, d, dtype, counts, offsets, perm_token, inv_slot, x_perm, disp_ws,
                             dbytes, status_dev, mass_blocks > 0 ? static_cast<const double*>(route_ws) : nullptr,

@@ -4,7 +4,7 @@
 #include <cfloat>
 #include <cstdint>
 
-#include "decomoe_internal.cuh"
+#include "dispatch_tile.cuh"
 
 namespace decomoe {
 
@@ -119,7 +119,7 @@ __global__ void __launch_bounds__(32 * GEMV_WARPS)
 // per expert, summed in token order, to part[block][e]; k_mass_finalize sums
 // the blocks in a fixed order in fp64, so the mass is bit-reproducible.
 constexpr int ROUTE_THREADS = 256;
-constexpr int ROUTE_TPB = 8;  // tokens per block: one per warp
+constexpr int ROUTE_TPB = ROUTE_TOKENS_PER_BLOCK;  // tokens per block: one per warp
 
 // Order-preserving 32-bit key of a float (larger float -> larger key; -0 and
 // +0 share a key so equal values tie). Key 0 is below every float's key and
@@ -182,11 +182,14 @@ __device__ __forceinline__ float pick_weight(float my_v, int lane, int k) {
 // vectors (all NP in flight), adding them in slice order and the bias last,
 // storing the sums to src.logits_out and, through shared memory, into the
 // key layout (E % 4 == 0, 16-byte aligned rows).
+// rd.counts set (one block, T <= ROUTE_TPB): after routing, the block
+// dispatches its own picks (dispatch_tile over the T*k pairs).
+static_assert(ROUTE_THREADS == DSP_THREADS, "the routing block runs the dispatch tile");
 template <int NP>
 __global__ void __launch_bounds__(ROUTE_THREADS)
     k_route(const float* __restrict__ logits, int64_t Tn, int E, int64_t ld, int K, int k,
             int32_t* __restrict__ idx_out, float* __restrict__ w_out, double* __restrict__ part,
-            const int32_t* __restrict__ K_dev, int64_t skip_at, int64_t skip_len, RouteSrc src) {
+            const int32_t* __restrict__ K_dev, int64_t skip_at, int64_t skip_len, RouteSrc src, RouteDispatch rd) {
   pdl_enter();
   if (K_dev != nullptr) K = *K_dev;  // prefix chosen on the device (k <= K <= E by construction)
   __shared__ int s_idx[ROUTE_TPB][DECOMOE_MAX_TOPK];
@@ -262,17 +265,23 @@ __global__ void __launch_bounds__(ROUTE_THREADS)
       }
     }
   }
-  if (!mass) return;
-  __syncthreads();
-  const int ntok = static_cast<int>(Tn - static_cast<int64_t>(blockIdx.x) * ROUTE_TPB < ROUTE_TPB
-                                        ? Tn - static_cast<int64_t>(blockIdx.x) * ROUTE_TPB
-                                        : ROUTE_TPB);
-  for (int e = threadIdx.x; e < E; e += ROUTE_THREADS) {
-    float acc = 0.f;
-    for (int tt = 0; tt < ntok; ++tt)
-      for (int j = 0; j < k; ++j)
-        if (s_idx[tt][j] == e) acc += s_w[tt][j];  // token order, then slot order
-    part[static_cast<int64_t>(blockIdx.x) * E + e] = static_cast<double>(acc);
+  if (mass) {
+    __syncthreads();
+    const int ntok = static_cast<int>(Tn - static_cast<int64_t>(blockIdx.x) * ROUTE_TPB < ROUTE_TPB
+                                          ? Tn - static_cast<int64_t>(blockIdx.x) * ROUTE_TPB
+                                          : ROUTE_TPB);
+    for (int e = threadIdx.x; e < E; e += ROUTE_THREADS) {
+      float acc = 0.f;
+      for (int tt = 0; tt < ntok; ++tt)
+        for (int j = 0; j < k; ++j)
+          if (s_idx[tt][j] == e) acc += s_w[tt][j];  // token order, then slot order
+      part[static_cast<int64_t>(blockIdx.x) * E + e] = static_cast<double>(acc);
+    }
+  }
+  if (rd.counts != nullptr) {
+    __syncthreads();  // the block's picks in idx_out are visible to all its threads
+    dispatch_tile<true>(idx_out, Tn * k, k, rd.Kd, nullptr, 1, 0, rd.counts, rd.offsets, rd.perm_token, rd.inv_slot,
+                        rd.status, static_cast<const uint4*>(rd.x), rd.row_vec, static_cast<uint4*>(rd.x_perm));
   }
 }
 
@@ -324,7 +333,8 @@ int launch_skip_mass(const float* logits, int64_t n, int E, int64_t ld, int k, i
                      double* part, double* mass, cudaStream_t s) {
   const int64_t nblocks = (n + ROUTE_TPB - 1) / ROUTE_TPB;
   k_route<1><<<static_cast<unsigned>(nblocks), ROUTE_THREADS, 0, s>>>(logits, n, E, ld, E, k, nullptr, nullptr, part,
-                                                                      nullptr, skip_at, skip_len, RouteSrc{});
+                                                                      nullptr, skip_at, skip_len, RouteSrc{},
+                                                                      RouteDispatch{});
   DM_LAUNCH_CHECK("k_route");
   k_mass_finalize<<<E, 256, 0, s>>>(part, static_cast<int>(nblocks), E, mass);
   DM_LAUNCH_CHECK("k_mass_finalize");
@@ -414,12 +424,14 @@ namespace decomoe {
 
 int route_prefix_src(const float* logits, const RouteSrc& src, int64_t T, int E, int64_t ld, int K, int k,
                      int32_t* topk_idx, float* topk_w, double* mass_out, void* ws, size_t ws_bytes,
-                     bool defer_finalize, int* mass_blocks, cudaStream_t s) {
+                     bool defer_finalize, int* mass_blocks, cudaStream_t s, const int32_t* K_dev,
+                     const RouteDispatch* rd) {
   if (mass_blocks != nullptr) *mass_blocks = 0;
   DM_ARG_CHECK(T >= 0, "route_prefix: T < 0");
   DM_ARG_CHECK(E >= 1 && E <= DECOMOE_MAX_E, "route_prefix: E=%d outside [1, %d]", E, DECOMOE_MAX_E);
   DM_ARG_CHECK(k >= 1 && k <= DECOMOE_MAX_TOPK, "route_prefix: k=%d outside [1, %d]", k, DECOMOE_MAX_TOPK);
-  DM_ARG_CHECK(K >= k && K <= E, "route_prefix: need k <= K <= E (k=%d K=%d E=%d)", k, K, E);
+  DM_ARG_CHECK(K_dev != nullptr || (K >= k && K <= E), "route_prefix: need k <= K <= E (k=%d K=%d E=%d)", k, K, E);
+  DM_ARG_CHECK(K_dev == nullptr || mass_out == nullptr, "route_prefix: a device prefix takes no mass");
   DM_ARG_CHECK(ld >= E, "route_prefix: ld < E");
   DM_ARG_CHECK(src.nparts == 1 || ((src.nparts == 4 || src.nparts == 16) && E % 4 == 0 && ld == E &&
                                     src.part_stride % 4 == 0 && aligned16(logits) &&
@@ -443,10 +455,15 @@ int route_prefix_src(const float* logits, const RouteSrc& src, int64_t T, int E,
     // finalize would only add zeros), so it is written in place
     part = nblocks == 1 ? mass_out : static_cast<double*>(ws);
   }
+  RouteDispatch rdv;
+  if (rd != nullptr && rd->counts != nullptr) {
+    DM_ARG_CHECK(nblocks == 1 && topk_idx != nullptr && T * k <= DSP_TILE,
+                 "route_prefix: dispatch in the routing block needs T <= %d", ROUTE_TPB);
+    rdv = *rd;
+  }
   auto kern = src.nparts == 16 ? k_route<16> : src.nparts == 4 ? k_route<4> : k_route<1>;
   DM_CUDA_CHECK(launch_pdl(kern, dim3(static_cast<unsigned>(nblocks)), dim3(ROUTE_THREADS), 0, s, logits, T, E, ld,
-                           K, k, topk_idx, topk_w, part, static_cast<const int32_t*>(nullptr), INT64_MAX,
-                           static_cast<int64_t>(0), src));
+                           K, k, topk_idx, topk_w, part, K_dev, INT64_MAX, static_cast<int64_t>(0), src, rdv));
   if (mass_out != nullptr && nblocks > 1) {
     if (defer_finalize && mass_blocks != nullptr) {
       *mass_blocks = static_cast<int>(nblocks);  // the caller's next kernel adds the partials up
@@ -481,12 +498,8 @@ int decomoe_route_prefix_dk(const float* logits, int64_t T, int E, int64_t ld, c
                "route_prefix_dk: bad sizes");
   if (T == 0) return DECOMOE_OK;
   DM_ARG_CHECK(logits && K_dev, "route_prefix_dk: null pointer");
-  const int64_t nblocks = (T + ROUTE_TPB - 1) / ROUTE_TPB;
-  DM_ARG_CHECK(nblocks <= 0x7fffffff, "route_prefix_dk: T too large");
-  DM_CUDA_CHECK(launch_pdl(k_route<1>, dim3(static_cast<unsigned>(nblocks)), dim3(ROUTE_THREADS), 0,
-                           reinterpret_cast<cudaStream_t>(stream), logits, T, E, ld, E, k, topk_idx, topk_w,
-                           static_cast<double*>(nullptr), K_dev, INT64_MAX, static_cast<int64_t>(0), RouteSrc{}));
-  return DECOMOE_OK;
+  return route_prefix_src(logits, RouteSrc{}, T, E, ld, E, k, topk_idx, topk_w, nullptr, nullptr, 0, false, nullptr,
+                          reinterpret_cast<cudaStream_t>(stream), K_dev);
 }
 
 }  // extern "C"
