@@ -51,14 +51,16 @@ struct DropRows {
   int64_t v0 = 0, nv = 0;
 };
 
-template <bool BF16, int KT, bool DROP>
-__global__ void __launch_bounds__(256)
+// WPT warps per token, each taking alternate 32-vector chunks of the row:
+// many tokens take one warp each (two blocks resident per SM), few tokens
+// spread each row over more warps.
+template <bool BF16, int KT, bool DROP, int WPT>
+__global__ void __launch_bounds__(256, WPT == 1 ? 2 : 1)
     k_combine(const uint4* __restrict__ y, const int32_t* __restrict__ inv_slot,
               const float* __restrict__ w, int64_t Tn, int k, int vec,
               const uint4* __restrict__ residual, uint4* __restrict__ out, DropRows drop) {
   pdl_enter();
   constexpr int NE = BF16 ? 8 : 4;
-  constexpr int WPT = 2;  // warps per token: each takes alternate 32-vector chunks
   const int lane = threadIdx.x & 31;
   const int64_t gw = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int64_t nw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
@@ -133,23 +135,35 @@ __global__ void __launch_bounds__(256)
   }
 }
 
-template <bool BF16, bool DROP>
-static cudaError_t launch_combine_k(int grid, cudaStream_t s, const uint4* y, const int32_t* inv, const float* w,
-                                    int64_t T, int k, int vec, const uint4* res, uint4* out, DropRows drop) {
+static int grid_for_warps(int64_t warps);
+
+template <bool BF16, bool DROP, int WPT>
+static cudaError_t launch_combine_w(cudaStream_t s, const uint4* y, const int32_t* inv, const float* w, int64_t T,
+                                    int k, int vec, const uint4* res, uint4* out, DropRows drop) {
+  const dim3 g(grid_for_warps(WPT * T)), b(256);
   switch (k) {
-    case 1: return launch_pdl(k_combine<BF16, 1, DROP>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out, drop);
-    case 2: return launch_pdl(k_combine<BF16, 2, DROP>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out, drop);
-    case 4: return launch_pdl(k_combine<BF16, 4, DROP>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out, drop);
-    case 8: return launch_pdl(k_combine<BF16, 8, DROP>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out, drop);
-    default:
-      return launch_pdl(k_combine<BF16, 0, DROP>, dim3(grid), dim3(256), 0, s, y, inv, w, T, k, vec, res, out, drop);
+    case 1: return launch_pdl(k_combine<BF16, 1, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop);
+    case 2: return launch_pdl(k_combine<BF16, 2, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop);
+    case 4: return launch_pdl(k_combine<BF16, 4, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop);
+    case 8: return launch_pdl(k_combine<BF16, 8, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop);
+    default: return launch_pdl(k_combine<BF16, 0, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop);
   }
 }
+// Warps per token by token count: one from 1024 tokens on, two from 256, four
+// from 32, eight below (a decode step's row then spans eight warps).
+template <bool BF16, bool DROP>
+static cudaError_t launch_combine_k(cudaStream_t s, const uint4* y, const int32_t* inv, const float* w, int64_t T,
+                                    int k, int vec, const uint4* res, uint4* out, DropRows drop) {
+  if (T >= 1024) return launch_combine_w<BF16, DROP, 1>(s, y, inv, w, T, k, vec, res, out, drop);
+  if (T >= 256) return launch_combine_w<BF16, DROP, 2>(s, y, inv, w, T, k, vec, res, out, drop);
+  if (T >= 32) return launch_combine_w<BF16, DROP, 4>(s, y, inv, w, T, k, vec, res, out, drop);
+  return launch_combine_w<BF16, DROP, 8>(s, y, inv, w, T, k, vec, res, out, drop);
+}
 template <bool BF16>
-static cudaError_t launch_combine(int grid, cudaStream_t s, const uint4* y, const int32_t* inv, const float* w,
-                                  int64_t T, int k, int vec, const uint4* res, uint4* out, DropRows drop) {
-  return drop.text != nullptr ? launch_combine_k<BF16, true>(grid, s, y, inv, w, T, k, vec, res, out, drop)
-                              : launch_combine_k<BF16, false>(grid, s, y, inv, w, T, k, vec, res, out, drop);
+static cudaError_t launch_combine(cudaStream_t s, const uint4* y, const int32_t* inv, const float* w, int64_t T,
+                                  int k, int vec, const uint4* res, uint4* out, DropRows drop) {
+  return drop.text != nullptr ? launch_combine_k<BF16, true>(s, y, inv, w, T, k, vec, res, out, drop)
+                              : launch_combine_k<BF16, false>(s, y, inv, w, T, k, vec, res, out, drop);
 }
 
 // ------------------------------------------------------------------ compaction
@@ -321,12 +335,11 @@ int combine_impl(const void* y_perm, const int32_t* inv_slot, const float* topk_
   }
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const int vec = static_cast<int>(row_bytes / 16);
-  const int grid = grid_for_warps(2 * T);  // two warps per token
   if (dtype == DECOMOE_BF16)
-    DM_CUDA_CHECK(launch_combine<true>(grid, s, static_cast<const uint4*>(y_perm), inv_slot, topk_w, T, k, vec,
+    DM_CUDA_CHECK(launch_combine<true>(s, static_cast<const uint4*>(y_perm), inv_slot, topk_w, T, k, vec,
                                        static_cast<const uint4*>(residual), static_cast<uint4*>(out), drop));
   else
-    DM_CUDA_CHECK(launch_combine<false>(grid, s, static_cast<const uint4*>(y_perm), inv_slot, topk_w, T, k, vec,
+    DM_CUDA_CHECK(launch_combine<false>(s, static_cast<const uint4*>(y_perm), inv_slot, topk_w, T, k, vec,
                                         static_cast<const uint4*>(residual), static_cast<uint4*>(out), drop));
   return DECOMOE_OK;
 }
