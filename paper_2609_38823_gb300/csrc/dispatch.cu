@@ -277,13 +277,6 @@ extern "C" int decomoe_dispatch_noalloc(const int32_t* topk_idx, int64_t T, int 
   k_dispatch_scatter<false><<<ntiles, DSP_THREADS, 0, s>>>(topk_idx, N, k, K, tile_hist, ntiles, counts, offsets,
                                                     perm_token, inv_slot);
   DM_LAUNCH_CHECK("k_dispatch_scatter");
-  if (x_perm != nullptr) {
-    const int vec = static_cast<int>(row_bytes / 16);
-    int blocks = static_cast<int>(std::min<int64_t>((N * 32 + 255) / 256, sm_count() * 8LL));
-    if (blocks < 1) blocks = 1;
-    DM_CUDA_CHECK(launch_pdl(k_gather_rows, dim3(blocks), dim3(256), 0, s, static_cast<const uint4*>(x),
-                             static_cast<const int32_t*>(perm_token), static_cast<const int32_t*>(offsets), K, vec,
-                             static_cast<uint4*>(x_perm)));
-  }
+  if (x_perm != nullptr) DM_RET(launch_gather_rows(x, perm_token, offsets, K, row_bytes, N, x_perm, s));
   return DECOMOE_OK;
 }
