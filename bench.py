@@ -425,9 +425,9 @@ def ours(args, ws, rank, local):
                 ev_in[b].record(s_in)
             s_comp.wait_event(ev_in[b])
             s_comp.wait_event(ev_out[b])          # out_dev[b] copied out by step i-2
+            # the layer with its output's visual-block removal (the exit layer)
             dm.decomoe_moe_layer(x_dev[b], L.w_r, L.bias, L.w_gu, L.w_down, k, out_dev[b], lws, K_fixed=K,
-                                 p=args.p, status=B.status)
-            dm.decomoe_drop_visual_block(out_dev[b], text, v0, nv)
+                                 p=args.p, status=B.status, text_out=text, v0=v0, nv=nv)
             ev_comp[b].record(s_comp)
             with torch.cuda.stream(s_out):
                 s_out.wait_event(ev_comp[b])
@@ -438,8 +438,7 @@ def ours(args, ws, rank, local):
             L = layers[i % len(layers)]
             x_dev[0].copy_(xs_host[i % len(layers)], non_blocking=True)
             dm.decomoe_moe_layer(x_dev[0], L.w_r, L.bias, L.w_gu, L.w_down, k, out_dev[0], lws, K_fixed=K,
-                                 p=args.p, status=B.status)
-            dm.decomoe_drop_visual_block(out_dev[0], text, v0, nv)
+                                 p=args.p, status=B.status, text_out=text, v0=v0, nv=nv)
             out_host[0].copy_(out_dev[0], non_blocking=True)
 
         def timed_all_streams(fn, steps, warmup):
@@ -466,8 +465,9 @@ def ours(args, ws, rank, local):
         e2e = {"value": round(job_rate(T * e_steps, ws, ms_e), 1), "unit": "tokens/s",
                "h2d_bytes_per_step": T * wl.d * 2, "d2h_bytes_per_step": T * wl.d * 2,
                "ms_per_step": round(ms_e / e_steps, 4), "steps": e_steps,
-               "path": "pinned host x -> decomoe_moe_layer + decomoe_drop_visual_block (C ABI, eager) -> pinned "
-                       "host out; copy-in, compute and copy-out on three streams, double-buffered",
+               "path": "pinned host x -> decomoe_moe_layer_exit (the layer and its output's visual-block removal; "
+                       "C ABI, eager) -> pinned host out; copy-in, compute and copy-out on three streams, "
+                       "double-buffered",
                "serial": {"value": round(job_rate(T * e_steps, ws, ms_s), 1),
                           "ms_per_step": round(ms_s / e_steps, 4)}}
 

@@ -460,6 +460,19 @@ DECOMOE_API int decomoe_moe_layer(const void* x, const void* w_r, const float* b
                       int* K_sel_host, void* ws, size_t ws_bytes, int32_t* status_dev,
                       decomoe_stream_t stream);
 
+/* The exit layer of Algorithm 2: decomoe_moe_layer whose output also leaves
+ * the visual block (Section 3.2) in the same combine launch: out [T, d] as
+ * decomoe_moe_layer writes it, and its text rows (outside [v0, v0 + nv)) in
+ * order in text_out [T - nv, d] — bit-identical to decomoe_moe_layer followed
+ * by decomoe_drop_visual_block(out, text_out, ...). Needs 0 <= v0, 0 <= nv,
+ * v0 + nv <= T, text_out 16-byte aligned and apart from out (may be NULL
+ * when nv == T). Other arguments as decomoe_moe_layer. */
+DECOMOE_API int decomoe_moe_layer_exit(const void* x, const void* w_r, const float* bias, const void* w_gate_up,
+                                       const void* w_down, int64_t T, int d, int E, int k, int m, int dtype,
+                                       int K_fixed, double p, const void* residual, void* out, void* text_out,
+                                       int64_t v0, int64_t nv, int* K_used_host, int* K_sel_host, void* ws,
+                                       size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream);
+
 /* Offsets (bytes) of the intermediates inside the decomoe_moe_layer workspace,
  * for inspection: logits, topk_idx, topk_w, mass, counts, offsets, perm_token,
  * inv_slot, x_perm, h, y_perm, device K (12 entries written to offs_host). */

@@ -81,6 +81,8 @@ SIGNATURES = {
     "decomoe_moe_layer_workspace_bytes": (_S, [_L, _I, _I, _I, _I, _I]),
     "decomoe_moe_layer": (_I, [_P, _P, _P, _P, _P, _L, _I, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P,
                                _P, _S, _P, _P]),
+    "decomoe_moe_layer_exit": (_I, [_P, _P, _P, _P, _P, _L, _I, _I, _I, _I, _I, _I, _D, _P, _P, _P, _L, _L, _P,
+                                    _P, _P, _S, _P, _P]),
     "decomoe_moe_layer_workspace_layout": (_I, [_L, _I, _I, _I, _I, _I, _P]),
     "decomoe_read_status": (_I, [_P, _P, _P]),
     "decomoe_set_wait_limit_ns": (_I, [_L]),
@@ -497,18 +499,28 @@ def decomoe_rmsnorm(x, y, eps=1e-6, stream=None):
 
 
 def decomoe_moe_layer(x, w_r, bias, w_gate_up, w_down, k, out, ws, K_fixed=0, p=0.0, residual=None,
-                      status=None, stream=None):
-    """One RCEP MoE invocation. Returns (K_used, K_selected or None)."""
-    _need_cuda(x, w_r, bias, w_gate_up, w_down, out, ws, residual, status)
+                      status=None, stream=None, text_out=None, v0=0, nv=0):
+    """One RCEP MoE invocation. Returns (K_used, K_selected or None). With
+    text_out, the exit layer: the output's text rows (outside [v0, v0 + nv))
+    are also stored, compacted, to text_out."""
+    _need_cuda(x, w_r, bias, w_gate_up, w_down, out, ws, residual, status, text_out)
     T, d = x.shape
     E = w_r.shape[0]
     m = w_down.shape[2]
     Ku, Ks = ctypes.c_int(0), ctypes.c_int(-1)
-    _check("decomoe_moe_layer",
-           lib().decomoe_moe_layer(_ptr(x), _ptr(w_r), _ptr(bias), _ptr(w_gate_up), _ptr(w_down), T, d, E,
-                                   k, m, _dt(x), int(K_fixed), float(p), _ptr(residual), _ptr(out),
-                                   ctypes.byref(Ku), ctypes.byref(Ks), _ptr(ws),
-                                   ws.numel() * ws.element_size(), _ptr(status), _stream(stream)))
+    if text_out is None:
+        _check("decomoe_moe_layer",
+               lib().decomoe_moe_layer(_ptr(x), _ptr(w_r), _ptr(bias), _ptr(w_gate_up), _ptr(w_down), T, d, E,
+                                       k, m, _dt(x), int(K_fixed), float(p), _ptr(residual), _ptr(out),
+                                       ctypes.byref(Ku), ctypes.byref(Ks), _ptr(ws),
+                                       ws.numel() * ws.element_size(), _ptr(status), _stream(stream)))
+    else:
+        _check("decomoe_moe_layer_exit",
+               lib().decomoe_moe_layer_exit(_ptr(x), _ptr(w_r), _ptr(bias), _ptr(w_gate_up), _ptr(w_down), T, d,
+                                            E, k, m, _dt(x), int(K_fixed), float(p), _ptr(residual), _ptr(out),
+                                            _ptr(text_out), int(v0), int(nv), ctypes.byref(Ku), ctypes.byref(Ks),
+                                            _ptr(ws), ws.numel() * ws.element_size(), _ptr(status),
+                                            _stream(stream)))
     return Ku.value, (Ks.value if Ks.value >= 0 else None)
 
 

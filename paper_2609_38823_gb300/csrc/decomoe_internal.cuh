@@ -154,6 +154,12 @@ int combine_impl(const void* y_perm, const int32_t* inv_slot, const float* topk_
 int drop_visual_block_impl(const int32_t* flag, const void* src, void* dst, int64_t rows, int64_t row_bytes,
                            int64_t v0, int64_t nv, int64_t nbatch, int64_t src_batch_stride,
                            int64_t dst_batch_stride, decomoe_stream_t stream);
+// decomoe_moe_layer; with text_out also the visual-block removal of its output
+// (decomoe_moe_layer_exit).
+int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void* w_gate_up, const void* w_down,
+                   int64_t T, int d, int E, int k, int m, int dtype, int K_fixed, double p, const void* residual,
+                   void* out, void* text_out, int64_t v0, int64_t nv, int* K_used_host, int* K_sel_host, void* ws,
+                   size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream);
 // The k-split router's GEMM alone: KS slices of partial logits [KS][T][E]
 // (no bias) into scratch; returns KS (1: no split at this size, nothing
 // launched).

@@ -253,6 +253,32 @@ int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const v
                       double p, const void* residual, void* out, int* K_used_host, int* K_sel_host, void* ws,
                       size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream) {
   clear_error();
+  return moe_layer_impl(x, w_r, bias, w_gate_up, w_down, T, d, E, k, m, dtype, K_fixed, p, residual, out, nullptr,
+                        0, 0, K_used_host, K_sel_host, ws, ws_bytes, status_dev, stream);
+}
+
+int decomoe_moe_layer_exit(const void* x, const void* w_r, const float* bias, const void* w_gate_up,
+                           const void* w_down, int64_t T, int d, int E, int k, int m, int dtype, int K_fixed,
+                           double p, const void* residual, void* out, void* text_out, int64_t v0, int64_t nv,
+                           int* K_used_host, int* K_sel_host, void* ws, size_t ws_bytes, int32_t* status_dev,
+                           decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(v0 >= 0 && nv >= 0 && v0 + nv <= T, "moe_layer_exit: visual block [%lld, %lld) outside [0, %lld)",
+               (long long)v0, (long long)(v0 + nv), (long long)T);
+  DM_ARG_CHECK(text_out != nullptr || T - nv == 0, "moe_layer_exit: text_out is null");
+  return moe_layer_impl(x, w_r, bias, w_gate_up, w_down, T, d, E, k, m, dtype, K_fixed, p, residual, out,
+                        T - nv > 0 ? text_out : nullptr, v0, nv, K_used_host, K_sel_host, ws, ws_bytes, status_dev,
+                        stream);
+}
+
+}  // extern "C"
+
+namespace decomoe {
+
+int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void* w_gate_up, const void* w_down,
+                   int64_t T, int d, int E, int k, int m, int dtype, int K_fixed, double p, const void* residual,
+                   void* out, void* text_out, int64_t v0, int64_t nv, int* K_used_host, int* K_sel_host, void* ws,
+                   size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream) {
   DM_ARG_CHECK(T >= 0 && d > 0 && m > 0, "moe_layer: bad sizes");
   DM_ARG_CHECK(E >= 1 && E <= DECOMOE_MAX_E && k >= 1 && k <= DECOMOE_MAX_TOPK && k <= E,
                "moe_layer: need 1 <= k <= E <= %d, k <= %d", DECOMOE_MAX_E, DECOMOE_MAX_TOPK);
@@ -330,9 +356,8 @@ int decomoe_moe_layer(const void* x, const void* w_r, const float* bias, const v
   // reset between the launches, which keeps them chained programmatically)
   DM_RET(decomoe_expert_swiglu(x_perm, offsets, T * k, K, d, m, dtype, w_gate_up, w_down, h, y_perm,
                                status_dev, nullptr, stream));
-  // a7: combine (+ residual)
-  DM_RET(decomoe_combine(y_perm, inv, topk_w, T, k, d, dtype, residual, out, stream));
-  return DECOMOE_OK;
+  // a7: combine (+ residual); with text_out also a8 on the layer output
+  return combine_impl(y_perm, inv, topk_w, T, k, d, dtype, residual, out, text_out, v0, nv, stream);
 }
 
-}  // extern "C"
+}  // namespace decomoe

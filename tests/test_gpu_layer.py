@@ -275,3 +275,30 @@ def test_layer_intermediates_equal_separate_calls(T, K_fixed, p):
     assert torch.equal(got["xp"].view(torch.int16), xp.view(torch.int16))
     if K_fixed == -1 or p > 0:
         assert torch.equal(mass_l.view(torch.int64), mass.cpu().view(torch.int64))
+
+
+@pytest.mark.parametrize("T,K_fixed,v0,nv", [(2048, 64, 0, 1792), (300, -1, 16, 200), (8, 64, 7, 1), (64, 40, 0, 64)])
+def test_layer_exit_equals_layer_then_removal(prefill_layer, T, K_fixed, v0, nv):
+    """decomoe_moe_layer_exit writes the same layer output as
+    decomoe_moe_layer and the same compacted text rows as a
+    decomoe_drop_visual_block of that output, bit for bit."""
+    wl, g, _ = prefill_layer
+    x = g["x"][:T].contiguous()
+    w_gu = dm.fuse_gate_up(g["w_gate"], g["w_up"])
+    d, E, k, m = wl.d, wl.E, wl.k, wl.m
+    ws1 = dm.workspace(dm.decomoe_moe_layer_workspace_bytes(T, d, E, k, m, dm.DECOMOE_BF16), DEV)
+    ws2 = dm.workspace(dm.decomoe_moe_layer_workspace_bytes(T, d, E, k, m, dm.DECOMOE_BF16), DEV)
+    out1, out2 = torch.empty_like(x), torch.empty_like(x)
+    text1 = torch.full((T - nv, d), 5.0, dtype=x.dtype, device=DEV)
+    text2 = torch.full((T - nv, d), -5.0, dtype=x.dtype, device=DEV)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    dm.decomoe_moe_layer(x, g["w_r"], g["bias"], w_gu, g["w_down"], k, out1, ws1, K_fixed=K_fixed, p=0.7,
+                         status=st, text_out=text1, v0=v0, nv=nv)
+    dm.decomoe_moe_layer(x, g["w_r"], g["bias"], w_gu, g["w_down"], k, out2, ws2, K_fixed=K_fixed, p=0.7,
+                         status=st)
+    if T - nv > 0:
+        dm.decomoe_drop_visual_block(out2, text2, v0, nv)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(st) == 0
+    assert torch.equal(out1.view(torch.int16), out2.view(torch.int16))
+    assert torch.equal(text1.view(torch.int16), text2.view(torch.int16))
