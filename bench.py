@@ -211,6 +211,7 @@ class Buffers:
         self.inv = torch.empty(R, dtype=torch.int32, device=dev)
         self.rd_ws = dm.workspace(dm.decomoe_route_dispatch_workspace_bytes(T, k, E), dev)
         self.rrd_ws = dm.workspace(dm.decomoe_router_route_dispatch_workspace_bytes(T, wl.d, E, k), dev)
+        self.lws = dm.workspace(dm.decomoe_moe_layer_workspace_bytes(T, wl.d, E, k, wl.m, dm.DECOMOE_BF16), dev)
         self.x_perm = torch.empty(R, d, dtype=torch.bfloat16, device=dev)
         self.h = torch.empty(R, m, dtype=torch.bfloat16, device=dev)
         self.y = torch.empty(R, d, dtype=torch.bfloat16, device=dev)
@@ -219,20 +220,24 @@ class Buffers:
 
 
 def run_step(dm, wl, L, B, K, v0, nv, text, ev=None):
-    """One pass of the hot path, every step a C-ABI call."""
+    """One pass of the hot path. Without events: one C-ABI call, the layer
+    (with its output's visual-block removal when text is given), K fixed and
+    the activated mass computed. With events (to time the two expert GEMMs):
+    the same kernels through the calls of the individual steps."""
     k, E = wl.k, wl.E
+    if ev is None:
+        dm.decomoe_moe_layer(L.x, L.w_r, L.bias, L.w_gu, L.w_down, k, B.out, B.lws, K_fixed=K, p=0.7,
+                             status=B.status, text_out=text, v0=v0, nv=nv)
+        return
     # a1 + a2 (Eq. 11) + a4 + a5: router logits, routing with the activated
     # mass, dispatch
     dm.decomoe_router_route_dispatch(L.x, L.w_r, L.bias, B.logits, K, k, B.idx, B.w, B.counts[:K], B.offsets[:K + 1],
                                      B.perm, B.inv, B.x_perm, B.rrd_ws, mass_out=B.mass, status=B.status)
-    if ev is not None:
-        ev[0].record()
+    ev[0].record()
     dm.decomoe_expert_gate_up(B.x_perm, B.offsets[:K + 1], K, L.w_gu, B.h, B.status)  # a6 gate/up
-    if ev is not None:
-        ev[1].record()
+    ev[1].record()
     dm.decomoe_expert_down(B.h, B.offsets[:K + 1], K, L.w_down, B.y, B.status)  # a6 down
-    if ev is not None:
-        ev[2].record()
+    ev[2].record()
     if text is not None:
         # a7 + a8: combine, the text rows also stored to the compacted buffer
         dm.decomoe_combine_drop_visual_block(B.y, B.inv, B.w, B.out, text, v0, nv)
@@ -357,10 +362,12 @@ def ours(args, ws, rank, local):
         del ev_graphs
     # distinct active experts per layer (for the algorithmic bytes)
     Ds = []
+    c_off = dm.decomoe_moe_layer_workspace_layout(T, wl.d, wl.E, k, wl.m, dm.DECOMOE_BF16)[4]
+    layer_counts = B.lws[c_off:c_off + 4 * wl.E].view(torch.int32)
     for l in range(len(layers)):
         run_step(dm, wl, layers[l], B, K, v0, nv, text)
         torch.cuda.synchronize()
-        Ds.append(int((B.counts[:K] > 0).sum()))
+        Ds.append(int((layer_counts[:K] > 0).sum()))
     D = statistics.mean(Ds)
     gu_flops = 2.0 * R * wl.d * 2 * wl.m
     dn_flops = 2.0 * R * wl.m * wl.d

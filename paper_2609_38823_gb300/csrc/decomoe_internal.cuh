@@ -130,10 +130,12 @@ struct RouteDispatch {
 // kernel to add up (launch_dispatch's extra blocks) instead of a separate
 // finalize launch. K_dev: the prefix is read on the device (no mass).
 // rd: with one routing block, that block also dispatches its picks.
+// zero_ints: n_zero int32 that the launch clears (for a later launch of the
+// same chain).
 int route_prefix_src(const float* logits, const RouteSrc& src, int64_t T, int E, int64_t ld, int K, int k,
                      int32_t* topk_idx, float* topk_w, double* mass_out, void* ws, size_t ws_bytes,
                      bool defer_finalize, int* mass_blocks, cudaStream_t s, const int32_t* K_dev = nullptr,
-                     const RouteDispatch* rd = nullptr);
+                     const RouteDispatch* rd = nullptr, int32_t* zero_ints = nullptr, int n_zero = 0);
 // The row gather of decomoe_dispatch: x_perm[r] = x[perm_token[r]] for the
 // offsets[K] routed rows (N = T*k rows at most).
 int launch_gather_rows(const void* x, const int32_t* perm_token, const int32_t* offsets, int K, size_t row_bytes,
@@ -160,6 +162,12 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
                    int64_t T, int d, int E, int k, int m, int dtype, int K_fixed, double p, const void* residual,
                    void* out, void* text_out, int64_t v0, int64_t nv, int* K_used_host, int* K_sel_host, void* ws,
                    size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream);
+// Both expert GEMMs of a decode-size invocation (bf16, at most 8 rows per
+// expert on average) in one launch; ready: K int32, zero at launch. Sets
+// *launched = false (and launches nothing) at other sizes.
+int launch_expert_ffn_fused(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m, int dtype,
+                            const void* w_gate_up, const void* w_down, void* h, void* y_perm, int32_t* ready,
+                            int32_t* status, cudaStream_t s, bool* launched);
 // The k-split router's GEMM alone: KS slices of partial logits [KS][T][E]
 // (no bias) into scratch; returns KS (1: no split at this size, nothing
 // launched).

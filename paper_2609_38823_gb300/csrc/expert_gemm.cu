@@ -1125,6 +1125,448 @@ __global__ void __launch_bounds__(192, 1)
 #undef DRAIN_BAR
 }
 
+// ------------------------------------------------------------------ fused decode FFN
+// Gate/up and down of the weights-stationary decode path in one persistent
+// launch. Work items: every gate/up tile of k_moe_ws<true> first, then every
+// down tile of k_moe_ws<false> (each list in k_moe_ws's order), handed out
+// round robin. A down tile of expert e reads h rows that the gate/up tiles
+// of e write, so after storing its h slice a gate/up tile bumps ready[e]
+// (release), and a down tile first issues the loads of its own weight
+// k-blocks (they depend on nothing), then waits until ready[e] counts all of
+// e's gate/up tiles (acquire, bounded) before loading its h rows. CTAs whose
+// first item is a down tile thus stream their weights while the gate/up
+// tiles run, and no launch separates the two GEMMs. Deadlock-free with at
+// most one CTA per SM and grid <= SMs: gate/up items never wait, and every
+// CTA reaches its gate/up items before any down item. ready[] must be zero at
+// launch (the layer's routing launch clears it).
+struct WsFfnArgs {
+  const int32_t* offsets;  // [G + 1] token row offsets per expert
+  int G;
+  int rows;
+  int wrows1, kdim1;  // gate/up: 2m weight rows per expert, K = d
+  int wrows2, kdim2;  // down: d weight rows per expert, K = m
+  void* h;            // [rows, m] bf16, gate/up output and down input
+  int64_t h_ld;
+  void* y;  // [rows, d] bf16
+  int64_t y_ld;
+  int32_t* ready;  // [G] finished gate/up tiles per expert; zero at launch
+  int32_t* status;
+  uint64_t limit_ns;
+};
+
+template <int STAGES, int BN>
+struct WsFfnCfg {
+  static constexpr int A_BYTES = WS_BM * WS_BK * 2;
+  static constexpr int B_BYTES = BN * WS_BK * 2;
+  static constexpr int BOX_BYTES = WS_BOX * WS_BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int TMEM_COLS = 2 * BN;
+  static constexpr int MAXG = DECOMOE_MAX_E;
+  static constexpr int NBARS = 2 * STAGES + 5;
+  static constexpr int XCH_BYTES = 2 * 2 * 32 * 32 * 4;   // SwiGLU up values, double-buffered
+  static constexpr int STILE_BYTES = 2 * 32 * WS_BM * 2;  // [2][32 tokens][128 features] bf16
+  static constexpr size_t SMEM = 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + XCH_BYTES + STILE_BYTES +
+                                 NBARS * 8 + 3 * (MAXG + 1) * 4 + 16;
+};
+
+template <int BN>
+constexpr int ffn_ws_max_stages() {
+  constexpr size_t fixed = WsFfnCfg<1, BN>::SMEM - WsFfnCfg<1, BN>::STAGE_BYTES - 2 * 8;
+  constexpr size_t per = WsFfnCfg<1, BN>::STAGE_BYTES + 2 * 8;
+  constexpr int n = static_cast<int>((232448 - fixed) / per);
+  return n > 12 ? 12 : n;
+}
+
+__device__ __forceinline__ void fence_proxy_async_all() { asm volatile("fence.proxy.async;" ::: "memory"); }
+
+template <int STAGES, int BN>
+__global__ void __launch_bounds__(192, 1)
+    k_ffn_ws(const __grid_constant__ CUtensorMap tma_w1, const __grid_constant__ CUtensorMap tma_x1,
+             const __grid_constant__ CUtensorMap tma_w2, const __grid_constant__ CUtensorMap tma_x2,
+             const WsFfnArgs g) {
+  using C = WsFfnCfg<STAGES, BN>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
+  uint8_t* smem = smem_raw + pad;
+  const uint32_t sA = raw + pad;
+  const uint32_t sB = sA + STAGES * C::A_BYTES;
+  float* xch = reinterpret_cast<float*>(smem + STAGES * C::STAGE_BYTES);
+  __nv_bfloat16* stile = reinterpret_cast<__nv_bfloat16*>(smem + STAGES * C::STAGE_BYTES + C::XCH_BYTES);
+  uint64_t* bars =
+      reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES + C::XCH_BYTES + C::STILE_BYTES);
+  int* s_off = reinterpret_cast<int*>(bars + C::NBARS);
+  int* s_tt1 = s_off + (C::MAXG + 1);
+  int* s_tt2 = s_tt1 + (C::MAXG + 1);
+  volatile uint32_t* s_tmem = reinterpret_cast<volatile uint32_t*>(s_tt2 + (C::MAXG + 1));
+  volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t bar0 = smem_u32(bars);
+#define FULL_BAR(s) (bar0 + 8u * (s))
+#define EMPTY_BAR(s) (bar0 + 8u * (STAGES + (s)))
+#define TFULL_BAR(a) (bar0 + 8u * (2 * STAGES + (a)))
+#define TEMPTY_BAR(a) (bar0 + 8u * (2 * STAGES + 2 + (a)))
+#define DRAIN_BAR (bar0 + 8u * (2 * STAGES + 4))
+
+  const int G = g.G;
+  const int nwb1 = g.wrows1 / WS_BM, nwb2 = g.wrows2 / WS_BM;
+  if (threadIdx.x == 0) {
+    *s_abort = 0;
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(FULL_BAR(s), 1);
+      mbar_init(EMPTY_BAR(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(TFULL_BAR(a), 1);
+      mbar_init(TEMPTY_BAR(a), 128);
+    }
+    mbar_init(DRAIN_BAR, 1);
+    fence_mbar_init();
+  }
+  pdl_wait();
+  for (int i = threadIdx.x; i <= G; i += blockDim.x) s_off[i] = g.offsets[i];
+  __syncthreads();
+  if (warp == 2 || warp == 3) {
+    // s_tt1 / s_tt2[e] = first gate/up / down item of expert e
+    const int nwb = warp == 2 ? nwb1 : nwb2;
+    int* s_tt = warp == 2 ? s_tt1 : s_tt2;
+    const int per = (G + 31) / 32;
+    int loc[8];
+    int sum = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      loc[i] = 0;
+      const int gi = lane * per + i;
+      if (i < per && gi < G) {
+        const int n = s_off[gi + 1] - s_off[gi];
+        loc[i] = n > 0 ? ((n + BN - 1) / BN) * nwb : 0;
+      }
+      sum += loc[i];
+    }
+    int incl = sum;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += v;
+    }
+    int run = incl - sum;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int gi = lane * per + i;
+      if (i < per && gi < G) s_tt[gi] = run;
+      run += loc[i];
+    }
+    if (lane == 31) s_tt[G] = incl;
+  }
+  __syncthreads();
+  const int total1 = s_tt1[G], total2 = s_tt2[G];
+  const int total = total1 + total2;
+  if (static_cast<int>(blockIdx.x) >= total) return;
+
+  if (warp == 1) {
+    tmem_alloc(smem_u32(const_cast<uint32_t*>(s_tmem)), C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *s_tmem;
+  // work item t -> (down?, tile)
+  auto item = [&](int t, bool& dn) -> WsTile {
+    dn = t >= total1;
+    return dn ? ws_tile<BN>(t - total1, total2, s_tt2, s_off, G, nwb2) : ws_tile<BN>(t, total1, s_tt1, s_off, G, nwb1);
+  };
+
+  if (warp == 0) {
+    // ------------------------------------------------ TMA producer (lane 0)
+    if (lane == 0) {
+      tma_prefetch_desc(&tma_w1);
+      tma_prefetch_desc(&tma_x1);
+      tma_prefetch_desc(&tma_w2);
+      tma_prefetch_desc(&tma_x2);
+    }
+    int stage = 0;
+    uint32_t ph = 0;
+    bool ok = true;
+    uint32_t armed = 0, armed_ph = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+      bool dn;
+      const WsTile T = item(t, dn);
+      if (lane == 0) {
+        const CUtensorMap* tw = dn ? &tma_w2 : &tma_w1;
+        const CUtensorMap* tx = dn ? &tma_x2 : &tma_x1;
+        const int wrow0 = T.g * (dn ? g.wrows2 : g.wrows1) + T.wb * WS_BM;
+        const int KB = (dn ? g.kdim2 : g.kdim1) / WS_BK;
+        const int nload = (T.ntok + WS_BOX - 1) / WS_BOX;
+        const uint32_t bytes = C::A_BYTES + nload * C::BOX_BYTES;
+        int pre = 0;  // k-blocks whose weights go out before the dependency is met
+        if (dn) {
+          pre = KB < STAGES ? KB : STAGES;
+          const int st0 = stage;
+          for (int kb = 0; kb < pre; ++kb) {
+            if (!mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(FULL_BAR(stage), bytes);
+            tma_load_2d(sA + stage * C::A_BYTES, tw, FULL_BAR(stage), kb * WS_BK, wrow0);
+            armed |= 1u << stage;
+            armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
+            if (++stage == STAGES) {
+              stage = 0;
+              ph ^= 1u;
+            }
+          }
+          if (ok) {
+            // every gate/up item of expert T.g has stored its h slice
+            const int n = s_off[T.g + 1] - s_off[T.g];
+            const int need = ((n + BN - 1) / BN) * nwb1;
+            const volatile int32_t* rp = g.ready + T.g;
+            const uint64_t t0 = globaltimer_ns();
+            while (*rp < need) {
+              if (*s_abort || globaltimer_ns() - t0 > g.limit_ns) {
+                ok = false;
+                break;
+              }
+            }
+            __threadfence();
+            fence_proxy_async_all();  // the h rows, written by generic stores, read through the tensor map
+          }
+          if (ok) {
+            int st = st0;
+            for (int kb = 0; kb < pre; ++kb) {
+              const uint32_t dB = sB + st * C::B_BYTES;
+              for (int i = 0; i < nload; ++i)
+                tma_load_2d(dB + i * C::BOX_BYTES, tx, FULL_BAR(st), kb * WS_BK, T.row0 + i * WS_BOX);
+              if (++st == STAGES) st = 0;
+            }
+          }
+        }
+        for (int kb = pre; ok && kb < KB; ++kb) {
+          if (!mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(FULL_BAR(stage), bytes);
+          tma_load_2d(sA + stage * C::A_BYTES, tw, FULL_BAR(stage), kb * WS_BK, wrow0);
+          const uint32_t dB = sB + stage * C::B_BYTES;
+          for (int i = 0; i < nload; ++i)
+            tma_load_2d(dB + i * C::BOX_BYTES, tx, FULL_BAR(stage), kb * WS_BK, T.row0 + i * WS_BOX);
+          armed |= 1u << stage;
+          armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            ph ^= 1u;
+          }
+        }
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+    }
+    if (lane == 0 && !ok) {
+      *s_abort = 1;
+      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+      // let the copies this thread started land before the CTA can exit (a
+      // stage whose activation rows were never requested runs to the limit)
+      int no_abort = 0;
+      for (int s = 0; s < STAGES; ++s)
+        if ((armed >> s) & 1u) mbar_wait(FULL_BAR(s), (armed_ph >> s) & 1u, g.limit_ns, &no_abort);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ------------------------------------------------ MMA issuer
+    int stage = 0;
+    uint32_t ph = 0;
+    bool ok = true, issued = false;
+    int it = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
+      bool dn;
+      const WsTile T = item(t, dn);
+      const int KB = (dn ? g.kdim2 : g.kdim1) / WS_BK;
+      const uint32_t idesc = idesc_bf16_f32(WS_BM, (T.ntok + 15) & ~15);
+      const int acc = it & 1;
+      const uint32_t aph = (it >> 1) & 1;
+      if (!mbar_wait(TEMPTY_BAR(acc), aph ^ 1u, g.limit_ns, s_abort)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t dt = tmem_base + static_cast<uint32_t>(acc * BN);
+      for (int kb = 0; kb < KB; ++kb) {
+        if (!mbar_wait(FULL_BAR(stage), ph, g.limit_ns, s_abort)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint64_t ad = smem_desc_kmajor<WS_BK>(sA + stage * C::A_BYTES);
+        const uint64_t bd = smem_desc_kmajor<WS_BK>(sB + stage * C::B_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < WS_BK / 16; ++kk)
+          tc_mma_f16(dt, ad + 2u * kk, bd + 2u * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+        tc_commit(EMPTY_BAR(stage));
+        issued = true;
+        if (++stage == STAGES) {
+          stage = 0;
+          ph ^= 1u;
+        }
+      }
+      if (!ok) break;
+      tc_commit(TFULL_BAR(acc));
+    }
+    if (!ok) {
+      *s_abort = 1;
+      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+      if (issued) {
+        int no_abort = 0;
+        tc_commit(DRAIN_BAR);
+        mbar_wait(DRAIN_BAR, 0, g.limit_ns, &no_abort);
+      }
+    }
+  } else if (warp >= 2) {
+    // ------------------------------------------------ epilogue (4 warps)
+    const int q = warp & 3;  // TMEM lanes [32q, 32q + 32)
+    int it = 0;
+    int xpar = 0;
+    bool ok = true;
+    const int et = threadIdx.x - 64;  // 0..127 among the epilogue warps
+    for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
+      bool dn;
+      const WsTile T = item(t, dn);
+      const int acc = it & 1;
+      const uint32_t aph = (it >> 1) & 1;
+      if (!mbar_wait(TFULL_BAR(acc), aph, g.limit_ns, s_abort)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t tb = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
+      // as k_moe_ws: 32-token chunks through a bf16 tile in shared memory;
+      // gate/up items write silu(gate) * up to h (64 features per item),
+      // down items write y (128 features per item)
+      const int OC = dn ? WS_BM : WS_BM / 2;
+      __nv_bfloat16* out = static_cast<__nv_bfloat16*>(dn ? g.y : g.h);
+      const int64_t ld = dn ? g.y_ld : g.h_ld;
+      const int fbase = T.wb * OC;
+#pragma unroll 1
+      for (int c0 = 0; c0 < T.ntok; c0 += 32) {
+        uint32_t r[32];
+        tmem_ld32(tb + c0, r);
+        tc_wait_ld();
+        __nv_bfloat16* st = stile + xpar * (32 * WS_BM);
+        if (!dn) {
+          const bool is_gate = q < 2;
+          const int pr = q & 1;
+          float* xb = xch + (xpar * 2 + pr) * 1024;  // [32 columns][32 lanes]
+          if (!is_gate) {
+#pragma unroll
+            for (int c = 0; c < 32; ++c) xb[c * 32 + lane] = __uint_as_float(r[c]);
+          }
+          named_bar_sync(1, 128);
+          if (is_gate) {
+#pragma unroll
+            for (int c = 0; c < 32; ++c)
+              st[c * OC + pr * 32 + lane] = __float2bfloat16_rn(silu_f(__uint_as_float(r[c])) * xb[c * 32 + lane]);
+          }
+        } else {
+#pragma unroll
+          for (int c = 0; c < 32; ++c) st[c * OC + q * 32 + lane] = __float2bfloat16_rn(__uint_as_float(r[c]));
+        }
+        named_bar_sync(1, 128);
+        const int nc = min(32, T.ntok - c0);
+        const int VPR = OC / 8;  // 16-byte vectors per token row
+        for (int v = et; v < 32 * VPR; v += 128) {
+          const int row = v / VPR, cv = v - row * VPR;
+          if (row < nc) {
+            const uint4 val = *reinterpret_cast<const uint4*>(st + row * OC + cv * 8);
+            *reinterpret_cast<uint4*>(out + static_cast<int64_t>(T.row0 + c0 + row) * ld + fbase + cv * 8) = val;
+          }
+        }
+        xpar ^= 1;
+      }
+      tc_fence_before();
+      mbar_arrive(TEMPTY_BAR(acc));
+      if (!dn) {
+        // this item's h slice is stored: publish it to the down items of T.g
+        fence_proxy_async_all();
+        named_bar_sync(1, 128);
+        if (et == 0) {
+          __threadfence();
+          atomicAdd(g.ready + T.g, 1);
+        }
+      }
+    }
+    if (!ok) {
+      *s_abort = 1;
+      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+    }
+  }
+  pdl_trigger();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+#undef FULL_BAR
+#undef EMPTY_BAR
+#undef TFULL_BAR
+#undef TEMPTY_BAR
+#undef DRAIN_BAR
+}
+
+template <int STAGES, int BN>
+static int launch_ffn_ws_bn(const void* x_perm, int rows, int d, int m, const void* w_gu, const void* w_down,
+                            const int32_t* offsets, int G, void* h, void* y, int32_t* ready, int32_t* status,
+                            cudaStream_t s) {
+  using C = WsFfnCfg<STAGES, BN>;
+  CUtensorMap tw1, tx1, tw2, tx2;
+  DM_RET(make_tmap_bf16(&tw1, w_gu, static_cast<uint64_t>(d), static_cast<uint64_t>(G) * 2 * m, WS_BM, WS_BK));
+  DM_RET(make_tmap_bf16(&tx1, x_perm, static_cast<uint64_t>(d), static_cast<uint64_t>(rows), WS_BOX, WS_BK));
+  DM_RET(make_tmap_bf16(&tw2, w_down, static_cast<uint64_t>(m), static_cast<uint64_t>(G) * d, WS_BM, WS_BK));
+  DM_RET(make_tmap_bf16(&tx2, h, static_cast<uint64_t>(m), static_cast<uint64_t>(rows), WS_BOX, WS_BK));
+  WsFfnArgs g;
+  g.offsets = offsets;
+  g.G = G;
+  g.rows = rows;
+  g.wrows1 = 2 * m;
+  g.kdim1 = d;
+  g.wrows2 = d;
+  g.kdim2 = m;
+  g.h = h;
+  g.h_ld = m;
+  g.y = y;
+  g.y_ld = d;
+  g.ready = ready;
+  g.status = status;
+  g.limit_ns = static_cast<uint64_t>(wait_limit_ns());
+  auto kern = k_ffn_ws<STAGES, BN>;
+  static_assert(C::SMEM <= 232448, "shared memory budget");
+  static_assert(C::SMEM > 232448 / 2, "one CTA per SM: the dependency waits need every CTA resident");
+  DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(C::SMEM)));
+  const int64_t ub = (static_cast<int64_t>(rows) / BN + G) * ((2 * m + d) / WS_BM);
+  const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(sm_count(), ub)));
+  DM_CUDA_CHECK(launch_pdl(kern, dim3(grid), dim3(192), C::SMEM, s, tw1, tx1, tw2, tx2, g));
+  return DECOMOE_OK;
+}
+
+// Token chunk by row count, as launch_ws_auto.
+static int launch_ffn_ws(const void* x_perm, int rows, int d, int m, const void* w_gu, const void* w_down,
+                         const int32_t* offsets, int G, void* h, void* y, int32_t* ready, int32_t* status,
+                         cudaStream_t s) {
+  if (rows <= 256)
+    return launch_ffn_ws_bn<ffn_ws_max_stages<32>(), 32>(x_perm, rows, d, m, w_gu, w_down, offsets, G, h, y, ready,
+                                                         status, s);
+  if (rows <= 512)
+    return launch_ffn_ws_bn<ffn_ws_max_stages<64>(), 64>(x_perm, rows, d, m, w_gu, w_down, offsets, G, h, y, ready,
+                                                         status, s);
+  if (rows <= 1024)
+    return launch_ffn_ws_bn<ffn_ws_max_stages<128>(), 128>(x_perm, rows, d, m, w_gu, w_down, offsets, G, h, y,
+                                                           ready, status, s);
+  return launch_ffn_ws_bn<ffn_ws_max_stages<256>(), 256>(x_perm, rows, d, m, w_gu, w_down, offsets, G, h, y, ready,
+                                                         status, s);
+}
+
 // X: [rows, kdim] token rows grouped by expert, or with GATHER_B the source
 // tensor [x_tensor_rows, kdim] whose row b_rows[r] is token row r;
 // W: [G * wrows, kdim].
@@ -1576,3 +2018,35 @@ int decomoe_expert_swiglu_ref(const void* x_perm, const int32_t* offsets, int64_
 }
 
 }  // extern "C"
+
+namespace decomoe {
+
+// Rows from which the fused launch is taken (with fewer, the gate/up tiles
+// leave SMs idle and the fused form gains nothing).
+#ifndef DECOMOE_FFN_FUSED_MIN_ROWS
+#define DECOMOE_FFN_FUSED_MIN_ROWS 16
+#endif
+// Both expert GEMMs of a decode-size invocation in one launch (k_ffn_ws)
+// when the weights-stationary kernel is the choice (bf16, rows <= 8 per
+// expert on average), else nothing launched and false returned.
+int launch_expert_ffn_fused(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m, int dtype,
+                            const void* w_gate_up, const void* w_down, void* h, void* y_perm, int32_t* ready,
+                            int32_t* status, cudaStream_t s, bool* launched) {
+  *launched = false;
+  static const int64_t min_rows = [] {
+    const char* e = getenv("DECOMOE_FFN_FUSED_MIN_ROWS");
+    return e != nullptr ? static_cast<int64_t>(atoll(e)) : static_cast<int64_t>(DECOMOE_FFN_FUSED_MIN_ROWS);
+  }();
+  if (dtype != DECOMOE_BF16 || rows < min_rows || rows <= 0 ||
+      rows > static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K)
+    return DECOMOE_OK;
+  DM_RET(expert_check("expert_gate_up", x_perm, offsets, rows, K, d, m, dtype, w_gate_up, h));
+  DM_RET(expert_check("expert_down", h, offsets, rows, K, d, m, dtype, w_down, y_perm));
+  DM_ARG_CHECK(ready != nullptr, "expert ffn: null ready counters");
+  DM_RET(launch_ffn_ws(x_perm, static_cast<int>(rows), d, m, w_gate_up, w_down, offsets, K, h, y_perm, ready, status,
+                       s));
+  *launched = true;
+  return DECOMOE_OK;
+}
+
+}  // namespace decomoe

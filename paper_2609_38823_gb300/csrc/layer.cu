@@ -24,6 +24,7 @@ enum {
   WS_KDEV,
   WS_SCHED,
   WS_RSPLIT,
+  WS_SYNC,
   WS_STATUS_PAD,
   WS_COUNT
 };
@@ -36,7 +37,7 @@ static int route_dispatch_src(const float* logits, const RouteSrc& src, int64_t 
                               int32_t* topk_idx, float* topk_w, double* mass_out, int32_t* K_dev, const void* x,
                               int d, int dtype, int32_t* counts, int32_t* offsets, int32_t* perm_token,
                               int32_t* inv_slot, void* x_perm, void* ws, size_t ws_bytes, int32_t* status_dev,
-                              cudaStream_t s) {
+                              cudaStream_t s, int32_t* zero_ints = nullptr, int n_zero = 0) {
   DM_ARG_CHECK(T >= 0, "route_dispatch: T < 0");
   DM_ARG_CHECK(E >= 1 && E <= DECOMOE_MAX_E && k >= 1 && k <= DECOMOE_MAX_TOPK && k <= E,
                "route_dispatch: need 1 <= k <= E <= %d, k <= %d", DECOMOE_MAX_E, DECOMOE_MAX_TOPK);
@@ -95,7 +96,7 @@ static int route_dispatch_src(const float* logits, const RouteSrc& src, int64_t 
     // mass pass, Eq. 12 on the device, routing over [0, *K_dev) (from the
     // summed logits when the first pass read the router's partials)
     DM_RET(route_prefix_src(logits, src, T, E, E, E, k, nullptr, nullptr, mass_out, route_ws, rbytes, false, nullptr,
-                            s));
+                            s, nullptr, nullptr, zero_ints, n_zero));
     DM_RET(decomoe_select_prefix_device(mass_out, E, k, p, K_dev, stream));
     DM_RET(route_prefix_src(src.logits_out != nullptr ? src.logits_out : logits, RouteSrc{}, T, E, E, E, k, topk_idx,
                             topk_w, nullptr, nullptr, 0, false, nullptr, s, K_dev, one_block ? &rd : nullptr));
@@ -103,7 +104,7 @@ static int route_dispatch_src(const float* logits, const RouteSrc& src, int64_t 
     // one launch: prefix routing and, with mass_out, the full-pool partial
     // masses (finished by the dispatch launch)
     DM_RET(route_prefix_src(logits, src, T, E, E, K, k, topk_idx, topk_w, mass_out, route_ws, rbytes, true,
-                            &mass_blocks, s, nullptr, one_block ? &rd : nullptr));
+                            &mass_blocks, s, nullptr, one_block ? &rd : nullptr, zero_ints, n_zero));
   }
   if (one_block) {
     // one routing block: the mass was written in place and the picks are dispatched
@@ -124,7 +125,7 @@ static int router_route_dispatch_impl(const void* x, const void* w_r, const floa
                                       float* topk_w, double* mass_out, int32_t* K_dev, int32_t* counts,
                                       int32_t* offsets, int32_t* perm_token, int32_t* inv_slot, void* x_perm,
                                       float* scratch, void* rd_ws, size_t rd_bytes, int32_t* status_dev,
-                                      cudaStream_t s) {
+                                      cudaStream_t s, int32_t* zero_ints = nullptr, int n_zero = 0) {
   DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "router_route_dispatch: bad dtype");
   RouteSrc src;
   const float* lg = logits;
@@ -149,7 +150,7 @@ static int router_route_dispatch_impl(const void* x, const void* w_r, const floa
     }
   }
   return route_dispatch_src(lg, src, T, E, K, k, p, topk_idx, topk_w, mass_out, K_dev, x, d, dtype, counts, offsets,
-                            perm_token, inv_slot, x_perm, rd_ws, rd_bytes, status_dev, s);
+                            perm_token, inv_slot, x_perm, rd_ws, rd_bytes, status_dev, s, zero_ints, n_zero);
 }
 
 struct LayerLayout {
@@ -177,6 +178,7 @@ static LayerLayout layer_layout(int64_t T, int d, int E, int k, int m, int dtype
   sz[WS_KDEV] = 16;
   sz[WS_SCHED] = 16;
   sz[WS_RSPLIT] = decomoe_router_logits_ws_bytes(T, d, E);
+  sz[WS_SYNC] = static_cast<size_t>(E) * 4;  // per-expert counters of the fused decode expert launch
   sz[WS_STATUS_PAD] = 256;
   size_t o = 0;
   for (int i = 0; i < WS_COUNT; ++i) {
@@ -318,6 +320,9 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
   int K = K_fixed;
   int32_t* K_dev = reinterpret_cast<int32_t*>(base + L.off[WS_KDEV]);
   float* rsplit = reinterpret_cast<float*>(base + L.off[WS_RSPLIT]);
+  // per-expert counters of the fused decode expert launch, cleared by the
+  // first routing launch of this call
+  int32_t* sync = reinterpret_cast<int32_t*>(base + L.off[WS_SYNC]);
   if (K_fixed != 0) {
     // a1-a5: router logits over all E reordered experts, full-pool mass
     // (Eq. 11), prefix (fixed, or Eq. 12 on the device), prefix routing and
@@ -325,7 +330,8 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
     // over all E groups (those at or beyond *K_dev are empty)
     DM_RET(router_route_dispatch_impl(x, w_r, bias, T, d, E, dtype, K_fixed, k, p, logits, topk_idx, topk_w,
                                       (K_fixed == -1 || p > 0.0) ? mass : nullptr, K_dev, counts, offsets, perm, inv,
-                                      x_perm, rsplit, route_ws, L.off[WS_KDEV] - L.off[WS_ROUTE], status_dev, s));
+                                      x_perm, rsplit, route_ws, L.off[WS_KDEV] - L.off[WS_ROUTE], status_dev, s, sync,
+                                      E));
     if (K_fixed == -1) {
       K = E;
       if (K_sel_host) *K_sel_host = -1;
@@ -336,8 +342,8 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
     // read, Eq. 12 in C
     DM_RET(decomoe_router_logits_ws(x, w_r, bias, T, d, E, dtype, logits, rsplit,
                                     decomoe_router_logits_ws_bytes(T, d, E), status_dev, stream));
-    DM_RET(decomoe_route_prefix(logits, T, E, E, E, k, nullptr, nullptr, mass, route_ws,
-                                decomoe_route_workspace_bytes(T, E), stream));
+    DM_RET(route_prefix_src(logits, RouteSrc{}, T, E, E, E, k, nullptr, nullptr, mass, route_ws,
+                            decomoe_route_workspace_bytes(T, E), false, nullptr, s, nullptr, nullptr, sync, E));
     static thread_local std::vector<double> h_mass;
     h_mass.resize(E);
     DM_CUDA_CHECK(cudaMemcpyAsync(h_mass.data(), mass, sizeof(double) * E, cudaMemcpyDeviceToHost, s));
@@ -351,11 +357,16 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
                                   status_dev, stream));
   }
   if (K_used_host && K_fixed != -1) *K_used_host = K;
-  // a6: grouped SwiGLU experts over [0, K)
-  // static tile order (as fast as the dynamic queue here, and no counter
-  // reset between the launches, which keeps them chained programmatically)
-  DM_RET(decomoe_expert_swiglu(x_perm, offsets, T * k, K, d, m, dtype, w_gate_up, w_down, h, y_perm,
-                               status_dev, nullptr, stream));
+  // a6: grouped SwiGLU experts over [0, K): at decode sizes gate/up and down
+  // in one launch, else the two GEMMs (static tile order: as fast as the
+  // dynamic queue here, and no counter reset between the launches, which
+  // keeps them chained programmatically)
+  bool fused = false;
+  DM_RET(launch_expert_ffn_fused(x_perm, offsets, T * k, K, d, m, dtype, w_gate_up, w_down, h, y_perm, sync,
+                                 status_dev, s, &fused));
+  if (!fused)
+    DM_RET(decomoe_expert_swiglu(x_perm, offsets, T * k, K, d, m, dtype, w_gate_up, w_down, h, y_perm, status_dev,
+                                 nullptr, stream));
   // a7: combine (+ residual); with text_out also a8 on the layer output
   return combine_impl(y_perm, inv, topk_w, T, k, d, dtype, residual, out, text_out, v0, nv, stream);
 }

@@ -189,8 +189,12 @@ template <int NP>
 __global__ void __launch_bounds__(ROUTE_THREADS)
     k_route(const float* __restrict__ logits, int64_t Tn, int E, int64_t ld, int K, int k,
             int32_t* __restrict__ idx_out, float* __restrict__ w_out, double* __restrict__ part,
-            const int32_t* __restrict__ K_dev, int64_t skip_at, int64_t skip_len, RouteSrc src, RouteDispatch rd) {
+            const int32_t* __restrict__ K_dev, int64_t skip_at, int64_t skip_len, RouteSrc src, RouteDispatch rd,
+            int32_t* __restrict__ zero_ints, int n_zero) {
   pdl_enter();
+  // block 0 clears a small int array for a later launch of the caller's chain
+  if (zero_ints != nullptr && blockIdx.x == 0)
+    for (int i = threadIdx.x; i < n_zero; i += ROUTE_THREADS) zero_ints[i] = 0;
   if (K_dev != nullptr) K = *K_dev;  // prefix chosen on the device (k <= K <= E by construction)
   __shared__ int s_idx[ROUTE_TPB][DECOMOE_MAX_TOPK];
   __shared__ float s_w[ROUTE_TPB][DECOMOE_MAX_TOPK];
@@ -334,7 +338,7 @@ int launch_skip_mass(const float* logits, int64_t n, int E, int64_t ld, int k, i
   const int64_t nblocks = (n + ROUTE_TPB - 1) / ROUTE_TPB;
   k_route<1><<<static_cast<unsigned>(nblocks), ROUTE_THREADS, 0, s>>>(logits, n, E, ld, E, k, nullptr, nullptr, part,
                                                                       nullptr, skip_at, skip_len, RouteSrc{},
-                                                                      RouteDispatch{});
+                                                                      RouteDispatch{}, nullptr, 0);
   DM_LAUNCH_CHECK("k_route");
   k_mass_finalize<<<E, 256, 0, s>>>(part, static_cast<int>(nblocks), E, mass);
   DM_LAUNCH_CHECK("k_mass_finalize");
@@ -425,7 +429,7 @@ namespace decomoe {
 int route_prefix_src(const float* logits, const RouteSrc& src, int64_t T, int E, int64_t ld, int K, int k,
                      int32_t* topk_idx, float* topk_w, double* mass_out, void* ws, size_t ws_bytes,
                      bool defer_finalize, int* mass_blocks, cudaStream_t s, const int32_t* K_dev,
-                     const RouteDispatch* rd) {
+                     const RouteDispatch* rd, int32_t* zero_ints, int n_zero) {
   if (mass_blocks != nullptr) *mass_blocks = 0;
   DM_ARG_CHECK(T >= 0, "route_prefix: T < 0");
   DM_ARG_CHECK(E >= 1 && E <= DECOMOE_MAX_E, "route_prefix: E=%d outside [1, %d]", E, DECOMOE_MAX_E);
@@ -463,7 +467,8 @@ int route_prefix_src(const float* logits, const RouteSrc& src, int64_t T, int E,
   }
   auto kern = src.nparts == 16 ? k_route<16> : src.nparts == 4 ? k_route<4> : k_route<1>;
   DM_CUDA_CHECK(launch_pdl(kern, dim3(static_cast<unsigned>(nblocks)), dim3(ROUTE_THREADS), 0, s, logits, T, E, ld,
-                           K, k, topk_idx, topk_w, part, K_dev, INT64_MAX, static_cast<int64_t>(0), src, rdv));
+                           K, k, topk_idx, topk_w, part, K_dev, INT64_MAX, static_cast<int64_t>(0), src, rdv,
+                           zero_ints, n_zero));
   if (mass_out != nullptr && nblocks > 1) {
     if (defer_finalize && mass_blocks != nullptr) {
       *mass_blocks = static_cast<int>(nblocks);  // the caller's next kernel adds the partials up
