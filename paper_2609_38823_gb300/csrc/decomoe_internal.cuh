@@ -162,9 +162,10 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
                    int64_t T, int d, int E, int k, int m, int dtype, int K_fixed, double p, const void* residual,
                    void* out, void* text_out, int64_t v0, int64_t nv, int* K_used_host, int* K_sel_host, void* ws,
                    size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream);
-// Both expert GEMMs of a decode-size invocation (bf16, at most 8 rows per
-// expert on average) in one launch; ready: K int32, zero at launch. Sets
-// *launched = false (and launches nothing) at other sizes.
+// Both expert GEMMs in one launch (bf16): ready holds
+// expert_ffn_sync_ints(rows, K) int32, zero at launch. Sets *launched = false
+// (and launches nothing) where the two-launch form is kept.
+size_t expert_ffn_sync_ints(int64_t rows, int E);
 int launch_expert_ffn_fused(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m, int dtype,
                             const void* w_gate_up, const void* w_down, void* h, void* y_perm, int32_t* ready,
                             int32_t* status, cudaStream_t s, bool* launched);

@@ -1567,6 +1567,389 @@ static int launch_ffn_ws(const void* x_perm, int rows, int d, int m, const void*
                                                          status, s);
 }
 
+// ------------------------------------------------------------------ fused prefill FFN
+// Gate/up and down of the tokens-as-M path in one persistent launch, with
+// k_gemm_tc's tiles (128 rows x 256, 4-stage ring, two TMEM accumulators,
+// 8 epilogue warps). Work items: every gate/up tile (tile_coords order),
+// then every down tile (same order); static round robin. A down tile of
+// M-tile j reads the h rows that the 2m/256 gate/up tiles of j store: those
+// bump ready[j] after their stores (release); the down tile issues its
+// weight k-blocks first, polls ready[j] (acquire, bounded), then requests the
+// h rows. The early CTAs of the down phase start while the last gate/up
+// tiles still run, instead of after a launch boundary. Deadlock-free as
+// k_ffn_ws (gate/up items never wait; one CTA per SM, grid <= SMs). ready[]
+// (one int per M-tile) is zero at launch.
+struct TcFfnArgs {
+  const int32_t* offsets;  // [G + 1]
+  int G;
+  int rows;
+  int d, m;
+  void* h;  // [rows, m] bf16
+  void* y;  // [rows, d] bf16
+  int32_t* ready;
+  int32_t* status;
+  uint64_t limit_ns;
+};
+
+constexpr int FFN_BN = 256, FFN_BK = 64, FFN_STAGES = 4, FFN_EW = 8;
+using FfnCfg = TcCfg<FFN_BN, FFN_STAGES, FFN_BK, 1, 1>;
+
+__global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
+    k_ffn_tc(const __grid_constant__ CUtensorMap tma_a1, const __grid_constant__ CUtensorMap tma_b1,
+             const __grid_constant__ CUtensorMap tma_a2, const __grid_constant__ CUtensorMap tma_b2,
+             const TcFfnArgs g) {
+  using C = FfnCfg;
+  constexpr int BN = FFN_BN, STAGES = FFN_STAGES, EW = FFN_EW;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
+  uint8_t* smem = smem_raw + pad;
+  const uint32_t sA = raw + pad;
+  const uint32_t sB = sA + STAGES * C::A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
+  int* s_off = reinterpret_cast<int*>(bars + C::NBARS);
+  int* s_mt = s_off + (C::MAXG + 1);
+  volatile uint32_t* s_tmem = reinterpret_cast<volatile uint32_t*>(s_mt + (C::MAXG + 1));
+  volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t bar0 = smem_u32(bars);
+#define FULL_BAR(s) (bar0 + 8u * (s))
+#define EMPTY_BAR(s) (bar0 + 8u * (STAGES + (s)))
+#define TFULL_BAR(a) (bar0 + 8u * (2 * STAGES + (a)))
+#define TEMPTY_BAR(a) (bar0 + 8u * (2 * STAGES + 2 + (a)))
+#define DRAIN_BAR (bar0 + 8u * (2 * STAGES + 4))
+
+  const int G = g.G;
+  if (threadIdx.x == 0) {
+    *s_abort = 0;
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(FULL_BAR(s), 1);
+      mbar_init(EMPTY_BAR(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(TFULL_BAR(a), 1);
+      mbar_init(TEMPTY_BAR(a), 32 * EW);
+    }
+    mbar_init(DRAIN_BAR, 1);
+    fence_mbar_init();
+  }
+  pdl_wait();
+  for (int i = threadIdx.x; i <= G; i += blockDim.x) s_off[i] = g.offsets[i];
+  __syncthreads();
+  if (warp == 2) {
+    // exclusive scan of M-tiles per group: s_mt[e] = first M-tile of e
+    const int per = (G + 31) / 32;  // <= 8
+    int loc[8];
+    int sum = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      loc[i] = 0;
+      const int gi = lane * per + i;
+      if (i < per && gi < G) {
+        const int n = s_off[gi + 1] - s_off[gi];
+        loc[i] = n > 0 ? (n + C::BM - 1) / C::BM : 0;
+      }
+      sum += loc[i];
+    }
+    int incl = sum;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += v;
+    }
+    int run = incl - sum;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int gi = lane * per + i;
+      if (i < per && gi < G) s_mt[gi] = run;
+      run += loc[i];
+    }
+    if (lane == 31) s_mt[G] = incl;
+  }
+  __syncthreads();
+  const int NT1 = 2 * g.m / BN, NT2 = g.d / BN;
+  const int total1 = s_mt[G] * NT1, total2 = s_mt[G] * NT2;
+  const int total = total1 + total2;
+  if (static_cast<int>(blockIdx.x) >= total) return;  // before any TMEM or TMA use
+
+  if (warp == 1) {
+    tmem_alloc(smem_u32(const_cast<uint32_t*>(s_tmem)), C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *s_tmem;
+  // work item t -> (down?, group, M-tile of the group, N-tile, M-tile index)
+  struct Item {
+    bool dn;
+    int grp, mt, nb, mtg;
+  };
+  auto item = [&](int t) -> Item {
+    Item r;
+    r.dn = t >= total1;
+    const int tl = r.dn ? t - total1 : t;
+    tile_coords(tl, r.dn ? NT2 : NT1, s_mt, G, r.grp, r.mt, r.nb);
+    r.mtg = s_mt[r.grp] + r.mt;
+    return r;
+  };
+
+  if (warp == 0) {
+    // ------------------------------------------------ TMA producer (lane 0)
+    if (lane == 0) {
+      tma_prefetch_desc(&tma_a1);
+      tma_prefetch_desc(&tma_b1);
+      tma_prefetch_desc(&tma_a2);
+      tma_prefetch_desc(&tma_b2);
+    }
+    int stage = 0;
+    uint32_t ph = 0;
+    bool ok = true;
+    uint32_t armed = 0, armed_ph = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+      const Item it = item(t);
+      if (lane == 0) {
+        const CUtensorMap* ta = it.dn ? &tma_a2 : &tma_a1;
+        const CUtensorMap* tb = it.dn ? &tma_b2 : &tma_b1;
+        const int row0 = s_off[it.grp] + it.mt * C::BM;
+        const int brow = it.grp * (it.dn ? g.d : 2 * g.m) + it.nb * BN;
+        const int KB = (it.dn ? g.m : g.d) / FFN_BK;
+        int pre = 0;  // k-blocks whose weights go out before the dependency is met
+        if (it.dn) {
+          pre = KB < STAGES ? KB : STAGES;
+          const int st0 = stage;
+          for (int kb = 0; kb < pre; ++kb) {
+            if (!mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(FULL_BAR(stage), C::A_BYTES + C::B_BYTES);
+            tma_load_2d(sB + stage * C::B_BYTES, tb, FULL_BAR(stage), kb * FFN_BK, brow);
+            armed |= 1u << stage;
+            armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
+            if (++stage == STAGES) {
+              stage = 0;
+              ph ^= 1u;
+            }
+          }
+          if (ok) {
+            // every gate/up tile of this M-tile has stored its h columns
+            const volatile int32_t* rp = g.ready + it.mtg;
+            const uint64_t t0 = globaltimer_ns();
+            while (*rp < NT1) {
+              if (*s_abort || globaltimer_ns() - t0 > g.limit_ns) {
+                ok = false;
+                break;
+              }
+            }
+            __threadfence();
+            fence_proxy_async_all();  // h, written by generic stores, read through the tensor map
+          }
+          if (ok) {
+            int st = st0;
+            for (int kb = 0; kb < pre; ++kb) {
+              tma_load_2d(sA + st * C::A_BYTES, ta, FULL_BAR(st), kb * FFN_BK, row0);
+              if (++st == STAGES) st = 0;
+            }
+          }
+        }
+        for (int kb = pre; ok && kb < KB; ++kb) {
+          if (!mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(FULL_BAR(stage), C::A_BYTES + C::B_BYTES);
+          tma_load_2d(sA + stage * C::A_BYTES, ta, FULL_BAR(stage), kb * FFN_BK, row0);
+          tma_load_2d(sB + stage * C::B_BYTES, tb, FULL_BAR(stage), kb * FFN_BK, brow);
+          armed |= 1u << stage;
+          armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            ph ^= 1u;
+          }
+        }
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+    }
+    if (lane == 0 && !ok) {
+      *s_abort = 1;
+      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+      int no_abort = 0;
+      for (int s = 0; s < STAGES; ++s)
+        if ((armed >> s) & 1u) mbar_wait(FULL_BAR(s), (armed_ph >> s) & 1u, g.limit_ns, &no_abort);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ------------------------------------------------ MMA issuer
+    constexpr uint32_t IDESC = idesc_bf16_f32(C::BM, BN);
+    int stage = 0;
+    uint32_t ph = 0;
+    bool ok = true, issued = false;
+    int n = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x, ++n) {
+      const bool dn = t >= total1;
+      const int KB = (dn ? g.m : g.d) / FFN_BK;
+      const int acc = n & 1;
+      const uint32_t aph = (n >> 1) & 1;
+      if (!mbar_wait(TEMPTY_BAR(acc), aph ^ 1u, g.limit_ns, s_abort)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t dt = tmem_base + static_cast<uint32_t>(acc * BN);
+      for (int kb = 0; kb < KB; ++kb) {
+        if (!mbar_wait(FULL_BAR(stage), ph, g.limit_ns, s_abort)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint64_t ad = smem_desc_kmajor<FFN_BK>(sA + stage * C::A_BYTES);
+        const uint64_t bd = smem_desc_kmajor<FFN_BK>(sB + stage * C::B_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < FFN_BK / 16; ++kk)
+          tc_mma_f16(dt, ad + 2u * kk, bd + 2u * kk, IDESC, (kb | kk) != 0 ? 1u : 0u);
+        tc_commit(EMPTY_BAR(stage));
+        issued = true;
+        if (++stage == STAGES) {
+          stage = 0;
+          ph ^= 1u;
+        }
+      }
+      if (!ok) break;
+      tc_commit(TFULL_BAR(acc));
+    }
+    if (!ok) {
+      *s_abort = 1;
+      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+      if (issued) {
+        int no_abort = 0;
+        tc_commit(DRAIN_BAR);
+        mbar_wait(DRAIN_BAR, 0, g.limit_ns, &no_abort);
+      }
+    }
+  } else if (warp >= 2) {
+    // ------------------------------------------------ epilogue (k_gemm_tc's)
+    const int q = warp & 3;
+    const int wp = (warp - 2) >> 2;
+    constexpr int WPQ = EW / 4;
+    bool ok = true;
+    int n = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x, ++n) {
+      const Item it = item(t);
+      const int acc = n & 1;
+      const uint32_t aph = (n >> 1) & 1;
+      const int row0 = s_off[it.grp] + it.mt * C::BM;
+      const int row_end = s_off[it.grp + 1];
+      if (!mbar_wait(TFULL_BAR(acc), aph, g.limit_ns, s_abort)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const int grow = row0 + q * 32 + lane;
+      const bool valid = grow < row_end;
+      const uint32_t tb = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
+      if (!it.dn) {
+        constexpr int GU = DECOMOE_GU_BLOCK;
+        __nv_bfloat16* out = static_cast<__nv_bfloat16*>(g.h);
+#pragma unroll 1
+        for (int cc = 32 * wp; cc < BN / 2; cc += 32 * WPQ) {
+          const int half = cc / GU, c = cc % GU;
+          uint32_t gr[32], ur[32];
+          tmem_ld32(tb + half * 2 * GU + c, gr);
+          tmem_ld32(tb + half * 2 * GU + GU + c, ur);
+          tc_wait_ld();
+          uint32_t pk[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const float g0 = __uint_as_float(gr[2 * i]), g1 = __uint_as_float(gr[2 * i + 1]);
+            const float u0 = __uint_as_float(ur[2 * i]), u1 = __uint_as_float(ur[2 * i + 1]);
+            pk[i] = pack_bf16x2(silu_f(g0) * u0, silu_f(g1) * u1);
+          }
+          if (valid) {
+            uint4* dst = reinterpret_cast<uint4*>(out + static_cast<int64_t>(grow) * g.m + it.nb * (BN / 2) + cc);
+#pragma unroll
+            for (int v = 0; v < 4; ++v) dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+          }
+        }
+      } else {
+        __nv_bfloat16* out = static_cast<__nv_bfloat16*>(g.y);
+#pragma unroll 1
+        for (int c = 32 * wp; c < BN; c += 32 * WPQ) {
+          uint32_t r[32];
+          tmem_ld32(tb + c, r);
+          tc_wait_ld();
+          uint32_t pk[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) pk[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
+          if (valid) {
+            uint4* dst = reinterpret_cast<uint4*>(out + static_cast<int64_t>(grow) * g.d + it.nb * BN + c);
+#pragma unroll
+            for (int v = 0; v < 4; ++v) dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(TEMPTY_BAR(acc));
+      if (!it.dn) {
+        // this tile's h columns are stored: publish them to the down tiles
+        fence_proxy_async_all();
+        named_bar_sync(1, 32 * EW);
+        if (warp == 2 && lane == 0) {
+          __threadfence();
+          atomicAdd(g.ready + it.mtg, 1);
+        }
+      }
+    }
+    if (!ok) {
+      *s_abort = 1;
+      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+    }
+  }
+  pdl_trigger();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+#undef FULL_BAR
+#undef EMPTY_BAR
+#undef TFULL_BAR
+#undef TEMPTY_BAR
+#undef DRAIN_BAR
+}
+
+static int launch_ffn_tc(const void* x_perm, int rows, int d, int m, const void* w_gu, const void* w_down,
+                         const int32_t* offsets, int G, void* h, void* y, int32_t* ready, int32_t* status,
+                         cudaStream_t s) {
+  using C = FfnCfg;
+  CUtensorMap ta1, tb1, ta2, tb2;
+  DM_RET(make_tmap_bf16(&ta1, x_perm, static_cast<uint64_t>(d), static_cast<uint64_t>(rows), C::BM, FFN_BK));
+  DM_RET(make_tmap_bf16(&tb1, w_gu, static_cast<uint64_t>(d), static_cast<uint64_t>(G) * 2 * m, FFN_BN, FFN_BK));
+  DM_RET(make_tmap_bf16(&ta2, h, static_cast<uint64_t>(m), static_cast<uint64_t>(rows), C::BM, FFN_BK));
+  DM_RET(make_tmap_bf16(&tb2, w_down, static_cast<uint64_t>(m), static_cast<uint64_t>(G) * d, FFN_BN, FFN_BK));
+  TcFfnArgs g;
+  g.offsets = offsets;
+  g.G = G;
+  g.rows = rows;
+  g.d = d;
+  g.m = m;
+  g.h = h;
+  g.y = y;
+  g.ready = ready;
+  g.status = status;
+  g.limit_ns = static_cast<uint64_t>(wait_limit_ns());
+  static_assert(C::SMEM <= 232448, "shared memory budget");
+  static_assert(C::SMEM > 232448 / 2, "one CTA per SM: the dependency waits need every CTA resident");
+  DM_CUDA_CHECK(cudaFuncSetAttribute(k_ffn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(C::SMEM)));
+  const int64_t ub = (static_cast<int64_t>(rows) / C::BM + G) * static_cast<int64_t>((2 * m + d) / FFN_BN);
+  const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(sm_count(), ub)));
+  DM_CUDA_CHECK(launch_pdl(k_ffn_tc, dim3(grid), dim3(64 + 32 * FFN_EW), C::SMEM, s, ta1, tb1, ta2, tb2, g));
+  return DECOMOE_OK;
+}
+
 // X: [rows, kdim] token rows grouped by expert, or with GATHER_B the source
 // tensor [x_tensor_rows, kdim] whose row b_rows[r] is token row r;
 // W: [G * wrows, kdim].
@@ -2022,13 +2405,21 @@ int decomoe_expert_swiglu_ref(const void* x_perm, const int32_t* offsets, int64_
 namespace decomoe {
 
 // Rows from which the fused launch is taken (with fewer, the gate/up tiles
-// leave SMs idle and the fused form gains nothing).
+// leave SMs idle and the fused form gains nothing), and up to which the
+// tokens-as-M form is fused (measured: 4.6-5.8 us faster per layer at
+// 1024-4096 rows, 3-17 us slower from 8192 rows, where the two launches'
+// waves already fill the SMs and the fused list's dependency stalls cost
+// more than the launch boundary).
 #ifndef DECOMOE_FFN_FUSED_MIN_ROWS
 #define DECOMOE_FFN_FUSED_MIN_ROWS 16
 #endif
-// Both expert GEMMs of a decode-size invocation in one launch (k_ffn_ws)
-// when the weights-stationary kernel is the choice (bf16, rows <= 8 per
-// expert on average), else nothing launched and false returned.
+#ifndef DECOMOE_FFN_FUSED_TC_MAX_ROWS
+#define DECOMOE_FFN_FUSED_TC_MAX_ROWS 4096
+#endif
+// Both expert GEMMs in one launch: k_ffn_ws at decode sizes (bf16, at most 8
+// rows per expert on average), k_ffn_tc above up to
+// DECOMOE_FFN_FUSED_TC_MAX_ROWS rows; nothing launched (and *launched false)
+// for fp32, fewer than DECOMOE_FFN_FUSED_MIN_ROWS rows or more than that.
 int launch_expert_ffn_fused(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m, int dtype,
                             const void* w_gate_up, const void* w_down, void* h, void* y_perm, int32_t* ready,
                             int32_t* status, cudaStream_t s, bool* launched) {
@@ -2037,16 +2428,28 @@ int launch_expert_ffn_fused(const void* x_perm, const int32_t* offsets, int64_t 
     const char* e = getenv("DECOMOE_FFN_FUSED_MIN_ROWS");
     return e != nullptr ? static_cast<int64_t>(atoll(e)) : static_cast<int64_t>(DECOMOE_FFN_FUSED_MIN_ROWS);
   }();
-  if (dtype != DECOMOE_BF16 || rows < min_rows || rows <= 0 ||
-      rows > static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K)
-    return DECOMOE_OK;
+  static const bool tc_fused = [] {
+    const char* e = getenv("DECOMOE_FFN_FUSED_TC");
+    return e == nullptr || e[0] != '0';
+  }();
+  if (dtype != DECOMOE_BF16 || rows < min_rows || rows <= 0) return DECOMOE_OK;
+  const bool ws = rows <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K;
+  if (!ws && (!tc_fused || rows > DECOMOE_FFN_FUSED_TC_MAX_ROWS)) return DECOMOE_OK;
   DM_RET(expert_check("expert_gate_up", x_perm, offsets, rows, K, d, m, dtype, w_gate_up, h));
   DM_RET(expert_check("expert_down", h, offsets, rows, K, d, m, dtype, w_down, y_perm));
   DM_ARG_CHECK(ready != nullptr, "expert ffn: null ready counters");
-  DM_RET(launch_ffn_ws(x_perm, static_cast<int>(rows), d, m, w_gate_up, w_down, offsets, K, h, y_perm, ready, status,
-                       s));
+  if (ws)
+    DM_RET(launch_ffn_ws(x_perm, static_cast<int>(rows), d, m, w_gate_up, w_down, offsets, K, h, y_perm, ready,
+                         status, s));
+  else
+    DM_RET(launch_ffn_tc(x_perm, static_cast<int>(rows), d, m, w_gate_up, w_down, offsets, K, h, y_perm, ready,
+                         status, s));
   *launched = true;
   return DECOMOE_OK;
 }
+
+// int32 counters the fused expert launch needs (zero at launch): one per
+// expert (decode kernel) or per M-tile (prefill kernel).
+size_t expert_ffn_sync_ints(int64_t rows, int E) { return static_cast<size_t>(rows / 128 + E + 1); }
 
 }  // namespace decomoe

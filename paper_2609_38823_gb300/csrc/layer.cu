@@ -178,7 +178,7 @@ static LayerLayout layer_layout(int64_t T, int d, int E, int k, int m, int dtype
   sz[WS_KDEV] = 16;
   sz[WS_SCHED] = 16;
   sz[WS_RSPLIT] = decomoe_router_logits_ws_bytes(T, d, E);
-  sz[WS_SYNC] = static_cast<size_t>(E) * 4;  // per-expert counters of the fused decode expert launch
+  sz[WS_SYNC] = expert_ffn_sync_ints(static_cast<int64_t>(T) * k, E) * 4;  // counters of the fused expert launch
   sz[WS_STATUS_PAD] = 256;
   size_t o = 0;
   for (int i = 0; i < WS_COUNT; ++i) {
@@ -320,9 +320,10 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
   int K = K_fixed;
   int32_t* K_dev = reinterpret_cast<int32_t*>(base + L.off[WS_KDEV]);
   float* rsplit = reinterpret_cast<float*>(base + L.off[WS_RSPLIT]);
-  // per-expert counters of the fused decode expert launch, cleared by the
-  // first routing launch of this call
+  // counters of the fused expert launch (per expert or per M-tile), cleared
+  // by the first routing launch of this call
   int32_t* sync = reinterpret_cast<int32_t*>(base + L.off[WS_SYNC]);
+  const int n_sync = static_cast<int>(expert_ffn_sync_ints(T * k, E));
   if (K_fixed != 0) {
     // a1-a5: router logits over all E reordered experts, full-pool mass
     // (Eq. 11), prefix (fixed, or Eq. 12 on the device), prefix routing and
@@ -331,7 +332,7 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
     DM_RET(router_route_dispatch_impl(x, w_r, bias, T, d, E, dtype, K_fixed, k, p, logits, topk_idx, topk_w,
                                       (K_fixed == -1 || p > 0.0) ? mass : nullptr, K_dev, counts, offsets, perm, inv,
                                       x_perm, rsplit, route_ws, L.off[WS_KDEV] - L.off[WS_ROUTE], status_dev, s, sync,
-                                      E));
+                                      n_sync));
     if (K_fixed == -1) {
       K = E;
       if (K_sel_host) *K_sel_host = -1;
@@ -343,7 +344,7 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
     DM_RET(decomoe_router_logits_ws(x, w_r, bias, T, d, E, dtype, logits, rsplit,
                                     decomoe_router_logits_ws_bytes(T, d, E), status_dev, stream));
     DM_RET(route_prefix_src(logits, RouteSrc{}, T, E, E, E, k, nullptr, nullptr, mass, route_ws,
-                            decomoe_route_workspace_bytes(T, E), false, nullptr, s, nullptr, nullptr, sync, E));
+                            decomoe_route_workspace_bytes(T, E), false, nullptr, s, nullptr, nullptr, sync, n_sync));
     static thread_local std::vector<double> h_mass;
     h_mass.resize(E);
     DM_CUDA_CHECK(cudaMemcpyAsync(h_mass.data(), mass, sizeof(double) * E, cudaMemcpyDeviceToHost, s));

@@ -221,12 +221,15 @@ def test_layer_device_selected_prefix_in_cuda_graph(prefill_layer):
     assert Kdev == dm.decomoe_select_prefix(mass, k, 0.8)
 
 
-@pytest.mark.parametrize("T,K_fixed,p", [(1, 64, 0.7), (8, 64, 0.7), (32, 40, 0.0), (100, 128, 0.7), (256, 96, 0.7),
-                                         (1, -1, 0.7), (8, -1, 0.5), (129, -1, 0.9), (256, -1, 1.0)])
+@pytest.mark.parametrize("T,K_fixed,p", [(1, 64, 0.7), (2, 64, 0.7), (8, 64, 0.7), (32, 40, 0.0), (100, 128, 0.7),
+                                         (256, 96, 0.7), (1, -1, 0.7), (8, -1, 0.5), (129, -1, 0.9), (256, -1, 1.0),
+                                         (2048, 64, 0.7), (2048, -1, 0.7)])
 def test_layer_intermediates_equal_separate_calls(T, K_fixed, p):
-    """The layer's routing, mass, prefix and dispatch intermediates (left in
-    its workspace) equal, bit for bit, the separate C-ABI calls on the same
-    router logits, for fixed and device-selected prefixes."""
+    """The layer's routing, mass, prefix and dispatch intermediates and its
+    expert outputs h and y (left in its workspace) equal, bit for bit, the
+    separate C-ABI calls on the same router logits, for fixed and
+    device-selected prefixes, at decode sizes (one expert launch from 16 rows)
+    and prefill sizes."""
     wl = W.with_(W.PREFILL, T=T)
     E, k, d, m = wl.E, wl.k, wl.d, wl.m
     g = W.make_layer(wl, device="cuda", seed=T)
@@ -275,6 +278,18 @@ def test_layer_intermediates_equal_separate_calls(T, K_fixed, p):
     assert torch.equal(got["xp"].view(torch.int16), xp.view(torch.int16))
     if K_fixed == -1 or p > 0:
         assert torch.equal(mass_l.view(torch.int64), mass.cpu().view(torch.int64))
+    # the layer's expert launch (both GEMMs in one launch where it fuses them)
+    # writes the same h and y as the two separate expert calls
+    h_l = view(9, T * k * m, torch.bfloat16).view(T * k, m)
+    y_l = view(10, T * k * d, torch.bfloat16).view(T * k, d)
+    h2 = torch.empty(T * k, m, dtype=torch.bfloat16, device=DEV)
+    y2 = torch.empty(T * k, d, dtype=torch.bfloat16, device=DEV)
+    dm.decomoe_expert_gate_up(xp, offsets, Kd, w_gu, h2, st)
+    dm.decomoe_expert_down(h2, offsets, Kd, g["w_down"], y2, st)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(st) == 0
+    assert torch.equal(h_l.view(torch.int16), h2.view(torch.int16))
+    assert torch.equal(y_l.view(torch.int16), y2.view(torch.int16))
 
 
 @pytest.mark.parametrize("T,K_fixed,v0,nv", [(2048, 64, 0, 1792), (300, -1, 16, 200), (8, 64, 7, 1), (64, 40, 0, 64)])
