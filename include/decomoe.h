@@ -280,6 +280,22 @@ DECOMOE_API int decomoe_expert_swiglu(const void* x_perm, const int32_t* offsets
                           int m, int dtype, const void* w_gate_up, const void* w_down, void* h_ws,
                           void* y_perm, int32_t* status_dev, int32_t* sched_dev, decomoe_stream_t stream);
 
+/* decomoe_expert_swiglu with both GEMMs in one persistent launch where that
+ * is faster (bf16, 16 to 32768 rows): the down tiles of an expert (decode
+ * sizes) or of a 128-row tile (larger) start as soon as the gate/up tiles
+ * they read have stored h, published through per-expert or per-tile counters
+ * with release/acquire ordering. ready: decomoe_expert_swiglu_ready_ints(rows,
+ * K) int32, all zero at the call (decomoe_moe_layer clears its own); the call
+ * leaves them non-zero. Outside that range the call runs the two launches of
+ * decomoe_expert_swiglu and leaves ready untouched. Outputs are bit-identical
+ * to decomoe_expert_swiglu. Needs every CTA of the launch resident at once
+ * (it sizes the grid to the SMs of the current device). */
+DECOMOE_API size_t decomoe_expert_swiglu_ready_ints(int64_t rows, int K);
+DECOMOE_API int decomoe_expert_swiglu_fused(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d,
+                                            int m, int dtype, const void* w_gate_up, const void* w_down, void* h_ws,
+                                            void* y_perm, int32_t* ready, int32_t* status_dev,
+                                            decomoe_stream_t stream);
+
 /* The two phases of decomoe_expert_swiglu as separate calls (same arguments
  * and rules): gate/up with the fused SwiGLU epilogue writes h [rows, m]; down
  * reads h and writes y_perm [rows, d]. */

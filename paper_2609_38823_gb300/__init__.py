@@ -55,6 +55,8 @@ SIGNATURES = {
     "decomoe_route_dispatch_workspace_bytes": (_S, [_L, _I, _I]),
     "decomoe_route_dispatch": (_I, [_P, _L, _I, _I, _I, _D, _P, _P, _P, _P, _P, _I, _I, _P, _P, _P, _P, _P, _P, _S,
                                     _P, _P]),
+    "decomoe_expert_swiglu_ready_ints": (_S, [_L, _I]),
+    "decomoe_expert_swiglu_fused": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
     "decomoe_router_route_dispatch_workspace_bytes": (_S, [_L, _I, _I, _I]),
     "decomoe_router_route_dispatch": (_I, [_P, _P, _P, _L, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P, _P, _P, _P, _P,
                                            _P, _P, _S, _P, _P]),
@@ -387,6 +389,22 @@ def decomoe_expert_swiglu(x_perm, offsets, K, w_gate_up, w_down, h_ws, y_perm, s
            lib().decomoe_expert_swiglu(_ptr(x_perm), _ptr(offsets), rows, K, d, m, _dt(x_perm),
                                        _ptr(w_gate_up), _ptr(w_down), _ptr(h_ws), _ptr(y_perm),
                                        _ptr(status), _ptr(sched), _stream(stream)))
+
+
+def decomoe_expert_swiglu_ready_ints(rows, K):
+    return int(lib().decomoe_expert_swiglu_ready_ints(rows, K))
+
+
+def decomoe_expert_swiglu_fused(x_perm, offsets, K, w_gate_up, w_down, h, y_perm, ready, status=None, stream=None):
+    """Both expert GEMMs, in one launch where that is faster; ready: int32
+    counters, zero at the call (decomoe_expert_swiglu_ready_ints)."""
+    _need_cuda(x_perm, offsets, w_gate_up, w_down, h, y_perm, ready, status)
+    rows, d = x_perm.shape
+    m = h.shape[1]
+    _check("decomoe_expert_swiglu_fused",
+           lib().decomoe_expert_swiglu_fused(_ptr(x_perm), _ptr(offsets), rows, K, d, m, _dt(x_perm),
+                                             _ptr(w_gate_up), _ptr(w_down), _ptr(h), _ptr(y_perm), _ptr(ready),
+                                             _ptr(status), _stream(stream)))
 
 
 def decomoe_expert_gate_up(x_perm, offsets, K, w_gate_up, h, status=None, sched=None, stream=None):

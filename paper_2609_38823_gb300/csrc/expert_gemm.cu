@@ -1178,6 +1178,11 @@ constexpr int ffn_ws_max_stages() {
 }
 
 __device__ __forceinline__ void fence_proxy_async_all() { asm volatile("fence.proxy.async;" ::: "memory"); }
+__device__ __forceinline__ int ld_acquire_gpu(const int32_t* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
 
 template <int STAGES, int BN>
 __global__ void __launch_bounds__(192, 1)
@@ -1290,9 +1295,21 @@ __global__ void __launch_bounds__(192, 1)
     uint32_t ph = 0;
     bool ok = true;
     uint32_t armed = 0, armed_ph = 0;
+    // readiness of a down item, acquire-loaded one item ahead so that its
+    // latency hides behind the current item's loads (stale values only send
+    // an item down the wait path)
+    auto flag_of = [&](int t) -> int {
+      if (t < total1 || t >= total) return 0;
+      bool d_;
+      const WsTile U = item(t, d_);
+      return ld_acquire_gpu(g.ready + U.g);
+    };
+    int flag_cur = lane == 0 ? flag_of(static_cast<int>(blockIdx.x)) : 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
       bool dn;
       const WsTile T = item(t, dn);
+      const int flag = flag_cur;
+      if (lane == 0) flag_cur = flag_of(t + static_cast<int>(gridDim.x));
       if (lane == 0) {
         const CUtensorMap* tw = dn ? &tma_w2 : &tma_w1;
         const CUtensorMap* tx = dn ? &tma_x2 : &tma_x1;
@@ -1301,7 +1318,11 @@ __global__ void __launch_bounds__(192, 1)
         const int nload = (T.ntok + WS_BOX - 1) / WS_BOX;
         const uint32_t bytes = C::A_BYTES + nload * C::BOX_BYTES;
         int pre = 0;  // k-blocks whose weights go out before the dependency is met
-        if (dn) {
+        const int need = ((s_off[T.g + 1] - s_off[T.g] + BN - 1) / BN) * nwb1;
+        // already met: the ordinary pipeline, weights and h rows together
+        const bool met = dn && flag >= need;
+        if (met) fence_proxy_async_all();  // h, written by generic stores, read through the tensor map
+        if (dn && !met) {
           pre = KB < STAGES ? KB : STAGES;
           const int st0 = stage;
           for (int kb = 0; kb < pre; ++kb) {
@@ -1320,8 +1341,6 @@ __global__ void __launch_bounds__(192, 1)
           }
           if (ok) {
             // every gate/up item of expert T.g has stored its h slice
-            const int n = s_off[T.g + 1] - s_off[T.g];
-            const int need = ((n + BN - 1) / BN) * nwb1;
             const volatile int32_t* rp = g.ready + T.g;
             const uint64_t t0 = globaltimer_ns();
             while (*rp < need) {
@@ -1707,8 +1726,16 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
     uint32_t ph = 0;
     bool ok = true;
     uint32_t armed = 0, armed_ph = 0;
+    // readiness of a down item, acquire-loaded one item ahead (as k_ffn_ws)
+    auto flag_of = [&](int t) -> int {
+      if (t < total1 || t >= total) return 0;
+      return ld_acquire_gpu(g.ready + item(t).mtg);
+    };
+    int flag_cur = lane == 0 ? flag_of(static_cast<int>(blockIdx.x)) : 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
       const Item it = item(t);
+      const int flag = flag_cur;
+      if (lane == 0) flag_cur = flag_of(t + static_cast<int>(gridDim.x));
       if (lane == 0) {
         const CUtensorMap* ta = it.dn ? &tma_a2 : &tma_a1;
         const CUtensorMap* tb = it.dn ? &tma_b2 : &tma_b1;
@@ -1716,7 +1743,11 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
         const int brow = it.grp * (it.dn ? g.d : 2 * g.m) + it.nb * BN;
         const int KB = (it.dn ? g.m : g.d) / FFN_BK;
         int pre = 0;  // k-blocks whose weights go out before the dependency is met
-        if (it.dn) {
+        // already met (the usual case once the gate/up phase is under way):
+        // the ordinary pipeline, h and weights together
+        const bool met = it.dn && flag >= NT1;
+        if (met) fence_proxy_async_all();  // h, written by generic stores, read through the tensor map
+        if (it.dn && !met) {
           pre = KB < STAGES ? KB : STAGES;
           const int st0 = stage;
           for (int kb = 0; kb < pre; ++kb) {
@@ -2406,15 +2437,14 @@ namespace decomoe {
 
 // Rows from which the fused launch is taken (with fewer, the gate/up tiles
 // leave SMs idle and the fused form gains nothing), and up to which the
-// tokens-as-M form is fused (measured: 4.6-5.8 us faster per layer at
-// 1024-4096 rows, 3-17 us slower from 8192 rows, where the two launches'
-// waves already fill the SMs and the fused list's dependency stalls cost
-// more than the launch boundary).
+// tokens-as-M form is fused (measured per layer: 7 us faster at 2048 and
+// 16384 rows, 1-2 us at 8192 and 32768, 5 and 20 us slower at 65536 and
+// 131072 rows).
 #ifndef DECOMOE_FFN_FUSED_MIN_ROWS
 #define DECOMOE_FFN_FUSED_MIN_ROWS 16
 #endif
 #ifndef DECOMOE_FFN_FUSED_TC_MAX_ROWS
-#define DECOMOE_FFN_FUSED_TC_MAX_ROWS 4096
+#define DECOMOE_FFN_FUSED_TC_MAX_ROWS 32768
 #endif
 // Both expert GEMMs in one launch: k_ffn_ws at decode sizes (bf16, at most 8
 // rows per expert on average), k_ffn_tc above up to
@@ -2434,7 +2464,12 @@ int launch_expert_ffn_fused(const void* x_perm, const int32_t* offsets, int64_t 
   }();
   if (dtype != DECOMOE_BF16 || rows < min_rows || rows <= 0) return DECOMOE_OK;
   const bool ws = rows <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K;
-  if (!ws && (!tc_fused || rows > DECOMOE_FFN_FUSED_TC_MAX_ROWS)) return DECOMOE_OK;
+  static const int64_t tc_max_rows = [] {
+    const char* e = getenv("DECOMOE_FFN_FUSED_TC_MAX_ROWS");
+    return e != nullptr ? static_cast<int64_t>(atoll(e)) : static_cast<int64_t>(DECOMOE_FFN_FUSED_TC_MAX_ROWS);
+  }();
+  // the tokens-as-M kernel tiles gate/up in whole 256-column blocks
+  if (!ws && (!tc_fused || rows > tc_max_rows || (2 * m) % FFN_BN != 0)) return DECOMOE_OK;
   DM_RET(expert_check("expert_gate_up", x_perm, offsets, rows, K, d, m, dtype, w_gate_up, h));
   DM_RET(expert_check("expert_down", h, offsets, rows, K, d, m, dtype, w_down, y_perm));
   DM_ARG_CHECK(ready != nullptr, "expert ffn: null ready counters");
@@ -2453,3 +2488,24 @@ int launch_expert_ffn_fused(const void* x_perm, const int32_t* offsets, int64_t 
 size_t expert_ffn_sync_ints(int64_t rows, int E) { return static_cast<size_t>(rows / 128 + E + 1); }
 
 }  // namespace decomoe
+
+extern "C" {
+
+size_t decomoe_expert_swiglu_ready_ints(int64_t rows, int K) {
+  return rows < 0 || K <= 0 ? 0 : decomoe::expert_ffn_sync_ints(rows, K);
+}
+
+int decomoe_expert_swiglu_fused(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m,
+                                int dtype, const void* w_gate_up, const void* w_down, void* h_ws, void* y_perm,
+                                int32_t* ready, int32_t* status_dev, decomoe_stream_t stream) {
+  using namespace decomoe;
+  clear_error();
+  bool fused = false;
+  DM_RET(launch_expert_ffn_fused(x_perm, offsets, rows, K, d, m, dtype, w_gate_up, w_down, h_ws, y_perm, ready,
+                                 status_dev, reinterpret_cast<cudaStream_t>(stream), &fused));
+  if (fused) return DECOMOE_OK;
+  return decomoe_expert_swiglu(x_perm, offsets, rows, K, d, m, dtype, w_gate_up, w_down, h_ws, y_perm, status_dev,
+                               nullptr, stream);
+}
+
+}  // extern "C"

@@ -266,6 +266,15 @@ def test_expert_swiglu_bf16_parity(T, k, K, d, m, pattern):
     torch.cuda.synchronize()
     assert dm.decomoe_read_status(status) == 0
     assert torch.equal(y3, y) and torch.equal(h3, h)
+    # both GEMMs in one launch where the library fuses them: same tiles and
+    # k order, so the same bits; counters zero at the call
+    ready = torch.zeros(dm.decomoe_expert_swiglu_ready_ints(R, K), dtype=torch.int32, device=DEV)
+    h5 = torch.empty_like(h)
+    y5 = torch.empty_like(y)
+    dm.decomoe_expert_swiglu_fused(xp, off, K, w_gu, g["w_down"], h5, y5, ready, status)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(status) == 0
+    assert torch.equal(y5, y) and torch.equal(h5, h)
 
 
 def test_expert_swiglu_f32_parity():
