@@ -268,7 +268,9 @@ DECOMOE_API int decomoe_weight_layout(const void* w_gate, const void* w_up, void
  * maps; offsets stay on the device). Experts with no rows cost nothing.
  * bf16: tcgen05 tensor-core kernels for rows > 64, a weight-streaming kernel
  * for rows <= 64 (decode); fp32 accumulate, h rounded to bf16. f32: CUDA-core
- * kernels with h kept in fp32. Needs d % 64 == 0 and m % 128 == 0 (bf16).
+ * kernels with h kept in fp32. Needs m % 64 == 0; bf16 also m % 128 == 0,
+ * d % 256 == 0 and 16-byte aligned pointers (DECOMOE_ERR_INVALID_ARG
+ * otherwise, before any launch).
  * status_dev: optional device int32 collecting bounded-wait timeouts.
  * sched_dev: optional device int32 (4 bytes, caller-owned). Given, the
  * tensor-core kernels hand tiles out dynamically from this counter (the call

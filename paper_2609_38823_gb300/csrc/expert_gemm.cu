@@ -2273,6 +2273,8 @@ static int expert_check(const char* name, const void* a, const int32_t* offsets,
   if (rows == 0) return DECOMOE_OK;
   DM_ARG_CHECK(a && offsets && w && out, "%s: null pointer", name);
   if (dtype == DECOMOE_BF16) {
+    // tensor-core tiles: 256 output columns (gate/up interleaved 2m, down d)
+    DM_ARG_CHECK(m % 128 == 0, "%s: bf16 needs m %% 128 == 0 (m=%d)", name, m);
     DM_ARG_CHECK(d % 256 == 0, "%s: bf16 needs d %% 256 == 0 (d=%d)", name, d);
     DM_ARG_CHECK(aligned16(a) && aligned16(w) && aligned16(out), "%s: pointers must be 16-byte aligned", name);
   }

@@ -289,6 +289,10 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
   DM_ARG_CHECK(K_fixed > 0 || (p > 0.0 && p <= 1.0), "moe_layer: mass mode needs 0 < p <= 1");
   DM_ARG_CHECK(p >= 0.0 && p <= 1.0, "moe_layer: p outside [0, 1]");
   DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "moe_layer: bad dtype");
+  // the expert call's shape rules, checked before the first launch
+  DM_ARG_CHECK(m % DECOMOE_GU_BLOCK == 0, "moe_layer: m must be a multiple of %d", DECOMOE_GU_BLOCK);
+  DM_ARG_CHECK(dtype != DECOMOE_BF16 || (m % 128 == 0 && d % 256 == 0),
+               "moe_layer: bf16 needs m %% 128 == 0 and d %% 256 == 0 (m=%d, d=%d)", m, d);
   if (T == 0) {
     if (K_used_host) *K_used_host = K_fixed > 0 ? K_fixed : k;
     if (K_sel_host) *K_sel_host = k;

@@ -83,6 +83,17 @@ def test_argument_errors_are_caught_before_launch():
     assert L.decomoe_drop_visual_block(fake, fake, 10, 16, 8, 3, 1, 160, 112, None) == 1
     # m not a multiple of the gate/up block
     assert L.decomoe_expert_swiglu(fake, fake, 100, 4, 256, 100, 0, fake, fake, fake, fake, None, None, None) == 1
+    # bf16: m a multiple of the block but not of 128 (the tensor-core tiles span
+    # 256 interleaved gate/up columns); the fused form and the layer refuse it too
+    assert L.decomoe_expert_swiglu(fake, fake, 100, 4, 256, 192, 0, fake, fake, fake, fake, None, None, None) == 1
+    assert "m % 128" in L.decomoe_last_error().decode()
+    assert L.decomoe_expert_swiglu_fused(fake, fake, 100, 4, 256, 192, 0, fake, fake, fake, fake, fake, None,
+                                         None) == 1
+    assert L.decomoe_expert_swiglu_fused(fake, fake, 20, 4, 256, 192, 0, fake, fake, fake, fake, fake, None,
+                                         None) == 1
+    assert L.decomoe_moe_layer(fake, fake, None, fake, fake, 4, 256, 16, 4, 192, 0, 4, 0.0, None, fake,
+                               None, None, fake, 1 << 30, None, None) == 1
+    assert "m % 128" in L.decomoe_last_error().decode()
     # K_fixed < k
     assert L.decomoe_moe_layer(fake, fake, None, fake, fake, 4, 256, 16, 4, 128, 0, 2, 0.0, None, fake,
                                None, None, fake, 1 << 30, None, None) == 1
