@@ -82,8 +82,10 @@ DECOMOE_API int decomoe_device_info(int* sm_count_host, int* cc_major_host, int*
  *   logits[t, e] = sum_j x[t, j] * w_r[e, j] + bias[e]      (fp32 out)
  * x: [T, d] row-major, dtype; w_r: [E, d] row-major, dtype, rows in reordered
  * expert order; bias: [E] fp32 or NULL; logits: [T, E] fp32 row-major.
- * bf16 with d % 64 == 0 and E in {128, 256} runs on the tensor cores (fp32
- * accumulate); f32 and other bf16 shapes run a CUDA-core kernel.
+ * bf16 with T <= 6 and d % 8 == 0 runs a CUDA-core dot-product kernel (one
+ * block per router row); above that, d % 64 == 0 and E in {128, 256} run on
+ * the tensor cores (fp32 accumulate); f32 and other bf16 shapes run a
+ * CUDA-core kernel.
  * status_dev: optional device int32 that collects bounded-wait timeouts.
  * ------------------------------------------------------------------------ */
 DECOMOE_API int decomoe_router_logits(const void* x, const void* w_r, const float* bias, int64_t T, int d,
@@ -199,7 +201,7 @@ DECOMOE_API int decomoe_route_dispatch(const float* logits, int64_t T, int E, in
  * then decomoe_route_dispatch on them. Outputs (logits included) are
  * bit-identical to decomoe_router_logits_ws followed by
  * decomoe_route_dispatch with the same arguments. Where the router splits
- * its k loop (bf16, 96 < T, k slices that fit the SMs), the routing kernel
+ * its k loop (bf16, 6 < T, k slices that fit the SMs), the routing kernel
  * reads the router's partial sums itself, adding them in slice order and the
  * bias last exactly as the router's own reduction does, and writes the summed
  * logits; with a fixed K and mass_out the activated mass is added up by the

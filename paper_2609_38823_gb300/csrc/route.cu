@@ -35,14 +35,11 @@ __global__ void k_router_simt(const T* __restrict__ x, const T* __restrict__ w_r
   logits[i] = acc;
 }
 
-// Router for few tokens (decode): one warp per (expert row, group of
-// GEMV_TPW tokens). The warp loads its 16-byte slices of the router row and
-// of the tokens' rows (all loads in flight before any arithmetic), forms the
-// fp32 dot products of the bf16 values, and combines the lane partial sums
-// with a shuffle tree. The router matrix is read from HBM once and spread
-// over many SMs instead of one tensor-core tile.
+// Router for few tokens (decode) on CUDA cores: fp32 dot products of the bf16
+// router rows and token rows. The router matrix is read from HBM once and
+// spread over many SMs instead of one tensor-core tile.
 #ifndef DECOMOE_ROUTER_GEMV_MAX_T
-#define DECOMOE_ROUTER_GEMV_MAX_T 96  // token counts up to which the router runs on CUDA cores
+#define DECOMOE_ROUTER_GEMV_MAX_T 6  // token counts up to which the router runs on CUDA cores
 #endif
 // DECOMOE_ROUTER_GEMV_MAX_T in the environment overrides the compiled value
 // (read once per process).
@@ -53,8 +50,15 @@ static int64_t router_gemv_max_t() {
   }();
   return v;
 }
-constexpr int GEMV_WARPS = 4;
-constexpr int GEMV_TPW = 4;  // tokens per warp
+// One block per expert row and GEMV_TPB tokens: the block's 128 threads split
+// the row's 16-byte vectors (thread i takes vectors i, i + 128, ...), so a
+// row's loads are spread over four warps and the E rows over E blocks (one per
+// SM at decode sizes) instead of piling every row of a block onto one SM; all
+// of a thread's loads are issued before its first multiply. Partial dots are
+// reduced by warp shuffles, then over the four warps in a fixed order.
+constexpr int GEMV_THREADS = 128;
+constexpr int GEMV_TPB = 8;  // tokens per block
+constexpr int GEMV_VPT = 2;  // vectors per thread per pass (d = 2048: one pass)
 __device__ __forceinline__ float dot8_bf16(const uint4 a, const uint4 b, float acc) {
   acc = fmaf(bf16_lo(a.x), bf16_lo(b.x), acc);
   acc = fmaf(bf16_hi(a.x), bf16_hi(b.x), acc);
@@ -67,41 +71,48 @@ __device__ __forceinline__ float dot8_bf16(const uint4 a, const uint4 b, float a
   return acc;
 }
 
-__global__ void __launch_bounds__(32 * GEMV_WARPS)
+__global__ void __launch_bounds__(GEMV_THREADS)
     k_router_gemv(const uint4* __restrict__ x, const uint4* __restrict__ w_r, const float* __restrict__ bias,
                   int64_t Tn, int vpr, int E, float* __restrict__ logits) {
   pdl_enter();
+  __shared__ float red[GEMV_THREADS / 32][GEMV_TPB];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int e = blockIdx.x * GEMV_WARPS + warp;
-  const int64_t t0 = static_cast<int64_t>(blockIdx.y) * GEMV_TPW;
-  if (e >= E) return;
+  const int e = blockIdx.x;
+  const int64_t t0 = static_cast<int64_t>(blockIdx.y) * GEMV_TPB;
+  const int nt = Tn - t0 < GEMV_TPB ? static_cast<int>(Tn - t0) : GEMV_TPB;
   const uint4* wr = w_r + static_cast<int64_t>(e) * vpr;
-  float acc[GEMV_TPW];
+  float acc[GEMV_TPB];
 #pragma unroll
-  for (int j = 0; j < GEMV_TPW; ++j) acc[j] = 0.f;
+  for (int j = 0; j < GEMV_TPB; ++j) acc[j] = 0.f;
   const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
-  for (int c0 = 0; c0 < vpr; c0 += 32 * 8) {  // 8 vectors per lane per pass
-    uint4 wv[8], xv[GEMV_TPW][8];
+  for (int c0 = 0; c0 < vpr; c0 += GEMV_THREADS * GEMV_VPT) {
+    uint4 wv[GEMV_VPT], xv[GEMV_TPB][GEMV_VPT];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int c = c0 + lane + 32 * i;
+    for (int i = 0; i < GEMV_VPT; ++i) {
+      const int c = c0 + static_cast<int>(threadIdx.x) + GEMV_THREADS * i;
       wv[i] = (c < vpr) ? __ldg(wr + c) : zero;
 #pragma unroll
-      for (int j = 0; j < GEMV_TPW; ++j)
-        xv[j][i] = (c < vpr && t0 + j < Tn) ? __ldg(x + (t0 + j) * vpr + c) : zero;
+      for (int j = 0; j < GEMV_TPB; ++j) xv[j][i] = (c < vpr && j < nt) ? __ldg(x + (t0 + j) * vpr + c) : zero;
     }
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
+    for (int i = 0; i < GEMV_VPT; ++i)
 #pragma unroll
-      for (int j = 0; j < GEMV_TPW; ++j) acc[j] = dot8_bf16(wv[i], xv[j][i], acc[j]);
+      for (int j = 0; j < GEMV_TPB; ++j) acc[j] = dot8_bf16(wv[i], xv[j][i], acc[j]);
   }
-  const float b = bias != nullptr ? bias[e] : 0.f;
 #pragma unroll
-  for (int j = 0; j < GEMV_TPW; ++j) {
+  for (int j = 0; j < GEMV_TPB; ++j) {
     float v = acc[j];
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-    if (lane == 0 && t0 + j < Tn) logits[(t0 + j) * E + e] = v + b;
+    if (lane == 0) red[warp][j] = v;
+  }
+  __syncthreads();
+  if (static_cast<int>(threadIdx.x) < nt) {
+    const int j = threadIdx.x;
+    float v = red[0][j];
+#pragma unroll
+    for (int w = 1; w < GEMV_THREADS / 32; ++w) v += red[w][j];
+    logits[(t0 + j) * E + e] = v + (bias != nullptr ? bias[e] : 0.f);
   }
 }
 
@@ -361,8 +372,8 @@ int decomoe_router_logits(const void* x, const void* w_r, const float* bias, int
   DM_ARG_CHECK(x && w_r && logits, "router_logits: null pointer");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (dtype == DECOMOE_BF16 && T <= router_gemv_max_t() && d % 8 == 0 && aligned16(x) && aligned16(w_r)) {
-    const dim3 grid((E + GEMV_WARPS - 1) / GEMV_WARPS, static_cast<unsigned>((T + GEMV_TPW - 1) / GEMV_TPW));
-    DM_CUDA_CHECK(launch_pdl(k_router_gemv, grid, dim3(32 * GEMV_WARPS), 0, s, static_cast<const uint4*>(x),
+    const dim3 grid(static_cast<unsigned>(E), static_cast<unsigned>((T + GEMV_TPB - 1) / GEMV_TPB));
+    DM_CUDA_CHECK(launch_pdl(k_router_gemv, grid, dim3(GEMV_THREADS), 0, s, static_cast<const uint4*>(x),
                              static_cast<const uint4*>(w_r), bias, static_cast<int64_t>(T), d / 8, E, logits));
     return DECOMOE_OK;
   }

@@ -432,7 +432,8 @@ def test_drop_visual_block_if_follows_the_device_flag(shape, v0, nv, dt):
 
 @pytest.mark.parametrize("T,d,E", [(2048, 2048, 128), (1, 2048, 128), (300, 2048, 256), (1552, 2048, 128),
                                    (129, 256, 128), (7, 2048, 128), (192, 2048, 128), (193, 2048, 256),
-                                   (33, 4096, 64), (5, 2056, 16)])
+                                   (33, 4096, 64), (5, 2056, 16), (8, 2048, 128), (9, 2048, 256), (96, 2048, 128),
+                                   (3, 4096, 64), (6, 2048, 256)])
 def test_router_logits_bf16_tensor_cores(T, d, E):
     g = torch.Generator().manual_seed(T + E)
     x = torch.randn(T, d, generator=g).to(torch.bfloat16)
@@ -566,7 +567,8 @@ def test_router_logits_k_split(T, E):
     assert (err <= logit_error_bound(x64[rows], w64, b64)).all(), f"max err {err.max():.3e}"
 
 
-@pytest.mark.parametrize("T,E,K,p", [(1, 128, 64, 0.7), (96, 128, 64, 0.7), (97, 128, 64, 0.7), (100, 128, -1, 0.7),
+@pytest.mark.parametrize("T,E,K,p", [(1, 128, 64, 0.7), (6, 128, 64, 0.7), (7, 128, -1, 0.7), (8, 128, 64, 0.7),
+                                     (96, 128, 64, 0.7), (97, 128, 64, 0.7), (100, 128, -1, 0.7),
                                      (193, 128, 64, 0.7), (300, 256, -1, 0.7),
                                      (576, 128, 64, 0.0), (577, 128, -1, 0.5), (2048, 128, 64, 0.7),
                                      (2048, 128, -1, 0.7), (2432, 256, 40, 0.7), (2433, 128, 64, 0.7),

@@ -221,7 +221,8 @@ def test_layer_device_selected_prefix_in_cuda_graph(prefill_layer):
     assert Kdev == dm.decomoe_select_prefix(mass, k, 0.8)
 
 
-@pytest.mark.parametrize("T,K_fixed,p", [(1, 64, 0.7), (2, 64, 0.7), (8, 64, 0.7), (32, 40, 0.0), (100, 128, 0.7),
+@pytest.mark.parametrize("T,K_fixed,p", [(1, 64, 0.7), (2, 64, 0.7), (6, 64, 0.7), (7, 64, 0.7), (8, 64, 0.7),
+                                         (32, 40, 0.0), (100, 128, 0.7),
                                          (256, 96, 0.7), (1, -1, 0.7), (8, -1, 0.5), (129, -1, 0.9), (256, -1, 1.0),
                                          (2048, 64, 0.7), (2048, -1, 0.7)])
 def test_layer_intermediates_equal_separate_calls(T, K_fixed, p):
