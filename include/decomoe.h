@@ -495,7 +495,10 @@ DECOMOE_API int decomoe_moe_layer_exit(const void* x, const void* w_r, const flo
 
 /* Offsets (bytes) of the intermediates inside the decomoe_moe_layer workspace,
  * for inspection: logits, topk_idx, topk_w, mass, counts, offsets, perm_token,
- * inv_slot, x_perm, h, y_perm, device K (12 entries written to offs_host). */
+ * inv_slot, x_perm, h, y_perm, device K (12 entries written to offs_host).
+ * The layer's scratch rows are dropped from L2 after their last read (see
+ * decomoe_set_discard_scratch): turn that off before a call whose y_perm is
+ * to be inspected. */
 DECOMOE_API int decomoe_moe_layer_workspace_layout(int64_t T, int d, int E, int k, int m, int dtype,
                                        size_t* offs_host);
 
@@ -514,6 +517,16 @@ DECOMOE_API int decomoe_moe_layer_workspace_layout(int64_t T, int d, int E, int 
 DECOMOE_API int decomoe_read_status(int32_t* status_dev, int32_t* code_host, decomoe_stream_t stream);
 DECOMOE_API int decomoe_set_wait_limit_ns(int64_t limit_ns);
 DECOMOE_API int decomoe_selftest_wait(int32_t* status_dev, int64_t limit_ns, decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Scratch lines in L2. With on != 0 (the default), decomoe_moe_layer and
+ * decomoe_moe_layer_exit drop the L2 lines of their workspace's y_perm rows
+ * once the combine has read them (discard.global.L2): the rows are not
+ * written back to HBM, and the next layer's writes find clean lines to
+ * evict. Those workspace rows are undefined after the call. on == 0 keeps
+ * them (for inspection). Process-wide; applies to later calls.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API int decomoe_set_discard_scratch(int on);
 
 #ifdef __cplusplus
 }

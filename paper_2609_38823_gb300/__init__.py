@@ -88,6 +88,7 @@ SIGNATURES = {
     "decomoe_moe_layer_workspace_layout": (_I, [_L, _I, _I, _I, _I, _I, _P]),
     "decomoe_read_status": (_I, [_P, _P, _P]),
     "decomoe_set_wait_limit_ns": (_I, [_L]),
+    "decomoe_set_discard_scratch": (_I, [_I]),
     "decomoe_selftest_wait": (_I, [_P, _L, _P]),
 }
 
@@ -192,6 +193,10 @@ def decomoe_moe_layer_workspace_layout(T, d, E, k, m, dtype):
 
 def decomoe_set_wait_limit_ns(limit_ns: int):
     _check("decomoe_set_wait_limit_ns", lib().decomoe_set_wait_limit_ns(int(limit_ns)))
+
+
+def decomoe_set_discard_scratch(on: bool):
+    _check("decomoe_set_discard_scratch", lib().decomoe_set_discard_scratch(1 if on else 0))
 
 
 def decomoe_device_info():

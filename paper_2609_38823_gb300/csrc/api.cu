@@ -26,6 +26,9 @@ void clear_error() { t_last_error.clear(); }
 
 int64_t wait_limit_ns() { return g_wait_limit_ns.load(std::memory_order_relaxed); }
 
+static std::atomic<int> g_discard_scratch{1};
+bool discard_scratch() { return g_discard_scratch.load(std::memory_order_relaxed) != 0; }
+
 // Programmatic launch pays for grids of at most one block per SM (the
 // persistent GEMMs and the decode-size kernels); kernels of many blocks ran
 // slower with it, so they launch plainly. DECOMOE_PDL=0 turns it off;
@@ -111,6 +114,11 @@ int decomoe_read_status(int32_t* status_dev, int32_t* code_host, decomoe_stream_
 int decomoe_set_wait_limit_ns(int64_t limit_ns) {
   DM_ARG_CHECK(limit_ns > 0, "set_wait_limit_ns: limit must be positive");
   g_wait_limit_ns.store(limit_ns, std::memory_order_relaxed);
+  return DECOMOE_OK;
+}
+
+int decomoe_set_discard_scratch(int on) {
+  g_discard_scratch.store(on != 0 ? 1 : 0, std::memory_order_relaxed);
   return DECOMOE_OK;
 }
 

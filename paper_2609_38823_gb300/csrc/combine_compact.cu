@@ -54,11 +54,19 @@ struct DropRows {
 // WPT warps per token, each taking alternate 32-vector chunks of the row:
 // many tokens take one warp each (two blocks resident per SM), few tokens
 // spread each row over more warps.
+// discard (y is the caller's scratch, rows 128-byte aligned): every y line is
+// read exactly once (inv_slot is a bijection), so once a warp has summed its
+// rows it drops their L2 lines (discard.global.L2): the lines are not written
+// back to HBM, and the next writer of the scratch finds clean lines to evict.
+__device__ __forceinline__ void l2_discard_line(const void* p) {
+  asm volatile("discard.global.L2 [%0], 128;" ::"l"(p) : "memory");
+}
+
 template <bool BF16, int KT, bool DROP, int WPT>
 __global__ void __launch_bounds__(256, WPT == 1 ? 2 : 1)
     k_combine(const uint4* __restrict__ y, const int32_t* __restrict__ inv_slot,
               const float* __restrict__ w, int64_t Tn, int k, int vec,
-              const uint4* __restrict__ residual, uint4* __restrict__ out, DropRows drop) {
+              const uint4* __restrict__ residual, uint4* __restrict__ out, DropRows drop, int discard) {
   pdl_enter();
   constexpr int NE = BF16 ? 8 : 4;
   const int lane = threadIdx.x & 31;
@@ -102,6 +110,18 @@ __global__ void __launch_bounds__(256, WPT == 1 ? 2 : 1)
             acc_vec<BF16>(acc, v[j], wts[j]);
             acc_vec<BF16>(acc2, v2[j], wts[j]);
           }
+        if (discard) {
+          // every lane's loads of these lines have been consumed above
+          __syncwarp();
+          if ((lane & 7) == 0) {
+#pragma unroll
+            for (int j = 0; j < KT; ++j)
+              if (rows[j] >= 0) {
+                l2_discard_line(y + static_cast<int64_t>(rows[j]) * vec + c);
+                if (two) l2_discard_line(y + static_cast<int64_t>(rows[j]) * vec + c2);
+              }
+          }
+        }
         const uint4 o1 = finish_vec<BF16>(acc, residual, t * vec + c);
         out[t * vec + c] = o1;
         if (text_row) drop.text[trow * vec + c] = o1;
@@ -139,31 +159,31 @@ static int grid_for_warps(int64_t warps);
 
 template <bool BF16, bool DROP, int WPT>
 static cudaError_t launch_combine_w(cudaStream_t s, const uint4* y, const int32_t* inv, const float* w, int64_t T,
-                                    int k, int vec, const uint4* res, uint4* out, DropRows drop) {
+                                    int k, int vec, const uint4* res, uint4* out, DropRows drop, int dc) {
   const dim3 g(grid_for_warps(WPT * T)), b(256);
   switch (k) {
-    case 1: return launch_pdl(k_combine<BF16, 1, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop);
-    case 2: return launch_pdl(k_combine<BF16, 2, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop);
-    case 4: return launch_pdl(k_combine<BF16, 4, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop);
-    case 8: return launch_pdl(k_combine<BF16, 8, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop);
-    default: return launch_pdl(k_combine<BF16, 0, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop);
+    case 1: return launch_pdl(k_combine<BF16, 1, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop, dc);
+    case 2: return launch_pdl(k_combine<BF16, 2, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop, dc);
+    case 4: return launch_pdl(k_combine<BF16, 4, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop, dc);
+    case 8: return launch_pdl(k_combine<BF16, 8, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop, dc);
+    default: return launch_pdl(k_combine<BF16, 0, DROP, WPT>, g, b, 0, s, y, inv, w, T, k, vec, res, out, drop, 0);
   }
 }
 // Warps per token by token count: one from 1024 tokens on, two from 256, four
 // from 32, eight below (a decode step's row then spans eight warps).
 template <bool BF16, bool DROP>
 static cudaError_t launch_combine_k(cudaStream_t s, const uint4* y, const int32_t* inv, const float* w, int64_t T,
-                                    int k, int vec, const uint4* res, uint4* out, DropRows drop) {
-  if (T >= 1024) return launch_combine_w<BF16, DROP, 1>(s, y, inv, w, T, k, vec, res, out, drop);
-  if (T >= 256) return launch_combine_w<BF16, DROP, 2>(s, y, inv, w, T, k, vec, res, out, drop);
-  if (T >= 32) return launch_combine_w<BF16, DROP, 4>(s, y, inv, w, T, k, vec, res, out, drop);
-  return launch_combine_w<BF16, DROP, 8>(s, y, inv, w, T, k, vec, res, out, drop);
+                                    int k, int vec, const uint4* res, uint4* out, DropRows drop, int dc) {
+  if (T >= 1024) return launch_combine_w<BF16, DROP, 1>(s, y, inv, w, T, k, vec, res, out, drop, dc);
+  if (T >= 256) return launch_combine_w<BF16, DROP, 2>(s, y, inv, w, T, k, vec, res, out, drop, dc);
+  if (T >= 32) return launch_combine_w<BF16, DROP, 4>(s, y, inv, w, T, k, vec, res, out, drop, dc);
+  return launch_combine_w<BF16, DROP, 8>(s, y, inv, w, T, k, vec, res, out, drop, dc);
 }
 template <bool BF16>
 static cudaError_t launch_combine(cudaStream_t s, const uint4* y, const int32_t* inv, const float* w, int64_t T,
-                                  int k, int vec, const uint4* res, uint4* out, DropRows drop) {
-  return drop.text != nullptr ? launch_combine_k<BF16, true>(s, y, inv, w, T, k, vec, res, out, drop)
-                              : launch_combine_k<BF16, false>(s, y, inv, w, T, k, vec, res, out, drop);
+                                  int k, int vec, const uint4* res, uint4* out, DropRows drop, int dc) {
+  return drop.text != nullptr ? launch_combine_k<BF16, true>(s, y, inv, w, T, k, vec, res, out, drop, dc)
+                              : launch_combine_k<BF16, false>(s, y, inv, w, T, k, vec, res, out, drop, dc);
 }
 
 // ------------------------------------------------------------------ compaction
@@ -311,7 +331,7 @@ namespace decomoe {
 
 int combine_impl(const void* y_perm, const int32_t* inv_slot, const float* topk_w, int64_t T, int k, int d,
                  int dtype, const void* residual, void* out, void* text_out, int64_t v0, int64_t nv,
-                 decomoe_stream_t stream) {
+                 decomoe_stream_t stream, bool discard_y) {
   DM_ARG_CHECK(T >= 0 && k >= 1 && k <= DECOMOE_MAX_TOPK && d > 0, "combine: bad sizes");
   DM_ARG_CHECK(dtype == DECOMOE_BF16 || dtype == DECOMOE_F32, "combine: bad dtype");
   if (T == 0) return DECOMOE_OK;
@@ -335,12 +355,14 @@ int combine_impl(const void* y_perm, const int32_t* inv_slot, const float* topk_
   }
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const int vec = static_cast<int>(row_bytes / 16);
+  // whole 128-byte lines only
+  const int dc = discard_y && row_bytes % 128 == 0 && reinterpret_cast<uintptr_t>(y_perm) % 128 == 0 ? 1 : 0;
   if (dtype == DECOMOE_BF16)
     DM_CUDA_CHECK(launch_combine<true>(s, static_cast<const uint4*>(y_perm), inv_slot, topk_w, T, k, vec,
-                                       static_cast<const uint4*>(residual), static_cast<uint4*>(out), drop));
+                                       static_cast<const uint4*>(residual), static_cast<uint4*>(out), drop, dc));
   else
     DM_CUDA_CHECK(launch_combine<false>(s, static_cast<const uint4*>(y_perm), inv_slot, topk_w, T, k, vec,
-                                        static_cast<const uint4*>(residual), static_cast<uint4*>(out), drop));
+                                        static_cast<const uint4*>(residual), static_cast<uint4*>(out), drop, dc));
   return DECOMOE_OK;
 }
 

@@ -151,7 +151,10 @@ int dispatch_with_mass(const int32_t* topk_idx, int64_t T, int k, int K, const v
 // output rows (decomoe_combine_drop_visual_block).
 int combine_impl(const void* y_perm, const int32_t* inv_slot, const float* topk_w, int64_t T, int k, int d,
                  int dtype, const void* residual, void* out, void* text_out, int64_t v0, int64_t nv,
-                 decomoe_stream_t stream);
+                 decomoe_stream_t stream, bool discard_y = false);
+// Whether calls that own scratch rows drop them from L2 after their last read
+// (decomoe_set_discard_scratch; on by default).
+bool discard_scratch();
 // decomoe_drop_visual_block; with flag, only when *flag == 1 on the device.
 int drop_visual_block_impl(const int32_t* flag, const void* src, void* dst, int64_t rows, int64_t row_bytes,
                            int64_t v0, int64_t nv, int64_t nbatch, int64_t src_batch_stride,

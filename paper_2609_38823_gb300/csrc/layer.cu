@@ -373,7 +373,9 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
     DM_RET(decomoe_expert_swiglu(x_perm, offsets, T * k, K, d, m, dtype, w_gate_up, w_down, h, y_perm, status_dev,
                                  nullptr, stream));
   // a7: combine (+ residual); with text_out also a8 on the layer output
-  return combine_impl(y_perm, inv, topk_w, T, k, d, dtype, residual, out, text_out, v0, nv, stream);
+  // y_perm is the call's own scratch: its lines leave L2 without a write-back
+  return combine_impl(y_perm, inv, topk_w, T, k, d, dtype, residual, out, text_out, v0, nv, stream,
+                      discard_scratch());
 }
 
 }  // namespace decomoe

@@ -238,10 +238,21 @@ def test_layer_intermediates_equal_separate_calls(T, K_fixed, p):
     out = torch.empty_like(g["x"])
     ws = dm.workspace(dm.decomoe_moe_layer_workspace_bytes(T, d, E, k, m, dm.DECOMOE_BF16), DEV)
     st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    # by default the combine drops the y rows from L2 after reading them: the
+    # output must not depend on it; the run that keeps them is inspected below
     dm.decomoe_moe_layer(g["x"], g["w_r"], g["bias"], w_gu, g["w_down"], k, out, ws, K_fixed=K_fixed, p=p,
                          status=st)
     torch.cuda.synchronize()
+    out_discard = out.clone()
+    dm.decomoe_set_discard_scratch(False)
+    try:
+        dm.decomoe_moe_layer(g["x"], g["w_r"], g["bias"], w_gu, g["w_down"], k, out, ws, K_fixed=K_fixed, p=p,
+                             status=st)
+        torch.cuda.synchronize()
+    finally:
+        dm.decomoe_set_discard_scratch(True)
     assert dm.decomoe_read_status(st) == 0
+    assert torch.equal(out.view(torch.int16), out_discard.view(torch.int16))
     offs = dm.decomoe_moe_layer_workspace_layout(T, d, E, k, m, dm.DECOMOE_BF16)
     view = lambda i, n, dt: ws[offs[i]:offs[i] + n * torch.tensor([], dtype=dt).element_size()].view(dt)
     logits = view(0, T * E, torch.float32).view(T, E).clone()
