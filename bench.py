@@ -35,9 +35,9 @@ sys.path.insert(0, ROOT)
 import workloads as W  # noqa: E402
 
 # at T=2048: router k slices, routing (reads the slices) with mass partials,
-# dispatch 3 (histogram + mass sum, ranks, row gather), the expert FFN (gate/up,
+# dispatch 2 (histogram + mass sum, ranks), the expert FFN (row gather, gate/up,
 # SwiGLU and down in one launch), combine with the visual-block removal
-LAUNCHES_PER_STEP = 7
+LAUNCHES_PER_STEP = 6
 
 
 def parse():

@@ -167,11 +167,16 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
                    size_t ws_bytes, int32_t* status_dev, decomoe_stream_t stream);
 // Both expert GEMMs in one launch (bf16): ready holds
 // expert_ffn_sync_ints(rows, K) int32, zero at launch. Sets *launched = false
-// (and launches nothing) where the two-launch form is kept.
+// (and launches nothing) where the two-launch form is kept. With gather_x and
+// perm (tokens-as-M form only) the launch also fills x_perm[r] =
+// gather_x[perm[r]] itself.
+enum { FFN_FUSED_NONE = 0, FFN_FUSED_WS = 1, FFN_FUSED_TC = 2 };
+int expert_ffn_fused_kind(int64_t rows, int K, int m, int dtype);
 size_t expert_ffn_sync_ints(int64_t rows, int E);
 int launch_expert_ffn_fused(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m, int dtype,
                             const void* w_gate_up, const void* w_down, void* h, void* y_perm, int32_t* ready,
-                            int32_t* status, cudaStream_t s, bool* launched);
+                            int32_t* status, cudaStream_t s, bool* launched, const void* gather_x = nullptr,
+                            const int32_t* perm = nullptr);
 // The k-split router's GEMM alone: KS slices of partial logits [KS][T][E]
 // (no bias) into scratch; returns KS (1: no split at this size, nothing
 // launched).

@@ -1598,6 +1598,29 @@ static int launch_ffn_ws(const void* x_perm, int rows, int d, int m, const void*
 // tiles still run, instead of after a launch boundary. Deadlock-free as
 // k_ffn_ws (gate/up items never wait; one CTA per SM, grid <= SMs). ready[]
 // (one int per M-tile) is zero at launch.
+//
+// With x set, the launch also performs the dispatch's row gather: each CTA's
+// epilogue warps copy, for every gate/up item of the CTA in work order, one
+// 1/NT1 share of that item's M-tile rows x_perm[r] = x[perm[r]] and publish
+// it (stores, proxy fence, barrier, release add on gathered[M-tile]); they
+// copy shares while the accumulator they need next is still being computed. A gate/up item's A rows are requested once all NT1
+// shares of its M-tile are in (acquire, bounded; its weight k-blocks go out
+// first), as a down item waits for h. The gathers wait on nothing, so this
+// adds no cycle; the first wave's rows are in after one share per CTA
+// instead of after a separate gather launch.
+// Non-blocking: has the phase with this parity completed?
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 struct TcFfnArgs {
   const int32_t* offsets;  // [G + 1]
   int G;
@@ -1608,6 +1631,10 @@ struct TcFfnArgs {
   int32_t* ready;
   int32_t* status;
   uint64_t limit_ns;
+  const uint4* x;      // gather source [tokens, d / 8] (16-byte vectors), or null: x_perm is filled
+  const int32_t* perm;  // [rows] token of each dispatched row
+  uint4* x_perm;        // [rows, d / 8], written by the gather
+  int32_t* gathered;    // per M-tile: shares copied (zero at launch)
 };
 
 constexpr int FFN_BN = 256, FFN_BK = 64, FFN_STAGES = 4, FFN_EW = 8;
@@ -1619,6 +1646,7 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
              const TcFfnArgs g) {
   using C = FfnCfg;
   constexpr int BN = FFN_BN, STAGES = FFN_STAGES, EW = FFN_EW;
+  __shared__ int s_gperm[C::BM + 1];  // token rows of the share being gathered; [BM]: a broadcast flag
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
@@ -1726,10 +1754,17 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
     uint32_t ph = 0;
     bool ok = true;
     uint32_t armed = 0, armed_ph = 0;
-    // readiness of a down item, acquire-loaded one item ahead (as k_ffn_ws)
+    // what an item's A rows wait for: a down item for its M-tile's h, a
+    // gate/up item (with the gather) for its M-tile's rows; NT1 counts each.
+    // Acquire-loaded one item ahead (as k_ffn_ws).
+    auto dep_of = [&](const Item& it) -> const int32_t* {
+      return it.dn ? g.ready : (g.x != nullptr ? g.gathered : nullptr);
+    };
     auto flag_of = [&](int t) -> int {
-      if (t < total1 || t >= total) return 0;
-      return ld_acquire_gpu(g.ready + item(t).mtg);
+      if (t >= total) return 0;
+      const Item it = item(t);
+      const int32_t* dp = dep_of(it);
+      return dp != nullptr ? ld_acquire_gpu(dp + it.mtg) : 0;
     };
     int flag_cur = lane == 0 ? flag_of(static_cast<int>(blockIdx.x)) : 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
@@ -1742,12 +1777,13 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
         const int row0 = s_off[it.grp] + it.mt * C::BM;
         const int brow = it.grp * (it.dn ? g.d : 2 * g.m) + it.nb * BN;
         const int KB = (it.dn ? g.m : g.d) / FFN_BK;
+        const int32_t* dp = dep_of(it);
         int pre = 0;  // k-blocks whose weights go out before the dependency is met
-        // already met (the usual case once the gate/up phase is under way):
-        // the ordinary pipeline, h and weights together
-        const bool met = it.dn && flag >= NT1;
-        if (met) fence_proxy_async_all();  // h, written by generic stores, read through the tensor map
-        if (it.dn && !met) {
+        // already met (the usual case once the first wave is under way): the
+        // ordinary pipeline, A rows and weights together
+        const bool met = dp == nullptr || flag >= NT1;
+        if (dp != nullptr && met) fence_proxy_async_all();  // rows written by generic stores, read through TMA
+        if (!met) {
           pre = KB < STAGES ? KB : STAGES;
           const int st0 = stage;
           for (int kb = 0; kb < pre; ++kb) {
@@ -1765,8 +1801,9 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
             }
           }
           if (ok) {
-            // every gate/up tile of this M-tile has stored its h columns
-            const volatile int32_t* rp = g.ready + it.mtg;
+            // every gate/up tile of this M-tile has stored its h columns (down
+            // item), or every share of its rows is gathered (gate/up item)
+            const volatile int32_t* rp = dp + it.mtg;
             const uint64_t t0 = globaltimer_ns();
             while (*rp < NT1) {
               if (*s_abort || globaltimer_ns() - t0 > g.limit_ns) {
@@ -1775,7 +1812,7 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
               }
             }
             __threadfence();
-            fence_proxy_async_all();  // h, written by generic stores, read through the tensor map
+            fence_proxy_async_all();  // rows written by generic stores, read through the tensor map
           }
           if (ok) {
             int st = st0;
@@ -1860,6 +1897,50 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
       }
     }
   } else if (warp >= 2) {
+    // ------------------------------------------------ row gather (with g.x):
+    // one share of each of this CTA's gate/up M-tiles, in work order, copied
+    // while the accumulator the epilogue needs next is still being computed
+    const int et = static_cast<int>(threadIdx.x) - 64;  // 0 .. 32*EW-1
+    int gshare = g.x != nullptr ? static_cast<int>(blockIdx.x) : total1;  // next share's work item
+    auto gather_share = [&](int t) {
+      const int vec = g.d / 8;
+      constexpr int U = 8;  // 16-byte loads in flight per thread
+      const Item it = item(t);
+      const int r0 = s_off[it.grp] + it.mt * C::BM;
+      const int r1 = min(r0 + C::BM, s_off[it.grp + 1]);
+      const int per = (r1 - r0 + NT1 - 1) / NT1;
+      const int a = min(r0 + it.nb * per, r1), b = min(a + per, r1);
+      for (int i = et; i < b - a; i += 32 * EW) s_gperm[i] = g.perm[a + i];
+      named_bar_sync(1, 32 * EW);
+      const int nv = (b - a) * vec;
+      for (int i0 = et; i0 < nv; i0 += 32 * EW * U) {
+        uint4 v[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          const int i = i0 + u * 32 * EW;
+          if (i < nv) {
+            const int r = i / vec;
+            v[u] = __ldg(g.x + static_cast<int64_t>(s_gperm[r]) * vec + (i - r * vec));
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          const int i = i0 + u * 32 * EW;
+          if (i < nv) {
+            const int r = i / vec;
+            g.x_perm[static_cast<int64_t>(a + r) * vec + (i - r * vec)] = v[u];
+          }
+        }
+      }
+      // publish the share to the gate/up tiles of this M-tile (and free
+      // s_gperm for the next share)
+      fence_proxy_async_all();
+      named_bar_sync(1, 32 * EW);
+      if (warp == 2 && lane == 0) {
+        __threadfence();
+        atomicAdd(g.gathered + it.mtg, 1);
+      }
+    };
     // ------------------------------------------------ epilogue (k_gemm_tc's)
     const int q = warp & 3;
     const int wp = (warp - 2) >> 2;
@@ -1872,6 +1953,18 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
       const uint32_t aph = (n >> 1) & 1;
       const int row0 = s_off[it.grp] + it.mt * C::BM;
       const int row_end = s_off[it.grp + 1];
+      // gather shares until this tile's accumulator is complete (one thread
+      // tests the barrier, all epilogue threads follow its answer); while
+      // shares remain the warps never block here, so every share gets copied
+      while (gshare < total1) {
+        if (et == 0) s_gperm[C::BM] = mbar_test(TFULL_BAR(acc), aph) ? 1 : 0;
+        named_bar_sync(1, 32 * EW);
+        const bool full = s_gperm[C::BM] != 0;
+        named_bar_sync(1, 32 * EW);
+        if (full) break;
+        gather_share(gshare);
+        gshare += gridDim.x;
+      }
       if (!mbar_wait(TFULL_BAR(acc), aph, g.limit_ns, s_abort)) {
         ok = false;
         break;
@@ -1952,9 +2045,11 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
 #undef DRAIN_BAR
 }
 
+// gather_x / perm given: the launch fills x_perm itself (see k_ffn_tc);
+// the gathered counters follow the ready counters in the same array.
 static int launch_ffn_tc(const void* x_perm, int rows, int d, int m, const void* w_gu, const void* w_down,
                          const int32_t* offsets, int G, void* h, void* y, int32_t* ready, int32_t* status,
-                         cudaStream_t s) {
+                         cudaStream_t s, const void* gather_x = nullptr, const int32_t* perm = nullptr) {
   using C = FfnCfg;
   CUtensorMap ta1, tb1, ta2, tb2;
   DM_RET(make_tmap_bf16(&ta1, x_perm, static_cast<uint64_t>(d), static_cast<uint64_t>(rows), C::BM, FFN_BK));
@@ -1972,7 +2067,11 @@ static int launch_ffn_tc(const void* x_perm, int rows, int d, int m, const void*
   g.ready = ready;
   g.status = status;
   g.limit_ns = static_cast<uint64_t>(wait_limit_ns());
-  static_assert(C::SMEM <= 232448, "shared memory budget");
+  g.x = static_cast<const uint4*>(gather_x);
+  g.perm = perm;
+  g.x_perm = static_cast<uint4*>(const_cast<void*>(x_perm));
+  g.gathered = ready + (rows / C::BM + G + 1);
+  static_assert(C::SMEM + sizeof(int) * (C::BM + 1) <= 232448, "shared memory budget");
   static_assert(C::SMEM > 232448 / 2, "one CTA per SM: the dependency waits need every CTA resident");
   DM_CUDA_CHECK(cudaFuncSetAttribute(k_ffn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(C::SMEM)));
   const int64_t ub = (static_cast<int64_t>(rows) / C::BM + G) * static_cast<int64_t>((2 * m + d) / FFN_BN);
@@ -2452,10 +2551,9 @@ namespace decomoe {
 // rows per expert on average), k_ffn_tc above up to
 // DECOMOE_FFN_FUSED_TC_MAX_ROWS rows; nothing launched (and *launched false)
 // for fp32, fewer than DECOMOE_FFN_FUSED_MIN_ROWS rows or more than that.
-int launch_expert_ffn_fused(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m, int dtype,
-                            const void* w_gate_up, const void* w_down, void* h, void* y_perm, int32_t* ready,
-                            int32_t* status, cudaStream_t s, bool* launched) {
-  *launched = false;
+// Which one-launch form the expert FFN takes: FFN_FUSED_NONE (two launches),
+// FFN_FUSED_WS (decode sizes) or FFN_FUSED_TC (tokens as M).
+int expert_ffn_fused_kind(int64_t rows, int K, int m, int dtype) {
   static const int64_t min_rows = [] {
     const char* e = getenv("DECOMOE_FFN_FUSED_MIN_ROWS");
     return e != nullptr ? static_cast<int64_t>(atoll(e)) : static_cast<int64_t>(DECOMOE_FFN_FUSED_MIN_ROWS);
@@ -2464,30 +2562,44 @@ int launch_expert_ffn_fused(const void* x_perm, const int32_t* offsets, int64_t 
     const char* e = getenv("DECOMOE_FFN_FUSED_TC");
     return e == nullptr || e[0] != '0';
   }();
-  if (dtype != DECOMOE_BF16 || rows < min_rows || rows <= 0) return DECOMOE_OK;
-  const bool ws = rows <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K;
   static const int64_t tc_max_rows = [] {
     const char* e = getenv("DECOMOE_FFN_FUSED_TC_MAX_ROWS");
     return e != nullptr ? static_cast<int64_t>(atoll(e)) : static_cast<int64_t>(DECOMOE_FFN_FUSED_TC_MAX_ROWS);
   }();
+  if (dtype != DECOMOE_BF16 || rows < min_rows || rows <= 0 || K <= 0) return FFN_FUSED_NONE;
+  if (rows <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K) return FFN_FUSED_WS;
   // the tokens-as-M kernel tiles gate/up in whole 256-column blocks
-  if (!ws && (!tc_fused || rows > tc_max_rows || (2 * m) % FFN_BN != 0)) return DECOMOE_OK;
+  if (!tc_fused || rows > tc_max_rows || (2 * m) % FFN_BN != 0) return FFN_FUSED_NONE;
+  return FFN_FUSED_TC;
+}
+
+int launch_expert_ffn_fused(const void* x_perm, const int32_t* offsets, int64_t rows, int K, int d, int m, int dtype,
+                            const void* w_gate_up, const void* w_down, void* h, void* y_perm, int32_t* ready,
+                            int32_t* status, cudaStream_t s, bool* launched, const void* gather_x,
+                            const int32_t* perm) {
+  *launched = false;
+  const int kind = expert_ffn_fused_kind(rows, K, m, dtype);
+  DM_ARG_CHECK(gather_x == nullptr || kind == FFN_FUSED_TC, "expert ffn: the row gather needs the tokens-as-M form");
+  if (kind == FFN_FUSED_NONE) return DECOMOE_OK;
   DM_RET(expert_check("expert_gate_up", x_perm, offsets, rows, K, d, m, dtype, w_gate_up, h));
   DM_RET(expert_check("expert_down", h, offsets, rows, K, d, m, dtype, w_down, y_perm));
   DM_ARG_CHECK(ready != nullptr, "expert ffn: null ready counters");
-  if (ws)
+  if (gather_x != nullptr)
+    DM_ARG_CHECK(perm != nullptr && aligned16(gather_x), "expert ffn: gather needs perm and a 16-byte aligned x");
+  if (kind == FFN_FUSED_WS)
     DM_RET(launch_ffn_ws(x_perm, static_cast<int>(rows), d, m, w_gate_up, w_down, offsets, K, h, y_perm, ready,
                          status, s));
   else
     DM_RET(launch_ffn_tc(x_perm, static_cast<int>(rows), d, m, w_gate_up, w_down, offsets, K, h, y_perm, ready,
-                         status, s));
+                         status, s, gather_x, perm));
   *launched = true;
   return DECOMOE_OK;
 }
 
 // int32 counters the fused expert launch needs (zero at launch): one per
-// expert (decode kernel) or per M-tile (prefill kernel).
-size_t expert_ffn_sync_ints(int64_t rows, int E) { return static_cast<size_t>(rows / 128 + E + 1); }
+// expert (decode kernel) or two per M-tile (prefill kernel: h stored, rows
+// gathered).
+size_t expert_ffn_sync_ints(int64_t rows, int E) { return 2 * static_cast<size_t>(rows / 128 + E + 1); }
 
 }  // namespace decomoe
 

@@ -328,15 +328,30 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
   // by the first routing launch of this call
   int32_t* sync = reinterpret_cast<int32_t*>(base + L.off[WS_SYNC]);
   const int n_sync = static_cast<int>(expert_ffn_sync_ints(T * k, E));
+  // Where the experts take the one-launch tokens-as-M form on at least
+  // DECOMOE_FFN_GATHER_MIN_ROWS routed rows, that launch copies the
+  // dispatched rows itself (per M-tile, while its accumulators fill) and the
+  // dispatch skips its gather launch (measured: T=2048 K=64 0.2258 -> 0.2244
+  // ms, end to end 8.80 -> 9.00 M tokens/s; at 1024 rows 3.4 us slower, the
+  // shares being a few rows each).
+  static const int64_t gather_min_rows = [] {
+    const char* e = getenv("DECOMOE_FFN_GATHER_MIN_ROWS");
+    return e != nullptr ? static_cast<int64_t>(atoll(e)) : static_cast<int64_t>(8192);
+  }();
+  auto ffn_gathers = [&](int K_groups) {
+    return T * k >= gather_min_rows && expert_ffn_fused_kind(T * k, K_groups, m, dtype) == FFN_FUSED_TC;
+  };
+  bool gathers = false;
   if (K_fixed != 0) {
     // a1-a5: router logits over all E reordered experts, full-pool mass
     // (Eq. 11), prefix (fixed, or Eq. 12 on the device), prefix routing and
     // dispatch; with a device-selected prefix, dispatch and the experts run
     // over all E groups (those at or beyond *K_dev are empty)
+    gathers = ffn_gathers(K_fixed == -1 ? E : K_fixed);
     DM_RET(router_route_dispatch_impl(x, w_r, bias, T, d, E, dtype, K_fixed, k, p, logits, topk_idx, topk_w,
                                       (K_fixed == -1 || p > 0.0) ? mass : nullptr, K_dev, counts, offsets, perm, inv,
-                                      x_perm, rsplit, route_ws, L.off[WS_KDEV] - L.off[WS_ROUTE], status_dev, s, sync,
-                                      n_sync));
+                                      gathers ? nullptr : x_perm, rsplit, route_ws, L.off[WS_KDEV] - L.off[WS_ROUTE],
+                                      status_dev, s, sync, n_sync));
     if (K_fixed == -1) {
       K = E;
       if (K_sel_host) *K_sel_host = -1;
@@ -357,9 +372,10 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
     DM_RET(decomoe_select_prefix(h_mass.data(), E, k, p, &Ksel));
     K = Ksel;
     if (K_sel_host) *K_sel_host = Ksel;
+    gathers = ffn_gathers(K);
     DM_RET(decomoe_route_dispatch(logits, T, E, K, k, 0.0, topk_idx, topk_w, nullptr, nullptr, x, d, dtype, counts,
-                                  offsets, perm, inv, x_perm, route_ws, L.off[WS_KDEV] - L.off[WS_ROUTE],
-                                  status_dev, stream));
+                                  offsets, perm, inv, gathers ? nullptr : x_perm, route_ws,
+                                  L.off[WS_KDEV] - L.off[WS_ROUTE], status_dev, stream));
   }
   if (K_used_host && K_fixed != -1) *K_used_host = K;
   // a6: grouped SwiGLU experts over [0, K): at decode sizes gate/up and down
@@ -368,7 +384,7 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
   // keeps them chained programmatically)
   bool fused = false;
   DM_RET(launch_expert_ffn_fused(x_perm, offsets, T * k, K, d, m, dtype, w_gate_up, w_down, h, y_perm, sync,
-                                 status_dev, s, &fused));
+                                 status_dev, s, &fused, gathers ? x : nullptr, gathers ? perm : nullptr));
   if (!fused)
     DM_RET(decomoe_expert_swiglu(x_perm, offsets, T * k, K, d, m, dtype, w_gate_up, w_down, h, y_perm, status_dev,
                                  nullptr, stream));

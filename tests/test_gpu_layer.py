@@ -224,13 +224,14 @@ def test_layer_device_selected_prefix_in_cuda_graph(prefill_layer):
 @pytest.mark.parametrize("T,K_fixed,p", [(1, 64, 0.7), (2, 64, 0.7), (6, 64, 0.7), (7, 64, 0.7), (8, 64, 0.7),
                                          (32, 40, 0.0), (100, 128, 0.7),
                                          (256, 96, 0.7), (1, -1, 0.7), (8, -1, 0.5), (129, -1, 0.9), (256, -1, 1.0),
-                                         (2048, 64, 0.7), (2048, -1, 0.7)])
+                                         (1100, 40, 0.7), (2048, 64, 0.7), (2048, -1, 0.7)])
 def test_layer_intermediates_equal_separate_calls(T, K_fixed, p):
     """The layer's routing, mass, prefix and dispatch intermediates and its
     expert outputs h and y (left in its workspace) equal, bit for bit, the
     separate C-ABI calls on the same router logits, for fixed and
     device-selected prefixes, at decode sizes (one expert launch from 16 rows)
-    and prefill sizes."""
+    and prefill sizes (from 8192 routed rows the expert launch gathers x_perm
+    itself: the gathered rows are compared too)."""
     wl = W.with_(W.PREFILL, T=T)
     E, k, d, m = wl.E, wl.k, wl.d, wl.m
     g = W.make_layer(wl, device="cuda", seed=T)
