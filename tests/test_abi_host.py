@@ -120,3 +120,12 @@ def test_workspace_queries():
     assert b >= 2048 * 8 * (2048 * 2 * 2 + 768 * 2)  # x_perm, y_perm and h
     offs = dm.decomoe_moe_layer_workspace_layout(2048, 2048, 128, 8, 768, 0)
     assert offs == sorted(offs) and all(o % 256 == 0 for o in offs)
+
+
+def test_expert_ready_counter_count():
+    # the one-launch expert FFN needs two counters per possible M-tile
+    # (h stored, rows gathered): at most rows/128 + K M-tiles, one spare each
+    for rows, K in ((16384, 64), (1, 1), (1000, 128), (0, 8)):
+        assert dm.decomoe_expert_swiglu_ready_ints(rows, K) == 2 * (rows // 128 + K + 1)
+    assert dm.decomoe_expert_swiglu_ready_ints(-1, 8) == 0
+    assert dm.decomoe_expert_swiglu_ready_ints(100, 0) == 0
