@@ -1767,6 +1767,7 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
       return dp != nullptr ? ld_acquire_gpu(dp + it.mtg) : 0;
     };
     int flag_cur = lane == 0 ? flag_of(static_cast<int>(blockIdx.x)) : 0;
+    const uint64_t pol_once = policy_evict_first();
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
       const Item it = item(t);
       const int flag = flag_cur;
@@ -1778,6 +1779,9 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
         const int brow = it.grp * (it.dn ? g.d : 2 * g.m) + it.nb * BN;
         const int KB = (it.dn ? g.m : g.d) / FFN_BK;
         const int32_t* dp = dep_of(it);
+        // an expert of one M-tile reads its weights once: they go to L2 as
+        // evict-first, leaving room for the weights that later M-tiles reuse
+        const bool once = s_mt[it.grp + 1] - s_mt[it.grp] == 1;
         int pre = 0;  // k-blocks whose weights go out before the dependency is met
         // already met (the usual case once the first wave is under way): the
         // ordinary pipeline, A rows and weights together
@@ -1792,7 +1796,10 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
               break;
             }
             mbar_arrive_expect_tx(FULL_BAR(stage), C::A_BYTES + C::B_BYTES);
-            tma_load_2d(sB + stage * C::B_BYTES, tb, FULL_BAR(stage), kb * FFN_BK, brow);
+            if (once)
+              tma_load_2d_hint(sB + stage * C::B_BYTES, tb, FULL_BAR(stage), kb * FFN_BK, brow, pol_once);
+            else
+              tma_load_2d(sB + stage * C::B_BYTES, tb, FULL_BAR(stage), kb * FFN_BK, brow);
             armed |= 1u << stage;
             armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
             if (++stage == STAGES) {
@@ -1829,7 +1836,10 @@ __global__ void __launch_bounds__(64 + 32 * FFN_EW, 1)
           }
           mbar_arrive_expect_tx(FULL_BAR(stage), C::A_BYTES + C::B_BYTES);
           tma_load_2d(sA + stage * C::A_BYTES, ta, FULL_BAR(stage), kb * FFN_BK, row0);
-          tma_load_2d(sB + stage * C::B_BYTES, tb, FULL_BAR(stage), kb * FFN_BK, brow);
+          if (once)
+            tma_load_2d_hint(sB + stage * C::B_BYTES, tb, FULL_BAR(stage), kb * FFN_BK, brow, pol_once);
+          else
+            tma_load_2d(sB + stage * C::B_BYTES, tb, FULL_BAR(stage), kb * FFN_BK, brow);
           armed |= 1u << stage;
           armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
           if (++stage == STAGES) {
