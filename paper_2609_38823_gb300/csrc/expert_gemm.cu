@@ -943,9 +943,13 @@ __global__ void __launch_bounds__(192, 1)
     uint32_t ph = 0;
     bool ok = true;
     uint32_t armed = 0, armed_ph = 0;
+    // an expert of one token chunk reads each weight block once: evict-first
+    // in L2 (blocks of larger experts are re-read by their next chunks)
+    const uint64_t pol_once = policy_evict_first();
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
       const WsTile T = ws_tile<WS_BN>(t, total, s_tt, s_off, G, nwb);
       const int wrow0 = T.g * g.wrows + T.wb * WS_BM;
+      const bool once = s_off[T.g + 1] - s_off[T.g] <= WS_BN;
       int nload;       // TMA copies for B per k-block
       uint32_t bytes;  // bytes landing per stage
       if constexpr (GATHER_B) {
@@ -965,7 +969,10 @@ __global__ void __launch_bounds__(192, 1)
             break;
           }
           mbar_arrive_expect_tx(FULL_BAR(stage), bytes);
-          tma_load_2d(sA + stage * C::A_BYTES, &tma_w, FULL_BAR(stage), kb * WS_BK, wrow0);
+          if (once)
+            tma_load_2d_hint(sA + stage * C::A_BYTES, &tma_w, FULL_BAR(stage), kb * WS_BK, wrow0, pol_once);
+          else
+            tma_load_2d(sA + stage * C::A_BYTES, &tma_w, FULL_BAR(stage), kb * WS_BK, wrow0);
           const uint32_t dB = sB + stage * C::B_BYTES;
           if constexpr (GATHER_B) {
             for (int i = 0; i < nload; ++i)
@@ -1305,6 +1312,7 @@ __global__ void __launch_bounds__(192, 1)
       return ld_acquire_gpu(g.ready + U.g);
     };
     int flag_cur = lane == 0 ? flag_of(static_cast<int>(blockIdx.x)) : 0;
+    const uint64_t pol_once = policy_evict_first();
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
       bool dn;
       const WsTile T = item(t, dn);
@@ -1314,6 +1322,8 @@ __global__ void __launch_bounds__(192, 1)
         const CUtensorMap* tw = dn ? &tma_w2 : &tma_w1;
         const CUtensorMap* tx = dn ? &tma_x2 : &tma_x1;
         const int wrow0 = T.g * (dn ? g.wrows2 : g.wrows1) + T.wb * WS_BM;
+        // an expert of one token chunk reads each weight block once: evict-first
+        const bool once = s_off[T.g + 1] - s_off[T.g] <= BN;
         const int KB = (dn ? g.kdim2 : g.kdim1) / WS_BK;
         const int nload = (T.ntok + WS_BOX - 1) / WS_BOX;
         const uint32_t bytes = C::A_BYTES + nload * C::BOX_BYTES;
@@ -1331,7 +1341,10 @@ __global__ void __launch_bounds__(192, 1)
               break;
             }
             mbar_arrive_expect_tx(FULL_BAR(stage), bytes);
-            tma_load_2d(sA + stage * C::A_BYTES, tw, FULL_BAR(stage), kb * WS_BK, wrow0);
+            if (once)
+              tma_load_2d_hint(sA + stage * C::A_BYTES, tw, FULL_BAR(stage), kb * WS_BK, wrow0, pol_once);
+            else
+              tma_load_2d(sA + stage * C::A_BYTES, tw, FULL_BAR(stage), kb * WS_BK, wrow0);
             armed |= 1u << stage;
             armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
             if (++stage == STAGES) {
@@ -1368,7 +1381,10 @@ __global__ void __launch_bounds__(192, 1)
             break;
           }
           mbar_arrive_expect_tx(FULL_BAR(stage), bytes);
-          tma_load_2d(sA + stage * C::A_BYTES, tw, FULL_BAR(stage), kb * WS_BK, wrow0);
+          if (once)
+            tma_load_2d_hint(sA + stage * C::A_BYTES, tw, FULL_BAR(stage), kb * WS_BK, wrow0, pol_once);
+          else
+            tma_load_2d(sA + stage * C::A_BYTES, tw, FULL_BAR(stage), kb * WS_BK, wrow0);
           const uint32_t dB = sB + stage * C::B_BYTES;
           for (int i = 0; i < nload; ++i)
             tma_load_2d(dB + i * C::BOX_BYTES, tx, FULL_BAR(stage), kb * WS_BK, T.row0 + i * WS_BOX);
