@@ -235,7 +235,11 @@ DECOMOE_API int decomoe_router_route_dispatch(const void* x, const void* w_r, co
  * DECOMOE_ERR_INVALID_ARG with a message and nothing launched.
  *   - The first call on a device looks up the array's device address (once
  *     per device, with that device current); make that first call before any
- *     stream capture.
+ *     stream capture. A first call made while its stream is capturing returns
+ *     DECOMOE_ERR_INVALID_ARG and launches nothing.
+ *   - The address is cached per device ordinal for the life of the process:
+ *     it assumes the device's primary context outlives every call and is not
+ *     looked up again after cudaDeviceReset.
  *   - Calls never allocate or free device memory.
  *   - All calls on a device share the one array and it keeps the last call's
  *     contents; nothing in it needs to start at zero (each call writes every
@@ -527,6 +531,16 @@ DECOMOE_API int decomoe_selftest_wait(int32_t* status_dev, int64_t limit_ns, dec
  * them (for inspection). Process-wide; applies to later calls.
  * ------------------------------------------------------------------------ */
 DECOMOE_API int decomoe_set_discard_scratch(int on);
+
+/* ------------------------------------------------------------------------
+ * Programmatic dependent launch. With on != 0 (the default) kernels of at
+ * most one block per SM are launched so that their blocks are scheduled while
+ * the previous kernel on the stream drains; each waits (griddepcontrol.wait)
+ * before it reads what earlier kernels wrote, so results are the same bits
+ * either way. on == 0 launches every kernel plainly. Process-wide; applies
+ * to later launches and to graphs captured after the call.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API int decomoe_set_pdl(int on);
 
 #ifdef __cplusplus
 }

@@ -89,6 +89,7 @@ SIGNATURES = {
     "decomoe_read_status": (_I, [_P, _P, _P]),
     "decomoe_set_wait_limit_ns": (_I, [_L]),
     "decomoe_set_discard_scratch": (_I, [_I]),
+    "decomoe_set_pdl": (_I, [_I]),
     "decomoe_selftest_wait": (_I, [_P, _L, _P]),
 }
 
@@ -197,6 +198,10 @@ def decomoe_set_wait_limit_ns(limit_ns: int):
 
 def decomoe_set_discard_scratch(on: bool):
     _check("decomoe_set_discard_scratch", lib().decomoe_set_discard_scratch(1 if on else 0))
+
+
+def decomoe_set_pdl(on: bool):
+    _check("decomoe_set_pdl", lib().decomoe_set_pdl(1 if on else 0))
 
 
 def decomoe_device_info():

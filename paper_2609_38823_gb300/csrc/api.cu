@@ -31,17 +31,10 @@ bool discard_scratch() { return g_discard_scratch.load(std::memory_order_relaxed
 
 // Programmatic launch pays for grids of at most one block per SM (the
 // persistent GEMMs and the decode-size kernels); kernels of many blocks ran
-// slower with it, so they launch plainly. DECOMOE_PDL=0 turns it off;
-// DECOMOE_PDL_MAX_BLOCKS overrides the grid-size limit.
+// slower with it, so they launch plainly. decomoe_set_pdl(0) turns it off.
+static std::atomic<int> g_pdl{1};
 bool pdl_enabled(int64_t blocks) {
-  static const int64_t max_blocks = [] {
-    const char* on = getenv("DECOMOE_PDL");
-    if (on != nullptr && on[0] == '0') return static_cast<int64_t>(-1);
-    const char* v = getenv("DECOMOE_PDL_MAX_BLOCKS");
-    if (v != nullptr) return static_cast<int64_t>(atoll(v));
-    return static_cast<int64_t>(0);  // 0: one block per SM of the current device
-  }();
-  return blocks <= (max_blocks == 0 ? static_cast<int64_t>(sm_count()) : max_blocks);
+  return g_pdl.load(std::memory_order_relaxed) != 0 && blocks <= static_cast<int64_t>(sm_count());
 }
 
 int sm_count() {
@@ -114,6 +107,11 @@ int decomoe_read_status(int32_t* status_dev, int32_t* code_host, decomoe_stream_
 int decomoe_set_wait_limit_ns(int64_t limit_ns) {
   DM_ARG_CHECK(limit_ns > 0, "set_wait_limit_ns: limit must be positive");
   g_wait_limit_ns.store(limit_ns, std::memory_order_relaxed);
+  return DECOMOE_OK;
+}
+
+int decomoe_set_pdl(int on) {
+  g_pdl.store(on != 0 ? 1 : 0, std::memory_order_relaxed);
   return DECOMOE_OK;
 }
 

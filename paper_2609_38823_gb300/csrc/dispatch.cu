@@ -214,9 +214,12 @@ namespace decomoe {
 
 static __device__ __align__(256) int32_t g_noalloc_dispatch_scratch[DECOMOE_NOALLOC_DISPATCH_SCRATCH_INTS];
 
-// Device address of the array, looked up once per device (host code cannot
-// use the symbol itself as a device pointer).
-static int noalloc_scratch_ptr(int32_t** out) {
+// Device address of the array, looked up once per device ordinal (host code
+// cannot use the symbol itself as a device pointer). The cached address
+// belongs to the device's primary context as it was at the first call: it is
+// not looked up again after cudaDeviceReset. The first call on a device must
+// not be made while `s` is being captured into a graph.
+static int noalloc_scratch_ptr(int32_t** out, cudaStream_t s) {
   static std::mutex mu;
   static int32_t* ptrs[64] = {nullptr};
   int dev = 0;
@@ -227,6 +230,13 @@ static int noalloc_scratch_ptr(int32_t** out) {
   }
   std::lock_guard<std::mutex> lk(mu);
   if (ptrs[dev] == nullptr) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    DM_CUDA_CHECK(cudaStreamIsCapturing(s, &cs));
+    if (cs != cudaStreamCaptureStatusNone) {
+      set_error("dispatch_noalloc: the first call on device %d is inside a stream capture; make one call on "
+                "this device before capturing", dev);
+      return DECOMOE_ERR_INVALID_ARG;
+    }
     void* p = nullptr;
     DM_CUDA_CHECK(cudaGetSymbolAddress(&p, g_noalloc_dispatch_scratch));
     ptrs[dev] = static_cast<int32_t*>(p);
@@ -268,7 +278,7 @@ extern "C" int decomoe_dispatch_noalloc(const int32_t* topk_idx, int64_t T, int 
                  "dispatch_noalloc: rows must be 16-byte multiples and 16-byte aligned");
   }
   int32_t* tile_hist = nullptr;
-  DM_RET(noalloc_scratch_ptr(&tile_hist));
+  DM_RET(noalloc_scratch_ptr(&tile_hist, s));
   // k_dispatch_hist writes every entry the scatter pass reads, so nothing
   // left in the array by an earlier call is ever used.
   const int ntiles = static_cast<int>(ntiles64);

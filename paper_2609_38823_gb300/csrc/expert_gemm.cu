@@ -30,11 +30,6 @@
 // when the average expert gets at most DECOMOE_WS_MAX_AVG_ROWS rows (decode
 // sizes: every tile streams its own weight slice), the tokens-as-M k_gemm_tc
 // otherwise (prefill: faster when many rows share an expert's weights).
-// How the gathered gate/up entry loads its A rows: 2 = cp.async rows by four
-// extra warps, 1 = TMA tile::gather4.
-#ifndef DECOMOE_GATHER_MODE
-#define DECOMOE_GATHER_MODE 2
-#endif
 #ifndef DECOMOE_WS_MAX_AVG_ROWS
 #define DECOMOE_WS_MAX_AVG_ROWS 8
 #endif
@@ -137,28 +132,12 @@ struct TcCfg {
 // experts whose weights stream from HBM once; mixing them in every wave keeps
 // both HBM and the tensor pipes busy instead of running the two phases one
 // after the other.
-#ifndef DECOMOE_TILE_ORDER
-#define DECOMOE_TILE_ORDER 1
-#endif
 __device__ __forceinline__ void tile_coords(int tile, int NT, const int* s_mt, int G, int& grp, int& mt,
                                             int& nb) {
   const int mtot = s_mt[G];
-#if DECOMOE_TILE_ORDER == 2
-  {
-    // multiplicative permutation of the work items (a bijection when the
-    // multiplier is coprime with their count)
-    const int total = mtot * NT;
-    const int P = (total % 7919 != 0) ? 7919 : 7907;
-    tile = static_cast<int>((static_cast<long long>(tile) * P) % total);
-  }
-#endif
   const int j = tile / NT;
   nb = tile - j * NT;
-#if DECOMOE_TILE_ORDER == 1
   const int mtg = (j & 1) ? (mtot - 1 - (j >> 1)) : (j >> 1);
-#else
-  const int mtg = j;
-#endif
   int lo = 0, hi = G - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
@@ -174,10 +153,9 @@ __device__ __forceinline__ void tile_coords(int tile, int NT, const int* s_mt, i
 // EW epilogue warps (4 or 8): with 8, two warps share each 32-lane TMEM
 // quarter and split its column chunks, so the epilogue's latency is hidden.
 // GA: how A tiles reach shared memory. 0: tiled TMA of rows [row0, row0+128)
-// of A. 1: TMA tile::gather4 of the rows a_rows[row0 ..] (warp 0). 2: four
-// extra warps, one A row per thread, 16-byte cp.async of the rows
-// a_rows[row0 ..] into the 128-byte-swizzled layout the TMA would produce;
-// each thread's copies complete on the stage's full barrier.
+// of A. 2: four extra warps, one A row per thread, 16-byte cp.async of the
+// rows a_rows[row0 ..] into the 128-byte-swizzled layout the TMA would
+// produce; each thread's copies complete on the stage's full barrier.
 // KS: split of the k loop. Work item = (output tile, k slice); slice s runs
 // k-blocks [s*KB/KS, (s+1)*KB/KS) and writes its partial sums to
 // out + s * split_stride (EPI_F32_BIAS_T only; the caller adds the slices).
@@ -186,11 +164,10 @@ __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
     k_gemm_tc(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b,
               const TcArgs g) {
   using C = TcCfg<BN, STAGES, BK, MP, OCC>;
+  static_assert(GA == 0 || GA == 2, "A rows by tiled TMA (0) or by cp.async gather (2)");
   static_assert(!(GA != 0 && MP != 1), "gathered A takes one M-tile per work item");
   static_assert(GA != 2 || BK == 64, "the cp.async gather writes 128-byte swizzled rows");
   static_assert(KS == 1 || (EPI == EPI_F32_BIAS_T && MP == 1 && GA == 0), "k split: transposed fp32 partials only");
-  constexpr bool GATHER_A = GA == 1;
-  __shared__ int s_arow[GATHER_A ? 128 : 1];
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
@@ -314,9 +291,7 @@ __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
   };
 
   if (warp == 0) {
-    // ------------------------------------------------ TMA producer (lane 0
-    // issues; with GATHER_A the whole warp first reads the tile's 128 A row
-    // indices into shared memory)
+    // ------------------------------------------------ TMA producer (lane 0 issues)
     if (lane == 0) {
       tma_prefetch_desc(&tma_a);
       tma_prefetch_desc(&tma_b);
@@ -341,40 +316,7 @@ __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
       const int brow = grp * g.n_per_group + nb * BN;
       const int kbase = (tile % KS) * KB;  // first k-block of this work item's slice
       const bool has2 = MP == 2 && row0 + C::BM < s_off[grp + 1];  // second M-tile has rows
-      if constexpr (GATHER_A) {
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int r = row0 + lane * 4 + i;
-          s_arow[lane * 4 + i] = (r < g.rows) ? g.a_rows[r] : 0;  // rows past the end: any valid row, not stored
-        }
-        __syncwarp();
-      }
-      if constexpr (GATHER_A) {
-        // the warp issues the 32 four-row gathers of a k-block in parallel
-        for (int kb = 0; kb < KB; ++kb) {
-          bool got = true;
-          if (lane == 0) got = mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort);
-          got = __shfl_sync(0xffffffffu, got, 0);
-          if (!got) {
-            ok = false;
-            break;
-          }
-          if (lane == 0) {
-            mbar_arrive_expect_tx(FULL_BAR(stage), C::STAGE_BYTES);
-            tma_load_2d(sB + stage * C::B_BYTES, &tma_b, FULL_BAR(stage), kb * C::BK, brow);
-          }
-          __syncwarp();
-          const uint32_t dA = sA + stage * C::A_BYTES;
-          tma_gather4(dA + lane * 4 * (C::BK * 2), &tma_a, FULL_BAR(stage), kb * C::BK, s_arow[4 * lane],
-                      s_arow[4 * lane + 1], s_arow[4 * lane + 2], s_arow[4 * lane + 3]);
-          armed |= 1u << stage;
-          armed_ph = (armed_ph & ~(1u << stage)) | (ph << stage);
-          if (++stage == STAGES) {
-            stage = 0;
-            ph ^= 1u;
-          }
-        }
-      } else if (lane == 0) {
+      if (lane == 0) {
         for (int kb = 0; kb < KB; ++kb) {
           if (!mbar_wait(EMPTY_BAR(stage), ph ^ 1u, g.limit_ns, s_abort)) {
             ok = false;
@@ -683,7 +625,7 @@ __global__ void __launch_bounds__(64 + 32 * EW + (GA == 2 ? 128 : 0), OCC)
 #undef TQE_BAR
 }
 
-// A: [rows, kdim], or with GATHER_A the source tensor [a_tensor_rows, kdim]
+// A: [rows, kdim], or with GA == 2 the source tensor [a_tensor_rows, kdim]
 // whose row a_rows[r] is A row r.
 template <int BN, int EPI, int STAGES, int BK, int GA = 0, int MP = 1, int EW = 8, int OCC = 1, int KS = 1>
 static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b_rows,
@@ -693,9 +635,7 @@ static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b
                      int64_t split_stride = 0) {
   using C = TcCfg<BN, STAGES, BK, MP, OCC>;
   CUtensorMap ta, tb;
-  if (GA == 1)
-    DM_RET(make_tmap_bf16(&ta, A, static_cast<uint64_t>(kdim), static_cast<uint64_t>(a_tensor_rows), 1, BK));
-  else if (GA == 2)
+  if (GA == 2)
     ta = CUtensorMap{};  // A is read with cp.async, not TMA
   else
     DM_RET(make_tmap_bf16(&ta, A, static_cast<uint64_t>(kdim), static_cast<uint64_t>(rows), C::BM, BK));
@@ -723,11 +663,7 @@ static int launch_tc(const void* A, int rows, int kdim, const void* B, int64_t b
                                      static_cast<int>(C::SMEM)));
   const int64_t ub_tiles =
       (static_cast<int64_t>(rows) / C::BM + ngroups) * static_cast<int64_t>(n_per_group / BN) * KS;
-#ifdef DECOMOE_GRID_CAP
-  const int64_t cap = std::min<int64_t>(static_cast<int64_t>(sm_count()) * OCC, DECOMOE_GRID_CAP);
-#else
   const int64_t cap = static_cast<int64_t>(sm_count()) * OCC;
-#endif
   const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(cap, ub_tiles)));
   DM_CUDA_CHECK(launch_pdl(kern, dim3(grid), dim3(64 + 32 * EW + (GA == 2 ? 128 : 0)), C::SMEM, s, ta, tb, g));
   return DECOMOE_OK;
@@ -767,9 +703,6 @@ struct WsArgs {
 
 #ifndef DECOMOE_WS_BOX
 #define DECOMOE_WS_BOX 32
-#endif
-#ifndef DECOMOE_WS_ORDER
-#define DECOMOE_WS_ORDER 0  // 0: weight block outer, token chunk inner; 1: chunk outer
 #endif
 constexpr int WS_BM = 128, WS_BK = 64, WS_BOX = DECOMOE_WS_BOX;
 
@@ -822,13 +755,8 @@ __device__ __forceinline__ WsTile ws_tile(int t, int total, const int* s_tt, con
   const int n = s_off[lo + 1] - s_off[lo];
   const int nch = (n + WS_BN - 1) / WS_BN;
   const int local = tp - s_tt[lo];
-#if DECOMOE_WS_ORDER == 1
-  const int c = local / nwb;
-  r.wb = local - c * nwb;
-#else
   r.wb = local / nch;
   const int c = local - r.wb * nch;
-#endif
   r.row0 = s_off[lo] + c * WS_BN;
   r.ntok = min(WS_BN, n - c * WS_BN);
   return r;
@@ -2510,7 +2438,7 @@ int decomoe_expert_gate_up_gather(const void* x, int64_t T, const int32_t* perm_
   }
   if (static_cast<int64_t>(R) <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K)
     return launch_ws<true, 4, true>(x, R, d, w_gate_up, 2 * m, offsets, K, h, m, status_dev, s, perm_token, T);
-  return launch_tc<256, EPI_SWIGLU, GU_STAGES, GU_BK, DECOMOE_GATHER_MODE>(
+  return launch_tc<256, EPI_SWIGLU, GU_STAGES, GU_BK, 2>(
       x, R, d, w_gate_up, static_cast<int64_t>(K) * 2 * m, offsets, K, 2 * m, h, m, nullptr, status_dev, s, 0,
       perm_token, T);
 }
@@ -2580,22 +2508,12 @@ namespace decomoe {
 // Which one-launch form the expert FFN takes: FFN_FUSED_NONE (two launches),
 // FFN_FUSED_WS (decode sizes) or FFN_FUSED_TC (tokens as M).
 int expert_ffn_fused_kind(int64_t rows, int K, int m, int dtype) {
-  static const int64_t min_rows = [] {
-    const char* e = getenv("DECOMOE_FFN_FUSED_MIN_ROWS");
-    return e != nullptr ? static_cast<int64_t>(atoll(e)) : static_cast<int64_t>(DECOMOE_FFN_FUSED_MIN_ROWS);
-  }();
-  static const bool tc_fused = [] {
-    const char* e = getenv("DECOMOE_FFN_FUSED_TC");
-    return e == nullptr || e[0] != '0';
-  }();
-  static const int64_t tc_max_rows = [] {
-    const char* e = getenv("DECOMOE_FFN_FUSED_TC_MAX_ROWS");
-    return e != nullptr ? static_cast<int64_t>(atoll(e)) : static_cast<int64_t>(DECOMOE_FFN_FUSED_TC_MAX_ROWS);
-  }();
+  constexpr int64_t min_rows = DECOMOE_FFN_FUSED_MIN_ROWS;
+  constexpr int64_t tc_max_rows = DECOMOE_FFN_FUSED_TC_MAX_ROWS;
   if (dtype != DECOMOE_BF16 || rows < min_rows || rows <= 0 || K <= 0) return FFN_FUSED_NONE;
   if (rows <= static_cast<int64_t>(DECOMOE_WS_MAX_AVG_ROWS) * K) return FFN_FUSED_WS;
   // the tokens-as-M kernel tiles gate/up in whole 256-column blocks
-  if (!tc_fused || rows > tc_max_rows || (2 * m) % FFN_BN != 0) return FFN_FUSED_NONE;
+  if (rows > tc_max_rows || (2 * m) % FFN_BN != 0) return FFN_FUSED_NONE;
   return FFN_FUSED_TC;
 }
 

@@ -329,15 +329,12 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
   int32_t* sync = reinterpret_cast<int32_t*>(base + L.off[WS_SYNC]);
   const int n_sync = static_cast<int>(expert_ffn_sync_ints(T * k, E));
   // Where the experts take the one-launch tokens-as-M form on at least
-  // DECOMOE_FFN_GATHER_MIN_ROWS routed rows, that launch copies the
+  // gather_min_rows routed rows, that launch copies the
   // dispatched rows itself (per M-tile, while its accumulators fill) and the
   // dispatch skips its gather launch (measured: T=2048 K=64 0.2258 -> 0.2244
   // ms, end to end 8.80 -> 9.00 M tokens/s; at 1024 rows 3.4 us slower, the
   // shares being a few rows each).
-  static const int64_t gather_min_rows = [] {
-    const char* e = getenv("DECOMOE_FFN_GATHER_MIN_ROWS");
-    return e != nullptr ? static_cast<int64_t>(atoll(e)) : static_cast<int64_t>(8192);
-  }();
+  constexpr int64_t gather_min_rows = 8192;
   auto ffn_gathers = [&](int K_groups) {
     return T * k >= gather_min_rows && expert_ffn_fused_kind(T * k, K_groups, m, dtype) == FFN_FUSED_TC;
   };

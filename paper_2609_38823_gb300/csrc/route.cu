@@ -41,15 +41,7 @@ __global__ void k_router_simt(const T* __restrict__ x, const T* __restrict__ w_r
 #ifndef DECOMOE_ROUTER_GEMV_MAX_T
 #define DECOMOE_ROUTER_GEMV_MAX_T 6  // token counts up to which the router runs on CUDA cores
 #endif
-// DECOMOE_ROUTER_GEMV_MAX_T in the environment overrides the compiled value
-// (read once per process).
-static int64_t router_gemv_max_t() {
-  static const int64_t v = [] {
-    const char* e = getenv("DECOMOE_ROUTER_GEMV_MAX_T");
-    return e != nullptr ? static_cast<int64_t>(atoll(e)) : static_cast<int64_t>(DECOMOE_ROUTER_GEMV_MAX_T);
-  }();
-  return v;
-}
+static constexpr int64_t router_gemv_max_t() { return DECOMOE_ROUTER_GEMV_MAX_T; }
 // One block per expert row and GEMV_TPB tokens: the block's 128 threads split
 // the row's 16-byte vectors (thread i takes vectors i, i + 128, ...), so a
 // row's loads are spread over four warps and the E rows over E blocks (one per

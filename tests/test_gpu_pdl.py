@@ -1,67 +1,53 @@
 """Programmatic dependent launch changes when kernels start, never what they
 compute: the layer's output and its routing/dispatch intermediates are
-bit-identical with it on (the default) and off (DECOMOE_PDL=0), at prefill and
-decode sizes, over several graph replays. A kernel that read its
+bit-identical with it on (the default) and off (decomoe_set_pdl(0)), at
+prefill and decode sizes, over several graph replays. A kernel that read its
 predecessor's output before griddepcontrol.wait would show up here as a
-mismatch. The setting is read once per process, so each run is a subprocess.
+mismatch.
 """
-import os
-import subprocess
-import sys
-
 import pytest
 import torch
 
-pytestmark = pytest.mark.gpu
-ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-
-SCRIPT = r"""
-import sys, torch
-sys.path.insert(0, sys.argv[1])
 import paper_2609_38823_gb300 as dm
 import workloads as W
+
+pytestmark = pytest.mark.gpu
 DEV = torch.device("cuda")
-out_path = sys.argv[2]
-res = {}
-for T, K in ((2048, 64), (8, 64), (1, -1)):
-    wl = W.with_(W.PREFILL, T=T)
-    g = W.make_layer(wl, device="cuda", seed=5)
-    wgu = dm.fuse_gate_up(g["w_gate"], g["w_up"])
-    out = torch.empty_like(g["x"])
-    ws = dm.workspace(dm.decomoe_moe_layer_workspace_bytes(T, wl.d, wl.E, wl.k, wl.m, 0), DEV)
-    ws.zero_()  # padding between sub-buffers compares equal too
-    st = torch.zeros(1, dtype=torch.int32, device=DEV)
-    fn = lambda: dm.decomoe_moe_layer(g["x"], g["w_r"], g["bias"], wgu, g["w_down"], wl.k, out, ws, K_fixed=K,
-                                      p=0.7, residual=g["x"], status=st)
-    gr = dm.capture_graph(fn)
-    for _ in range(5):
-        gr.replay()
-    torch.cuda.synchronize()
-    assert dm.decomoe_read_status(st) == 0
-    res[f"{T}_{K}_out"] = out.cpu().clone()
-    res[f"{T}_{K}_ws"] = ws[: dm.decomoe_moe_layer_workspace_layout(T, wl.d, wl.E, wl.k, wl.m, 0)[8]].cpu().clone()
-torch.save(res, out_path)
-"""
 
 
-def _run(tmp_path, env_extra, name):
-    path = tmp_path / f"{name}.pt"
-    script = tmp_path / "pdl_run.py"
-    script.write_text(SCRIPT)
-    env = dict(os.environ)
-    env.update(env_extra)
-    r = subprocess.run([sys.executable, str(script), ROOT, str(path)], env=env, capture_output=True, text=True,
-                       timeout=600)
-    assert r.returncode == 0, r.stderr[-3000:]
-    return torch.load(path)
+def _run():
+    res = {}
+    for T, K in ((2048, 64), (8, 64), (1, -1)):
+        wl = W.with_(W.PREFILL, T=T)
+        g = W.make_layer(wl, device="cuda", seed=5)
+        wgu = dm.fuse_gate_up(g["w_gate"], g["w_up"])
+        out = torch.empty_like(g["x"])
+        ws = dm.workspace(dm.decomoe_moe_layer_workspace_bytes(T, wl.d, wl.E, wl.k, wl.m, 0), DEV)
+        ws.zero_()  # padding between sub-buffers compares equal too
+        st = torch.zeros(1, dtype=torch.int32, device=DEV)
+        fn = lambda: dm.decomoe_moe_layer(g["x"], g["w_r"], g["bias"], wgu, g["w_down"], wl.k, out, ws, K_fixed=K,
+                                          p=0.7, residual=g["x"], status=st)
+        gr = dm.capture_graph(fn)
+        for _ in range(5):
+            gr.replay()
+        torch.cuda.synchronize()
+        assert dm.decomoe_read_status(st) == 0
+        res[f"{T}_{K}_out"] = out.cpu().clone()
+        res[f"{T}_{K}_ws"] = ws[: dm.decomoe_moe_layer_workspace_layout(T, wl.d, wl.E, wl.k, wl.m, 0)[8]].cpu().clone()
+        del gr
+    return res
 
 
-def test_pdl_on_and_off_give_identical_bits(tmp_path):
+def test_pdl_on_and_off_give_identical_bits():
     import __graft_entry__
 
     __graft_entry__.build()
-    on = _run(tmp_path, {}, "on")
-    off = _run(tmp_path, {"DECOMOE_PDL": "0"}, "off")
+    on = _run()
+    dm.decomoe_set_pdl(False)
+    try:
+        off = _run()
+    finally:
+        dm.decomoe_set_pdl(True)
     assert on.keys() == off.keys()
     for key in on:
         a, b = on[key], off[key]

@@ -239,6 +239,69 @@ def test_route_prefix_K_equals_k_takes_whole_prefix():
     assert all(sorted(r) == [0, 1, 2] for r in idx.tolist())
 
 
+# ---------------------------------------------------------------- prefix margin (near-tie rule)
+
+def test_prefix_margin_closed_forms():
+    # prefix [0, 5) sorted is 5, 4, 3, 2, 1: the gap between the 2nd and 3rd is
+    # 4 - 3; the 100 at index 5 lies outside the prefix and must be ignored
+    a = np.array([[5.0, 1.0, 3.0, 2.0, 4.0, 100.0, -7.0]])
+    assert O.prefix_margin(a, 5, 2)[0] == 1.0
+    assert O.prefix_margin(a, 5, 1)[0] == 1.0   # 5 - 4
+    assert O.prefix_margin(a, 5, 4)[0] == 1.0   # 2 - 1
+    assert O.prefix_margin(a, 7, 1)[0] == 95.0  # full span: 100 - 5
+    assert O.prefix_margin(a, 6, 2)[0] == 1.0   # 100, 5 | 4: 5 - 4
+    # an exact tie at the boundary gives 0; ties above it do not matter
+    t = np.array([[2.0, 1.0, 1.0, 0.0], [3.0, 3.0, 1.0, 0.0]])
+    np.testing.assert_array_equal(O.prefix_margin(t, 4, 2), [0.0, 2.0])
+    # K == k: the whole prefix is selected, nothing can swap in
+    assert np.isinf(O.prefix_margin(a, 3, 3)).all()
+    # one value per row is returned, in row order
+    assert O.prefix_margin(np.zeros((0, 6)), 4, 2).shape == (0,)
+
+
+def test_prefix_margin_bruteforce_best_subset():
+    # the margin is min over the best k-subset minus max over the rest of the
+    # prefix; the best subset comes from enumerating all k-subsets
+    for seed in range(40):
+        r = np.random.default_rng(500 + seed)
+        E = int(r.integers(3, 9))
+        K = int(r.integers(1, E + 1))
+        k = int(r.integers(1, K + 1))
+        row = r.standard_normal(E)
+        if seed % 5 == 0:
+            row = np.round(row * 2) / 2  # coarse grid: frequent exact ties
+        got = O.prefix_margin(row[None, :], K, k)[0]
+        if K == k:
+            assert np.isinf(got)
+            continue
+        pre = [float(v) for v in row[:K]]
+        best = max(itertools.combinations(range(K), k), key=lambda S: sum(pre[e] for e in S))
+        rest = [pre[e] for e in range(K) if e not in best]
+        assert got == min(pre[e] for e in best) - max(rest)
+        srt = sorted(pre)
+        assert got == srt[-k] - srt[-k - 1]
+
+
+def test_prefix_margin_decides_stability_of_the_routed_set():
+    # perturbing every prefix logit by less than half the margin leaves the
+    # prefix top-k set unchanged; moving the k-th down and the (k+1)-th up by
+    # a little more than half swaps them
+    for seed in range(30):
+        a = _logits(1, 16, 900 + seed).astype(np.float64)
+        K, k = 12, 4
+        m = O.prefix_margin(a, K, k)[0]
+        S = set(O.route_prefix(a, K, k)[0][0].tolist())
+        r = np.random.default_rng(seed)
+        noise = r.uniform(-0.49, 0.49, a.shape) * m
+        assert set(O.route_prefix(a + noise, K, k)[0][0].tolist()) == S
+        order = np.argsort(-a[0, :K], kind="stable")
+        b = a.copy()
+        b[0, order[k - 1]] -= 0.51 * m
+        b[0, order[k]] += 0.51 * m
+        S2 = set(O.route_prefix(b, K, k)[0][0].tolist())
+        assert S2 != S and int(order[k]) in S2 and int(order[k - 1]) not in S2
+
+
 # ---------------------------------------------------------------- dispatch
 
 def test_dispatch_is_stable_sort_by_expert():
