@@ -554,42 +554,60 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
     out += run_stack(dm, ws, pk)
     out += run_calib_gate(dm, ws, pk)
     # decode-size layers, K=64: weight streaming, reported against HBM
+    out += run_decode(dm, wl, layers, B, ws, pk, n)
+    return out
+
+
+def run_decode(dm, wl, layers, B, ws, pk, n):
+    """Decode-size layers (T in {1, 8, 32, 128} text tokens, K = 64): one
+    decomoe_moe_layer call per layer step (at most 32 tokens: the one-launch
+    decode layer). Bytes per step are the algorithmic ones of that step's
+    rotated layer (its own active experts D_l x 9.44 MB of weights, the router
+    rows, the activations), averaged over the rotated layers. Timed three
+    ways: eager calls, one CUDA graph per layer replayed one after another,
+    and the rotated layers captured back to back in one graph (as a decode
+    step runs its layers), reported per layer."""
+    out = []
+    K = 64
     for Td in W.DECODE_T:
         Bd = Buffers(wl, Td, B.out.device, dm)
         xs = [W.make_x(W.DECODE, T=Td, layer=l, device=B.out.device) for l in range(len(layers))]
 
-        class LV:
-            pass
-
-        def dec_step(i, ev, Td=Td, Bd=Bd, xs=xs):
+        def dec_call(i, Td=Td, Bd=Bd, xs=xs):
             L = layers[i % len(layers)]
-            lv = LV()
-            lv.x, lv.w_r, lv.bias, lv.w_gu, lv.w_down = xs[i % len(xs)], L.w_r, L.bias, L.w_gu, L.w_down
-            run_step(dm, wl, lv, Bd, 64, 0, 0, None, ev)
+            dm.decomoe_moe_layer(xs[i % len(xs)], L.w_r, L.bias, L.w_gu, L.w_down, wl.k, Bd.out, Bd.lws, K_fixed=K,
+                                 p=0.7, status=Bd.status)
 
-        ms, _ = timed(dec_step, n, 5, ws)
-        D = int((Bd.counts[:64] > 0).sum())
-        wbytes = D * 3 * wl.m * wl.d * 2
-        step_bytes = wbytes + wl.E * wl.d * 2 + Td * wl.d * 2 * (2 + 3 * wl.k)
-        # graph replay (no host launch gaps); events captured in each graph
-        # bracket its expert FFN
-        graphs = [dm.capture_graph(lambda i=i: dec_step(i, None)) for i in range(len(layers))]
+        c_off = dm.decomoe_moe_layer_workspace_layout(Td, wl.d, wl.E, wl.k, wl.m, dm.DECOMOE_BF16)[4]
+        Ds = []
+        for l in range(len(layers)):
+            dec_call(l)
+            torch.cuda.synchronize()
+            Ds.append(int((Bd.lws[c_off:c_off + 4 * K].view(torch.int32) > 0).sum()))
+        step_bytes = [D * 3 * wl.m * wl.d * 2 + wl.E * wl.d * 2 + Td * wl.d * 2 * (2 + 3 * wl.k) for D in Ds]
+        mean_bytes = statistics.mean(step_bytes)
+        ms, _ = timed(lambda i, ev: dec_call(i), n, 5, ws)
+        graphs = [dm.capture_graph(lambda i=i: dec_call(i)) for i in range(len(layers))]
         msg, _ = timed(lambda i, ev: graphs[i % len(graphs)].replay(), n, 5, ws)
-        gevs = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)] for _ in layers]
-        ev_graphs = [dm.capture_graph(lambda i=i: dec_step(i, gevs[i])) for i in range(len(layers))]
-        for _ in range(3):
-            for gr in ev_graphs:
-                gr.replay()
-        torch.cuda.synchronize()
-        ffn = statistics.mean(e[0].elapsed_time(e[1]) for e in gevs)
-        del ev_graphs
-        out.append({"mode": "decode", "T": Td, "K": 64, "active_experts": D,
+        del graphs
+        nl = len(layers)
+        g_all = dm.capture_graph(lambda: [dec_call(i) for i in range(nl)])
+        reps = max(5, n // nl)
+        msa, _ = timed(lambda i, ev: g_all.replay(), reps, 3, ws)
+        del g_all
+        per_layer = msa / (reps * nl)
+        if dm.decomoe_read_status(Bd.status) != 0:
+            raise RuntimeError("device status set during the decode run")
+        out.append({"mode": "decode", "T": Td, "K": K, "active_experts_per_layer": Ds,
+                    "algo_bytes_per_step_mean": round(mean_bytes),
                     "tokens_per_s": round(Td * n / (ms / 1e3), 1), "ms_per_step": round(ms / n, 4),
                     "graph_tokens_per_s": round(Td * n / (msg / 1e3), 1), "graph_ms_per_step": round(msg / n, 4),
-                    "graph_step_hbm_frac": round(step_bytes / (msg / n * 1e-3) / 1e9 / pk["hbm_gbs"], 4),
-                    "ffn_ms": round(ffn, 4),
-                    "ffn_hbm_frac": round(wbytes / (ffn * 1e-3) / 1e9 / pk["hbm_gbs"], 4)})
-        del Bd, xs, graphs
+                    "graph_step_hbm_frac": round(mean_bytes / (msg / n * 1e-3) / 1e9 / pk["hbm_gbs"], 4),
+                    "graph8_ms_per_layer": round(per_layer, 4),
+                    "graph8_tokens_per_s": round(Td / (per_layer * 1e-3), 1),
+                    "graph8_hbm_frac": round(mean_bytes / (per_layer * 1e-3) / 1e9 / pk["hbm_gbs"], 4),
+                    "path": "one launch per layer" if Td <= 32 else "router, routing + dispatch, expert FFN, combine"})
+        del Bd, xs
     return out
 
 
@@ -775,9 +793,15 @@ def only_decode(args, local):
 
     graphs = [dm.capture_graph(lambda i=i: dec_step(i)) for i in range(len(layers))]
     ms, _ = timed(lambda i, ev: graphs[i % len(graphs)].replay(), args.steps, args.warmup, 1)
+    del graphs
+    nl = len(layers)
+    g_all = dm.capture_graph(lambda: [dec_step(i) for i in range(nl)])
+    reps = max(5, args.steps // nl)
+    msa, _ = timed(lambda i, ev: g_all.replay(), reps, max(3, args.warmup // nl), 1)
     if dm.decomoe_read_status(Bd.status) != 0:
         raise RuntimeError("device status set during the decode run")
-    return {"mode": "decode only", "T": Td, "K": 64, "steps": args.steps, "ms_per_step": round(ms / args.steps, 4)}
+    return {"mode": "decode only", "T": Td, "K": 64, "steps": args.steps, "ms_per_step": round(ms / args.steps, 4),
+            "graph8_ms_per_layer": round(msa / (reps * nl), 4)}
 
 
 def _kernel_hash():

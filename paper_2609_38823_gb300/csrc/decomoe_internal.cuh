@@ -86,6 +86,11 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
 }
 
 // Internal entry points shared between translation units.
+// TMA map of a 2-D bf16 tensor [outer, inner] row-major; box = box_outer rows x
+// box_inner columns (64 -> 128-byte swizzle, 32 -> 64-byte swizzle), zero fill
+// out of bounds.
+int make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint32_t box_outer,
+                   uint32_t box_inner);
 int launch_router_tc(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E,
                      float* logits, int32_t* status, cudaStream_t s);
 bool router_tc_supported(int d, int E);
@@ -177,6 +182,17 @@ int launch_expert_ffn_fused(const void* x_perm, const int32_t* offsets, int64_t 
                             const void* w_gate_up, const void* w_down, void* h, void* y_perm, int32_t* ready,
                             int32_t* status, cudaStream_t s, bool* launched, const void* gather_x = nullptr,
                             const int32_t* perm = nullptr);
+// One launch for a whole decode-size layer (router, routing, dispatch,
+// experts, combine, and with text_out the visual-block removal of the
+// output; fixed or device-selected prefix). sync: decode_layer_sync_ints(T, d, E) int32 of the caller's
+// workspace, 8-byte aligned, any content (the launch clears what it uses).
+bool decode_layer_supported(int64_t T, int d, int E, int k, int m, int dtype, int K_fixed);
+size_t decode_layer_sync_ints(int64_t T, int d, int E);
+int launch_decode_layer(const void* x, const void* w_r, const float* bias, const void* w_gate_up, const void* w_down,
+                        int64_t T, int d, int E, int k, int m, int K_fixed, double p, const void* residual, void* out,
+                        void* text_out, int64_t v0, int64_t nv, float* logits, int32_t* topk_idx, float* topk_w, double* mass, int32_t* counts,
+                        int32_t* offsets, int32_t* perm, int32_t* inv, void* x_perm, void* h, void* y, int32_t* K_dev,
+                        int32_t* sync, int32_t* status, cudaStream_t s);
 // The k-split router's GEMM alone: KS slices of partial logits [KS][T][E]
 // (no bias) into scratch; returns KS (1: no split at this size, nothing
 // launched).
@@ -226,6 +242,19 @@ __device__ __forceinline__ void pdl_enter() {
 // Record the first error code in the caller's status word (if given).
 __device__ __forceinline__ void report_status(int32_t* status, int32_t code) {
   if (status != nullptr) atomicCAS(status, 0, code);
+}
+
+// Barrier over a subset of the block's warps (named barrier id, thread count).
+__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+// Order this thread's generic-proxy global writes before later async-proxy
+// (TMA) accesses of the same memory.
+__device__ __forceinline__ void fence_proxy_async_all() { asm volatile("fence.proxy.async;" ::: "memory"); }
+__device__ __forceinline__ int ld_acquire_gpu(const int32_t* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
 }
 
 // ---- cp.async (16-byte copies into shared memory, completion on an mbarrier)

@@ -54,7 +54,7 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 // 2-D bf16 tensor [outer, inner] row-major; box = box_outer rows x box_inner
 // columns (64 -> 128-byte swizzle, 32 -> 64-byte swizzle), zero fill out of
 // bounds.
-static int make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
+int make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
                           uint32_t box_outer, uint32_t box_inner) {
   auto fn = encode_fn();
   if (fn == nullptr) {
@@ -762,9 +762,6 @@ __device__ __forceinline__ WsTile ws_tile(int t, int total, const int* s_tt, con
   return r;
 }
 
-__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
-}
 
 template <bool SWIGLU, int STAGES, bool GATHER_B = false, int BN = 256>
 __global__ void __launch_bounds__(192, 1)
@@ -1112,12 +1109,6 @@ constexpr int ffn_ws_max_stages() {
   return n > 12 ? 12 : n;
 }
 
-__device__ __forceinline__ void fence_proxy_async_all() { asm volatile("fence.proxy.async;" ::: "memory"); }
-__device__ __forceinline__ int ld_acquire_gpu(const int32_t* p) {
-  int v;
-  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
 
 template <int STAGES, int BN>
 __global__ void __launch_bounds__(192, 1)

@@ -25,6 +25,7 @@ enum {
   WS_SCHED,
   WS_RSPLIT,
   WS_SYNC,
+  WS_DSYNC,
   WS_STATUS_PAD,
   WS_COUNT
 };
@@ -179,6 +180,7 @@ static LayerLayout layer_layout(int64_t T, int d, int E, int k, int m, int dtype
   sz[WS_SCHED] = 16;
   sz[WS_RSPLIT] = decomoe_router_logits_ws_bytes(T, d, E);
   sz[WS_SYNC] = expert_ffn_sync_ints(static_cast<int64_t>(T) * k, E) * 4;  // counters of the fused expert launch
+  sz[WS_DSYNC] = decode_layer_sync_ints(T, d, E) * 4;  // counters of the one-launch decode layer
   sz[WS_STATUS_PAD] = 256;
   size_t o = 0;
   for (int i = 0; i < WS_COUNT; ++i) {
@@ -328,6 +330,16 @@ int moe_layer_impl(const void* x, const void* w_r, const float* bias, const void
   // by the first routing launch of this call
   int32_t* sync = reinterpret_cast<int32_t*>(base + L.off[WS_SYNC]);
   const int n_sync = static_cast<int>(expert_ffn_sync_ints(T * k, E));
+  // Decode sizes: the whole layer as one launch (router, routing, dispatch,
+  // experts and combine; its counters in their own workspace slot).
+  if (decode_layer_supported(T, d, E, k, m, dtype, K_fixed)) {
+    if (K_used_host) *K_used_host = K_fixed;
+    if (K_sel_host && K_fixed == -1) *K_sel_host = -1;
+    return launch_decode_layer(x, w_r, bias, w_gate_up, w_down, T, d, E, k, m, K_fixed, p, residual, out, text_out,
+                               v0, nv, logits,
+                               topk_idx, topk_w, mass, counts, offsets, perm, inv, x_perm, h, y_perm, K_dev,
+                               reinterpret_cast<int32_t*>(base + L.off[WS_DSYNC]), status_dev, s);
+  }
   // Where the experts take the one-launch tokens-as-M form on at least
   // gather_min_rows routed rows, that launch copies the
   // dispatched rows itself (per M-tile, while its accumulators fill) and the

@@ -5,6 +5,7 @@
 #include <cstdint>
 
 #include "dispatch_tile.cuh"
+#include "route_common.cuh"
 
 namespace decomoe {
 
@@ -48,21 +49,6 @@ static constexpr int64_t router_gemv_max_t() { return DECOMOE_ROUTER_GEMV_MAX_T;
 // SM at decode sizes) instead of piling every row of a block onto one SM; all
 // of a thread's loads are issued before its first multiply. Partial dots are
 // reduced by warp shuffles, then over the four warps in a fixed order.
-constexpr int GEMV_THREADS = 128;
-constexpr int GEMV_TPB = 8;  // tokens per block
-constexpr int GEMV_VPT = 2;  // vectors per thread per pass (d = 2048: one pass)
-__device__ __forceinline__ float dot8_bf16(const uint4 a, const uint4 b, float acc) {
-  acc = fmaf(bf16_lo(a.x), bf16_lo(b.x), acc);
-  acc = fmaf(bf16_hi(a.x), bf16_hi(b.x), acc);
-  acc = fmaf(bf16_lo(a.y), bf16_lo(b.y), acc);
-  acc = fmaf(bf16_hi(a.y), bf16_hi(b.y), acc);
-  acc = fmaf(bf16_lo(a.z), bf16_lo(b.z), acc);
-  acc = fmaf(bf16_hi(a.z), bf16_hi(b.z), acc);
-  acc = fmaf(bf16_lo(a.w), bf16_lo(b.w), acc);
-  acc = fmaf(bf16_hi(a.w), bf16_hi(b.w), acc);
-  return acc;
-}
-
 __global__ void __launch_bounds__(GEMV_THREADS)
     k_router_gemv(const uint4* __restrict__ x, const uint4* __restrict__ w_r, const float* __restrict__ bias,
                   int64_t Tn, int vpr, int E, float* __restrict__ logits) {
@@ -123,62 +109,6 @@ __global__ void __launch_bounds__(GEMV_THREADS)
 // the blocks in a fixed order in fp64, so the mass is bit-reproducible.
 constexpr int ROUTE_THREADS = 256;
 constexpr int ROUTE_TPB = ROUTE_TOKENS_PER_BLOCK;  // tokens per block: one per warp
-
-// Order-preserving 32-bit key of a float (larger float -> larger key; -0 and
-// +0 share a key so equal values tie). Key 0 is below every float's key and
-// marks entries that are out of range or already picked.
-__device__ __forceinline__ uint32_t fkey(float f) {
-  const uint32_t u = (f == 0.0f) ? 0u : __float_as_uint(f);
-  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-}
-__device__ __forceinline__ float fkey_inv(uint32_t k) {
-  return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
-}
-
-// k rounds of warp arg-max over entries e < lim: each round one redux.sync
-// max over the lanes' best keys, then one redux.sync min over the indices of
-// the lanes holding that key (lower index wins a tie). Pick j ends in lane j.
-__device__ __forceinline__ void warp_topk(const uint32_t (&key_in)[8], int lim, int k, int lane, float& my_v,
-                                          int& my_i) {
-  uint32_t key[8];
-#pragma unroll
-  for (int i = 0; i < 8; ++i) key[i] = (lane + 32 * i < lim) ? key_in[i] : 0u;
-  my_v = 0.f;
-  my_i = 0;
-  for (int j = 0; j < k; ++j) {
-    uint32_t bk = 0;
-    int bs = 0;  // slot of the lane's best (entries ascend with the slot, so strict > keeps the lowest index)
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-      if (key[i] > bk) {
-        bk = key[i];
-        bs = i;
-      }
-    const uint32_t mk = __reduce_max_sync(0xffffffffu, bk);
-    const uint32_t cand = (bk == mk) ? static_cast<uint32_t>(lane + 32 * bs) : 0xffffffffu;
-    const uint32_t wi = __reduce_min_sync(0xffffffffu, cand);
-    {
-      const bool mine = (wi & 31u) == static_cast<uint32_t>(lane);
-      const int sl = static_cast<int>(wi >> 5);
-#pragma unroll
-      for (int i = 0; i < 8; ++i) key[i] = (mine && i == sl) ? 0u : key[i];  // selects keep key[] in registers
-    }
-    if (lane == j) {
-      my_v = fkey_inv(mk);
-      my_i = static_cast<int>(wi);
-    }
-  }
-}
-
-// Renormalised weight of this lane's pick (lanes >= k get 0).
-__device__ __forceinline__ float pick_weight(float my_v, int lane, int k) {
-  const float v0 = __shfl_sync(0xffffffffu, my_v, 0);
-  const float z = (lane < k) ? __expf(my_v - v0) : 0.f;
-  float zs = z;
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) zs += __shfl_xor_sync(0xffffffffu, zs, off);
-  return z / zs;
-}
 
 // NP: 1 reads plain logit rows; NP > 1 reads NP k slices of the split
 // router (src), each warp loading its row's slices as coalesced 16-byte
@@ -299,31 +229,6 @@ __global__ void __launch_bounds__(256)
     k_mass_finalize(const double* __restrict__ part, int nblocks, int E, double* __restrict__ mass) {
   pdl_enter();
   mass_finalize_block(part, nblocks, E, static_cast<int>(blockIdx.x), mass);
-}
-
-// Eq. 12, sequentially in fp64 with round-to-nearest adds and division, as
-// the host decomoe_select_prefix does: K_hat = smallest K whose prefix mass
-// ratio reaches p (E when p >= 1 or none does), K = max(k, K_hat); k when the
-// total mass is zero.
-__device__ int select_prefix_seq(const double* mass, int E, int k, double p) {
-  double tot = 0.0;
-  for (int e = 0; e < E; ++e) tot = __dadd_rn(tot, mass[e]);
-  int K = k;
-  if (tot > 0.0) {
-    int K_hat = E;
-    if (p < 1.0) {
-      double acc = 0.0;
-      for (int Kc = 1; Kc <= E; ++Kc) {
-        acc = __dadd_rn(acc, mass[Kc - 1]);
-        if (__ddiv_rn(acc, tot) >= p) {
-          K_hat = Kc;
-          break;
-        }
-      }
-    }
-    K = K_hat > k ? K_hat : k;
-  }
-  return K;
 }
 
 // Eq. 12 on the device, one thread (bit-identical to decomoe_select_prefix).

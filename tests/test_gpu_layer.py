@@ -17,8 +17,7 @@ import paper_2609_38823_gb300 as dm
 import workloads as W
 from oracle import decomoe_oracle as O
 from tests.helpers import (BF16_MAX_ABS, BF16_REL_L2, F32_MAX_ABS, F32_REL_L2, MASS_P_BAND, MASS_REL, W_ABS,
-                           assert_close_out, f64,
-                           logit_error_bound)
+                           Experts, check_layer_tokens, f64)
 
 pytestmark = pytest.mark.gpu
 DEV = torch.device("cuda")
@@ -68,61 +67,13 @@ def _run_layer(g, k, T, K_fixed=0, p=0.0, residual=None):
 
 
 def _compare(g_cpu, out, logits, idx, w, K, k, sample, tol, residual=None):
-    """Compare the layer's routing and output with the oracle on the sampled
-    tokens. A token whose oracle prefix margin exceeds twice its own largest
-    logit error bound must get the oracle's experts exactly. For the others
-    (near-ties) several expert sets are correct: the GPU's set must be one
-    that some logits within the bounds rank first, and its weights and output
-    are compared with the oracle evaluated on that set. Returns the number of
-    near-tie tokens."""
-    x64 = f64(g_cpu["x"][sample])
-    wr64 = f64(g_cpu["w_r"])
-    b64 = g_cpu["bias"].numpy().astype(np.float64)
-    ref_logits = O.router_logits(x64, wr64, b64).astype(np.float64)
-    bound = logit_error_bound(x64, wr64, b64)
-    err = np.abs(f64(logits[sample]) - ref_logits)
-    assert (err <= bound).all(), f"logit error {err.max():.3e} above bound"
-    keep = O.prefix_margin(ref_logits, K, k) > 2.0 * bound[:, :K].max(axis=1)
-    n = len(sample)
-    n_tie = int((~keep).sum())
-    print(f"[layer parity] K={K}: {n_tie} of {n} sampled tokens near a tie (compared on the GPU's valid set)")
-    assert n_tie <= max(0.1 * n, 4), f"{n_tie} of {n} tokens near a tie: the logit bound is too loose"
-    ref = O.moe_layer(x64, wr64, b64, ExpertView(g_cpu["w_gate"]), ExpertView(g_cpu["w_up"]),
-                      ExpertView(g_cpu["w_down"]), k=k, K=K,
-                      residual=None if residual is None else f64(residual[sample]))
-    gi = idx[sample]
-    ref_w = np.array(ref["w"])
-    ref_out = np.array(ref["out"])
-    # the expert set is unique on the kept tokens; the slot order inside it
-    # is unique where every gap between consecutive prefix logits down to the
-    # (k+1)-th exceeds twice the token's bound
-    srt = -np.sort(-ref_logits[:, :K], axis=-1)[:, :min(k + 1, K)]
-    ordered = keep & (np.diff(-srt, axis=-1).min(axis=-1, initial=np.inf) > 2.0 * bound[:, :K].max(axis=1))
-    assert np.array_equal(gi[ordered], ref["idx"][ordered])
-    assert np.array_equal(np.sort(gi[keep], -1), np.sort(ref["idx"][keep], -1))
-    wg, wu, wd = ExpertView(g_cpu["w_gate"]), ExpertView(g_cpu["w_up"]), ExpertView(g_cpu["w_down"])
-    for i in range(n):
-        S = [int(e) for e in gi[i]]
-        assert len(set(S)) == k and all(0 <= e < K for e in S)
-        a, b = ref_logits[i, :K], bound[i, :K]
-        # slot order: descending logits up to the bounds
-        assert all(a[S[j]] + b[S[j]] >= a[S[j + 1]] - b[S[j + 1]] for j in range(k - 1)), f"token {i}: slot order"
-        if keep[i]:
-            pos = {int(e): j for j, e in enumerate(ref["idx"][i])}
-            ref_w[i] = [ref["w"][i][pos[e]] for e in S]
-            continue
-        rest = [e for e in range(K) if e not in S]
-        assert min(a[S] + b[S]) >= max(a[rest] - b[rest]), f"token {i}: GPU experts {S} are not a valid top-{k}"
-        a_S = ref_logits[i].copy()
-        a_S[rest] = -1e30  # the oracle evaluated on the GPU's set
-        o_i, idx_i, w_i = O.moe_token(x64[i], a_S, wg, wu, wd, K, k)
-        assert sorted(idx_i.tolist()) == sorted(S)
-        pos = {int(e): j for j, e in enumerate(idx_i)}
-        ref_w[i] = [w_i[pos[e]] for e in S]
-        ref_out[i] = o_i + (0.0 if residual is None else f64(residual[sample])[i])
-    assert np.abs(w[sample] - ref_w).max() <= 2e-5
-    assert_close_out(f64(out[sample]), ref_out, tol[0], tol[1], "layer output")
-    return n_tie
+    """The sampled tokens' routing and output against the oracle (rule in
+    tests.helpers.check_layer_tokens). Returns the near-tie count."""
+    return check_layer_tokens(f64(g_cpu["x"][sample]), f64(g_cpu["w_r"]), g_cpu["bias"].numpy().astype(np.float64),
+                              Experts(g_cpu["w_gate"]), Experts(g_cpu["w_up"]), Experts(g_cpu["w_down"]),
+                              f64(logits[sample]), idx[sample], w[sample], f64(out[sample]), K, k,
+                              residual64=None if residual is None else f64(residual[sample]), tol=tol,
+                              label="layer parity")
 
 
 # ----------------------------------------------------------------- tiny fp32 layer (all tokens)
