@@ -551,6 +551,7 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
                 "tokens_per_s": round(T * n / (ms / 1e3), 1), "ms_per_step": round(ms / n, 4)})
     del graphs
     out += run_large(dm, ws, pk, n)
+    out += run_large_stack(dm, ws, pk)
     out += run_stack(dm, ws, pk)
     out += run_calib_gate(dm, ws, pk)
     # decode-size layers, K=64: weight streaming, reported against HBM
@@ -560,7 +561,7 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
 
 def run_decode(dm, wl, layers, B, ws, pk, n):
     """Decode-size layers (T in {1, 8, 32, 128} text tokens, K = 64): one
-    decomoe_moe_layer call per layer step (at most 32 tokens: the one-launch
+    decomoe_moe_layer call per layer step (2 to 32 tokens: the one-launch
     decode layer). Bytes per step are the algorithmic ones of that step's
     rotated layer (its own active experts D_l x 9.44 MB of weights, the router
     rows, the activations), averaged over the rotated layers. Timed three
@@ -606,7 +607,8 @@ def run_decode(dm, wl, layers, B, ws, pk, n):
                     "graph8_ms_per_layer": round(per_layer, 4),
                     "graph8_tokens_per_s": round(Td / (per_layer * 1e-3), 1),
                     "graph8_hbm_frac": round(mean_bytes / (per_layer * 1e-3) / 1e9 / pk["hbm_gbs"], 4),
-                    "path": "one launch per layer" if Td <= 32 else "router, routing + dispatch, expert FFN, combine"})
+                    "path": ("one launch per layer" if 2 <= Td <= 32 else
+                             "router, routing + dispatch, expert FFN, combine (separate launches)")})
         del Bd, xs
     return out
 
@@ -666,6 +668,59 @@ def run_large(dm, ws, pk, n):
             del gr, gr2, Bl
         del g, w_gu, lws
     del kv, kv_out
+    torch.cuda.empty_cache()
+    return out
+
+
+def run_large_stack(dm, ws, pk):
+    """The large workload as a 48-layer pass: T = 16384 rows (14336 visual +
+    2048 text); layers 0..11 run the full pool (K = 128) on all rows; at layer
+    12 the visual block leaves the hidden state and both 48-layer KV caches
+    (2 x 48 x 16384 x 512 bf16 in); layers 12..47 run on the 2048 text rows at
+    K = ceil(f * 128). Attention is not part of the path (RMSNorm, then MoE
+    plus residual). One graph replay per (Zipf exponent, prefix fraction);
+    useful FLOPs are 6 k d m per routed token and layer plus the router."""
+    from paper_2609_38823_gb300.stack import Stack, StackLayer
+
+    base = W.LARGE
+    dev = torch.device("cuda")
+    torch.cuda.empty_cache()
+    weights = []
+    for l in range(base.layers):
+        g = W.make_layer(base, layer=l, device=dev, with_x=False)
+        weights.append((g["w_r"], dm.fuse_gate_up(g["w_gate"], g["w_up"]), g["w_down"]))
+        del g
+    h0 = W.make_x(base, device=dev)
+    kv = [W.make_kv(base, device=dev, seed=s) for s in (0, 1)]
+    kv_out = [torch.empty(base.layers, base.T - base.nv, base.kv_width, dtype=torch.bfloat16, device=dev)
+              for _ in range(2)]
+    Tt = base.T - base.nv
+    out = []
+    for zipf in W.LARGE_ZIPF:
+        bias = W._bias(W.with_(base, zipf_s=zipf)).to(dev)
+        layers = [StackLayer(w_r, bias, w_gu, w_d) for (w_r, w_gu, w_d) in weights]
+        for f in W.LARGE_FRACTIONS:
+            K = W.large_K(f)
+            K_sched = [base.E] * base.exit_layer + [K] * (base.layers - base.exit_layer)
+            st = Stack(layers, K_sched, base.k, base.exit_layer, base.v0, base.nv, base.T)
+            gr = dm.capture_graph(lambda st=st: st.forward(h0, kv, kv_out))
+            nn = 5
+            ms, _ = timed(lambda i, ev: gr.replay(), nn, 2, ws)
+            if dm.decomoe_read_status(st.status) != 0:
+                raise RuntimeError("device status set during the 48-layer pass")
+            ms_pass = ms / nn
+            fl = sum((6.0 * base.k * base.d * base.m + 2.0 * base.d * base.E) * (base.T if l < base.exit_layer else Tt)
+                     for l in range(base.layers))
+            out.append({"mode": "stack48 T=16384", "zipf_s": zipf, "K_after_exit": K, "fraction": f,
+                        "exit_layer": base.exit_layer, "pass_ms": round(ms_pass, 3),
+                        "tokens_per_s": round(base.T / (ms_pass * 1e-3), 1),
+                        "useful_tflops": round(fl / (ms_pass * 1e-3) / 1e12, 1),
+                        "useful_tflop_per_pass": round(fl / 1e12, 2),
+                        "tensor_frac": round(fl / (ms_pass * 1e-3) / 1e12 / pk["bf16_tflops"], 4),
+                        "includes": "12 full-sequence layers, hidden + 2x48-layer KV compaction, 36 text-only "
+                                    "layers (RMSNorm, MoE, residual)"})
+            del gr, st
+    del weights, kv, kv_out, h0
     torch.cuda.empty_cache()
     return out
 

@@ -98,12 +98,16 @@ class Stack:
         return dst
 
     def forward(self, h0: torch.Tensor, kv: Optional[List[torch.Tensor]] = None,
-                kv_out: Optional[List[torch.Tensor]] = None) -> torch.Tensor:
+                kv_out: Optional[List[torch.Tensor]] = None, trace=None) -> torch.Tensor:
         """Run every layer on h0 [T, d]; returns the final hidden state (text
         rows only once the visual block has left). kv: K and V caches
         [L, T, w]; kv_out: their compacted destinations [L, T - nv, w]. With a
         gate, each candidate layer's decision is read back to the host (one
-        4-byte copy) because the exit changes the shapes of later launches."""
+        4-byte copy) because the exit changes the shapes of later launches.
+        trace, if given, is called after each layer's launches are queued as
+        trace(l, layer_input, normed_input, layer_output, workspace), so a
+        caller can inspect any layer's inputs and results (the buffers are
+        reused by later layers)."""
         cur = self.hf[0]
         cur.copy_(h0)
         bufs, xn, nxt = self.hf, self.xn_f, 1
@@ -123,6 +127,8 @@ class Stack:
             else:
                 decomoe_moe_layer(xn, Lw.w_r, Lw.bias, Lw.w_gate_up, Lw.w_down, self.k, out, self.ws,
                                   K_fixed=self.K[l], p=0.0, residual=cur, status=self.status)
+            if trace is not None:
+                trace(l, cur, xn, out, self.ws)
             cur, nxt = out, 1 - nxt
             if self.gate is not None and not exited and l in self.gate.params and l + 1 < len(self.layers):
                 w1, b1, w2, b2 = self.gate.params[l]

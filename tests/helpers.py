@@ -71,7 +71,7 @@ class Experts:
     def __getitem__(self, e):
         e = int(e)
         if e not in self.cache:
-            self.cache[e] = self.t[e].double().cpu().numpy()
+            self.cache[e] = self.t[e].cpu().double().numpy()
         return self.cache[e]
 
 

@@ -15,7 +15,7 @@ import paper_2609_38823_gb300 as dm
 import workloads as W
 from oracle import decomoe_oracle as O
 from paper_2609_38823_gb300.stack import Stack, StackLayer
-from tests.helpers import MASS_P_BAND, assert_close_out, bf16_round, f64
+from tests.helpers import MASS_P_BAND, Experts, assert_close_out, bf16_round, check_layer_tokens, f64
 
 pytestmark = pytest.mark.gpu
 DEV = torch.device("cuda")
@@ -87,38 +87,66 @@ def stack48():
     return wl, L, R
 
 
-def test_stack48_exit_layer_compaction_and_window_parity(stack48):
-    """Full 48-layer stack at its real size: finite text-only output, KV
-    compaction bit-exact, and sampled tokens followed by the oracle through a
-    three-layer window around the exit layer (19, 20, 21), where the bf16
-    drift of the hidden state stays within the output tolerance."""
+def test_stack48_teacher_forced_every_layer(stack48):
+    """The 48-layer stack at its real size (1552 rows, exit at layer 20,
+    K_l drawn from 32..96 after it): every layer is checked against the
+    oracle from the GPU's own bf16 input to that layer (teacher forcing: bf16
+    drift over 48 layers would otherwise flip near-tie routing), on 16
+    sampled text tokens (4 system rows, 12 trailing text rows) followed
+    through all 48 layers, plus the KV compaction bit-exact. The RMSNorm
+    output is compared with the oracle's on the same layer input. The
+    end-to-end relative L2 of the oracle's own trajectory is printed, not
+    gated."""
     wl, L, R = stack48
+    d, E, k, m = wl.d, wl.E, wl.k, wl.m
     K_sched = W.stack_K_schedule(wl)
     assert K_sched[:20] == [128] * 20 and all(32 <= v <= 96 for v in K_sched[20:])
     h0 = W.make_x(wl, device="cuda")
     kv = [W.make_kv(wl, device="cuda", seed=s) for s in (0, 1)]
     kv_out = [torch.empty(wl.layers, wl.T - wl.nv, wl.kv_width, dtype=torch.bfloat16, device=DEV) for _ in range(2)]
-    st = Stack(L, K_sched, wl.k, exit_layer=wl.exit_layer, v0=wl.v0, nv=wl.nv, T=wl.T)
-    out = st.forward(h0, kv, kv_out)
+    r = np.random.default_rng(7)
+    rows = sorted(r.choice(wl.v0, 4, replace=False).tolist() +
+                  r.choice(np.arange(wl.v0 + wl.nv, wl.T), 12, replace=False).tolist())
+    rows_after = [t if t < wl.v0 else t - wl.nv for t in rows]
+    rec = {}
+
+    def trace(l, cur, xn, out, ws):
+        Tc = cur.shape[0]
+        idx = torch.tensor(rows if Tc == wl.T else rows_after, device=DEV)
+        o = dm.decomoe_moe_layer_workspace_layout(Tc, d, E, k, m, dm.DECOMOE_BF16)
+        lg = ws[o[0]:o[0] + Tc * E * 4].view(torch.float32).view(Tc, E)
+        ti = ws[o[1]:o[1] + Tc * k * 4].view(torch.int32).view(Tc, k)
+        tw = ws[o[2]:o[2] + Tc * k * 4].view(torch.float32).view(Tc, k)
+        rec[l] = tuple(t[idx].cpu() for t in (cur, xn, out, lg, ti, tw))
+
+    st = Stack(L, K_sched, k, exit_layer=wl.exit_layer, v0=wl.v0, nv=wl.nv, T=wl.T)
+    out = st.forward(h0, kv, kv_out, trace=trace)
     torch.cuda.synchronize()
     assert dm.decomoe_read_status(st.status) == 0
-    assert out.shape == (wl.T - wl.nv, wl.d) and torch.isfinite(out.float()).all()
+    assert out.shape == (wl.T - wl.nv, d) and torch.isfinite(out.float()).all()
     for src, dst in zip(kv, kv_out):
         for l in (0, 19, 20, 47):
             ref = O.drop_visual_block(src[l].view(torch.int16).cpu().numpy(), wl.v0, wl.nv)
             assert np.array_equal(dst[l].view(torch.int16).cpu().numpy(), ref)
-    # window around the exit: layers 19 (full sequence), 20 and 21 (text only)
-    win = Stack(L[19:22], K_sched[19:22], wl.k, exit_layer=1, v0=wl.v0, nv=wl.nv, T=wl.T)
-    hw = win.forward(h0)
-    torch.cuda.synchronize()
-    text = [t for t in range(wl.T) if not (wl.v0 <= t < wl.v0 + wl.nv)]
-    r = np.random.default_rng(7)
-    pick = np.sort(r.choice(len(text), 12, replace=False))
-    rows = [text[i] for i in pick]
-    ref, margins = _trajectories(f64(h0), R[19:22], K_sched[19:22], wl.k, rows, bf16_round)
-    keep = margins > 2e-2
-    assert keep.sum() >= 3, f"only {keep.sum()} sampled tokens clear of near-ties"
-    assert_close_out(f64(hw)[pick][keep], ref[keep], 5e-3, 2e-2, "stack window output")
+    assert sorted(rec) == list(range(wl.layers))
+    h_ref = f64(h0[torch.tensor(rows, device=DEV)])
+    ties = 0
+    for l in range(wl.layers):
+        cur, xn, o, lg, ti, tw = rec[l]
+        wg, wu, wd = Experts(R[l]["w_gate"].t), Experts(R[l]["w_up"].t), Experts(R[l]["w_down"].t)
+        wr64, b64 = R[l]["w_r"], R[l]["bias"].astype(np.float64)
+        # RMSNorm of the layer input (stored in bf16)
+        assert_close_out(f64(xn), O.rmsnorm(f64(cur)), 5e-3, 2e-2, f"layer {l} rmsnorm")
+        # the layer from the GPU's own normed input, residual = its input
+        ties += check_layer_tokens(f64(xn), wr64, b64, wg, wu, wd, f64(lg), ti.numpy(), tw.numpy(), f64(o),
+                                   K_sched[l], k, residual64=f64(cur), label=f"stack layer {l}")
+        # the oracle's own trajectory (bf16 storage between layers), reported
+        xr = bf16_round(O.rmsnorm(h_ref))
+        h_ref = bf16_round(h_ref + O.moe_layer(xr, wr64, b64, wg, wu, wd, k=k, K=K_sched[l])["out"])
+    got = f64(out[torch.tensor(rows_after, device=DEV)])
+    rel = np.linalg.norm(got - h_ref) / np.linalg.norm(h_ref)
+    print(f"[stack48] {ties} near-tie token-layers of {16 * wl.layers}; end-to-end rel-L2 of the oracle's own "
+          f"trajectory vs the GPU output after 48 layers: {rel:.3e} (reported, not gated)")
 
 
 @pytest.mark.parametrize("K,zipf", [(39, 1.2), (128, 0.8)])
