@@ -53,6 +53,8 @@ def parse():
     ap.add_argument("--only-decode", type=int, default=0, metavar="T",
                     help="run only the decode layer at T tokens (K=64) for --steps graph replays (profiling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--only-isolated", default="", metavar="NAME",
+                    help="time one isolated memory-bound kernel (compaction, gather, combine, permute) and exit")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     return ap.parse_args()
 
@@ -232,13 +234,20 @@ def run_step(dm, wl, L, B, K, v0, nv, text, ev=None):
                              status=B.status, text_out=text, v0=v0, nv=nv)
         return
     # a1 + a2 (Eq. 11) + a4 + a5: router logits, routing with the activated
-    # mass, dispatch
+    # mass, dispatch (from 8192 routed rows the layer leaves the row gather to
+    # the expert launch, and so does this)
+    gather = L.x.shape[0] * k >= 8192
     dm.decomoe_router_route_dispatch(L.x, L.w_r, L.bias, B.logits, K, k, B.idx, B.w, B.counts[:K], B.offsets[:K + 1],
-                                     B.perm, B.inv, B.x_perm, B.rrd_ws, mass_out=B.mass, status=B.status)
+                                     B.perm, B.inv, None if gather else B.x_perm, B.rrd_ws, mass_out=B.mass,
+                                     status=B.status)
     B.ready.zero_()
     ev[0].record()
-    dm.decomoe_expert_swiglu_fused(B.x_perm, B.offsets[:K + 1], K, L.w_gu, L.w_down, B.h, B.y, B.ready,
-                                   B.status)  # a6
+    if gather:
+        dm.decomoe_expert_swiglu_fused_gather(L.x, B.perm, B.offsets[:K + 1], K, L.w_gu, L.w_down, B.x_perm, B.h,
+                                              B.y, B.ready, B.status)  # a6 with the row gather
+    else:
+        dm.decomoe_expert_swiglu_fused(B.x_perm, B.offsets[:K + 1], K, L.w_gu, L.w_down, B.h, B.y, B.ready,
+                                       B.status)  # a6
     ev[1].record()
     if text is not None:
         # a7 + a8: combine, the text rows also stored to the compacted buffer
@@ -271,13 +280,17 @@ def timed(fn, steps, warmup, ws, clocks=None, name="sweep"):
     return ms, evs
 
 
-def algo_bytes_ffn(wl, R, D):
+def algo_bytes_ffn(wl, R, D, T=None):
     """Expert FFN as one launch: the gate/up and down weights of the D active
-    experts, the R dispatched rows read, h written once (an output of the
-    call) and y written. The read of h back by the down tiles is not counted:
-    in the one-launch form it follows the write within microseconds and is
-    served from L2."""
-    return D * 3 * wl.m * wl.d * 2 + R * wl.d * 2 + R * wl.m * 2 + R * wl.d * 2
+    experts, the activations read once (the R dispatched rows, or with the
+    row gather in the launch the T token rows x, each read once), h written
+    once (an output of the call) and y written. The read of h back by the
+    down tiles is not counted: in the one-launch form it follows the write
+    within microseconds and is served from L2. With the row gather the launch
+    also writes the gathered rows to its x_perm scratch: that is not
+    algorithmic traffic (the DRAM counters show it)."""
+    act = (T if T is not None else R) * wl.d * 2
+    return D * 3 * wl.m * wl.d * 2 + act + R * wl.m * 2 + R * wl.d * 2
 
 
 def ours(args, ws, rank, local):
@@ -372,7 +385,7 @@ def ours(args, ws, rank, local):
     D = statistics.mean(Ds)
     ffn_flops = 6.0 * R * wl.d * wl.m
     useful_flops = ffn_flops + 2.0 * T * wl.d * wl.E
-    ffn_bytes = algo_bytes_ffn(wl, R, D)
+    ffn_bytes = algo_bytes_ffn(wl, R, D, T if R >= 8192 else None)
     ffn_tflops = ffn_flops / (ffn_ms * 1e-3) / 1e12
     ffn_gbs = ffn_bytes / (ffn_ms * 1e-3) / 1e9
     t_compute = ffn_flops / (pk["bf16_tflops"] * 1e12)
@@ -382,7 +395,7 @@ def ours(args, ws, rank, local):
     prof = os.path.join(ROOT, "profiles", "traffic.json")
     if os.path.exists(prof):
         try:
-            tr = json.load(open(prof)).get(f"expert_ffn_K{K}")
+            tr = json.load(open(prof)).get(f"expert_ffn_gather_K{K}")
             if tr and tr.get("source_hash") == _kernel_hash():
                 traffic = tr["bytes_per_launch"]
         except Exception:
@@ -393,7 +406,8 @@ def ours(args, ws, rank, local):
     else:
         roof = {"bound": "hbm", "achieved": round(ffn_gbs, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
                 "frac": round(ffn_gbs / pk["hbm_gbs"], 4), "traffic": traffic}
-    roof.update({"kernel": "k_ffn_tc (expert gate/up + SwiGLU + down in one persistent launch)",
+    roof.update({"kernel": "k_ffn_tc as the layer launches it (row gather, gate/up + SwiGLU, down in one "
+                           "persistent launch)",
                  "peak_source": f"{pk['source']} burst", "ms_per_launch": round(ffn_ms, 4),
                  "flops_per_launch": ffn_flops, "algo_bytes_per_launch": ffn_bytes,
                  "tensor_frac": round(ffn_tflops / pk["bf16_tflops"], 4),
@@ -521,7 +535,7 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
         ffn = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
         D = int((B.counts[:K] > 0).sum())
         ffn_fl = 6.0 * R * wl.d * wl.m
-        ffn_by = algo_bytes_ffn(wl, R, D)
+        ffn_by = algo_bytes_ffn(wl, R, D, T if R >= 8192 else None)
         out.append({"mode": "fixed (eager launches)", "K": K, "tokens_per_s": round(T * n / (ms / 1e3), 1),
                     "ms_per_step": round(ms / n, 4), "ffn_ms": round(ffn, 4),
                     "ffn_tflops": round(ffn_fl / (ffn * 1e-3) / 1e12, 2),
@@ -550,6 +564,7 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
     out.append({"mode": f"mass p={args.p}, device-selected K (graph replay)",
                 "tokens_per_s": round(T * n / (ms / 1e3), 1), "ms_per_step": round(ms / n, 4)})
     del graphs
+    out += run_isolated(dm, ws, pk)
     out += run_large(dm, ws, pk, n)
     out += run_large_stack(dm, ws, pk)
     out += run_stack(dm, ws, pk)
@@ -668,6 +683,102 @@ def run_large(dm, ws, pk, n):
             del gr, gr2, Bl
         del g, w_gu, lws
     del kv, kv_out
+    torch.cuda.empty_cache()
+    return out
+
+
+ISOLATED = ("compaction", "gather", "combine", "permute")
+
+
+def run_isolated(dm, ws, pk, only=None, steps=10, warmup=3):
+    """The memory-bound steps alone, each timed with CUDA events (L2 flushed
+    before every repetition, median reported) and reported as GB/s of
+    algorithmic bytes against the measured HBM copy peak:
+      compaction: the visual block (14336 of 16384 rows) removed from both
+        48-layer KV caches [48, 16384, 512] bf16 (reads and writes the 2048
+        kept rows of every layer slice);
+      gather: the dispatch's row copy at T=2048, k=8, K=64 (x read once,
+        16384 rows of x_perm written; the routing launches are outside the
+        events);
+      combine: T=2048, k=8 (y_perm read, out written);
+      permute: the one-time expert reorder of one layer's gate/up tensor
+        [128, 1536, 2048] bf16 (read and written once)."""
+    dev = torch.device("cuda")
+    out = []
+    names = [only] if only else list(ISOLATED)
+
+    flush = torch.empty(512 * 2 ** 20, dtype=torch.uint8, device=dev)  # 4x the L2
+
+    def timed_ev(fn):
+        # L2 flushed (a 512 MB write) before every repetition; events bracket
+        # the kernel alone; the median repetition is reported
+        for _ in range(warmup):
+            fn()
+        torch.cuda.synchronize()
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        for a, b in evs:
+            flush.fill_(1)
+            a.record()
+            fn()
+            b.record()
+        torch.cuda.synchronize()
+        return statistics.median(a.elapsed_time(b) for a, b in evs)
+
+    def row(name, ms, nbytes, kernel, shape):
+        gbs = nbytes / (ms * 1e-3) / 1e9
+        out.append({"mode": f"isolated {name}", "kernel": kernel, "shape": shape, "ms": round(ms, 4),
+                    "algo_bytes": int(nbytes), "gbs": round(gbs, 1), "hbm_frac": round(gbs / pk["hbm_gbs"], 4)})
+
+    wl = W.PREFILL
+    T, d, k, E, K = wl.T, wl.d, wl.k, wl.E, 64
+    if "compaction" in names:
+        big = W.LARGE
+        kv = [W.make_kv(big, device=dev, seed=s) for s in (0, 1)]
+        kv_out = [torch.empty(big.layers, big.T - big.nv, big.kv_width, dtype=torch.bfloat16, device=dev)
+                  for _ in range(2)]
+        ms = timed_ev(lambda: [dm.decomoe_drop_visual_block(a, b, big.v0, big.nv) for a, b in zip(kv, kv_out)])
+        nb = 2 * 2 * big.layers * (big.T - big.nv) * big.kv_width * 2
+        row("compaction", ms, nb, "k_compact_vec", "2 x [48, 16384, 512] bf16 -> [48, 2048, 512]")
+        del kv, kv_out
+    if "gather" in names or "combine" in names:
+        g = W.make_layer(wl, device=dev)
+        logits = torch.empty(T, E, dtype=torch.float32, device=dev)
+        dm.decomoe_router_logits(g["x"], g["w_r"], g["bias"], logits)
+        idx = torch.empty(T, k, dtype=torch.int32, device=dev)
+        wts = torch.empty(T, k, dtype=torch.float32, device=dev)
+        rws = dm.workspace(dm.decomoe_route_workspace_bytes(T, E), dev)
+        dm.decomoe_route_prefix(logits, K, k, idx, wts, None, rws)
+        counts = torch.empty(K, dtype=torch.int32, device=dev)
+        offsets = torch.empty(K + 1, dtype=torch.int32, device=dev)
+        perm = torch.empty(T * k, dtype=torch.int32, device=dev)
+        inv = torch.empty(T * k, dtype=torch.int32, device=dev)
+        xp = torch.empty(T * k, d, dtype=torch.bfloat16, device=dev)
+        dws = dm.workspace(dm.decomoe_dispatch_workspace_bytes(T, k, K), dev)
+        dm.decomoe_dispatch(idx, K, g["x"], counts, offsets, perm, inv, xp, dws)
+        if "gather" in names:
+            # the row copy alone (the index pass is repeated inside the call;
+            # ncu separates k_gather_rows from the two index kernels)
+            ms = timed_ev(lambda: dm.decomoe_gather_rows(g["x"], perm, offsets, K, xp))
+            row("gather", ms, T * d * 2 + T * k * d * 2, "k_gather_rows", "x [2048, 2048] -> x_perm [16384, 2048]")
+        if "combine" in names:
+            y = torch.randn(T * k, d, device=dev).to(torch.bfloat16)
+            o = torch.empty(T, d, dtype=torch.bfloat16, device=dev)
+            ms = timed_ev(lambda: dm.decomoe_combine(y, inv, wts, o))
+            row("combine", ms, T * k * d * 2 + T * d * 2 + T * k * 8, "k_combine",
+                "y_perm [16384, 2048] -> out [2048, 2048]")
+            del y, o
+        del g, xp
+    if "permute" in names:
+        gl = W.make_layer(wl, device=dev, with_x=False)
+        wgu = dm.fuse_gate_up(gl["w_gate"], gl["w_up"])
+        del gl
+        dst = torch.empty_like(wgu)
+        pi = torch.randperm(E, device=dev).to(torch.int32)
+        ms = timed_ev(lambda: dm.decomoe_permute_experts(wgu, dst, pi))
+        nb = 2 * wgu.numel() * 2
+        row("permute", ms, nb, "k_permute_vec", "w_gate_up [128, 1536, 2048] bf16")
+        del wgu, dst
+    del flush
     torch.cuda.empty_cache()
     return out
 
@@ -969,6 +1080,15 @@ def main():
         line = only_decode(args, local)
         if rank == 0:
             print(json.dumps(line), flush=True)
+        return
+    if args.only_isolated:
+        import paper_2609_38823_gb300 as dm
+
+        dm.lib()
+        rows = run_isolated(dm, ws, peaks(), only=args.only_isolated, steps=max(1, args.steps),
+                            warmup=max(1, args.warmup))
+        if rank == 0:
+            print(json.dumps(rows), flush=True)
         return
     line = ours(args, ws, rank, local)
     if rank == 0:

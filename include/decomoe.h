@@ -166,6 +166,13 @@ DECOMOE_API int decomoe_route_prefix_dk(const float* logits, int64_t T, int E, i
  * ws: decomoe_dispatch_workspace_bytes(T, k, K) bytes.
  * ------------------------------------------------------------------------ */
 DECOMOE_API size_t decomoe_dispatch_workspace_bytes(int64_t T, int k, int K);
+/* The row gather of the dispatch alone: x_perm[r, :] = x[perm_token[r], :]
+ * for the offsets[K] (<= N) rows counted on the device (from a dispatch run
+ * without x_perm). x: [T, d] dtype, x_perm: [N, d] dtype, both 16-byte
+ * aligned with rows of a multiple of 16 bytes (DECOMOE_ERR_INVALID_ARG
+ * otherwise). */
+DECOMOE_API int decomoe_gather_rows(const void* x, const int32_t* perm_token, const int32_t* offsets, int K,
+                                    int64_t N, int d, int dtype, void* x_perm, decomoe_stream_t stream);
 DECOMOE_API int decomoe_dispatch(const int32_t* topk_idx, int64_t T, int k, int K, const void* x, int d,
                      int dtype, int32_t* counts, int32_t* offsets, int32_t* perm_token,
                      int32_t* inv_slot, void* x_perm, void* ws, size_t ws_bytes,
@@ -303,6 +310,22 @@ DECOMOE_API int decomoe_expert_swiglu_fused(const void* x_perm, const int32_t* o
                                             int m, int dtype, const void* w_gate_up, const void* w_down, void* h_ws,
                                             void* y_perm, int32_t* ready, int32_t* status_dev,
                                             decomoe_stream_t stream);
+
+/* The same one launch as decomoe_moe_layer runs it from 8192 routed rows: the
+ * dispatch's row gather inside the expert launch (Algorithm 2, dispatch and
+ * expert evaluation). x: [T, d] token rows; perm_token: [rows] from
+ * decomoe_dispatch (called without x_perm); x_perm: [rows, d] scratch the
+ * launch fills with x[perm_token[r]] on its way to the tiles (caller-owned,
+ * 16-byte aligned). Other arguments as decomoe_expert_swiglu_fused; ready
+ * needs decomoe_expert_swiglu_ready_ints(rows, K) zeroed int32. Only for
+ * sizes the one-launch tokens-as-M form takes (bf16, 8*K < rows <= 32768):
+ * DECOMOE_ERR_INVALID_ARG otherwise, nothing launched. Outputs equal those of
+ * decomoe_dispatch with x_perm followed by decomoe_expert_swiglu, bit for bit. */
+DECOMOE_API int decomoe_expert_swiglu_fused_gather(const void* x, int64_t T, const int32_t* perm_token,
+                                                   const int32_t* offsets, int64_t rows, int K, int d, int m,
+                                                   int dtype, const void* w_gate_up, const void* w_down,
+                                                   void* x_perm, void* h_ws, void* y_perm, int32_t* ready,
+                                                   int32_t* status_dev, decomoe_stream_t stream);
 
 /* The two phases of decomoe_expert_swiglu as separate calls (same arguments
  * and rules): gate/up with the fused SwiGLU epilogue writes h [rows, m]; down

@@ -57,6 +57,9 @@ SIGNATURES = {
                                     _P, _P]),
     "decomoe_expert_swiglu_ready_ints": (_S, [_L, _I]),
     "decomoe_expert_swiglu_fused": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
+    "decomoe_gather_rows": (_I, [_P, _P, _P, _I, _L, _I, _I, _P, _P]),
+    "decomoe_expert_swiglu_fused_gather": (_I, [_P, _L, _P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P,
+                                                _P]),
     "decomoe_router_route_dispatch_workspace_bytes": (_S, [_L, _I, _I, _I]),
     "decomoe_router_route_dispatch": (_I, [_P, _P, _P, _L, _I, _I, _I, _I, _I, _D, _P, _P, _P, _P, _P, _P, _P, _P, _P,
                                            _P, _P, _S, _P, _P]),
@@ -415,6 +418,31 @@ def decomoe_expert_swiglu_fused(x_perm, offsets, K, w_gate_up, w_down, h, y_perm
            lib().decomoe_expert_swiglu_fused(_ptr(x_perm), _ptr(offsets), rows, K, d, m, _dt(x_perm),
                                              _ptr(w_gate_up), _ptr(w_down), _ptr(h), _ptr(y_perm), _ptr(ready),
                                              _ptr(status), _stream(stream)))
+
+
+def decomoe_gather_rows(x, perm_token, offsets, K, x_perm, stream=None):
+    """The dispatch's row gather alone: x_perm[r] = x[perm_token[r]] for the
+    offsets[K] rows on the device."""
+    _need_cuda(x, perm_token, offsets, x_perm)
+    d = x.shape[1]
+    _check("decomoe_gather_rows",
+           lib().decomoe_gather_rows(_ptr(x), _ptr(perm_token), _ptr(offsets), K, x_perm.shape[0], d, _dt(x),
+                                     _ptr(x_perm), _stream(stream)))
+
+
+def decomoe_expert_swiglu_fused_gather(x, perm_token, offsets, K, w_gate_up, w_down, x_perm, h, y_perm, ready,
+                                       status=None, stream=None):
+    """The one-launch expert FFN as the layer runs it from 8192 routed rows:
+    it gathers x_perm[r] = x[perm_token[r]] itself (dispatch called without
+    x_perm); ready: int32 counters, zero at the call."""
+    _need_cuda(x, perm_token, offsets, w_gate_up, w_down, x_perm, h, y_perm, ready, status)
+    T, d = x.shape
+    rows = x_perm.shape[0]
+    m = h.shape[1]
+    _check("decomoe_expert_swiglu_fused_gather",
+           lib().decomoe_expert_swiglu_fused_gather(_ptr(x), T, _ptr(perm_token), _ptr(offsets), rows, K, d, m,
+                                                    _dt(x), _ptr(w_gate_up), _ptr(w_down), _ptr(x_perm), _ptr(h),
+                                                    _ptr(y_perm), _ptr(ready), _ptr(status), _stream(stream)))
 
 
 def decomoe_expert_gate_up(x_perm, offsets, K, w_gate_up, h, status=None, sched=None, stream=None):

@@ -111,6 +111,19 @@ size_t decomoe_dispatch_workspace_bytes(int64_t T, int k, int K) {
   return align_up(static_cast<size_t>(ntiles > 0 ? ntiles : 1) * K * sizeof(int32_t), 256);
 }
 
+int decomoe_gather_rows(const void* x, const int32_t* perm_token, const int32_t* offsets, int K, int64_t N,
+                        int d, int dtype, void* x_perm, decomoe_stream_t stream) {
+  clear_error();
+  DM_ARG_CHECK(N >= 0 && K >= 1 && d > 0 && (dtype == DECOMOE_BF16 || dtype == DECOMOE_F32),
+               "gather_rows: bad sizes or dtype");
+  if (N == 0) return DECOMOE_OK;
+  const size_t row_bytes = static_cast<size_t>(d) * dtype_bytes(dtype);
+  DM_ARG_CHECK(x && perm_token && offsets && x_perm, "gather_rows: null pointer");
+  DM_ARG_CHECK(row_bytes % 16 == 0 && aligned16(x) && aligned16(x_perm),
+               "gather_rows: rows must be 16-byte multiples and 16-byte aligned");
+  return launch_gather_rows(x, perm_token, offsets, K, row_bytes, N, x_perm, reinterpret_cast<cudaStream_t>(stream));
+}
+
 int decomoe_dispatch(const int32_t* topk_idx, int64_t T, int k, int K, const void* x, int d,
                      int dtype, int32_t* counts, int32_t* offsets, int32_t* perm_token,
                      int32_t* inv_slot, void* x_perm, void* ws, size_t ws_bytes,

@@ -2557,4 +2557,20 @@ int decomoe_expert_swiglu_fused(const void* x_perm, const int32_t* offsets, int6
                                nullptr, stream);
 }
 
+int decomoe_expert_swiglu_fused_gather(const void* x, int64_t T, const int32_t* perm_token, const int32_t* offsets,
+                                       int64_t rows, int K, int d, int m, int dtype, const void* w_gate_up,
+                                       const void* w_down, void* x_perm, void* h_ws, void* y_perm, int32_t* ready,
+                                       int32_t* status_dev, decomoe_stream_t stream) {
+  using namespace decomoe;
+  clear_error();
+  DM_ARG_CHECK(x != nullptr && perm_token != nullptr && T >= 0, "expert_swiglu_fused_gather: null pointer");
+  DM_ARG_CHECK(expert_ffn_fused_kind(rows, K, m, dtype) == FFN_FUSED_TC,
+               "expert_swiglu_fused_gather: %lld rows at K=%d take no one-launch tokens-as-M form",
+               (long long)rows, K);
+  bool fused = false;
+  DM_RET(launch_expert_ffn_fused(x_perm, offsets, rows, K, d, m, dtype, w_gate_up, w_down, h_ws, y_perm, ready,
+                                 status_dev, reinterpret_cast<cudaStream_t>(stream), &fused, x, perm_token));
+  return fused ? DECOMOE_OK : DECOMOE_ERR_UNSUPPORTED;
+}
+
 }  // extern "C"

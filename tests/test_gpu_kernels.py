@@ -179,6 +179,11 @@ def test_dispatch_parity(T, k, K, d, dt, pattern):
     assert np.array_equal(perm.cpu().numpy(), p)
     assert np.array_equal(inv.cpu().numpy(), i)
     assert torch.equal(xp, x[perm.long()])
+    # the row gather alone, after the index passes: the same rows
+    xp2 = torch.zeros_like(xp)
+    dm.decomoe_gather_rows(x, perm, offsets, K, xp2)
+    torch.cuda.synchronize()
+    assert torch.equal(xp2, xp)
 
 
 def test_dispatch_flags_bad_expert_id():
@@ -217,6 +222,7 @@ EXPERT_CASES = [
     (64, 2, 16, 256, 128, "route"),
     (300, 1, 3, 256, 256, "one_expert"),  # one expert, 3 M tiles (300 rows)
     (512, 8, 64, 2048, 768, "route"),     # full layer width, 4096 rows
+    (1100, 8, 64, 2048, 768, "route"),    # 8800 rows: the layer's launch gathers its own rows
     (129, 8, 16, 2048, 768, "uniform"),
     (1, 8, 64, 2048, 768, "route"),       # decode T=1 (8 rows)
     (8, 8, 64, 2048, 768, "route"),       # decode T=8 (64 rows)
@@ -275,6 +281,26 @@ def test_expert_swiglu_bf16_parity(T, k, K, d, m, pattern):
     torch.cuda.synchronize()
     assert dm.decomoe_read_status(status) == 0
     assert torch.equal(y5, y) and torch.equal(h5, h)
+    # the one launch that also gathers the dispatched rows (as the layer runs
+    # it from 8192 routed rows): same tiles, same bits, and the gathered rows
+    # are x[perm_token]
+    if 8 * K < R <= 32768 and (2 * m) % 256 == 0:
+        ready.zero_()
+        xg = torch.zeros_like(xp)
+        h6 = torch.empty_like(h)
+        y6 = torch.empty_like(y)
+        dm.decomoe_expert_swiglu_fused_gather(L["x"].to(DEV), perm_d, off, K, w_gu, g["w_down"], xg, h6, y6, ready,
+                                              status)
+        torch.cuda.synchronize()
+        assert dm.decomoe_read_status(status) == 0
+        assert torch.equal(y6, y) and torch.equal(h6, h)
+        assert torch.equal(xg.view(torch.int16), xp.view(torch.int16))
+    else:
+        with pytest.raises(dm.DecomoeError) as e:
+            dm.decomoe_expert_swiglu_fused_gather(L["x"].to(DEV), perm_d, off, K, w_gu, g["w_down"],
+                                                  torch.empty_like(xp), torch.empty_like(h), torch.empty_like(y),
+                                                  ready, status)
+        assert e.value.code == dm.DECOMOE_ERR_INVALID_ARG
 
 
 def test_expert_swiglu_f32_parity():
