@@ -443,3 +443,45 @@ def stack_token(h_t, layers, K_sched, k, eps=1e-6, round_bf16=None):
         if round_bf16 is not None:
             h = round_bf16(h[None, :])[0]
     return h, margins
+
+
+# ---------------------------------------------------------------------------
+# Self-attention on the compacted sequence and over the text-only KV cache
+# (Section 3.2: once the visual block exits, attention in that layer and every
+# later one runs on the shortened text-only sequence; Algorithm 2, last step:
+# decoding reuses the shortened text-only cache; Appendix FLOPs: 2qS(S+1) per
+# prefill layer, 4qC per decode forward with cache length C)
+# ---------------------------------------------------------------------------
+
+def attention(q, k_cache, v_cache, scale=None):
+    """Causal scaled-dot-product attention with grouped KV heads.
+
+    q: [n, Hq, D] queries of the last n positions of a sequence whose keys and
+    values are k_cache, v_cache: [C, Hkv, D] (C >= n; the queries' own keys are
+    the last n rows). Query i sits at position C - n + i and attends to keys
+    j <= C - n + i: n = C is a prefill over the sequence, n < C a decode step
+    over a cache. Query head h reads KV head h // (Hq // Hkv). The score is
+    q . k * scale (scale = 1 / sqrt(D) unless given); weights are the softmax
+    over the visible keys; the output is the weighted sum of their values.
+    The paper does not restate attention; this is the standard causal form of
+    the decoder it accelerates. Float64. Returns [n, Hq, D].
+    """
+    q = np.asarray(q, F64)
+    k_cache = np.asarray(k_cache, F64)
+    v_cache = np.asarray(v_cache, F64)
+    n, Hq, D = q.shape
+    C, Hkv, _ = k_cache.shape
+    if not (1 <= n <= C) or Hq % Hkv != 0:
+        raise ValueError("need 1 <= n <= C and Hq a multiple of Hkv")
+    if scale is None:
+        scale = 1.0 / np.sqrt(D)
+    group = Hq // Hkv
+    out = np.zeros((n, Hq, D), F64)
+    for i in range(n):
+        last = C - n + i  # position of query i: keys 0..last are visible
+        for h in range(Hq):
+            g = h // group
+            s = (k_cache[:last + 1, g, :] @ q[i, h, :]) * scale
+            w = softmax(s)
+            out[i, h, :] = w @ v_cache[:last + 1, g, :]
+    return out

@@ -588,3 +588,82 @@ def test_gate_mlp_closed_form_sigmoid():
     z = O.gate_logits(np.array([-1.0, 0, 0, 0]), np.array([[1.0, 0, 0, 0]]), np.zeros(1),
                       np.array([[0.0], [5.0]]), np.array([0.25, 0.0]))
     assert np.allclose(z, [0.25, 0.0])
+
+
+# ---------------------------------------------------------------- attention on the compacted sequence
+
+def test_attention_single_key_returns_its_value():
+    r = np.random.default_rng(3)
+    q = r.standard_normal((1, 4, 8))
+    k = r.standard_normal((1, 2, 8))
+    v = r.standard_normal((1, 2, 8))
+    out = O.attention(q, k, v)
+    for h in range(4):
+        np.testing.assert_allclose(out[0, h], v[0, h // 2], rtol=0, atol=1e-15)
+
+
+def test_attention_two_keys_closed_form_and_equal_keys_mean():
+    r = np.random.default_rng(4)
+    D = 16
+    q = r.standard_normal((1, 1, D))
+    k = r.standard_normal((2, 1, D))
+    v = r.standard_normal((2, 1, D))
+    s0, s1 = (float(k[j, 0] @ q[0, 0]) / np.sqrt(D) for j in range(2))
+    w1 = 1.0 / (1.0 + math.exp(s0 - s1))
+    np.testing.assert_allclose(O.attention(q, k, v)[0, 0], (1 - w1) * v[0, 0] + w1 * v[1, 0], rtol=1e-13)
+    # identical keys: every visible key weighs the same (the mean of the values)
+    k_same = np.repeat(k[:1], 5, axis=0)
+    v5 = r.standard_normal((5, 1, D))
+    np.testing.assert_allclose(O.attention(q, k_same, v5)[0, 0], v5[:, 0].mean(0), rtol=1e-13)
+
+
+def test_attention_matches_torch_sdpa_with_grouped_heads():
+    # prefill (n = C, causal) and a decode step (n < C) against torch's
+    # scaled_dot_product_attention with the KV heads repeated per group and
+    # the visibility written as a mask
+    r = np.random.default_rng(5)
+    for (n, C, Hq, Hkv, D) in ((7, 7, 8, 2, 16), (1, 9, 4, 1, 8), (3, 11, 6, 3, 32)):
+        q = r.standard_normal((n, Hq, D))
+        k = r.standard_normal((C, Hkv, D))
+        v = r.standard_normal((C, Hkv, D))
+        got = O.attention(q, k, v)
+        g = Hq // Hkv
+        qt = torch.from_numpy(q).permute(1, 0, 2)                      # [Hq, n, D]
+        kt = torch.from_numpy(k).permute(1, 0, 2).repeat_interleave(g, 0)
+        vt = torch.from_numpy(v).permute(1, 0, 2).repeat_interleave(g, 0)
+        mask = torch.tensor([[j <= C - n + i for j in range(C)] for i in range(n)])
+        ref = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, attn_mask=mask)
+        np.testing.assert_allclose(got, ref.permute(1, 0, 2).numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_attention_on_compacted_sequence_equals_masking_the_visual_keys():
+    # removing the visual block [v0, v0 + nv) from the keys and values (the
+    # SAVB exit) gives each text query the same output as attending over the
+    # full sequence with the visual keys hidden: the removal changes the work,
+    # not what text tokens see
+    r = np.random.default_rng(6)
+    S, v0, nv, Hq, Hkv, D = 20, 3, 11, 4, 2, 16
+    x_q = r.standard_normal((S, Hq, D))
+    k = r.standard_normal((S, Hkv, D))
+    v = r.standard_normal((S, Hkv, D))
+    text = [i for i in range(S) if not (v0 <= i < v0 + nv)]
+    comp = O.attention(x_q[text], O.drop_visual_block(k, v0, nv), O.drop_visual_block(v, v0, nv))
+    # brute force on the full sequence: causal, visual keys excluded
+    for a, i in enumerate(text):
+        for h in range(Hq):
+            vis = [j for j in text if j <= i]
+            s = np.array([k[j, h // 2] @ x_q[i, h] for j in vis]) / np.sqrt(D)
+            w = np.exp(s - s.max())
+            w /= w.sum()
+            np.testing.assert_allclose(comp[a, h], w @ v[vis, h // 2], rtol=1e-12, atol=1e-12)
+
+
+def test_attention_decode_step_equals_last_row_of_prefill():
+    # the decode step over the cache gives what the prefill gives its last rows
+    r = np.random.default_rng(8)
+    C, Hq, Hkv, D = 13, 4, 2, 8
+    q = r.standard_normal((C, Hq, D))
+    k = r.standard_normal((C, Hkv, D))
+    v = r.standard_normal((C, Hkv, D))
+    full = O.attention(q, k, v)
+    np.testing.assert_allclose(O.attention(q[-2:], k, v), full[-2:], rtol=1e-13, atol=1e-14)
