@@ -687,7 +687,7 @@ def run_large(dm, ws, pk, n):
     return out
 
 
-ISOLATED = ("compaction", "gather", "combine", "permute")
+ISOLATED = ("compaction", "gather", "combine", "permute", "attention")
 
 
 def run_isolated(dm, ws, pk, only=None, steps=10, warmup=3):
@@ -702,7 +702,10 @@ def run_isolated(dm, ws, pk, only=None, steps=10, warmup=3):
         events);
       combine: T=2048, k=8 (y_perm read, out written);
       permute: the one-time expert reorder of one layer's gate/up tensor
-        [128, 1536, 2048] bf16 (read and written once)."""
+        [128, 1536, 2048] bf16 (read and written once);
+      attention: one decode step of one layer's attention over the text-only
+        cache the visual exit leaves and over the uncompacted cache (K and V
+        read once)."""
     dev = torch.device("cuda")
     out = []
     names = [only] if only else list(ISOLATED)
@@ -778,6 +781,25 @@ def run_isolated(dm, ws, pk, only=None, steps=10, warmup=3):
         nb = 2 * wgu.numel() * 2
         row("permute", ms, nb, "k_permute_vec", "w_gate_up [128, 1536, 2048] bf16")
         del wgu, dst
+    if "attention" in names:
+        # one decode step (one new token) of one layer's attention, 32 query
+        # heads on 4 KV heads of 128, over the text-only cache the exit leaves
+        # and over the uncompacted cache: the stack workload (16 + 1280 + 256
+        # rows) and the large one (14336 + 2048 rows), next token appended
+        Hq, Hkv, Dh = 32, 4, 128
+        for name, C_text, C_full in (("stack", 16 + 256 + 1, 1552 + 1), ("large", 2048 + 1, 16384 + 1)):
+            for kind, C in (("text-only cache", C_text), ("full cache", C_full)):
+                gq = torch.Generator(device=dev).manual_seed(C)
+                q = torch.randn(1, Hq, Dh, device=dev, generator=gq).to(torch.bfloat16)
+                kc = torch.randn(C, Hkv, Dh, device=dev, generator=gq).to(torch.bfloat16)
+                vc = torch.randn(C, Hkv, Dh, device=dev, generator=gq).to(torch.bfloat16)
+                o = torch.empty(1, Hq, Dh, dtype=torch.bfloat16, device=dev)
+                aws = dm.workspace(dm.decomoe_attention_workspace_bytes(1, C, Hq, Hkv, Dh), dev)
+                ms = timed_ev(lambda: dm.decomoe_attention(q, kc, vc, o, aws))
+                nb = 2 * C * Hkv * Dh * 2 + 2 * Hq * Dh * 2
+                row(f"attention decode, {name}, {kind}", ms, nb, "k_attn_split + k_attn_combine",
+                    f"q [1, 32, 128], K and V [{C}, 4, 128] bf16 (4qC = {4 * Hq * Dh * C / 1e6:.1f} MFLOP)")
+                del q, kc, vc, o, aws
     del flush
     torch.cuda.empty_cache()
     return out

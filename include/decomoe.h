@@ -530,6 +530,29 @@ DECOMOE_API int decomoe_moe_layer_workspace_layout(int64_t T, int d, int E, int 
                                        size_t* offs_host);
 
 /* ------------------------------------------------------------------------
+ * Attention on the compacted sequence and over the text-only KV cache
+ * (Section 3.2: once the visual block exits, attention in that layer and
+ * every later one runs on the shortened text-only sequence; Algorithm 2,
+ * last step: decoding reuses the shortened cache; Appendix FLOPs 2qS(S+1)
+ * per prefill layer, 4qC per decode forward with cache length C).
+ *   q: [n, Hq, D] queries of the last n positions; k_cache, v_cache:
+ *   [C, Hkv, D] keys and values of the whole (compacted) sequence, the
+ *   queries' own rows last (n <= C); out: [n, Hq, D]. All bf16, row-major,
+ *   16-byte aligned; D = 128; Hq a multiple of Hkv. Query i sits at position
+ *   C - n + i and sees keys 0 .. C - n + i; query head h reads KV head
+ *   h / (Hq / Hkv). scale <= 0 means 1 / sqrt(D). fp32 scores, softmax and
+ *   accumulation; out rounded to bf16.
+ *   Decode sizes: n * (Hq / Hkv) <= 64 queries per KV head (split-key
+ *   partials over 128-key chunks and a combine in chunk order; deterministic).
+ *   ws: decomoe_attention_workspace_bytes(n, C, Hq, Hkv, D) bytes.
+ *   DECOMOE_ERR_INVALID_ARG for other shapes, before any launch.
+ * ------------------------------------------------------------------------ */
+DECOMOE_API size_t decomoe_attention_workspace_bytes(int64_t n, int64_t C, int Hq, int Hkv, int D);
+DECOMOE_API int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void* v_cache, int64_t C,
+                                  int Hq, int Hkv, int D, float scale, void* out, void* ws, size_t ws_bytes,
+                                  int32_t* status_dev, decomoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * Bounded-wait status. Kernels that wait on device barriers give up after a
  * time limit, record DECOMOE_ERR_TIMEOUT (or DECOMOE_ERR_BAD_INPUT) in the
  * caller's status word and return, leaving the context usable.

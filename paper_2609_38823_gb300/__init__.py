@@ -58,6 +58,8 @@ SIGNATURES = {
     "decomoe_expert_swiglu_ready_ints": (_S, [_L, _I]),
     "decomoe_expert_swiglu_fused": (_I, [_P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
     "decomoe_gather_rows": (_I, [_P, _P, _P, _I, _L, _I, _I, _P, _P]),
+    "decomoe_attention_workspace_bytes": (_S, [_L, _L, _I, _I, _I]),
+    "decomoe_attention": (_I, [_P, _L, _P, _P, _L, _I, _I, _I, _F, _P, _P, _S, _P, _P]),
     "decomoe_expert_swiglu_fused_gather": (_I, [_P, _L, _P, _P, _L, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P,
                                                 _P]),
     "decomoe_router_route_dispatch_workspace_bytes": (_S, [_L, _I, _I, _I]),
@@ -418,6 +420,22 @@ def decomoe_expert_swiglu_fused(x_perm, offsets, K, w_gate_up, w_down, h, y_perm
            lib().decomoe_expert_swiglu_fused(_ptr(x_perm), _ptr(offsets), rows, K, d, m, _dt(x_perm),
                                              _ptr(w_gate_up), _ptr(w_down), _ptr(h), _ptr(y_perm), _ptr(ready),
                                              _ptr(status), _stream(stream)))
+
+
+def decomoe_attention_workspace_bytes(n, C, Hq, Hkv, D=128):
+    return int(lib().decomoe_attention_workspace_bytes(n, C, Hq, Hkv, D))
+
+
+def decomoe_attention(q, k_cache, v_cache, out, ws, scale=0.0, status=None, stream=None):
+    """Causal grouped-head attention of the last n positions over a
+    (compacted) sequence: q [n, Hq, D], k_cache / v_cache [C, Hkv, D], out
+    [n, Hq, D], bf16."""
+    _need_cuda(q, k_cache, v_cache, out, ws, status)
+    n, Hq, D = q.shape
+    C, Hkv, _ = k_cache.shape
+    _check("decomoe_attention",
+           lib().decomoe_attention(_ptr(q), n, _ptr(k_cache), _ptr(v_cache), C, Hq, Hkv, D, float(scale), _ptr(out),
+                                   _ptr(ws), ws.numel() * ws.element_size(), _ptr(status), _stream(stream)))
 
 
 def decomoe_gather_rows(x, perm_token, offsets, K, x_perm, stream=None):

@@ -17,7 +17,7 @@ ROOT = os.path.dirname(HERE)
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(HERE, "libdecomoe.so")
 
-CU_SOURCES = ["api.cu", "route.cu", "dispatch.cu", "expert_gemm.cu", "combine_compact.cu", "calib_gate.cu", "layer.cu", "decode_layer.cu"]
+CU_SOURCES = ["api.cu", "route.cu", "dispatch.cu", "expert_gemm.cu", "combine_compact.cu", "calib_gate.cu", "layer.cu", "decode_layer.cu", "attention.cu"]
 C_SOURCES = ["prefix.c"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

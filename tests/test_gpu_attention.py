@@ -1,0 +1,93 @@
+"""Attention on the compacted sequence and over the text-only KV cache
+(decomoe_attention) against the oracle's causal grouped-head attention.
+
+The layer shape is the 30B-A3B decoder's: 32 query heads and 4 KV heads of
+128 (q = 4096, k_v = 512); the caches are one layer slice of the KV buffers
+that the visual-block removal compacts ([T, 4, 128] bf16). Outputs are
+compared at the bf16 output tolerance (fp32 scores, softmax and sums).
+"""
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_38823_gb300 as dm
+import workloads as W
+from oracle import decomoe_oracle as O
+from tests.helpers import BF16_MAX_ABS, BF16_REL_L2, assert_close_out, f64
+
+pytestmark = pytest.mark.gpu
+DEV = torch.device("cuda")
+HQ, HKV, D = 32, 4, 128
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    import __graft_entry__
+
+    __graft_entry__.build()
+    dm.lib()
+
+
+def _qkv(n, C, seed, Hq=HQ, Hkv=HKV):
+    g = torch.Generator().manual_seed(seed)
+    q = torch.randn(n, Hq, D, generator=g).to(torch.bfloat16)
+    k = torch.randn(C, Hkv, D, generator=g).to(torch.bfloat16)
+    v = torch.randn(C, Hkv, D, generator=g).to(torch.bfloat16)
+    return q, k, v
+
+
+def _run(q, k, v, scale=0.0):
+    n, Hq, _ = q.shape
+    C, Hkv, _ = k.shape
+    out = torch.full((n, Hq, D), 9.0, dtype=torch.bfloat16, device=DEV)
+    ws = dm.workspace(dm.decomoe_attention_workspace_bytes(n, C, Hq, Hkv, D), DEV)
+    dm.decomoe_attention(q.to(DEV), k.to(DEV), v.to(DEV), out, ws, scale=scale)
+    torch.cuda.synchronize()
+    return out
+
+
+@pytest.mark.parametrize("n,C", [(1, 1), (1, 127), (1, 128), (1, 272), (1, 2049), (2, 300), (8, 1552),
+                                 (1, 16384), (3, 129)])
+def test_attention_decode_parity(n, C):
+    q, k, v = _qkv(n, C, seed=C + n)
+    out = _run(q, k, v)
+    ref = O.attention(f64(q), f64(k), f64(v))
+    assert_close_out(f64(out), ref, BF16_REL_L2, BF16_MAX_ABS, f"attention n={n} C={C}")
+
+
+def test_attention_grouping_and_scale():
+    # 8 query heads on 2 KV heads and an explicit scale
+    q, k, v = _qkv(2, 200, seed=5, Hq=8, Hkv=2)
+    out = _run(q, k, v, scale=0.05)
+    ref = O.attention(f64(q), f64(k), f64(v), scale=0.05)
+    assert_close_out(f64(out), ref, BF16_REL_L2, BF16_MAX_ABS, "grouping and scale")
+
+
+def test_attention_on_compacted_cache_equals_masked_full_cache():
+    """The stack workload's sequence (16 system rows, 1280 visual, 256 text):
+    a text token's decode step over the compacted cache (the visual block
+    removed by decomoe_drop_visual_block) matches the oracle run on the full
+    cache with the visual rows removed, and equals what the oracle gives on
+    the full sequence with those keys hidden (oracle pin)."""
+    wl = W.STACK
+    C_full = wl.T
+    q, k, v = _qkv(1, C_full, seed=11)
+    kc = torch.empty(C_full - wl.nv, HKV, D, dtype=torch.bfloat16, device=DEV)
+    vc = torch.empty_like(kc)
+    dm.decomoe_drop_visual_block(k.to(DEV).view(C_full, HKV * D), kc.view(-1, HKV * D), wl.v0, wl.nv)
+    dm.decomoe_drop_visual_block(v.to(DEV).view(C_full, HKV * D), vc.view(-1, HKV * D), wl.v0, wl.nv)
+    out = _run(q, kc.cpu(), vc.cpu())
+    ref = O.attention(f64(q), O.drop_visual_block(f64(k), wl.v0, wl.nv), O.drop_visual_block(f64(v), wl.v0, wl.nv))
+    assert_close_out(f64(out), ref, BF16_REL_L2, BF16_MAX_ABS, "decode over the compacted cache")
+
+
+def test_attention_rejects_unsupported_shapes():
+    q, k, v = _qkv(1, 10, seed=1)
+    ws = dm.workspace(1 << 20, DEV)
+    out = torch.empty(1, HQ, D, dtype=torch.bfloat16, device=DEV)
+    with pytest.raises(dm.DecomoeError) as e:  # more queries than keys
+        dm.decomoe_attention(q.to(DEV).repeat(11, 1, 1), k.to(DEV), v.to(DEV), out.repeat(11, 1, 1), ws)
+    assert e.value.code == dm.DECOMOE_ERR_INVALID_ARG
+    with pytest.raises(dm.DecomoeError) as e:  # 31 query heads on 4 KV heads
+        dm.decomoe_attention(q.to(DEV)[:, :31].contiguous(), k.to(DEV), v.to(DEV), out[:, :31].contiguous(), ws)
+    assert e.value.code == dm.DECOMOE_ERR_INVALID_ARG
