@@ -687,7 +687,7 @@ def run_large(dm, ws, pk, n):
     return out
 
 
-ISOLATED = ("compaction", "gather", "combine", "permute", "attention")
+ISOLATED = ("compaction", "gather", "combine", "permute", "attention", "attention_prefill")
 
 
 def run_isolated(dm, ws, pk, only=None, steps=10, warmup=3):
@@ -705,7 +705,10 @@ def run_isolated(dm, ws, pk, only=None, steps=10, warmup=3):
         [128, 1536, 2048] bf16 (read and written once);
       attention: one decode step of one layer's attention over the text-only
         cache the visual exit leaves and over the uncompacted cache (K and V
-        read once)."""
+        read once);
+      attention_prefill: one layer's causal prefill attention over the
+        compacted sequence and over the full one, as TFLOP/s of the
+        Appendix's 2 q S (S + 1) against the measured bf16 tensor peak."""
     dev = torch.device("cuda")
     out = []
     names = [only] if only else list(ISOLATED)
@@ -799,6 +802,27 @@ def run_isolated(dm, ws, pk, only=None, steps=10, warmup=3):
                 nb = 2 * C * Hkv * Dh * 2 + 2 * Hq * Dh * 2
                 row(f"attention decode, {name}, {kind}", ms, nb, "k_attn_split + k_attn_combine",
                     f"q [1, 32, 128], K and V [{C}, 4, 128] bf16 (4qC = {4 * Hq * Dh * C / 1e6:.1f} MFLOP)")
+                del q, kc, vc, o, aws
+    if "attention_prefill" in names:
+        # one layer's prefill attention (n = C = S, 32 query heads on 4 KV
+        # heads of 128): the stack workload's sequence (1552 rows, 272 once
+        # the visual block has left) and the large one's (16384 rows, 2048)
+        Hq, Hkv, Dh = 32, 4, 128
+        for name, S_text, S_full in (("stack", 272, 1552), ("large", 2048, 16384)):
+            for kind, S in (("compacted sequence", S_text), ("full sequence", S_full)):
+                gq = torch.Generator(device=dev).manual_seed(S)
+                q = torch.randn(S, Hq, Dh, device=dev, generator=gq).to(torch.bfloat16)
+                kc = torch.randn(S, Hkv, Dh, device=dev, generator=gq).to(torch.bfloat16)
+                vc = torch.randn(S, Hkv, Dh, device=dev, generator=gq).to(torch.bfloat16)
+                o = torch.empty(S, Hq, Dh, dtype=torch.bfloat16, device=dev)
+                aws = dm.workspace(dm.decomoe_attention_workspace_bytes(S, S, Hq, Hkv, Dh), dev)
+                ms = timed_ev(lambda: dm.decomoe_attention(q, kc, vc, o, aws))
+                fl = 2.0 * Hq * Dh * S * (S + 1)
+                tf = fl / (ms * 1e-3) / 1e12
+                out.append({"mode": f"isolated attention prefill, {name}, {kind}", "kernel": "k_attn_vt + k_attn_prefill",
+                            "shape": f"q [{S}, 32, 128], K and V [{S}, 4, 128] bf16", "ms": round(ms, 4),
+                            "algo_flops": fl, "tflops": round(tf, 1),
+                            "tensor_frac": round(tf / pk["bf16_tflops"], 4)})
                 del q, kc, vc, o, aws
     del flush
     torch.cuda.empty_cache()

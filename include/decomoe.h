@@ -544,7 +544,13 @@ DECOMOE_API int decomoe_moe_layer_workspace_layout(int64_t T, int d, int E, int 
  *   accumulation; out rounded to bf16.
  *   Decode sizes: n * (Hq / Hkv) <= 64 queries per KV head (split-key
  *   partials over 128-key chunks and a combine in chunk order; deterministic).
- *   ws: decomoe_attention_workspace_bytes(n, C, Hq, Hkv, D) bytes.
+ *   Prefill sizes (more queries per KV head, n = C or a chunk n < C): V is
+ *   transposed into the workspace, then one tensor-core CTA per (query head,
+ *   128-query tile) runs the online softmax over 128-key blocks up to its
+ *   causal limit (P rounded to bf16 before the P V product; deterministic).
+ *   ws: decomoe_attention_workspace_bytes(n, C, Hq, Hkv, D) bytes, 16-byte
+ *   aligned. A wait that runs past the time limit records
+ *   DECOMOE_ERR_TIMEOUT in status_dev (may be null).
  *   DECOMOE_ERR_INVALID_ARG for other shapes, before any launch.
  * ------------------------------------------------------------------------ */
 DECOMOE_API size_t decomoe_attention_workspace_bytes(int64_t n, int64_t C, int Hq, int Hkv, int D);

@@ -91,6 +91,10 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
 // out of bounds.
 int make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint32_t box_outer,
                    uint32_t box_inner);
+// 3-D bf16 tensor (dims[0] contiguous; byte strides of dims 1 and 2), box[0]
+// = 64 elements with 128-byte swizzle, zero fill out of bounds.
+int make_tmap_bf16_3d(CUtensorMap* m, const void* base, const uint64_t dims[3], const uint64_t strides[2],
+                      const uint32_t box[3]);
 int launch_router_tc(const void* x, const void* w_r, const float* bias, int64_t T, int d, int E,
                      float* logits, int32_t* status, cudaStream_t s);
 bool router_tc_supported(int d, int E);
@@ -323,6 +327,14 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* m, 
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* m, uint32_t bar, int32_t x, int32_t y,
+                                            int32_t z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(bar)
       : "memory");
 }
 // Four rows (row0..row3, any order) of a 2-D tensor whose map has a

@@ -77,6 +77,31 @@ int make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t ou
   return DECOMOE_OK;
 }
 
+// 3-D bf16 tensor, dims[0] innermost (contiguous), byte strides of dims 1 and
+// 2, box[0] = 64 elements (128-byte swizzle); zero fill out of bounds.
+int make_tmap_bf16_3d(CUtensorMap* m, const void* base, const uint64_t dims[3], const uint64_t strides[2],
+                      const uint32_t box[3]) {
+  auto fn = encode_fn();
+  if (fn == nullptr) {
+    set_error("cuTensorMapEncodeTiled is not available from the driver");
+    return DECOMOE_ERR_CUDA;
+  }
+  cuuint64_t d[3] = {dims[0], dims[1], dims[2]};
+  cuuint64_t st[2] = {strides[0], strides[1]};
+  cuuint32_t bx[3] = {box[0], box[1], box[2]};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), d, st, bx, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    set_error("cuTensorMapEncodeTiled (3-D) failed (%d): dims=%llu x %llu x %llu box=%u x %u x %u", (int)r,
+              (unsigned long long)dims[0], (unsigned long long)dims[1], (unsigned long long)dims[2], box[0], box[1],
+              box[2]);
+    return DECOMOE_ERR_CUDA;
+  }
+  return DECOMOE_OK;
+}
+
 // ------------------------------------------------------------------ tcgen05 GEMM
 // EPI_SWIGLU: columns [0, BN/2) gate, [BN/2, BN) up -> bf16 silu(g)*u.
 // EPI_BF16: bf16 store. EPI_F32_BIAS: fp32 + bias[col]. EPI_F32_BIAS_T: the

@@ -1,5 +1,8 @@
 """Attention on the compacted sequence and over the text-only KV cache
-(decomoe_attention) against the oracle's causal grouped-head attention.
+(decomoe_attention) against the oracle's causal grouped-head attention:
+decode steps (up to 64 queries per KV head, split-key CUDA-core kernel) and
+prefill (more, the tensor-core kernel), with ragged tiles, chunked prefill
+(n < C), sampled rows at the full 16384-token sequence.
 
 The layer shape is the 30B-A3B decoder's: 32 query heads and 4 KV heads of
 128 (q = 4096, k_v = 512); the caches are one layer slice of the KV buffers
@@ -55,6 +58,51 @@ def test_attention_decode_parity(n, C):
     assert_close_out(f64(out), ref, BF16_REL_L2, BF16_MAX_ABS, f"attention n={n} C={C}")
 
 
+@pytest.mark.parametrize("n,C", [(9, 9), (9, 300), (128, 128), (129, 200), (300, 300), (640, 1000), (1024, 1024)])
+def test_attention_prefill_parity(n, C):
+    q, k, v = _qkv(n, C, seed=7 * C + n)
+    out = _run(q, k, v)
+    ref = O.attention(f64(q), f64(k), f64(v))
+    assert_close_out(f64(out), ref, BF16_REL_L2, BF16_MAX_ABS, f"prefill attention n={n} C={C}")
+
+
+def _sampled_rows(out, q, k, v, rows, label):
+    """Query row i of a launch over (n, C) is attention at position C - n + i
+    over keys 0..C - n + i: the oracle on that one row and prefix."""
+    n, C = q.shape[0], k.shape[0]
+    got = f64(out[rows].cpu())
+    ref = np.concatenate([O.attention(f64(q[i:i + 1]), f64(k[:C - n + i + 1]), f64(v[:C - n + i + 1]))
+                          for i in rows])
+    assert_close_out(got, ref, BF16_REL_L2, BF16_MAX_ABS, label)
+
+
+@pytest.mark.parametrize("n,C", [(2048, 2048), (16384, 16384), (2048, 16384)])
+def test_attention_prefill_full_sizes_sampled(n, C):
+    """The two prefill sizes of the 16384-token workload: the full sequence
+    (layers before the exit) and its 2048 text rows (after it), plus a
+    2048-query chunk at the end of the full cache."""
+    q, k, v = _qkv(n, C, seed=n + C)
+    out = _run(q, k, v)
+    rng = np.random.default_rng(n)
+    rows = sorted(set([0, 1, 127, 128, n - 129, n - 1] + rng.integers(0, n, 10).tolist()))
+    _sampled_rows(out, q, k, v, rows, f"prefill attention n={n} C={C} (sampled rows)")
+
+
+def test_attention_prefill_grouping_and_scale():
+    # 8 query heads on 2 KV heads: 40 queries make 160 per KV head
+    q, k, v = _qkv(40, 333, seed=6, Hq=8, Hkv=2)
+    out = _run(q, k, v, scale=0.05)
+    ref = O.attention(f64(q), f64(k), f64(v), scale=0.05)
+    assert_close_out(f64(out), ref, BF16_REL_L2, BF16_MAX_ABS, "prefill grouping and scale")
+
+
+def test_attention_prefill_is_deterministic():
+    q, k, v = _qkv(300, 700, seed=9)
+    a = _run(q, k, v)
+    b = _run(q, k, v)
+    assert torch.equal(a, b)
+
+
 def test_attention_grouping_and_scale():
     # 8 query heads on 2 KV heads and an explicit scale
     q, k, v = _qkv(2, 200, seed=5, Hq=8, Hkv=2)
@@ -79,6 +127,25 @@ def test_attention_on_compacted_cache_equals_masked_full_cache():
     out = _run(q, kc.cpu(), vc.cpu())
     ref = O.attention(f64(q), O.drop_visual_block(f64(k), wl.v0, wl.nv), O.drop_visual_block(f64(v), wl.v0, wl.nv))
     assert_close_out(f64(out), ref, BF16_REL_L2, BF16_MAX_ABS, "decode over the compacted cache")
+
+
+def test_attention_prefill_on_compacted_sequence():
+    """Prefill after the visual block has left: the compacted hidden rows'
+    queries over the compacted K and V (1552 - 1280 = 272 rows) equal the
+    oracle's attention on the full sequence's caches with the visual rows
+    removed."""
+    wl = W.STACK
+    C_full = wl.T
+    q, k, v = _qkv(C_full, C_full, seed=12)
+    dev = [t.to(DEV).view(C_full, -1) for t in (q, k, v)]
+    comp = [torch.empty(C_full - wl.nv, t.shape[1], dtype=torch.bfloat16, device=DEV) for t in dev]
+    for src, dst in zip(dev, comp):
+        dm.decomoe_drop_visual_block(src, dst, wl.v0, wl.nv)
+    qc, kc, vc = (comp[0].view(-1, HQ, D).cpu(), comp[1].view(-1, HKV, D).cpu(), comp[2].view(-1, HKV, D).cpu())
+    out = _run(qc, kc, vc)
+    drop = lambda t: O.drop_visual_block(f64(t), wl.v0, wl.nv)  # noqa: E731
+    ref = O.attention(drop(q), drop(k), drop(v))
+    assert_close_out(f64(out), ref, BF16_REL_L2, BF16_MAX_ABS, "prefill over the compacted sequence")
 
 
 def test_attention_rejects_unsupported_shapes():
