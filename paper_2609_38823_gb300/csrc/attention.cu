@@ -230,29 +230,40 @@ __global__ void __launch_bounds__(32 * ATT_CWARPS)
 
 // ------------------------------------------------------------------ prefill (tensor cores)
 // Many queries per KV head (the compacted sequence's prefill): flash-style
-// attention on tcgen05. CTA = (query head h, tile of 128 query rows). Per
-// block j of 128 keys: S = Q K_j^T (M = 128 queries, N = 128 keys, K = 128
-// features) into tensor memory; four warps (one query row per thread) take
-// the row's running maximum m and sum l, write p = exp(s - m) as bf16 into a
-// 128-byte-swizzled shared-memory tile (the next MMA's A operand) and scale
-// their fp32 output row by exp(m_old - m); then O_j = P V_j (N = 128
-// features, K = 128 keys, V pre-transposed so both operands are K-major)
-// into tensor memory, added to the row in registers. Warp 0 streams K_j and
-// V_j^T blocks by TMA into a two-stage ring; warp 1 issues the MMAs. Every
-// wait is bounded; on a timeout the CTA records DECOMOE_ERR_TIMEOUT, lets
-// its copies and MMAs land, frees its tensor memory and returns.
+// attention on tcgen05. A CTA takes one tile of 128 query rows for two query
+// heads of the same KV group, so each K and V block it streams serves both.
+// Per block j of 64 keys and head x: S_x = Q_x K_j^T (M = 128 queries, N = 64
+// keys, K = 128 features) into tensor memory; four warps per head (one query
+// row per thread) take the row maximum, write p = 2^(s*scale*log2e - m) as
+// bf16 into tensor memory (the A operand of the next product) and add p to
+// the row sum l; then O_x += P_x V_j (N = 128 features, K = 64 keys, V
+// transposed beforehand so that the B operand is K-major) accumulates in
+// tensor memory. The reference maximum m of a row moves only when the block
+// maximum exceeds it by more than 8 (a factor 256): then that row's O and l
+// are scaled by 2^(m_old - m_new) before the next product (otherwise p stays
+// below 256, well inside bf16 and fp32); the final output is O / l either
+// way. Tensor-core work of one head overlaps the other head's softmax: the
+// issue order is PV_0(j), S_0(j+1), PV_1(j), S_1(j+1). Warp 0 streams K_j and
+// V_j^T blocks by TMA into a four-stage ring; warp 1 issues the MMAs. Every
+// wait is bounded; on a timeout the CTA records DECOMOE_ERR_TIMEOUT, lets its
+// copies and MMAs land, frees its tensor memory and returns.
 constexpr int ATP_BM = 128;                 // query rows per CTA
-constexpr int ATP_BN = 128;                 // keys per block
-constexpr int ATP_HALF = 128 * 64 * 2;      // one 128-row x 64-column swizzled tile (16 KB)
-constexpr int ATP_THREADS = 192;
-constexpr int ATP_TMEM_COLS = 256;          // S (128 columns) and O_j (128 columns)
-constexpr size_t ATP_SMEM = 1024 + 2 * ATP_HALF /* Q */ + 2 * 2 * ATP_HALF /* K ring */ +
-                            2 * 2 * ATP_HALF /* V^T ring */ + 2 * ATP_HALF /* P */ + 16 * 8 + 16;
+constexpr int ATP_BN = 64;                  // keys per block
+constexpr int ATP_HEADS = 2;                // query heads per CTA (same KV head)
+constexpr int ATP_NST = 4;                  // K / V ring stages
+constexpr int ATP_QHALF = 128 * 64 * 2;     // Q: 128 rows x 64 features, 128-byte swizzle (16 KB)
+constexpr int ATP_KHALF = ATP_BN * 64 * 2;  // K block: 64 keys x 64 features (8 KB)
+constexpr int ATP_VT = 128 * ATP_BN * 2;    // V^T block: 128 features x 64 keys (16 KB)
+constexpr int ATP_STAGE = 2 * ATP_KHALF + ATP_VT;
+constexpr int ATP_THREADS = 64 + ATP_HEADS * 128;
+constexpr int ATP_TMEM_COLS = 512;          // per head: S [0,64), P [64,96), O [128,256)
+constexpr float ATP_RESCALE = 8.0f;         // log2 of the largest unnormalised p
+constexpr size_t ATP_SMEM = 1024 + ATP_HEADS * 2 * ATP_QHALF + ATP_NST * ATP_STAGE + 32 * 8 + 16;
 
 struct AttPreArgs {
   int64_t n, C;        // queries (the last n positions), keys
-  int Hq, Hkv;
-  float scale;
+  int Hq, group;       // query heads, query heads per KV head
+  float scale_log2;    // scale * log2(e)
   __nv_bfloat16* out;  // [n, Hq, D]
   int32_t* status;
   uint64_t limit_ns;
@@ -278,6 +289,42 @@ __global__ void __launch_bounds__(256)
   }
 }
 
+// D(tmem) (+)= A(tmem) * B(smem desc)^T: A is 128 rows (lanes) x 16 bf16
+// (8 columns, two elements per 32-bit column, the lower index in the low half).
+__device__ __forceinline__ void tc_mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                              uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
+      "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+      "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]),
+      "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]),
+      "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+__device__ __forceinline__ void tc_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+// Values loaded by tcgen05.ld are defined only after tcgen05.wait::ld: route
+// them through an empty asm placed after the wait so no use moves above it.
+template <int N>
+__device__ __forceinline__ void after_wait(uint32_t (&r)[N]) {
+#pragma unroll
+  for (int i = 0; i < N; ++i) asm volatile("" : "+r"(r[i]));
+}
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __global__ void __launch_bounds__(ATP_THREADS, 1)
     k_attn_prefill(const __grid_constant__ CUtensorMap tma_q, const __grid_constant__ CUtensorMap tma_k,
                    const __grid_constant__ CUtensorMap tma_vt, const AttPreArgs a) {
@@ -285,27 +332,27 @@ __global__ void __launch_bounds__(ATP_THREADS, 1)
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
   uint8_t* smem = smem_raw + pad;
-  const uint32_t sQ = raw + pad;                 // 2 halves (features 0-63, 64-127)
-  const uint32_t sK = sQ + 2 * ATP_HALF;         // [stage][half]
-  const uint32_t sV = sK + 4 * ATP_HALF;         // [stage][half of the keys]
-  const uint32_t sP = sV + 4 * ATP_HALF;         // [half of the keys]
-  uint8_t* pP = smem + (sP - sQ);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 12 * ATP_HALF);
-  volatile uint32_t* s_tmem = reinterpret_cast<volatile uint32_t*>(bars + 16);
+  const uint32_t sQ = raw + pad;                              // [head][feature half]
+  const uint32_t sKV = sQ + ATP_HEADS * 2 * ATP_QHALF;        // [stage]{K half 0, K half 1, V^T}
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + ATP_HEADS * 2 * ATP_QHALF + ATP_NST * ATP_STAGE);
+  volatile uint32_t* s_tmem = reinterpret_cast<volatile uint32_t*>(bars + 32);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
   const uint32_t bar0 = smem_u32(bars);
-  const uint32_t Q_BAR = bar0, S_FULL = bar0 + 8, P_FULL = bar0 + 16, O_FULL = bar0 + 24, O_EMPTY = bar0 + 32,
-                 DRAIN = bar0 + 40;
-  auto FULL = [&](int st) { return bar0 + 48u + 8u * st; };
-  auto EMPTY = [&](int st) { return bar0 + 64u + 8u * st; };
+  const uint32_t Q_BAR = bar0, DRAIN = bar0 + 8;
+  auto S_FULL = [&](int x) { return bar0 + 16u + 8u * x; };
+  auto P_FULL = [&](int x) { return bar0 + 32u + 8u * x; };
+  auto O_FINAL = [&](int x) { return bar0 + 48u + 8u * x; };
+  auto FULL = [&](int st) { return bar0 + 64u + 8u * st; };
+  auto EMPTY = [&](int st) { return bar0 + 96u + 8u * st; };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int G = a.Hq / a.Hkv;
+  const int npair = a.Hq / ATP_HEADS;
   const int ntile = static_cast<int>((a.n + ATP_BM - 1) / ATP_BM);
-  // heaviest tiles (most key blocks) first; the heads of a KV group adjacent
-  const int h = blockIdx.x % a.Hq;
-  const int qt = ntile - 1 - static_cast<int>(blockIdx.x / a.Hq);
-  const int g = h / G;
+  // heaviest tiles (most key blocks) first
+  const int hp = blockIdx.x % npair;
+  const int qt = ntile - 1 - static_cast<int>(blockIdx.x / npair);
+  const int h0 = hp * ATP_HEADS;
+  const int g = h0 / a.group;  // both heads read KV head g (the group size is even)
   const int64_t p0 = a.C - a.n + static_cast<int64_t>(qt) * ATP_BM;  // position of the tile's first row
   const int64_t last = p0 + ATP_BM - 1 < a.C - 1 ? p0 + ATP_BM - 1 : a.C - 1;
   const int nblk = static_cast<int>(last / ATP_BN) + 1;  // key blocks any row of the tile can see
@@ -313,12 +360,13 @@ __global__ void __launch_bounds__(ATP_THREADS, 1)
   if (threadIdx.x == 0) {
     *s_abort = 0;
     mbar_init(Q_BAR, 1);
-    mbar_init(S_FULL, 1);
-    mbar_init(P_FULL, 128);
-    mbar_init(O_FULL, 1);
-    mbar_init(O_EMPTY, 128);
     mbar_init(DRAIN, 1);
-    for (int st = 0; st < 2; ++st) {
+    for (int x = 0; x < ATP_HEADS; ++x) {
+      mbar_init(S_FULL(x), 1);
+      mbar_init(P_FULL(x), 128);
+      mbar_init(O_FINAL(x), 1);
+    }
+    for (int st = 0; st < ATP_NST; ++st) {
       mbar_init(FULL(st), 1);
       mbar_init(EMPTY(st), 1);
     }
@@ -333,8 +381,11 @@ __global__ void __launch_bounds__(ATP_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *s_tmem;
-  const uint32_t S_TM = tmem, O_TM = tmem + ATP_BN;
-  constexpr uint32_t IDESC = idesc_bf16_f32(ATP_BM, ATP_BN);
+  auto S_TM = [&](int x) { return tmem + 256u * x; };
+  auto P_TM = [&](int x) { return tmem + 256u * x + 64u; };
+  auto O_TM = [&](int x) { return tmem + 256u * x + 128u; };
+  constexpr uint32_t IDESC_S = idesc_bf16_f32(ATP_BM, ATP_BN);
+  constexpr uint32_t IDESC_O = idesc_bf16_f32(ATP_BM, ATT_D);
 
   if (warp == 0) {
     // ------------------------------------------------ TMA producer (lane 0)
@@ -344,23 +395,23 @@ __global__ void __launch_bounds__(ATP_THREADS, 1)
       tma_prefetch_desc(&tma_vt);
       bool ok = true;
       uint32_t armed = 0, armed_ph = 0;
-      mbar_arrive_expect_tx(Q_BAR, 2 * ATP_HALF);
+      mbar_arrive_expect_tx(Q_BAR, ATP_HEADS * 2 * ATP_QHALF);
       const int qrow0 = qt * ATP_BM;
-      tma_load_3d(sQ, &tma_q, Q_BAR, 0, h, qrow0);
-      tma_load_3d(sQ + ATP_HALF, &tma_q, Q_BAR, 64, h, qrow0);
+      for (int x = 0; x < ATP_HEADS; ++x)
+        for (int kb = 0; kb < 2; ++kb) tma_load_3d(sQ + (2 * x + kb) * ATP_QHALF, &tma_q, Q_BAR, 64 * kb, h0 + x, qrow0);
       for (int j = 0; j < nblk; ++j) {
-        const int st = j & 1;
-        const uint32_t ph = (j >> 1) & 1;
+        const int st = j % ATP_NST;
+        const uint32_t ph = (j / ATP_NST) & 1;
         if (!mbar_wait(EMPTY(st), ph ^ 1u, a.limit_ns, s_abort)) {
           ok = false;
           break;
         }
-        mbar_arrive_expect_tx(FULL(st), 4 * ATP_HALF);
+        mbar_arrive_expect_tx(FULL(st), ATP_STAGE);
         const int key0 = j * ATP_BN;
-        tma_load_3d(sK + (2 * st) * ATP_HALF, &tma_k, FULL(st), 0, g, key0);
-        tma_load_3d(sK + (2 * st + 1) * ATP_HALF, &tma_k, FULL(st), 64, g, key0);
-        tma_load_3d(sV + (2 * st) * ATP_HALF, &tma_vt, FULL(st), key0, 0, g);
-        tma_load_3d(sV + (2 * st + 1) * ATP_HALF, &tma_vt, FULL(st), key0 + 64, 0, g);
+        const uint32_t base = sKV + st * ATP_STAGE;
+        tma_load_3d(base, &tma_k, FULL(st), 0, g, key0);
+        tma_load_3d(base + ATP_KHALF, &tma_k, FULL(st), 64, g, key0);
+        tma_load_3d(base + 2 * ATP_KHALF, &tma_vt, FULL(st), key0, 0, g);
         armed |= 1u << st;
         armed_ph = (armed_ph & ~(1u << st)) | (ph << st);
       }
@@ -369,48 +420,67 @@ __global__ void __launch_bounds__(ATP_THREADS, 1)
         report_status(a.status, DECOMOE_ERR_TIMEOUT);
         int no_abort = 0;
         mbar_wait(Q_BAR, 0, a.limit_ns, &no_abort);
-        for (int st = 0; st < 2; ++st)
+        for (int st = 0; st < ATP_NST; ++st)
           if ((armed >> st) & 1u) mbar_wait(FULL(st), (armed_ph >> st) & 1u, a.limit_ns, &no_abort);
       }
     }
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer (lane 0)
     if (lane == 0) {
-      bool ok = mbar_wait(Q_BAR, 0, a.limit_ns, s_abort), issued = false;
-      for (int j = 0; ok && j < nblk; ++j) {
-        const int st = j & 1;
-        if (!mbar_wait(FULL(st), (j >> 1) & 1, a.limit_ns, s_abort)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        // S = Q K_j^T over the 128 features (two 64-column halves)
+      // S_x = Q_x K^T over the 128 features (two 64-feature halves)
+      auto issue_s = [&](int x, int st) {
+        const uint32_t base = sKV + st * ATP_STAGE;
 #pragma unroll
         for (int kb = 0; kb < 2; ++kb) {
-          const uint64_t ad = smem_desc_kmajor<64>(sQ + kb * ATP_HALF);
-          const uint64_t bd = smem_desc_kmajor<64>(sK + (2 * st + kb) * ATP_HALF);
+          const uint64_t ad = smem_desc_kmajor<64>(sQ + (2 * x + kb) * ATP_QHALF);
+          const uint64_t bd = smem_desc_kmajor<64>(base + kb * ATP_KHALF);
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk) tc_mma_f16(S_TM, ad + 2u * kk, bd + 2u * kk, IDESC, (kb | kk) != 0 ? 1u : 0u);
+          for (int kk = 0; kk < 4; ++kk)
+            tc_mma_f16(S_TM(x), ad + 2u * kk, bd + 2u * kk, IDESC_S, (kb | kk) != 0 ? 1u : 0u);
         }
-        tc_commit(S_FULL);
+      };
+      // O_x += P_x V_j over the block's 64 keys
+      auto issue_pv = [&](int x, int st, bool acc) {
+        const uint64_t bd = smem_desc_kmajor<64>(sKV + st * ATP_STAGE + 2 * ATP_KHALF);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          tc_mma_f16_ts(O_TM(x), P_TM(x) + 8u * kk, bd + 2u * kk, IDESC_O, (acc || kk > 0) ? 1u : 0u);
+      };
+      bool ok = mbar_wait(Q_BAR, 0, a.limit_ns, s_abort) && mbar_wait(FULL(0), 0, a.limit_ns, s_abort);
+      bool issued = false;
+      if (ok) {
+        tc_fence_after();
+        for (int x = 0; x < ATP_HEADS; ++x) {
+          issue_s(x, 0);
+          tc_commit(S_FULL(x));
+        }
         issued = true;
-        // O_j = P V_j once the softmax rows have written P and read O_{j-1}
-        if (!mbar_wait(P_FULL, j & 1, a.limit_ns, s_abort) ||
-            (j > 0 && !mbar_wait(O_EMPTY, (j - 1) & 1, a.limit_ns, s_abort))) {
-          ok = false;
-          break;
+      }
+      for (int j = 0; ok && j < nblk; ++j) {
+        const int st = j % ATP_NST;
+        for (int x = 0; x < ATP_HEADS; ++x) {
+          if (!mbar_wait(P_FULL(x), j & 1, a.limit_ns, s_abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          issue_pv(x, st, j > 0);
+          if (x == ATP_HEADS - 1) tc_commit(EMPTY(st));  // K_j and V_j read by every product
+          if (j + 1 < nblk) {
+            const int st1 = (j + 1) % ATP_NST;
+            if (x == 0) {
+              if (!mbar_wait(FULL(st1), ((j + 1) / ATP_NST) & 1, a.limit_ns, s_abort)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+            }
+            issue_s(x, st1);
+            tc_commit(S_FULL(x));
+          } else {
+            tc_commit(O_FINAL(x));
+          }
         }
-        tc_fence_after();
-        fence_proxy_async_smem();  // P came through the generic proxy
-#pragma unroll
-        for (int kb = 0; kb < 2; ++kb) {
-          const uint64_t ad = smem_desc_kmajor<64>(sP + kb * ATP_HALF);
-          const uint64_t bd = smem_desc_kmajor<64>(sV + (2 * st + kb) * ATP_HALF);
-#pragma unroll
-          for (int kk = 0; kk < 4; ++kk) tc_mma_f16(O_TM, ad + 2u * kk, bd + 2u * kk, IDESC, (kb | kk) != 0 ? 1u : 0u);
-        }
-        tc_commit(O_FULL);
-        tc_commit(EMPTY(st));
       }
       if (!ok) {
         *s_abort = 1;
@@ -423,95 +493,99 @@ __global__ void __launch_bounds__(ATP_THREADS, 1)
       }
     }
   } else {
-    // ------------------------------------------------ softmax and output rows
+    // ------------------------------------------------ softmax rows
+    const int x = (warp - 2) >> 2;          // head of this warp
     const int q = warp & 3;                 // tensor-memory lane quarter of this warp
     const int r = q * 32 + lane;            // query row of the tile
-    const int64_t qpos = p0 + r;            // its position
+    const int64_t climit = a.C - 1;
+    const int64_t qlim = p0 + r < climit ? p0 + r : climit;                    // last visible key of the row
+    const int64_t wlim = p0 + q * 32 < climit ? p0 + q * 32 : climit;          // smallest of the warp's rows
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
-    float o[ATT_D];
-#pragma unroll
-    for (int d = 0; d < ATT_D; ++d) o[d] = 0.f;
-    float m = -FLT_MAX, l = 0.f;
+    const float sl2 = a.scale_log2;
+    float m = 0.f, l = 0.f;
     bool ok = true;
     for (int j = 0; j < nblk; ++j) {
-      if (!__all_sync(0xffffffffu, mbar_wait(S_FULL, j & 1, a.limit_ns, s_abort))) {  // warp-uniform tensor-memory loads
+      if (!__all_sync(0xffffffffu, mbar_wait(S_FULL(x), j & 1, a.limit_ns, s_abort))) {  // warp-uniform loads
         ok = false;
         break;
       }
       tc_fence_after();
       const int64_t key0 = static_cast<int64_t>(j) * ATP_BN;
-      // pass 1: the block's maximum over visible keys
-      float bmax = -FLT_MAX;
+      uint32_t sv[ATP_BN];
+      tmem_ld32(S_TM(x) + lane_off, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
+      tmem_ld32(S_TM(x) + lane_off + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
+      tc_wait_ld();
+      after_wait(sv);
+      if (key0 + ATP_BN - 1 > wlim) {  // the causal edge or the end of the keys crosses this warp's rows
+        const int64_t d = qlim - key0;
+        const int lim = d < 0 ? -1 : static_cast<int>(d);  // d < 64 here
 #pragma unroll
-      for (int c = 0; c < ATP_BN / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld32(S_TM + lane_off + 32 * c, v);
-        tc_wait_ld();
+        for (int c = 0; c < ATP_BN; ++c)
+          if (c > lim) sv[c] = __float_as_uint(-INFINITY);
+      }
+      float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const int64_t kp = key0 + 32 * c + i;
-          if (kp <= qpos && kp < a.C) bmax = fmaxf(bmax, __uint_as_float(v[i]) * a.scale);
+      for (int c = 0; c < ATP_BN; ++c) mx[c & 3] = fmaxf(mx[c & 3], __uint_as_float(sv[c]));
+      const float m_blk = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * sl2;
+      float factor = 1.0f;
+      if (j == 0) {
+        m = m_blk;  // key 0 is visible to every row
+      } else if (m_blk > m + ATP_RESCALE) {
+        factor = ex2_approx(m - m_blk);
+        m = m_blk;
+        l *= factor;
+      }
+      if (__any_sync(0xffffffffu, factor != 1.0f)) {
+        // the previous product into O has completed (S_FULL is committed after it)
+#pragma unroll
+        for (int c = 0; c < ATT_D / 32; ++c) {
+          uint32_t ov[32];
+          tmem_ld32(O_TM(x) + lane_off + 32 * c, ov);
+          tc_wait_ld();
+          after_wait(ov);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) ov[i] = __float_as_uint(__uint_as_float(ov[i]) * factor);
+          tmem_st32(O_TM(x) + lane_off + 32 * c, ov);
         }
       }
-      const float m_new = fmaxf(m, bmax);
-      const float alpha = m == -FLT_MAX ? 0.f : __expf(m - m_new);
-      // pass 2: p = exp(s - m_new) as bf16 into the swizzled P tile, and the sum
-      float psum = 0.f;
+      float ls[4] = {0.f, 0.f, 0.f, 0.f};
+      uint32_t pk[32];
 #pragma unroll
-      for (int c = 0; c < ATP_BN / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld32(S_TM + lane_off + 32 * c, v);
-        tc_wait_ld();
-        uint32_t pk[16];
-#pragma unroll
-        for (int i = 0; i < 32; i += 2) {
-          const int64_t kp = key0 + 32 * c + i;
-          const float e0 = (kp <= qpos && kp < a.C) ? __expf(__uint_as_float(v[i]) * a.scale - m_new) : 0.f;
-          const float e1 = (kp + 1 <= qpos && kp + 1 < a.C) ? __expf(__uint_as_float(v[i + 1]) * a.scale - m_new) : 0.f;
-          psum += e0 + e1;
-          pk[i / 2] = pack_bf16x2(e0, e1);
-        }
-        // columns 32c .. 32c + 31: half kb = c / 2, 16-byte chunks (c % 2) * 4 .. + 3
-        const int kb = c >> 1;
-        uint8_t* rowp = pP + kb * ATP_HALF + r * 128;
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int chunk = (c & 1) * 4 + u;
-          *reinterpret_cast<uint4*>(rowp + ((chunk ^ (r & 7)) << 4)) =
-              make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
-        }
+      for (int c = 0; c < ATP_BN; c += 2) {
+        const float e0 = ex2_approx(fmaf(__uint_as_float(sv[c]), sl2, -m));
+        const float e1 = ex2_approx(fmaf(__uint_as_float(sv[c + 1]), sl2, -m));
+        ls[(c >> 1) & 3] += e0 + e1;
+        pk[c >> 1] = pack_bf16x2(e0, e1);
       }
-      l = l * alpha + psum;
-      m = m_new;
-      fence_proxy_async_smem();
+      l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+      tmem_st32(P_TM(x) + lane_off, pk);
+      tc_wait_st();
       tc_fence_before();
-      mbar_arrive(P_FULL);
-      if (!__all_sync(0xffffffffu, mbar_wait(O_FULL, j & 1, a.limit_ns, s_abort))) {
-        ok = false;
-        break;
-      }
+      mbar_arrive(P_FULL(x));
+    }
+    if (ok && __all_sync(0xffffffffu, mbar_wait(O_FINAL(x), 0, a.limit_ns, s_abort))) {
       tc_fence_after();
+      const float inv = 1.0f / l;
+      const int64_t row = static_cast<int64_t>(qt) * ATP_BM + r;
+      uint4* dst = reinterpret_cast<uint4*>(a.out + (row * a.Hq + h0 + x) * ATT_D);
 #pragma unroll
       for (int c = 0; c < ATT_D / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld32(O_TM + lane_off + 32 * c, v);
+        uint32_t ov[32];
+        tmem_ld32(O_TM(x) + lane_off + 32 * c, ov);
         tc_wait_ld();
+        after_wait(ov);
+        if (row < a.n) {
 #pragma unroll
-        for (int i = 0; i < 32; ++i) o[32 * c + i] = fmaf(o[32 * c + i], alpha, __uint_as_float(v[i]));
+          for (int u = 0; u < 4; ++u) {
+            const float* o = reinterpret_cast<const float*>(&ov[8 * u]);
+            dst[4 * c + u] = make_uint4(pack_bf16x2(o[0] * inv, o[1] * inv), pack_bf16x2(o[2] * inv, o[3] * inv),
+                                        pack_bf16x2(o[4] * inv, o[5] * inv), pack_bf16x2(o[6] * inv, o[7] * inv));
+          }
+        }
       }
-      tc_fence_before();
-      mbar_arrive(O_EMPTY);
-    }
-    if (!ok) {
+    } else {
       *s_abort = 1;
       report_status(a.status, DECOMOE_ERR_TIMEOUT);
-    } else if (qt * ATP_BM + r < a.n) {
-      const float inv = 1.0f / l;
-      uint4* dst = reinterpret_cast<uint4*>(a.out + ((static_cast<int64_t>(qt) * ATP_BM + r) * a.Hq + h) * ATT_D);
-#pragma unroll
-      for (int c = 0; c < ATT_D / 8; ++c)
-        dst[c] = make_uint4(pack_bf16x2(o[8 * c] * inv, o[8 * c + 1] * inv), pack_bf16x2(o[8 * c + 2] * inv, o[8 * c + 3] * inv),
-                            pack_bf16x2(o[8 * c + 4] * inv, o[8 * c + 5] * inv), pack_bf16x2(o[8 * c + 6] * inv, o[8 * c + 7] * inv));
     }
   }
   pdl_trigger();
@@ -563,6 +637,8 @@ int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void*
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const float sc = scale > 0.f ? scale : 1.0f / sqrtf(static_cast<float>(D));
   if (att_use_prefill(n, Hq, Hkv)) {
+    DM_ARG_CHECK(G % ATP_HEADS == 0, "attention: prefill sizes need an even number of query heads per KV head (%d)",
+                 G);
     // V transposed (keys contiguous) so that P V_j takes K-major operands
     const int64_t C_pad = att_c_pad(C);
     __nv_bfloat16* vt = static_cast<__nv_bfloat16*>(ws);
@@ -575,7 +651,7 @@ int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void*
     const uint64_t sk[2] = {static_cast<uint64_t>(D) * 2, static_cast<uint64_t>(Hkv) * D * 2};
     const uint64_t dv[3] = {static_cast<uint64_t>(C_pad), static_cast<uint64_t>(D), static_cast<uint64_t>(Hkv)};
     const uint64_t sv[2] = {static_cast<uint64_t>(C_pad) * 2, static_cast<uint64_t>(D) * C_pad * 2};
-    const uint32_t bq[3] = {64, 1, ATP_BM}, bk[3] = {64, 1, ATP_BN}, bv[3] = {64, ATT_D, 1};
+    const uint32_t bq[3] = {64, 1, ATP_BM}, bk[3] = {64, 1, ATP_BN}, bv[3] = {ATP_BN, ATT_D, 1};
     DM_RET(make_tmap_bf16_3d(&tq, q, dq, sq, bq));
     DM_RET(make_tmap_bf16_3d(&tk, k_cache, dk, sk, bk));
     DM_RET(make_tmap_bf16_3d(&tv, vt, dv, sv, bv));
@@ -583,16 +659,17 @@ int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void*
     pa.n = n;
     pa.C = C;
     pa.Hq = Hq;
-    pa.Hkv = Hkv;
-    pa.scale = sc;
+    pa.group = G;
+    pa.scale_log2 = sc * 1.4426950408889634f;
     pa.out = static_cast<__nv_bfloat16*>(out);
     pa.status = status_dev;
     pa.limit_ns = static_cast<uint64_t>(wait_limit_ns());
     const int64_t ntile = (n + ATP_BM - 1) / ATP_BM;
-    DM_ARG_CHECK(ntile * Hq < 0x7fffffffLL, "attention: too many query tiles");
+    DM_ARG_CHECK(ntile * (Hq / ATP_HEADS) < 0x7fffffffLL, "attention: too many query tiles");
     DM_CUDA_CHECK(cudaFuncSetAttribute(k_attn_prefill, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(ATP_SMEM)));
-    DM_CUDA_CHECK(launch_pdl(k_attn_prefill, dim3(static_cast<unsigned>(ntile * Hq)), dim3(ATP_THREADS), ATP_SMEM, s,
+    DM_CUDA_CHECK(launch_pdl(k_attn_prefill, dim3(static_cast<unsigned>(ntile * (Hq / ATP_HEADS))), dim3(ATP_THREADS),
+                             ATP_SMEM, s,
                              tq, tk, tv, pa));
     return DECOMOE_OK;
   }
