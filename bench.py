@@ -221,6 +221,14 @@ class Buffers:
         self.ready = torch.zeros(dm.decomoe_expert_swiglu_ready_ints(R, E), dtype=torch.int32, device=dev)
 
 
+def layer_gathers(R):
+    """Whether the layer's one-launch expert FFN also does the dispatch's row
+    gather at R routed rows (from 8192 rows up to the one-launch limit of
+    32768; above it the layer gathers in the dispatch and runs the two expert
+    GEMMs as separate launches)."""
+    return 8192 <= R <= 32768
+
+
 def run_step(dm, wl, L, B, K, v0, nv, text, ev=None):
     """One pass of the hot path. Without events: one C-ABI call, the layer
     (with its output's visual-block removal when text is given), K fixed and
@@ -236,7 +244,7 @@ def run_step(dm, wl, L, B, K, v0, nv, text, ev=None):
     # a1 + a2 (Eq. 11) + a4 + a5: router logits, routing with the activated
     # mass, dispatch (from 8192 routed rows the layer leaves the row gather to
     # the expert launch, and so does this)
-    gather = L.x.shape[0] * k >= 8192
+    gather = layer_gathers(L.x.shape[0] * k)
     dm.decomoe_router_route_dispatch(L.x, L.w_r, L.bias, B.logits, K, k, B.idx, B.w, B.counts[:K], B.offsets[:K + 1],
                                      B.perm, B.inv, None if gather else B.x_perm, B.rrd_ws, mass_out=B.mass,
                                      status=B.status)
@@ -385,7 +393,7 @@ def ours(args, ws, rank, local):
     D = statistics.mean(Ds)
     ffn_flops = 6.0 * R * wl.d * wl.m
     useful_flops = ffn_flops + 2.0 * T * wl.d * wl.E
-    ffn_bytes = algo_bytes_ffn(wl, R, D, T if R >= 8192 else None)
+    ffn_bytes = algo_bytes_ffn(wl, R, D, T if layer_gathers(R) else None)
     ffn_tflops = ffn_flops / (ffn_ms * 1e-3) / 1e12
     ffn_gbs = ffn_bytes / (ffn_ms * 1e-3) / 1e9
     t_compute = ffn_flops / (pk["bf16_tflops"] * 1e12)
@@ -535,7 +543,7 @@ def run_sweep(args, dm, wl, layers, B, text, ws, pk):
         ffn = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
         D = int((B.counts[:K] > 0).sum())
         ffn_fl = 6.0 * R * wl.d * wl.m
-        ffn_by = algo_bytes_ffn(wl, R, D, T if R >= 8192 else None)
+        ffn_by = algo_bytes_ffn(wl, R, D, T if layer_gathers(R) else None)
         out.append({"mode": "fixed (eager launches)", "K": K, "tokens_per_s": round(T * n / (ms / 1e3), 1),
                     "ms_per_step": round(ms / n, 4), "ffn_ms": round(ffn, 4),
                     "ffn_tflops": round(ffn_fl / (ffn * 1e-3) / 1e12, 2),
