@@ -542,12 +542,17 @@ DECOMOE_API int decomoe_moe_layer_workspace_layout(int64_t T, int d, int E, int 
  *   C - n + i and sees keys 0 .. C - n + i; query head h reads KV head
  *   h / (Hq / Hkv). scale <= 0 means 1 / sqrt(D). fp32 scores, softmax and
  *   accumulation; out rounded to bf16.
- *   Decode sizes: n * (Hq / Hkv) <= 64 queries per KV head (split-key
- *   partials over 128-key chunks and a combine in chunk order; deterministic).
- *   Prefill sizes (more queries per KV head, n = C or a chunk n < C): V is
- *   transposed into the workspace, then one tensor-core CTA per (query head,
- *   128-query tile) runs the online softmax over 128-key blocks up to its
- *   causal limit (P rounded to bf16 before the P V product; deterministic).
+ *   Decode sizes: n * (Hq / Hkv) <= 64 queries per KV head: one launch;
+ *   each block streams a range of keys and keeps the online softmax of up to
+ *   32 queries of its KV head, and the ranges of a head (one thread-block
+ *   cluster of up to 16 blocks) are merged in key order through the
+ *   cluster's shared memory (deterministic). No workspace (0 bytes; ws may
+ *   be null).
+ *   Prefill sizes (more queries per KV head, n = C or a chunk n < C; Hq / Hkv
+ *   even): V is transposed into the workspace, then one tensor-core CTA per
+ *   (pair of query heads, 128-query tile) runs the online softmax over 64-key
+ *   blocks up to its causal limit (P rounded to bf16 before the P V product;
+ *   deterministic).
  *   ws: decomoe_attention_workspace_bytes(n, C, Hq, Hkv, D) bytes, 16-byte
  *   aligned. A wait that runs past the time limit records
  *   DECOMOE_ERR_TIMEOUT in status_dev (may be null).

@@ -9,13 +9,11 @@
 // D = 128. Query i is at position C - n + i and sees keys 0 .. C - n + i;
 // query head h reads KV head h / (Hq / Hkv).
 //
-// Decode sizes (few queries per KV head): split-key partials. CTA (s, g)
-// takes one chunk of keys (32 to 128) of KV head g and every query of its
-// head group: K and V chunk rows staged in shared memory (cp.async), one warp
-// per query, scores and weighted values on CUDA cores with fp32 accumulation;
-// the chunk's softmax maximum, sum and weighted value row go out as partials
-// and a second launch combines the partials of each query in a fixed order
-// (deterministic).
+// Decode sizes (few queries per KV head): one launch of split-key blocks on
+// warp-level tensor-core products, the splits of a head merged through the
+// shared memory of their thread-block cluster (below). Prefill sizes: a
+// transpose of V, then the tcgen05 flash-style kernel (further below).
+#include <atomic>
 #include <cfloat>
 
 #include "decomoe_internal.cuh"
@@ -23,209 +21,424 @@
 namespace decomoe {
 
 constexpr int ATT_D = 128;
-constexpr int ATT_CH_MAX = 128;                 // keys per split (at most)
-constexpr int ATT_THREADS = 256;                // 8 warps: one query at a time each
-constexpr int ATT_KROW = ATT_D * 2 + 16;        // padded K row in shared memory (bytes): conflict-free 16-byte reads
-constexpr int ATT_MAXQ = 64;                    // queries per KV head handled by one split CTA
+constexpr int ATT_MAXQ = 64;                    // queries per KV head taken by the decode kernel
 constexpr int ATT_PROW = ATT_D + 4;             // floats per partial row: acc[D], m, l, 2 unused (16-byte rows)
 
-struct AttArgs {
+// ------------------------------------------------------------------ decode sizes
+// Few queries per KV head (a decode step over the cache, or a short chunk):
+// block (split s, KV head g, query tile group z) streams keys
+// [s * kps, (s + 1) * kps) of head g through a three-chunk TMA ring of 128
+// keys (128-byte swizzled 64-feature halves; rows past C read as zero) and
+// runs the online softmax of up to 32 of the group's
+// nq = n * Hq / Hkv queries on the tensor cores with warp-level
+// mma.m16n8k16 (bf16 in, fp32 accumulate): per 16 keys a warp computes
+// S = Q K^T for 16 query rows, turns the scores into bf16 weights in
+// registers (the accumulator layout of one product is the operand layout of
+// the next) and adds P V into its output tile. The eight warps of a block take
+// 16 keys of each chunk apiece; their states are merged in warp order into
+// the block's partial (m, l, unnormalised output) per query, kept in shared
+// memory. The splits of one (KV head, query tile group) form one thread-block
+// cluster: after a cluster barrier, block r merges queries r, r + nsplit, ...
+// over the blocks in rank order, reading their partials through distributed
+// shared memory, and stores the output; a second barrier keeps every block's
+// shared memory alive until it has been read. No workspace, no counters, and
+// the result does not depend on timing.
+constexpr int ATD_WARPS = 8;
+constexpr int ATD_CH = 16 * ATD_WARPS;          // keys per staged chunk (16 per warp)
+constexpr int ATD_THREADS = 32 * ATD_WARPS;
+constexpr int ATD_ROW = ATT_D * 2 + 16;         // padded query row (bytes): conflict-free ldmatrix
+constexpr int ATD_QT = 2;                       // 16-row query tiles per block (at most)
+constexpr int ATD_HALF = ATD_CH * 64 * 2;       // 128 keys x 64 features, 128-byte swizzle (16 KB)
+constexpr int ATD_STAGE = 4 * ATD_HALF;         // K and V halves of one chunk
+constexpr int ATD_NST = 3;                      // chunks in flight
+constexpr int ATD_PART = ATD_QT * 16 * ATT_PROW * 4;  // the block's partial rows (bytes)
+constexpr size_t ATD_SMEM =
+    1024 + static_cast<size_t>(ATD_NST) * ATD_STAGE + ATD_QT * 16 * ATD_ROW + ATD_PART + 8 * ATD_NST + 16;
+constexpr int ATD_OROW = ATT_D + 4;             // floats per row of the warp merge (padded)
+static_assert(ATD_WARPS * ATD_QT * 16 * (ATD_OROW + 2) * 4 <= ATD_NST * ATD_STAGE, "warp merge fits in the ring");
+
+struct AttDecArgs {
   const uint4* q;   // [n, Hq, D]
   const uint4* k;   // [C, Hkv, D]
   const uint4* v;
   int64_t n, C;
-  int Hq, Hkv, nsplit, chunk;
-  float scale;
-  float* part;      // [nsplit][Hkv][nq][ATT_PROW]: acc[D], m, l
+  int Hq, Hkv, kps; // keys per block; the cluster (grid.x) is the head's splits
+  float sl2;        // scale * log2(e)
+  __nv_bfloat16* out;
+  int32_t* status;
+  uint64_t limit_ns;
 };
 
-__host__ __device__ constexpr size_t att_split_smem() {
-  return static_cast<size_t>(ATT_CH_MAX) * ATT_KROW + static_cast<size_t>(ATT_CH_MAX) * ATT_D * 2 +
-         static_cast<size_t>(ATT_MAXQ) * ATT_D * 2;
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ float att_ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+// Four 8x8 bf16 matrices from shared memory; thread t gives the address of
+// row t % 8 of matrix t / 8 and receives (row t / 4, columns 2 (t % 4), +1)
+// of each (with .trans: of each matrix transposed).
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Address of the same shared-memory location in block `rank` of the cluster.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float ld_dsmem_f32(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+  return v;
+}
+// Every thread of every block of the cluster: writes before it (shared and
+// global) are visible to the cluster's blocks after it.
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// D (16x8 fp32) += A (16x16 bf16, row) * B (16x8 bf16, col)
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                               uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// Keys per split: 128 when that already gives a CTA per SM, else smaller
-// chunks (multiples of 32) so that short caches still spread over the SMs.
-static int att_chunk(int64_t C, int Hkv) {
-  const int64_t want = std::max<int64_t>(1, sm_count() / std::max(1, Hkv));
-  int64_t ch = (C + want - 1) / want;
-  ch = (ch + 31) / 32 * 32;
-  return static_cast<int>(std::min<int64_t>(ATT_CH_MAX, std::max<int64_t>(32, ch)));
-}
-
-// nq = n * (Hq / Hkv) <= ATT_MAXQ queries of KV head g against one key chunk
-// (query qi = i * G + j is head g * G + j of token i). Warp w takes queries
-// w, w + 8, ...: lane l owns keys l, l + 32, ... for the scores (the query's
-// 32-feature slices held in registers, the key rows read from shared
-// memory), then features 4l .. 4l + 3 for the weighted value rows (each key's
-// weight passed from its lane by a shuffle).
-__global__ void __launch_bounds__(ATT_THREADS)
-    k_attn_split(const AttArgs a) {
-  pdl_enter();
-  extern __shared__ uint8_t smem[];
+template <int QT>
+__global__ void __launch_bounds__(ATD_THREADS)
+    k_attn_dec(const __grid_constant__ CUtensorMap tma_k, const __grid_constant__ CUtensorMap tma_v,
+               const AttDecArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
+  uint8_t* sKV = smem_raw + pad;                                 // [NST]{K lo, K hi, V lo, V hi}
+  uint8_t* sQ = sKV + ATD_NST * ATD_STAGE;                       // [QT * 16][ROW]
+  float* s_part = reinterpret_cast<float*>(sQ + ATD_QT * 16 * ATD_ROW);  // [QT*16][PROW]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(s_part) + ATD_PART);
+  volatile int* s_abort = reinterpret_cast<volatile int*>(bars + ATD_NST);
+  const uint32_t sKVa = smem_u32(sKV);
+  const uint32_t bar0 = smem_u32(bars);
   const int s = blockIdx.x, g = blockIdx.y;
   const int G = a.Hq / a.Hkv;
   const int nq = static_cast<int>(a.n) * G;
+  const int qbase = static_cast<int>(blockIdx.z) * ATD_QT * 16;  // first query row of this block
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  uint8_t* sK = smem;                                                          // [CH][KROW]
-  const __nv_bfloat16* sV = reinterpret_cast<const __nv_bfloat16*>(sK + ATT_CH_MAX * ATT_KROW);  // [CH][D]
-  uint4* sQ = reinterpret_cast<uint4*>(sK + ATT_CH_MAX * ATT_KROW + ATT_CH_MAX * ATT_D * 2);     // [nq][D] bf16
-  const int64_t c0 = static_cast<int64_t>(s) * a.chunk;
-  const int nk = static_cast<int>(a.C - c0 < a.chunk ? a.C - c0 : a.chunk);
+  const int grp = lane >> 2, tig = lane & 3;
   constexpr int VPR = ATT_D / 8;  // 16-byte vectors per head row
-  // stage this chunk's K and V rows of head g (16-byte copies, all in flight)
-  for (int i = tid; i < nk * VPR; i += ATT_THREADS) {
-    const int r = i / VPR, c = i - r * VPR;
-    const int64_t src = ((c0 + r) * a.Hkv + g) * VPR + c;
-    cp_async16(smem_u32(sK + r * ATT_KROW + c * 16), a.k + src);
-    cp_async16(smem_u32(const_cast<__nv_bfloat16*>(sV) + r * ATT_D + c * 8), a.v + src);
+  const int64_t k0 = static_cast<int64_t>(s) * a.kps;
+  const int64_t k1 = k0 + a.kps < a.C ? k0 + a.kps : a.C;
+  const int nch = static_cast<int>((k1 - k0 + ATD_CH - 1) / ATD_CH);
+  if (tid == 0) {
+    *s_abort = 0;
+    for (int st = 0; st < ATD_NST; ++st) mbar_init(bar0 + 8u * st, 1);
+    fence_mbar_init();
+    tma_prefetch_desc(&tma_k);
+    tma_prefetch_desc(&tma_v);
   }
-  // and the group's query rows (query qi = i * G + j is head g * G + j of token i)
-  for (int i = tid; i < nq * VPR; i += ATT_THREADS) {
-    const int qi = i / VPR, c = i - qi * VPR;
-    const int ti = qi / G, hj = qi - ti * G;
-    cp_async16(smem_u32(sQ + i), a.q + (static_cast<int64_t>(ti) * a.Hq + g * G + hj) * VPR + c);
+  __syncthreads();
+  pdl_wait();  // q, K and V are ready
+  // chunk c into stage st: K and V, features 0-63 and 64-127 (keys past C read as zero)
+  auto issue = [&](int c, int st) {
+    const uint32_t bar = bar0 + 8u * st;
+    const uint32_t base = sKVa + st * ATD_STAGE;
+    const int key0 = static_cast<int>(k0) + c * ATD_CH;
+    mbar_arrive_expect_tx(bar, ATD_STAGE);
+    tma_load_3d(base, &tma_k, bar, 0, g, key0);
+    tma_load_3d(base + ATD_HALF, &tma_k, bar, 64, g, key0);
+    tma_load_3d(base + 2 * ATD_HALF, &tma_v, bar, 0, g, key0);
+    tma_load_3d(base + 3 * ATD_HALF, &tma_v, bar, 64, g, key0);
+  };
+  int issued = nch < ATD_NST ? nch : ATD_NST;  // chunks whose copies were requested (thread 0)
+  if (tid == 0)
+    for (int c = 0; c < issued; ++c) issue(c, c);
+
+  // query rows (zero rows past the group's queries)
+  for (int i = tid; i < QT * 16 * VPR; i += ATD_THREADS) {
+    const int r = i / VPR, c = i - r * VPR;
+    const int qi = qbase + r;
+    uint8_t* dst = sQ + r * ATD_ROW + c * 16;
+    if (qi < nq) {
+      const int ti = qi / G, hj = qi - ti * G;
+      cp_async16(smem_u32(dst), a.q + (static_cast<int64_t>(ti) * a.Hq + g * G + hj) * VPR + c);
+    } else {
+      *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
+    }
   }
   cp_async_wait_all();
-  __syncthreads();
-  float* part = a.part + (static_cast<int64_t>(s) * a.Hkv + g) * nq * ATT_PROW;
-  for (int qi = warp; qi < nq; qi += ATT_THREADS / 32) {
-    const int ti = qi / G;
-    const uint4* qrow = sQ + qi * VPR;
-    const int64_t last = a.C - a.n + ti;  // the query's position: keys up to it are visible
-    // scores of keys lane, lane + 32, lane + 64, lane + 96
-    float sc[ATT_CH_MAX / 32];
+  __syncthreads();  // the query rows are in place
+
+  // last visible key of this thread's two rows in each query tile
+  int64_t lim[QT][2];
 #pragma unroll
-    for (int u = 0; u < ATT_CH_MAX / 32; ++u) sc[u] = 0.f;
+  for (int qt = 0; qt < QT; ++qt)
 #pragma unroll
-    for (int c4 = 0; c4 < VPR; c4 += 4) {
-      // 32 features of the query (four 16-byte vectors, the same for every lane)
-      float qf[32];
+    for (int h = 0; h < 2; ++h) {
+      const int qi = qbase + qt * 16 + grp + 8 * h;
+      lim[qt][h] = qi < nq ? a.C - a.n + qi / G : a.C - 1;
+    }
+  float m[QT][2], l[QT][2], o[QT][16][4];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const uint4 u = qrow[c4 + c];
-        qf[8 * c + 0] = bf16_lo(u.x); qf[8 * c + 1] = bf16_hi(u.x);
-        qf[8 * c + 2] = bf16_lo(u.y); qf[8 * c + 3] = bf16_hi(u.y);
-        qf[8 * c + 4] = bf16_lo(u.z); qf[8 * c + 5] = bf16_hi(u.z);
-        qf[8 * c + 6] = bf16_lo(u.w); qf[8 * c + 7] = bf16_hi(u.w);
+  for (int qt = 0; qt < QT; ++qt) {
+    m[qt][0] = m[qt][1] = -INFINITY;
+    l[qt][0] = l[qt][1] = 0.f;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) o[qt][j][0] = o[qt][j][1] = o[qt][j][2] = o[qt][j][3] = 0.f;
+  }
+  const uint32_t sQa = smem_u32(sQ);
+  bool ok = true;
+  int c_fail = nch;  // first chunk whose wait ran out
+  for (int c = 0; c < nch; ++c) {
+    const int buf = c % ATD_NST;
+    ok = ok && __all_sync(0xffffffffu, mbar_wait(bar0 + 8u * buf, (c / ATD_NST) & 1, a.limit_ns, s_abort));
+    if (!ok && c_fail == nch) c_fail = c;
+    const uint32_t sKa = sKVa + buf * ATD_STAGE;  // K halves; V halves follow
+    const uint32_t sVa = sKa + 2 * ATD_HALF;
+    const int64_t kw = k0 + static_cast<int64_t>(c) * ATD_CH + 16 * warp;  // this warp's first key
+    if (ok && kw < k1) {
+      // S = Q K^T for this warp's 16 keys (two 8-key n-tiles), per query tile
+      float sc[QT][2][4];
+#pragma unroll
+      for (int qt = 0; qt < QT; ++qt)
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt) sc[qt][nt][0] = sc[qt][nt][1] = sc[qt][nt][2] = sc[qt][nt][3] = 0.f;
+      const int mi = lane >> 3, rr = lane & 7;
+#pragma unroll
+      for (int ks = 0; ks < ATT_D / 16; ++ks) {
+        uint32_t b00, b01, b10, b11;  // n-tile 0 (keys 0-7) and 1 (keys 8-15), features ks*16 + 0-7 / 8-15
+        {
+          const int key = 16 * warp + (mi >> 1) * 8 + rr, f = ks * 16 + (mi & 1) * 8;
+          ldsm_x4(sKa + (f >> 6) * ATD_HALF + key * 128 + ((((f & 63) >> 3) ^ (key & 7)) << 4), b00, b01, b10, b11);
+        }
+#pragma unroll
+        for (int qt = 0; qt < QT; ++qt) {
+          uint32_t a0, a1, a2, a3;
+          ldsm_x4(sQa + (qt * 16 + (mi & 1) * 8 + rr) * ATD_ROW + (ks * 16 + (mi >> 1) * 8) * 2, a0, a1, a2, a3);
+          mma_bf16_16816(sc[qt][0], a0, a1, a2, a3, b00, b01);
+          mma_bf16_16816(sc[qt][1], a0, a1, a2, a3, b10, b11);
+        }
       }
+      // online softmax (log2 units), weights packed as the A operand of P V
+      uint32_t pa[QT][4];
 #pragma unroll
-      for (int u = 0; u < ATT_CH_MAX / 32; ++u) {
-        const int t = lane + 32 * u;
-        if (t < nk) {
-          const uint4* kr = reinterpret_cast<const uint4*>(sK + t * ATT_KROW) + c4;
-          float acc = sc[u];
+      for (int qt = 0; qt < QT; ++qt) {
+        float t[2][4];
 #pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            const uint4 kv = kr[c];
-            acc = fmaf(bf16_lo(kv.x), qf[8 * c + 0], acc);
-            acc = fmaf(bf16_hi(kv.x), qf[8 * c + 1], acc);
-            acc = fmaf(bf16_lo(kv.y), qf[8 * c + 2], acc);
-            acc = fmaf(bf16_hi(kv.y), qf[8 * c + 3], acc);
-            acc = fmaf(bf16_lo(kv.z), qf[8 * c + 4], acc);
-            acc = fmaf(bf16_hi(kv.z), qf[8 * c + 5], acc);
-            acc = fmaf(bf16_lo(kv.w), qf[8 * c + 6], acc);
-            acc = fmaf(bf16_hi(kv.w), qf[8 * c + 7], acc);
+        for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int64_t kp = kw + nt * 8 + 2 * tig + (e & 1);
+            const bool vis = kp < k1 && kp <= lim[qt][e >> 1];
+            t[nt][e] = vis ? sc[qt][nt][e] * a.sl2 : -INFINITY;
           }
-          sc[u] = acc;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          float mx = fmaxf(fmaxf(t[0][2 * h], t[0][2 * h + 1]), fmaxf(t[1][2 * h], t[1][2 * h + 1]));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+          const float mn = fmaxf(m[qt][h], mx);
+          float alpha = 1.f;
+          if (mn == -INFINITY) {  // nothing visible yet in this row
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) t[nt][2 * h] = t[nt][2 * h + 1] = 0.f;
+          } else {
+            alpha = att_ex2(m[qt][h] - mn);
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) {
+              t[nt][2 * h] = att_ex2(t[nt][2 * h] - mn);
+              t[nt][2 * h + 1] = att_ex2(t[nt][2 * h + 1] - mn);
+            }
+            m[qt][h] = mn;
+          }
+          l[qt][h] = fmaf(l[qt][h], alpha, (t[0][2 * h] + t[0][2 * h + 1]) + (t[1][2 * h] + t[1][2 * h + 1]));
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            o[qt][j][2 * h] *= alpha;
+            o[qt][j][2 * h + 1] *= alpha;
+          }
+        }
+        pa[qt][0] = pack_bf16x2(t[0][0], t[0][1]);  // row grp,     keys 2 tig, +1
+        pa[qt][1] = pack_bf16x2(t[0][2], t[0][3]);  // row grp + 8
+        pa[qt][2] = pack_bf16x2(t[1][0], t[1][1]);  // row grp,     keys 8 + 2 tig, +1
+        pa[qt][3] = pack_bf16x2(t[1][2], t[1][3]);  // row grp + 8
+      }
+      // O += P V: V rows are keys, so the B operand comes through ldmatrix.trans
+#pragma unroll
+      for (int j = 0; j < ATT_D / 16; ++j) {
+        uint32_t v00, v01, v10, v11;  // features 16j + 0-7 (keys 0-7, 8-15), 16j + 8-15 (keys 0-7, 8-15)
+        {
+          const int key = 16 * warp + (mi & 1) * 8 + rr, f = 16 * j + (mi >> 1) * 8;
+          ldsm_x4_t(sVa + (f >> 6) * ATD_HALF + key * 128 + ((((f & 63) >> 3) ^ (key & 7)) << 4), v00, v01, v10,
+                    v11);
+        }
+#pragma unroll
+        for (int qt = 0; qt < QT; ++qt) {
+          mma_bf16_16816(o[qt][2 * j], pa[qt][0], pa[qt][1], pa[qt][2], pa[qt][3], v00, v01);
+          mma_bf16_16816(o[qt][2 * j + 1], pa[qt][0], pa[qt][1], pa[qt][2], pa[qt][3], v10, v11);
         }
       }
     }
-    // softmax partials over the chunk's visible keys
-    float mx = -FLT_MAX;
-#pragma unroll
-    for (int u = 0; u < ATT_CH_MAX / 32; ++u) {
-      const int t = lane + 32 * u;
-      const bool vis = t < nk && c0 + t <= last;
-      sc[u] = vis ? sc[u] * a.scale : -FLT_MAX;
-      mx = fmaxf(mx, sc[u]);
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-    float sum = 0.f;
-#pragma unroll
-    for (int u = 0; u < ATT_CH_MAX / 32; ++u) {
-      sc[u] = sc[u] == -FLT_MAX ? 0.f : __expf(sc[u] - mx);
-      sum += sc[u];
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-    // weighted value rows: lane l sums features 4l .. 4l + 3 over the keys
-    float o[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-    for (int u = 0; u < ATT_CH_MAX / 32; ++u) {
-      const int tb = 32 * u;
-      const int nt = nk - tb < 32 ? nk - tb : 32;
-      for (int j = 0; j < nt; ++j) {
-        const float p = __shfl_sync(0xffffffffu, sc[u], j);
-        const uint2 vv = *reinterpret_cast<const uint2*>(sV + (tb + j) * ATT_D + 4 * lane);
-        o[0] = fmaf(p, bf16_lo(vv.x), o[0]);
-        o[1] = fmaf(p, bf16_hi(vv.x), o[1]);
-        o[2] = fmaf(p, bf16_lo(vv.y), o[2]);
-        o[3] = fmaf(p, bf16_hi(vv.y), o[3]);
-      }
-    }
-    float* pr = part + qi * ATT_PROW;
-    *reinterpret_cast<float4*>(pr + 4 * lane) = make_float4(o[0], o[1], o[2], o[3]);
-    if (lane == 0) {
-      pr[ATT_D] = sum > 0.f ? mx : -FLT_MAX;
-      pr[ATT_D + 1] = sum;
+    __syncthreads();  // every warp is done with this stage
+    if (tid == 0 && ok && c + ATD_NST < nch) {
+      issue(c + ATD_NST, buf);
+      ++issued;
     }
   }
+  if (!ok) {
+    // a stage never arrived: record it, let the copies still in flight land
+    // (bounded), and finish without results; the cluster barriers below still
+    // meet
+    *s_abort = 1;
+    if (tid == 0) {
+      report_status(a.status, DECOMOE_ERR_TIMEOUT);
+      int no_abort = 0;
+      for (int c = c_fail; c < issued; ++c) mbar_wait(bar0 + 8u * (c % ATD_NST), (c / ATD_NST) & 1, a.limit_ns, &no_abort);
+    }
+  }
+  __syncthreads();
+
+  // merge the warps (warp order) through shared memory: per warp and row m, l
+  // and the 128 output columns
+  float* sm_o = reinterpret_cast<float*>(sKV);                   // [WARPS][QT*16][OROW]
+  float* sm_m = sm_o + ATD_WARPS * ATD_QT * 16 * ATD_OROW;        // [WARPS][QT*16]
+  float* sm_l = sm_m + ATD_WARPS * ATD_QT * 16;
+#pragma unroll
+  for (int qt = 0; qt < QT; ++qt)
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      float ls = l[qt][h];
+      ls += __shfl_xor_sync(0xffffffffu, ls, 1);
+      ls += __shfl_xor_sync(0xffffffffu, ls, 2);
+      const int r = qt * 16 + grp + 8 * h;
+      if (tig == 0) {
+        sm_m[warp * ATD_QT * 16 + r] = m[qt][h];
+        sm_l[warp * ATD_QT * 16 + r] = ls;
+      }
+      float* orow = sm_o + (warp * ATD_QT * 16 + r) * ATD_OROW;
+#pragma unroll
+      for (int j = 0; j < 16; ++j)
+        *reinterpret_cast<float2*>(orow + 8 * j + 2 * tig) = make_float2(o[qt][j][2 * h], o[qt][j][2 * h + 1]);
+    }
+  __syncthreads();
+  // this block's partial rows: m (log2 units), l and the unnormalised output
+  for (int r = 0; r < QT * 16; r += 2) {
+    // two rows at a time: threads 0-127 and 128-255 take one output column each
+    const int rh = r + (tid >> 7);
+    const int col = tid & (ATT_D - 1);
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < ATD_WARPS; ++w) M = fmaxf(M, sm_m[w * ATD_QT * 16 + rh]);
+    float acc = 0.f, L = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int w = 0; w < ATD_WARPS; ++w) {
+        const float mw = sm_m[w * ATD_QT * 16 + rh];
+        const float ww = mw == -INFINITY ? 0.f : att_ex2(mw - M);
+        acc = fmaf(ww, sm_o[(w * ATD_QT * 16 + rh) * ATD_OROW + col], acc);
+        L = fmaf(ww, sm_l[w * ATD_QT * 16 + rh], L);
+      }
+    }
+    float* pr = s_part + rh * ATT_PROW;
+    pr[col] = acc;
+    if (col == 0) {
+      pr[ATT_D] = M;
+      pr[ATT_D + 1] = L;
+    }
+  }
+  cluster_sync_all();  // every block's partial rows are in place
+  // block `rank` merges rows rank, rank + nsplit, ... over the blocks in rank
+  // order (threads 0-127 and 128-255: two rows per pass, one column each)
+  const uint32_t nsplit = gridDim.x;
+  const uint32_t rank = cluster_ctarank();
+  const uint32_t part_a = smem_u32(s_part);
+  for (int r0 = static_cast<int>(rank); r0 < QT * 16; r0 += 2 * static_cast<int>(nsplit)) {
+    const int r = r0 + (tid >> 7) * static_cast<int>(nsplit);
+    const int col = tid & (ATT_D - 1);
+    const int qi = qbase + r;
+    if (r < QT * 16 && qi < nq) {
+      float M = -INFINITY;
+      for (uint32_t t = 0; t < nsplit; ++t)
+        M = fmaxf(M, ld_dsmem_f32(mapa_shared(part_a + (r * ATT_PROW + ATT_D) * 4, t)));
+      float acc = 0.f, L = 0.f;
+      for (uint32_t t = 0; t < nsplit; ++t) {
+        const uint32_t row = mapa_shared(part_a + r * ATT_PROW * 4, t);
+        const float mt = ld_dsmem_f32(row + ATT_D * 4);
+        const float w = mt == -INFINITY ? 0.f : att_ex2(mt - M);  // a split with no visible key weighs 0
+        acc = fmaf(w, ld_dsmem_f32(row + col * 4), acc);
+        L = fmaf(w, ld_dsmem_f32(row + (ATT_D + 1) * 4), L);
+      }
+      const int ti = qi / G, hj = qi - ti * G;
+      a.out[(static_cast<int64_t>(ti) * a.Hq + g * G + hj) * ATT_D + col] = __float2bfloat16_rn(acc / L);
+    }
+  }
+  cluster_sync_all();  // no block leaves while its partial rows may still be read
   pdl_trigger();
 }
 
-// out[i, h, :] = sum_s e^(m_s - M) acc_s / sum_s e^(m_s - M) l_s over the
-// splits s (M = max m_s). Block (token i x head h, 32-feature slice), 32
-// warps: warp w sums the splits s = w, w + 32, ... in order (lane = feature),
-// then the warp sums are added in warp order: a fixed order, so the result
-// does not depend on timing, and each pass is about one round of loads.
-constexpr int ATT_MAX_SPLITS = 1024;
-constexpr int ATT_CWARPS = 32;
-__global__ void __launch_bounds__(32 * ATT_CWARPS)
-    k_attn_combine(const float* __restrict__ part, int64_t n, int Hq, int Hkv, int nsplit,
-                   __nv_bfloat16* __restrict__ out) {
-  pdl_enter();
-  __shared__ float s_m[ATT_CWARPS], s_num[ATT_CWARPS][32], s_den[ATT_CWARPS];
-  const int64_t ih = blockIdx.x;  // token i * Hq + head h
-  const int64_t i = ih / Hq;
-  const int h = static_cast<int>(ih - i * Hq);
-  const int G = Hq / Hkv;
-  const int g = h / G;
-  const int nq = static_cast<int>(n) * G;
-  const int qi = static_cast<int>(i) * G + (h - g * G);
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int d = blockIdx.y * 32 + lane;
-  auto prow = [&](int s) { return part + ((static_cast<int64_t>(s) * Hkv + g) * nq + qi) * ATT_PROW; };
-  float mx = -FLT_MAX;
-  for (int s = warp; s < nsplit; s += ATT_CWARPS) mx = fmaxf(mx, __ldg(prow(s) + ATT_D));
-  if (lane == 0) s_m[warp] = mx;
-  __syncthreads();
-  float M = s_m[0];
-#pragma unroll
-  for (int w = 1; w < ATT_CWARPS; ++w) M = fmaxf(M, s_m[w]);
-  float num = 0.f, den = 0.f;
-  for (int s = warp; s < nsplit; s += ATT_CWARPS) {
-    const float* p = prow(s);
-    const float ms = __ldg(p + ATT_D);
-    const float ls = __ldg(p + ATT_D + 1);
-    const float as = __ldg(p + d);
-    const float w = ms == -FLT_MAX ? 0.f : __expf(ms - M);  // no visible key in this split: weight 0
-    num = fmaf(w, as, num);
-    den = fmaf(w, ls, den);
+// Keys per block, in whole chunks: the splits of a head form one cluster of
+// at most att_max_cluster() blocks, one chunk each where C allows.
+static int att_max_cluster();
+static int64_t att_kps(int64_t C) {
+  const int64_t maxc = att_max_cluster();
+  const int64_t nsplit = std::max<int64_t>(1, std::min<int64_t>((C + ATD_CH - 1) / ATD_CH, maxc));
+  int64_t kps = (C + nsplit - 1) / nsplit;
+  return (kps + ATD_CH - 1) / ATD_CH * ATD_CH;
+}
+static int att_nz(int64_t nq) { return static_cast<int>((nq + ATD_QT * 16 - 1) / (ATD_QT * 16)); }
+
+// Largest cluster of decode blocks this device schedules (16 where the
+// non-portable size fits, else the portable 8), per device ordinal.
+static std::atomic<int> g_att_cluster[64];
+static int att_max_cluster() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 8;
+  int v = g_att_cluster[dev].load();
+  if (v != 0) return v;
+  v = 8;
+  bool ok = true;
+  for (auto kern : {k_attn_dec<1>, k_attn_dec<2>}) {
+    ok = ok && cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(ATD_SMEM)) ==
+                   cudaSuccess;
+    ok = ok && cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess;
   }
-  s_num[warp][lane] = num;
-  if (lane == 0) s_den[warp] = den;
-  __syncthreads();
-  if (warp == 0) {
-    float a = s_num[0][lane], b = s_den[0];
-#pragma unroll
-    for (int w = 1; w < ATT_CWARPS; ++w) {
-      a += s_num[w][lane];
-      b += s_den[w];
-    }
-    out[ih * ATT_D + d] = __float2bfloat16_rn(a / b);
+  if (ok) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(16, 1, 1);
+    cfg.blockDim = dim3(ATD_THREADS);
+    cfg.dynamicSmemBytes = ATD_SMEM;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 16;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n1 = 0, n2 = 0;
+    if (cudaOccupancyMaxActiveClusters(&n1, k_attn_dec<1>, &cfg) == cudaSuccess &&
+        cudaOccupancyMaxActiveClusters(&n2, k_attn_dec<2>, &cfg) == cudaSuccess && n1 >= 1 && n2 >= 1)
+      v = 16;
   }
+  cudaGetLastError();  // a refused query leaves no error behind
+  g_att_cluster[dev].store(v);
+  return v;
 }
 
 // ------------------------------------------------------------------ prefill (tensor cores)
@@ -611,9 +824,7 @@ size_t decomoe_attention_workspace_bytes(int64_t n, int64_t C, int Hq, int Hkv, 
   if (n <= 0 || C <= 0 || Hq <= 0 || Hkv <= 0 || D != ATT_D || Hq % Hkv != 0) return 0;
   if (att_use_prefill(n, Hq, Hkv))  // the transposed values [Hkv][D][C padded to 64]
     return align_up(static_cast<size_t>(Hkv) * ATT_D * att_c_pad(C) * 2, 256);
-  const int64_t nsplit = (C + att_chunk(C, Hkv) - 1) / att_chunk(C, Hkv);
-  const int64_t nq = n * (Hq / Hkv);
-  return align_up(static_cast<size_t>(nsplit) * Hkv * nq * ATT_PROW * sizeof(float), 256);
+  return 0;  // decode sizes: the splits merge through the cluster's shared memory
 }
 
 int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void* v_cache, int64_t C, int Hq,
@@ -629,11 +840,11 @@ int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void*
                "attention: pointers must be 16-byte aligned");
   const int G = Hq / Hkv;
   const size_t need = decomoe_attention_workspace_bytes(n, C, Hq, Hkv, D);
-  if (ws == nullptr || ws_bytes < need) {
+  if (need > 0 && (ws == nullptr || ws_bytes < need)) {
     set_error("attention: workspace needs %zu bytes", need);
     return DECOMOE_ERR_WORKSPACE;
   }
-  DM_ARG_CHECK(aligned16(ws), "attention: workspace must be 16-byte aligned");
+  DM_ARG_CHECK(need == 0 || aligned16(ws), "attention: workspace must be 16-byte aligned");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const float sc = scale > 0.f ? scale : 1.0f / sqrtf(static_cast<float>(D));
   if (att_use_prefill(n, Hq, Hkv)) {
@@ -673,7 +884,7 @@ int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void*
                              tq, tk, tv, pa));
     return DECOMOE_OK;
   }
-  AttArgs a;
+  AttDecArgs a;
   a.q = static_cast<const uint4*>(q);
   a.k = static_cast<const uint4*>(k_cache);
   a.v = static_cast<const uint4*>(v_cache);
@@ -681,20 +892,42 @@ int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void*
   a.C = C;
   a.Hq = Hq;
   a.Hkv = Hkv;
-  a.chunk = att_chunk(C, Hkv);
-  a.nsplit = static_cast<int>((C + a.chunk - 1) / a.chunk);
-  DM_ARG_CHECK(a.nsplit <= ATT_MAX_SPLITS, "attention: C=%lld is more than %d keys", (long long)C,
-               ATT_MAX_SPLITS * ATT_CH_MAX);
-  a.scale = sc;
-  a.part = static_cast<float*>(ws);
-  const size_t smem = att_split_smem();
-  DM_CUDA_CHECK(cudaFuncSetAttribute(k_attn_split, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     static_cast<int>(smem)));
-  DM_CUDA_CHECK(launch_pdl(k_attn_split, dim3(a.nsplit, Hkv), dim3(ATT_THREADS), smem, s, a));
-  DM_CUDA_CHECK(launch_pdl(k_attn_combine, dim3(static_cast<unsigned>(n * Hq), ATT_D / 32), dim3(32 * ATT_CWARPS), 0, s,
-                           static_cast<const float*>(a.part), n, Hq, Hkv, a.nsplit,
-                           static_cast<__nv_bfloat16*>(out)));
-  return DECOMOE_OK;
+  const int nq = static_cast<int>(n) * G;
+  const int nz = att_nz(nq);
+  const int64_t kps = att_kps(C);
+  DM_ARG_CHECK(kps <= 0x7fffffffLL, "attention: C=%lld keys is too long", (long long)C);
+  a.kps = static_cast<int>(kps);
+  const int nsplit = static_cast<int>((C + kps - 1) / kps);  // <= att_max_cluster()
+  a.sl2 = sc * 1.4426950408889634f;
+  a.out = static_cast<__nv_bfloat16*>(out);
+  a.status = status_dev;
+  a.limit_ns = static_cast<uint64_t>(wait_limit_ns());
+  CUtensorMap tk, tv;  // [C][Hkv][D]: boxes of 128 keys x 64 features of one head
+  const uint64_t dkv[3] = {static_cast<uint64_t>(D), static_cast<uint64_t>(Hkv), static_cast<uint64_t>(C)};
+  const uint64_t skv[2] = {static_cast<uint64_t>(D) * 2, static_cast<uint64_t>(Hkv) * D * 2};
+  const uint32_t bkv[3] = {64, 1, ATD_CH};
+  DM_RET(make_tmap_bf16_3d(&tk, k_cache, dkv, skv, bkv));
+  DM_RET(make_tmap_bf16_3d(&tv, v_cache, dkv, skv, bkv));
+  const dim3 grid(static_cast<unsigned>(nsplit), static_cast<unsigned>(Hkv), static_cast<unsigned>(nz));
+  auto go = [&](auto kern) -> int {
+    DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(ATD_SMEM)));
+    if (nsplit > 8) DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1));
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(ATD_THREADS);
+    cfg.dynamicSmemBytes = ATD_SMEM;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;  // one cluster per (KV head, query tile group)
+    attr[0].val.clusterDim.x = static_cast<unsigned>(nsplit);
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    DM_CUDA_CHECK(cudaLaunchKernelEx(&cfg, kern, tk, tv, a));
+    return DECOMOE_OK;
+  };
+  return nq <= 16 ? go(k_attn_dec<1>) : go(k_attn_dec<2>);
 }
 
 }  // extern "C"

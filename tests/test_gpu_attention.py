@@ -1,8 +1,9 @@
 """Attention on the compacted sequence and over the text-only KV cache
 (decomoe_attention) against the oracle's causal grouped-head attention:
-decode steps (up to 64 queries per KV head, split-key CUDA-core kernel) and
-prefill (more, the tensor-core kernel), with ragged tiles, chunked prefill
-(n < C), sampled rows at the full 16384-token sequence.
+decode steps (up to 64 queries per KV head: split keys in one thread-block
+cluster per KV head, warp-level tensor-core products) and prefill (more: the
+tcgen05 kernel), with ragged tiles, chunked prefill (n < C), sampled rows at
+the full 16384-token sequence.
 
 The layer shape is the 30B-A3B decoder's: 32 query heads and 4 KV heads of
 128 (q = 4096, k_v = 512); the caches are one layer slice of the KV buffers
@@ -49,8 +50,8 @@ def _run(q, k, v, scale=0.0):
     return out
 
 
-@pytest.mark.parametrize("n,C", [(1, 1), (1, 127), (1, 128), (1, 272), (1, 2049), (2, 300), (8, 1552),
-                                 (1, 16384), (3, 129)])
+@pytest.mark.parametrize("n,C", [(1, 1), (1, 63), (1, 64), (1, 65), (1, 127), (1, 128), (1, 272), (1, 2049),
+                                 (2, 300), (8, 1552), (1, 16384), (3, 129), (5, 40000)])
 def test_attention_decode_parity(n, C):
     q, k, v = _qkv(n, C, seed=C + n)
     out = _run(q, k, v)
@@ -101,6 +102,29 @@ def test_attention_prefill_is_deterministic():
     a = _run(q, k, v)
     b = _run(q, k, v)
     assert torch.equal(a, b)
+
+
+def test_attention_decode_needs_no_workspace_and_repeats_bitwise():
+    """Decode sizes take no workspace (a null pointer is accepted) and give the
+    same bits on every call, in any order of sizes."""
+    sizes = [(1, 16384), (1, 300), (8, 2049), (2, 64), (1, 1), (4, 5000)]
+    for n, C in sizes:
+        assert dm.decomoe_attention_workspace_bytes(n, C, HQ, HKV, D) == 0
+    first = {}
+    for rep in range(2):
+        for n, C in sizes:
+            q, k, v = _qkv(n, C, seed=31 * C + n)
+            out = torch.empty(n, HQ, D, dtype=torch.bfloat16, device=DEV)
+            lib = dm.lib()
+            rc = lib.decomoe_attention(q.to(DEV).data_ptr(), n, k.to(DEV).data_ptr(), v.to(DEV).data_ptr(), C, HQ,
+                                       HKV, D, 0.0, out.data_ptr(), None, 0, None,
+                                       torch.cuda.current_stream().cuda_stream)
+            torch.cuda.synchronize()
+            assert rc == 0
+            if rep == 0:
+                first[(n, C)] = out.cpu()
+            else:
+                assert torch.equal(out.cpu(), first[(n, C)]), (n, C)
 
 
 def test_attention_grouping_and_scale():
@@ -157,4 +181,9 @@ def test_attention_rejects_unsupported_shapes():
     assert e.value.code == dm.DECOMOE_ERR_INVALID_ARG
     with pytest.raises(dm.DecomoeError) as e:  # 31 query heads on 4 KV heads
         dm.decomoe_attention(q.to(DEV)[:, :31].contiguous(), k.to(DEV), v.to(DEV), out[:, :31].contiguous(), ws)
+    assert e.value.code == dm.DECOMOE_ERR_INVALID_ARG
+    q3, k3, v3 = _qkv(40, 100, seed=2, Hq=12, Hkv=4)  # prefill sizes with an odd group (3 heads per KV head)
+    with pytest.raises(dm.DecomoeError) as e:
+        dm.decomoe_attention(q3.to(DEV), k3.to(DEV), v3.to(DEV), torch.empty(40, 12, D, dtype=torch.bfloat16,
+                                                                               device=DEV), ws)
     assert e.value.code == dm.DECOMOE_ERR_INVALID_ARG
