@@ -54,7 +54,11 @@ def parse():
                     help="run only the decode layer at T tokens (K=64) for --steps graph replays (profiling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--only-isolated", default="", metavar="NAME",
-                    help="time one isolated memory-bound kernel (compaction, gather, combine, permute) and exit")
+                    help="time one isolated step (compaction, gather, combine, permute, attention, "
+                         "attention_prefill) and exit")
+    ap.add_argument("--att-len", type=int, default=0, metavar="C",
+                    help="with --only-isolated attention / attention_prefill: only the cache or sequence of this "
+                         "length (profiling)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     return ap.parse_args()
 
@@ -698,7 +702,7 @@ def run_large(dm, ws, pk, n):
 ISOLATED = ("compaction", "gather", "combine", "permute", "attention", "attention_prefill")
 
 
-def run_isolated(dm, ws, pk, only=None, steps=10, warmup=3):
+def run_isolated(dm, ws, pk, only=None, steps=10, warmup=3, att_len=0):
     """The memory-bound steps alone, each timed with CUDA events (L2 flushed
     before every repetition, median reported) and reported as GB/s of
     algorithmic bytes against the measured HBM copy peak:
@@ -802,6 +806,8 @@ def run_isolated(dm, ws, pk, only=None, steps=10, warmup=3):
         Hq, Hkv, Dh = 32, 4, 128
         for name, C_text, C_full in (("stack", 16 + 256 + 1, 1552 + 1), ("large", 2048 + 1, 16384 + 1)):
             for kind, C in (("text-only cache", C_text), ("full cache", C_full)):
+                if att_len and C != att_len:
+                    continue
                 gq = torch.Generator(device=dev).manual_seed(C)
                 nb = 2 * C * Hkv * Dh * 2 + 2 * Hq * Dh * 2
                 # R distinct caches, together at least twice the L2, replayed as
@@ -838,6 +844,8 @@ def run_isolated(dm, ws, pk, only=None, steps=10, warmup=3):
         Hq, Hkv, Dh = 32, 4, 128
         for name, S_text, S_full in (("stack", 272, 1552), ("large", 2048, 16384)):
             for kind, S in (("compacted sequence", S_text), ("full sequence", S_full)):
+                if att_len and S != att_len:
+                    continue
                 gq = torch.Generator(device=dev).manual_seed(S)
                 q = torch.randn(S, Hq, Dh, device=dev, generator=gq).to(torch.bfloat16)
                 kc = torch.randn(S, Hkv, Dh, device=dev, generator=gq).to(torch.bfloat16)
@@ -1160,7 +1168,7 @@ def main():
 
         dm.lib()
         rows = run_isolated(dm, ws, peaks(), only=args.only_isolated, steps=max(1, args.steps),
-                            warmup=max(1, args.warmup))
+                            warmup=max(1, args.warmup), att_len=args.att_len)
         if rank == 0:
             print(json.dumps(rows), flush=True)
         return
