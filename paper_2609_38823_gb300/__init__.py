@@ -435,7 +435,8 @@ def decomoe_attention(q, k_cache, v_cache, out, ws, scale=0.0, status=None, stre
     C, Hkv, _ = k_cache.shape
     _check("decomoe_attention",
            lib().decomoe_attention(_ptr(q), n, _ptr(k_cache), _ptr(v_cache), C, Hq, Hkv, D, float(scale), _ptr(out),
-                                   _ptr(ws), ws.numel() * ws.element_size(), _ptr(status), _stream(stream)))
+                                   _ptr(ws), 0 if ws is None else ws.numel() * ws.element_size(), _ptr(status),
+                                   _stream(stream)))
 
 
 def decomoe_gather_rows(x, perm_token, offsets, K, x_perm, stream=None):
