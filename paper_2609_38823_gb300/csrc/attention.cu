@@ -58,9 +58,7 @@ constexpr int ATD_OROW = ATT_D + 4;             // floats per row of the warp me
 static_assert(ATD_WARPS * ATD_QT * 16 * (ATD_OROW + 2) * 4 <= ATD_NST * ATD_STAGE, "warp merge fits in the ring");
 
 struct AttDecArgs {
-  const uint4* q;   // [n, Hq, D]
-  const uint4* k;   // [C, Hkv, D]
-  const uint4* v;
+  const uint4* q;   // [n, Hq, D] (K and V [C, Hkv, D] come through the tensor maps)
   int64_t n, C;
   int Hq, Hkv, kps; // keys per block; the cluster (grid.x) is the head's splits
   float sl2;        // scale * log2(e)
@@ -69,11 +67,6 @@ struct AttDecArgs {
   uint64_t limit_ns;
 };
 
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait_group() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
 __device__ __forceinline__ float att_ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -886,8 +879,6 @@ int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void*
   }
   AttDecArgs a;
   a.q = static_cast<const uint4*>(q);
-  a.k = static_cast<const uint4*>(k_cache);
-  a.v = static_cast<const uint4*>(v_cache);
   a.n = n;
   a.C = C;
   a.Hq = Hq;
