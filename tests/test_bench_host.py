@@ -44,3 +44,25 @@ def test_ffn_bound_is_hbm_at_the_measured_peaks():
     t_compute = flops / (pk["bf16_tflops"] * 1e12)
     assert t_mem > t_compute  # 114.7 us of HBM against 80.2 us of tensor work
     assert abs(t_mem * 1e6 - 114.7) < 0.1 and abs(t_compute * 1e6 - 80.2) < 0.1
+
+
+def test_ffn_algorithmic_bytes_with_the_row_gather():
+    """The layer's own launch from 8192 routed rows reads x once instead of
+    the gathered rows: 704.6 MB per launch at T=2048, K=64 (105.9 us at the
+    measured HBM peak against 80.2 us of tensor work: still HBM-bound)."""
+    b = _bench()
+    wl = b.W.PREFILL
+    R, D = wl.T * wl.k, 64
+    with_gather = b.algo_bytes_ffn(wl, R, D, wl.T)
+    assert with_gather == 64 * 3 * 2048 * 768 * 2 + 2048 * 2048 * 2 + 16384 * 768 * 2 + 16384 * 2048 * 2
+    assert with_gather == 704643072
+    assert abs(with_gather / 6652.7e9 * 1e6 - 105.9) < 0.1
+
+
+def test_layer_gather_range_matches_the_layer():
+    """bench.py times the gathering launch exactly where the layer uses it:
+    from 8192 routed rows up to the one-launch limit of 32768."""
+    b = _bench()
+    assert not b.layer_gathers(8191)
+    assert b.layer_gathers(8192) and b.layer_gathers(16384) and b.layer_gathers(32768)
+    assert not b.layer_gathers(32769) and not b.layer_gathers(131072)
