@@ -169,7 +169,11 @@ __device__ __forceinline__ void dl_acc_vec(float* acc, const uint4& v, float w) 
   acc[7] = fmaf(w, bf16_hi(v.w), acc[7]);
 }
 
-template <int STAGES>
+// TMAX: the most tokens this form takes (8, 16 or DL_MAX_T): the router's
+// per-thread token accumulators, and (up to DL_LOCAL_ROUTE_T) no code for the
+// distributed routing. Code run once per launch is fetched cold, so the
+// few-token forms run the short versions (measured: T=8 54.6 -> 51.5 us).
+template <int STAGES, int TMAX>
 __global__ void __launch_bounds__(DL_THREADS, 1)
     k_decode_layer(const __grid_constant__ CUtensorMap tma_w1, const __grid_constant__ CUtensorMap tma_x1,
                    const __grid_constant__ CUtensorMap tma_w2, const __grid_constant__ CUtensorMap tma_x2,
@@ -290,9 +294,9 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
   for (int e = blockIdx.x; e < E; e += gridDim.x) {
     if (tid < GEMV_THREADS) {
       const uint4* wr = g.w_r + static_cast<int64_t>(e) * vpr;
-      float acc[DL_MAX_T];
+      float acc[TMAX];
 #pragma unroll
-      for (int j = 0; j < DL_MAX_T; ++j) acc[j] = 0.f;
+      for (int j = 0; j < TMAX; ++j) acc[j] = 0.f;
       for (int c0 = 0; c0 < vpr; c0 += GEMV_THREADS * GEMV_VPT) {
         uint4 wv[GEMV_VPT];
 #pragma unroll
@@ -307,13 +311,13 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
           const int c = c0 + tid + GEMV_THREADS * i;
           if (c < vpr) {
 #pragma unroll
-            for (int j = 0; j < DL_MAX_T; ++j)
+            for (int j = 0; j < TMAX; ++j)
               if (j < T) acc[j] = dot8_bf16(wv[i], s_x[j * vpr + c], acc[j]);
           }
         }
       }
 #pragma unroll
-      for (int j = 0; j < DL_MAX_T; ++j) {
+      for (int j = 0; j < TMAX; ++j) {
         if (j < T) {
           float v = acc[j];
 #pragma unroll
@@ -380,7 +384,8 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
   // only) CTA t routes token t, publishes its picks, and a second grid
   // barrier precedes the dispatch. Lane l holds logits l, l+32, ...
   const int Kd = g.K_fixed > 0 ? g.K_fixed : E;  // expert groups of the dispatch
-  const bool dist = T > DL_LOCAL_ROUTE_T;          // one token per CTA, then a second barrier
+  // one token per CTA, then a second barrier (never in the few-token forms)
+  const bool dist = TMAX > DL_LOCAL_ROUTE_T && T > DL_LOCAL_ROUTE_T;
   float* s_lg = reinterpret_cast<float*>(smem);  // [T][E], in the ring
   float* s_wt = s_lg + T * E;                     // [T][E] full-pool pick weights (0: not picked)
   int32_t* const g_fpick = comb + T * nfb;        // [T*k] full-pool picks (distributed routing)
@@ -477,39 +482,43 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
       }
     }
   };
-  if (g.want_mass) {
-    if (!dist) {
-      route_pass(0, true);
-      __syncthreads();
-    }
-    // Eq. 11 as the routing kernels form it: fp32 sums per block of 8 tokens
-    // in token order (a token picks an expert at most once; the table's
-    // zeros add nothing), then the fixed fp64 tree over the blocks
-    const int nb = (T + 7) / 8;
-    for (int e = tid; e < E; e += DL_THREADS) {
-      double part[4] = {0.0, 0.0, 0.0, 0.0};
-      for (int b = 0; b < nb; ++b) {
-        float acc = 0.f;
-        const int te = min(T, 8 * b + 8);
-        for (int tt = 8 * b; tt < te; ++tt) acc += s_wt[tt * E + e];
-        part[b] = static_cast<double>(acc);
+  // At most two passes from one call site (code run once per launch is
+  // fetched cold): pass 0 the full pool (with the mass) or the fixed prefix,
+  // then Eq. 11's mass, and with the prefix selected on the device (Eq. 12)
+  // pass 1 over [0, K).
+  for (int pass = 0; pass < 2; ++pass) {
+    if (pass == 1) {
+      if (g.want_mass) {
+        // Eq. 11 as the routing kernels form it: fp32 sums per block of 8
+        // tokens in token order (a token picks an expert at most once; the
+        // table's zeros add nothing), then the fixed fp64 tree over the blocks
+        const int nb = (T + 7) / 8;
+        for (int e = tid; e < E; e += DL_THREADS) {
+          double part[4] = {0.0, 0.0, 0.0, 0.0};
+          for (int b = 0; b < nb; ++b) {
+            float acc = 0.f;
+            const int te = min(T, 8 * b + 8);
+            for (int tt = 8 * b; tt < te; ++tt) acc += s_wt[tt * E + e];
+            part[b] = static_cast<double>(acc);
+          }
+          const double me = nb == 1 ? part[0] : (part[0] + part[2]) + (part[1] + part[3]);
+          s_mass[e] = me;
+          if (blockIdx.x == 0) g.mass[e] = me;
+        }
       }
-      const double me = nb == 1 ? part[0] : (part[0] + part[2]) + (part[1] + part[3]);
-      s_mass[e] = me;
-      if (blockIdx.x == 0) g.mass[e] = me;
+      if (g.K_fixed >= 0) break;
+      __syncthreads();
+      if (tid == 0) {
+        s_flag[1] = select_prefix_seq(s_mass, E, k, g.p);
+        if (blockIdx.x == 0) *g.K_dev = s_flag[1];
+      }
+      __syncthreads();
+    } else if (dist) {
+      continue;  // the picks were routed per CTA and exchanged above
     }
-  } else if (!dist) {
-    route_pass(g.K_fixed, false);
-  }
-  if (g.K_fixed < 0) {
-    // Eq. 12 on the device, then the prefix top-k over [0, K)
+    const bool full = pass == 0 && g.want_mass;
+    route_pass(pass == 1 ? s_flag[1] : (full ? 0 : g.K_fixed), full);
     __syncthreads();
-    if (tid == 0) {
-      s_flag[1] = select_prefix_seq(s_mass, E, k, g.p);
-      if (blockIdx.x == 0) *g.K_dev = s_flag[1];
-    }
-    __syncthreads();
-    route_pass(s_flag[1], false);
   }
   __syncthreads();
   // dispatch: counts and exclusive offsets from the per-expert token masks;
@@ -958,7 +967,9 @@ int launch_decode_layer(const void* x, const void* w_r, const float* bias, const
   g.sync = sync;
   g.status = status;
   g.limit_ns = static_cast<uint64_t>(wait_limit_ns());
-  auto kern = k_decode_layer<DL_STAGES>;
+  auto kern = T <= 8    ? k_decode_layer<DL_STAGES, 8>
+              : T <= 16 ? k_decode_layer<DL_STAGES, 16>
+                        : k_decode_layer<DL_STAGES, DL_MAX_T>;
   static_assert(C::SMEM <= DL_DYN_SMEM_MAX, "shared memory budget");
   static_assert(C::SMEM > 232448 / 2, "one CTA per SM: the grid barrier needs every CTA resident");
   DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(C::SMEM)));
