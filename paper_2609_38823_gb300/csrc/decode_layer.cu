@@ -46,7 +46,7 @@ constexpr int DL_MAX_T = 32;
 constexpr int DL_MAX_ROWS = 256;           // routed rows T * k
 constexpr int DL_BN = 32;                  // token columns of a tile (MMA N, TMA box rows)
 constexpr int DL_BM = 128, DL_BK = 64;     // weight rows per tile, k-block
-constexpr int DL_THREADS = 192;            // TMA warp, MMA warp, four epilogue warps
+constexpr int DL_THREADS = 256;            // TMA warp, MMA warp, four epilogue warps, two more for routing
 constexpr int DL_FB = 128;                 // features per combine block (= down tile rows)
 constexpr int DL_LOCAL_ROUTE_T = 12;       // up to this many tokens every CTA routes them all itself
 constexpr uint32_t DL_BULK_CHUNK = 32768;  // bytes per bulk copy of the token rows
@@ -767,7 +767,7 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
         mbar_wait(DRAIN_BAR, 0, g.limit_ns, &no_abort);
       }
     }
-  } else if (warp >= 2) {
+  } else if (warp >= 2 && warp < 6) {
     // ------------------------------------------------ epilogue (4 warps)
     const int q = warp & 3;  // TMEM lanes [32q, 32q + 32)
     const int et = tid - 64;  // 0..127
