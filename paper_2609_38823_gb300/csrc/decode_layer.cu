@@ -12,8 +12,11 @@
 //
 // Phases (one CTA per SM, every CTA resident):
 //  A  router: CTA c computes logits[:, e] for e = c, c + grid, ... on CUDA
-//     cores (the arithmetic of the router's decode-size kernel), then all
-//     CTAs meet at a grid barrier (bounded wait).
+//     cores (the arithmetic of the router's decode-size kernel) and stores
+//     each logit together with the launch's tag in one 64-bit word; every
+//     CTA then reads all T x E words, polling (bounded) until each carries
+//     the tag. No grid barrier: the tag is the launch number, which each CTA
+//     learns from its arrival on a launch counter at its start.
 //  B  routing: full-pool top-k and mass when wanted, Eq. 12 on the device,
 //     prefix top-k and renormalised weights. For a few tokens every CTA
 //     routes all of them itself (no second exchange); for more, each token is
@@ -30,18 +33,24 @@
 //     that completes a (token, block) pair sums that pair's k slot rows in
 //     slot order (+ residual) into out, with the combine kernel's arithmetic.
 // Counters live in the caller's workspace and every launch leaves them at
-// zero: the grid barrier reverses a sense word, an expert's readiness count
+// zero: the grid barrier (distributed routing only) bumps a generation, the
+// launch counter's arrivals return to zero when the last CTA arrives (its
+// launch number goes up by one), an expert's readiness count
 // is reset by the last of its down tiles, and a (token, block) count by the
 // tile that completes it. The first launch on a workspace may find anything
-// there: CTA 0 clears the counters unless the word it publishes (the launch's
-// grid id, which a graph's kernel node keeps from one replay to the next)
-// shows that this launch node has run on the workspace before, and the other
-// CTAs wait for that word before their first counter use.
+// there: the launch counter carries a 24-bit signature, and an arrival that
+// finds it missing (a fresh workspace, or one a timed-out launch marked as
+// such) makes CTA 0 clear every counter and the tagged logits and write the
+// signature back (release); the other CTAs wait for it (acquire) and arrive
+// again. Tags are launch number + 1, never 0, so cleared words never pass
+// for logits; the launch number is 24 bits wide, and its wrap carries into
+// the signature, which re-initialises the block, so no tag recurs while
+// older words can still be read.
 #include "route_common.cuh"
 
 namespace decomoe {
 
-constexpr int DL_MIN_T = 2;                // tokens per launch
+constexpr int DL_MIN_T = 1;                // tokens per launch
 constexpr int DL_MAX_T = 32;
 constexpr int DL_MAX_ROWS = 256;           // routed rows T * k
 constexpr int DL_BN = 32;                  // token columns of a tile (MMA N, TMA box rows)
@@ -50,11 +59,20 @@ constexpr int DL_THREADS = 256;            // TMA warp, MMA warp, four epilogue 
 constexpr int DL_FB = 128;                 // features per combine block (= down tile rows)
 constexpr int DL_LOCAL_ROUTE_T = 12;       // up to this many tokens every CTA routes them all itself
 constexpr uint32_t DL_BULK_CHUNK = 32768;  // bytes per bulk copy of the token rows
+constexpr int DL_QN = 4;                   // work items the TMA warp may publish ahead of the MMA and epilogue
 
-// int32 slots of the counter block: [0, 2) grid id of the launch that last
-// cleared it, [2] grid barrier word, [3] spare, then ready[E], done[E] (down
-// tiles finished per expert), comb[T * d / 128].
-constexpr int DL_SYNC_HEAD = 4;
+// int32 slots of the counter block (the same for every T of a layer shape):
+// [0, 2) spare, [2] grid barrier word, [3] work-item counter, [4, 6) launch counter
+// (u64: signature in bits 40-63, launch number in bits 16-39, arrivals in
+// bits 0-15), [6, 8) spare, then ready[E], done[E] (down tiles finished per
+// expert), comb[DL_MAX_T * d / 128], the full-pool picks and weights of the
+// distributed routing [2][DL_MAX_ROWS], and the tagged logits
+// [DL_MAX_T][E] (u64: logit bits low, tag high).
+constexpr int DL_SYNC_HEAD = 8;
+constexpr uint64_t DL_SIGNATURE = 0xD3C0AEull;  // 24 bits
+__host__ __device__ constexpr int dl_sync_tagged_offset(int E, int d) {
+  return DL_SYNC_HEAD + 2 * E + DL_MAX_T * (d / DL_FB) + 2 * DL_MAX_ROWS;
+}
 
 struct DlArgs {
   const uint4* x;  // [T, d] bf16
@@ -91,7 +109,7 @@ struct DlCfg {
   static constexpr int B_BYTES = DL_BN * DL_BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int TMEM_COLS = 2 * DL_BN;
-  static constexpr int NBARS = 2 * STAGES + 6;
+  static constexpr int NBARS = 2 * STAGES + 6 + 2 * DL_QN;
   static constexpr int XCH_BYTES = 2 * 2 * 32 * 32 * 4;   // SwiGLU up values, double-buffered
   static constexpr int STILE_BYTES = 2 * 32 * DL_BM * 2;  // [2][32 columns][128 features] bf16
   static constexpr int MAXE = DECOMOE_MAX_E;
@@ -115,11 +133,6 @@ constexpr int dl_max_stages_from<1>() {
 }
 constexpr int DL_STAGES = dl_max_stages_from<12>();
 
-__device__ __forceinline__ uint64_t grid_id() {
-  uint64_t g;
-  asm volatile("mov.u64 %0, %%gridid;" : "=l"(g));
-  return g;
-}
 __device__ __forceinline__ uint64_t ld_acquire_u64(const void* p) {
   uint64_t v;
   asm volatile("ld.acquire.gpu.global.b64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
@@ -134,6 +147,26 @@ __device__ __forceinline__ void bulk_load_g2s(uint32_t dst, const void* src, uin
   asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
                "l"(src), "r"(bytes), "r"(bar)
                : "memory");
+}
+__device__ __forceinline__ uint64_t ld_relaxed_u64(const uint64_t* p) {
+  uint64_t v;
+  asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+// two adjacent words (16-byte aligned), each read single-copy atomically
+__device__ __forceinline__ void ld_relaxed_u64x2(const uint64_t* p, uint64_t& a, uint64_t& b) {
+  asm volatile("ld.relaxed.gpu.global.v2.b64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "l"(p) : "memory");
+}
+__device__ __forceinline__ void st_relaxed_u64(uint64_t* p, uint64_t v) {
+  asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+__device__ __forceinline__ uint64_t atom_add_acquire_u64(uint64_t* p, uint64_t v) {
+  uint64_t old;
+  asm volatile("atom.acquire.gpu.global.add.u64 %0, [%1], %2;" : "=l"(old) : "l"(p), "l"(v) : "memory");
+  return old;
+}
+__device__ __forceinline__ void red_add_relaxed_u64(uint64_t* p, uint64_t v) {
+  asm volatile("red.relaxed.gpu.global.add.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 __device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
   uint32_t v;
@@ -181,8 +214,11 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
   using C = DlCfg<STAGES>;
   extern __shared__ uint8_t smem_raw[];
   __shared__ float s_red[4][DL_MAX_T];
-  __shared__ int s_flag[4];  // [0] counters usable, [1] K, [2] finisher count
+  __shared__ int s_flag[4];  // [0] counters usable, [1] K, [2] finisher count, [3] the launch's tag (0: not yet)
   __shared__ int s_fin[DL_BN];
+  __shared__ int s_q[DL_QN];  // work items in the order this CTA takes them (-1: no more)
+  __shared__ int s_qt_store;   // the epilogue's current item
+  volatile int* const s_qt = &s_qt_store;
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
   uint8_t* smem = smem_raw + pad;
@@ -216,19 +252,28 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
 #define TEMPTY_BAR(a) (bar0 + 8u * (2 * STAGES + 2 + (a)))
 #define DRAIN_BAR (bar0 + 8u * (2 * STAGES + 4))
 #define XROWS_BAR (bar0 + 8u * (2 * STAGES + 5))
+#define QFULL_BAR(q) (bar0 + 8u * (2 * STAGES + 6 + (q)))
+#define QEMPTY_BAR(q) (bar0 + 8u * (2 * STAGES + 6 + DL_QN + (q)))
 
   const int T = g.T, E = g.E, k = g.k, d = g.d;
   const int N = T * k;
   const int nfb = d / DL_FB;
   uint32_t* const bar_word = reinterpret_cast<uint32_t*>(g.sync + 2);
+  uint64_t* const lcount = reinterpret_cast<uint64_t*>(g.sync + 4);
   int32_t* const ready = g.sync + DL_SYNC_HEAD;
   int32_t* const done = ready + E;
   int32_t* const comb = done + E;
-  const int n_clear = 2 * E + T * nfb + (DL_SYNC_HEAD - 2);  // barrier, spare, ready, done, comb
-  const uint64_t gid = grid_id();
+  uint64_t* const tagged = reinterpret_cast<uint64_t*>(g.sync + dl_sync_tagged_offset(E, d));  // [T][E] used
+  // a timed-out wait: the status says so, and the missing signature makes the
+  // next launch re-initialise the counter block
+  auto fail = [&]() {
+    report_status(g.status, DECOMOE_ERR_TIMEOUT);
+    st_relaxed_u64(lcount, 0u);
+  };
 
   if (tid == 0) {
     *s_abort = 0;
+    s_flag[3] = 0;
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(FULL_BAR(s), 1);
       mbar_init(EMPTY_BAR(s), 1);
@@ -239,6 +284,10 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
     }
     mbar_init(DRAIN_BAR, 1);
     mbar_init(XROWS_BAR, 1);
+    for (int q = 0; q < DL_QN; ++q) {
+      mbar_init(QFULL_BAR(q), 1);
+      mbar_init(QEMPTY_BAR(q), 2);  // the MMA thread and the epilogue
+    }
     fence_mbar_init();
   }
   __syncthreads();
@@ -246,29 +295,13 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
   // has completed and its writes are visible
   pdl_wait();
 
-  // ---------------------------------------------------------------- counters
-  // CTA 0 clears them once per launch (unless this grid id already did) and
-  // publishes the grid id; nothing else of the launch touches them before it
-  // has seen that id.
-  if (blockIdx.x == 0) {
-    if (tid == 0) s_flag[0] = ld_acquire_u64(g.sync) == gid;
-    __syncthreads();
-    if (!s_flag[0]) {
-      for (int i = tid; i < n_clear; i += DL_THREADS) g.sync[2 + i] = 0;
-      __syncthreads();
-      if (tid == 0) {
-        __threadfence();
-        st_release_u64(g.sync, gid);
-      }
-    }
-  }
-
   // ---------------------------------------------------------------- A: router
   // logits[t, e] = sum_j x[t, j] w_r[e, j] + bias[e] with the router's
   // decode-size arithmetic: threads 0..127 split the row's 16-byte vectors
   // (thread i takes i, i + 128, ...), warp shuffles, then the four warps in
   // order. The T token rows are staged in shared memory first (the TMA ring,
-  // unused until the expert phase), all copies in flight at once.
+  // unused until the expert phase), all copies in flight at once. Warps 0-3
+  // compute; warp 4 meanwhile learns the launch's tag.
   const int vpr = d / 8;
   const uint4* s_x = reinterpret_cast<const uint4*>(smem);
   // the first router row's loads go out with the staging copies (d <= 2048:
@@ -290,9 +323,10 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
       bulk_load_g2s(sA + off, reinterpret_cast<const uint8_t*>(g.x) + off,
                     bytes - off < DL_BULK_CHUNK ? bytes - off : DL_BULK_CHUNK, XROWS_BAR);
   }
-  if (!mbar_wait(XROWS_BAR, 0, g.limit_ns, s_abort)) report_status(g.status, DECOMOE_ERR_TIMEOUT);
-  for (int e = blockIdx.x; e < E; e += gridDim.x) {
-    if (tid < GEMV_THREADS) {
+  volatile int* const vflag = s_flag;
+  if (tid < GEMV_THREADS) {
+    if (!mbar_wait(XROWS_BAR, 0, g.limit_ns, s_abort)) fail();
+    for (int e = blockIdx.x; e < E; e += gridDim.x) {
       const uint4* wr = g.w_r + static_cast<int64_t>(e) * vpr;
       float acc[TMAX];
 #pragma unroll
@@ -325,57 +359,104 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
           if (lane == 0) s_red[warp][j] = v;
         }
       }
-    }
-    __syncthreads();
-    if (tid < T) {
-      float v = s_red[0][tid];
+      named_bar_sync(2, GEMV_THREADS);
+      if (tid < T) {
+        float v = s_red[0][tid];
 #pragma unroll
-      for (int w = 1; w < GEMV_THREADS / 32; ++w) v += s_red[w][tid];
-      g.logits[static_cast<int64_t>(tid) * E + e] = v + (g.bias != nullptr ? g.bias[e] : 0.f);
+        for (int w = 1; w < GEMV_THREADS / 32; ++w) v += s_red[w][tid];
+        v += g.bias != nullptr ? g.bias[e] : 0.f;
+        // the logit and the launch's tag in one single-copy-atomic word
+        int tg = vflag[3];
+        const uint64_t t0 = globaltimer_ns();
+        while (tg == 0 && !*s_abort && globaltimer_ns() - t0 <= g.limit_ns) tg = vflag[3];
+        if (tg != 0)
+          st_relaxed_u64(tagged + tid * E + e,
+                         (static_cast<uint64_t>(static_cast<uint32_t>(tg)) << 32) | __float_as_uint(v));
+      }
+      named_bar_sync(2, GEMV_THREADS);
     }
-    __syncthreads();
-  }
-
-  // ---------------------------------------------------------------- grid barrier
-  // One word: arrivals in the low 16 bits, a generation in the high bits. The
-  // last arrival (acquire-release, after every CTA's writes) adds
-  // 0x10000 - grid, which empties the count and bumps the generation. The
-  // first use also waits for CTA 0's counter clear (the published grid id).
-  auto grid_sync = [&](bool first) -> bool {
-    __syncthreads();
-    if (tid == 0) {
-      bool ok = true;
-      const uint64_t t0 = globaltimer_ns();
-      if (first && blockIdx.x != 0)
-        while (ld_acquire_u64(g.sync) != gid)
+  } else if (warp == GEMV_THREADS / 32) {
+    // Arrive on the launch counter: the launch number in the returned word is
+    // this launch's for every CTA (the round cannot complete before all of
+    // them have arrived), and the last arrival moves it to the next number.
+    // Without the signature, CTA 0 (re)initialises the counter block and the
+    // other CTAs wait for that, then arrive again.
+    const uint32_t G = gridDim.x;
+    uint64_t old = 0;
+    if (lane == 0) old = atom_add_acquire_u64(lcount, 1u);
+    old = __shfl_sync(0xffffffffu, old, 0);
+    bool ok = true;
+    if ((old >> 40) != DL_SIGNATURE) {
+      if (blockIdx.x == 0) {
+        // the barrier word, the work-item counter, ready, done, comb, the
+        // distributed picks and the tagged logits, then the signature
+        // (launch 0, no arrivals)
+        const int n = dl_sync_tagged_offset(E, d) + 2 * DL_MAX_T * E;
+        g.sync[2] = 0;
+        g.sync[3] = 0;
+        for (int i = DL_SYNC_HEAD + lane; i < n; i += 32) g.sync[i] = 0;
+        __syncwarp();
+        if (lane == 0) {
+          __threadfence();
+          st_release_u64(lcount, DL_SIGNATURE << 40);
+          old = atom_add_acquire_u64(lcount, 1u);
+        }
+      } else if (lane == 0) {
+        const uint64_t t0 = globaltimer_ns();
+        while ((ld_acquire_u64(lcount) >> 40) != DL_SIGNATURE)
           if (globaltimer_ns() - t0 > g.limit_ns) {
             ok = false;
             break;
           }
-      if (ok) {
-        const uint32_t G = gridDim.x;
-        const uint32_t old = atom_add_acq_rel_u32(bar_word, 1u);
-        if ((old & 0xFFFFu) == G - 1u) {
-          red_add_release_u32(bar_word, 0x10000u - G);
-        } else {
-          // short sleeps between polls keep the waiting CTAs' loads off the
-          // word the last arrival has to update
-          while ((ld_acquire_u32(bar_word) >> 16) == (old >> 16)) {
-            __nanosleep(64);
-            if (globaltimer_ns() - t0 > g.limit_ns) {
-              ok = false;
-              break;
-            }
+        if (ok) old = atom_add_acquire_u64(lcount, 1u);
+      }
+    }
+    if (lane == 0) {
+      if (ok && (old >> 40) == DL_SIGNATURE) {
+        if ((old & 0xFFFFu) == G - 1u) red_add_relaxed_u64(lcount, 0x10000u - G);
+        vflag[3] = static_cast<int>(static_cast<uint32_t>((old >> 16) & 0xFFFFFFu) + 1u);  // never 0
+      } else {
+        *s_abort = 1;
+        fail();
+      }
+    }
+  }
+
+  // ---------------------------------------------------------------- grid barrier
+  // (distributed routing only) One word: arrivals in the low 16 bits, a
+  // generation in the high bits. The last arrival (acquire-release, after
+  // every CTA's writes) adds 0x10000 - grid, which empties the count and
+  // bumps the generation.
+  auto grid_sync = [&]() -> bool {
+    __syncthreads();
+    if (tid == 0) {
+      bool ok = true;
+      const uint64_t t0 = globaltimer_ns();
+      const uint32_t G = gridDim.x;
+      const uint32_t old = atom_add_acq_rel_u32(bar_word, 1u);
+      if ((old & 0xFFFFu) == G - 1u) {
+        red_add_release_u32(bar_word, 0x10000u - G);
+      } else {
+        // short sleeps between polls keep the waiting CTAs' loads off the
+        // word the last arrival has to update
+        while ((ld_acquire_u32(bar_word) >> 16) == (old >> 16)) {
+          __nanosleep(64);
+          if (globaltimer_ns() - t0 > g.limit_ns) {
+            ok = false;
+            break;
           }
         }
       }
       s_flag[0] = ok;
-      if (!ok) report_status(g.status, DECOMOE_ERR_TIMEOUT);
+      if (!ok) fail();
     }
     __syncthreads();
     return s_flag[0] != 0;
   };
-  if (!grid_sync(true)) return;  // nothing allocated yet
+  // every thread past the router (the ring's x rows are no longer read)
+  __syncthreads();
+  if (*s_abort) return;  // nothing allocated yet
+  const uint32_t tag = static_cast<uint32_t>(s_flag[3]);
 
   // ---------------------------------------------------------------- B: routing
   // Up to DL_LOCAL_ROUTE_T tokens every CTA routes them all itself (same
@@ -388,29 +469,99 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
   const bool dist = TMAX > DL_LOCAL_ROUTE_T && T > DL_LOCAL_ROUTE_T;
   float* s_lg = reinterpret_cast<float*>(smem);  // [T][E], in the ring
   float* s_wt = s_lg + T * E;                     // [T][E] full-pool pick weights (0: not picked)
-  int32_t* const g_fpick = comb + T * nfb;        // [T*k] full-pool picks (distributed routing)
+  int32_t* const g_fpick = comb + DL_MAX_T * nfb;  // [T*k] full-pool picks (distributed routing)
   float* const g_fpw = reinterpret_cast<float*>(g_fpick + N);
   {
-    const float4* src = reinterpret_cast<const float4*>(g.logits);
-    float4* dst = reinterpret_cast<float4*>(s_lg);
-    for (int i = tid; i < T * E / 4; i += DL_THREADS) {
-      if (!dist) dst[i] = __ldcg(src + i);
+    for (int i = tid; i < T * E / 4; i += DL_THREADS)
       reinterpret_cast<float4*>(s_wt)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-    }
     for (int i = tid; i < C::MAXE; i += DL_THREADS) s_tmask[i] = 0u;
+    if (!dist) {
+      // every logit, once its word carries this launch's tag (pairs of
+      // words, up to four pairs per thread in flight per round; bounded)
+      bool ok = true;
+      const uint64_t t0 = globaltimer_ns();
+      const int npair = T * E / 2;  // E is a multiple of 4
+      for (int i0 = 0; ok && i0 < npair; i0 += 4 * DL_THREADS) {
+        uint64_t w[8];
+        for (;;) {
+          bool pend = false;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int i = i0 + tid + DL_THREADS * j;
+            if (i < npair) {
+              ld_relaxed_u64x2(tagged + 2 * i, w[2 * j], w[2 * j + 1]);
+            } else {
+              w[2 * j] = w[2 * j + 1] = static_cast<uint64_t>(tag) << 32;
+            }
+          }
+#pragma unroll
+          for (int j = 0; j < 8; ++j) pend |= static_cast<uint32_t>(w[j] >> 32) != tag;
+          if (!pend) break;
+          if (*s_abort || globaltimer_ns() - t0 > g.limit_ns) {
+            ok = false;
+            break;
+          }
+          __nanosleep(64);
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int i = i0 + tid + DL_THREADS * j;
+          if (i < npair) {
+            s_lg[2 * i] = __uint_as_float(static_cast<uint32_t>(w[2 * j]));
+            s_lg[2 * i + 1] = __uint_as_float(static_cast<uint32_t>(w[2 * j + 1]));
+          }
+        }
+      }
+      if (!ok) {
+        *s_abort = 1;
+        fail();
+      }
+    }
   }
   __syncthreads();
+  if (*s_abort) return;  // nothing allocated yet
+  if (!dist && blockIdx.x == 0)
+    for (int i = tid; i < T * E; i += DL_THREADS) g.logits[i] = s_lg[i];
   if (dist) {
     // CTA t < T routes token t (warp 0; fixed prefix) and publishes its picks
     if (static_cast<int>(blockIdx.x) < T && warp == 0) {
       const int t = blockIdx.x;
-      const float* row = g.logits + static_cast<int64_t>(t) * E;
+      const uint64_t* row = tagged + t * E;
       const int lim = g.want_mass ? E : g.K_fixed;
+      // row t, once each word carries this launch's tag (bounded; on time-out
+      // the status says so and the launch goes on with what it read)
+      float lv[8];
+      {
+        const uint64_t t0 = globaltimer_ns();
+        uint64_t wv[8];
+        for (;;) {
+          bool pend = false;
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int e = lane + 32 * i;
+            wv[i] = e < E ? ld_relaxed_u64(row + e) : static_cast<uint64_t>(tag) << 32;
+          }
+#pragma unroll
+          for (int i = 0; i < 8; ++i) pend |= static_cast<uint32_t>(wv[i] >> 32) != tag;
+          if (!__any_sync(0xffffffffu, pend)) break;
+          if (__any_sync(0xffffffffu, globaltimer_ns() - t0 > g.limit_ns)) {  // warp-uniform exit
+            if (lane == 0) fail();
+            break;
+          }
+          __nanosleep(64);
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int e = lane + 32 * i;
+          lv[i] = __uint_as_float(static_cast<uint32_t>(wv[i]));
+          if (e < E) g.logits[t * E + e] = lv[i];
+        }
+      }
       uint32_t v[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         const int e = lane + 32 * i;
-        v[i] = (e < lim) ? fkey(__ldcg(row + e)) : 0u;
+        v[i] = (e < lim) ? fkey(lv[i]) : 0u;
       }
       float my_v;
       int my_i;
@@ -430,7 +581,7 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
         g.topk_w[t * k + lane] = w;
       }
     }
-    if (!grid_sync(false)) return;  // nothing allocated yet
+    if (!grid_sync()) return;  // nothing allocated yet
     for (int f = tid; f < N; f += DL_THREADS) {
       const int t = f / k;
       const int e = __ldcg(g.topk_idx + f);
@@ -635,7 +786,39 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
     bool ok = true;
     uint32_t armed = 0, armed_ph = 0;
     const uint64_t pol_once = policy_evict_first();  // every weight block is read once per step
-    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+    // Work items: the first is this CTA's index, every later one comes from
+    // the shared counter (item grid + n for the n-th draw), drawn once the
+    // current item's last load is out (the draw's round trip hides behind
+    // the loads in flight), so CTAs that finish early take more. Each CTA
+    // draws until it gets an index past the list (a CTA without a first item
+    // draws once): max(total, grid) draws in all, and the last of them
+    // returns the counter to zero for the next launch.
+    int32_t* const sched = g.sync + 3;
+    const int G = static_cast<int>(gridDim.x);
+    const int ndraw = total > G ? total : G;
+    auto draw = [&]() -> int {
+      const int f = atomicAdd(sched, 1);
+      if (f == ndraw - 1) *sched = 0;
+      return G + f;
+    };
+    int t = blockIdx.x;
+    for (int n = 0;; ++n) {
+      // publish the item (or the end) to the MMA and epilogue warps
+      if (lane == 0) {
+        const int qs = n % DL_QN;
+        if (!mbar_wait(QEMPTY_BAR(qs), ((n / DL_QN) & 1u) ^ 1u, g.limit_ns, s_abort)) {
+          ok = false;
+        } else {
+          s_q[qs] = t < total ? t : -1;
+          mbar_arrive(QFULL_BAR(qs));
+        }
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      if (t >= total) {
+        if (n == 0 && lane == 0) draw();
+        break;
+      }
       bool dn;
       int eg, wb;
       item(t, dn, eg, wb);
@@ -708,10 +891,12 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
+      const int tn = lane == 0 ? draw() : 0;
+      t = __shfl_sync(0xffffffffu, tn, 0);
     }
     if (lane == 0 && !ok) {
       *s_abort = 1;
-      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+      fail();
       int no_abort = 0;
       for (int s = 0; s < STAGES; ++s)
         if ((armed >> s) & 1u) mbar_wait(FULL_BAR(s), (armed_ph >> s) & 1u, g.limit_ns, &no_abort);
@@ -721,8 +906,15 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
     int stage = 0;
     uint32_t ph = 0;
     bool ok = true, issued = false;
-    int it = 0;
-    for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
+    for (int it = 0;; ++it) {
+      const int qs = it % DL_QN;
+      if (!mbar_wait(QFULL_BAR(qs), (it / DL_QN) & 1u, g.limit_ns, s_abort)) {
+        ok = false;
+        break;
+      }
+      const int t = *reinterpret_cast<volatile int*>(&s_q[qs]);
+      mbar_arrive(QEMPTY_BAR(qs));
+      if (t < 0) break;
       bool dn;
       int eg, wb;
       item(t, dn, eg, wb);
@@ -760,7 +952,7 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
     }
     if (!ok) {
       *s_abort = 1;
-      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+      fail();
       if (issued) {
         int no_abort = 0;
         tc_commit(DRAIN_BAR);
@@ -778,10 +970,27 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
       uint4* dst = g.x_perm + static_cast<int64_t>(r) * vpr;
       for (int c = lane; c < vpr; c += 32) dst[c] = __ldg(src + c);
     }
-    int it = 0;
     int xpar = 0;
     bool ok = true;
-    for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
+    for (int it = 0;; ++it) {
+      // one thread takes the item from the queue and hands it (or -2 for a
+      // wait that gave up) to the other 127 through s_qt
+      if (et == 0) {
+        const int qs = it % DL_QN;
+        if (mbar_wait(QFULL_BAR(qs), (it / DL_QN) & 1u, g.limit_ns, s_abort)) {
+          *s_qt = *reinterpret_cast<volatile int*>(&s_q[qs]);
+          mbar_arrive(QEMPTY_BAR(qs));
+        } else {
+          *s_qt = -2;
+        }
+      }
+      named_bar_sync(1, 128);
+      const int t = *s_qt;
+      if (t == -2) {
+        ok = false;
+        break;
+      }
+      if (t < 0) break;
       bool dn;
       int eg, wb;
       item(t, dn, eg, wb);
@@ -885,7 +1094,7 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
     }
     if (!ok) {
       *s_abort = 1;
-      report_status(g.status, DECOMOE_ERR_TIMEOUT);
+      fail();
     }
   }
   pdl_trigger();
@@ -902,14 +1111,13 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
 #undef TEMPTY_BAR
 #undef DRAIN_BAR
 #undef XROWS_BAR
+#undef QFULL_BAR
+#undef QEMPTY_BAR
 }
 
 bool decode_layer_supported(int64_t T, int d, int E, int k, int m, int dtype, int K_fixed) {
   // x rows and the logits are staged in the TMA ring during the first phases
   constexpr size_t ring = static_cast<size_t>(DL_STAGES) * DlCfg<DL_STAGES>::STAGE_BYTES;
-  // one token: the separate launches measured faster (the expert phase's
-  // handoff from gate/up to down dominates there, and 96 weight tiles use
-  // 96 SMs either way)
   return dtype == DECOMOE_BF16 && T >= DL_MIN_T && T <= DL_MAX_T && T * k <= DL_MAX_ROWS &&
          (K_fixed > 0 || (K_fixed == -1 && T <= DL_LOCAL_ROUTE_T)) && E >= 1 &&
          E <= DECOMOE_MAX_E && E % 4 == 0 && k >= 1 && k <= 32 && k <= E && d % 256 == 0 && m % 128 == 0 &&
@@ -917,7 +1125,8 @@ bool decode_layer_supported(int64_t T, int d, int E, int k, int m, int dtype, in
 }
 
 size_t decode_layer_sync_ints(int64_t T, int d, int E) {
-  return align_up(static_cast<size_t>(DL_SYNC_HEAD + 2 * E + T * (d / DL_FB) + 2 * T * DL_MAX_ROWS / DL_MAX_T), 64);
+  if (T < DL_MIN_T || T > DL_MAX_T) return 0;  // the one-launch layer never runs there
+  return align_up(static_cast<size_t>(dl_sync_tagged_offset(E, d) + 2 * DL_MAX_T * E), 64);
 }
 
 int launch_decode_layer(const void* x, const void* w_r, const float* bias, const void* w_gate_up, const void* w_down,
@@ -929,7 +1138,7 @@ int launch_decode_layer(const void* x, const void* w_r, const float* bias, const
   DM_ARG_CHECK(aligned16(x) && aligned16(w_r) && aligned16(w_gate_up) && aligned16(w_down) && aligned16(out) &&
                    (residual == nullptr || aligned16(residual)) && (text_out == nullptr || aligned16(text_out)),
                "moe_layer: bf16 operands must be 16-byte aligned");
-  DM_ARG_CHECK((reinterpret_cast<uintptr_t>(sync) & 7u) == 0, "moe_layer: workspace misaligned");
+  DM_ARG_CHECK((reinterpret_cast<uintptr_t>(sync) & 15u) == 0, "moe_layer: workspace misaligned");
   CUtensorMap tw1, tx1, tw2, tx2;
   DM_RET(make_tmap_bf16(&tw1, w_gate_up, static_cast<uint64_t>(d), static_cast<uint64_t>(E) * 2 * m, DL_BM, DL_BK));
   DM_RET(make_tmap_bf16(&tx1, x, static_cast<uint64_t>(d), static_cast<uint64_t>(T), DL_BN, DL_BK));

@@ -189,7 +189,7 @@ int launch_expert_ffn_fused(const void* x_perm, const int32_t* offsets, int64_t 
 // One launch for a whole decode-size layer (router, routing, dispatch,
 // experts, combine, and with text_out the visual-block removal of the
 // output; fixed or device-selected prefix). sync: decode_layer_sync_ints(T, d, E) int32 of the caller's
-// workspace, 8-byte aligned, any content (the launch clears what it uses).
+// workspace, 16-byte aligned, any content (the launch clears what it uses).
 bool decode_layer_supported(int64_t T, int d, int E, int k, int m, int dtype, int K_fixed);
 size_t decode_layer_sync_ints(int64_t T, int d, int E);
 int launch_decode_layer(const void* x, const void* w_r, const float* bias, const void* w_gate_up, const void* w_down,

@@ -1,10 +1,12 @@
 """The decode-size layer as one launch (router, routing, dispatch, experts and
-combine in a single persistent kernel, 2 <= T <= 32 tokens).
+combine in a single persistent kernel, 1 <= T <= 32 tokens).
 
 Its counters live in the layer workspace and must reset themselves: these
-tests start from a workspace full of garbage, replay several CUDA graphs that
-share one workspace with different inputs in a rotating order, and compare
-every output with a fresh eager call. The combine done inside the kernel must
+tests start from a workspace full of garbage or zeros (no signature: the
+launch initialises the block), replay several CUDA graphs that share one
+workspace with different inputs in a rotating order (also after the
+workspace was zeroed between replays), and compare every output with a
+fresh eager call. The combine done inside the kernel must
 equal, bit for bit, decomoe_combine run on the kernel's own expert outputs;
 the oracle comparison of the same layer sits in test_gpu_layer.py.
 """
@@ -62,7 +64,7 @@ class _Experts:
         return self.c[e]
 
 
-@pytest.mark.parametrize("T,K", [(2, 64), (5, 8), (16, 128), (12, -1), (3, -1), (32, 64)])
+@pytest.mark.parametrize("T,K", [(1, 64), (2, 64), (5, 8), (16, 128), (12, -1), (3, -1), (32, 64), (1, -1)])
 def test_garbage_workspace_first_call(layer, T, K):
     wl, g = layer
     x = W.make_x(W.DECODE, T=T, device="cuda", seed=T)
@@ -82,11 +84,12 @@ def test_garbage_workspace_first_call(layer, T, K):
         assert torch.equal(_bits(out), _bits(ref))
 
 
-@pytest.mark.parametrize("T,K", [(2, 64), (8, 64), (32, 40), (8, -1), (13, 64)])
+@pytest.mark.parametrize("T,K", [(1, 64), (2, 64), (8, 64), (32, 40), (8, -1), (13, 64)])
 def test_rotating_graph_replays_share_one_workspace(layer, T, K):
-    """Each graph keeps its kernel's grid id from one replay to the next; the
-    counters must be back at zero after every launch for the next replay (of
-    the same or another graph) to be right."""
+    """The counters must be back at zero after every launch, and the launch
+    counter one number further, for the next replay (of the same or another
+    graph) to be right; a zeroed workspace (no signature) between two replays
+    is initialised again by the next one."""
     wl, g = layer
     xs = [W.make_x(W.DECODE, T=T, device="cuda", seed=10 + i) for i in range(3)]
     res = torch.zeros_like(xs[0])
@@ -100,11 +103,13 @@ def test_rotating_graph_replays_share_one_workspace(layer, T, K):
     outs = [torch.empty_like(x) for x in xs]
     graphs = [dm.capture_graph(lambda i=i: _call(wl, g, xs[i], outs[i], ws, K, residual=res, status=st))
               for i in range(3)]
-    for i in (0, 1, 2, 0, 0, 1, 2, 2, 1, 0, 1):
+    for n, i in enumerate((0, 1, 2, 0, 0, 1, 2, 2, 1, 0, 1, 2, 0)):
+        if n in (5, 11):
+            ws.zero_()
         outs[i].fill_(-3.0)
         graphs[i].replay()
         torch.cuda.synchronize()
-        assert torch.equal(_bits(outs[i]), _bits(refs[i])), f"replay of graph {i}"
+        assert torch.equal(_bits(outs[i]), _bits(refs[i])), f"replay {n} of graph {i}"
     assert dm.decomoe_read_status(st) == 0
 
 
@@ -168,3 +173,41 @@ def test_edge_prefixes_against_oracle(layer, T, K, p):
     wg, wu, wd = (_Experts(g[n]) for n in ("w_gate", "w_up", "w_down"))
     ref = np.stack([O.moe_token(f64(x[t]), logits[t].astype(np.float32), wg, wu, wd, Ku, k)[0] for t in range(T)])
     assert_close_out(f64(out)[keep], ref[keep], BF16_REL_L2, BF16_MAX_ABS, "decode layer output")
+
+
+@pytest.mark.parametrize("T,K,p", [(1, 64, 0.7), (5, 64, 0.7), (8, -1, 0.7), (16, 64, 0.7), (3, 40, 0.0),
+                                   (24, 64, 0.0)])
+def test_tied_logits_take_the_lower_index(layer, T, K, p):
+    """A router whose rows come in identical pairs gives every logit twice:
+    the one-launch routing (a bitonic top-8 network for E <= 128, k <= 8)
+    must order equal logits by index exactly as the routing kernel's arg-max
+    rounds do, picks and weights bit for bit, on the layer's own logits."""
+    wl, g = layer
+    w_r = g["w_r"].clone()
+    w_r[1::2] = w_r[0::2]
+    bias = None
+    if g["bias"] is not None:
+        bias = g["bias"].clone()
+        bias[1::2] = bias[0::2]
+    x = W.make_x(W.DECODE, T=T, device="cuda", seed=400 + T)
+    ws = _ws(wl, T)
+    out = torch.empty_like(x)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    dm.decomoe_moe_layer(x, w_r, bias, g["w_gu"], g["w_down"], wl.k, out, ws, K_fixed=K, p=p, status=st)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(st) == 0
+    offs = dm.decomoe_moe_layer_workspace_layout(T, wl.d, wl.E, wl.k, wl.m, dm.DECOMOE_BF16)
+    E, k = wl.E, wl.k
+    logits = ws[offs[0]:offs[0] + T * E * 4].view(torch.float32).view(T, E).clone()
+    assert torch.equal(logits[:, 0::2].view(torch.int32), logits[:, 1::2].view(torch.int32))
+    idx = ws[offs[1]:offs[1] + T * k * 4].view(torch.int32).view(T, k).clone()
+    wts = ws[offs[2]:offs[2] + T * k * 4].view(torch.float32).view(T, k).clone()
+    Ku = int(ws[offs[11]:offs[11] + 4].view(torch.int32).cpu()) if K == -1 else K
+    ri = torch.empty(T, k, dtype=torch.int32, device=DEV)
+    rw = torch.empty(T, k, dtype=torch.float32, device=DEV)
+    dm.decomoe_route_prefix(logits, Ku, k, topk_idx=ri, topk_w=rw)
+    torch.cuda.synchronize()
+    assert torch.equal(idx, ri)
+    assert torch.equal(wts.view(torch.int32), rw.view(torch.int32))
+    oi, _ = O.route_prefix(logits.cpu().numpy(), Ku, k)
+    assert np.array_equal(idx.cpu().numpy(), oi)
