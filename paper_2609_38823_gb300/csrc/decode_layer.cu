@@ -46,6 +46,8 @@
 // for logits; the launch number is 24 bits wide, and its wrap carries into
 // the signature, which re-initialises the block, so no tag recurs while
 // older words can still be read.
+#include <type_traits>
+
 #include "route_common.cuh"
 
 namespace decomoe {
@@ -290,7 +292,25 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
     }
     fence_mbar_init();
   }
+  // the accumulators' tensor memory, held to the end (every return below
+  // frees it first)
+  if (warp == 1) {
+    tmem_alloc(smem_u32(const_cast<uint32_t*>(s_tmem)), C::TMEM_COLS);
+    tmem_relinquish();
+  } else if (warp == 5 && lane == 0) {
+    tma_prefetch_desc(&tma_w1);
+    tma_prefetch_desc(&tma_x1);
+    tma_prefetch_desc(&tma_w2);
+    tma_prefetch_desc(&tma_x2);
+  }
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *s_tmem;
+  // leave early (a timed-out wait): free the tensor memory first
+  auto leave = [&]() {
+    if (warp == 1) tmem_dealloc(tmem_base, C::TMEM_COLS);
+  };
   // the previous kernel on the stream (which may have used this workspace)
   // has completed and its writes are visible
   pdl_wait();
@@ -308,6 +328,8 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
   // one pass of GEMV_VPT vectors per thread)
   uint4 wv0[GEMV_VPT];
   const bool pre_w = vpr <= GEMV_THREADS * GEMV_VPT && static_cast<int>(blockIdx.x) < E && tid < GEMV_THREADS;
+  // the first router row's bias too (read after the products otherwise)
+  const float b0 = (tid < T && g.bias != nullptr && static_cast<int>(blockIdx.x) < E) ? __ldg(g.bias + blockIdx.x) : 0.f;
   if (pre_w) {
 #pragma unroll
     for (int i = 0; i < GEMV_VPT; ++i) {
@@ -364,11 +386,13 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
         float v = s_red[0][tid];
 #pragma unroll
         for (int w = 1; w < GEMV_THREADS / 32; ++w) v += s_red[w][tid];
-        v += g.bias != nullptr ? g.bias[e] : 0.f;
+        v += g.bias == nullptr ? 0.f : e == static_cast<int>(blockIdx.x) ? b0 : __ldg(g.bias + e);
         // the logit and the launch's tag in one single-copy-atomic word
         int tg = vflag[3];
-        const uint64_t t0 = globaltimer_ns();
-        while (tg == 0 && !*s_abort && globaltimer_ns() - t0 <= g.limit_ns) tg = vflag[3];
+        if (tg == 0) {
+          const uint64_t t0 = globaltimer_ns();
+          while (tg == 0 && !*s_abort && globaltimer_ns() - t0 <= g.limit_ns) tg = vflag[3];
+        }
         if (tg != 0)
           st_relaxed_u64(tagged + tid * E + e,
                          (static_cast<uint64_t>(static_cast<uint32_t>(tg)) << 32) | __float_as_uint(v));
@@ -455,7 +479,10 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
   };
   // every thread past the router (the ring's x rows are no longer read)
   __syncthreads();
-  if (*s_abort) return;  // nothing allocated yet
+  if (*s_abort) {
+    leave();
+    return;
+  }
   const uint32_t tag = static_cast<uint32_t>(s_flag[3]);
 
   // ---------------------------------------------------------------- B: routing
@@ -479,24 +506,28 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
       // every logit, once its word carries this launch's tag (pairs of
       // words, up to four pairs per thread in flight per round; bounded)
       bool ok = true;
-      const uint64_t t0 = globaltimer_ns();
+      uint64_t t0 = 0;  // the clock is read once a round finds words missing
       const int npair = T * E / 2;  // E is a multiple of 4
       for (int i0 = 0; ok && i0 < npair; i0 += 4 * DL_THREADS) {
         uint64_t w[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) w[j] = 0u;  // tag 0: not read yet
         for (;;) {
-          bool pend = false;
+          // (re)read the pairs not complete yet
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
             const int i = i0 + tid + DL_THREADS * j;
-            if (i < npair) {
-              ld_relaxed_u64x2(tagged + 2 * i, w[2 * j], w[2 * j + 1]);
-            } else {
+            if (i >= npair) {
               w[2 * j] = w[2 * j + 1] = static_cast<uint64_t>(tag) << 32;
+            } else if (static_cast<uint32_t>(w[2 * j] >> 32) != tag || static_cast<uint32_t>(w[2 * j + 1] >> 32) != tag) {
+              ld_relaxed_u64x2(tagged + 2 * i, w[2 * j], w[2 * j + 1]);
             }
           }
+          bool pend = false;
 #pragma unroll
           for (int j = 0; j < 8; ++j) pend |= static_cast<uint32_t>(w[j] >> 32) != tag;
           if (!pend) break;
+          if (t0 == 0) t0 = globaltimer_ns();
           if (*s_abort || globaltimer_ns() - t0 > g.limit_ns) {
             ok = false;
             break;
@@ -519,7 +550,10 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
     }
   }
   __syncthreads();
-  if (*s_abort) return;  // nothing allocated yet
+  if (*s_abort) {
+    leave();
+    return;
+  }
   if (!dist && blockIdx.x == 0)
     for (int i = tid; i < T * E; i += DL_THREADS) g.logits[i] = s_lg[i];
   if (dist) {
@@ -581,7 +615,10 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
         g.topk_w[t * k + lane] = w;
       }
     }
-    if (!grid_sync()) return;  // nothing allocated yet
+    if (!grid_sync()) {
+      leave();
+      return;
+    }
     for (int f = tid; f < N; f += DL_THREADS) {
       const int t = f / k;
       const int e = __ldcg(g.topk_idx + f);
@@ -598,40 +635,49 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
     }
     __syncthreads();
   }
-  auto route_pass = [&](int lim_fixed, bool full) {
-    // full: picks over [0, E) into s_fidx / s_fw (and, with a fixed prefix,
-    // the prefix picks from them); else picks over [0, lim_fixed)
+  // one routing pass; NSL key slots per lane (4 cover up to 128 experts).
+  // The full pool's picks (with the mass) and the prefix picks come from one
+  // loop body, so its code is fetched once for both rounds.
+  auto route_tokens = [&](auto nsl, int lim_fixed, bool full) {
+    constexpr int NSL = decltype(nsl)::value;
+    // full: picks over [0, E) into s_fidx / s_fw, then, with a fixed prefix,
+    // the prefix picks; else picks over [0, lim_fixed)
+    const int Kp = full ? g.K_fixed : lim_fixed;
     for (int t = warp; t < T; t += DL_THREADS / 32) {
       const float* row = s_lg + t * E;
-      const int lim = full ? E : lim_fixed;
-      uint32_t v[8];
+      uint32_t v[NSL];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
+      for (int i = 0; i < NSL; ++i) {
         const int e = lane + 32 * i;
-        v[i] = (e < lim) ? fkey(row[e]) : 0u;
+        v[i] = (e < E) ? fkey(row[e]) : 0u;
       }
-      float my_v;
-      int my_i;
-      warp_topk(v, lim, k, lane, my_v, my_i);
-      if (full) {
-        const float wf = pick_weight(my_v, lane, k);
+      float my_v = 0.f;
+      int my_i = 0;
+      for (int r = full ? 0 : 1; r < 2; ++r) {
+        if (r == 1 && Kp <= 0) break;  // the prefix is chosen after the mass
+        // full-pool picks all inside the prefix are the prefix picks too
+        const bool reuse = r == 1 && full && __all_sync(0xffffffffu, lane >= k || my_i < Kp);
+        if (!reuse) warp_topk_n<NSL>(v, r == 0 ? E : Kp, k, lane, my_v, my_i);
+        const float w = pick_weight(my_v, lane, k);
         if (lane < k) {
-          s_fidx[t * k + lane] = my_i;
-          s_fw[t * k + lane] = wf;
-          s_wt[t * E + my_i] = wf;
+          if (r == 0) {
+            s_fidx[t * k + lane] = my_i;
+            s_fw[t * k + lane] = w;
+            s_wt[t * E + my_i] = w;
+          } else {
+            s_idx[t * k + lane] = my_i;
+            s_w[t * k + lane] = w;
+            atomicOr(&s_tmask[my_i], 1u << t);
+          }
         }
-        if (g.K_fixed <= 0) continue;
-        // full-pool picks all inside the prefix: they are the prefix picks too
-        const bool inside = __all_sync(0xffffffffu, lane >= k || my_i < g.K_fixed);
-        if (!inside) warp_topk(v, g.K_fixed, k, lane, my_v, my_i);
-      }
-      const float w = pick_weight(my_v, lane, k);
-      if (lane < k) {
-        s_idx[t * k + lane] = my_i;
-        s_w[t * k + lane] = w;
-        atomicOr(&s_tmask[my_i], 1u << t);
       }
     }
+  };
+  auto route_pass = [&](int lim_fixed, bool full) {
+    if (E <= 128)
+      route_tokens(std::integral_constant<int, 4>(), lim_fixed, full);
+    else
+      route_tokens(std::integral_constant<int, 8>(), lim_fixed, full);
   };
   // At most two passes from one call site (code run once per launch is
   // fetched cold): pass 0 the full pool (with the mass) or the fixed prefix,
@@ -643,16 +689,14 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
         // Eq. 11 as the routing kernels form it: fp32 sums per block of 8
         // tokens in token order (a token picks an expert at most once; the
         // table's zeros add nothing), then the fixed fp64 tree over the blocks
-        const int nb = (T + 7) / 8;
         for (int e = tid; e < E; e += DL_THREADS) {
-          double part[4] = {0.0, 0.0, 0.0, 0.0};
-          for (int b = 0; b < nb; ++b) {
-            float acc = 0.f;
-            const int te = min(T, 8 * b + 8);
-            for (int tt = 8 * b; tt < te; ++tt) acc += s_wt[tt * E + e];
-            part[b] = static_cast<double>(acc);
-          }
-          const double me = nb == 1 ? part[0] : (part[0] + part[2]) + (part[1] + part[3]);
+          float a[4] = {0.f, 0.f, 0.f, 0.f};  // blocks of 8 tokens (T <= 32)
+#pragma unroll
+          for (int b = 0; b < 4; ++b)
+            for (int tt = 8 * b; tt < T && tt < 8 * b + 8; ++tt) a[b] += s_wt[tt * E + e];
+          const double me = T <= 8 ? static_cast<double>(a[0])
+                                   : (static_cast<double>(a[0]) + static_cast<double>(a[2])) +
+                                         (static_cast<double>(a[1]) + static_cast<double>(a[3]));
           s_mass[e] = me;
           if (blockIdx.x == 0) g.mass[e] = me;
         }
@@ -746,14 +790,7 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
   const int total1 = s_tt1[Kd], total = total1 + s_tt2[Kd];
 
   // ---------------------------------------------------------------- C, D: experts and combine
-  if (warp == 1) {
-    tmem_alloc(smem_u32(const_cast<uint32_t*>(s_tmem)), C::TMEM_COLS);
-    tmem_relinquish();
-  }
-  tc_fence_before();
   __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem_base = *s_tmem;
   // item -> (down?, expert, weight block); expert = last e with s_tt[e] <= i
   auto item = [&](int t, bool& dn, int& eg, int& wb) {
     dn = t >= total1;
@@ -775,12 +812,6 @@ __global__ void __launch_bounds__(DL_THREADS, 1)
 
   if (warp == 0) {
     // ------------------------------------------------ TMA producer (lane 0)
-    if (lane == 0) {
-      tma_prefetch_desc(&tma_w1);
-      tma_prefetch_desc(&tma_x1);
-      tma_prefetch_desc(&tma_w2);
-      tma_prefetch_desc(&tma_x2);
-    }
     int stage = 0;
     uint32_t ph = 0;
     bool ok = true;

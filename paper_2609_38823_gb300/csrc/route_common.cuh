@@ -35,23 +35,25 @@ __device__ __forceinline__ float fkey_inv(uint32_t k) {
   return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
 }
 
-// k rounds of warp arg-max over entries e < lim: each round one redux.sync
-// max over the lanes' best keys; when a single lane holds that key (no tie)
-// a ballot names it, otherwise one redux.sync min over the indices of the
-// lanes holding it picks the lower index. Only the winning lane clears its
-// key, so the next round waits on nothing else; pick j ends in lane j.
-__device__ __forceinline__ void warp_topk(const uint32_t (&key_in)[8], int lim, int k, int lane, float& my_v,
-                                          int& my_i) {
-  uint32_t key[8];
+// k rounds of warp arg-max over entries e < lim (entry lane + 32 i in slot
+// i; NSL slots cover 32 NSL entries): each round one redux.sync max over the
+// lanes' best keys; when a single lane holds that key (no tie) a ballot
+// names it, otherwise one redux.sync min over the indices of the lanes
+// holding it picks the lower index. Only the winning lane clears its key, so
+// the next round waits on nothing else; pick j ends in lane j.
+template <int NSL>
+__device__ __forceinline__ void warp_topk_n(const uint32_t (&key_in)[NSL], int lim, int k, int lane, float& my_v,
+                                            int& my_i) {
+  uint32_t key[NSL];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) key[i] = (lane + 32 * i < lim) ? key_in[i] : 0u;
+  for (int i = 0; i < NSL; ++i) key[i] = (lane + 32 * i < lim) ? key_in[i] : 0u;
   my_v = 0.f;
   my_i = 0;
   for (int j = 0; j < k; ++j) {
     uint32_t bk = 0;
     int bs = 0;  // slot of the lane's best (entries ascend with the slot, so strict > keeps the lowest index)
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
+    for (int i = 0; i < NSL; ++i)
       if (key[i] > bk) {
         bk = key[i];
         bs = i;
@@ -71,7 +73,7 @@ __device__ __forceinline__ void warp_topk(const uint32_t (&key_in)[8], int lim, 
     {
       const bool mine = wl == lane;
 #pragma unroll
-      for (int i = 0; i < 8; ++i) key[i] = (mine && i == ws) ? 0u : key[i];  // selects keep key[] in registers
+      for (int i = 0; i < NSL; ++i) key[i] = (mine && i == ws) ? 0u : key[i];  // selects keep key[] in registers
     }
     const int wi = wl + 32 * __shfl_sync(0xffffffffu, ws, wl);
     if (lane == j) {
@@ -79,6 +81,11 @@ __device__ __forceinline__ void warp_topk(const uint32_t (&key_in)[8], int lim, 
       my_i = wi;
     }
   }
+}
+
+__device__ __forceinline__ void warp_topk(const uint32_t (&key_in)[8], int lim, int k, int lane, float& my_v,
+                                          int& my_i) {
+  warp_topk_n<8>(key_in, lim, k, lane, my_v, my_i);
 }
 
 // Renormalised weight of this lane's pick (lanes >= k get 0).
