@@ -634,7 +634,7 @@ def run_decode(dm, wl, layers, B, ws, pk, n):
                     "graph8_ms_per_layer": round(per_layer, 4),
                     "graph8_tokens_per_s": round(Td / (per_layer * 1e-3), 1),
                     "graph8_hbm_frac": round(mean_bytes / (per_layer * 1e-3) / 1e9 / pk["hbm_gbs"], 4),
-                    "path": ("one launch per layer" if 2 <= Td <= 32 else
+                    "path": ("one launch per layer" if 1 <= Td <= 32 else
                              "router, routing + dispatch, expert FFN, combine (separate launches)")})
         del Bd, xs
     return out
