@@ -542,12 +542,15 @@ DECOMOE_API int decomoe_moe_layer_workspace_layout(int64_t T, int d, int E, int 
  *   C - n + i and sees keys 0 .. C - n + i; query head h reads KV head
  *   h / (Hq / Hkv). scale <= 0 means 1 / sqrt(D). fp32 scores, softmax and
  *   accumulation; out rounded to bf16.
- *   Decode sizes: n * (Hq / Hkv) <= 64 queries per KV head: one launch;
- *   each block streams a range of keys and keeps the online softmax of up to
- *   32 queries of its KV head, and the ranges of a head (one thread-block
- *   cluster of up to 16 blocks) are merged in key order through the
- *   cluster's shared memory (deterministic). No workspace (0 bytes; ws may
- *   be null).
+ *   Decode sizes: n * (Hq / Hkv) <= 64 queries per KV head: each block
+ *   streams a range of keys and keeps the online softmax of up to 32 queries
+ *   of its KV head, and the ranges of a thread-block cluster (up to 16
+ *   blocks) are merged in key order through the cluster's shared memory. One
+ *   cluster per head and no workspace (0 bytes; ws may be null) while that
+ *   streams at most four 128-key chunks per block; a longer cache is split
+ *   over several clusters per head where the SMs allow, each leaving its
+ *   merged rows in the workspace, and a second small launch merges them in
+ *   cluster order (deterministic in both cases).
  *   Prefill sizes (more queries per KV head, n = C or a chunk n < C; Hq / Hkv
  *   even): V is transposed into the workspace, then one tensor-core CTA per
  *   (pair of query heads, 128-query tile) runs the online softmax over 64-key

@@ -41,8 +41,11 @@ constexpr int ATT_PROW = ATT_D + 4;             // floats per partial row: acc[D
 // cluster: after a cluster barrier, block r merges queries r, r + nsplit, ...
 // over the blocks in rank order, reading their partials through distributed
 // shared memory, and stores the output; a second barrier keeps every block's
-// shared memory alive until it has been read. No workspace, no counters, and
-// the result does not depend on timing.
+// shared memory alive until it has been read. A long cache (more than four
+// chunks per block with one cluster per head) is split over S clusters per
+// head where the SMs allow: each cluster stores its merged (m, l, output)
+// rows in a workspace and a second small launch merges the S clusters in
+// cluster order. No counters, and the result does not depend on timing.
 constexpr int ATD_WARPS = 8;
 constexpr int ATD_CH = 16 * ATD_WARPS;          // keys per staged chunk (16 per warp)
 constexpr int ATD_THREADS = 32 * ATD_WARPS;
@@ -60,9 +63,11 @@ static_assert(ATD_WARPS * ATD_QT * 16 * (ATD_OROW + 2) * 4 <= ATD_NST * ATD_STAG
 struct AttDecArgs {
   const uint4* q;   // [n, Hq, D] (K and V [C, Hkv, D] come through the tensor maps)
   int64_t n, C;
-  int Hq, Hkv, kps; // keys per block; the cluster (grid.x) is the head's splits
+  int Hq, Hkv, kps; // keys per block; a cluster (grid.x) is a run of the head's splits
+  int S;            // clusters per (KV head, query tile group): grid.y = Hkv * S
   float sl2;        // scale * log2(e)
   __nv_bfloat16* out;
+  float* part;      // S > 1: [Hkv][nz][S][QT * 16][ATT_PROW] merged rows of each cluster
   int32_t* status;
   uint64_t limit_ns;
 };
@@ -130,16 +135,16 @@ __global__ void __launch_bounds__(ATD_THREADS)
   volatile int* s_abort = reinterpret_cast<volatile int*>(bars + ATD_NST);
   const uint32_t sKVa = smem_u32(sKV);
   const uint32_t bar0 = smem_u32(bars);
-  const int s = blockIdx.x, g = blockIdx.y;
+  const int s = blockIdx.x, g = static_cast<int>(blockIdx.y) / a.S, cset = static_cast<int>(blockIdx.y) % a.S;
   const int G = a.Hq / a.Hkv;
   const int nq = static_cast<int>(a.n) * G;
   const int qbase = static_cast<int>(blockIdx.z) * ATD_QT * 16;  // first query row of this block
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int grp = lane >> 2, tig = lane & 3;
   constexpr int VPR = ATT_D / 8;  // 16-byte vectors per head row
-  const int64_t k0 = static_cast<int64_t>(s) * a.kps;
+  const int64_t k0 = static_cast<int64_t>(cset * static_cast<int>(gridDim.x) + s) * a.kps;
   const int64_t k1 = k0 + a.kps < a.C ? k0 + a.kps : a.C;
-  const int nch = static_cast<int>((k1 - k0 + ATD_CH - 1) / ATD_CH);
+  const int nch = k1 > k0 ? static_cast<int>((k1 - k0 + ATD_CH - 1) / ATD_CH) : 0;  // a split past C: none
   if (tid == 0) {
     *s_abort = 0;
     for (int st = 0; st < ATD_NST; ++st) mbar_init(bar0 + 8u * st, 1);
@@ -378,24 +383,109 @@ __global__ void __launch_bounds__(ATD_THREADS)
         acc = fmaf(w, ld_dsmem_f32(row + col * 4), acc);
         L = fmaf(w, ld_dsmem_f32(row + (ATT_D + 1) * 4), L);
       }
-      const int ti = qi / G, hj = qi - ti * G;
-      a.out[(static_cast<int64_t>(ti) * a.Hq + g * G + hj) * ATT_D + col] = __float2bfloat16_rn(acc / L);
+      if (a.S == 1) {
+        const int ti = qi / G, hj = qi - ti * G;
+        a.out[(static_cast<int64_t>(ti) * a.Hq + g * G + hj) * ATT_D + col] = __float2bfloat16_rn(acc / L);
+      } else {
+        // this cluster's merged row, for the merge launch
+        float* pr = a.part + ((static_cast<int64_t>(g * gridDim.z + blockIdx.z) * a.S + cset) * (QT * 16) + r) * ATT_PROW;
+        pr[col] = acc;
+        if (col == 0) {
+          pr[ATT_D] = M;
+          pr[ATT_D + 1] = L;
+        }
+      }
     }
   }
   cluster_sync_all();  // no block leaves while its partial rows may still be read
   pdl_trigger();
 }
 
-// Keys per block, in whole chunks: the splits of a head form one cluster of
-// at most att_max_cluster() blocks, one chunk each where C allows.
+// The S <= ATT_MAX_SETS clusters of a (KV head g = blockIdx.x, query tile
+// group z = blockIdx.y) merged in cluster order; block blockIdx.z takes two
+// of the rows (threads 0-127 and 128-255, one output column each), with all
+// S partials' loads in flight at once.
+constexpr int ATT_MAX_SETS = 16;
+__global__ void __launch_bounds__(ATD_THREADS)
+    k_attn_dec_merge(const float* __restrict__ part, int S, int rows, int64_t n, int Hq, int Hkv,
+                     __nv_bfloat16* __restrict__ out) {
+  pdl_wait();
+  const int g = blockIdx.x, z = blockIdx.y, tid = threadIdx.x;
+  const int G = Hq / Hkv;
+  const int nq = static_cast<int>(n) * G;
+  const int r = static_cast<int>(blockIdx.z) * 2 + (tid >> 7), col = tid & (ATT_D - 1);
+  const int qi = z * rows + r;
+  if (r < rows && qi < nq) {
+    const float* base = part + (static_cast<int64_t>(g * gridDim.y + z) * S * rows + r) * ATT_PROW;
+    float mc[ATT_MAX_SETS], ac[ATT_MAX_SETS], lc[ATT_MAX_SETS];
+#pragma unroll
+    for (int c = 0; c < ATT_MAX_SETS; ++c) {
+      const float* row = base + static_cast<int64_t>(c) * rows * ATT_PROW;
+      mc[c] = c < S ? __ldcg(row + ATT_D) : -INFINITY;
+      ac[c] = c < S ? __ldcg(row + col) : 0.f;
+      lc[c] = c < S ? __ldcg(row + ATT_D + 1) : 0.f;
+    }
+    float M = -INFINITY;
+#pragma unroll
+    for (int c = 0; c < ATT_MAX_SETS; ++c) M = fmaxf(M, mc[c]);
+    float acc = 0.f, L = 0.f;
+#pragma unroll
+    for (int c = 0; c < ATT_MAX_SETS; ++c) {
+      if (c < S) {
+        const float w = mc[c] == -INFINITY ? 0.f : att_ex2(mc[c] - M);  // a cluster with no visible key weighs 0
+        acc = fmaf(w, ac[c], acc);
+        L = fmaf(w, lc[c], L);
+      }
+    }
+    const int ti = qi / G, hj = qi - ti * G;
+    out[(static_cast<int64_t>(ti) * Hq + g * G + hj) * ATT_D + col] = __float2bfloat16_rn(acc / L);
+  }
+  pdl_trigger();
+}
+
 static int att_max_cluster();
-static int64_t att_kps(int64_t C) {
-  const int64_t maxc = att_max_cluster();
-  const int64_t nsplit = std::max<int64_t>(1, std::min<int64_t>((C + ATD_CH - 1) / ATD_CH, maxc));
+static int att_active_clusters(int cs);
+static int att_nz(int64_t nq) { return static_cast<int>((nq + ATD_QT * 16 - 1) / (ATD_QT * 16)); }
+// The split of a head's keys: S clusters of at most cs blocks each. One
+// cluster per (KV head, query tile group), of the largest size (16, 8, 4) of
+// which that many clusters are resident at once, while that streams at most
+// four chunks per block; a longer cache takes the cluster size and S that
+// put the most blocks to work with every cluster resident at once (the
+// device's limit on active clusters of that size) and each block keeping at
+// least two chunks.
+struct AttPlan {
+  int cs, S;
+};
+static AttPlan att_plan(int64_t C, int Hkv, int nz) {
+  const int maxc = att_max_cluster();
+  const int64_t sets = static_cast<int64_t>(Hkv) * nz;
+  int cs1 = maxc;
+  for (int cs : {16, 8, 4})
+    if (cs <= maxc && sets <= att_active_clusters(cs)) {
+      cs1 = cs;
+      break;
+    }
+  if (C <= static_cast<int64_t>(cs1) * ATD_CH * 4) return {cs1, 1};
+  AttPlan best = {cs1, 1};
+  int64_t best_blocks = cs1;
+  for (int cs : {16, 8, 4}) {
+    if (cs > maxc) continue;
+    const int64_t by_res = att_active_clusters(cs) / sets;
+    const int64_t by_keys = C / (static_cast<int64_t>(cs) * ATD_CH * 2);
+    const int64_t S = std::min<int64_t>({by_res, by_keys, static_cast<int64_t>(ATT_MAX_SETS)});
+    if (S >= 1 && S * cs > best_blocks) {
+      best = {cs, static_cast<int>(S)};
+      best_blocks = S * cs;
+    }
+  }
+  return best;
+}
+// Keys per block, in whole chunks, for the plan's cs * S splits.
+static int64_t att_kps(int64_t C, const AttPlan& pl) {
+  const int64_t nsplit = std::max<int64_t>(1, std::min<int64_t>((C + ATD_CH - 1) / ATD_CH, pl.cs)) * pl.S;
   int64_t kps = (C + nsplit - 1) / nsplit;
   return (kps + ATD_CH - 1) / ATD_CH * ATD_CH;
 }
-static int att_nz(int64_t nq) { return static_cast<int>((nq + ATD_QT * 16 - 1) / (ATD_QT * 16)); }
 
 // Largest cluster of decode blocks this device schedules (16 where the
 // non-portable size fits, else the portable 8), per device ordinal.
@@ -432,6 +522,37 @@ static int att_max_cluster() {
   cudaGetLastError();  // a refused query leaves no error behind
   g_att_cluster[dev].store(v);
   return v;
+}
+
+// Clusters of cs decode blocks the device keeps resident at once (per device
+// ordinal and cluster size 4, 8 or 16; 0 when the query is refused).
+static std::atomic<int> g_att_active[64][3];
+static int att_active_clusters(int cs) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  const int slot = cs == 4 ? 0 : cs == 8 ? 1 : 2;
+  int v = g_att_active[dev][slot].load();
+  if (v != 0) return v > 0 ? v : 0;
+  att_max_cluster();  // sets the kernels' shared-memory and cluster-size attributes
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(cs), 1, 1);
+  cfg.blockDim = dim3(ATD_THREADS);
+  cfg.dynamicSmemBytes = ATD_SMEM;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(cs);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n1 = 0, n2 = 0;
+  if (cudaOccupancyMaxActiveClusters(&n1, k_attn_dec<1>, &cfg) != cudaSuccess ||
+      cudaOccupancyMaxActiveClusters(&n2, k_attn_dec<2>, &cfg) != cudaSuccess)
+    n1 = n2 = 0;
+  cudaGetLastError();  // a refused query leaves no error behind
+  v = std::min(n1, n2);
+  g_att_active[dev][slot].store(v > 0 ? v : -1);
+  return v > 0 ? v : 0;
 }
 
 // ------------------------------------------------------------------ prefill (tensor cores)
@@ -817,7 +938,13 @@ size_t decomoe_attention_workspace_bytes(int64_t n, int64_t C, int Hq, int Hkv, 
   if (n <= 0 || C <= 0 || Hq <= 0 || Hkv <= 0 || D != ATT_D || Hq % Hkv != 0) return 0;
   if (att_use_prefill(n, Hq, Hkv))  // the transposed values [Hkv][D][C padded to 64]
     return align_up(static_cast<size_t>(Hkv) * ATT_D * att_c_pad(C) * 2, 256);
-  return 0;  // decode sizes: the splits merge through the cluster's shared memory
+  // decode sizes: a cluster's splits merge through its shared memory; several
+  // clusters per head (long caches) leave their merged rows here
+  const int nq = static_cast<int>(n) * (Hq / Hkv);
+  const int nz = att_nz(nq);
+  const int S = att_plan(C, Hkv, nz).S;
+  const int rows = (nq <= 16 ? 1 : 2) * 16;
+  return S == 1 ? 0 : align_up(static_cast<size_t>(Hkv) * nz * S * rows * ATT_PROW * 4, 256);
 }
 
 int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void* v_cache, int64_t C, int Hq,
@@ -885,10 +1012,16 @@ int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void*
   a.Hkv = Hkv;
   const int nq = static_cast<int>(n) * G;
   const int nz = att_nz(nq);
-  const int64_t kps = att_kps(C);
+  const AttPlan pl = att_plan(C, Hkv, nz);
+  const int S = pl.S;
+  const int64_t kps = att_kps(C, pl);
   DM_ARG_CHECK(kps <= 0x7fffffffLL, "attention: C=%lld keys is too long", (long long)C);
   a.kps = static_cast<int>(kps);
-  const int nsplit = static_cast<int>((C + kps - 1) / kps);  // <= att_max_cluster()
+  a.S = S;
+  a.part = static_cast<float*>(ws);
+  // blocks per cluster (<= pl.cs); with S > 1 the last blocks may find no
+  // key left (they weigh 0 in the merge)
+  const int nsplit = static_cast<int>((C + kps * S - 1) / (kps * S));
   a.sl2 = sc * 1.4426950408889634f;
   a.out = static_cast<__nv_bfloat16*>(out);
   a.status = status_dev;
@@ -899,7 +1032,7 @@ int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void*
   const uint32_t bkv[3] = {64, 1, ATD_CH};
   DM_RET(make_tmap_bf16_3d(&tk, k_cache, dkv, skv, bkv));
   DM_RET(make_tmap_bf16_3d(&tv, v_cache, dkv, skv, bkv));
-  const dim3 grid(static_cast<unsigned>(nsplit), static_cast<unsigned>(Hkv), static_cast<unsigned>(nz));
+  const dim3 grid(static_cast<unsigned>(nsplit), static_cast<unsigned>(Hkv * S), static_cast<unsigned>(nz));
   auto go = [&](auto kern) -> int {
     DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(ATD_SMEM)));
     if (nsplit > 8) DM_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1));
@@ -916,6 +1049,11 @@ int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void*
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     DM_CUDA_CHECK(cudaLaunchKernelEx(&cfg, kern, tk, tv, a));
+    if (S > 1)
+      DM_CUDA_CHECK(launch_pdl(k_attn_dec_merge,
+                               dim3(static_cast<unsigned>(Hkv), static_cast<unsigned>(nz), (nq <= 16 ? 1 : 2) * 8),
+                               dim3(ATD_THREADS), 0, s, static_cast<const float*>(ws), S, (nq <= 16 ? 1 : 2) * 16, n,
+                               Hq, Hkv, static_cast<__nv_bfloat16*>(out)));
     return DECOMOE_OK;
   };
   return nq <= 16 ? go(k_attn_dec<1>) : go(k_attn_dec<2>);

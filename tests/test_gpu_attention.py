@@ -51,7 +51,8 @@ def _run(q, k, v, scale=0.0):
 
 
 @pytest.mark.parametrize("n,C", [(1, 1), (1, 63), (1, 64), (1, 65), (1, 127), (1, 128), (1, 272), (1, 2049),
-                                 (2, 300), (8, 1552), (1, 16384), (3, 129), (5, 40000)])
+                                 (2, 300), (8, 1552), (1, 8192), (1, 8193), (1, 16384), (1, 16385), (3, 129),
+                                 (5, 40000), (8, 20000)])
 def test_attention_decode_parity(n, C):
     q, k, v = _qkv(n, C, seed=C + n)
     out = _run(q, k, v)
@@ -104,21 +105,31 @@ def test_attention_prefill_is_deterministic():
     assert torch.equal(a, b)
 
 
-def test_attention_decode_needs_no_workspace_and_repeats_bitwise():
-    """Decode sizes take no workspace (a null pointer is accepted) and give the
-    same bits on every call, in any order of sizes."""
-    sizes = [(1, 16384), (1, 300), (8, 2049), (2, 64), (1, 1), (4, 5000)]
+def test_attention_decode_workspace_and_repeats_bitwise():
+    """Decode sizes take no workspace while one cluster per KV head streams
+    at most four chunks per block (a null pointer is accepted there); a
+    longer cache is split over several clusters per head where the SMs allow
+    and takes a small workspace for their merged rows (a missing one is
+    rejected). Every call gives the same bits, in any order of sizes."""
+    sizes = [(1, 16384), (1, 300), (8, 2049), (2, 64), (1, 1), (4, 5000), (1, 40000)]
     for n, C in sizes:
-        assert dm.decomoe_attention_workspace_bytes(n, C, HQ, HKV, D) == 0
+        if C <= 16 * 128 * 4:
+            assert dm.decomoe_attention_workspace_bytes(n, C, HQ, HKV, D) == 0
+    lib = dm.lib()
     first = {}
     for rep in range(2):
         for n, C in sizes:
-            q, k, v = _qkv(n, C, seed=31 * C + n)
+            # device copies held in variables: a temporary's memory could be
+            # handed to the next copy before the launch reads it
+            q, k, v = (t.to(DEV) for t in _qkv(n, C, seed=31 * C + n))
             out = torch.empty(n, HQ, D, dtype=torch.bfloat16, device=DEV)
-            lib = dm.lib()
-            rc = lib.decomoe_attention(q.to(DEV).data_ptr(), n, k.to(DEV).data_ptr(), v.to(DEV).data_ptr(), C, HQ,
-                                       HKV, D, 0.0, out.data_ptr(), None, 0, None,
-                                       torch.cuda.current_stream().cuda_stream)
+            nbytes = dm.decomoe_attention_workspace_bytes(n, C, HQ, HKV, D)
+            ws = dm.workspace(nbytes, DEV)
+            args = (q.data_ptr(), n, k.data_ptr(), v.data_ptr(), C, HQ, HKV, D, 0.0, out.data_ptr())
+            stream = torch.cuda.current_stream().cuda_stream
+            if nbytes > 0 and rep == 0:
+                assert lib.decomoe_attention(*args, None, 0, None, stream) == dm.DECOMOE_ERR_WORKSPACE
+            rc = lib.decomoe_attention(*args, None if ws is None else ws.data_ptr(), nbytes, None, stream)
             torch.cuda.synchronize()
             assert rc == 0
             if rep == 0:
