@@ -211,3 +211,42 @@ def test_tied_logits_take_the_lower_index(layer, T, K, p):
     assert torch.equal(wts.view(torch.int32), rw.view(torch.int32))
     oi, _ = O.route_prefix(logits.cpu().numpy(), Ku, k)
     assert np.array_equal(idx.cpu().numpy(), oi)
+
+
+@pytest.mark.parametrize("E,k,T,K,p", [(256, 16, 1, 200, 0.7), (256, 16, 4, -1, 0.7), (256, 16, 13, 240, 0.7),
+                                       (256, 16, 16, 64, 0.0), (64, 4, 8, 32, 0.7), (64, 4, 32, 48, 0.7)])
+def test_other_pool_shapes_against_oracle(E, k, T, K, p):
+    """Pools other than 128 experts with k = 8: 256 experts (eight key slots
+    per lane in the routing rounds) with k = 16, where up to 16 tokens fill
+    the 256 routed rows and 13 or more tokens take the per-CTA routing with
+    its exchanged picks, and 64 experts with k = 4. Routing, mass and the
+    device-selected prefix against the oracle on the layer's own logits;
+    outputs within the bf16 tolerance."""
+    wl = W.with_(W.PREFILL, E=E, k=k, d=256, m=128)
+    g = W.make_layer(wl, device="cuda", with_x=False, seed=5)
+    x = W.make_x(wl, T=T, device="cuda", seed=600 + T)
+    ws = _ws(wl, T)
+    out = torch.empty_like(x)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    dm.decomoe_moe_layer(x, g["w_r"], g["bias"], dm.fuse_gate_up(g["w_gate"], g["w_up"]), g["w_down"], k, out, ws,
+                         K_fixed=K, p=p, status=st)
+    torch.cuda.synchronize()
+    assert dm.decomoe_read_status(st) == 0
+    offs = dm.decomoe_moe_layer_workspace_layout(T, wl.d, E, k, wl.m, dm.DECOMOE_BF16)
+    logits = f64(ws[offs[0]:offs[0] + T * E * 4].view(torch.float32).view(T, E))
+    idx = ws[offs[1]:offs[1] + T * k * 4].view(torch.int32).view(T, k).cpu().numpy()
+    wts = ws[offs[2]:offs[2] + T * k * 4].view(torch.float32).view(T, k).cpu().numpy()
+    if K == -1:
+        mass = ws[offs[3]:offs[3] + E * 8].view(torch.float64).cpu().numpy()
+        assert np.allclose(mass, O.activated_mass(logits.astype(np.float32), k), rtol=4e-6, atol=1e-5)
+        Ku = int(ws[offs[11]:offs[11] + 4].view(torch.int32).cpu())
+        assert Ku == O.select_prefix(mass, p, k)
+    else:
+        Ku = K
+    ref_idx, ref_w = O.route_prefix(logits.astype(np.float32), Ku, k)
+    keep = O.prefix_margin(logits.astype(np.float32), Ku, k) > 1e-6
+    assert np.array_equal(idx[keep], ref_idx[keep])
+    assert np.abs(wts[keep] - ref_w[keep]).max(initial=0.0) <= 1e-6
+    wg, wu, wd = (_Experts(g[n]) for n in ("w_gate", "w_up", "w_down"))
+    ref = np.stack([O.moe_token(f64(x[t]), logits[t].astype(np.float32), wg, wu, wd, Ku, k)[0] for t in range(T)])
+    assert_close_out(f64(out)[keep], ref[keep], BF16_REL_L2, BF16_MAX_ABS, f"decode layer E={E} k={k} T={T}")
