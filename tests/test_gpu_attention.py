@@ -198,3 +198,15 @@ def test_attention_rejects_unsupported_shapes():
         dm.decomoe_attention(q3.to(DEV), k3.to(DEV), v3.to(DEV), torch.empty(40, 12, D, dtype=torch.bfloat16,
                                                                                device=DEV), ws)
     assert e.value.code == dm.DECOMOE_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("n,C,Hq,Hkv", [(1, 20000, 16, 8), (2, 12000, 32, 2), (1, 9000, 8, 8), (4, 30000, 8, 1)])
+def test_attention_decode_long_caches_other_groupings(n, C, Hq, Hkv):
+    """Long caches split over several clusters per KV head (the cluster size
+    and count follow the number of (head, query tile) sets) for other head
+    groupings, against the oracle, and bit-identical on a second call."""
+    q, k, v = _qkv(n, C, seed=C + Hkv, Hq=Hq, Hkv=Hkv)
+    out = _run(q, k, v)
+    ref = O.attention(f64(q), f64(k), f64(v))
+    assert_close_out(f64(out), ref, BF16_REL_L2, BF16_MAX_ABS, f"attention n={n} C={C} Hq={Hq} Hkv={Hkv}")
+    assert torch.equal(_run(q, k, v), out)
