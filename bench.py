@@ -1144,7 +1144,8 @@ def reference(args, ws, rank):
             "value": v, "unit": "tokens/s", "n_gpus": 0, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(dt / args.steps * 1e3, 3), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": wl.name, "T": wl.T, "d": wl.d, "E": wl.E, "k": wl.k, "m": wl.m, "K": K},
+            "config": {"workload": wl.name, "T": wl.T, "visual_block": [wl.v0, wl.nv], "d": wl.d, "E": wl.E,
+                       "k": wl.k, "m": wl.m, "K": K},
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": _cores(), "kind": "oracle",
                              "sample": f"{ntok} tokens of the {wl.T}-token layer per step"},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
