@@ -36,16 +36,21 @@ constexpr int ATT_PROW = ATT_D + 4;             // floats per partial row: acc[D
 // registers (the accumulator layout of one product is the operand layout of
 // the next) and adds P V into its output tile. The eight warps of a block take
 // 16 keys of each chunk apiece; their states are merged in warp order into
-// the block's partial (m, l, unnormalised output) per query, kept in shared
-// memory. The splits of one (KV head, query tile group) form one thread-block
-// cluster: after a cluster barrier, block r merges queries r, r + nsplit, ...
-// over the blocks in rank order, reading their partials through distributed
-// shared memory, and stores the output; a second barrier keeps every block's
-// shared memory alive until it has been read. A long cache (more than four
-// chunks per block with one cluster per head) is split over S clusters per
-// head where the SMs allow: each cluster stores its merged (m, l, output)
-// rows in a workspace and a second small launch merges the S clusters in
-// cluster order. No counters, and the result does not depend on timing.
+// the block's partial (m, l, unnormalised output) per query. The splits of
+// one (KV head, query tile group) form one thread-block cluster: each block
+// pushes its partial of query row r into the shared memory of block
+// r % nsplit (distributed shared-memory stores, fire and forget), one cluster
+// barrier (release / acquire) makes them visible, and block r then merges
+// its rows over the blocks in rank order from its own shared memory and
+// stores the output. A barrier split around the launch's start (arrive
+// first thing, wait before the first push) keeps pushes out of blocks that
+// are not running yet; after the second barrier no block touches another's
+// shared memory, so blocks leave freely. A long cache (more than four chunks
+// per block with one cluster per head) is split over S clusters per head
+// where the SMs allow: each cluster stores its merged (m, l, output) rows in
+// a workspace and a second small launch, allowed to be scheduled from this
+// launch's start, merges the S clusters in cluster order. No counters, and
+// the result does not depend on timing.
 constexpr int ATD_WARPS = 8;
 constexpr int ATD_CH = 16 * ATD_WARPS;          // keys per staged chunk (16 per warp)
 constexpr int ATD_THREADS = 32 * ATD_WARPS;
@@ -54,10 +59,16 @@ constexpr int ATD_QT = 2;                       // 16-row query tiles per block 
 constexpr int ATD_HALF = ATD_CH * 64 * 2;       // 128 keys x 64 features, 128-byte swizzle (16 KB)
 constexpr int ATD_STAGE = 4 * ATD_HALF;         // K and V halves of one chunk
 constexpr int ATD_NST = 3;                      // chunks in flight
-constexpr int ATD_PART = ATD_QT * 16 * ATT_PROW * 4;  // the block's partial rows (bytes)
+// Partial rows pushed into a block by the blocks of its cluster: row r of
+// the query tile goes to block r % nsplit, slot (r / nsplit) * nsplit +
+// sender rank, so ceil(rows / nsplit) * nsplit <= rows + 15 slots
+// (nsplit <= 16).
+constexpr int ATD_RSLOTS = ATD_QT * 16 + 15;
+constexpr int ATD_RECV = ATD_RSLOTS * ATT_PROW * 4;
 constexpr size_t ATD_SMEM =
-    1024 + static_cast<size_t>(ATD_NST) * ATD_STAGE + ATD_QT * 16 * ATD_ROW + ATD_PART + 8 * ATD_NST + 16;
-constexpr int ATD_OROW = ATT_D + 4;             // floats per row of the warp merge (padded)
+    1024 + static_cast<size_t>(ATD_NST) * ATD_STAGE + ATD_QT * 16 * ATD_ROW + ATD_RECV + 8 * ATD_NST + 16;
+static_assert(ATD_SMEM <= 232448, "decode attention shared memory");
+constexpr int ATD_OROW = ATT_D + 8;             // floats per row of the warp merge (conflict-free float2 stores)
 static_assert(ATD_WARPS * ATD_QT * 16 * (ATD_OROW + 2) * 4 <= ATD_NST * ATD_STAGE, "warp merge fits in the ring");
 
 struct AttDecArgs {
@@ -101,15 +112,25 @@ __device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
   return r;
 }
-__device__ __forceinline__ float ld_dsmem_f32(uint32_t addr) {
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
-  return v;
+__device__ __forceinline__ void st_dsmem_v4(uint32_t addr, float4 v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+               : "memory");
 }
-// Every thread of every block of the cluster: writes before it (shared and
-// global) are visible to the cluster's blocks after it.
-__device__ __forceinline__ void cluster_sync_all() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+__device__ __forceinline__ void st_dsmem_v2(uint32_t addr, float x, float y) {
+  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(addr), "f"(x), "f"(y) : "memory");
+}
+// Split cluster barrier, every thread of every block: arrive (relaxed: no
+// ordering) and the matching wait; arrive with release and wait with
+// acquire: writes before the arrive (shared, distributed shared and global)
+// are visible to the cluster's blocks after the wait.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_arrive_release() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait_acquire() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 // D (16x8 fp32) += A (16x16 bf16, row) * B (16x8 bf16, col)
 __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
@@ -130,8 +151,8 @@ __global__ void __launch_bounds__(ATD_THREADS)
   const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
   uint8_t* sKV = smem_raw + pad;                                 // [NST]{K lo, K hi, V lo, V hi}
   uint8_t* sQ = sKV + ATD_NST * ATD_STAGE;                       // [QT * 16][ROW]
-  float* s_part = reinterpret_cast<float*>(sQ + ATD_QT * 16 * ATD_ROW);  // [QT*16][PROW]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(s_part) + ATD_PART);
+  float* s_recv = reinterpret_cast<float*>(sQ + ATD_QT * 16 * ATD_ROW);  // [RSLOTS][PROW]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(s_recv) + ATD_RECV);
   volatile int* s_abort = reinterpret_cast<volatile int*>(bars + ATD_NST);
   const uint32_t sKVa = smem_u32(sKV);
   const uint32_t bar0 = smem_u32(bars);
@@ -153,6 +174,12 @@ __global__ void __launch_bounds__(ATD_THREADS)
     tma_prefetch_desc(&tma_v);
   }
   __syncthreads();
+  // first half of the barrier that keeps pushes out of blocks not yet
+  // running (its wait comes before the first push)
+  cluster_arrive_relaxed();
+  // several clusters per head: the merge launch may be scheduled now (its
+  // griddepcontrol.wait still waits for this grid's completion)
+  if (a.S > 1) pdl_trigger();
   pdl_wait();  // q, K and V are ready
   // chunk c into stage st: K and V, features 0-63 and 64-127 (keys past C read as zero)
   auto issue = [&](int c, int st) {
@@ -165,11 +192,8 @@ __global__ void __launch_bounds__(ATD_THREADS)
     tma_load_3d(base + 2 * ATD_HALF, &tma_v, bar, 0, g, key0);
     tma_load_3d(base + 3 * ATD_HALF, &tma_v, bar, 64, g, key0);
   };
-  int issued = nch < ATD_NST ? nch : ATD_NST;  // chunks whose copies were requested (thread 0)
-  if (tid == 0)
-    for (int c = 0; c < issued; ++c) issue(c, c);
-
-  // query rows (zero rows past the group's queries)
+  // query rows (zero rows past the group's queries), requested ahead of the
+  // key and value chunks so that they do not queue behind them
   for (int i = tid; i < QT * 16 * VPR; i += ATD_THREADS) {
     const int r = i / VPR, c = i - r * VPR;
     const int qi = qbase + r;
@@ -181,6 +205,9 @@ __global__ void __launch_bounds__(ATD_THREADS)
       *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
     }
   }
+  int issued = nch < ATD_NST ? nch : ATD_NST;  // chunks whose copies were requested (thread 0)
+  if (tid == 0)
+    for (int c = 0; c < issued; ++c) issue(c, c);
   cp_async_wait_all();
   __syncthreads();  // the query rows are in place
 
@@ -313,8 +340,9 @@ __global__ void __launch_bounds__(ATD_THREADS)
   }
   __syncthreads();
 
-  // merge the warps (warp order) through shared memory: per warp and row m, l
-  // and the 128 output columns
+  // merge the warps (warp order) through shared memory: per warp and valid
+  // row m, l and the 128 output columns
+  const int rv = min(ATD_QT * 16, nq - qbase);  // this block's query rows (>= 1)
   float* sm_o = reinterpret_cast<float*>(sKV);                   // [WARPS][QT*16][OROW]
   float* sm_m = sm_o + ATD_WARPS * ATD_QT * 16 * ATD_OROW;        // [WARPS][QT*16]
   float* sm_l = sm_m + ATD_WARPS * ATD_QT * 16;
@@ -326,63 +354,88 @@ __global__ void __launch_bounds__(ATD_THREADS)
       ls += __shfl_xor_sync(0xffffffffu, ls, 1);
       ls += __shfl_xor_sync(0xffffffffu, ls, 2);
       const int r = qt * 16 + grp + 8 * h;
-      if (tig == 0) {
-        sm_m[warp * ATD_QT * 16 + r] = m[qt][h];
-        sm_l[warp * ATD_QT * 16 + r] = ls;
-      }
-      float* orow = sm_o + (warp * ATD_QT * 16 + r) * ATD_OROW;
+      if (r < rv) {
+        if (tig == 0) {
+          sm_m[warp * ATD_QT * 16 + r] = m[qt][h];
+          sm_l[warp * ATD_QT * 16 + r] = ls;
+        }
+        float* orow = sm_o + (warp * ATD_QT * 16 + r) * ATD_OROW;
 #pragma unroll
-      for (int j = 0; j < 16; ++j)
-        *reinterpret_cast<float2*>(orow + 8 * j + 2 * tig) = make_float2(o[qt][j][2 * h], o[qt][j][2 * h + 1]);
+        for (int j = 0; j < 16; ++j)
+          *reinterpret_cast<float2*>(orow + 8 * j + 2 * tig) = make_float2(o[qt][j][2 * h], o[qt][j][2 * h + 1]);
+      }
     }
   __syncthreads();
-  // this block's partial rows: m (log2 units), l and the unnormalised output
-  for (int r = 0; r < QT * 16; r += 2) {
-    // two rows at a time: threads 0-127 and 128-255 take one output column each
-    const int rh = r + (tid >> 7);
-    const int col = tid & (ATT_D - 1);
+  // this block's partial rows (m in log2 units, l, unnormalised output), one
+  // (row, 4 columns) piece per thread summed over the warps in warp order,
+  // pushed into the shared memory of the row's owner, block r % nsplit
+  cluster_wait_acquire();  // every block of the cluster is running
+  const uint32_t nsplit = gridDim.x;
+  const uint32_t rank = cluster_ctarank();
+  const uint32_t recv_a = smem_u32(s_recv);
+  for (int it = tid; it < rv * (ATT_D / 4); it += ATD_THREADS) {
+    const int r = it / (ATT_D / 4), c4 = it - r * (ATT_D / 4);
+    float mw[ATD_WARPS], lw[ATD_WARPS];
+    float4 ow[ATD_WARPS];
+#pragma unroll
+    for (int w = 0; w < ATD_WARPS; ++w) {  // every load in flight at once
+      mw[w] = sm_m[w * ATD_QT * 16 + r];
+      lw[w] = sm_l[w * ATD_QT * 16 + r];
+      ow[w] = *reinterpret_cast<const float4*>(sm_o + (w * ATD_QT * 16 + r) * ATD_OROW + 4 * c4);
+    }
     float M = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < ATD_WARPS; ++w) M = fmaxf(M, sm_m[w * ATD_QT * 16 + rh]);
-    float acc = 0.f, L = 0.f;
+    for (int w = 0; w < ATD_WARPS; ++w) M = fmaxf(M, mw[w]);
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    float L = 0.f;
     if (M != -INFINITY) {
 #pragma unroll
       for (int w = 0; w < ATD_WARPS; ++w) {
-        const float mw = sm_m[w * ATD_QT * 16 + rh];
-        const float ww = mw == -INFINITY ? 0.f : att_ex2(mw - M);
-        acc = fmaf(ww, sm_o[(w * ATD_QT * 16 + rh) * ATD_OROW + col], acc);
-        L = fmaf(ww, sm_l[w * ATD_QT * 16 + rh], L);
+        const float ww = mw[w] == -INFINITY ? 0.f : att_ex2(mw[w] - M);
+        acc.x = fmaf(ww, ow[w].x, acc.x);
+        acc.y = fmaf(ww, ow[w].y, acc.y);
+        acc.z = fmaf(ww, ow[w].z, acc.z);
+        acc.w = fmaf(ww, ow[w].w, acc.w);
+        L = fmaf(ww, lw[w], L);
       }
     }
-    float* pr = s_part + rh * ATT_PROW;
-    pr[col] = acc;
-    if (col == 0) {
-      pr[ATT_D] = M;
-      pr[ATT_D + 1] = L;
-    }
+    const uint32_t owner = static_cast<uint32_t>(r) % nsplit;
+    const uint32_t slot = (static_cast<uint32_t>(r) / nsplit) * nsplit + rank;
+    const uint32_t dst = mapa_shared(recv_a + slot * (ATT_PROW * 4), owner);
+    st_dsmem_v4(dst + 16u * c4, acc);
+    if (c4 == 0) st_dsmem_v2(dst + ATT_D * 4, M, L);
   }
-  cluster_sync_all();  // every block's partial rows are in place
-  // block `rank` merges rows rank, rank + nsplit, ... over the blocks in rank
-  // order (threads 0-127 and 128-255: two rows per pass, one column each)
-  const uint32_t nsplit = gridDim.x;
-  const uint32_t rank = cluster_ctarank();
-  const uint32_t part_a = smem_u32(s_part);
-  for (int r0 = static_cast<int>(rank); r0 < QT * 16; r0 += 2 * static_cast<int>(nsplit)) {
+  cluster_arrive_release();
+  cluster_wait_acquire();  // every block's rows are in their owners' shared memory
+  // block `rank` merges its rows rank, rank + nsplit, ... over the blocks in
+  // rank order (threads 0-127 and 128-255: two rows per pass, one column each)
+  for (int r0 = static_cast<int>(rank); r0 < rv; r0 += 2 * static_cast<int>(nsplit)) {
     const int r = r0 + (tid >> 7) * static_cast<int>(nsplit);
     const int col = tid & (ATT_D - 1);
-    const int qi = qbase + r;
-    if (r < QT * 16 && qi < nq) {
-      float M = -INFINITY;
-      for (uint32_t t = 0; t < nsplit; ++t)
-        M = fmaxf(M, ld_dsmem_f32(mapa_shared(part_a + (r * ATT_PROW + ATT_D) * 4, t)));
-      float acc = 0.f, L = 0.f;
-      for (uint32_t t = 0; t < nsplit; ++t) {
-        const uint32_t row = mapa_shared(part_a + r * ATT_PROW * 4, t);
-        const float mt = ld_dsmem_f32(row + ATT_D * 4);
-        const float w = mt == -INFINITY ? 0.f : att_ex2(mt - M);  // a split with no visible key weighs 0
-        acc = fmaf(w, ld_dsmem_f32(row + col * 4), acc);
-        L = fmaf(w, ld_dsmem_f32(row + (ATT_D + 1) * 4), L);
+    if (r < rv) {
+      const float* base = s_recv + (r / static_cast<int>(nsplit)) * static_cast<int>(nsplit) * ATT_PROW;
+      constexpr int MAXS = 16;  // cluster size limit
+      float mt[MAXS], at[MAXS], lt[MAXS];
+#pragma unroll
+      for (int t = 0; t < MAXS; ++t) {  // every load in flight at once
+        const float* row = base + t * ATT_PROW;
+        mt[t] = t < static_cast<int>(nsplit) ? row[ATT_D] : -INFINITY;
+        at[t] = t < static_cast<int>(nsplit) ? row[col] : 0.f;
+        lt[t] = t < static_cast<int>(nsplit) ? row[ATT_D + 1] : 0.f;
       }
+      float M = -INFINITY;
+#pragma unroll
+      for (int t = 0; t < MAXS; ++t) M = fmaxf(M, mt[t]);
+      float acc = 0.f, L = 0.f;
+#pragma unroll
+      for (int t = 0; t < MAXS; ++t) {
+        if (t < static_cast<int>(nsplit)) {
+          const float w = mt[t] == -INFINITY ? 0.f : att_ex2(mt[t] - M);  // a split with no visible key weighs 0
+          acc = fmaf(w, at[t], acc);
+          L = fmaf(w, lt[t], L);
+        }
+      }
+      const int qi = qbase + r;
       if (a.S == 1) {
         const int ti = qi / G, hj = qi - ti * G;
         a.out[(static_cast<int64_t>(ti) * a.Hq + g * G + hj) * ATT_D + col] = __float2bfloat16_rn(acc / L);
@@ -397,8 +450,7 @@ __global__ void __launch_bounds__(ATD_THREADS)
       }
     }
   }
-  cluster_sync_all();  // no block leaves while its partial rows may still be read
-  pdl_trigger();
+  if (a.S == 1) pdl_trigger();
 }
 
 // The S <= ATT_MAX_SETS clusters of a (KV head g = blockIdx.x, query tile
@@ -1041,13 +1093,18 @@ int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void*
     cfg.blockDim = dim3(ATD_THREADS);
     cfg.dynamicSmemBytes = ATD_SMEM;
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;  // one cluster per (KV head, query tile group)
     attr[0].val.clusterDim.x = static_cast<unsigned>(nsplit);
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    // at most one block per SM: scheduled while the previous kernel drains,
+    // waiting on griddepcontrol.wait before it reads q, K or V
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed =
+        pdl_enabled(static_cast<int64_t>(grid.x) * grid.y * grid.z) ? 1 : 0;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     DM_CUDA_CHECK(cudaLaunchKernelEx(&cfg, kern, tk, tv, a));
     if (S > 1)
       DM_CUDA_CHECK(launch_pdl(k_attn_dec_merge,
