@@ -52,8 +52,10 @@ def _run(q, k, v, scale=0.0):
 
 @pytest.mark.parametrize("n,C", [(1, 1), (1, 63), (1, 64), (1, 65), (1, 127), (1, 128), (1, 272), (1, 2049),
                                  (2, 300), (8, 1552), (1, 8192), (1, 8193), (1, 16384), (1, 16385), (3, 129),
-                                 (5, 40000), (8, 20000)])
+                                 (5, 40000), (8, 20000), (4, 1900), (4, 2049), (7, 1000)])
 def test_attention_decode_parity(n, C):
+    # (4, 1900): 32 query rows on a cluster of 15, the most receive slots
+    # (ceil(32 / 15) * 15 = 45); (7, 1000): a second query tile of 24 rows
     q, k, v = _qkv(n, C, seed=C + n)
     out = _run(q, k, v)
     ref = O.attention(f64(q), f64(k), f64(v))
