@@ -1074,6 +1074,12 @@ int decomoe_attention(const void* q, int64_t n, const void* k_cache, const void*
   // blocks per cluster (<= pl.cs); with S > 1 the last blocks may find no
   // key left (they weigh 0 in the merge)
   const int nsplit = static_cast<int>((C + kps * S - 1) / (kps * S));
+  // the receive slots of the pushed partial rows are sized for clusters of
+  // at most 16 blocks (att_plan never picks more)
+  if (nsplit < 1 || nsplit > 16) {
+    set_error("attention: internal split of %d blocks per cluster (at most 16)", nsplit);
+    return DECOMOE_ERR_UNSUPPORTED;
+  }
   a.sl2 = sc * 1.4426950408889634f;
   a.out = static_cast<__nv_bfloat16*>(out);
   a.status = status_dev;
