@@ -52,10 +52,12 @@ def _run(q, k, v, scale=0.0):
 
 @pytest.mark.parametrize("n,C", [(1, 1), (1, 63), (1, 64), (1, 65), (1, 127), (1, 128), (1, 272), (1, 2049),
                                  (2, 300), (8, 1552), (1, 8192), (1, 8193), (1, 16384), (1, 16385), (3, 129),
-                                 (5, 40000), (8, 20000), (4, 1900), (4, 2049), (7, 1000)])
+                                 (5, 40000), (8, 20000), (4, 1900), (4, 2049), (7, 1000), (2, 2), (3, 3),
+                                 (8, 8)])
 def test_attention_decode_parity(n, C):
     # (4, 1900): 32 query rows on a cluster of 15, the most receive slots
-    # (ceil(32 / 15) * 15 = 45); (7, 1000): a second query tile of 24 rows
+    # (ceil(32 / 15) * 15 = 45); (7, 1000): a second query tile of 24 rows;
+    # (2, 2), (3, 3), (8, 8): every query's causal limit inside the one chunk
     q, k, v = _qkv(n, C, seed=C + n)
     out = _run(q, k, v)
     ref = O.attention(f64(q), f64(k), f64(v))
@@ -212,3 +214,42 @@ def test_attention_decode_long_caches_other_groupings(n, C, Hq, Hkv):
     ref = O.attention(f64(q), f64(k), f64(v))
     assert_close_out(f64(out), ref, BF16_REL_L2, BF16_MAX_ABS, f"attention n={n} C={C} Hq={Hq} Hkv={Hkv}")
     assert torch.equal(_run(q, k, v), out)
+
+
+def test_attention_decode_chained_calls_in_a_graph():
+    """Three decode steps in a row, each step's query the previous step's
+    output, over a long cache (several clusters per head and the merge
+    launch), the text-only one and the long one again, all sharing one
+    workspace: the launches are programmatic, so each must wait for the one
+    before it both to read its output and to reuse the workspace. Captured
+    in a CUDA graph and replayed, the outputs equal the eager calls'
+    bits."""
+    sizes = [16385, 2049, 16385]
+    g = torch.Generator().manual_seed(77)
+    q0 = torch.randn(1, HQ, D, generator=g).to(torch.bfloat16).to(DEV)
+    kv = [(torch.randn(C, HKV, D, generator=g).to(torch.bfloat16).to(DEV),
+           torch.randn(C, HKV, D, generator=g).to(torch.bfloat16).to(DEV)) for C in sizes]
+    nbytes = max(dm.decomoe_attention_workspace_bytes(1, C, HQ, HKV, D) for C in sizes)
+    assert nbytes > 0
+    ws = dm.workspace(nbytes, DEV)
+
+    def chain(outs):
+        q = q0
+        for (k, v), o in zip(kv, outs):
+            dm.decomoe_attention(q, k, v, o, ws)
+            q = o
+
+    eager = [torch.empty(1, HQ, D, dtype=torch.bfloat16, device=DEV) for _ in sizes]
+    chain(eager)
+    torch.cuda.synchronize()
+    graphed = [torch.full((1, HQ, D), 7.0, dtype=torch.bfloat16, device=DEV) for _ in sizes]
+    gr = dm.capture_graph(lambda: chain(graphed))
+    for _ in range(3):
+        for o in graphed:
+            o.fill_(7.0)
+        gr.replay()
+        torch.cuda.synchronize()
+        for i, (a, b) in enumerate(zip(eager, graphed)):
+            assert torch.equal(a, b), i
+    ref = O.attention(f64(q0.cpu()), f64(kv[0][0].cpu()), f64(kv[0][1].cpu()))
+    assert_close_out(f64(eager[0].cpu()), ref, BF16_REL_L2, BF16_MAX_ABS, "chained step 1")
